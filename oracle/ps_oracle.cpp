@@ -1,0 +1,341 @@
+// Oracle for the PackServe scheduler hot path: TEST INFRASTRUCTURE, not part of the product.
+//
+// Only the tests, __graft_entry__.smoke() and bench.py's CPU-baseline / reference arm load this
+// library.  It shares no code, header, table or constant generator with the CUDA library: it is a
+// plain, single-threaded restatement of the paper's Algorithm 1 applied to one request at a time
+// in arrival order, with instance state updated after every decision (Section 4, "Metadata
+// service": state tracked along request paths).
+//
+// Data structures: one std::unordered_set<uint64_t> of cached block hashes per instance (the
+// paper's Section 6 prefix tree, flattened: a block hash covers its whole prefix, so "prefix
+// cached" == "block hash present").  Hit length = a linear walk along the request's chain until
+// the first hash that is not in the set (exact whether or not the set is prefix-closed).
+//
+// Arithmetic: IEEE fp32 in the fixed operation order written below, built with
+// -ffp-contract=off (no fused multiply-add) so that x86-64 and aarch64 give identical bits.
+// Integer -> float conversions round to nearest.
+//
+// Readings where the paper is silent (each also listed in the design notes):
+//  * Eq. 6 with the configuration's coefficients: T_pf(N,C) =
+//    ((((a0 + a1 N) + a2 (N C)) + a3 (N N)) + a4 C) + a5 (C C); a4, a5 are the Section 5.3
+//    empirical C and C^2 terms.
+//  * Capacity guard (Alg. 1 CapacityCandidates): b + qr + 1 <= B_max and S + L <= M_KV.
+//  * Eq. 8 is tested as (W - W_min) <= eta * Z (no division); Z <= 0 keeps all of A.
+//  * TPOT, configuration form: ((b0 + b1 B) + b2 S') f + g_q (q + n), B = b + qr + 1, S' = S + L,
+//    f = EMA factor of B's decode-batch segment (Section 5.3).  Paper form (Eq. 9):
+//    ((b0 + b1 B) + b2 S') f + [b + qr > 0] T_pf(n,c) / max(1, L_out).
+//  * TTFT (Eq. 4): T_pf(n,c) + (a0 qr + a1 q), overhead neglected; the budget is
+//    max(target, T_pf(L,0)) (Section 7.1 Metrics); TTFT uses <=, TPOT uses strict < (Alg. 1).
+//  * Packing key D-C-Q (Section 5.5, Table 4): more decoding b, then more cached blocks h, then
+//    fewer queued requests qr, then the lowest instance id.  Fallback CacheAwareLB = LMetric
+//    (Section 6, Section 7.1 Baselines): min over C of (q + n)(b + qr + 1), lowest id on ties.
+
+#include <cstdint>
+#include <cstring>
+#include <vector>
+#include <unordered_set>
+#include <unordered_map>
+#include <algorithm>
+
+extern "C" {
+
+typedef struct {
+  float a0, a1, a2, a3, a4, a5;    // Eq. 6 (+ Section 5.3 C, C^2 terms)
+  float b0, b1, b2;                // Eq. 7
+  float g_q;                       // TPOT per queued prefill token (configuration form)
+  float eta;                       // recompute budget (Eq. 8)
+  float lout_median;               // Eq. 9 amortisation length
+  int32_t interference_mode;       // 0 configuration form, 1 paper Eq. 9 form
+  int32_t ttft_filter;             // 1: TTFT test in the admission set, 0: Alg. 1 exactly
+  int32_t nseg;                    // decode-batch segments of the EMA factor table
+  int32_t seg_lo[16];              // segment s covers B >= seg_lo[s] (ascending)
+  float ema_factor[16];
+} orc_model;
+
+typedef struct { int32_t b, qr; int64_t q, S, M_KV; int32_t B_max; } orc_inst;
+
+}  // extern "C"
+
+namespace {
+
+struct BlockMeta { uint64_t parent; uint32_t children; uint32_t last_use; };
+
+struct Oracle {
+  uint32_t I;
+  orc_model m;
+  std::vector<std::unordered_set<uint64_t>> cache;
+  std::vector<orc_inst> st;
+  // Leaf-first LRU bookkeeping (streaming windows only): per instance, block -> metadata.
+  bool track = false;
+  std::vector<std::unordered_map<uint64_t, BlockMeta>> meta;
+};
+
+// Eq. 6 in the fixed order above.
+float t_pf(const orc_model& m, float N, float C) {
+  float t = m.a0 + m.a1 * N;
+  t = t + m.a2 * (N * C);
+  t = t + m.a3 * (N * N);
+  t = t + m.a4 * C;
+  t = t + m.a5 * (C * C);
+  return t;
+}
+
+// Hit length: cached prefix blocks of the chain on instance i (Section 6 prefix-tree lookup).
+uint64_t hit_len(const Oracle& o, uint32_t i, const uint64_t* chain, uint64_t nb) {
+  uint64_t h = 0;
+  while (h < nb && o.cache[i].count(chain[h])) ++h;
+  return h;
+}
+
+float ema_factor(const orc_model& m, int64_t B) {
+  int s = 0;
+  for (int k = 0; k < m.nseg; ++k)
+    if ((int64_t)m.seg_lo[k] <= B) s = k;
+  return m.ema_factor[s];
+}
+
+struct Row {
+  std::vector<uint64_t> hit;
+  std::vector<float> tpot, ttft;
+  std::vector<uint8_t> cls;    // 0: in T, 1: in C \ T, 2: in A \ C, 3: not in A
+  int32_t pick = -1;
+  uint8_t path = 2;            // 0 packed (from T), 1 fallback (LMetric over C), 2 reject
+};
+
+// Algorithm 1 for one request against the current caches and state.
+void decide(const Oracle& o, const uint64_t* chain, uint64_t nb, uint32_t L, float ttft_target,
+            float tpot_target, Row& row) {
+  const orc_model& m = o.m;
+  const uint32_t I = o.I;
+  row.hit.assign(I, 0); row.tpot.assign(I, 0.f); row.ttft.assign(I, 0.f); row.cls.assign(I, 3);
+  row.pick = -1; row.path = 2;
+  const float Lf = (float)L;
+  const float t_cached = t_pf(m, 0.0f, Lf);       // fully cached input
+  const float t_cold = t_pf(m, Lf, 0.0f);         // fully uncached input
+  const float Z = t_cold - t_cached;              // CacheBenefit (Alg. 1, Section 5.4)
+  const float etaZ = m.eta * Z;
+  const float ttft_budget = t_cold > ttft_target ? t_cold : ttft_target;
+  std::vector<float> W(I, 0.f), tpf(I, 0.f);
+  std::vector<int64_t> n_tok(I, 0);
+  std::vector<char> inA(I, 0);
+  bool anyA = false;
+  float Wmin = 0.f;
+  // Capacity guard + RecomputeCost (Alg. 1, KVC-first filtering; Section 5.4).
+  for (uint32_t i = 0; i < I; ++i) {
+    const orc_inst& s = o.st[i];
+    uint64_t h = hit_len(o, i, chain, nb);
+    row.hit[i] = h;
+    int64_t c = 16 * (int64_t)h;
+    int64_t n = (int64_t)L - c;
+    n_tok[i] = n;
+    tpf[i] = t_pf(m, (float)n, (float)c);
+    W[i] = tpf[i] - t_cached;
+    inA[i] = ((int64_t)s.b + s.qr + 1 <= (int64_t)s.B_max) && (s.S + (int64_t)L <= s.M_KV);
+    if (inA[i]) {
+      if (!anyA || W[i] < Wmin) Wmin = W[i];
+      anyA = true;
+    }
+    // Predicted latencies for every instance (Eq. 4, Eq. 7, Eq. 9 / configuration form).
+    const int64_t Bp = (int64_t)s.b + s.qr + 1;
+    const int64_t Sp = s.S + (int64_t)L;
+    const float f = ema_factor(m, Bp);
+    float dec = m.b0 + m.b1 * (float)Bp;
+    dec = dec + m.b2 * (float)Sp;
+    dec = dec * f;
+    float tp;
+    if (m.interference_mode == 0) {
+      tp = dec + m.g_q * (float)(s.q + n);
+    } else {
+      const float den = m.lout_median > 1.0f ? m.lout_median : 1.0f;
+      const float interf = ((int64_t)s.b + s.qr > 0) ? tpf[i] / den : 0.0f;
+      tp = dec + interf;
+    }
+    const float tq = m.a0 * (float)s.qr + m.a1 * (float)s.q;
+    row.tpot[i] = tp;
+    row.ttft[i] = tpf[i] + tq;
+  }
+  if (!anyA) return;  // Reject (Alg. 1: A empty)
+  // Normalised recompute filter, Eq. 8; SLO admission (Alg. 1 TPOT filter, plus TTFT budget).
+  bool anyT = false;
+  for (uint32_t i = 0; i < I; ++i) {
+    if (!inA[i]) continue;
+    bool inC = (Z > 0.0f) ? ((W[i] - Wmin) <= etaZ) : true;
+    if (!inC) { row.cls[i] = 2; continue; }
+    bool ok = row.tpot[i] < tpot_target;
+    if (m.ttft_filter) ok = ok && (row.ttft[i] <= ttft_budget);
+    row.cls[i] = ok ? 0 : 1;
+    anyT = anyT || ok;
+  }
+  int32_t best = -1;
+  if (anyT) {
+    // Decode-batch-size-centric key: more decoding, more cached, fewer queued, lowest id.
+    for (uint32_t i = 0; i < I; ++i) {
+      if (row.cls[i] != 0) continue;
+      if (best < 0) { best = (int32_t)i; continue; }
+      const orc_inst& a = o.st[i];
+      const orc_inst& z = o.st[best];
+      bool better;
+      if (a.b != z.b) better = a.b > z.b;
+      else if (row.hit[i] != row.hit[best]) better = row.hit[i] > row.hit[best];
+      else better = a.qr < z.qr;
+      if (better) best = (int32_t)i;
+    }
+    row.pick = best; row.path = 0;
+  } else {
+    // CacheAwareLB = LMetric over C: pending uncached prefill tokens x active requests,
+    // both including the arriving request.
+    uint64_t bestv = 0;
+    for (uint32_t i = 0; i < I; ++i) {
+      if (row.cls[i] != 1) continue;
+      const orc_inst& s = o.st[i];
+      uint64_t v = (uint64_t)(s.q + n_tok[i]) * (uint64_t)((int64_t)s.b + s.qr + 1);
+      if (best < 0 || v < bestv) { best = (int32_t)i; bestv = v; }
+    }
+    row.pick = best; row.path = best >= 0 ? 1 : 2;
+  }
+}
+
+void insert_block(Oracle& o, uint32_t i, uint64_t h, uint64_t parent, uint32_t last_use) {
+  bool added = o.cache[i].insert(h).second;
+  if (!o.track) return;
+  auto& mm = o.meta[i];
+  if (added) {
+    mm[h] = BlockMeta{parent, 0, last_use};
+    if (parent) {
+      auto it = mm.find(parent);
+      if (it != mm.end()) it->second.children += 1;
+    }
+  } else {
+    auto it = mm.find(h);
+    if (it != mm.end() && it->second.last_use < last_use) it->second.last_use = last_use;
+  }
+}
+
+}  // namespace
+
+extern "C" {
+
+void* orc_create(uint32_t I, const orc_model* m, int32_t track_lru) {
+  if (!m || m->nseg < 1 || m->nseg > 16) return nullptr;
+  Oracle* o = new Oracle();
+  o->I = I;
+  o->m = *m;
+  o->cache.resize(I);
+  o->st.assign(I, orc_inst{0, 0, 0, 0, 0, 0});
+  o->track = track_lru != 0;
+  if (o->track) o->meta.resize(I);
+  return o;
+}
+
+void orc_destroy(void* h) { delete static_cast<Oracle*>(h); }
+
+void orc_reserve(void* h, uint32_t inst, uint64_t n) {
+  Oracle* o = static_cast<Oracle*>(h);
+  o->cache[inst].reserve(n);
+  if (o->track) o->meta[inst].reserve(n);
+}
+
+// Insert n chained blocks into instance inst: block 0's parent is `parent` (0 = root), block k's
+// parent is block k-1.
+void orc_insert_chain(void* h, uint32_t inst, const uint64_t* chain, uint64_t n, uint64_t parent,
+                      uint32_t last_use) {
+  Oracle* o = static_cast<Oracle*>(h);
+  for (uint64_t k = 0; k < n; ++k) insert_block(*o, inst, chain[k], k ? chain[k - 1] : parent, last_use);
+}
+
+// Bulk form of the above over a CSR of chains.
+void orc_insert_chains(void* h, uint64_t nchains, const uint32_t* inst, const uint64_t* off,
+                       const uint64_t* hash, const uint64_t* parent, uint32_t last_use) {
+  for (uint64_t c = 0; c < nchains; ++c)
+    orc_insert_chain(h, inst[c], hash + off[c], off[c + 1] - off[c], parent[c], last_use);
+}
+
+uint64_t orc_cached_blocks(void* h, uint32_t inst) {
+  return static_cast<Oracle*>(h)->cache[inst].size();
+}
+
+int32_t orc_contains(void* h, uint32_t inst, uint64_t block) {
+  return static_cast<Oracle*>(h)->cache[inst].count(block) ? 1 : 0;
+}
+
+void orc_set_state(void* h, const orc_inst* s) {
+  Oracle* o = static_cast<Oracle*>(h);
+  std::memcpy(o->st.data(), s, sizeof(orc_inst) * o->I);
+}
+
+void orc_get_state(void* h, orc_inst* s) {
+  Oracle* o = static_cast<Oracle*>(h);
+  std::memcpy(s, o->st.data(), sizeof(orc_inst) * o->I);
+}
+
+uint64_t orc_hit(void* h, uint32_t inst, const uint64_t* chain, uint64_t nb) {
+  return hit_len(*static_cast<Oracle*>(h), inst, chain, nb);
+}
+
+// Hit lengths of selected (request, instance) pairs.
+void orc_hit_pairs(void* h, const uint64_t* off, const uint64_t* hash, uint64_t npairs,
+                   const uint32_t* req, const uint32_t* inst, uint32_t* out) {
+  Oracle* o = static_cast<Oracle*>(h);
+  for (uint64_t k = 0; k < npairs; ++k) {
+    const uint64_t* ch = hash + off[req[k]];
+    out[k] = (uint32_t)hit_len(*o, inst[k], ch, off[req[k] + 1] - off[req[k]]);
+  }
+}
+
+// Score mode: each listed request against the current state, independently (no state change).
+// Outputs are row-major [nrows x I]; any output pointer may be null.
+void orc_score_rows(void* h, const uint64_t* off, const uint64_t* hash, const uint32_t* L,
+                    const float* ttft_target, const float* tpot_target, uint64_t nrows,
+                    const uint32_t* rows, uint32_t* hits, float* tpot, float* ttft, uint8_t* cls,
+                    int32_t* best, uint8_t* path) {
+  Oracle* o = static_cast<Oracle*>(h);
+  Row row;
+  for (uint64_t k = 0; k < nrows; ++k) {
+    uint32_t r = rows[k];
+    decide(*o, hash + off[r], off[r + 1] - off[r], L[r], ttft_target[r], tpot_target[r], row);
+    for (uint32_t i = 0; i < o->I; ++i) {
+      size_t x = (size_t)k * o->I + i;
+      if (hits) hits[x] = (uint32_t)row.hit[i];
+      if (tpot) tpot[x] = row.tpot[i];
+      if (ttft) ttft[x] = row.ttft[i];
+      if (cls) cls[x] = row.cls[i];
+    }
+    if (best) best[k] = row.pick;
+    if (path) path[k] = row.path;
+  }
+}
+
+// Greedy in-window assignment: requests in arrival order, each decided by Algorithm 1 on the
+// state left by all earlier decisions; an admitted request adds qr += 1, q += n, S += L on its
+// instance and its uncached blocks chain[h..nb) to that instance's cache.  `hit_chosen` receives
+// the hit length on the chosen instance (0 on reject).  window_id stamps LRU use times.
+void orc_schedule(void* h, uint32_t R, const uint64_t* off, const uint64_t* hash, const uint32_t* L,
+                  const float* ttft_target, const float* tpot_target, int32_t* assign,
+                  uint8_t* path, uint32_t* hit_chosen, uint32_t window_id) {
+  Oracle* o = static_cast<Oracle*>(h);
+  Row row;
+  for (uint32_t r = 0; r < R; ++r) {
+    const uint64_t* ch = hash + off[r];
+    const uint64_t nb = off[r + 1] - off[r];
+    decide(*o, ch, nb, L[r], ttft_target[r], tpot_target[r], row);
+    if (assign) assign[r] = row.pick;
+    if (path) path[r] = row.path;
+    if (hit_chosen) hit_chosen[r] = row.pick >= 0 ? (uint32_t)row.hit[row.pick] : 0;
+    if (row.pick < 0) continue;
+    const uint32_t j = (uint32_t)row.pick;
+    const uint64_t hj = row.hit[j];
+    orc_inst& s = o->st[j];
+    s.qr += 1;
+    s.q += (int64_t)L[r] - 16 * (int64_t)hj;
+    s.S += (int64_t)L[r];
+    if (o->track) {
+      for (uint64_t k = 0; k < hj; ++k) {
+        auto it = o->meta[j].find(ch[k]);
+        if (it != o->meta[j].end() && it->second.last_use < window_id) it->second.last_use = window_id;
+      }
+    }
+    for (uint64_t k = hj; k < nb; ++k) insert_block(*o, j, ch[k], k ? ch[k - 1] : 0, window_id);
+  }
+}
+
+}  // extern "C"
