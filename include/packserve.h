@@ -1,0 +1,244 @@
+/*
+ * packserve.h -- C ABI of the GB300 scheduler hot path of PackServe (KVC-first, SLO-aware request
+ * packing for agentic LLM serving, arXiv 2609.33224).
+ *
+ * For a window of requests against every serving instance the library computes, on one GPU:
+ *   1. the KV-cache prefix-hit length of each (request, instance) pair (Section 6: the scheduler's
+ *      prefix tree of cached prefixes, here per-instance hash tables of chained block hashes);
+ *   2. predicted TTFT and TPOT from the white-box prefill/decode model (Eq. 4-7, Eq. 9);
+ *   3. the capacity guard, the normalised recompute filter (Eq. 8) and the SLO admission test
+ *      (Algorithm 1), and the decode-batch-size-centric packing key or the cache-aware fallback;
+ *   4. the greedy in-window assignment: requests in arrival order, each decided on the state left
+ *      by the earlier decisions of the window (Section 4: state tracked along request paths).
+ *
+ * Conventions (all calls):
+ *   - Every call returns a ps_status; on failure ps_last_error() describes the first error.
+ *   - Calls are ordered on the context's CUDA stream and return after their results are in the
+ *     caller's buffers (they synchronise the stream), so device-side errors surface in the same call.
+ *   - Caller buffers are host memory unless the call's *_on_device flag says device memory of the
+ *     context's device.  The caller owns them; the library never keeps a pointer to a host buffer.
+ *     Host buffers that are page-locked (cudaHostAlloc / torch pin_memory) copy fastest.
+ *   - The library owns its tables, instance state and scratch, all allocated in ps_create and
+ *     released in ps_destroy.  One context must not be used from two threads at once.
+ *   - Block hashes are 64-bit chained hashes: block k's hash covers the request's first 16(k+1)
+ *     tokens, so a cached block hash means its whole prefix is cached.  The values 0 and
+ *     0xFFFFFFFFFFFFFFFF are reserved (empty / deleted slot): ps_insert_* rejects them and a request
+ *     block with either value never counts as cached.
+ *   - Instance ids are 0..num_instances-1; ties are broken towards the lowest id.
+ */
+#ifndef PACKSERVE_H
+#define PACKSERVE_H
+
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define PS_API __attribute__((visibility("default")))
+#else
+#define PS_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct ps_ctx ps_ctx; /* opaque, owned by the library */
+
+typedef enum {
+  PS_OK = 0,
+  PS_ERR_INVALID = 1,    /* bad argument, size or layout; nothing was changed */
+  PS_ERR_CUDA = 2,       /* a CUDA runtime call failed (message in ps_last_error) */
+  PS_ERR_OOM = 3,        /* device or pinned allocation failed in ps_create */
+  PS_ERR_TABLE_FULL = 4, /* a hash table has no free slot left for an insert */
+  PS_ERR_TIMEOUT = 5,    /* a bounded device-side wait gave up (reserved; no kernel waits today) */
+  PS_ERR_CAPACITY = 6,   /* an instance holds more blocks than its cache capacity */
+  PS_ERR_STATE = 7       /* call out of order (e.g. commit with no pending window) */
+} ps_status;
+
+enum { PS_MAX_EMA_SEGMENTS = 16, PS_BLOCK_TOKENS = 16 };
+
+/* Performance model (Section 5; all times in ms, fp32).
+ * Prefill, Eq. 6 plus the Section 5.3 empirical C and C^2 terms, evaluated in exactly this order:
+ *   T_pf(N, C) = ((((a0 + a1*N) + a2*(N*C)) + a3*(N*N)) + a4*C) + a5*(C*C)
+ * Decode iteration, Eq. 7:  T_iter(B, S) = (b0 + b1*B) + b2*S, scaled by the online EMA factor of
+ * B's decode-batch segment (Section 5.3): segment s covers B >= seg_lo[s] (ascending, seg_lo[0] <= 1).
+ * TPOT (Eq. 5), with B = b + qr + 1 and S = S_tokens + L after admission:
+ *   interference_mode 0:  T_iter * f + g_q * (q_tokens + n)           (queued-prefill form)
+ *   interference_mode 1:  T_iter * f + [b + qr > 0] T_pf(n, c) / max(1, lout_median)   (Eq. 9)
+ * TTFT (Eq. 4, overhead neglected): T_pf(n, c) + (a0*qr + a1*q_tokens).
+ * eta: recompute budget of Eq. 8 (>= 0; the paper's default is 0.5).
+ * ttft_filter: 1 adds "TTFT <= max(ttft_target, T_pf(L, 0))" to the TPOT admission test of
+ * Algorithm 1 (the TTFT SLO of Section 7.1 Metrics); 0 applies Algorithm 1 exactly.
+ * All coefficients must be finite with magnitude <= 1e9; EMA factors finite and > 0. */
+typedef struct {
+  float a0, a1, a2, a3, a4, a5;
+  float b0, b1, b2;
+  float g_q;
+  float eta;
+  float lout_median;
+  int32_t interference_mode;
+  int32_t ttft_filter;
+  int32_t nseg;
+  int32_t seg_lo[PS_MAX_EMA_SEGMENTS];
+  float ema_factor[PS_MAX_EMA_SEGMENTS];
+} ps_model;
+
+/* Context configuration (ps_create).
+ *   device, cuda_stream   CUDA device ordinal and the cudaStream_t to launch on (NULL: the
+ *                         library creates and owns a non-blocking stream).
+ *   num_instances         1..4096.
+ *   max_window_requests   largest R a window may have (1..131072).
+ *   max_window_chain_blocks  largest total chain length (sum over requests) of a window.
+ *   block_tokens          must be 16 (PS_BLOCK_TOKENS).
+ *   cap_blocks            host array [num_instances]: cache capacity of each instance in blocks.
+ *   table_load_factor     slots of instance i = ceil(cap_blocks[i] / table_load_factor), rounded
+ *                         up to 16-slot buckets; (0, 0.95].
+ *   model                 the performance model above. */
+typedef struct {
+  int32_t device;
+  void* cuda_stream;
+  uint32_t num_instances;
+  uint32_t max_window_requests;
+  uint64_t max_window_chain_blocks;
+  uint32_t block_tokens;
+  const uint64_t* cap_blocks;
+  float table_load_factor;
+  ps_model model;
+} ps_config;
+
+/* Scheduler-tracked state of one instance (Section 4 Metadata service; Section 5.5):
+ * b decoding requests, qr queued (not yet decoding) requests, q_tokens queued uncached prefill
+ * tokens, S_tokens KV tokens held by the active requests, M_KV_tokens KV capacity, B_max decode-slot
+ * limit.  Capacity guard of Algorithm 1: b + qr + 1 <= B_max and S_tokens + L <= M_KV_tokens.
+ * Limits: 0 <= b, qr < 2^17; 0 <= q_tokens < 2^40; 0 <= S_tokens, M_KV_tokens < 2^50. */
+typedef struct {
+  int32_t b, qr;
+  int64_t q_tokens, S_tokens, M_KV_tokens;
+  int32_t B_max;
+} ps_instance_state;
+
+/* One window of requests in arrival order (Algorithm 1's request r: a session's token prefix as a
+ * chain of block hashes, plus its SLO targets).
+ *   chain_off      [R+1], chain_off[0] = 0, non-decreasing; request r's chain is
+ *                  chain_hash[chain_off[r] .. chain_off[r+1]).
+ *   chain_hash     [chain_off[R]] block hashes.
+ *   prompt_tokens  [R] input length L_r in tokens; its chain must have exactly L_r / 16 blocks
+ *                  (full blocks only).  L_r < 2^30.
+ *   ttft_target, tpot_target  [R] per-request SLO targets in ms.
+ *   inputs_on_device  0: all arrays are host memory, 1: all are device memory.
+ * A window with device inputs is read in place; its buffers must stay unchanged until the window is
+ * committed or discarded (ps_commit_window / the next ps_schedule_window). */
+typedef struct {
+  uint32_t R;
+  const uint64_t* chain_off;
+  const uint64_t* chain_hash;
+  const uint32_t* prompt_tokens;
+  const float* ttft_target;
+  const float* tpot_target;
+  int32_t inputs_on_device;
+} ps_window;
+
+/* Per-pair and per-request scoring outputs.  Any pointer may be NULL (not wanted).
+ *   hits  [R*I] row-major (request-major) prefix-hit length in blocks.
+ *   tpot, ttft  [R*I] predicted latencies in ms (computed for every pair).
+ *   cls   [R*I] 0: in T (capacity, recompute and SLO tests pass), 1: in C but not T,
+ *               2: in A but filtered by Eq. 8, 3: not capacity-eligible (not in A).
+ *   best  [R] Algorithm 1's pick against the current state, -1 = Reject.
+ *   path  [R] 0: packed (from T), 1: fallback (CacheAwareLB over C), 2: Reject.
+ *   outputs_on_device  0: host buffers, 1: device buffers. */
+typedef struct {
+  uint32_t* hits;
+  float* tpot;
+  float* ttft;
+  uint8_t* cls;
+  int32_t* best;
+  uint8_t* path;
+  int32_t outputs_on_device;
+} ps_scores;
+
+/* Greedy decisions of a window (ps_schedule_window).
+ *   assign      [R] chosen instance, -1 = Reject.
+ *   path        [R] 0 packed, 1 fallback, 2 reject.
+ *   hit_chosen  [R] prefix-hit length (blocks) on the chosen instance at decision time (0 on reject).
+ * Any pointer may be NULL.  outputs_on_device as in ps_scores. */
+typedef struct {
+  int32_t* assign;
+  uint8_t* path;
+  uint32_t* hit_chosen;
+  int32_t outputs_on_device;
+} ps_decisions;
+
+/* Create a context: allocates every table and buffer up front (instance hash tables sized by
+ * cap_blocks / table_load_factor, a window-scoped delta table of 2 * max_window_chain_blocks
+ * slots, window staging and score scratch).  Instances start empty with zero state.
+ * Errors: PS_ERR_INVALID (config), PS_ERR_CUDA, PS_ERR_OOM.  *out is NULL on failure. */
+PS_API ps_status ps_create(const ps_config* cfg, ps_ctx** out);
+
+/* Replace the committed state of all instances (host array of n = num_instances entries).
+ * Discards any pending window.  Errors: PS_ERR_INVALID (n or a field out of range). */
+PS_API ps_status ps_load_instances(ps_ctx* ctx, const ps_instance_state* s, uint32_t n);
+
+/* Read the committed state (host array of n = num_instances entries). */
+PS_API ps_status ps_get_instances(ps_ctx* ctx, ps_instance_state* out, uint32_t n);
+
+/* Read the state a pending window would commit (the committed state updated by each of the
+ * window's admitted requests: qr += 1, q_tokens += n, S_tokens += L).  PS_ERR_STATE if none. */
+PS_API ps_status ps_get_pending_instances(ps_ctx* ctx, ps_instance_state* out, uint32_t n);
+
+/* Cache a chain of n blocks on instance inst (host array): block 0 continues parent_hash (0 = the
+ * chain starts at the root), block k continues block k-1.  Blocks already cached are skipped.
+ * last_use stamps the blocks for LRU bookkeeping.
+ * Errors: PS_ERR_INVALID (inst, reserved hash), PS_ERR_TABLE_FULL (no slot left; the blocks before
+ * the failing one stay cached), PS_ERR_CAPACITY (the instance now holds more than cap_blocks
+ * blocks; the blocks stay cached). */
+PS_API ps_status ps_insert_blocks(ps_ctx* ctx, uint32_t inst, const uint64_t* chain, uint64_t n,
+                           uint64_t parent_hash, uint32_t last_use);
+
+/* Bulk form of ps_insert_blocks over nchains chains in CSR form: chain c goes to instance inst[c],
+ * its blocks are hash[off[c] .. off[c+1]) and its first block continues parent[c].  on_device
+ * selects host (0) or device (1) arrays.  Same errors as ps_insert_blocks. */
+PS_API ps_status ps_insert_chains(ps_ctx* ctx, uint64_t nchains, const uint32_t* inst, const uint64_t* off,
+                           const uint64_t* hash, const uint64_t* parent, uint32_t last_use,
+                           int32_t on_device);
+
+/* Number of blocks cached on each instance (host array [n = num_instances]). */
+PS_API ps_status ps_cached_blocks(ps_ctx* ctx, uint64_t* out, uint32_t n);
+
+/* Score a window: every request independently against the committed state (no state change).
+ * Runs the probe kernel (hit lengths of all R x I pairs) and the fused score kernel (latencies,
+ * filters, packing key and per-request argmin).  Errors: PS_ERR_INVALID (window layout, R too
+ * large, chain length != L/16, total blocks too large), PS_ERR_CUDA. */
+PS_API ps_status ps_score_window(ps_ctx* ctx, const ps_window* w, ps_scores* out);
+
+/* Greedy in-window assignment (Algorithm 1 per request in arrival order, each admitted request
+ * updating its instance's state and caching its blocks there before the next decision).
+ * The result is a pending window: the committed state and caches are unchanged until
+ * ps_commit_window; the next ps_schedule_window or ps_load_instances discards it.
+ * opt_scores (may be NULL) receives the window's independent scores against the committed state
+ * (hits = the hit lengths before the window; best/path as ps_score_window).
+ * Errors: as ps_score_window, plus PS_ERR_TABLE_FULL if the delta table overflowed (cannot happen
+ * within max_window_chain_blocks). */
+PS_API ps_status ps_schedule_window(ps_ctx* ctx, const ps_window* w, ps_decisions* out,
+                             ps_scores* opt_scores);
+
+/* Commit the pending window: the pending state becomes the committed state and each admitted
+ * request's uncached blocks are cached on its instance (stamped last_use).  The window's buffers
+ * are read again here.  Errors: PS_ERR_STATE (no pending window), PS_ERR_TABLE_FULL,
+ * PS_ERR_CAPACITY (as ps_insert_blocks; the commit is still applied). */
+PS_API ps_status ps_commit_window(ps_ctx* ctx, uint32_t last_use);
+
+/* Device time in ms (CUDA events recorded on the context's stream around each kernel) of the last
+ * ps_score_window / ps_schedule_window call and of the commit after it: ms[0] probe, ms[1] fused
+ * score, ms[2] greedy, ms[3] commit; -1 where that kernel did not run.  n must be >= 4. */
+PS_API ps_status ps_last_timings(ps_ctx* ctx, float* ms, uint32_t n);
+
+/* Text of the last error on this context ("" if none).  Valid until the next call. */
+PS_API const char* ps_last_error(const ps_ctx* ctx);
+
+/* Release every resource of the context.  NULL is accepted. */
+PS_API void ps_destroy(ps_ctx* ctx);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* PACKSERVE_H */

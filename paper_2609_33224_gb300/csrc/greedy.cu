@@ -1,0 +1,255 @@
+// Greedy in-window assignment (Algorithm 1 applied to the window's requests in arrival order).
+//
+// The paper's gateway decides each request online and updates the instance records along the
+// request path before the next decision (Section 4, Metadata service; Section 6).  This kernel
+// replays that sequence for a whole window on the GPU: one persistent thread block whose threads
+// each own up to IPT instances.  Per request r:
+//   1. hit of r on instance i = hit0[r][i] (the probe kernel's walk over the committed tables)
+//      extended through the window's delta table: an instance that has received blocks in this
+//      window is re-probed at position hit0 (and walked 32 positions per warp step, over delta and
+//      main, if that block is now cached).  Instances untouched in the window need no probe.
+//   2. the whole row is re-evaluated from the current state (capacity guard, W, W_min, Eq. 8
+//      filter, TPOT/TTFT admission, D-C-Q key or LMetric fallback), reduced block-wide to the pick;
+//   3. the pick's state is updated (qr += 1, q += n, S += L) and its uncached blocks
+//      chain[h..nb) are inserted into the delta table for instance j.
+// Committed tables are never written here; the decisions and the updated state are a pending
+// window that ps_commit_window applies.  No step waits on another block: a single thread block with
+// __syncthreads barriers only.
+#include "ps_internal.cuh"
+
+namespace {
+
+template <int IPT>
+__global__ void __launch_bounds__(1024, 1)
+greedy_kernel(const uint64_t* __restrict__ slots, const psk::TableDesc* __restrict__ tdesc, uint32_t I,
+              psk::WindowDev w, const uint32_t* __restrict__ hit0, psk::StateSoA committed,
+              psk::StateSoA pending, psk::DevModel m, psk::DeltaSlot* delta, uint32_t delta_nbkt,
+              unsigned long long* dlog, unsigned long long* dlog_n, int32_t* __restrict__ assign,
+              uint8_t* __restrict__ path, uint32_t* __restrict__ hit_chosen, uint32_t* err) {
+  extern __shared__ unsigned long long smem_raw[];
+  int64_t* s_q = reinterpret_cast<int64_t*>(smem_raw);
+  int64_t* s_S = s_q + I;
+  int64_t* s_M = s_S + I;
+  int32_t* s_b = reinterpret_cast<int32_t*>(s_M + I);
+  int32_t* s_qr = s_b + I;
+  int32_t* s_Bmax = s_qr + I;
+  uint32_t* s_h = reinterpret_cast<uint32_t*>(s_Bmax + I);
+  uint32_t* s_walk = s_h + I;
+  uint8_t* s_touched = reinterpret_cast<uint8_t*>(s_walk + I);
+  __shared__ float s_red_w[32];
+  __shared__ int s_red_a[32];
+  __shared__ psk::ArgKey s_red_k[32];
+  __shared__ uint32_t s_nwalk;
+
+  const int t = threadIdx.x;
+  const int NT = blockDim.x;
+  const int lane = t & 31;
+  const int warp = t >> 5;
+  const int NW = NT >> 5;
+
+  for (uint32_t i = t; i < I; i += NT) {
+    s_b[i] = committed.b[i];
+    s_qr[i] = committed.qr[i];
+    s_q[i] = committed.q[i];
+    s_S[i] = committed.S[i];
+    s_M[i] = committed.M[i];
+    s_Bmax[i] = committed.Bmax[i];
+    s_touched[i] = 0;
+  }
+  if (t == 0) s_nwalk = 0;
+  uint32_t hn[IPT];
+#pragma unroll
+  for (int k = 0; k < IPT; ++k) {
+    const uint32_t i = t + k * NT;
+    hn[k] = (i < I && w.R > 0) ? __ldg(hit0 + i) : 0u;
+  }
+  __syncthreads();
+
+  for (uint32_t r = 0; r < w.R; ++r) {
+    const uint64_t o = w.off[r];
+    const uint64_t nb = w.off[r + 1] - o;
+    const psk::RowConst rc = psk::row_const(m, w.L[r], w.ttft_t[r], w.tpot_t[r]);
+    uint32_t hc[IPT];
+#pragma unroll
+    for (int k = 0; k < IPT; ++k) {
+      const uint32_t i = t + k * NT;
+      hc[k] = hn[k];
+      if (i < I) {
+        if (s_touched[i] && hc[k] < nb &&
+            psk::delta_contains(delta, delta_nbkt, i, w.hash[o + hc[k]])) {
+          const uint32_t at = atomicAdd(&s_nwalk, 1u);
+          s_walk[at] = i;
+        }
+        s_h[i] = hc[k];
+      }
+    }
+    if (r + 1 < w.R) {
+#pragma unroll
+      for (int k = 0; k < IPT; ++k) {
+        const uint32_t i = t + k * NT;
+        if (i < I) hn[k] = __ldg(hit0 + (uint64_t)(r + 1) * I + i);
+      }
+    }
+    __syncthreads();  // (A) hits staged, walk list complete
+    const uint32_t nwalk = s_nwalk;
+    if (nwalk) {
+      for (uint32_t x = warp; x < nwalk; x += NW) {
+        const uint32_t i = s_walk[x];
+        const psk::TableDesc d = tdesc[i];
+        uint64_t hnew = nb;
+        for (uint64_t base = (uint64_t)s_h[i] + 1; base < nb; base += 32) {
+          const uint64_t k = base + lane;
+          bool present = true;
+          if (k < nb) {
+            const uint64_t key = w.hash[o + k];
+            present = psk::delta_contains(delta, delta_nbkt, i, key) || psk::main_contains(slots, d, key);
+          }
+          const unsigned miss = __ballot_sync(0xffffffffu, !present);
+          if (miss) {
+            hnew = base + (uint64_t)(__ffs(miss) - 1);
+            break;
+          }
+        }
+        if (lane == 0) s_h[i] = (uint32_t)hnew;
+      }
+      __syncthreads();  // (B) extended hits visible
+#pragma unroll
+      for (int k = 0; k < IPT; ++k) {
+        const uint32_t i = t + k * NT;
+        if (i < I) hc[k] = s_h[i];
+      }
+    }
+    // Pass 1: capacity guard and recompute cost; W_min over A.
+    psk::PairEval ev[IPT];
+    float wmin = INFINITY;
+    bool anyA = false;
+#pragma unroll
+    for (int k = 0; k < IPT; ++k) {
+      const uint32_t i = t + k * NT;
+      if (i < I) {
+        ev[k] = psk::eval_pair(m, rc, hc[k], s_b[i], s_qr[i], s_q[i], s_S[i], s_M[i], s_Bmax[i]);
+        if (ev[k].inA) {
+          wmin = fminf(wmin, ev[k].W);
+          anyA = true;
+        }
+      } else {
+        ev[k].inA = false;
+      }
+    }
+    wmin = psk::warp_fmin(wmin);
+    anyA = __any_sync(0xffffffffu, anyA);
+    if (lane == 0) {
+      s_red_w[warp] = wmin;
+      s_red_a[warp] = anyA ? 1 : 0;
+    }
+    __syncthreads();  // (C)
+    wmin = INFINITY;
+    anyA = false;
+    for (int x = 0; x < NW; ++x) {
+      wmin = fminf(wmin, s_red_w[x]);
+      anyA = anyA || (s_red_a[x] != 0);
+    }
+    // Pass 2: admission classes and the lexicographic argmin.
+    psk::ArgKey best{psk::kNoKeyCi, ~0ull};
+#pragma unroll
+    for (int k = 0; k < IPT; ++k) {
+      const uint32_t i = t + k * NT;
+      if (i < I && ev[k].inA) {
+        const uint32_t cls = psk::pair_class(m, rc, ev[k], wmin);
+        if (cls <= 1u) {
+          const psk::ArgKey kk{(cls << 28) | i, psk::pair_value(cls, hc[k], s_b[i], s_qr[i], s_q[i], ev[k].n)};
+          if (psk::key_less(kk, best)) best = kk;
+        }
+      }
+    }
+    best = psk::warp_argmin(best);
+    if (lane == 0) s_red_k[warp] = best;
+    __syncthreads();  // (D)
+    best = s_red_k[0];
+    for (int x = 1; x < NW; ++x)
+      if (psk::key_less(s_red_k[x], best)) best = s_red_k[x];
+    const bool pick = anyA && best.ci != psk::kNoKeyCi;
+    const uint32_t j = best.ci & 0x0FFFFFFFu;
+    const uint32_t hj = pick ? s_h[j] : 0u;
+    if (t == 0) {
+      assign[r] = pick ? (int32_t)j : -1;
+      path[r] = pick ? (uint8_t)(best.ci >> 28) : (uint8_t)2;
+      hit_chosen[r] = hj;
+      if (pick) {
+        s_qr[j] += 1;
+        s_q[j] += (int64_t)rc.L - 16 * (int64_t)hj;
+        s_S[j] += (int64_t)rc.L;
+        s_touched[j] = 1;
+      }
+      s_nwalk = 0;
+    }
+    if (pick) {
+      for (uint64_t k = (uint64_t)hj + t; k < nb; k += NT)
+        if (!psk::delta_insert(delta, delta_nbkt, j, w.hash[o + k], dlog, dlog_n)) atomicOr(err, psk::kErrDeltaFull);
+    }
+    __syncthreads();  // (E) state, delta and walk counter ready for the next request
+  }
+  for (uint32_t i = t; i < I; i += NT) {
+    pending.b[i] = s_b[i];
+    pending.qr[i] = s_qr[i];
+    pending.q[i] = s_q[i];
+    pending.S[i] = s_S[i];
+    pending.M[i] = s_M[i];
+    pending.Bmax[i] = s_Bmax[i];
+  }
+}
+
+__global__ void delta_clear_kernel(psk::DeltaSlot* delta, const unsigned long long* dlog,
+                                   const unsigned long long* dlog_n, uint64_t max_entries) {
+  uint64_t n = *dlog_n;
+  if (n > max_entries) n = max_entries;
+  for (uint64_t x = blockIdx.x * (uint64_t)blockDim.x + threadIdx.x; x < n; x += (uint64_t)gridDim.x * blockDim.x)
+    delta[dlog[x]].hash = psk::kEmpty;
+}
+
+size_t greedy_smem(uint32_t I) {
+  return (size_t)I * (3 * sizeof(int64_t) + 3 * sizeof(int32_t) + 2 * sizeof(uint32_t) + 1) + 16;
+}
+
+}  // namespace
+
+namespace pskl {
+
+cudaError_t launch_greedy(const uint64_t* slots, const psk::TableDesc* tdesc, uint32_t I,
+                          const psk::WindowDev& w, const uint32_t* hit0, psk::StateSoA committed,
+                          psk::StateSoA pending, const psk::DevModel& m, psk::DeltaSlot* delta,
+                          uint32_t delta_nbkt, unsigned long long* dlog, unsigned long long* dlog_n,
+                          int32_t* assign, uint8_t* path, uint32_t* hit_chosen, uint32_t* err,
+                          cudaStream_t s) {
+  uint32_t nt = (I + 31) / 32 * 32;
+  if (nt > 1024) nt = 1024;
+  const uint32_t ipt = (I + nt - 1) / nt;
+  const size_t smem = greedy_smem(I);
+  if (ipt <= 1) {
+    cudaFuncSetAttribute(greedy_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    greedy_kernel<1><<<1, nt, smem, s>>>(slots, tdesc, I, w, hit0, committed, pending, m, delta, delta_nbkt,
+                                         dlog, dlog_n, assign, path, hit_chosen, err);
+  } else if (ipt <= 2) {
+    cudaFuncSetAttribute(greedy_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    greedy_kernel<2><<<1, nt, smem, s>>>(slots, tdesc, I, w, hit0, committed, pending, m, delta, delta_nbkt,
+                                         dlog, dlog_n, assign, path, hit_chosen, err);
+  } else if (ipt <= 4) {
+    cudaFuncSetAttribute(greedy_kernel<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    greedy_kernel<4><<<1, nt, smem, s>>>(slots, tdesc, I, w, hit0, committed, pending, m, delta, delta_nbkt,
+                                         dlog, dlog_n, assign, path, hit_chosen, err);
+  } else {
+    return cudaErrorInvalidValue;
+  }
+  return cudaGetLastError();
+}
+
+cudaError_t launch_delta_clear(psk::DeltaSlot* delta, const unsigned long long* dlog,
+                               unsigned long long* dlog_n, uint64_t max_entries, int num_sms,
+                               cudaStream_t s) {
+  delta_clear_kernel<<<num_sms * 4, 256, 0, s>>>(delta, dlog, dlog_n, max_entries);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  return cudaMemsetAsync(dlog_n, 0, sizeof(unsigned long long), s);
+}
+
+}  // namespace pskl

@@ -1,0 +1,329 @@
+// Device-side data layout and shared device functions of the scheduler library (sm_103a).
+//
+// HBM layout
+//   main tables   one u64 slot array for all instances; instance i owns buckets [0, nbkt_i) starting
+//                 at slot base_i.  A bucket is 16 slots = one 128-byte line.  A key's home bucket
+//                 is fastrange(key, nbkt_i) (the high 64 bits of key * nbkt_i); collisions go to the
+//                 next bucket (linear probing over buckets).  Slot value 0 = empty.
+//   delta table   window-scoped set of (instance, block) pairs cached by the window's own earlier
+//                 decisions: 16-byte slots {hash, instance}, 8 per 128-byte bucket, sized at twice the
+//                 window's block bound so it can never fill.  Cleared (through its insert log) after
+//                 each window.
+//   state         structure of arrays per instance (b, qr, q, S, M_KV, B_max).
+//   hits          u32 [R x I], request-major.
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+
+namespace psk {
+
+constexpr uint64_t kEmpty = 0ull;
+constexpr uint64_t kTomb = ~0ull;
+constexpr int kBucketSlots = 16;   // main table: 16 x 8 B
+constexpr int kDeltaSlots = 8;     // delta table: 8 x 16 B
+constexpr uint32_t kDeltaNoInst = 0xFFFFFFFFu;
+
+// Device error bits, OR-ed into one word per context and turned into a ps_status on the host.
+enum : uint32_t {
+  kErrTableFull = 1u,
+  kErrReservedHash = 2u,
+  kErrDeltaFull = 4u,
+  kErrWindowLayout = 8u,
+  kErrBadInstance = 16u,
+};
+
+struct TableDesc {
+  uint64_t base;   // first slot of the instance's table
+  uint32_t nbkt;   // buckets
+  uint32_t pad;
+};
+
+struct DeltaSlot {
+  unsigned long long hash;
+  unsigned int inst;
+  unsigned int pad;
+};
+
+struct DevModel {
+  float a0, a1, a2, a3, a4, a5, b0, b1, b2, g_q, eta, lout;
+  int32_t interference_mode, ttft_filter, nseg;
+  int32_t seg_lo[16];
+  float ema[16];
+};
+
+struct StateSoA {
+  int32_t* b;
+  int32_t* qr;
+  int64_t* q;
+  int64_t* S;
+  int64_t* M;
+  int32_t* Bmax;
+};
+
+struct WindowDev {
+  const uint64_t* off;
+  const uint64_t* hash;
+  const uint32_t* L;
+  const float* ttft_t;
+  const float* tpot_t;
+  uint32_t R;
+};
+
+__device__ __forceinline__ uint32_t fastrange32(uint64_t h, uint32_t n) {
+  return (uint32_t)__umul64hi(h, (unsigned long long)n);
+}
+
+// Membership in an instance's main table.  Read-only during every kernel that calls it, so the
+// non-coherent read-only path is used.  A probe reads whole 128-byte buckets as 8 x 16-byte loads.
+__device__ __forceinline__ bool main_contains(const uint64_t* __restrict__ slots, const TableDesc d,
+                                              uint64_t key) {
+  if (key == kEmpty || key == kTomb) return false;
+  uint32_t b = fastrange32(key, d.nbkt);
+  for (uint32_t p = 0; p < d.nbkt; ++p) {
+    const ulonglong2* line = reinterpret_cast<const ulonglong2*>(slots + d.base + (uint64_t)b * kBucketSlots);
+    bool empty = false;
+#pragma unroll
+    for (int k = 0; k < kBucketSlots / 2; ++k) {
+      const ulonglong2 v = __ldg(line + k);
+      if (v.x == key || v.y == key) return true;
+      empty |= (v.x == kEmpty) | (v.y == kEmpty);
+    }
+    if (empty) return false;
+    b = (b + 1 == d.nbkt) ? 0u : b + 1;
+  }
+  return false;
+}
+
+// Insert into a main table.  Returns 1 if inserted, 0 if already present, -1 if the table is full.
+// Concurrent inserts of the same key are safe: they scan the same slot sequence, and a failed CAS
+// that returns the key itself means another thread inserted it.
+__device__ __forceinline__ int main_insert(uint64_t* slots, const TableDesc d, uint64_t key) {
+  uint32_t b = fastrange32(key, d.nbkt);
+  for (uint32_t p = 0; p < d.nbkt; ++p) {
+    unsigned long long* line = reinterpret_cast<unsigned long long*>(slots + d.base + (uint64_t)b * kBucketSlots);
+    for (int k = 0; k < kBucketSlots; ++k) {
+      const unsigned long long v = __ldcg(line + k);
+      if (v == key) return 0;
+      if (v == kEmpty) {
+        const unsigned long long old = atomicCAS(line + k, kEmpty, (unsigned long long)key);
+        if (old == kEmpty) return 1;
+        if (old == key) return 0;
+      }
+    }
+    b = (b + 1 == d.nbkt) ? 0u : b + 1;
+  }
+  return -1;
+}
+
+__device__ __forceinline__ uint32_t delta_home(uint64_t key, uint32_t inst, uint32_t nbkt) {
+  return fastrange32(key ^ ((uint64_t)(inst + 1) * 0x9E3779B97F4A7C15ull), nbkt);
+}
+
+// Membership of (inst, key) in the delta table.  The delta table is written by the same thread
+// block between reads (separated by __syncthreads), so it is read through the coherent path.
+__device__ __forceinline__ bool delta_contains(const DeltaSlot* delta, uint32_t nbkt, uint32_t inst,
+                                               uint64_t key) {
+  if (key == kEmpty || key == kTomb) return false;
+  uint32_t b = delta_home(key, inst, nbkt);
+  for (uint32_t p = 0; p < nbkt; ++p) {
+    const ulonglong2* line = reinterpret_cast<const ulonglong2*>(delta + (uint64_t)b * kDeltaSlots);
+#pragma unroll
+    for (int k = 0; k < kDeltaSlots; ++k) {
+      const ulonglong2 v = __ldcg(line + k);
+      if (v.x == key && (uint32_t)v.y == inst) return true;
+      if (v.x == kEmpty) return false;
+    }
+    b = (b + 1 == nbkt) ? 0u : b + 1;
+  }
+  return false;
+}
+
+// Insert (inst, key) into the delta table; appends the slot index to the clear log.  All concurrent
+// inserts come from one greedy step and target one instance.  Returns false if the table is full.
+__device__ __forceinline__ bool delta_insert(DeltaSlot* delta, uint32_t nbkt, uint32_t inst, uint64_t key,
+                                             unsigned long long* log, unsigned long long* log_n) {
+  if (key == kEmpty || key == kTomb) return true;
+  uint32_t b = delta_home(key, inst, nbkt);
+  for (uint32_t p = 0; p < nbkt; ++p) {
+    DeltaSlot* line = delta + (uint64_t)b * kDeltaSlots;
+    for (int k = 0; k < kDeltaSlots; ++k) {
+      const unsigned long long h = __ldcg(&line[k].hash);
+      if (h == key && __ldcg(&line[k].inst) == inst) return true;
+      if (h == kEmpty) {
+        const unsigned long long old = atomicCAS(&line[k].hash, kEmpty, (unsigned long long)key);
+        if (old == kEmpty) {
+          line[k].inst = inst;
+          const unsigned long long at = atomicAdd(log_n, 1ull);
+          log[at] = (uint64_t)b * kDeltaSlots + k;
+          return true;
+        }
+        if (old == key && __ldcg(&line[k].inst) == inst) return true;
+      }
+    }
+    b = (b + 1 == nbkt) ? 0u : b + 1;
+  }
+  return false;
+}
+
+// ---------------------------------------------------------------------------- performance model --
+// Every operation is an explicitly rounded fp32 intrinsic in the order the header documents, so
+// nothing is fused or reassociated.
+
+// Eq. 6 with the Section 5.3 empirical C and C^2 terms.
+__device__ __forceinline__ float t_pf(const DevModel& m, float N, float C) {
+  float t = __fadd_rn(m.a0, __fmul_rn(m.a1, N));
+  t = __fadd_rn(t, __fmul_rn(m.a2, __fmul_rn(N, C)));
+  t = __fadd_rn(t, __fmul_rn(m.a3, __fmul_rn(N, N)));
+  t = __fadd_rn(t, __fmul_rn(m.a4, C));
+  t = __fadd_rn(t, __fmul_rn(m.a5, __fmul_rn(C, C)));
+  return t;
+}
+
+// Per-request constants of Algorithm 1 and Eq. 8.
+struct RowConst {
+  float t_cached;     // T_pf(0, L): fully cached input
+  float Z;            // CacheBenefit: T_pf(L, 0) - T_pf(0, L)
+  float etaZ;         // eta * Z
+  float ttft_budget;  // max(target, T_pf(L, 0))
+  float tpot_target;
+  uint32_t L;
+};
+
+__device__ __forceinline__ RowConst row_const(const DevModel& m, uint32_t L, float ttft_t, float tpot_t) {
+  RowConst rc;
+  const float Lf = __uint2float_rn(L);
+  rc.t_cached = t_pf(m, 0.0f, Lf);
+  const float t_cold = t_pf(m, Lf, 0.0f);
+  rc.Z = __fsub_rn(t_cold, rc.t_cached);
+  rc.etaZ = __fmul_rn(m.eta, rc.Z);
+  rc.ttft_budget = t_cold > ttft_t ? t_cold : ttft_t;
+  rc.tpot_target = tpot_t;
+  rc.L = L;
+  return rc;
+}
+
+struct PairEval {
+  float W, tpot, ttft;
+  int64_t n;   // uncached tokens
+  bool inA;    // capacity-eligible
+};
+
+__device__ __forceinline__ float ema_factor(const DevModel& m, int64_t B) {
+  int s = 0;
+  for (int k = 0; k < m.nseg; ++k)
+    if ((int64_t)m.seg_lo[k] <= B) s = k;
+  return m.ema[s];
+}
+
+// RecomputeCost, capacity guard and the latency predictions of one (request, instance) pair.
+__device__ __forceinline__ PairEval eval_pair(const DevModel& m, const RowConst& rc, uint32_t h,
+                                              int32_t b, int32_t qr, int64_t q, int64_t S, int64_t M,
+                                              int32_t Bmax) {
+  PairEval e;
+  const int64_t c = 16 * (int64_t)h;
+  const int64_t n = (int64_t)rc.L - c;
+  const float tpf = t_pf(m, __ll2float_rn(n), __ll2float_rn(c));
+  e.n = n;
+  e.W = __fsub_rn(tpf, rc.t_cached);
+  const int64_t Bp = (int64_t)b + qr + 1;
+  const int64_t Sp = S + (int64_t)rc.L;
+  e.inA = (Bp <= (int64_t)Bmax) && (Sp <= M);
+  float dec = __fadd_rn(m.b0, __fmul_rn(m.b1, __ll2float_rn(Bp)));
+  dec = __fadd_rn(dec, __fmul_rn(m.b2, __ll2float_rn(Sp)));
+  dec = __fmul_rn(dec, ema_factor(m, Bp));
+  if (m.interference_mode == 0) {
+    e.tpot = __fadd_rn(dec, __fmul_rn(m.g_q, __ll2float_rn(q + n)));
+  } else {
+    const float den = m.lout > 1.0f ? m.lout : 1.0f;
+    const float interf = ((int64_t)b + qr > 0) ? __fdiv_rn(tpf, den) : 0.0f;
+    e.tpot = __fadd_rn(dec, interf);
+  }
+  const float tq = __fadd_rn(__fmul_rn(m.a0, __int2float_rn(qr)), __fmul_rn(m.a1, __ll2float_rn(q)));
+  e.ttft = __fadd_rn(tpf, tq);
+  return e;
+}
+
+// Class of a capacity-eligible pair once W_min is known (Eq. 8, Alg. 1 TPOT filter + TTFT budget):
+// 0 in T, 1 in C \ T, 2 filtered by the recompute budget.
+__device__ __forceinline__ uint32_t pair_class(const DevModel& m, const RowConst& rc, const PairEval& e,
+                                               float Wmin) {
+  const bool inC = (rc.Z > 0.0f) ? (__fsub_rn(e.W, Wmin) <= rc.etaZ) : true;
+  if (!inC) return 2u;
+  bool ok = e.tpot < rc.tpot_target;
+  if (m.ttft_filter) ok = ok && (e.ttft <= rc.ttft_budget);
+  return ok ? 0u : 1u;
+}
+
+// Ordering value inside a class.  Class 0 (Section 5.5, D-C-Q): more decoding requests, then more
+// cached blocks, then fewer queued requests: (2^18-1-b) | (2^26-1-h) | qr in 18/26/18 bits.
+// Class 1 (CacheAwareLB = LMetric): (q + n) * (b + qr + 1) as an unsigned 64-bit product.
+__device__ __forceinline__ uint64_t pair_value(uint32_t cls, uint32_t h, int32_t b, int32_t qr, int64_t q,
+                                               int64_t n) {
+  if (cls == 0u)
+    return ((uint64_t)((1u << 18) - 1u - (uint32_t)b) << 44) |
+           ((uint64_t)((1u << 26) - 1u - h) << 18) | (uint64_t)(uint32_t)qr;
+  return (uint64_t)(q + n) * (uint64_t)((int64_t)b + qr + 1);
+}
+
+// Lexicographic (class, value, instance) argmin element; ci packs class << 28 | instance.
+struct ArgKey {
+  uint32_t ci;
+  uint64_t v;
+};
+
+__device__ __forceinline__ bool key_less(const ArgKey& a, const ArgKey& z) {
+  const uint32_t ca = a.ci >> 28, cz = z.ci >> 28;
+  if (ca != cz) return ca < cz;
+  if (a.v != z.v) return a.v < z.v;
+  return (a.ci & 0x0FFFFFFFu) < (z.ci & 0x0FFFFFFFu);
+}
+
+__device__ __forceinline__ ArgKey warp_argmin(ArgKey k) {
+#pragma unroll
+  for (int s = 16; s > 0; s >>= 1) {
+    ArgKey o;
+    o.ci = __shfl_xor_sync(0xffffffffu, k.ci, s);
+    o.v = __shfl_xor_sync(0xffffffffu, k.v, s);
+    if (key_less(o, k)) k = o;
+  }
+  return k;
+}
+
+__device__ __forceinline__ float warp_fmin(float x) {
+#pragma unroll
+  for (int s = 16; s > 0; s >>= 1) x = fminf(x, __shfl_xor_sync(0xffffffffu, x, s));
+  return x;
+}
+
+constexpr uint32_t kNoKeyCi = 0xFFFFFFFFu;  // class 15: worse than any real pair
+
+}  // namespace psk
+
+// Kernel launchers (one translation unit each).
+namespace pskl {
+cudaError_t launch_probe(const uint64_t* slots, const psk::TableDesc* tdesc, uint32_t I,
+                         const psk::WindowDev& w, uint32_t* hits, int grid, cudaStream_t s);
+int probe_max_grid(uint32_t I, int num_sms);
+cudaError_t launch_score(const uint32_t* hits, psk::StateSoA st, uint32_t I, const psk::WindowDev& w,
+                         const psk::DevModel& m, float* tpot, float* ttft, uint8_t* cls, int32_t* best,
+                         uint8_t* path, int num_sms, cudaStream_t s);
+cudaError_t launch_greedy(const uint64_t* slots, const psk::TableDesc* tdesc, uint32_t I,
+                          const psk::WindowDev& w, const uint32_t* hit0, psk::StateSoA committed,
+                          psk::StateSoA pending, const psk::DevModel& m, psk::DeltaSlot* delta,
+                          uint32_t delta_nbkt, unsigned long long* dlog, unsigned long long* dlog_n,
+                          int32_t* assign, uint8_t* path, uint32_t* hit_chosen, uint32_t* err,
+                          cudaStream_t s);
+cudaError_t launch_delta_clear(psk::DeltaSlot* delta, const unsigned long long* dlog,
+                               unsigned long long* dlog_n, uint64_t max_entries, int num_sms,
+                               cudaStream_t s);
+cudaError_t launch_insert_chains(uint64_t* slots, const psk::TableDesc* tdesc, uint32_t I,
+                                 unsigned long long* count, uint64_t nchains, const uint32_t* inst,
+                                 const uint64_t* off, const uint64_t* hash, uint64_t total,
+                                 uint32_t* err, int num_sms, cudaStream_t s);
+cudaError_t launch_commit(uint64_t* slots, const psk::TableDesc* tdesc, uint32_t I,
+                          unsigned long long* count, const psk::WindowDev& w, const int32_t* assign,
+                          const uint32_t* hit_chosen, uint32_t* err, int num_sms, cudaStream_t s);
+cudaError_t launch_validate_window(const psk::WindowDev& w, uint64_t max_blocks, uint32_t* err,
+                                   cudaStream_t s);
+}  // namespace pskl
