@@ -112,12 +112,50 @@ class ClockSampler:
                 "samples": len(sm)}
 
 
-def probe_algorithmic_bytes(hits: np.ndarray, nb: np.ndarray) -> int:
-    """Bytes the linear probe walk must move per launch: one 32-byte sector per probed position
-    (positions 0..h, capped at the chain length), the chain read once per request, the u32 hit
-    written per pair."""
-    probes = np.minimum(hits.astype(np.int64) + 1, nb[:, None]).sum()
-    return int(32 * probes + 8 * nb.sum() + 4 * hits.size)
+def search_probe_count(h: np.ndarray, nb: np.ndarray) -> np.ndarray:
+    """Probes the 32-ary first-miss search makes for hit h on a chain of nb blocks: 32 per step
+    while the interval spans more than 32 positions, then one probe per remaining position."""
+    h = h.astype(np.int64)
+    lo = np.zeros_like(h)
+    hi = np.broadcast_to(nb, h.shape).astype(np.int64).copy()
+    cnt = np.zeros_like(h)
+    live = np.ones(h.shape, bool)
+    for _ in range(8):
+        span = hi - lo
+        fin = live & (span <= 32)
+        cnt[fin] += span[fin]
+        live &= ~fin
+        if not live.any():
+            break
+        cnt[live] += 32
+        # first j with p_j = lo + (j+1) span / 32 - 1 >= h; none -> done (h = hi)
+        j = np.zeros_like(h)
+        found = np.zeros(h.shape, bool)
+        for jj in range(32):
+            p = lo + ((jj + 1) * span) // 32 - 1
+            hit = live & ~found & (p >= h)
+            j[hit] = jj
+            found |= hit
+        done = live & ~found
+        live &= found
+        newhi = lo + ((j + 1) * span) // 32 - 1
+        newlo = lo + (j * span) // 32
+        hi = np.where(live, newhi, hi)
+        lo = np.where(live, newlo, lo)
+        live &= ~done
+    return cnt
+
+
+def probe_algorithmic_bytes(hits: np.ndarray, nb: np.ndarray, search: bool) -> int:
+    """Bytes the probe kernel's algorithm must move per launch: one 32-byte sector per probed
+    position (linear walk: positions 0..h capped at the chain length; search: the search's own probe
+    count), the chain read once per request, the u32 hit written per pair."""
+    if search:
+        probes = int(sum(search_probe_count(hits[r0:r0 + 512], nb[r0:r0 + 512, None]).sum()
+                         for r0 in range(0, hits.shape[0], 512)))
+    else:
+        probes = int(np.minimum(hits.astype(np.int64) + 1, nb[:, None]).sum())
+    return int(32 * probes + 8 * nb.sum() + 4 * hits.size), probes
 
 
 def oracle_sample(wl, seconds: float, max_rows: int | None = None):
@@ -203,6 +241,7 @@ def main():
     ap.add_argument("--tpot", type=float, default=None)
     ap.add_argument("--cpu-seconds", type=float, default=20.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--probe-mode", type=int, default=1, choices=[0, 1])
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
@@ -227,7 +266,7 @@ def main():
     I, R = ins.I, win.R
     nb = np.diff(win.chain_off).astype(np.int64)
     stream = torch.cuda.current_stream()
-    sched = P.scheduler_for(wl, device=local, stream=stream.cuda_stream)
+    sched = P.scheduler_for(wl, device=local, stream=stream.cuda_stream, probe_mode=args.probe_mode)
 
     def to_dev(a):
         a = np.ascontiguousarray(a)
@@ -242,7 +281,7 @@ def main():
     for _ in range(args.warmup):
         step()
     hits = sched.score_window(win, want=("hits",))["hits"]
-    probe_bytes = probe_algorithmic_bytes(hits, nb)
+    probe_bytes, n_probes = probe_algorithmic_bytes(hits, nb, args.probe_mode == 1)
     dist_on = world > 1
     if dist_on:
         import torch.distributed as dist
@@ -311,7 +350,8 @@ def main():
             "decisions_per_s": world * R / (ms / 1000),
             "config": {"workload": WORKLOADS.get(args.config, str(args.config)), "instances": I,
                        "window_requests": R, "window_chain_blocks": int(nb.sum()),
-                       "tpot_target_ms": float(win.tpot_target[0]), "probe": "linear 32-wide warp walk",
+                       "tpot_target_ms": float(win.tpot_target[0]), "probe": ("32-ary first-miss search (prefix-closed caches)" if args.probe_mode == 1
+                                 else "linear 32-wide warp walk"), "probes_per_window": n_probes,
                        "l2": "inputs larger than L2 (no flush)", "path_counts": path_counts},
             "kernel_ms": km,
             "probe_roofline": {"achieved": probe_achieved, "peak": peak, "frac": probe_achieved / peak,

@@ -92,7 +92,19 @@ typedef struct {
  *   cap_blocks            host array [num_instances]: cache capacity of each instance in blocks.
  *   table_load_factor     slots of instance i = ceil(cap_blocks[i] / table_load_factor), rounded
  *                         up to 16-slot buckets; (0, 0.95].
- *   model                 the performance model above. */
+ *   model                 the performance model above.
+ *   probe_mode            how hit lengths are found (both give the same hits on the caches they
+ *                         accept):
+ *     PS_PROBE_LINEAR  (0) walk the chain 32 blocks per warp step until the first block that is
+ *                          not cached; exact for any cache contents.
+ *     PS_PROBE_SEARCH  (1) the caches must be prefix-closed (every cached block's parent is
+ *                          cached, as in the paper's Section 6 prefix tree).  Then "block k is
+ *                          cached" is monotone along a chain and a warp finds the first miss by a
+ *                          32-ary search (32 evenly spaced probes per step, at most 4 steps for
+ *                          65536 blocks).  ps_insert_* checks the closure: a chain whose parent_hash
+ *                          is neither 0 nor cached after the call fails with PS_ERR_INVALID. */
+enum { PS_PROBE_LINEAR = 0, PS_PROBE_SEARCH = 1 };
+
 typedef struct {
   int32_t device;
   void* cuda_stream;
@@ -103,6 +115,7 @@ typedef struct {
   const uint64_t* cap_blocks;
   float table_load_factor;
   ps_model model;
+  int32_t probe_mode;
 } ps_config;
 
 /* Scheduler-tracked state of one instance (Section 4 Metadata service; Section 5.5):
@@ -187,9 +200,10 @@ PS_API ps_status ps_get_pending_instances(ps_ctx* ctx, ps_instance_state* out, u
 /* Cache a chain of n blocks on instance inst (host array): block 0 continues parent_hash (0 = the
  * chain starts at the root), block k continues block k-1.  Blocks already cached are skipped.
  * last_use stamps the blocks for LRU bookkeeping.
- * Errors: PS_ERR_INVALID (inst, reserved hash), PS_ERR_TABLE_FULL (no slot left; the blocks before
- * the failing one stay cached), PS_ERR_CAPACITY (the instance now holds more than cap_blocks
- * blocks; the blocks stay cached). */
+ * Errors: PS_ERR_INVALID (inst, reserved hash, or in PS_PROBE_SEARCH mode a parent_hash that is not
+ * cached once the call's blocks are in), PS_ERR_TABLE_FULL (no slot left), PS_ERR_CAPACITY (the
+ * instance now holds more than cap_blocks blocks).  On any of these errors the blocks that could be
+ * inserted stay cached. */
 PS_API ps_status ps_insert_blocks(ps_ctx* ctx, uint32_t inst, const uint64_t* chain, uint64_t n,
                            uint64_t parent_hash, uint32_t last_use);
 
@@ -221,9 +235,10 @@ PS_API ps_status ps_schedule_window(ps_ctx* ctx, const ps_window* w, ps_decision
                              ps_scores* opt_scores);
 
 /* Commit the pending window: the pending state becomes the committed state and each admitted
- * request's uncached blocks are cached on its instance (stamped last_use).  The window's buffers
- * are read again here.  Errors: PS_ERR_STATE (no pending window), PS_ERR_TABLE_FULL,
- * PS_ERR_CAPACITY (as ps_insert_blocks; the commit is still applied). */
+ * request's uncached blocks are cached on its instance.  The window's buffers are read again here.
+ * An instance may end above its cache capacity (ps_cached_blocks shows it); the table keeps working
+ * as long as it has free slots.  Errors: PS_ERR_STATE (no pending window), PS_ERR_TABLE_FULL (no
+ * free slot left; the state is still committed). */
 PS_API ps_status ps_commit_window(ps_ctx* ctx, uint32_t last_use);
 
 /* Device time in ms (CUDA events recorded on the context's stream around each kernel) of the last

@@ -40,7 +40,9 @@ class PsConfig(ctypes.Structure):
                 ("num_instances", ctypes.c_uint32), ("max_window_requests", ctypes.c_uint32),
                 ("max_window_chain_blocks", ctypes.c_uint64), ("block_tokens", ctypes.c_uint32),
                 ("cap_blocks", ctypes.c_void_p), ("table_load_factor", ctypes.c_float),
-                ("model", PsModel)]
+                ("model", PsModel), ("probe_mode", ctypes.c_int32)]
+
+PS_PROBE_LINEAR, PS_PROBE_SEARCH = 0, 1
 
 
 class PsInstanceState(ctypes.Structure):
@@ -156,7 +158,7 @@ class Scheduler:
 
     def __init__(self, num_instances: int, cap_blocks, max_window_requests: int,
                  max_window_chain_blocks: int, model: dict, table_load_factor: float = 0.5,
-                 device: int = 0, stream=None):
+                 device: int = 0, stream=None, probe_mode: int = PS_PROBE_SEARCH):
         self.I = int(num_instances)
         self._cap = np.ascontiguousarray(cap_blocks, dtype=np.uint64)
         cfg = PsConfig()
@@ -169,6 +171,8 @@ class Scheduler:
         cfg.cap_blocks = self._cap.ctypes.data
         cfg.table_load_factor = float(table_load_factor)
         cfg.model = make_model(model)
+        cfg.probe_mode = int(probe_mode)
+        self.probe_mode = int(probe_mode)
         h = ctypes.c_void_p()
         s = lib().ps_create(ctypes.byref(cfg), ctypes.byref(h))
         if s != PS_OK:
@@ -322,12 +326,14 @@ class Scheduler:
 
 
 def scheduler_for(workload, max_window_chain_blocks: int | None = None, device: int = 0, stream=None,
-                  model: dict | None = None, load: bool = True) -> Scheduler:
+                  model: dict | None = None, load: bool = True,
+                  probe_mode: int = PS_PROBE_SEARCH) -> Scheduler:
     """A context sized for a workload.Workload, optionally seeded with its instances."""
     win, ins = workload.window, workload.instances
     mb = max_window_chain_blocks or max(1, int(win.chain_off[-1]))
     s = Scheduler(ins.I, ins.cap_blocks, max(1, win.R), mb, model or workload.model,
-                  table_load_factor=workload.table_load_factor, device=device, stream=stream)
+                  table_load_factor=workload.table_load_factor, device=device, stream=stream,
+                  probe_mode=probe_mode)
     if load:
         s.load_workload_instances(ins)
     return s

@@ -38,6 +38,7 @@ struct ps_ctx {
   uint64_t max_blocks = 0;
   psk::DevModel model{};
   int num_sms = 0, probe_grid = 0;
+  int search = 0;  // PS_PROBE_SEARCH
   std::vector<uint64_t> cap;
   uint64_t total_slots = 0;
   uint64_t* d_slots = nullptr;
@@ -139,6 +140,8 @@ ps_status device_errors(ps_ctx* c) {
                                    "request, L < 2^30, and stay within max_window_chain_blocks");
   if (e & psk::kErrBadInstance) return fail(c, PS_ERR_INVALID, "instance id out of range");
   if (e & psk::kErrReservedHash) return fail(c, PS_ERR_INVALID, "block hash 0 or 2^64-1 is reserved");
+  if (e & psk::kErrParentMissing)
+    return fail(c, PS_ERR_INVALID, "a chain's parent_hash is not cached (PS_PROBE_SEARCH needs prefix-closed caches)");
   if (e & psk::kErrDeltaFull) return fail(c, PS_ERR_TABLE_FULL, "window delta table full");
   if (e & psk::kErrTableFull) return fail(c, PS_ERR_TABLE_FULL, "instance hash table full");
   return fail(c, PS_ERR_CUDA, "unknown device error");
@@ -173,7 +176,7 @@ ps_status stage_window(ps_ctx* c, const ps_window* w, psk::WindowDev* out) {
   if (w->R > c->Rmax) return fail(c, PS_ERR_INVALID, "window has more than max_window_requests requests");
   if (w->inputs_on_device != 0 && w->inputs_on_device != 1)
     return fail(c, PS_ERR_INVALID, "inputs_on_device must be 0 or 1");
-  if (!w->chain_off || !w->prompt_tokens || !w->ttft_target || !w->tpot_target)
+  if (!w->chain_off || (w->R > 0 && (!w->prompt_tokens || !w->ttft_target || !w->tpot_target)))
     return fail(c, PS_ERR_INVALID, "window array is NULL");
   out->R = w->R;
   if (w->inputs_on_device) {
@@ -232,7 +235,7 @@ ps_status run_probe_and_score(ps_ctx* c, const psk::WindowDev& wd, ps_scores* ou
   const int dev_out = out ? out->outputs_on_device : 0;
   uint32_t* hits = (out && out->hits && dev_out) ? out->hits : c->d_hits;
   record(c, kEvProbe0);
-  PS_TRY_CUDA(c, pskl::launch_probe(c->d_slots, c->d_tdesc, c->I, wd, hits, c->probe_grid, c->stream));
+  PS_TRY_CUDA(c, pskl::launch_probe(c->d_slots, c->d_tdesc, c->I, wd, hits, c->probe_grid, c->search, c->stream));
   record(c, kEvProbe1);
   c->ev_used[0] = true;
   *hits_used = hits;
@@ -285,6 +288,8 @@ ps_status ps_create(const ps_config* cfg, ps_ctx** out) {
   if (cfg->block_tokens != PS_BLOCK_TOKENS || !cfg->cap_blocks) return bail(PS_ERR_INVALID);
   if (!(cfg->table_load_factor > 0.0f && cfg->table_load_factor <= 0.95f)) return bail(PS_ERR_INVALID);
   if (check_model(c, cfg->model) != PS_OK) return bail(PS_ERR_INVALID);
+  if (cfg->probe_mode != PS_PROBE_LINEAR && cfg->probe_mode != PS_PROBE_SEARCH) return bail(PS_ERR_INVALID);
+  c->search = cfg->probe_mode == PS_PROBE_SEARCH ? 1 : 0;
   c->device = cfg->device;
   c->I = cfg->num_instances;
   c->Rmax = cfg->max_window_requests;
@@ -446,12 +451,14 @@ ps_status ps_insert_chains(ps_ctx* c, uint64_t nchains, const uint32_t* inst, co
   (void)last_use;
   if (!c) return PS_ERR_INVALID;
   if (nchains == 0) return PS_OK;
-  if (!inst || !off || (on_device != 0 && on_device != 1)) return fail(c, PS_ERR_INVALID, "bad chain arrays");
+  if (!inst || !off || !parent || (on_device != 0 && on_device != 1))
+    return fail(c, PS_ERR_INVALID, "bad chain arrays");
   DeviceGuard g(c->device);
   uint64_t total = 0;
   const uint32_t* d_inst = inst;
   const uint64_t* d_off = off;
   const uint64_t* d_hash = hash;
+  const uint64_t* d_parent = parent;
   void* tmp = nullptr;
   if (!on_device) {
     if (off[0] != 0) return fail(c, PS_ERR_INVALID, "off[0] must be 0");
@@ -461,12 +468,14 @@ ps_status ps_insert_chains(ps_ctx* c, uint64_t nchains, const uint32_t* inst, co
     }
     total = off[nchains];
     if (total && !hash) return fail(c, PS_ERR_INVALID, "hash is NULL");
-    const size_t bytes = nchains * 4 + (nchains + 1) * 8 + total * 8 + 16;
+    const size_t bytes = nchains * 4 + (nchains + 1) * 8 + nchains * 8 + total * 8 + 16;
     PS_TRY_CUDA(c, cudaMalloc(&tmp, bytes));
     uint64_t* t_off = static_cast<uint64_t*>(tmp);
-    uint64_t* t_hash = t_off + nchains + 1;
+    uint64_t* t_parent = t_off + nchains + 1;
+    uint64_t* t_hash = t_parent + nchains;
     uint32_t* t_inst = reinterpret_cast<uint32_t*>(t_hash + total);
     cudaError_t e = cudaMemcpyAsync(t_off, off, (nchains + 1) * 8, cudaMemcpyHostToDevice, c->stream);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(t_parent, parent, nchains * 8, cudaMemcpyHostToDevice, c->stream);
     if (e == cudaSuccess && total) e = cudaMemcpyAsync(t_hash, hash, total * 8, cudaMemcpyHostToDevice, c->stream);
     if (e == cudaSuccess) e = cudaMemcpyAsync(t_inst, inst, nchains * 4, cudaMemcpyHostToDevice, c->stream);
     if (e != cudaSuccess) {
@@ -476,11 +485,15 @@ ps_status ps_insert_chains(ps_ctx* c, uint64_t nchains, const uint32_t* inst, co
     d_off = t_off;
     d_hash = t_hash;
     d_inst = t_inst;
+    d_parent = t_parent;
   } else {
     PS_TRY_CUDA(c, cudaMemcpy(&total, off + nchains, 8, cudaMemcpyDeviceToHost));
   }
   cudaError_t e = pskl::launch_insert_chains(c->d_slots, c->d_tdesc, c->I, c->d_count, nchains, d_inst, d_off,
                                              d_hash, total, c->d_err, c->num_sms, c->stream);
+  if (e == cudaSuccess && c->search)
+    e = pskl::launch_check_parents(c->d_slots, c->d_tdesc, c->I, nchains, d_inst, d_parent, c->d_err, c->num_sms,
+                                   c->stream);
   ps_status s = e == cudaSuccess ? finish(c) : fail(c, PS_ERR_CUDA, cudaGetErrorString(e));
   if (tmp) cudaFree(tmp);
   if (s != PS_OK) return s;
@@ -537,7 +550,7 @@ ps_status ps_schedule_window(ps_ctx* c, const ps_window* w, ps_decisions* out, p
   record(c, kEvGreedy0);
   PS_TRY_CUDA(c, pskl::launch_greedy(c->d_slots, c->d_tdesc, c->I, wd, hit0, c->st, c->pend, c->model, c->d_delta,
                                      c->delta_nbkt, c->d_dlog, c->d_dlog_n, c->d_assign, c->d_dpath, c->d_hchosen,
-                                     c->d_err, c->stream));
+                                     c->d_err, c->search, c->stream));
   record(c, kEvGreedy1);
   c->ev_used[2] = true;
   PS_TRY_CUDA(c, pskl::launch_delta_clear(c->d_delta, c->d_dlog, c->d_dlog_n, c->max_blocks, c->num_sms, c->stream));
@@ -571,9 +584,7 @@ ps_status ps_commit_window(ps_ctx* c, uint32_t last_use) {
   record(c, kEvCommit1);
   c->ev_used[3] = true;
   c->pending = false;
-  ps_status s = finish(c);
-  if (s != PS_OK) return s;
-  return check_capacity(c);
+  return finish(c);
 }
 
 ps_status ps_last_timings(ps_ctx* c, float* ms, uint32_t n) {

@@ -4,10 +4,12 @@
 // request path before the next decision (Section 4, Metadata service; Section 6).  This kernel
 // replays that sequence for a whole window on the GPU: one persistent thread block whose threads
 // each own up to IPT instances.  Per request r:
-//   1. hit of r on instance i = hit0[r][i] (the probe kernel's walk over the committed tables)
+//   1. hit of r on instance i = hit0[r][i] (the probe kernel's result on the committed tables)
 //      extended through the window's delta table: an instance that has received blocks in this
-//      window is re-probed at position hit0 (and walked 32 positions per warp step, over delta and
-//      main, if that block is now cached).  Instances untouched in the window need no probe.
+//      window is re-probed at position hit0, and if that block is now cached a warp finds the new
+//      first miss over delta and main (linear walk, or 32-ary search on prefix-closed caches: the
+//      delta only ever adds a chain's continuation to a cached prefix, so closure is kept).
+//      Instances untouched in the window need no probe.
 //   2. the whole row is re-evaluated from the current state (capacity guard, W, W_min, Eq. 8
 //      filter, TPOT/TTFT admission, D-C-Q key or LMetric fallback), reduced block-wide to the pick;
 //   3. the pick's state is updated (qr += 1, q += n, S += L) and its uncached blocks
@@ -19,7 +21,7 @@
 
 namespace {
 
-template <int IPT>
+template <int IPT, bool SEARCH>
 __global__ void __launch_bounds__(1024, 1)
 greedy_kernel(const uint64_t* __restrict__ slots, const psk::TableDesc* __restrict__ tdesc, uint32_t I,
               psk::WindowDev w, const uint32_t* __restrict__ hit0, psk::StateSoA committed,
@@ -96,20 +98,13 @@ greedy_kernel(const uint64_t* __restrict__ slots, const psk::TableDesc* __restri
       for (uint32_t x = warp; x < nwalk; x += NW) {
         const uint32_t i = s_walk[x];
         const psk::TableDesc d = tdesc[i];
-        uint64_t hnew = nb;
-        for (uint64_t base = (uint64_t)s_h[i] + 1; base < nb; base += 32) {
-          const uint64_t k = base + lane;
-          bool present = true;
-          if (k < nb) {
-            const uint64_t key = w.hash[o + k];
-            present = psk::delta_contains(delta, delta_nbkt, i, key) || psk::main_contains(slots, d, key);
-          }
-          const unsigned miss = __ballot_sync(0xffffffffu, !present);
-          if (miss) {
-            hnew = base + (uint64_t)(__ffs(miss) - 1);
-            break;
-          }
-        }
+        auto cached = [&](uint64_t k) {
+          const uint64_t key = w.hash[o + k];
+          return psk::delta_contains(delta, delta_nbkt, i, key) || psk::main_contains(slots, d, key);
+        };
+        const uint64_t from = (uint64_t)s_h[i] + 1;
+        const uint64_t hnew = SEARCH ? psk::warp_first_miss_search(from, nb, cached)
+                                     : psk::warp_first_miss_linear(from, nb, cached);
         if (lane == 0) s_h[i] = (uint32_t)hnew;
       }
       __syncthreads();  // (B) extended hits visible
@@ -215,32 +210,40 @@ size_t greedy_smem(uint32_t I) {
 
 namespace pskl {
 
+template <int IPT, bool SEARCH>
+cudaError_t greedy_launch(const uint64_t* slots, const psk::TableDesc* tdesc, uint32_t I, const psk::WindowDev& w,
+                          const uint32_t* hit0, psk::StateSoA committed, psk::StateSoA pending,
+                          const psk::DevModel& m, psk::DeltaSlot* delta, uint32_t delta_nbkt,
+                          unsigned long long* dlog, unsigned long long* dlog_n, int32_t* assign, uint8_t* path,
+                          uint32_t* hit_chosen, uint32_t* err, uint32_t nt, cudaStream_t s) {
+  const size_t smem = greedy_smem(I);
+  cudaError_t e = cudaFuncSetAttribute(greedy_kernel<IPT, SEARCH>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)smem);
+  if (e != cudaSuccess) return e;
+  greedy_kernel<IPT, SEARCH><<<1, nt, smem, s>>>(slots, tdesc, I, w, hit0, committed, pending, m, delta,
+                                                 delta_nbkt, dlog, dlog_n, assign, path, hit_chosen, err);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_greedy(const uint64_t* slots, const psk::TableDesc* tdesc, uint32_t I,
                           const psk::WindowDev& w, const uint32_t* hit0, psk::StateSoA committed,
                           psk::StateSoA pending, const psk::DevModel& m, psk::DeltaSlot* delta,
                           uint32_t delta_nbkt, unsigned long long* dlog, unsigned long long* dlog_n,
                           int32_t* assign, uint8_t* path, uint32_t* hit_chosen, uint32_t* err,
-                          cudaStream_t s) {
+                          int search, cudaStream_t s) {
   uint32_t nt = (I + 31) / 32 * 32;
   if (nt > 1024) nt = 1024;
   const uint32_t ipt = (I + nt - 1) / nt;
-  const size_t smem = greedy_smem(I);
-  if (ipt <= 1) {
-    cudaFuncSetAttribute(greedy_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    greedy_kernel<1><<<1, nt, smem, s>>>(slots, tdesc, I, w, hit0, committed, pending, m, delta, delta_nbkt,
-                                         dlog, dlog_n, assign, path, hit_chosen, err);
-  } else if (ipt <= 2) {
-    cudaFuncSetAttribute(greedy_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    greedy_kernel<2><<<1, nt, smem, s>>>(slots, tdesc, I, w, hit0, committed, pending, m, delta, delta_nbkt,
-                                         dlog, dlog_n, assign, path, hit_chosen, err);
-  } else if (ipt <= 4) {
-    cudaFuncSetAttribute(greedy_kernel<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    greedy_kernel<4><<<1, nt, smem, s>>>(slots, tdesc, I, w, hit0, committed, pending, m, delta, delta_nbkt,
-                                         dlog, dlog_n, assign, path, hit_chosen, err);
-  } else {
-    return cudaErrorInvalidValue;
-  }
-  return cudaGetLastError();
+#define PS_GREEDY(IPT)                                                                                  \
+  return search ? greedy_launch<IPT, true>(slots, tdesc, I, w, hit0, committed, pending, m, delta, delta_nbkt, \
+                                           dlog, dlog_n, assign, path, hit_chosen, err, nt, s)           \
+                : greedy_launch<IPT, false>(slots, tdesc, I, w, hit0, committed, pending, m, delta, delta_nbkt, \
+                                            dlog, dlog_n, assign, path, hit_chosen, err, nt, s)
+  if (ipt <= 1) PS_GREEDY(1);
+  if (ipt <= 2) PS_GREEDY(2);
+  if (ipt <= 4) PS_GREEDY(4);
+#undef PS_GREEDY
+  return cudaErrorInvalidValue;
 }
 
 cudaError_t launch_delta_clear(psk::DeltaSlot* delta, const unsigned long long* dlog,

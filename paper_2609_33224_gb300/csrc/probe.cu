@@ -5,17 +5,18 @@
 // quantity the paper's scheduler reads from its prefix tree (Section 6) to estimate KVC reuse.
 //
 // One thread block per request (grid-stride over requests).  The request's chain is staged in
-// shared memory once (coalesced 8-byte loads) and reused by every instance's walk.  Each warp walks
-// one instance at a time, 32 chain positions per step: lane k probes position base + k in the
-// instance's table, __ballot_sync collects the misses and __ffs finds the first.  Positions past the
-// staging capacity are read from global memory (L1/L2-resident: the same block re-reads them).
+// shared memory once (coalesced 8-byte loads) and reused by every instance's walk.  Each warp
+// handles one instance at a time with 32 probes per step, __ballot_sync collecting the misses and
+// __ffs finding the first: either a linear walk over 32 consecutive positions per step, or (for
+// prefix-closed caches) a 32-ary search over 32 evenly spaced positions.  Positions past the staging
+// capacity are read from global memory (L1/L2-resident: the same block re-reads them).
 #include "ps_internal.cuh"
 
 namespace {
 
 constexpr uint32_t kStageBlocks = 8192;  // 64 KB of staged chain per thread block
 
-template <int WARPS>
+template <int WARPS, bool SEARCH>
 __global__ void __launch_bounds__(WARPS * 32)
 probe_hits_kernel(const uint64_t* __restrict__ slots, const psk::TableDesc* __restrict__ tdesc,
                   uint32_t I, const uint64_t* __restrict__ off, const uint64_t* __restrict__ hash,
@@ -31,20 +32,12 @@ probe_hits_kernel(const uint64_t* __restrict__ slots, const psk::TableDesc* __re
     __syncthreads();
     for (uint32_t i = warp; i < I; i += WARPS) {
       const psk::TableDesc d = tdesc[i];
-      uint64_t h = nb;
-      for (uint64_t base = 0; base < nb; base += 32) {
-        const uint64_t k = base + lane;
-        bool present = true;  // positions past the chain end never count as a miss
-        if (k < nb) {
-          const uint64_t key = k < ns ? s_chain[k] : __ldg(hash + o + k);
-          present = psk::main_contains(slots, d, key);
-        }
-        const unsigned miss = __ballot_sync(0xffffffffu, !present);
-        if (miss) {
-          h = base + (uint64_t)(__ffs(miss) - 1);
-          break;
-        }
-      }
+      auto cached = [&](uint64_t k) {
+        const uint64_t key = k < ns ? s_chain[k] : __ldg(hash + o + k);
+        return psk::main_contains(slots, d, key);
+      };
+      const uint64_t h = SEARCH ? psk::warp_first_miss_search(0, nb, cached)
+                                : psk::warp_first_miss_linear(0, nb, cached);
       if (lane == 0) hits[(uint64_t)r * I + i] = (uint32_t)h;
     }
     __syncthreads();
@@ -53,11 +46,13 @@ probe_hits_kernel(const uint64_t* __restrict__ slots, const psk::TableDesc* __re
 
 template <int WARPS>
 int max_grid(int num_sms) {
-  int per_sm = 0;
-  cudaFuncSetAttribute(probe_hits_kernel<WARPS>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                       (int)(kStageBlocks * sizeof(uint64_t)));
-  cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, probe_hits_kernel<WARPS>, WARPS * 32,
-                                                kStageBlocks * sizeof(uint64_t));
+  int per_sm = 0, per_sm2 = 0;
+  const int smem = (int)(kStageBlocks * sizeof(uint64_t));
+  cudaFuncSetAttribute(probe_hits_kernel<WARPS, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  cudaFuncSetAttribute(probe_hits_kernel<WARPS, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, probe_hits_kernel<WARPS, false>, WARPS * 32, smem);
+  cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm2, probe_hits_kernel<WARPS, true>, WARPS * 32, smem);
+  if (per_sm2 < per_sm) per_sm = per_sm2;
   if (per_sm < 1) per_sm = 1;
   return per_sm * num_sms;
 }
@@ -71,14 +66,21 @@ int probe_max_grid(uint32_t I, int num_sms) {
 }
 
 cudaError_t launch_probe(const uint64_t* slots, const psk::TableDesc* tdesc, uint32_t I,
-                         const psk::WindowDev& w, uint32_t* hits, int grid, cudaStream_t s) {
+                         const psk::WindowDev& w, uint32_t* hits, int grid, int search, cudaStream_t s) {
   if (w.R == 0) return cudaSuccess;
   const int g = (int)((uint32_t)grid < w.R ? (uint32_t)grid : w.R);
   const size_t smem = kStageBlocks * sizeof(uint64_t);
-  if (I >= 64)
-    probe_hits_kernel<16><<<g, 16 * 32, smem, s>>>(slots, tdesc, I, w.off, w.hash, w.R, hits);
-  else
-    probe_hits_kernel<4><<<g, 4 * 32, smem, s>>>(slots, tdesc, I, w.off, w.hash, w.R, hits);
+  if (I >= 64) {
+    if (search)
+      probe_hits_kernel<16, true><<<g, 16 * 32, smem, s>>>(slots, tdesc, I, w.off, w.hash, w.R, hits);
+    else
+      probe_hits_kernel<16, false><<<g, 16 * 32, smem, s>>>(slots, tdesc, I, w.off, w.hash, w.R, hits);
+  } else {
+    if (search)
+      probe_hits_kernel<4, true><<<g, 4 * 32, smem, s>>>(slots, tdesc, I, w.off, w.hash, w.R, hits);
+    else
+      probe_hits_kernel<4, false><<<g, 4 * 32, smem, s>>>(slots, tdesc, I, w.off, w.hash, w.R, hits);
+  }
   return cudaGetLastError();
 }
 

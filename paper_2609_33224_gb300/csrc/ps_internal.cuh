@@ -31,6 +31,7 @@ enum : uint32_t {
   kErrDeltaFull = 4u,
   kErrWindowLayout = 8u,
   kErrBadInstance = 16u,
+  kErrParentMissing = 32u,
 };
 
 struct TableDesc {
@@ -164,6 +165,52 @@ __device__ __forceinline__ bool delta_insert(DeltaSlot* delta, uint32_t nbkt, ui
     b = (b + 1 == nbkt) ? 0u : b + 1;
   }
   return false;
+}
+
+// ------------------------------------------------------------------------------- first-miss walks --
+// All 32 lanes of a warp call these with the same arguments; present(k) is evaluated per lane.
+// Both return the first position k in [lo, nb) with present(k) false (nb if there is none), given
+// that every position below lo is known present.
+
+// Linear walk, 32 consecutive positions per step: exact for any membership pattern.
+template <class Pred>
+__device__ __forceinline__ uint64_t warp_first_miss_linear(uint64_t lo, uint64_t nb, Pred present) {
+  const int lane = threadIdx.x & 31;
+  for (uint64_t base = lo; base < nb; base += 32) {
+    const uint64_t k = base + lane;
+    const bool p = k < nb ? present(k) : true;
+    const unsigned miss = __ballot_sync(0xffffffffu, !p);
+    if (miss) return base + (uint64_t)(__ffs(miss) - 1);
+  }
+  return nb;
+}
+
+// 32-ary search, exact when membership is monotone along the chain (a prefix-closed cache).
+// Invariant: the answer h lies in [lo, hi], positions below lo are present and position hi is
+// absent (or hi = nb).  Each step probes 32 evenly spaced positions p_j = lo + (j+1) span / 32 - 1
+// (p_31 = hi - 1) and keeps [p_{j-1} + 1, p_j] around the first miss j, so an interval of span s
+// shrinks to at most ceil(s / 32); spans <= 32 are finished by one linear step.
+template <class Pred>
+__device__ __forceinline__ uint64_t warp_first_miss_search(uint64_t lo, uint64_t nb, Pred present) {
+  const int lane = threadIdx.x & 31;
+  uint64_t hi = nb;
+  for (;;) {
+    const uint64_t span = hi - lo;
+    if (span == 0) return lo;
+    if (span <= 32) {
+      const uint64_t k = lo + lane;
+      const bool p = k < hi ? present(k) : true;
+      const unsigned miss = __ballot_sync(0xffffffffu, !p);
+      return miss ? lo + (uint64_t)(__ffs(miss) - 1) : hi;
+    }
+    const uint64_t k = lo + ((uint64_t)(lane + 1) * span) / 32 - 1;
+    const unsigned miss = __ballot_sync(0xffffffffu, !present(k));
+    if (!miss) return hi;
+    const uint64_t j = (uint64_t)(__ffs(miss) - 1);
+    const uint64_t pj = lo + ((j + 1) * span) / 32 - 1;
+    lo = lo + (j * span) / 32;
+    hi = pj;
+  }
 }
 
 // ---------------------------------------------------------------------------- performance model --
@@ -303,7 +350,7 @@ constexpr uint32_t kNoKeyCi = 0xFFFFFFFFu;  // class 15: worse than any real pai
 // Kernel launchers (one translation unit each).
 namespace pskl {
 cudaError_t launch_probe(const uint64_t* slots, const psk::TableDesc* tdesc, uint32_t I,
-                         const psk::WindowDev& w, uint32_t* hits, int grid, cudaStream_t s);
+                         const psk::WindowDev& w, uint32_t* hits, int grid, int search, cudaStream_t s);
 int probe_max_grid(uint32_t I, int num_sms);
 cudaError_t launch_score(const uint32_t* hits, psk::StateSoA st, uint32_t I, const psk::WindowDev& w,
                          const psk::DevModel& m, float* tpot, float* ttft, uint8_t* cls, int32_t* best,
@@ -313,7 +360,7 @@ cudaError_t launch_greedy(const uint64_t* slots, const psk::TableDesc* tdesc, ui
                           psk::StateSoA pending, const psk::DevModel& m, psk::DeltaSlot* delta,
                           uint32_t delta_nbkt, unsigned long long* dlog, unsigned long long* dlog_n,
                           int32_t* assign, uint8_t* path, uint32_t* hit_chosen, uint32_t* err,
-                          cudaStream_t s);
+                          int search, cudaStream_t s);
 cudaError_t launch_delta_clear(psk::DeltaSlot* delta, const unsigned long long* dlog,
                                unsigned long long* dlog_n, uint64_t max_entries, int num_sms,
                                cudaStream_t s);
@@ -324,6 +371,9 @@ cudaError_t launch_insert_chains(uint64_t* slots, const psk::TableDesc* tdesc, u
 cudaError_t launch_commit(uint64_t* slots, const psk::TableDesc* tdesc, uint32_t I,
                           unsigned long long* count, const psk::WindowDev& w, const int32_t* assign,
                           const uint32_t* hit_chosen, uint32_t* err, int num_sms, cudaStream_t s);
+cudaError_t launch_check_parents(const uint64_t* slots, const psk::TableDesc* tdesc, uint32_t I,
+                                 uint64_t nchains, const uint32_t* inst, const uint64_t* parent,
+                                 uint32_t* err, int num_sms, cudaStream_t s);
 cudaError_t launch_validate_window(const psk::WindowDev& w, uint64_t max_blocks, uint32_t* err,
                                    cudaStream_t s);
 }  // namespace pskl

@@ -87,6 +87,18 @@ __global__ void commit_kernel(uint64_t* slots, const psk::TableDesc* __restrict_
   }
 }
 
+// Prefix closure check (search mode): every chain's parent must be cached once the chains are in.
+__global__ void check_parents_kernel(const uint64_t* slots, const psk::TableDesc* __restrict__ tdesc, uint32_t I,
+                                     uint64_t nchains, const uint32_t* __restrict__ inst,
+                                     const uint64_t* __restrict__ parent, uint32_t* err) {
+  for (uint64_t c = blockIdx.x * (uint64_t)blockDim.x + threadIdx.x; c < nchains; c += (uint64_t)gridDim.x * blockDim.x) {
+    const uint64_t p = parent[c];
+    const uint32_t i = inst[c];
+    if (p == psk::kEmpty || i >= I) continue;
+    if (!psk::main_contains(slots, tdesc[i], p)) atomicOr(err, psk::kErrParentMissing);
+  }
+}
+
 __global__ void validate_window_kernel(psk::WindowDev w, uint64_t max_blocks, uint32_t* err) {
   for (uint32_t r = blockIdx.x * blockDim.x + threadIdx.x; r < w.R; r += gridDim.x * blockDim.x) {
     const uint64_t a = w.off[r], b = w.off[r + 1];
@@ -121,6 +133,16 @@ cudaError_t launch_commit(uint64_t* slots, const psk::TableDesc* tdesc, uint32_t
   uint32_t blocks = (w.R + 7) / 8;
   if (blocks > (uint32_t)num_sms * 8) blocks = num_sms * 8;
   commit_kernel<<<blocks, 256, 0, s>>>(slots, tdesc, I, count, w, assign, hit_chosen, err);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_check_parents(const uint64_t* slots, const psk::TableDesc* tdesc, uint32_t I,
+                                 uint64_t nchains, const uint32_t* inst, const uint64_t* parent,
+                                 uint32_t* err, int num_sms, cudaStream_t s) {
+  if (nchains == 0) return cudaSuccess;
+  uint64_t blocks = (nchains + 255) / 256;
+  if (blocks > (uint64_t)num_sms * 8) blocks = (uint64_t)num_sms * 8;
+  check_parents_kernel<<<(unsigned)blocks, 256, 0, s>>>(slots, tdesc, I, nchains, inst, parent, err);
   return cudaGetLastError();
 }
 

@@ -83,3 +83,9 @@ def test_create_without_gpu_reports_an_error(lib):
         pytest.skip("a GPU is present")
     with pytest.raises(P.PSError):
         P.Scheduler(2, [16, 16], 4, 64, dict(__import__("workload").MODEL_DEFAULT))
+
+
+def test_graft_entry_build_runs_on_cpu():
+    import __graft_entry__ as g
+    g.build()
+    assert os.path.exists(P._LIB_PATH)

@@ -30,9 +30,12 @@ def _oracle(model, ins):
     return Oracle(ins.I, model).load(ins)
 
 
-def _sched(P, model, ins, win, max_blocks=None):
+MODES = [0, 1]  # PS_PROBE_LINEAR, PS_PROBE_SEARCH
+
+
+def _sched(P, model, ins, win, max_blocks=None, mode=1):
     s = P.Scheduler(ins.I, ins.cap_blocks, max(1, win.R), max(1, max_blocks or int(win.chain_off[-1])),
-                    model, table_load_factor=0.5)
+                    model, table_load_factor=0.5, probe_mode=mode)
     s.load_workload_instances(ins)
     return s
 
@@ -48,10 +51,10 @@ def _assert_scores(g, o, exact_floats=True):
             assert np.array_equal(g[k].view(np.uint32), o[k].view(np.uint32)), k
 
 
-def _check_window(P, model, ins, win, commit=True):
+def _check_window(P, model, ins, win, commit=True, mode=1):
     """Score and schedule one window on both sides and compare everything."""
     orc = _oracle(model, ins)
-    with _sched(P, model, ins, win) as s:
+    with _sched(P, model, ins, win, mode=mode) as s:
         g = s.score_window(win)
         o = orc.score_rows(win)
         _assert_scores(g, o)
@@ -83,9 +86,10 @@ def _check_window(P, model, ins, win, commit=True):
         return gd, od
 
 
-def test_hand_example_through_the_abi(P, hand):
+@pytest.mark.parametrize("mode", MODES)
+def test_hand_example_through_the_abi(P, hand, mode):
     model, ins, win, d = hand
-    with _sched(P, model, ins, win) as s:
+    with _sched(P, model, ins, win, mode=mode) as s:
         g = s.score_window(win)
         e = d["score_mode"]
         assert g["hits"].tolist() == e["hits"]
@@ -100,12 +104,13 @@ def test_hand_example_through_the_abi(P, hand):
         for i, f in enumerate(e["final_state"]):
             for k in ("b", "qr", "q", "S"):
                 assert int(pend[k][i]) == f[k]
-    _check_window(P, model, ins, win)
+    _check_window(P, model, ins, win, mode=mode)
 
 
-def test_config0_full_parity(P):
+@pytest.mark.parametrize("mode", MODES)
+def test_config0_full_parity(P, mode):
     wl = W.generate(0)
-    gd, od = _check_window(P, wl.model, wl.instances, wl.window)
+    gd, od = _check_window(P, wl.model, wl.instances, wl.window, mode=mode)
     assert (od["path"] == 0).any()
 
 
@@ -166,11 +171,41 @@ def _random_case(seed, I, R):
     return ins, win
 
 
+@pytest.mark.parametrize("mode", MODES)
 @pytest.mark.parametrize("seed,I,R", [(1, 1, 7), (2, 3, 64), (3, 33, 37), (4, 70, 200), (5, 130, 150),
-                                      (6, 8, 1), (7, 257, 90)])
-def test_random_ragged_windows(P, seed, I, R):
+                                      (6, 8, 1), (7, 257, 90), (8, 1100, 40)])
+def test_random_ragged_windows(P, seed, I, R, mode):
     ins, win = _random_case(seed, I, R)
-    _check_window(P, dict(W.MODEL_DEFAULT), ins, win)
+    _check_window(P, dict(W.MODEL_DEFAULT), ins, win, mode=mode)
+
+
+def test_linear_mode_is_exact_on_a_cache_that_is_not_prefix_closed(P):
+    """A gapped cache (blocks 0-2 and 5-29 of a chain): linear walks stop at block 3, like the
+    oracle; search mode refuses to build such a cache."""
+    ch = W.chain_from_tokens(seq_tokens("A", 16 * 40))
+    model = dict(W.MODEL_DEFAULT)
+    win = make_window([(seq_tokens("A", 16 * 40), 2000.0, 50.0), (seq_tokens("A", 16 * 4), 2000.0, 50.0)])
+    orc = Oracle(2, model)
+    orc.insert_chain(0, ch[:3])
+    orc.insert_chain(0, ch[5:30], parent=int(ch[4]))
+    st = dict(b=np.array([3, 1], np.int32), qr=np.zeros(2, np.int32), q=np.zeros(2, np.int64),
+              S=np.zeros(2, np.int64), M_KV=np.full(2, 10 ** 7, np.int64), B_max=np.full(2, 64, np.int32))
+    orc.set_state(**st)
+    with P.Scheduler(2, [4096, 4096], 2, 64, model, probe_mode=0) as s:
+        s.insert_blocks(0, ch[:3])
+        s.insert_blocks(0, ch[5:30], parent=int(ch[4]))
+        s.load_instances(**st)
+        g = s.score_window(win)
+        o = orc.score_rows(win)
+        _assert_scores(g, o)
+        assert g["hits"][0].tolist() == [3, 0]
+        gd, od = s.schedule_window(win), orc.schedule(win)
+        assert np.array_equal(gd["assign"], od["assign"]) and np.array_equal(gd["hit_chosen"], od["hit_chosen"])
+    with P.Scheduler(2, [4096, 4096], 2, 64, model, probe_mode=1) as s:
+        s.insert_blocks(0, ch[:3])
+        with pytest.raises(P.PSError) as e:
+            s.insert_blocks(0, ch[5:30], parent=int(ch[4]))
+        assert e.value.status == P.PS_ERR_INVALID
 
 
 def test_empty_window_and_short_prompts(P):
@@ -236,9 +271,9 @@ def test_capacity_and_table_full_errors(P):
         assert int(s.cached_blocks()[0]) == 25
 
 
-@pytest.mark.parametrize("tpot", [30.0, 50.0])
-def test_config1_full_parity(P, tpot):
+@pytest.mark.parametrize("tpot,mode", [(30.0, 1), (50.0, 1), (50.0, 0)])
+def test_config1_full_parity(P, tpot, mode):
     wl = W.generate(1, tpot_target_ms=tpot)
-    gd, od = _check_window(P, wl.model, wl.instances, wl.window, commit=(tpot == 50.0))
+    gd, od = _check_window(P, wl.model, wl.instances, wl.window, commit=(tpot == 50.0), mode=mode)
     counts = np.bincount(od["path"], minlength=3)
     print(f"config 1 tpot {tpot}: packed {counts[0]} fallback {counts[1]} reject {counts[2]}")
