@@ -246,6 +246,56 @@ PS_API ps_status ps_commit_window(ps_ctx* ctx, uint32_t last_use);
  * score, ms[2] greedy, ms[3] commit; -1 where that kernel did not run.  n must be >= 4. */
 PS_API ps_status ps_last_timings(ps_ctx* ctx, float* ms, uint32_t n);
 
+/* ---- Scoring without device allocation ------------------------------------------------------
+ * The paper has no counterpart to this call; it exists for callers that cannot allocate device
+ * memory: a serving process whose memory manager reserves the GPU at start-up (leaving the rest to
+ * the KV cache) and forbids later allocations, or a scheduler loop that must not call cudaMalloc
+ * because an allocation can synchronise the device and stall the serving streams.  Such callers
+ * cannot create a context (ps_create allocates), so this call takes every buffer from the caller
+ * and needs no context.
+ *
+ * It computes what ps_score_window computes (probe kernel + fused score kernel, same results) for
+ * caches laid out the way the library lays them out:
+ *   slots    device u64 array holding every instance's table; value 0 = empty slot.
+ *   tables   device array [num_instances] of ps_table_desc: instance i's table is num_buckets
+ *            buckets of 16 slots starting at slot `base`; block hash h lives in bucket
+ *            (h * num_buckets) >> 64 (high 64 bits of the 128-bit product) or, if that bucket is
+ *            full, in the following buckets (wrapping); each table must keep at least one empty slot.
+ *   state    device arrays of the instance state (ps_instance_state fields, structure of arrays).
+ *   window   inputs_on_device must be 1; out->outputs_on_device must be 1 (all device buffers).
+ *   probe_mode  as ps_config.probe_mode (PS_PROBE_SEARCH only for prefix-closed caches).
+ *   cuda_stream  the stream to run on; the call synchronises it before returning.
+ * The hit matrix it needs in between is kept in a fixed device array inside the library
+ * (PS_NOALLOC_MAX_PAIRS u32 entries, 8 MiB, held on every GPU that loads the library until the
+ * process exits), so R * num_instances may not exceed PS_NOALLOC_MAX_PAIRS (split larger windows).
+ * The first call on each device resolves that array's device address; make that first call before
+ * any stream capture.  All calls share the one array: calls that overlap on the GPU (other threads
+ * or streams) race and must be serialised by the caller.  The call allocates nothing (no
+ * cudaMalloc, cudaFree or allocating library routine).
+ * Errors: PS_ERR_INVALID (NULL or host buffers, sizes beyond the limit, bad window layout or model),
+ * PS_ERR_CUDA.  No context exists, so there is no message for ps_last_error. */
+#define PS_NOALLOC_MAX_PAIRS 2097152u
+
+typedef struct {
+  uint64_t base;
+  uint32_t num_buckets;
+  uint32_t reserved;
+} ps_table_desc;
+
+typedef struct {
+  const int32_t* b;
+  const int32_t* qr;
+  const int64_t* q_tokens;
+  const int64_t* S_tokens;
+  const int64_t* M_KV_tokens;
+  const int32_t* B_max;
+} ps_state_arrays;
+
+PS_API ps_status ps_score_window_noalloc(const uint64_t* slots, const ps_table_desc* tables,
+                                         uint32_t num_instances, const ps_state_arrays* state,
+                                         const ps_window* window, const ps_model* model,
+                                         int32_t probe_mode, ps_scores* out, void* cuda_stream);
+
 /* Text of the last error on this context ("" if none).  Valid until the next call. */
 PS_API const char* ps_last_error(const ps_ctx* ctx);
 

@@ -25,7 +25,7 @@ STATUS_NAMES = {0: "PS_OK", 1: "PS_ERR_INVALID", 2: "PS_ERR_CUDA", 3: "PS_ERR_OO
 ABI_FUNCTIONS = ("ps_create", "ps_load_instances", "ps_get_instances", "ps_get_pending_instances",
                  "ps_insert_blocks", "ps_insert_chains", "ps_cached_blocks", "ps_score_window",
                  "ps_schedule_window", "ps_commit_window", "ps_last_timings", "ps_last_error",
-                 "ps_destroy")
+                 "ps_destroy", "ps_score_window_noalloc")
 
 
 class PsModel(ctypes.Structure):
@@ -67,6 +67,16 @@ class PsDecisions(ctypes.Structure):
                 ("outputs_on_device", ctypes.c_int32)]
 
 
+class PsTableDesc(ctypes.Structure):
+    _fields_ = [("base", ctypes.c_uint64), ("num_buckets", ctypes.c_uint32), ("reserved", ctypes.c_uint32)]
+
+
+class PsStateArrays(ctypes.Structure):
+    _fields_ = [(k, ctypes.c_void_p) for k in ("b", "qr", "q_tokens", "S_tokens", "M_KV_tokens", "B_max")]
+
+
+PS_NOALLOC_MAX_PAIRS = 2097152
+
 STATE_DTYPE = np.dtype([("b", np.int32), ("qr", np.int32), ("q_tokens", np.int64), ("S_tokens", np.int64),
                         ("M_KV_tokens", np.int64), ("B_max", np.int32)], align=True)
 assert STATE_DTYPE.itemsize == ctypes.sizeof(PsInstanceState)
@@ -96,6 +106,8 @@ def lib() -> ctypes.CDLL:
                                    ctypes.POINTER(PsScores)],
             "ps_commit_window": [vp, u32],
             "ps_last_timings": [vp, vp, u32],
+            "ps_score_window_noalloc": [vp, vp, u32, ctypes.POINTER(PsStateArrays), ctypes.POINTER(PsWindow),
+                                        ctypes.POINTER(PsModel), i32, ctypes.POINTER(PsScores), vp],
         }
         for name, args in sigs.items():
             fn = getattr(L, name)

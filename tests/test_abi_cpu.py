@@ -29,7 +29,7 @@ def _declared():
 
 def test_every_declared_symbol_is_exported(lib):
     names = _declared()
-    assert len(names) >= 13
+    assert len(names) >= 14
     out = subprocess.run(["nm", "-D", "--defined-only", P._LIB_PATH], capture_output=True, text=True,
                          check=True).stdout
     exported = set(re.findall(r"\bT (ps_\w+)$", out, flags=re.M))
@@ -49,6 +49,7 @@ def test_struct_layouts_match_c(tmp_path):
 #define O(T, f) printf(#T "." #f " %zu\\n", offsetof(T, f));
 int main(void) {
   P(ps_model) P(ps_config) P(ps_instance_state) P(ps_window) P(ps_scores) P(ps_decisions)
+  P(ps_table_desc) P(ps_state_arrays)
   O(ps_config, model) O(ps_config, table_load_factor) O(ps_config, cap_blocks)
   O(ps_model, seg_lo) O(ps_model, ema_factor) O(ps_instance_state, B_max)
   O(ps_window, inputs_on_device) O(ps_scores, outputs_on_device) O(ps_decisions, outputs_on_device)
@@ -60,7 +61,8 @@ int main(void) {
     got = dict(line.rsplit(" ", 1) for line in subprocess.run([str(exe)], capture_output=True, text=True,
                                                                check=True).stdout.split("\n") if line)
     ct = {"ps_model": P.PsModel, "ps_config": P.PsConfig, "ps_instance_state": P.PsInstanceState,
-          "ps_window": P.PsWindow, "ps_scores": P.PsScores, "ps_decisions": P.PsDecisions}
+          "ps_window": P.PsWindow, "ps_scores": P.PsScores, "ps_decisions": P.PsDecisions,
+          "ps_table_desc": P.PsTableDesc, "ps_state_arrays": P.PsStateArrays}
     for k, v in got.items():
         if "." in k:
             t, f = k.split(".")

@@ -1,0 +1,167 @@
+"""ps_score_window_noalloc: scoring for callers that cannot allocate device memory.
+
+Such a caller (for example a serving process that reserves the GPU at start-up and forbids later
+allocations) owns every buffer, so this test plays that caller: it lays out the cache tables itself
+in the documented format, in device memory it allocated, and checks that two calls in a row give
+the same hits, latencies, classes and picks as the context-based ps_score_window.
+"""
+import ctypes
+import math
+
+import numpy as np
+import pytest
+
+import workload as W
+from tests.helpers import make_window, seq_tokens
+
+pytestmark = pytest.mark.gpu
+
+REL = 1e-5
+
+
+@pytest.fixture(scope="module")
+def P():
+    import torch
+    if not torch.cuda.is_available():
+        pytest.fail("a CUDA device is required for the gpu tests")
+    import paper_2609_33224_gb300 as P
+    P.build()
+    return P
+
+
+def _caller_tables(ins):
+    """The documented layout, built on the host: 16-slot buckets, home bucket (h * nbkt) >> 64,
+    linear probing over buckets, 0 = empty; two slots per cached block (load factor 0.5)."""
+    I = ins.I
+    per = np.bincount(ins.chain_inst, weights=np.diff(ins.chain_off).astype(np.float64), minlength=I)
+    nbkt = [max(1, math.ceil(2 * int(n) / 16) + 1) for n in per]
+    base = np.zeros(I, np.uint64)
+    base[1:] = np.cumsum(np.array(nbkt[:-1], np.uint64) * 16)
+    slots = np.zeros(int(sum(nbkt)) * 16, np.uint64)
+    for c in range(ins.chain_inst.shape[0]):
+        i = int(ins.chain_inst[c])
+        for key in ins.chain_hash[ins.chain_off[c]:ins.chain_off[c + 1]]:
+            key = int(key)
+            b = (key * nbkt[i]) >> 64
+            while True:
+                line = slots[int(base[i]) + 16 * b: int(base[i]) + 16 * b + 16]
+                if (line == key).any():
+                    break
+                empty = np.nonzero(line == 0)[0]
+                if empty.size:
+                    line[empty[0]] = key
+                    break
+                b = (b + 1) % nbkt[i]
+    desc = np.zeros(I, dtype=np.dtype([("base", np.uint64), ("num_buckets", np.uint32), ("reserved", np.uint32)]))
+    desc["base"], desc["num_buckets"] = base, nbkt
+    return slots, desc
+
+
+def _dev(a):
+    import torch
+    a = np.ascontiguousarray(a)
+    view = {np.dtype(np.uint64): np.int64, np.dtype(np.uint32): np.int32}.get(a.dtype)
+    if a.dtype.names:
+        return torch.from_numpy(a.view(np.uint8)).cuda()
+    return torch.from_numpy(a.view(view) if view else a).cuda()
+
+
+def _noalloc_score(P, ins, win, model, mode):
+    """One call of the allocation-free entry point with caller-owned device buffers."""
+    import torch
+    slots, desc = _caller_tables(ins)
+    d_slots, d_desc = _dev(slots), _dev(desc)
+    st = {k: _dev(getattr(ins, k)) for k in ("b", "qr", "q", "S", "M_KV", "B_max")}
+    sa = P.PsStateArrays(st["b"].data_ptr(), st["qr"].data_ptr(), st["q"].data_ptr(), st["S"].data_ptr(),
+                         st["M_KV"].data_ptr(), st["B_max"].data_ptr())
+    dwin = W.Window(**{k: _dev(getattr(win, k)) for k in win.__dataclass_fields__})
+    pw = P.Scheduler.make_window(dwin)
+    R, I = win.R, ins.I
+    out = {"hits": torch.empty((R, I), dtype=torch.int32, device="cuda"),
+           "tpot": torch.empty((R, I), dtype=torch.float32, device="cuda"),
+           "ttft": torch.empty((R, I), dtype=torch.float32, device="cuda"),
+           "cls": torch.empty((R, I), dtype=torch.uint8, device="cuda"),
+           "best": torch.empty(R, dtype=torch.int32, device="cuda"),
+           "path": torch.empty(R, dtype=torch.uint8, device="cuda")}
+    sc = P.PsScores(*(out[k].data_ptr() for k in ("hits", "tpot", "ttft", "cls", "best", "path")), 1)
+    m = P.make_model(model)
+    status = P.lib().ps_score_window_noalloc(d_slots.data_ptr(), d_desc.data_ptr(), I, ctypes.byref(sa),
+                                             ctypes.byref(pw), ctypes.byref(m), int(mode), ctypes.byref(sc),
+                                             torch.cuda.current_stream().cuda_stream)
+    assert status == P.PS_OK, P.STATUS_NAMES.get(status, status)
+    res = {k: v.cpu().numpy() for k, v in out.items()}
+    res["hits"] = res["hits"].view(np.uint32)
+    return res
+
+
+def _context_score(P, ins, win, model, mode):
+    with P.Scheduler(ins.I, ins.cap_blocks, max(1, win.R), max(1, int(win.chain_off[-1])), model,
+                     probe_mode=mode) as s:
+        s.load_workload_instances(ins)
+        return s.score_window(win)
+
+
+def _same(a, b):
+    for k in ("hits", "cls", "best", "path"):
+        assert np.array_equal(a[k], b[k]), k
+    for k in ("tpot", "ttft"):
+        np.testing.assert_allclose(a[k], b[k], rtol=REL, atol=0)
+
+
+def _random_case(seed, I, R):
+    rng = np.random.default_rng(seed)
+    base = [rng.integers(0, 1 << 17, 16 * 300).astype(np.uint32) for _ in range(3)]
+    reqs = []
+    for _ in range(R):
+        b = base[int(rng.integers(0, 3))]
+        L = int(rng.integers(0, 16 * 400))
+        cut = int(rng.integers(0, b.shape[0]))
+        toks = b[:L] if L <= cut else np.concatenate([b[:cut], rng.integers(0, 1 << 17, L - cut).astype(np.uint32)])
+        reqs.append((toks, 2000.0, float(rng.choice([20.0, 50.0]))))
+    win = make_window(reqs)
+    chains, inst = [], []
+    for i in range(I):
+        for _ in range(int(rng.integers(1, 3))):
+            b = base[int(rng.integers(0, 3))]
+            chains.append(W.chain_from_tokens(b[:16 * int(rng.integers(0, 300))]))
+            inst.append(i)
+    off = np.zeros(len(chains) + 1, np.uint64)
+    off[1:] = np.cumsum([c.shape[0] for c in chains])
+    ins = W.Instances(b=rng.integers(0, 40, I).astype(np.int32), qr=rng.integers(0, 5, I).astype(np.int32),
+                      q=rng.integers(0, 9000, I).astype(np.int64), S=rng.integers(0, 300000, I).astype(np.int64),
+                      M_KV=np.full(I, 10 ** 6, np.int64), B_max=np.full(I, 64, np.int32),
+                      cap_blocks=np.full(I, 4096, np.uint64), chain_inst=np.array(inst, np.uint32), chain_off=off,
+                      chain_hash=np.concatenate(chains).astype(np.uint64), chain_parent=np.zeros(len(chains), np.uint64))
+    return ins, win
+
+
+def test_noalloc_matches_context_scoring_on_two_calls_in_a_row(P):
+    wl = W.generate(0)
+    first = _noalloc_score(P, wl.instances, wl.window, wl.model, P.PS_PROBE_SEARCH)
+    _same(first, _context_score(P, wl.instances, wl.window, wl.model, P.PS_PROBE_SEARCH))
+    # the second call reuses the shared array left over from the first with other sizes
+    ins, win = _random_case(11, 70, 90)
+    second = _noalloc_score(P, ins, win, dict(W.MODEL_DEFAULT), P.PS_PROBE_LINEAR)
+    _same(second, _context_score(P, ins, win, dict(W.MODEL_DEFAULT), P.PS_PROBE_LINEAR))
+
+
+def test_noalloc_rejects_windows_beyond_its_fixed_scratch(P):
+    import torch
+    I = 1024
+    R = P.PS_NOALLOC_MAX_PAIRS // I + 1
+    win = make_window([(seq_tokens("A", 16), 2000.0, 50.0)] * R)
+    dwin = W.Window(**{k: _dev(getattr(win, k)) for k in win.__dataclass_fields__})
+    pw = P.Scheduler.make_window(dwin)
+    z32 = torch.zeros(I, dtype=torch.int32, device="cuda")
+    z64 = torch.zeros(I, dtype=torch.int64, device="cuda")
+    sa = P.PsStateArrays(z32.data_ptr(), z32.data_ptr(), z64.data_ptr(), z64.data_ptr(), z64.data_ptr(),
+                         z32.data_ptr())
+    best = torch.empty(R, dtype=torch.int32, device="cuda")
+    sc = P.PsScores(None, None, None, None, best.data_ptr(), None, 1)
+    slots = torch.zeros(16 * I, dtype=torch.int64, device="cuda")
+    desc = torch.zeros(2 * I, dtype=torch.int64, device="cuda")
+    m = P.make_model(dict(W.MODEL_DEFAULT))
+    status = P.lib().ps_score_window_noalloc(slots.data_ptr(), desc.data_ptr(), I, ctypes.byref(sa),
+                                             ctypes.byref(pw), ctypes.byref(m), 1, ctypes.byref(sc),
+                                             torch.cuda.current_stream().cuda_stream)
+    assert status == P.PS_ERR_INVALID
