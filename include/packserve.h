@@ -257,10 +257,15 @@ PS_API ps_status ps_last_timings(ps_ctx* ctx, float* ms, uint32_t n);
  * It computes what ps_score_window computes (probe kernel + fused score kernel, same results) for
  * caches laid out the way the library lays them out:
  *   slots    device u64 array holding every instance's table; value 0 = empty slot.
+ *   overflow_bits  device u64 array of overflow bitmaps, one bit per bucket.
  *   tables   device array [num_instances] of ps_table_desc: instance i's table is num_buckets
- *            buckets of 16 slots starting at slot `base`; block hash h lives in bucket
- *            (h * num_buckets) >> 64 (high 64 bits of the 128-bit product) or, if that bucket is
- *            full, in the following buckets (wrapping); each table must keep at least one empty slot.
+ *            buckets of 8 slots starting at slot `base`, and its overflow bitmap starts at word
+ *            `overflow_base` of overflow_bits (bit b of the bitmap = word b / 64, bit b % 64).
+ *            A block hash h has two candidate buckets, b1 = (h * num_buckets) >> 64 and
+ *            b2 = (g * num_buckets) >> 64 with g = (h ^ (h >> 31)) * 0x7FB5D329728EA185 mod 2^64
+ *            (high 64 bits of the 128-bit products), and is stored in one of them; if both were
+ *            full when it was inserted, it is stored in the first bucket after b1 (wrapping) that
+ *            had a free slot, and b1 and every bucket passed on the way carry overflow bit 1.
  *   state    device arrays of the instance state (ps_instance_state fields, structure of arrays).
  *   window   inputs_on_device must be 1; out->outputs_on_device must be 1 (all device buffers).
  *   probe_mode  as ps_config.probe_mode (PS_PROBE_SEARCH only for prefix-closed caches).
@@ -278,6 +283,7 @@ PS_API ps_status ps_last_timings(ps_ctx* ctx, float* ms, uint32_t n);
 
 typedef struct {
   uint64_t base;
+  uint64_t overflow_base;
   uint32_t num_buckets;
   uint32_t reserved;
 } ps_table_desc;
@@ -291,8 +297,9 @@ typedef struct {
   const int32_t* B_max;
 } ps_state_arrays;
 
-PS_API ps_status ps_score_window_noalloc(const uint64_t* slots, const ps_table_desc* tables,
-                                         uint32_t num_instances, const ps_state_arrays* state,
+PS_API ps_status ps_score_window_noalloc(const uint64_t* slots, const uint64_t* overflow_bits,
+                                         const ps_table_desc* tables, uint32_t num_instances,
+                                         const ps_state_arrays* state,
                                          const ps_window* window, const ps_model* model,
                                          int32_t probe_mode, ps_scores* out, void* cuda_stream);
 

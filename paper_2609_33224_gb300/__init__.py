@@ -68,7 +68,8 @@ class PsDecisions(ctypes.Structure):
 
 
 class PsTableDesc(ctypes.Structure):
-    _fields_ = [("base", ctypes.c_uint64), ("num_buckets", ctypes.c_uint32), ("reserved", ctypes.c_uint32)]
+    _fields_ = [("base", ctypes.c_uint64), ("overflow_base", ctypes.c_uint64), ("num_buckets", ctypes.c_uint32),
+                ("reserved", ctypes.c_uint32)]
 
 
 class PsStateArrays(ctypes.Structure):
@@ -106,7 +107,7 @@ def lib() -> ctypes.CDLL:
                                    ctypes.POINTER(PsScores)],
             "ps_commit_window": [vp, u32],
             "ps_last_timings": [vp, vp, u32],
-            "ps_score_window_noalloc": [vp, vp, u32, ctypes.POINTER(PsStateArrays), ctypes.POINTER(PsWindow),
+            "ps_score_window_noalloc": [vp, vp, vp, u32, ctypes.POINTER(PsStateArrays), ctypes.POINTER(PsWindow),
                                         ctypes.POINTER(PsModel), i32, ctypes.POINTER(PsScores), vp],
         }
         for name, args in sigs.items():

@@ -42,6 +42,8 @@ struct ps_ctx {
   std::vector<uint64_t> cap;
   uint64_t total_slots = 0;
   uint64_t* d_slots = nullptr;
+  uint64_t total_ovf = 0;
+  uint64_t* d_ovf = nullptr;
   psk::TableDesc* d_tdesc = nullptr;
   unsigned long long* d_count = nullptr;
   psk::DeltaSlot* d_delta = nullptr;
@@ -235,7 +237,7 @@ ps_status run_probe_and_score(ps_ctx* c, const psk::WindowDev& wd, ps_scores* ou
   const int dev_out = out ? out->outputs_on_device : 0;
   uint32_t* hits = (out && out->hits && dev_out) ? out->hits : c->d_hits;
   record(c, kEvProbe0);
-  PS_TRY_CUDA(c, pskl::launch_probe(c->d_slots, c->d_tdesc, c->I, wd, hits, c->probe_grid, c->search, c->stream));
+  PS_TRY_CUDA(c, pskl::launch_probe(c->d_slots, c->d_ovf, c->d_tdesc, c->I, wd, hits, c->probe_grid, c->search, c->stream));
   record(c, kEvProbe1);
   c->ev_used[0] = true;
   *hits_used = hits;
@@ -306,25 +308,30 @@ ps_status ps_create(const ps_config* cfg, ps_ctx** out) {
     if (cudaStreamCreateWithFlags(&c->stream, cudaStreamNonBlocking) != cudaSuccess) return bail(PS_ERR_CUDA);
     c->own_stream = true;
   }
-  // Instance tables: slots = ceil(cap / lf) rounded up to whole 16-slot buckets.
+  // Instance tables: slots = ceil(cap / lf) rounded up to whole 8-slot buckets; one overflow bit
+  // per bucket, each instance's bitmap starting on its own u64 word.
   std::vector<psk::TableDesc> td(c->I);
-  uint64_t base = 0;
+  uint64_t base = 0, obase = 0;
   for (uint32_t i = 0; i < c->I; ++i) {
     if (c->cap[i] < 1 || c->cap[i] > (1ull << 36)) return bail(PS_ERR_INVALID);
     const uint64_t slots = (uint64_t)std::ceil((double)c->cap[i] / (double)cfg->table_load_factor);
     const uint64_t nbkt = (slots + psk::kBucketSlots - 1) / psk::kBucketSlots;
     if (nbkt >= (1ull << 32)) return bail(PS_ERR_INVALID);
     td[i].base = base;
+    td[i].ovf = obase;
     td[i].nbkt = (uint32_t)nbkt;
+    td[i].pad = 0;
     base += nbkt * psk::kBucketSlots;
+    obase += (nbkt + 63) / 64;
   }
   c->total_slots = base;
+  c->total_ovf = obase;
   const uint64_t dn = (2 * c->max_blocks + psk::kDeltaSlots - 1) / psk::kDeltaSlots;
   if (dn >= (1ull << 32)) return bail(PS_ERR_INVALID);
   c->delta_nbkt = (uint32_t)dn;
   const size_t RI = (size_t)c->Rmax * c->I;
   const size_t I = c->I;
-  bool ok = dalloc(c, &c->d_slots, c->total_slots) == cudaSuccess &&
+  bool ok = dalloc(c, &c->d_slots, c->total_slots) == cudaSuccess && dalloc(c, &c->d_ovf, c->total_ovf) == cudaSuccess &&
             dalloc(c, &c->d_tdesc, I) == cudaSuccess && dalloc(c, &c->d_count, I) == cudaSuccess &&
             dalloc(c, &c->d_delta, (size_t)dn * psk::kDeltaSlots) == cudaSuccess &&
             dalloc(c, &c->d_dlog, c->max_blocks) == cudaSuccess && dalloc(c, &c->d_dlog_n, 1) == cudaSuccess;
@@ -350,6 +357,7 @@ ps_status ps_create(const ps_config* cfg, ps_ctx** out) {
   for (int e = 0; e < kNumEv; ++e)
     if (cudaEventCreate(&c->ev[e]) != cudaSuccess) return bail(PS_ERR_CUDA);
   bool set = cudaMemsetAsync(c->d_slots, 0, c->total_slots * sizeof(uint64_t), c->stream) == cudaSuccess &&
+             cudaMemsetAsync(c->d_ovf, 0, c->total_ovf * sizeof(uint64_t), c->stream) == cudaSuccess &&
              cudaMemcpyAsync(c->d_tdesc, td.data(), I * sizeof(psk::TableDesc), cudaMemcpyHostToDevice,
                              c->stream) == cudaSuccess &&
              cudaMemsetAsync(c->d_count, 0, I * sizeof(unsigned long long), c->stream) == cudaSuccess &&
@@ -489,10 +497,10 @@ ps_status ps_insert_chains(ps_ctx* c, uint64_t nchains, const uint32_t* inst, co
   } else {
     PS_TRY_CUDA(c, cudaMemcpy(&total, off + nchains, 8, cudaMemcpyDeviceToHost));
   }
-  cudaError_t e = pskl::launch_insert_chains(c->d_slots, c->d_tdesc, c->I, c->d_count, nchains, d_inst, d_off,
+  cudaError_t e = pskl::launch_insert_chains(c->d_slots, c->d_ovf, c->d_tdesc, c->I, c->d_count, nchains, d_inst, d_off,
                                              d_hash, total, c->d_err, c->num_sms, c->stream);
   if (e == cudaSuccess && c->search)
-    e = pskl::launch_check_parents(c->d_slots, c->d_tdesc, c->I, nchains, d_inst, d_parent, c->d_err, c->num_sms,
+    e = pskl::launch_check_parents(c->d_slots, c->d_ovf, c->d_tdesc, c->I, nchains, d_inst, d_parent, c->d_err, c->num_sms,
                                    c->stream);
   ps_status s = e == cudaSuccess ? finish(c) : fail(c, PS_ERR_CUDA, cudaGetErrorString(e));
   if (tmp) cudaFree(tmp);
@@ -548,7 +556,7 @@ ps_status ps_schedule_window(ps_ctx* c, const ps_window* w, ps_decisions* out, p
   s = run_probe_and_score(c, wd, opt_scores, &hit0);
   if (s != PS_OK) return s;
   record(c, kEvGreedy0);
-  PS_TRY_CUDA(c, pskl::launch_greedy(c->d_slots, c->d_tdesc, c->I, wd, hit0, c->st, c->pend, c->model, c->d_delta,
+  PS_TRY_CUDA(c, pskl::launch_greedy(c->d_slots, c->d_ovf, c->d_tdesc, c->I, wd, hit0, c->st, c->pend, c->model, c->d_delta,
                                      c->delta_nbkt, c->d_dlog, c->d_dlog_n, c->d_assign, c->d_dpath, c->d_hchosen,
                                      c->d_err, c->search, c->stream));
   record(c, kEvGreedy1);
@@ -572,7 +580,7 @@ ps_status ps_commit_window(ps_ctx* c, uint32_t last_use) {
   if (!c->pending) return fail(c, PS_ERR_STATE, "no pending window");
   DeviceGuard g(c->device);
   record(c, kEvCommit0);
-  PS_TRY_CUDA(c, pskl::launch_commit(c->d_slots, c->d_tdesc, c->I, c->d_count, c->pend_win, c->d_assign,
+  PS_TRY_CUDA(c, pskl::launch_commit(c->d_slots, c->d_ovf, c->d_tdesc, c->I, c->d_count, c->pend_win, c->d_assign,
                                      c->d_hchosen, c->d_err, c->num_sms, c->stream));
   const size_t I = c->I;
   PS_TRY_CUDA(c, cudaMemcpyAsync(c->st.b, c->pend.b, I * 4, cudaMemcpyDeviceToDevice, c->stream));

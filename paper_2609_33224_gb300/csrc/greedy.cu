@@ -23,7 +23,8 @@ namespace {
 
 template <int IPT, bool SEARCH>
 __global__ void __launch_bounds__(1024, 1)
-greedy_kernel(const uint64_t* __restrict__ slots, const psk::TableDesc* __restrict__ tdesc, uint32_t I,
+greedy_kernel(const uint64_t* __restrict__ slots, const uint64_t* __restrict__ ovf,
+              const psk::TableDesc* __restrict__ tdesc, uint32_t I,
               psk::WindowDev w, const uint32_t* __restrict__ hit0, psk::StateSoA committed,
               psk::StateSoA pending, psk::DevModel m, psk::DeltaSlot* delta, uint32_t delta_nbkt,
               unsigned long long* dlog, unsigned long long* dlog_n, int32_t* __restrict__ assign,
@@ -98,9 +99,12 @@ greedy_kernel(const uint64_t* __restrict__ slots, const psk::TableDesc* __restri
       for (uint32_t x = warp; x < nwalk; x += NW) {
         const uint32_t i = s_walk[x];
         const psk::TableDesc d = tdesc[i];
+        // Positions past hit0 are never in a prefix-closed main table (hit0 is its first miss), so
+        // the search only consults the delta; the linear walk checks both.
         auto cached = [&](uint64_t k) {
           const uint64_t key = w.hash[o + k];
-          return psk::delta_contains(delta, delta_nbkt, i, key) || psk::main_contains(slots, d, key);
+          return psk::delta_contains(delta, delta_nbkt, i, key) ||
+                 (!SEARCH && psk::main_contains(slots, ovf, d, key));
         };
         const uint64_t from = (uint64_t)s_h[i] + 1;
         const uint64_t hnew = SEARCH ? psk::warp_first_miss_search(from, nb, cached)
@@ -211,7 +215,8 @@ size_t greedy_smem(uint32_t I) {
 namespace pskl {
 
 template <int IPT, bool SEARCH>
-cudaError_t greedy_launch(const uint64_t* slots, const psk::TableDesc* tdesc, uint32_t I, const psk::WindowDev& w,
+cudaError_t greedy_launch(const uint64_t* slots, const uint64_t* ovf, const psk::TableDesc* tdesc, uint32_t I,
+                          const psk::WindowDev& w,
                           const uint32_t* hit0, psk::StateSoA committed, psk::StateSoA pending,
                           const psk::DevModel& m, psk::DeltaSlot* delta, uint32_t delta_nbkt,
                           unsigned long long* dlog, unsigned long long* dlog_n, int32_t* assign, uint8_t* path,
@@ -220,12 +225,12 @@ cudaError_t greedy_launch(const uint64_t* slots, const psk::TableDesc* tdesc, ui
   cudaError_t e = cudaFuncSetAttribute(greedy_kernel<IPT, SEARCH>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)smem);
   if (e != cudaSuccess) return e;
-  greedy_kernel<IPT, SEARCH><<<1, nt, smem, s>>>(slots, tdesc, I, w, hit0, committed, pending, m, delta,
+  greedy_kernel<IPT, SEARCH><<<1, nt, smem, s>>>(slots, ovf, tdesc, I, w, hit0, committed, pending, m, delta,
                                                  delta_nbkt, dlog, dlog_n, assign, path, hit_chosen, err);
   return cudaGetLastError();
 }
 
-cudaError_t launch_greedy(const uint64_t* slots, const psk::TableDesc* tdesc, uint32_t I,
+cudaError_t launch_greedy(const uint64_t* slots, const uint64_t* ovf, const psk::TableDesc* tdesc, uint32_t I,
                           const psk::WindowDev& w, const uint32_t* hit0, psk::StateSoA committed,
                           psk::StateSoA pending, const psk::DevModel& m, psk::DeltaSlot* delta,
                           uint32_t delta_nbkt, unsigned long long* dlog, unsigned long long* dlog_n,
@@ -235,9 +240,9 @@ cudaError_t launch_greedy(const uint64_t* slots, const psk::TableDesc* tdesc, ui
   if (nt > 1024) nt = 1024;
   const uint32_t ipt = (I + nt - 1) / nt;
 #define PS_GREEDY(IPT)                                                                                  \
-  return search ? greedy_launch<IPT, true>(slots, tdesc, I, w, hit0, committed, pending, m, delta, delta_nbkt, \
+  return search ? greedy_launch<IPT, true>(slots, ovf, tdesc, I, w, hit0, committed, pending, m, delta, delta_nbkt, \
                                            dlog, dlog_n, assign, path, hit_chosen, err, nt, s)           \
-                : greedy_launch<IPT, false>(slots, tdesc, I, w, hit0, committed, pending, m, delta, delta_nbkt, \
+                : greedy_launch<IPT, false>(slots, ovf, tdesc, I, w, hit0, committed, pending, m, delta, delta_nbkt, \
                                             dlog, dlog_n, assign, path, hit_chosen, err, nt, s)
   if (ipt <= 1) PS_GREEDY(1);
   if (ipt <= 2) PS_GREEDY(2);

@@ -87,10 +87,11 @@ static_assert(sizeof(ps_table_desc) == sizeof(psk::TableDesc), "ps_table_desc la
 
 extern "C" {
 
-ps_status ps_score_window_noalloc(const uint64_t* slots, const ps_table_desc* tables, uint32_t num_instances,
+ps_status ps_score_window_noalloc(const uint64_t* slots, const uint64_t* overflow_bits, const ps_table_desc* tables,
+                                  uint32_t num_instances,
                                   const ps_state_arrays* state, const ps_window* w, const ps_model* model,
                                   int32_t probe_mode, ps_scores* out, void* cuda_stream) {
-  if (!slots || !tables || !state || !w || !model || !out) return PS_ERR_INVALID;
+  if (!slots || !overflow_bits || !tables || !state || !w || !model || !out) return PS_ERR_INVALID;
   if (num_instances < 1 || num_instances > 4096) return PS_ERR_INVALID;
   if (w->inputs_on_device != 1 || out->outputs_on_device != 1) return PS_ERR_INVALID;
   if (probe_mode != PS_PROBE_LINEAR && probe_mode != PS_PROBE_SEARCH) return PS_ERR_INVALID;
@@ -122,7 +123,7 @@ ps_status ps_score_window_noalloc(const uint64_t* slots, const ps_table_desc* ta
   if (herr != 0 || (nblk > 0 && !w->chain_hash)) return PS_ERR_INVALID;
   const psk::TableDesc* td = reinterpret_cast<const psk::TableDesc*>(tables);
   const int grid = num_instances >= 64 ? d->probe_grid_large : d->probe_grid_small;
-  if (pskl::launch_probe(slots, td, num_instances, wd, hits, grid, probe_mode == PS_PROBE_SEARCH, s) != cudaSuccess)
+  if (pskl::launch_probe(slots, overflow_bits, td, num_instances, wd, hits, grid, probe_mode == PS_PROBE_SEARCH, s) != cudaSuccess)
     return PS_ERR_CUDA;
   const psk::StateSoA soa{const_cast<int32_t*>(state->b), const_cast<int32_t*>(state->qr),
                           const_cast<int64_t*>(state->q_tokens), const_cast<int64_t*>(state->S_tokens),

@@ -18,7 +18,8 @@ constexpr uint32_t kStageBlocks = 8192;  // 64 KB of staged chain per thread blo
 
 template <int WARPS, bool SEARCH>
 __global__ void __launch_bounds__(WARPS * 32)
-probe_hits_kernel(const uint64_t* __restrict__ slots, const psk::TableDesc* __restrict__ tdesc,
+probe_hits_kernel(const uint64_t* __restrict__ slots, const uint64_t* __restrict__ ovf,
+                  const psk::TableDesc* __restrict__ tdesc,
                   uint32_t I, const uint64_t* __restrict__ off, const uint64_t* __restrict__ hash,
                   uint32_t R, uint32_t* __restrict__ hits) {
   extern __shared__ uint64_t s_chain[];
@@ -34,7 +35,7 @@ probe_hits_kernel(const uint64_t* __restrict__ slots, const psk::TableDesc* __re
       const psk::TableDesc d = tdesc[i];
       auto cached = [&](uint64_t k) {
         const uint64_t key = k < ns ? s_chain[k] : __ldg(hash + o + k);
-        return psk::main_contains(slots, d, key);
+        return psk::main_contains(slots, ovf, d, key);
       };
       const uint64_t h = SEARCH ? psk::warp_first_miss_search(0, nb, cached)
                                 : psk::warp_first_miss_linear(0, nb, cached);
@@ -65,21 +66,21 @@ int probe_max_grid(uint32_t I, int num_sms) {
   return I >= 64 ? max_grid<16>(num_sms) : max_grid<4>(num_sms);
 }
 
-cudaError_t launch_probe(const uint64_t* slots, const psk::TableDesc* tdesc, uint32_t I,
+cudaError_t launch_probe(const uint64_t* slots, const uint64_t* ovf, const psk::TableDesc* tdesc, uint32_t I,
                          const psk::WindowDev& w, uint32_t* hits, int grid, int search, cudaStream_t s) {
   if (w.R == 0) return cudaSuccess;
   const int g = (int)((uint32_t)grid < w.R ? (uint32_t)grid : w.R);
   const size_t smem = kStageBlocks * sizeof(uint64_t);
   if (I >= 64) {
     if (search)
-      probe_hits_kernel<16, true><<<g, 16 * 32, smem, s>>>(slots, tdesc, I, w.off, w.hash, w.R, hits);
+      probe_hits_kernel<16, true><<<g, 16 * 32, smem, s>>>(slots, ovf, tdesc, I, w.off, w.hash, w.R, hits);
     else
-      probe_hits_kernel<16, false><<<g, 16 * 32, smem, s>>>(slots, tdesc, I, w.off, w.hash, w.R, hits);
+      probe_hits_kernel<16, false><<<g, 16 * 32, smem, s>>>(slots, ovf, tdesc, I, w.off, w.hash, w.R, hits);
   } else {
     if (search)
-      probe_hits_kernel<4, true><<<g, 4 * 32, smem, s>>>(slots, tdesc, I, w.off, w.hash, w.R, hits);
+      probe_hits_kernel<4, true><<<g, 4 * 32, smem, s>>>(slots, ovf, tdesc, I, w.off, w.hash, w.R, hits);
     else
-      probe_hits_kernel<4, false><<<g, 4 * 32, smem, s>>>(slots, tdesc, I, w.off, w.hash, w.R, hits);
+      probe_hits_kernel<4, false><<<g, 4 * 32, smem, s>>>(slots, ovf, tdesc, I, w.off, w.hash, w.R, hits);
   }
   return cudaGetLastError();
 }

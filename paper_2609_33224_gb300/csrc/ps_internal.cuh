@@ -1,14 +1,20 @@
 // Device-side data layout and shared device functions of the scheduler library (sm_103a).
 //
 // HBM layout
-//   main tables   one u64 slot array for all instances; instance i owns buckets [0, nbkt_i) starting
-//                 at slot base_i.  A bucket is 16 slots = one 128-byte line.  A key's home bucket
-//                 is fastrange(key, nbkt_i) (the high 64 bits of key * nbkt_i); collisions go to the
-//                 next bucket (linear probing over buckets).  Slot value 0 = empty.
+//   main tables   one u64 slot array for all instances; instance i owns nbkt_i buckets of 8 slots
+//                 (one 64-byte half line each) starting at slot base_i.  Balanced two-choice
+//                 hashing: a block hash h may live in bucket b1 = fastrange(h) or
+//                 b2 = fastrange(remix(h)) and is inserted into the emptier of the two (b1 on
+//                 ties).  A lookup reads both 64-byte buckets at once, so a hit or a miss costs one
+//                 memory round trip.  If both buckets are full the key goes to the first non-full
+//                 bucket after b1 (wrapping) and b1 plus every full bucket passed get their bit set
+//                 in the instance's overflow bitmap; at load factor 0.9 about 0.6% of keys take that
+//                 path.  Slot value 0 = empty.  Each table has a single writer (one warp per
+//                 instance), so placement needs no atomics and a key is never stored twice.
 //   delta table   window-scoped set of (instance, block) pairs cached by the window's own earlier
-//                 decisions: 16-byte slots {hash, instance}, 8 per 128-byte bucket, sized at twice the
-//                 window's block bound so it can never fill.  Cleared (through its insert log) after
-//                 each window.
+//                 decisions: 16-byte slots {hash, instance}, 8 per 128-byte bucket, linear probing,
+//                 sized at twice the window's block bound so it can never fill.  Cleared (through its
+//                 insert log) after each window.
 //   state         structure of arrays per instance (b, qr, q, S, M_KV, B_max).
 //   hits          u32 [R x I], request-major.
 #pragma once
@@ -20,7 +26,7 @@ namespace psk {
 
 constexpr uint64_t kEmpty = 0ull;
 constexpr uint64_t kTomb = ~0ull;
-constexpr int kBucketSlots = 16;   // main table: 16 x 8 B
+constexpr int kBucketSlots = 8;    // main table: 8 x 8 B = 64 B
 constexpr int kDeltaSlots = 8;     // delta table: 8 x 16 B
 constexpr uint32_t kDeltaNoInst = 0xFFFFFFFFu;
 
@@ -36,6 +42,7 @@ enum : uint32_t {
 
 struct TableDesc {
   uint64_t base;   // first slot of the instance's table
+  uint64_t ovf;    // first u64 word of the instance's overflow bitmap (one bit per bucket)
   uint32_t nbkt;   // buckets
   uint32_t pad;
 };
@@ -75,44 +82,88 @@ __device__ __forceinline__ uint32_t fastrange32(uint64_t h, uint32_t n) {
   return (uint32_t)__umul64hi(h, (unsigned long long)n);
 }
 
-// Membership in an instance's main table.  Read-only during every kernel that calls it, so the
-// non-coherent read-only path is used.  A probe reads whole 128-byte buckets as 8 x 16-byte loads.
-__device__ __forceinline__ bool main_contains(const uint64_t* __restrict__ slots, const TableDesc d,
-                                              uint64_t key) {
+// Second bucket choice: an odd-constant multiply of a folded key, so fastrange of it uses bits
+// independent of the ones that pick the first bucket.
+__device__ __forceinline__ uint64_t remix(uint64_t k) { return (k ^ (k >> 31)) * 0x7FB5D329728EA185ull; }
+
+__device__ __forceinline__ bool ovf_bit(const uint64_t* ovf, const TableDesc& d, uint32_t b) {
+  return (ovf[d.ovf + (b >> 6)] >> (b & 63)) & 1ull;
+}
+
+// Membership in an instance's main table.  Both candidate buckets (2 x 4 x 16-byte loads) and the
+// overflow word are requested before any comparison.  LOAD selects the read path: the read-only
+// path for kernels that never write the tables, the L2-coherent path for the table writers.
+template <bool RO = true>
+__device__ __forceinline__ bool main_contains(const uint64_t* __restrict__ slots, const uint64_t* __restrict__ ovf,
+                                              const TableDesc d, uint64_t key) {
   if (key == kEmpty || key == kTomb) return false;
-  uint32_t b = fastrange32(key, d.nbkt);
-  for (uint32_t p = 0; p < d.nbkt; ++p) {
-    const ulonglong2* line = reinterpret_cast<const ulonglong2*>(slots + d.base + (uint64_t)b * kBucketSlots);
-    bool empty = false;
+  const uint32_t b1 = fastrange32(key, d.nbkt);
+  const uint32_t b2 = fastrange32(remix(key), d.nbkt);
+  const ulonglong2* l1 = reinterpret_cast<const ulonglong2*>(slots + d.base + (uint64_t)b1 * kBucketSlots);
+  const ulonglong2* l2 = reinterpret_cast<const ulonglong2*>(slots + d.base + (uint64_t)b2 * kBucketSlots);
+  ulonglong2 v[8];
 #pragma unroll
-    for (int k = 0; k < kBucketSlots / 2; ++k) {
-      const ulonglong2 v = __ldg(line + k);
-      if (v.x == key || v.y == key) return true;
-      empty |= (v.x == kEmpty) | (v.y == kEmpty);
-    }
-    if (empty) return false;
+  for (int k = 0; k < 4; ++k) {
+    v[k] = RO ? __ldg(l1 + k) : __ldcg(l1 + k);
+    v[4 + k] = RO ? __ldg(l2 + k) : __ldcg(l2 + k);
+  }
+  const uint64_t* ow_p = ovf + d.ovf + (b1 >> 6);
+  const uint64_t ow = RO ? __ldg(ow_p) : __ldcg(ow_p);
+  bool hit = false;
+#pragma unroll
+  for (int k = 0; k < 8; ++k) hit |= (v[k].x == key) | (v[k].y == key);
+  if (hit) return true;
+  if (!((ow >> (b1 & 63)) & 1ull)) return false;
+  uint32_t b = b1;  // rare: follow the overflow run after b1
+  for (uint32_t p = 1; p < d.nbkt; ++p) {
     b = (b + 1 == d.nbkt) ? 0u : b + 1;
+    const ulonglong2* l = reinterpret_cast<const ulonglong2*>(slots + d.base + (uint64_t)b * kBucketSlots);
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const ulonglong2 x = RO ? __ldg(l + k) : __ldcg(l + k);
+      if (x.x == key || x.y == key) return true;
+    }
+    const uint64_t* q = ovf + d.ovf + (b >> 6);
+    if (!(((RO ? __ldg(q) : __ldcg(q)) >> (b & 63)) & 1ull)) return false;
   }
   return false;
 }
 
-// Insert into a main table.  Returns 1 if inserted, 0 if already present, -1 if the table is full.
-// Concurrent inserts of the same key are safe: they scan the same slot sequence, and a failed CAS
-// that returns the key itself means another thread inserted it.
-__device__ __forceinline__ int main_insert(uint64_t* slots, const TableDesc d, uint64_t key) {
-  uint32_t b = fastrange32(key, d.nbkt);
-  for (uint32_t p = 0; p < d.nbkt; ++p) {
-    unsigned long long* line = reinterpret_cast<unsigned long long*>(slots + d.base + (uint64_t)b * kBucketSlots);
-    for (int k = 0; k < kBucketSlots; ++k) {
-      const unsigned long long v = __ldcg(line + k);
-      if (v == key) return 0;
-      if (v == kEmpty) {
-        const unsigned long long old = atomicCAS(line + k, kEmpty, (unsigned long long)key);
-        if (old == kEmpty) return 1;
-        if (old == key) return 0;
-      }
-    }
+// Warp-cooperative insert of one key by the instance's only writer warp (all 32 lanes call it with
+// the same key).  Lanes 0-7 read bucket b1, lanes 8-15 bucket b2; the key goes to the emptier one.
+// Returns 1 if inserted, 0 if already present, -1 if the table is full.
+__device__ __forceinline__ int warp_insert(uint64_t* slots, uint64_t* ovf, const TableDesc d, uint64_t key) {
+  const int lane = threadIdx.x & 31;
+  if (main_contains<false>(slots, ovf, d, key)) return 0;
+  const uint32_t b1 = fastrange32(key, d.nbkt);
+  const uint32_t b2 = fastrange32(remix(key), d.nbkt);
+  uint64_t* p = nullptr;
+  if (lane < 8) p = slots + d.base + (uint64_t)b1 * kBucketSlots + lane;
+  else if (lane < 16) p = slots + d.base + (uint64_t)b2 * kBucketSlots + (lane - 8);
+  const uint64_t v = p ? __ldcg(reinterpret_cast<const unsigned long long*>(p)) : ~0ull;
+  const unsigned empty = __ballot_sync(0xffffffffu, p != nullptr && v == kEmpty);
+  const unsigned e1 = empty & 0xFFu, e2 = empty & 0xFF00u;
+  int target = -1;  // lane whose slot receives the key
+  if (e1 || e2) {
+    // emptier bucket (more empty slots), b1 on ties
+    target = (__popc(e1) >= __popc(e2)) ? __ffs(e1) - 1 : __ffs(e2) - 1;
+    if (lane == target) *p = key;
+    __syncwarp();
+    return 1;
+  }
+  // both full: first non-full bucket after b1; mark b1 and every full bucket passed
+  uint32_t b = b1;
+  for (uint32_t step = 0; step < d.nbkt; ++step) {
+    if (lane == 0) atomicOr(reinterpret_cast<unsigned long long*>(ovf + d.ovf + (b >> 6)), 1ull << (b & 63));
     b = (b + 1 == d.nbkt) ? 0u : b + 1;
+    uint64_t* q = slots + d.base + (uint64_t)b * kBucketSlots + (lane & 7);
+    const uint64_t w = lane < 8 ? __ldcg(reinterpret_cast<const unsigned long long*>(q)) : ~0ull;
+    const unsigned em = __ballot_sync(0xffffffffu, lane < 8 && w == kEmpty);
+    if (em) {
+      if (lane == __ffs(em) - 1) *q = key;
+      __syncwarp();
+      return 1;
+    }
   }
   return -1;
 }
@@ -349,13 +400,13 @@ constexpr uint32_t kNoKeyCi = 0xFFFFFFFFu;  // class 15: worse than any real pai
 
 // Kernel launchers (one translation unit each).
 namespace pskl {
-cudaError_t launch_probe(const uint64_t* slots, const psk::TableDesc* tdesc, uint32_t I,
+cudaError_t launch_probe(const uint64_t* slots, const uint64_t* ovf, const psk::TableDesc* tdesc, uint32_t I,
                          const psk::WindowDev& w, uint32_t* hits, int grid, int search, cudaStream_t s);
 int probe_max_grid(uint32_t I, int num_sms);
 cudaError_t launch_score(const uint32_t* hits, psk::StateSoA st, uint32_t I, const psk::WindowDev& w,
                          const psk::DevModel& m, float* tpot, float* ttft, uint8_t* cls, int32_t* best,
                          uint8_t* path, int num_sms, cudaStream_t s);
-cudaError_t launch_greedy(const uint64_t* slots, const psk::TableDesc* tdesc, uint32_t I,
+cudaError_t launch_greedy(const uint64_t* slots, const uint64_t* ovf, const psk::TableDesc* tdesc, uint32_t I,
                           const psk::WindowDev& w, const uint32_t* hit0, psk::StateSoA committed,
                           psk::StateSoA pending, const psk::DevModel& m, psk::DeltaSlot* delta,
                           uint32_t delta_nbkt, unsigned long long* dlog, unsigned long long* dlog_n,
@@ -364,14 +415,14 @@ cudaError_t launch_greedy(const uint64_t* slots, const psk::TableDesc* tdesc, ui
 cudaError_t launch_delta_clear(psk::DeltaSlot* delta, const unsigned long long* dlog,
                                unsigned long long* dlog_n, uint64_t max_entries, int num_sms,
                                cudaStream_t s);
-cudaError_t launch_insert_chains(uint64_t* slots, const psk::TableDesc* tdesc, uint32_t I,
+cudaError_t launch_insert_chains(uint64_t* slots, uint64_t* ovf, const psk::TableDesc* tdesc, uint32_t I,
                                  unsigned long long* count, uint64_t nchains, const uint32_t* inst,
                                  const uint64_t* off, const uint64_t* hash, uint64_t total,
                                  uint32_t* err, int num_sms, cudaStream_t s);
-cudaError_t launch_commit(uint64_t* slots, const psk::TableDesc* tdesc, uint32_t I,
+cudaError_t launch_commit(uint64_t* slots, uint64_t* ovf, const psk::TableDesc* tdesc, uint32_t I,
                           unsigned long long* count, const psk::WindowDev& w, const int32_t* assign,
                           const uint32_t* hit_chosen, uint32_t* err, int num_sms, cudaStream_t s);
-cudaError_t launch_check_parents(const uint64_t* slots, const psk::TableDesc* tdesc, uint32_t I,
+cudaError_t launch_check_parents(const uint64_t* slots, const uint64_t* ovf, const psk::TableDesc* tdesc, uint32_t I,
                                  uint64_t nchains, const uint32_t* inst, const uint64_t* parent,
                                  uint32_t* err, int num_sms, cudaStream_t s);
 cudaError_t launch_validate_window(const psk::WindowDev& w, uint64_t max_blocks, uint32_t* err,

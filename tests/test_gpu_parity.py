@@ -263,12 +263,52 @@ def test_invalid_windows_are_rejected(P):
 
 def test_capacity_and_table_full_errors(P):
     model = dict(W.MODEL_DEFAULT)
+    # capacity 20 at load factor 0.9: ceil(20 / 0.9) = 23 slots -> 3 buckets of 8 = 24 slots
     with P.Scheduler(2, [20, 20], 4, 64, model, table_load_factor=0.9) as s:
-        ch = np.arange(1, 30, dtype=np.uint64) * 0x9E3779B97F4A7C15 % (1 << 63) + 1
+        ch = np.arange(1, 40, dtype=np.uint64) * np.uint64(0x9E3779B97F4A7C15) % np.uint64(1 << 63) + np.uint64(1)
         with pytest.raises(P.PSError) as e:
-            s.insert_blocks(0, ch[:25])
+            s.insert_blocks(0, ch[:22])
         assert e.value.status == P.PS_ERR_CAPACITY
-        assert int(s.cached_blocks()[0]) == 25
+        assert int(s.cached_blocks()[0]) == 22
+        with pytest.raises(P.PSError) as e:
+            s.insert_blocks(0, ch[22:30], parent=int(ch[21]))
+        assert e.value.status == P.PS_ERR_TABLE_FULL
+        assert int(s.cached_blocks()[0]) == 24
+
+
+@pytest.mark.parametrize("mode", MODES)
+def test_overflow_runs_at_high_load_factor(P, mode):
+    """Tables at 95% load: many keys find both candidate buckets full and go to the overflow run;
+    hits must still equal the oracle's."""
+    rng = np.random.default_rng(21)
+    I, cap = 3, 2000
+    bases = [rng.integers(0, 1 << 17, 16 * 900).astype(np.uint32) for _ in range(3)]
+    chains, inst = [], []
+    for i in range(I):
+        n_seq = W.chain_from_tokens(bases[i][:16 * 800])
+        chains.append(n_seq)
+        inst.append(i)
+        filler = (rng.integers(1, 1 << 62, cap - 800, dtype=np.int64)).astype(np.uint64)
+        chains.append(filler)
+        inst.append(i)
+    off = np.zeros(len(chains) + 1, np.uint64)
+    off[1:] = np.cumsum([c.shape[0] for c in chains])
+    ins = W.Instances(b=np.array([5, 9, 1], np.int32), qr=np.zeros(I, np.int32), q=np.zeros(I, np.int64),
+                      S=np.zeros(I, np.int64), M_KV=np.full(I, 10 ** 8, np.int64), B_max=np.full(I, 64, np.int32),
+                      cap_blocks=np.full(I, cap, np.uint64), chain_inst=np.array(inst, np.uint32), chain_off=off,
+                      chain_hash=np.concatenate(chains).astype(np.uint64), chain_parent=np.zeros(len(chains), np.uint64))
+    reqs = [(bases[int(rng.integers(0, 3))][:int(rng.integers(0, 16 * 900))], 2000.0, 50.0) for _ in range(60)]
+    win = make_window(reqs)
+    model = dict(W.MODEL_DEFAULT)
+    orc = _oracle(model, ins)
+    with P.Scheduler(I, ins.cap_blocks, win.R, int(win.chain_off[-1]), model, table_load_factor=0.95,
+                     probe_mode=mode) as s:
+        s.load_workload_instances(ins)
+        assert s.cached_blocks().tolist() == [cap] * I
+        g = s.score_window(win)
+        _assert_scores(g, orc.score_rows(win))
+        gd, od = s.schedule_window(win), orc.schedule(win)
+        assert np.array_equal(gd["assign"], od["assign"]) and np.array_equal(gd["hit_chosen"], od["hit_chosen"])
 
 
 @pytest.mark.parametrize("tpot,mode", [(30.0, 1), (50.0, 1), (50.0, 0)])

@@ -30,31 +30,60 @@ def P():
 
 
 def _caller_tables(ins):
-    """The documented layout, built on the host: 16-slot buckets, home bucket (h * nbkt) >> 64,
-    linear probing over buckets, 0 = empty; two slots per cached block (load factor 0.5)."""
+    """The documented layout, built on the host: 8-slot buckets, candidate buckets
+    b1 = (h * nbkt) >> 64 and b2 = (((h ^ (h >> 31)) * 0x7FB5D329728EA185) mod 2^64 * nbkt) >> 64,
+    each key in the emptier candidate (b1 on ties), both-full keys in the first bucket with room after
+    b1 with overflow bits on b1 and every bucket passed; about two slots per cached block."""
     I = ins.I
+    M64 = (1 << 64) - 1
     per = np.bincount(ins.chain_inst, weights=np.diff(ins.chain_off).astype(np.float64), minlength=I)
-    nbkt = [max(1, math.ceil(2 * int(n) / 16) + 1) for n in per]
+    nbkt = [max(1, math.ceil(2 * int(n) / 8) + 1) for n in per]
     base = np.zeros(I, np.uint64)
-    base[1:] = np.cumsum(np.array(nbkt[:-1], np.uint64) * 16)
-    slots = np.zeros(int(sum(nbkt)) * 16, np.uint64)
+    base[1:] = np.cumsum(np.array(nbkt[:-1], np.uint64) * 8)
+    obase = np.zeros(I, np.uint64)
+    obase[1:] = np.cumsum(np.array([(n + 63) // 64 for n in nbkt[:-1]], np.uint64))
+    slots = np.zeros(int(sum(nbkt)) * 8, np.uint64)
+    ovf = np.zeros(max(1, int(sum((n + 63) // 64 for n in nbkt))), np.uint64)
+
+    def bucket(i, b):
+        return slots[int(base[i]) + 8 * b: int(base[i]) + 8 * b + 8]
+
+    def bit(i, b):
+        return (int(ovf[int(obase[i]) + b // 64]) >> (b % 64)) & 1
+
     for c in range(ins.chain_inst.shape[0]):
         i = int(ins.chain_inst[c])
+        n = nbkt[i]
         for key in ins.chain_hash[ins.chain_off[c]:ins.chain_off[c + 1]]:
             key = int(key)
-            b = (key * nbkt[i]) >> 64
+            b1 = (key * n) >> 64
+            b2 = ((((key ^ (key >> 31)) * 0x7FB5D329728EA185) & M64) * n) >> 64
+            present = (bucket(i, b1) == key).any() or (bucket(i, b2) == key).any()
+            b = b1
+            while not present and bit(i, b):
+                b = (b + 1) % n
+                present = (bucket(i, b) == key).any()
+            if present:
+                continue
+            e1, e2 = int((bucket(i, b1) == 0).sum()), int((bucket(i, b2) == 0).sum())
+            if e1 or e2:
+                tb = b1 if e1 >= e2 else b2
+                line = bucket(i, tb)
+                line[np.nonzero(line == 0)[0][0]] = key
+                continue
+            b = b1
             while True:
-                line = slots[int(base[i]) + 16 * b: int(base[i]) + 16 * b + 16]
-                if (line == key).any():
+                w = int(obase[i]) + b // 64
+                ovf[w] = np.uint64(int(ovf[w]) | (1 << (b % 64)))
+                b = (b + 1) % n
+                line = bucket(i, b)
+                if (line == 0).any():
+                    line[np.nonzero(line == 0)[0][0]] = key
                     break
-                empty = np.nonzero(line == 0)[0]
-                if empty.size:
-                    line[empty[0]] = key
-                    break
-                b = (b + 1) % nbkt[i]
-    desc = np.zeros(I, dtype=np.dtype([("base", np.uint64), ("num_buckets", np.uint32), ("reserved", np.uint32)]))
-    desc["base"], desc["num_buckets"] = base, nbkt
-    return slots, desc
+    desc = np.zeros(I, dtype=np.dtype([("base", np.uint64), ("overflow_base", np.uint64),
+                                       ("num_buckets", np.uint32), ("reserved", np.uint32)]))
+    desc["base"], desc["overflow_base"], desc["num_buckets"] = base, obase, nbkt
+    return slots, ovf, desc
 
 
 def _dev(a):
@@ -69,8 +98,8 @@ def _dev(a):
 def _noalloc_score(P, ins, win, model, mode):
     """One call of the allocation-free entry point with caller-owned device buffers."""
     import torch
-    slots, desc = _caller_tables(ins)
-    d_slots, d_desc = _dev(slots), _dev(desc)
+    slots, ovf, desc = _caller_tables(ins)
+    d_slots, d_ovf, d_desc = _dev(slots), _dev(ovf), _dev(desc)
     st = {k: _dev(getattr(ins, k)) for k in ("b", "qr", "q", "S", "M_KV", "B_max")}
     sa = P.PsStateArrays(st["b"].data_ptr(), st["qr"].data_ptr(), st["q"].data_ptr(), st["S"].data_ptr(),
                          st["M_KV"].data_ptr(), st["B_max"].data_ptr())
@@ -85,7 +114,8 @@ def _noalloc_score(P, ins, win, model, mode):
            "path": torch.empty(R, dtype=torch.uint8, device="cuda")}
     sc = P.PsScores(*(out[k].data_ptr() for k in ("hits", "tpot", "ttft", "cls", "best", "path")), 1)
     m = P.make_model(model)
-    status = P.lib().ps_score_window_noalloc(d_slots.data_ptr(), d_desc.data_ptr(), I, ctypes.byref(sa),
+    status = P.lib().ps_score_window_noalloc(d_slots.data_ptr(), d_ovf.data_ptr(), d_desc.data_ptr(), I,
+                                             ctypes.byref(sa),
                                              ctypes.byref(pw), ctypes.byref(m), int(mode), ctypes.byref(sc),
                                              torch.cuda.current_stream().cuda_stream)
     assert status == P.PS_OK, P.STATUS_NAMES.get(status, status)
@@ -158,10 +188,11 @@ def test_noalloc_rejects_windows_beyond_its_fixed_scratch(P):
                          z32.data_ptr())
     best = torch.empty(R, dtype=torch.int32, device="cuda")
     sc = P.PsScores(None, None, None, None, best.data_ptr(), None, 1)
-    slots = torch.zeros(16 * I, dtype=torch.int64, device="cuda")
-    desc = torch.zeros(2 * I, dtype=torch.int64, device="cuda")
+    slots = torch.zeros(8 * I, dtype=torch.int64, device="cuda")
+    ovf = torch.zeros(I, dtype=torch.int64, device="cuda")
+    desc = torch.zeros(3 * I, dtype=torch.int64, device="cuda")
     m = P.make_model(dict(W.MODEL_DEFAULT))
-    status = P.lib().ps_score_window_noalloc(slots.data_ptr(), desc.data_ptr(), I, ctypes.byref(sa),
+    status = P.lib().ps_score_window_noalloc(slots.data_ptr(), ovf.data_ptr(), desc.data_ptr(), I, ctypes.byref(sa),
                                              ctypes.byref(pw), ctypes.byref(m), 1, ctypes.byref(sc),
                                              torch.cuda.current_stream().cuda_stream)
     assert status == P.PS_ERR_INVALID
