@@ -113,37 +113,21 @@ class ClockSampler:
 
 
 def search_probe_count(h: np.ndarray, nb: np.ndarray) -> np.ndarray:
-    """Probes the 32-ary first-miss search makes for hit h on a chain of nb blocks: 32 per step
-    while the interval spans more than 32 positions, then one probe per remaining position."""
+    """Probes the per-lane binary search makes for hit h on a chain of nb blocks: one per step of
+    lo, hi = 0, nb; while lo < hi: mid = (lo + hi) // 2; lo = mid + 1 if mid < h else hi = mid."""
     h = h.astype(np.int64)
     lo = np.zeros_like(h)
     hi = np.broadcast_to(nb, h.shape).astype(np.int64).copy()
     cnt = np.zeros_like(h)
-    live = np.ones(h.shape, bool)
-    for _ in range(8):
-        span = hi - lo
-        fin = live & (span <= 32)
-        cnt[fin] += span[fin]
-        live &= ~fin
+    while True:
+        live = lo < hi
         if not live.any():
-            break
-        cnt[live] += 32
-        # first j with p_j = lo + (j+1) span / 32 - 1 >= h; none -> done (h = hi)
-        j = np.zeros_like(h)
-        found = np.zeros(h.shape, bool)
-        for jj in range(32):
-            p = lo + ((jj + 1) * span) // 32 - 1
-            hit = live & ~found & (p >= h)
-            j[hit] = jj
-            found |= hit
-        done = live & ~found
-        live &= found
-        newhi = lo + ((j + 1) * span) // 32 - 1
-        newlo = lo + (j * span) // 32
-        hi = np.where(live, newhi, hi)
-        lo = np.where(live, newlo, lo)
-        live &= ~done
-    return cnt
+            return cnt
+        mid = (lo + hi) >> 1
+        cnt += live
+        up = live & (mid < h)
+        lo = np.where(up, mid + 1, lo)
+        hi = np.where(live & ~up, mid, hi)
 
 
 def probe_algorithmic_bytes(hits: np.ndarray, nb: np.ndarray, search: bool) -> int:
@@ -350,7 +334,7 @@ def main():
             "decisions_per_s": world * R / (ms / 1000),
             "config": {"workload": WORKLOADS.get(args.config, str(args.config)), "instances": I,
                        "window_requests": R, "window_chain_blocks": int(nb.sum()),
-                       "tpot_target_ms": float(win.tpot_target[0]), "probe": ("32-ary first-miss search (prefix-closed caches)" if args.probe_mode == 1
+                       "tpot_target_ms": float(win.tpot_target[0]), "probe": ("per-lane binary first-miss search (prefix-closed caches)" if args.probe_mode == 1
                                  else "linear 32-wide warp walk"), "probes_per_window": n_probes,
                        "l2": "inputs larger than L2 (no flush)", "path_counts": path_counts},
             "kernel_ms": km,

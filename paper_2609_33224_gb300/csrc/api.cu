@@ -48,8 +48,6 @@ struct ps_ctx {
   unsigned long long* d_count = nullptr;
   psk::DeltaSlot* d_delta = nullptr;
   uint32_t delta_nbkt = 0;
-  unsigned long long* d_dlog = nullptr;
-  unsigned long long* d_dlog_n = nullptr;
   psk::StateSoA st{}, pend{};
   uint64_t* d_off = nullptr;
   uint64_t* d_hash = nullptr;
@@ -333,8 +331,7 @@ ps_status ps_create(const ps_config* cfg, ps_ctx** out) {
   const size_t I = c->I;
   bool ok = dalloc(c, &c->d_slots, c->total_slots) == cudaSuccess && dalloc(c, &c->d_ovf, c->total_ovf) == cudaSuccess &&
             dalloc(c, &c->d_tdesc, I) == cudaSuccess && dalloc(c, &c->d_count, I) == cudaSuccess &&
-            dalloc(c, &c->d_delta, (size_t)dn * psk::kDeltaSlots) == cudaSuccess &&
-            dalloc(c, &c->d_dlog, c->max_blocks) == cudaSuccess && dalloc(c, &c->d_dlog_n, 1) == cudaSuccess;
+            dalloc(c, &c->d_delta, (size_t)dn * psk::kDeltaSlots) == cudaSuccess;
   for (psk::StateSoA* s : {&c->st, &c->pend}) {
     ok = ok && dalloc(c, &s->b, I) == cudaSuccess && dalloc(c, &s->qr, I) == cudaSuccess &&
          dalloc(c, &s->q, I) == cudaSuccess && dalloc(c, &s->S, I) == cudaSuccess &&
@@ -363,7 +360,6 @@ ps_status ps_create(const ps_config* cfg, ps_ctx** out) {
              cudaMemsetAsync(c->d_count, 0, I * sizeof(unsigned long long), c->stream) == cudaSuccess &&
              cudaMemsetAsync(c->d_delta, 0, (size_t)dn * psk::kDeltaSlots * sizeof(psk::DeltaSlot), c->stream) ==
                  cudaSuccess &&
-             cudaMemsetAsync(c->d_dlog_n, 0, sizeof(unsigned long long), c->stream) == cudaSuccess &&
              cudaMemsetAsync(c->d_err, 0, sizeof(uint32_t), c->stream) == cudaSuccess;
   for (psk::StateSoA* s : {&c->st, &c->pend}) {
     set = set && cudaMemsetAsync(s->b, 0, I * 4, c->stream) == cudaSuccess &&
@@ -557,11 +553,11 @@ ps_status ps_schedule_window(ps_ctx* c, const ps_window* w, ps_decisions* out, p
   if (s != PS_OK) return s;
   record(c, kEvGreedy0);
   PS_TRY_CUDA(c, pskl::launch_greedy(c->d_slots, c->d_ovf, c->d_tdesc, c->I, wd, hit0, c->st, c->pend, c->model, c->d_delta,
-                                     c->delta_nbkt, c->d_dlog, c->d_dlog_n, c->d_assign, c->d_dpath, c->d_hchosen,
+                                     c->delta_nbkt, c->d_assign, c->d_dpath, c->d_hchosen,
                                      c->d_err, c->search, c->stream));
   record(c, kEvGreedy1);
   c->ev_used[2] = true;
-  PS_TRY_CUDA(c, pskl::launch_delta_clear(c->d_delta, c->d_dlog, c->d_dlog_n, c->max_blocks, c->num_sms, c->stream));
+  PS_TRY_CUDA(c, pskl::launch_delta_clear(c->d_delta, (uint64_t)c->delta_nbkt * psk::kDeltaSlots, c->stream));
   if (out) {
     PS_TRY_CUDA(c, deliver(c, out->assign, c->d_assign, wd.R, out->outputs_on_device));
     PS_TRY_CUDA(c, deliver(c, out->path, c->d_dpath, wd.R, out->outputs_on_device));

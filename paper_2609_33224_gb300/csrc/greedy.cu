@@ -14,6 +14,8 @@
 //      filter, TPOT/TTFT admission, D-C-Q key or LMetric fallback), reduced block-wide to the pick;
 //   3. the pick's state is updated (qr += 1, q += n, S += L) and its uncached blocks
 //      chain[h..nb) are inserted into the delta table for instance j.
+// The next request's row constants, hit row and the chain blocks at its hit positions are loaded
+// while the current request is decided, so a step starts with its inputs in registers.
 // Committed tables are never written here; the decisions and the updated state are a pending
 // window that ps_commit_window applies.  No step waits on another block: a single thread block with
 // __syncthreads barriers only.
@@ -21,14 +23,47 @@
 
 namespace {
 
+struct RowIn {
+  uint64_t o, nb;
+  uint32_t L;
+  float ttft_t, tpot_t;
+};
+
+__device__ __forceinline__ RowIn load_row(const psk::WindowDev& w, uint32_t r) {
+  RowIn x;
+  x.o = w.off[r];
+  x.nb = w.off[r + 1] - x.o;
+  x.L = w.L[r];
+  x.ttft_t = w.ttft_t[r];
+  x.tpot_t = w.tpot_t[r];
+  return x;
+}
+
+// Block-wide reductions without an extra barrier: after the per-warp partials are in shared
+// memory (and one __syncthreads), every warp reduces the (up to 32) partials with shuffles.
+__device__ __forceinline__ void cross_warp_min_any(const float* s_w, const int* s_a, int nw, float& wmin,
+                                                   bool& anyA) {
+  const int lane = threadIdx.x & 31;
+  const float v = lane < nw ? s_w[lane] : INFINITY;
+  const bool a = lane < nw ? (s_a[lane] != 0) : false;
+  wmin = psk::warp_fmin(v);
+  anyA = __any_sync(0xffffffffu, a);
+}
+
+__device__ __forceinline__ psk::ArgKey cross_warp_argmin(const psk::ArgKey* s_k, int nw) {
+  const int lane = threadIdx.x & 31;
+  psk::ArgKey k = lane < nw ? s_k[lane] : psk::ArgKey{psk::kNoKeyCi, ~0ull};
+  return psk::warp_argmin(k);
+}
+
 template <int IPT, bool SEARCH>
 __global__ void __launch_bounds__(1024, 1)
 greedy_kernel(const uint64_t* __restrict__ slots, const uint64_t* __restrict__ ovf,
               const psk::TableDesc* __restrict__ tdesc, uint32_t I,
               psk::WindowDev w, const uint32_t* __restrict__ hit0, psk::StateSoA committed,
               psk::StateSoA pending, psk::DevModel m, psk::DeltaSlot* delta, uint32_t delta_nbkt,
-              unsigned long long* dlog, unsigned long long* dlog_n, int32_t* __restrict__ assign,
-              uint8_t* __restrict__ path, uint32_t* __restrict__ hit_chosen, uint32_t* err) {
+              int32_t* __restrict__ assign, uint8_t* __restrict__ path, uint32_t* __restrict__ hit_chosen,
+              uint32_t* err) {
   extern __shared__ unsigned long long smem_raw[];
   int64_t* s_q = reinterpret_cast<int64_t*>(smem_raw);
   int64_t* s_S = s_q + I;
@@ -38,7 +73,9 @@ greedy_kernel(const uint64_t* __restrict__ slots, const uint64_t* __restrict__ o
   int32_t* s_Bmax = s_qr + I;
   uint32_t* s_h = reinterpret_cast<uint32_t*>(s_Bmax + I);
   uint32_t* s_walk = s_h + I;
-  uint8_t* s_touched = reinterpret_cast<uint8_t*>(s_walk + I);
+  uint32_t* s_end = s_walk + I;  // chain end of the last request assigned to the instance this window
+  psk::InstTerms* s_it = reinterpret_cast<psk::InstTerms*>(s_end + I);
+  uint8_t* s_touched = reinterpret_cast<uint8_t*>(s_it + I);
   __shared__ float s_red_w[32];
   __shared__ int s_red_a[32];
   __shared__ psk::ArgKey s_red_k[32];
@@ -57,36 +94,46 @@ greedy_kernel(const uint64_t* __restrict__ slots, const uint64_t* __restrict__ o
     s_S[i] = committed.S[i];
     s_M[i] = committed.M[i];
     s_Bmax[i] = committed.Bmax[i];
+    s_end[i] = 0;
     s_touched[i] = 0;
+    s_it[i] = psk::inst_terms(m, s_b[i], s_qr[i], s_q[i], s_Bmax[i]);
   }
   if (t == 0) s_nwalk = 0;
+  // Inputs of the next request: row constants, hit row, chain block at each hit position.
+  RowIn nx{};
   uint32_t hn[IPT];
+  uint64_t cn[IPT];
+  if (w.R > 0) nx = load_row(w, 0);
 #pragma unroll
   for (int k = 0; k < IPT; ++k) {
     const uint32_t i = t + k * NT;
     hn[k] = (i < I && w.R > 0) ? __ldg(hit0 + i) : 0u;
+    cn[k] = (i < I && hn[k] < nx.nb) ? w.hash[nx.o + hn[k]] : 0ull;
   }
   __syncthreads();
 
   for (uint32_t r = 0; r < w.R; ++r) {
-    const uint64_t o = w.off[r];
-    const uint64_t nb = w.off[r + 1] - o;
-    const psk::RowConst rc = psk::row_const(m, w.L[r], w.ttft_t[r], w.tpot_t[r]);
+    const RowIn cur = nx;
+    const uint64_t o = cur.o;
+    const uint64_t nb = cur.nb;
+    const psk::RowConst rc = psk::row_const(m, cur.L, cur.ttft_t, cur.tpot_t);
     uint32_t hc[IPT];
 #pragma unroll
     for (int k = 0; k < IPT; ++k) {
       const uint32_t i = t + k * NT;
       hc[k] = hn[k];
       if (i < I) {
-        if (s_touched[i] && hc[k] < nb &&
-            psk::delta_contains(delta, delta_nbkt, i, w.hash[o + hc[k]])) {
+        if (s_touched[i] && hc[k] < nb && psk::delta_contains(delta, delta_nbkt, i, cn[k])) {
           const uint32_t at = atomicAdd(&s_nwalk, 1u);
           s_walk[at] = i;
         }
         s_h[i] = hc[k];
       }
     }
-    if (r + 1 < w.R) {
+    // first half of the prefetch: row constants and hit row of request r + 1
+    const bool more = r + 1 < w.R;
+    if (more) {
+      nx = load_row(w, r + 1);
 #pragma unroll
       for (int k = 0; k < IPT; ++k) {
         const uint32_t i = t + k * NT;
@@ -106,8 +153,10 @@ greedy_kernel(const uint64_t* __restrict__ slots, const uint64_t* __restrict__ o
           return psk::delta_contains(delta, delta_nbkt, i, key) ||
                  (!SEARCH && psk::main_contains(slots, ovf, d, key));
         };
+        // Likely answer: where the last request assigned to i in this window ended (the same
+        // session's previous step usually ends exactly there).
         const uint64_t from = (uint64_t)s_h[i] + 1;
-        const uint64_t hnew = SEARCH ? psk::warp_first_miss_search(from, nb, cached)
+        const uint64_t hnew = SEARCH ? psk::warp_first_miss_search_hint(from, nb, s_end[i], cached)
                                      : psk::warp_first_miss_linear(from, nb, cached);
         if (lane == 0) s_h[i] = (uint32_t)hnew;
       }
@@ -126,7 +175,7 @@ greedy_kernel(const uint64_t* __restrict__ slots, const uint64_t* __restrict__ o
     for (int k = 0; k < IPT; ++k) {
       const uint32_t i = t + k * NT;
       if (i < I) {
-        ev[k] = psk::eval_pair(m, rc, hc[k], s_b[i], s_qr[i], s_q[i], s_S[i], s_M[i], s_Bmax[i]);
+        ev[k] = psk::eval_pair_terms(m, rc, hc[k], s_it[i], s_q[i], s_S[i], s_M[i]);
         if (ev[k].inA) {
           wmin = fminf(wmin, ev[k].W);
           anyA = true;
@@ -142,11 +191,14 @@ greedy_kernel(const uint64_t* __restrict__ slots, const uint64_t* __restrict__ o
       s_red_a[warp] = anyA ? 1 : 0;
     }
     __syncthreads();  // (C)
-    wmin = INFINITY;
-    anyA = false;
-    for (int x = 0; x < NW; ++x) {
-      wmin = fminf(wmin, s_red_w[x]);
-      anyA = anyA || (s_red_a[x] != 0);
+    cross_warp_min_any(s_red_w, s_red_a, NW, wmin, anyA);
+    // second half of the prefetch: chain blocks of request r + 1 at its hit positions
+    if (more) {
+#pragma unroll
+      for (int k = 0; k < IPT; ++k) {
+        const uint32_t i = t + k * NT;
+        if (i < I && hn[k] < nx.nb) cn[k] = w.hash[nx.o + hn[k]];
+      }
     }
     // Pass 2: admission classes and the lexicographic argmin.
     psk::ArgKey best{psk::kNoKeyCi, ~0ull};
@@ -164,9 +216,7 @@ greedy_kernel(const uint64_t* __restrict__ slots, const uint64_t* __restrict__ o
     best = psk::warp_argmin(best);
     if (lane == 0) s_red_k[warp] = best;
     __syncthreads();  // (D)
-    best = s_red_k[0];
-    for (int x = 1; x < NW; ++x)
-      if (psk::key_less(s_red_k[x], best)) best = s_red_k[x];
+    best = cross_warp_argmin(s_red_k, NW);
     const bool pick = anyA && best.ci != psk::kNoKeyCi;
     const uint32_t j = best.ci & 0x0FFFFFFFu;
     const uint32_t hj = pick ? s_h[j] : 0u;
@@ -178,13 +228,15 @@ greedy_kernel(const uint64_t* __restrict__ slots, const uint64_t* __restrict__ o
         s_qr[j] += 1;
         s_q[j] += (int64_t)rc.L - 16 * (int64_t)hj;
         s_S[j] += (int64_t)rc.L;
+        s_end[j] = (uint32_t)nb;
         s_touched[j] = 1;
+        s_it[j] = psk::inst_terms(m, s_b[j], s_qr[j], s_q[j], s_Bmax[j]);
       }
       s_nwalk = 0;
     }
     if (pick) {
       for (uint64_t k = (uint64_t)hj + t; k < nb; k += NT)
-        if (!psk::delta_insert(delta, delta_nbkt, j, w.hash[o + k], dlog, dlog_n)) atomicOr(err, psk::kErrDeltaFull);
+        if (!psk::delta_insert(delta, delta_nbkt, j, w.hash[o + k])) atomicOr(err, psk::kErrDeltaFull);
     }
     __syncthreads();  // (E) state, delta and walk counter ready for the next request
   }
@@ -198,52 +250,42 @@ greedy_kernel(const uint64_t* __restrict__ slots, const uint64_t* __restrict__ o
   }
 }
 
-__global__ void delta_clear_kernel(psk::DeltaSlot* delta, const unsigned long long* dlog,
-                                   const unsigned long long* dlog_n, uint64_t max_entries) {
-  uint64_t n = *dlog_n;
-  if (n > max_entries) n = max_entries;
-  for (uint64_t x = blockIdx.x * (uint64_t)blockDim.x + threadIdx.x; x < n; x += (uint64_t)gridDim.x * blockDim.x)
-    delta[dlog[x]].hash = psk::kEmpty;
+size_t greedy_smem(uint32_t I) {
+  return (size_t)I * (3 * sizeof(int64_t) + 3 * sizeof(int32_t) + 3 * sizeof(uint32_t) + sizeof(psk::InstTerms) + 1) + 16;
 }
 
-size_t greedy_smem(uint32_t I) {
-  return (size_t)I * (3 * sizeof(int64_t) + 3 * sizeof(int32_t) + 2 * sizeof(uint32_t) + 1) + 16;
+template <int IPT, bool SEARCH>
+cudaError_t greedy_launch(const uint64_t* slots, const uint64_t* ovf, const psk::TableDesc* tdesc, uint32_t I,
+                          const psk::WindowDev& w, const uint32_t* hit0, psk::StateSoA committed,
+                          psk::StateSoA pending, const psk::DevModel& m, psk::DeltaSlot* delta,
+                          uint32_t delta_nbkt, int32_t* assign, uint8_t* path, uint32_t* hit_chosen,
+                          uint32_t* err, uint32_t nt, cudaStream_t s) {
+  const size_t smem = greedy_smem(I);
+  cudaError_t e = cudaFuncSetAttribute(greedy_kernel<IPT, SEARCH>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)smem);
+  if (e != cudaSuccess) return e;
+  greedy_kernel<IPT, SEARCH><<<1, nt, smem, s>>>(slots, ovf, tdesc, I, w, hit0, committed, pending, m, delta,
+                                                 delta_nbkt, assign, path, hit_chosen, err);
+  return cudaGetLastError();
 }
 
 }  // namespace
 
 namespace pskl {
 
-template <int IPT, bool SEARCH>
-cudaError_t greedy_launch(const uint64_t* slots, const uint64_t* ovf, const psk::TableDesc* tdesc, uint32_t I,
-                          const psk::WindowDev& w,
-                          const uint32_t* hit0, psk::StateSoA committed, psk::StateSoA pending,
-                          const psk::DevModel& m, psk::DeltaSlot* delta, uint32_t delta_nbkt,
-                          unsigned long long* dlog, unsigned long long* dlog_n, int32_t* assign, uint8_t* path,
-                          uint32_t* hit_chosen, uint32_t* err, uint32_t nt, cudaStream_t s) {
-  const size_t smem = greedy_smem(I);
-  cudaError_t e = cudaFuncSetAttribute(greedy_kernel<IPT, SEARCH>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       (int)smem);
-  if (e != cudaSuccess) return e;
-  greedy_kernel<IPT, SEARCH><<<1, nt, smem, s>>>(slots, ovf, tdesc, I, w, hit0, committed, pending, m, delta,
-                                                 delta_nbkt, dlog, dlog_n, assign, path, hit_chosen, err);
-  return cudaGetLastError();
-}
-
 cudaError_t launch_greedy(const uint64_t* slots, const uint64_t* ovf, const psk::TableDesc* tdesc, uint32_t I,
                           const psk::WindowDev& w, const uint32_t* hit0, psk::StateSoA committed,
                           psk::StateSoA pending, const psk::DevModel& m, psk::DeltaSlot* delta,
-                          uint32_t delta_nbkt, unsigned long long* dlog, unsigned long long* dlog_n,
-                          int32_t* assign, uint8_t* path, uint32_t* hit_chosen, uint32_t* err,
-                          int search, cudaStream_t s) {
+                          uint32_t delta_nbkt, int32_t* assign, uint8_t* path, uint32_t* hit_chosen,
+                          uint32_t* err, int search, cudaStream_t s) {
   uint32_t nt = (I + 31) / 32 * 32;
   if (nt > 1024) nt = 1024;
   const uint32_t ipt = (I + nt - 1) / nt;
-#define PS_GREEDY(IPT)                                                                                  \
-  return search ? greedy_launch<IPT, true>(slots, ovf, tdesc, I, w, hit0, committed, pending, m, delta, delta_nbkt, \
-                                           dlog, dlog_n, assign, path, hit_chosen, err, nt, s)           \
-                : greedy_launch<IPT, false>(slots, ovf, tdesc, I, w, hit0, committed, pending, m, delta, delta_nbkt, \
-                                            dlog, dlog_n, assign, path, hit_chosen, err, nt, s)
+#define PS_GREEDY(IPT)                                                                                         \
+  return search ? greedy_launch<IPT, true>(slots, ovf, tdesc, I, w, hit0, committed, pending, m, delta,        \
+                                           delta_nbkt, assign, path, hit_chosen, err, nt, s)                   \
+                : greedy_launch<IPT, false>(slots, ovf, tdesc, I, w, hit0, committed, pending, m, delta,       \
+                                            delta_nbkt, assign, path, hit_chosen, err, nt, s)
   if (ipt <= 1) PS_GREEDY(1);
   if (ipt <= 2) PS_GREEDY(2);
   if (ipt <= 4) PS_GREEDY(4);
@@ -251,13 +293,9 @@ cudaError_t launch_greedy(const uint64_t* slots, const uint64_t* ovf, const psk:
   return cudaErrorInvalidValue;
 }
 
-cudaError_t launch_delta_clear(psk::DeltaSlot* delta, const unsigned long long* dlog,
-                               unsigned long long* dlog_n, uint64_t max_entries, int num_sms,
-                               cudaStream_t s) {
-  delta_clear_kernel<<<num_sms * 4, 256, 0, s>>>(delta, dlog, dlog_n, max_entries);
-  cudaError_t e = cudaGetLastError();
-  if (e != cudaSuccess) return e;
-  return cudaMemsetAsync(dlog_n, 0, sizeof(unsigned long long), s);
+// The delta table only holds one window's blocks: clear it whole after each window.
+cudaError_t launch_delta_clear(psk::DeltaSlot* delta, uint64_t nslots, cudaStream_t s) {
+  return cudaMemsetAsync(delta, 0, nslots * sizeof(psk::DeltaSlot), s);
 }
 
 }  // namespace pskl

@@ -28,7 +28,7 @@ struct DeviceScratch {
   uint32_t* base = nullptr;  // device address of g_noalloc_scratch on this device
   int num_sms = 0;
   int probe_grid_small = 0;  // probe grid for I < 64 (4-warp blocks)
-  int probe_grid_large = 0;  // probe grid for I >= 64 (16-warp blocks)
+  int probe_grid_large = 0;  // probe grid for I >= 64 (8-warp blocks)
 };
 
 std::mutex g_mu;

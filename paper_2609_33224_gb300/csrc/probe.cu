@@ -5,16 +5,19 @@
 // quantity the paper's scheduler reads from its prefix tree (Section 6) to estimate KVC reuse.
 //
 // One thread block per request (grid-stride over requests).  The request's chain is staged in
-// shared memory once (coalesced 8-byte loads) and reused by every instance's walk.  Each warp
-// handles one instance at a time with 32 probes per step, __ballot_sync collecting the misses and
-// __ffs finding the first: either a linear walk over 32 consecutive positions per step, or (for
-// prefix-closed caches) a 32-ary search over 32 evenly spaced positions.  Positions past the staging
-// capacity are read from global memory (L1/L2-resident: the same block re-reads them).
+// shared memory once (coalesced 8-byte loads) and reused by every instance's probe; positions past
+// the staging capacity are read from global memory (L1/L2-resident: the same block re-reads them).
+//   linear mode (any cache): each warp walks one instance at a time, 32 consecutive chain positions
+//     per step, __ballot_sync collecting the misses and __ffs finding the first.
+//   search mode (prefix-closed caches, where "block k cached" is monotone along the chain): each
+//     lane binary-searches its own instance.  All instances of a row share the chain length, so the
+//     32 lanes of a warp run the same number of steps in lock-step with 32 independent lookups in
+//     flight, and a pair costs about log2(nb) probes.
 #include "ps_internal.cuh"
 
 namespace {
 
-constexpr uint32_t kStageBlocks = 8192;  // 64 KB of staged chain per thread block
+constexpr uint32_t kStageBlocks = 4096;  // 32 KB of staged chain per thread block
 
 template <int WARPS, bool SEARCH>
 __global__ void __launch_bounds__(WARPS * 32)
@@ -31,15 +34,24 @@ probe_hits_kernel(const uint64_t* __restrict__ slots, const uint64_t* __restrict
     const uint64_t ns = nb < kStageBlocks ? nb : kStageBlocks;
     for (uint64_t k = threadIdx.x; k < ns; k += WARPS * 32) s_chain[k] = __ldg(hash + o + k);
     __syncthreads();
-    for (uint32_t i = warp; i < I; i += WARPS) {
-      const psk::TableDesc d = tdesc[i];
-      auto cached = [&](uint64_t k) {
-        const uint64_t key = k < ns ? s_chain[k] : __ldg(hash + o + k);
-        return psk::main_contains(slots, ovf, d, key);
-      };
-      const uint64_t h = SEARCH ? psk::warp_first_miss_search(0, nb, cached)
-                                : psk::warp_first_miss_linear(0, nb, cached);
-      if (lane == 0) hits[(uint64_t)r * I + i] = (uint32_t)h;
+    auto chain = [&](uint64_t k) { return k < ns ? s_chain[k] : __ldg(hash + o + k); };
+    if (SEARCH) {
+      for (uint32_t i = threadIdx.x; i < I; i += WARPS * 32) {
+        const psk::TableDesc d = tdesc[i];
+        uint64_t lo = 0, hi = nb;  // first miss in [lo, hi]
+        while (lo < hi) {
+          const uint64_t mid = (lo + hi) >> 1;
+          if (psk::main_contains(slots, ovf, d, chain(mid))) lo = mid + 1; else hi = mid;
+        }
+        hits[(uint64_t)r * I + i] = (uint32_t)lo;
+      }
+    } else {
+      for (uint32_t i = warp; i < I; i += WARPS) {
+        const psk::TableDesc d = tdesc[i];
+        auto cached = [&](uint64_t k) { return psk::main_contains(slots, ovf, d, chain(k)); };
+        const uint64_t h = psk::warp_first_miss_linear(0, nb, cached);
+        if (lane == 0) hits[(uint64_t)r * I + i] = (uint32_t)h;
+      }
     }
     __syncthreads();
   }
@@ -63,7 +75,7 @@ int max_grid(int num_sms) {
 namespace pskl {
 
 int probe_max_grid(uint32_t I, int num_sms) {
-  return I >= 64 ? max_grid<16>(num_sms) : max_grid<4>(num_sms);
+  return I >= 64 ? max_grid<8>(num_sms) : max_grid<4>(num_sms);
 }
 
 cudaError_t launch_probe(const uint64_t* slots, const uint64_t* ovf, const psk::TableDesc* tdesc, uint32_t I,
@@ -73,9 +85,9 @@ cudaError_t launch_probe(const uint64_t* slots, const uint64_t* ovf, const psk::
   const size_t smem = kStageBlocks * sizeof(uint64_t);
   if (I >= 64) {
     if (search)
-      probe_hits_kernel<16, true><<<g, 16 * 32, smem, s>>>(slots, ovf, tdesc, I, w.off, w.hash, w.R, hits);
+      probe_hits_kernel<8, true><<<g, 8 * 32, smem, s>>>(slots, ovf, tdesc, I, w.off, w.hash, w.R, hits);
     else
-      probe_hits_kernel<16, false><<<g, 16 * 32, smem, s>>>(slots, ovf, tdesc, I, w.off, w.hash, w.R, hits);
+      probe_hits_kernel<8, false><<<g, 8 * 32, smem, s>>>(slots, ovf, tdesc, I, w.off, w.hash, w.R, hits);
   } else {
     if (search)
       probe_hits_kernel<4, true><<<g, 4 * 32, smem, s>>>(slots, ovf, tdesc, I, w.off, w.hash, w.R, hits);

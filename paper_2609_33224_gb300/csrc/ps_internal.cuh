@@ -191,26 +191,21 @@ __device__ __forceinline__ bool delta_contains(const DeltaSlot* delta, uint32_t 
   return false;
 }
 
-// Insert (inst, key) into the delta table; appends the slot index to the clear log.  All concurrent
-// inserts come from one greedy step and target one instance.  Returns false if the table is full.
-__device__ __forceinline__ bool delta_insert(DeltaSlot* delta, uint32_t nbkt, uint32_t inst, uint64_t key,
-                                             unsigned long long* log, unsigned long long* log_n) {
+// Insert (inst, key) into the delta table.  All concurrent inserts come from one greedy step and
+// target one instance, and no lookup runs concurrently with them.  The key is CAS-ed into the first
+// slot of its home bucket that is free (the table is sized at twice the window's blocks, so the first
+// attempt nearly always succeeds); a duplicate (inst, key) entry is harmless for lookups.  Returns
+// false if the table is full.
+__device__ __forceinline__ bool delta_insert(DeltaSlot* delta, uint32_t nbkt, uint32_t inst, uint64_t key) {
   if (key == kEmpty || key == kTomb) return true;
   uint32_t b = delta_home(key, inst, nbkt);
   for (uint32_t p = 0; p < nbkt; ++p) {
     DeltaSlot* line = delta + (uint64_t)b * kDeltaSlots;
     for (int k = 0; k < kDeltaSlots; ++k) {
-      const unsigned long long h = __ldcg(&line[k].hash);
-      if (h == key && __ldcg(&line[k].inst) == inst) return true;
-      if (h == kEmpty) {
-        const unsigned long long old = atomicCAS(&line[k].hash, kEmpty, (unsigned long long)key);
-        if (old == kEmpty) {
-          line[k].inst = inst;
-          const unsigned long long at = atomicAdd(log_n, 1ull);
-          log[at] = (uint64_t)b * kDeltaSlots + k;
-          return true;
-        }
-        if (old == key && __ldcg(&line[k].inst) == inst) return true;
+      const unsigned long long old = atomicCAS(&line[k].hash, kEmpty, (unsigned long long)key);
+      if (old == kEmpty) {
+        line[k].inst = inst;
+        return true;
       }
     }
     b = (b + 1 == nbkt) ? 0u : b + 1;
@@ -242,9 +237,8 @@ __device__ __forceinline__ uint64_t warp_first_miss_linear(uint64_t lo, uint64_t
 // (p_31 = hi - 1) and keeps [p_{j-1} + 1, p_j] around the first miss j, so an interval of span s
 // shrinks to at most ceil(s / 32); spans <= 32 are finished by one linear step.
 template <class Pred>
-__device__ __forceinline__ uint64_t warp_first_miss_search(uint64_t lo, uint64_t nb, Pred present) {
+__device__ __forceinline__ uint64_t warp_search_range(uint64_t lo, uint64_t hi, Pred present) {
   const int lane = threadIdx.x & 31;
-  uint64_t hi = nb;
   for (;;) {
     const uint64_t span = hi - lo;
     if (span == 0) return lo;
@@ -262,6 +256,51 @@ __device__ __forceinline__ uint64_t warp_first_miss_search(uint64_t lo, uint64_t
     lo = lo + (j * span) / 32;
     hi = pj;
   }
+}
+
+template <class Pred>
+__device__ __forceinline__ uint64_t warp_first_miss_search(uint64_t lo, uint64_t nb, Pred present) {
+  return warp_search_range(lo, nb, present);
+}
+
+__device__ __forceinline__ uint64_t warp_min_u64(uint64_t x) {
+#pragma unroll
+  for (int s = 16; s > 0; s >>= 1) {
+    const uint64_t o = __shfl_xor_sync(0xffffffffu, x, s);
+    x = o < x ? o : x;
+  }
+  return x;
+}
+
+__device__ __forceinline__ uint64_t warp_max_u64(uint64_t x) {
+#pragma unroll
+  for (int s = 16; s > 0; s >>= 1) {
+    const uint64_t o = __shfl_xor_sync(0xffffffffu, x, s);
+    x = o > x ? o : x;
+  }
+  return x;
+}
+
+// The same search with a likely answer: the first step probes hint - 1 and hint next to 30 evenly
+// spaced positions.  Under monotone membership every probed position narrows the interval (a
+// present p raises lo to p + 1, an absent p lowers hi to p), so any positions keep it exact; when
+// the hint is the answer the first step ends the search.
+template <class Pred>
+__device__ __forceinline__ uint64_t warp_first_miss_search_hint(uint64_t lo, uint64_t nb, uint64_t hint,
+                                                                Pred present) {
+  const int lane = threadIdx.x & 31;
+  const uint64_t span = nb - lo;
+  if (span <= 32 || hint <= lo || hint > nb) return warp_search_range(lo, nb, present);
+  uint64_t p;
+  if (lane == 0) p = hint - 1;
+  else if (lane == 1) p = hint < nb ? hint : hint - 1;
+  else p = lo + ((uint64_t)(lane - 1) * span) / 31 - 1;
+  const bool pr = present(p);
+  const uint64_t new_hi = warp_min_u64(pr ? ~0ull : p);
+  const uint64_t last_present = warp_max_u64(pr ? p + 1 : 0ull);
+  const uint64_t hi = new_hi == ~0ull ? nb : new_hi;
+  const uint64_t lo2 = last_present > lo ? last_present : lo;
+  return warp_search_range(lo2, hi, present);
 }
 
 // ---------------------------------------------------------------------------- performance model --
@@ -342,6 +381,52 @@ __device__ __forceinline__ PairEval eval_pair(const DevModel& m, const RowConst&
   return e;
 }
 
+// Terms of eval_pair that depend only on the instance state (b, qr, q, B_max): they change only
+// when the instance is picked, so the greedy keeps them per instance.  Same rounded operations as
+// eval_pair, so results are bit-identical.
+struct InstTerms {
+  float dec0;   // b0 + b1 * B, B = b + qr + 1
+  float f;      // EMA factor of B's segment
+  float tq;     // a0 * qr + a1 * q (queueing part of TTFT)
+  int32_t Bp;   // b + qr + 1
+  int32_t okB;  // B <= B_max
+};
+
+__device__ __forceinline__ InstTerms inst_terms(const DevModel& m, int32_t b, int32_t qr, int64_t q, int32_t Bmax) {
+  InstTerms x;
+  const int64_t Bp = (int64_t)b + qr + 1;
+  x.dec0 = __fadd_rn(m.b0, __fmul_rn(m.b1, __ll2float_rn(Bp)));
+  x.f = ema_factor(m, Bp);
+  x.tq = __fadd_rn(__fmul_rn(m.a0, __int2float_rn(qr)), __fmul_rn(m.a1, __ll2float_rn(q)));
+  x.Bp = (int32_t)Bp;
+  x.okB = Bp <= (int64_t)Bmax;
+  return x;
+}
+
+// eval_pair with the instance terms precomputed.
+__device__ __forceinline__ PairEval eval_pair_terms(const DevModel& m, const RowConst& rc, uint32_t h,
+                                                    const InstTerms& it, int64_t q, int64_t S, int64_t M) {
+  PairEval e;
+  const int64_t c = 16 * (int64_t)h;
+  const int64_t n = (int64_t)rc.L - c;
+  const float tpf = t_pf(m, __ll2float_rn(n), __ll2float_rn(c));
+  e.n = n;
+  e.W = __fsub_rn(tpf, rc.t_cached);
+  const int64_t Sp = S + (int64_t)rc.L;
+  e.inA = it.okB && (Sp <= M);
+  float dec = __fadd_rn(it.dec0, __fmul_rn(m.b2, __ll2float_rn(Sp)));
+  dec = __fmul_rn(dec, it.f);
+  if (m.interference_mode == 0) {
+    e.tpot = __fadd_rn(dec, __fmul_rn(m.g_q, __ll2float_rn(q + n)));
+  } else {
+    const float den = m.lout > 1.0f ? m.lout : 1.0f;
+    const float interf = (it.Bp > 1) ? __fdiv_rn(tpf, den) : 0.0f;
+    e.tpot = __fadd_rn(dec, interf);
+  }
+  e.ttft = __fadd_rn(tpf, it.tq);
+  return e;
+}
+
 // Class of a capacity-eligible pair once W_min is known (Eq. 8, Alg. 1 TPOT filter + TTFT budget):
 // 0 in T, 1 in C \ T, 2 filtered by the recompute budget.
 __device__ __forceinline__ uint32_t pair_class(const DevModel& m, const RowConst& rc, const PairEval& e,
@@ -409,12 +494,9 @@ cudaError_t launch_score(const uint32_t* hits, psk::StateSoA st, uint32_t I, con
 cudaError_t launch_greedy(const uint64_t* slots, const uint64_t* ovf, const psk::TableDesc* tdesc, uint32_t I,
                           const psk::WindowDev& w, const uint32_t* hit0, psk::StateSoA committed,
                           psk::StateSoA pending, const psk::DevModel& m, psk::DeltaSlot* delta,
-                          uint32_t delta_nbkt, unsigned long long* dlog, unsigned long long* dlog_n,
-                          int32_t* assign, uint8_t* path, uint32_t* hit_chosen, uint32_t* err,
-                          int search, cudaStream_t s);
-cudaError_t launch_delta_clear(psk::DeltaSlot* delta, const unsigned long long* dlog,
-                               unsigned long long* dlog_n, uint64_t max_entries, int num_sms,
-                               cudaStream_t s);
+                          uint32_t delta_nbkt, int32_t* assign, uint8_t* path, uint32_t* hit_chosen,
+                          uint32_t* err, int search, cudaStream_t s);
+cudaError_t launch_delta_clear(psk::DeltaSlot* delta, uint64_t nslots, cudaStream_t s);
 cudaError_t launch_insert_chains(uint64_t* slots, uint64_t* ovf, const psk::TableDesc* tdesc, uint32_t I,
                                  unsigned long long* count, uint64_t nchains, const uint32_t* inst,
                                  const uint64_t* off, const uint64_t* hash, uint64_t total,
