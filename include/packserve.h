@@ -85,7 +85,7 @@ typedef struct {
 /* Context configuration (ps_create).
  *   device, cuda_stream   CUDA device ordinal and the cudaStream_t to launch on (NULL: the
  *                         library creates and owns a non-blocking stream).
- *   num_instances         1..4096.
+ *   num_instances         1..2048 (the greedy kernel keeps ~85 bytes of shared memory per instance).
  *   max_window_requests   largest R a window may have (1..131072).
  *   max_window_chain_blocks  largest total chain length (sum over requests) of a window.
  *   block_tokens          must be 16 (PS_BLOCK_TOKENS).

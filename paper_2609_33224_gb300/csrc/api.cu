@@ -143,6 +143,7 @@ ps_status device_errors(ps_ctx* c) {
   if (e & psk::kErrParentMissing)
     return fail(c, PS_ERR_INVALID, "a chain's parent_hash is not cached (PS_PROBE_SEARCH needs prefix-closed caches)");
   if (e & psk::kErrDeltaFull) return fail(c, PS_ERR_TABLE_FULL, "window delta table full");
+  if (e & psk::kErrTimeout) return fail(c, PS_ERR_TIMEOUT, "a bounded wait for a shared-memory bulk copy gave up");
   if (e & psk::kErrTableFull) return fail(c, PS_ERR_TABLE_FULL, "instance hash table full");
   return fail(c, PS_ERR_CUDA, "unknown device error");
 }
@@ -282,7 +283,7 @@ ps_status ps_create(const ps_config* cfg, ps_ctx** out) {
     ps_destroy(c);
     return s;
   };
-  if (cfg->num_instances < 1 || cfg->num_instances > 4096) return bail(PS_ERR_INVALID);
+  if (cfg->num_instances < 1 || cfg->num_instances > 2048) return bail(PS_ERR_INVALID);
   if (cfg->max_window_requests < 1 || cfg->max_window_requests > (1u << 17)) return bail(PS_ERR_INVALID);
   if (cfg->max_window_chain_blocks < 1 || cfg->max_window_chain_blocks > (1ull << 36)) return bail(PS_ERR_INVALID);
   if (cfg->block_tokens != PS_BLOCK_TOKENS || !cfg->cap_blocks) return bail(PS_ERR_INVALID);

@@ -38,6 +38,7 @@ enum : uint32_t {
   kErrWindowLayout = 8u,
   kErrBadInstance = 16u,
   kErrParentMissing = 32u,
+  kErrTimeout = 64u,
 };
 
 struct TableDesc {
@@ -49,7 +50,7 @@ struct TableDesc {
 
 struct DeltaSlot {
   unsigned long long hash;
-  unsigned int inst;
+  unsigned int inst1;  // instance id + 1; 0 while the slot is being claimed (never matches)
   unsigned int pad;
 };
 
@@ -183,7 +184,7 @@ __device__ __forceinline__ bool delta_contains(const DeltaSlot* delta, uint32_t 
 #pragma unroll
     for (int k = 0; k < kDeltaSlots; ++k) {
       const ulonglong2 v = __ldcg(line + k);
-      if (v.x == key && (uint32_t)v.y == inst) return true;
+      if (v.x == key && (uint32_t)v.y == inst + 1) return true;
       if (v.x == kEmpty) return false;
     }
     b = (b + 1 == nbkt) ? 0u : b + 1;
@@ -192,9 +193,11 @@ __device__ __forceinline__ bool delta_contains(const DeltaSlot* delta, uint32_t 
 }
 
 // Insert (inst, key) into the delta table.  All concurrent inserts come from one greedy step and
-// target one instance, and no lookup runs concurrently with them.  The key is CAS-ed into the first
-// slot of its home bucket that is free (the table is sized at twice the window's blocks, so the first
-// attempt nearly always succeeds); a duplicate (inst, key) entry is harmless for lookups.  Returns
+// target one instance.  The key is CAS-ed into the first free slot of its home bucket (the table is
+// sized at twice the window's blocks, so the first attempt nearly always succeeds), then the slot's
+// instance field is written.  A lookup that races with the insert sees either an empty slot or a
+// slot whose instance field is still 0, which matches no instance: it never reports a block that is
+// not in that instance's delta.  A duplicate (inst, key) entry is harmless for lookups.  Returns
 // false if the table is full.
 __device__ __forceinline__ bool delta_insert(DeltaSlot* delta, uint32_t nbkt, uint32_t inst, uint64_t key) {
   if (key == kEmpty || key == kTomb) return true;
@@ -204,7 +207,7 @@ __device__ __forceinline__ bool delta_insert(DeltaSlot* delta, uint32_t nbkt, ui
     for (int k = 0; k < kDeltaSlots; ++k) {
       const unsigned long long old = atomicCAS(&line[k].hash, kEmpty, (unsigned long long)key);
       if (old == kEmpty) {
-        line[k].inst = inst;
+        line[k].inst1 = inst + 1;
         return true;
       }
     }
@@ -281,8 +284,8 @@ __device__ __forceinline__ uint64_t warp_max_u64(uint64_t x) {
   return x;
 }
 
-// The same search with a likely answer: the first step probes hint - 1 and hint next to 30 evenly
-// spaced positions.  Under monotone membership every probed position narrows the interval (a
+// The same search with a likely answer (positions below lo are known present, lo itself need not
+// be): the first step probes hint - 1 and hint next to 30 evenly spaced positions.  Under monotone membership every probed position narrows the interval (a
 // present p raises lo to p + 1, an absent p lowers hi to p), so any positions keep it exact; when
 // the hint is the answer the first step ends the search.
 template <class Pred>
@@ -301,6 +304,52 @@ __device__ __forceinline__ uint64_t warp_first_miss_search_hint(uint64_t lo, uin
   const uint64_t hi = new_hi == ~0ull ? nb : new_hi;
   const uint64_t lo2 = last_present > lo ? last_present : lo;
   return warp_search_range(lo2, hi, present);
+}
+
+// --------------------------------------------------------------------- bulk copies (TMA, sm_90+) --
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return (uint32_t)__cvta_generic_to_shared(p);
+}
+
+__device__ __forceinline__ void mbar_init(uint64_t* mbar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(mbar)), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void fence_mbar_init() {
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+
+__device__ __forceinline__ void fence_proxy_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+// Arm the barrier for `bytes` of transaction count (one arrival) and start a global -> shared bulk
+// copy that completes against it.  dst, src 16-byte aligned, bytes a multiple of 16.
+__device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t bytes, uint64_t* mbar) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(mbar)), "r"(bytes)
+               : "memory");
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+          smem_u32(dst)),
+      "l"(src), "r"(bytes), "r"(smem_u32(mbar))
+      : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* mbar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}"
+      : "=r"(ok)
+      : "r"(smem_u32(mbar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+// Bounded wait for the barrier phase with the given parity; false after max_iter unsuccessful tries.
+__device__ __forceinline__ bool mbar_wait_bounded(uint64_t* mbar, uint32_t parity, uint32_t max_iter) {
+  for (uint32_t it = 0; it < max_iter; ++it)
+    if (mbar_try_wait(mbar, parity)) return true;
+  return false;
 }
 
 // ---------------------------------------------------------------------------- performance model --
