@@ -102,7 +102,12 @@ typedef struct {
  *                          cached" is monotone along a chain and a warp finds the first miss by a
  *                          32-ary search (32 evenly spaced probes per step, at most 4 steps for
  *                          65536 blocks).  ps_insert_* checks the closure: a chain whose parent_hash
- *                          is neither 0 nor cached after the call fails with PS_ERR_INVALID. */
+ *                          is neither 0 nor cached after the call fails with PS_ERR_INVALID.
+ *   track_lru             1: keep per-block (last_use, child count, parent) metadata so that
+ *                         ps_advance_window can evict leaf-first LRU; 0: no eviction.
+ *   max_active_requests   0: no request tracking.  > 0: each instance keeps up to this many queued
+ *                         and this many decoding requests for ps_advance_window (streaming windows);
+ *                         committed windows then need ps_window.out_tokens. */
 enum { PS_PROBE_LINEAR = 0, PS_PROBE_SEARCH = 1 };
 
 typedef struct {
@@ -116,6 +121,8 @@ typedef struct {
   float table_load_factor;
   ps_model model;
   int32_t probe_mode;
+  int32_t track_lru;
+  uint32_t max_active_requests;
 } ps_config;
 
 /* Scheduler-tracked state of one instance (Section 4 Metadata service; Section 5.5):
@@ -137,6 +144,8 @@ typedef struct {
  *   prompt_tokens  [R] input length L_r in tokens; its chain must have exactly L_r / 16 blocks
  *                  (full blocks only).  L_r < 2^30.
  *   ttft_target, tpot_target  [R] per-request SLO targets in ms.
+ *   out_tokens     [R] output length of each request (only read by ps_commit_window on a context
+ *                  with request tracking, to queue the admitted requests; may be NULL otherwise).
  *   inputs_on_device  0: all arrays are host memory, 1: all are device memory.
  * A window with device inputs is read in place; its buffers must stay unchanged until the window is
  * committed or discarded (ps_commit_window / the next ps_schedule_window). */
@@ -147,6 +156,7 @@ typedef struct {
   const uint32_t* prompt_tokens;
   const float* ttft_target;
   const float* tpot_target;
+  const uint32_t* out_tokens;
   int32_t inputs_on_device;
 } ps_window;
 
@@ -235,11 +245,48 @@ PS_API ps_status ps_schedule_window(ps_ctx* ctx, const ps_window* w, ps_decision
                              ps_scores* opt_scores);
 
 /* Commit the pending window: the pending state becomes the committed state and each admitted
- * request's uncached blocks are cached on its instance.  The window's buffers are read again here.
- * An instance may end above its cache capacity (ps_cached_blocks shows it); the table keeps working
- * as long as it has free slots.  Errors: PS_ERR_STATE (no pending window), PS_ERR_TABLE_FULL (no
- * free slot left; the state is still committed). */
+ * request's uncached blocks are cached on its instance.  With track_lru every block of an admitted
+ * request's chain on its instance (cached prefix and new blocks) gets last_use; with request
+ * tracking each admitted request joins its instance's FIFO queue (remaining prefill = its uncached
+ * tokens, output length from out_tokens).  The window's buffers are read again here.  An instance
+ * may end above its cache capacity (ps_cached_blocks shows it) until ps_advance_window evicts.
+ * Errors: PS_ERR_STATE (no pending window), PS_ERR_TABLE_FULL (no free slot left),
+ * PS_ERR_CAPACITY (an instance's request queue is full); the state is committed in every case. */
 PS_API ps_status ps_commit_window(ps_ctx* ctx, uint32_t last_use);
+
+/* ---- Streaming windows (between-window progress) ----------------------------------------------
+ * The paper's gateway tracks requests along their request and response paths (Section 4); the
+ * engine's progress between two windows is simulated with these rules (the serving engine's
+ * behaviour, which the paper leaves to the engine):
+ *   1. every decoding request emits k = max(1, floor(window_ms / ((b0 + b1 b) + b2 S))) tokens
+ *      (fp32, b and S at the window start); S grows by the tokens emitted; a request whose output
+ *      is exhausted leaves (b -= 1, S -= L + out);
+ *   2. each instance's queue drains prefill_tokens tokens in FIFO order; a request whose prefill
+ *      completes starts decoding (qr -= 1, b += 1, q falls by the tokens drained);
+ *   3. with evict = 1 (needs track_lru): while an instance holds more blocks than its capacity,
+ *      its leaf block (no cached child) with the smallest (last_use, hash) is evicted. */
+
+/* Requests in flight at the start of a stream (context created with max_active_requests > 0),
+ * host arrays of n entries: instance, state (0 queued, in FIFO order per instance; 1 decoding),
+ * prompt tokens L, output tokens out, rem (queued: remaining prefill tokens; decoding: remaining
+ * output tokens, 1..out).  Replaces all tracked requests; the committed state's b, qr, q_tokens
+ * and S_tokens are recomputed from them (S = queued L + decoding L + tokens already emitted).
+ * Errors: PS_ERR_INVALID (bad instance, state or rem), PS_ERR_CAPACITY (more than
+ * max_active_requests of one kind on an instance), PS_ERR_STATE (no request tracking). */
+PS_API ps_status ps_load_requests(ps_ctx* ctx, uint64_t n, const uint32_t* inst, const uint32_t* state,
+                                  const uint32_t* L, const uint32_t* out, const uint64_t* rem);
+
+typedef struct {
+  float window_ms;          /* engine time between two windows (ms), > 0 */
+  uint64_t prefill_tokens;  /* prefill tokens each instance processes in that time */
+  int32_t evict;            /* 1: evict to capacity (needs track_lru) */
+} ps_advance_params;
+
+/* Advance every instance by one window (rules above).  Errors: PS_ERR_STATE (a scheduled window
+ * is still pending, or no request tracking), PS_ERR_INVALID (params), PS_ERR_CAPACITY (a decoding
+ * list is full), PS_ERR_TABLE_FULL (an instance has more leaves than the eviction buffer holds,
+ * 4096; its eviction stops). */
+PS_API ps_status ps_advance_window(ps_ctx* ctx, const ps_advance_params* p);
 
 /* Device time in ms (CUDA events recorded on the context's stream around each kernel) of the last
  * ps_score_window / ps_schedule_window call and of the commit after it: ms[0] probe, ms[1] fused

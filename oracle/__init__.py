@@ -75,7 +75,12 @@ def _lib():
         lib.orc_hit.argtypes = [vp, u32, vp, u64]
         lib.orc_hit_pairs.argtypes = [vp, vp, vp, u64, vp, vp, vp]
         lib.orc_score_rows.argtypes = [vp] * 6 + [u64] + [vp] * 7
-        lib.orc_schedule.argtypes = [vp, u32] + [vp] * 8 + [u32]
+        lib.orc_schedule.argtypes = [vp, u32] + [vp] * 9 + [u32]
+        lib.orc_set_capacity.argtypes = [vp, vp]
+        lib.orc_load_requests.argtypes = [vp, u64, vp, vp, vp, vp, vp]
+        lib.orc_advance.argtypes = [vp, ctypes.c_float, u64, i32]
+        lib.orc_last_use.restype = u32
+        lib.orc_last_use.argtypes = [vp, u32, u64]
         _LIB = lib
     return _LIB
 
@@ -110,6 +115,7 @@ class Oracle:
 
     def __init__(self, I: int, model: dict, track_lru: bool = False):
         self.I = int(I)
+        self.track_lru = bool(track_lru)
         self._m = make_model(model)
         self._h = _lib().orc_create(self.I, ctypes.byref(self._m), 1 if track_lru else 0)
         if not self._h:
@@ -154,13 +160,14 @@ class Oracle:
         return {k: s[k].copy() for k in INST_DTYPE.names}
 
     def load(self, inst) -> "Oracle":
-        """Seed caches and state from a workload.Instances."""
+        """Seed caches and state from a workload.Instances (and capacities for eviction)."""
         counts = np.bincount(inst.chain_inst, weights=np.diff(inst.chain_off).astype(np.float64),
                              minlength=self.I)
         for i in range(self.I):
             _lib().orc_reserve(self._h, i, int(counts[i]))
         self.insert_chains(inst.chain_inst, inst.chain_off, inst.chain_hash, inst.chain_parent)
         self.set_state(inst.b, inst.qr, inst.q, inst.S, inst.M_KV, inst.B_max)
+        self.set_capacity(inst.cap_blocks)
         return self
 
     # -- scheduling --------------------------------------------------------------------------
@@ -191,14 +198,33 @@ class Oracle:
                               _p(out["best"]), _p(out["path"]))
         return out
 
-    def schedule(self, window, window_id: int = 0) -> dict:
+    def schedule(self, window, window_id: int = 0, streaming: bool = False) -> dict:
+        """Greedy window; with streaming=True admitted requests join their instance's queue."""
         R = window.R
         out = dict(assign=np.zeros(R, np.int32), path=np.zeros(R, np.uint8),
                    hit_chosen=np.zeros(R, np.uint32))
+        outs = _c(window.out_tokens, np.uint32) if streaming else None
         _lib().orc_schedule(self._h, R, _p(_c(window.chain_off, np.uint64)),
                             _p(_c(window.chain_hash, np.uint64)),
                             _p(_c(window.prompt_tokens, np.uint32)),
                             _p(_c(window.ttft_target, np.float32)),
-                            _p(_c(window.tpot_target, np.float32)), _p(out["assign"]),
+                            _p(_c(window.tpot_target, np.float32)), _p(outs), _p(out["assign"]),
                             _p(out["path"]), _p(out["hit_chosen"]), int(window_id))
         return out
+
+    # -- streaming windows ---------------------------------------------------------------------
+    def set_capacity(self, cap):
+        c = _c(cap, np.uint64)
+        _lib().orc_set_capacity(self._h, _p(c))
+
+    def load_requests(self, req: dict):
+        """req: inst, state (0 queued / 1 decoding), L, out, rem arrays (queued in FIFO order)."""
+        inst, state = _c(req["inst"], np.uint32), _c(req["state"], np.uint32)
+        L, out, rem = _c(req["L"], np.uint32), _c(req["out"], np.uint32), _c(req["rem"], np.uint64)
+        _lib().orc_load_requests(self._h, inst.shape[0], _p(inst), _p(state), _p(L), _p(out), _p(rem))
+
+    def advance(self, window_ms: float = 20.0, prefill_tokens: int = 1000, evict: bool = True):
+        _lib().orc_advance(self._h, float(window_ms), int(prefill_tokens), 1 if evict else 0)
+
+    def last_use(self, inst: int, block: int) -> int:
+        return int(_lib().orc_last_use(self._h, int(inst), int(block)))

@@ -29,6 +29,17 @@
 //  * Packing key D-C-Q (Section 5.5, Table 4): more decoding b, then more cached blocks h, then
 //    fewer queued requests qr, then the lowest instance id.  Fallback CacheAwareLB = LMetric
 //    (Section 6, Section 7.1 Baselines): min over C of (q + n)(b + qr + 1), lowest id on ties.
+//  * Streaming windows (the paper leaves engine progress to the serving engine; these are the
+//    simulation rules of the streaming workload).  Each instance keeps a FIFO queue of admitted
+//    requests (remaining uncached prefill tokens) and a set of decoding requests (remaining output
+//    tokens).  Advancing one window of window_ms: (1) every decoding request emits
+//    k = max(1, floor(window_ms / ((b0 + b1 b) + b2 S))) tokens (fp32, b and S at the window start),
+//    S grows by the tokens emitted, and a request whose output is exhausted leaves (b -= 1,
+//    S -= L + out); (2) the queue drains prefill_tokens tokens in FIFO order, a request whose prefill
+//    completes starts decoding (qr -= 1, b += 1); (3) while the cache holds more than cap blocks, the
+//    leaf block (no cached child) with the smallest (last_use, hash) is evicted.  Scheduling stamps
+//    last_use = window id on every block of an admitted request's chain (cached prefix and new
+//    blocks) on its instance.
 
 #include <cstdint>
 #include <cstring>
@@ -36,6 +47,8 @@
 #include <unordered_set>
 #include <unordered_map>
 #include <algorithm>
+#include <deque>
+#include <set>
 
 extern "C" {
 
@@ -65,9 +78,17 @@ struct Oracle {
   orc_model m;
   std::vector<std::unordered_set<uint64_t>> cache;
   std::vector<orc_inst> st;
-  // Leaf-first LRU bookkeeping (streaming windows only): per instance, block -> metadata.
+  // Leaf-first LRU bookkeeping (streaming windows only): per instance, block -> metadata, and the
+  // set of leaves ordered by (last_use, hash).
   bool track = false;
   std::vector<std::unordered_map<uint64_t, BlockMeta>> meta;
+  std::vector<std::set<std::pair<uint32_t, uint64_t>>> leaves;
+  // Requests in flight (streaming windows only).
+  struct Queued { uint32_t L, out; uint64_t rem; };
+  struct Decoding { uint32_t L, out, rem; };
+  std::vector<std::deque<Queued>> queue;
+  std::vector<std::vector<Decoding>> decoding;
+  std::vector<uint64_t> cap;
 };
 
 // Eq. 6 in the fixed order above.
@@ -195,19 +216,51 @@ void decide(const Oracle& o, const uint64_t* chain, uint64_t nb, uint32_t L, flo
   }
 }
 
+void touch_block(Oracle& o, uint32_t i, uint64_t h, uint32_t last_use) {
+  auto it = o.meta[i].find(h);
+  if (it == o.meta[i].end() || it->second.last_use >= last_use) return;
+  if (it->second.children == 0) {
+    o.leaves[i].erase({it->second.last_use, h});
+    o.leaves[i].insert({last_use, h});
+  }
+  it->second.last_use = last_use;
+}
+
 void insert_block(Oracle& o, uint32_t i, uint64_t h, uint64_t parent, uint32_t last_use) {
   bool added = o.cache[i].insert(h).second;
   if (!o.track) return;
   auto& mm = o.meta[i];
   if (added) {
     mm[h] = BlockMeta{parent, 0, last_use};
+    o.leaves[i].insert({last_use, h});
     if (parent) {
       auto it = mm.find(parent);
-      if (it != mm.end()) it->second.children += 1;
+      if (it != mm.end()) {
+        if (it->second.children == 0) o.leaves[i].erase({it->second.last_use, parent});
+        it->second.children += 1;
+      }
     }
   } else {
-    auto it = mm.find(h);
-    if (it != mm.end() && it->second.last_use < last_use) it->second.last_use = last_use;
+    touch_block(o, i, h, last_use);
+  }
+}
+
+// Leaf-first LRU eviction down to the instance's capacity.
+void evict_to_cap(Oracle& o, uint32_t i) {
+  while (o.cache[i].size() > o.cap[i] && !o.leaves[i].empty()) {
+    const auto victim = *o.leaves[i].begin();
+    o.leaves[i].erase(o.leaves[i].begin());
+    const uint64_t h = victim.second;
+    const uint64_t parent = o.meta[i][h].parent;
+    o.meta[i].erase(h);
+    o.cache[i].erase(h);
+    if (parent) {
+      auto it = o.meta[i].find(parent);
+      if (it != o.meta[i].end()) {
+        it->second.children -= 1;
+        if (it->second.children == 0) o.leaves[i].insert({it->second.last_use, parent});
+      }
+    }
   }
 }
 
@@ -223,7 +276,13 @@ void* orc_create(uint32_t I, const orc_model* m, int32_t track_lru) {
   o->cache.resize(I);
   o->st.assign(I, orc_inst{0, 0, 0, 0, 0, 0});
   o->track = track_lru != 0;
-  if (o->track) o->meta.resize(I);
+  if (o->track) {
+    o->meta.resize(I);
+    o->leaves.resize(I);
+  }
+  o->queue.resize(I);
+  o->decoding.resize(I);
+  o->cap.assign(I, UINT64_MAX);
   return o;
 }
 
@@ -310,8 +369,8 @@ void orc_score_rows(void* h, const uint64_t* off, const uint64_t* hash, const ui
 // instance and its uncached blocks chain[h..nb) to that instance's cache.  `hit_chosen` receives
 // the hit length on the chosen instance (0 on reject).  window_id stamps LRU use times.
 void orc_schedule(void* h, uint32_t R, const uint64_t* off, const uint64_t* hash, const uint32_t* L,
-                  const float* ttft_target, const float* tpot_target, int32_t* assign,
-                  uint8_t* path, uint32_t* hit_chosen, uint32_t window_id) {
+                  const float* ttft_target, const float* tpot_target, const uint32_t* out_tokens,
+                  int32_t* assign, uint8_t* path, uint32_t* hit_chosen, uint32_t window_id) {
   Oracle* o = static_cast<Oracle*>(h);
   Row row;
   for (uint32_t r = 0; r < R; ++r) {
@@ -328,14 +387,93 @@ void orc_schedule(void* h, uint32_t R, const uint64_t* off, const uint64_t* hash
     s.qr += 1;
     s.q += (int64_t)L[r] - 16 * (int64_t)hj;
     s.S += (int64_t)L[r];
-    if (o->track) {
-      for (uint64_t k = 0; k < hj; ++k) {
-        auto it = o->meta[j].find(ch[k]);
-        if (it != o->meta[j].end() && it->second.last_use < window_id) it->second.last_use = window_id;
+    if (o->track)
+      for (uint64_t k = 0; k < hj; ++k) touch_block(*o, j, ch[k], window_id);
+    for (uint64_t k = hj; k < nb; ++k) insert_block(*o, j, ch[k], k ? ch[k - 1] : 0, window_id);
+    if (out_tokens)
+      o->queue[j].push_back(Oracle::Queued{L[r], out_tokens[r], (uint64_t)((int64_t)L[r] - 16 * (int64_t)hj)});
+  }
+}
+
+// Cache capacities for eviction (blocks per instance).
+void orc_set_capacity(void* h, const uint64_t* cap) {
+  Oracle* o = static_cast<Oracle*>(h);
+  for (uint32_t i = 0; i < o->I; ++i) o->cap[i] = cap[i];
+}
+
+// Requests in flight at the start of a stream.  state 0: queued (FIFO in the given order, rem =
+// remaining prefill tokens), 1: decoding (rem = remaining output tokens).  The instance state's
+// b, qr, q and S are recomputed from them (S = sum of queued L + decoding L + emitted tokens).
+void orc_load_requests(void* h, uint64_t n, const uint32_t* inst, const uint32_t* state, const uint32_t* L,
+                       const uint32_t* out, const uint64_t* rem) {
+  Oracle* o = static_cast<Oracle*>(h);
+  for (uint32_t i = 0; i < o->I; ++i) {
+    o->queue[i].clear();
+    o->decoding[i].clear();
+    o->st[i].b = 0; o->st[i].qr = 0; o->st[i].q = 0; o->st[i].S = 0;
+  }
+  for (uint64_t k = 0; k < n; ++k) {
+    orc_inst& s = o->st[inst[k]];
+    if (state[k] == 0) {
+      o->queue[inst[k]].push_back(Oracle::Queued{L[k], out[k], rem[k]});
+      s.qr += 1;
+      s.q += (int64_t)rem[k];
+      s.S += (int64_t)L[k];
+    } else {
+      o->decoding[inst[k]].push_back(Oracle::Decoding{L[k], out[k], (uint32_t)rem[k]});
+      s.b += 1;
+      s.S += (int64_t)L[k] + (int64_t)(out[k] - (uint32_t)rem[k]);
+    }
+  }
+}
+
+// One window of engine progress, then eviction to capacity (see the header).
+void orc_advance(void* h, float window_ms, uint64_t prefill_tokens, int32_t evict) {
+  Oracle* o = static_cast<Oracle*>(h);
+  const orc_model& m = o->m;
+  for (uint32_t i = 0; i < o->I; ++i) {
+    orc_inst& s = o->st[i];
+    float t_iter = m.b0 + m.b1 * (float)s.b;
+    t_iter = t_iter + m.b2 * (float)s.S;
+    const float per = window_ms / t_iter;
+    int64_t k = (int64_t)per;  // per > 0: truncation is floor
+    if (k < 1) k = 1;
+    std::vector<Oracle::Decoding> keep;
+    for (auto& d : o->decoding[i]) {
+      const uint32_t e = (uint64_t)d.rem < (uint64_t)k ? d.rem : (uint32_t)k;
+      d.rem -= e;
+      s.S += e;
+      if (d.rem == 0) {
+        s.b -= 1;
+        s.S -= (int64_t)d.L + (int64_t)d.out;
+      } else {
+        keep.push_back(d);
       }
     }
-    for (uint64_t k = hj; k < nb; ++k) insert_block(*o, j, ch[k], k ? ch[k - 1] : 0, window_id);
+    o->decoding[i].swap(keep);
+    uint64_t budget = prefill_tokens;
+    while (budget > 0 && !o->queue[i].empty()) {
+      Oracle::Queued& qd = o->queue[i].front();
+      const uint64_t d = qd.rem < budget ? qd.rem : budget;
+      qd.rem -= d;
+      s.q -= (int64_t)d;
+      budget -= d;
+      if (qd.rem == 0) {
+        o->decoding[i].push_back(Oracle::Decoding{qd.L, qd.out, qd.out});
+        o->queue[i].pop_front();
+        s.qr -= 1;
+        s.b += 1;
+      }
+    }
+    if (evict && o->track) evict_to_cap(*o, i);
   }
+}
+
+uint32_t orc_last_use(void* h, uint32_t inst, uint64_t block) {
+  Oracle* o = static_cast<Oracle*>(h);
+  if (!o->track) return 0;
+  auto it = o->meta[inst].find(block);
+  return it == o->meta[inst].end() ? 0 : it->second.last_use;
 }
 
 }  // extern "C"

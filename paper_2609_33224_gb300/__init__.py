@@ -25,7 +25,7 @@ STATUS_NAMES = {0: "PS_OK", 1: "PS_ERR_INVALID", 2: "PS_ERR_CUDA", 3: "PS_ERR_OO
 ABI_FUNCTIONS = ("ps_create", "ps_load_instances", "ps_get_instances", "ps_get_pending_instances",
                  "ps_insert_blocks", "ps_insert_chains", "ps_cached_blocks", "ps_score_window",
                  "ps_schedule_window", "ps_commit_window", "ps_last_timings", "ps_last_error",
-                 "ps_destroy", "ps_score_window_noalloc")
+                 "ps_destroy", "ps_score_window_noalloc", "ps_load_requests", "ps_advance_window")
 
 
 class PsModel(ctypes.Structure):
@@ -40,7 +40,8 @@ class PsConfig(ctypes.Structure):
                 ("num_instances", ctypes.c_uint32), ("max_window_requests", ctypes.c_uint32),
                 ("max_window_chain_blocks", ctypes.c_uint64), ("block_tokens", ctypes.c_uint32),
                 ("cap_blocks", ctypes.c_void_p), ("table_load_factor", ctypes.c_float),
-                ("model", PsModel), ("probe_mode", ctypes.c_int32)]
+                ("model", PsModel), ("probe_mode", ctypes.c_int32), ("track_lru", ctypes.c_int32),
+                ("max_active_requests", ctypes.c_uint32)]
 
 PS_PROBE_LINEAR, PS_PROBE_SEARCH = 0, 1
 
@@ -53,7 +54,8 @@ class PsInstanceState(ctypes.Structure):
 class PsWindow(ctypes.Structure):
     _fields_ = [("R", ctypes.c_uint32), ("chain_off", ctypes.c_void_p), ("chain_hash", ctypes.c_void_p),
                 ("prompt_tokens", ctypes.c_void_p), ("ttft_target", ctypes.c_void_p),
-                ("tpot_target", ctypes.c_void_p), ("inputs_on_device", ctypes.c_int32)]
+                ("tpot_target", ctypes.c_void_p), ("out_tokens", ctypes.c_void_p),
+                ("inputs_on_device", ctypes.c_int32)]
 
 
 class PsScores(ctypes.Structure):
@@ -65,6 +67,10 @@ class PsScores(ctypes.Structure):
 class PsDecisions(ctypes.Structure):
     _fields_ = [("assign", ctypes.c_void_p), ("path", ctypes.c_void_p), ("hit_chosen", ctypes.c_void_p),
                 ("outputs_on_device", ctypes.c_int32)]
+
+
+class PsAdvanceParams(ctypes.Structure):
+    _fields_ = [("window_ms", ctypes.c_float), ("prefill_tokens", ctypes.c_uint64), ("evict", ctypes.c_int32)]
 
 
 class PsTableDesc(ctypes.Structure):
@@ -107,6 +113,8 @@ def lib() -> ctypes.CDLL:
                                    ctypes.POINTER(PsScores)],
             "ps_commit_window": [vp, u32],
             "ps_last_timings": [vp, vp, u32],
+            "ps_load_requests": [vp, u64, vp, vp, vp, vp, vp],
+            "ps_advance_window": [vp, ctypes.POINTER(PsAdvanceParams)],
             "ps_score_window_noalloc": [vp, vp, vp, u32, ctypes.POINTER(PsStateArrays), ctypes.POINTER(PsWindow),
                                         ctypes.POINTER(PsModel), i32, ctypes.POINTER(PsScores), vp],
         }
@@ -171,7 +179,8 @@ class Scheduler:
 
     def __init__(self, num_instances: int, cap_blocks, max_window_requests: int,
                  max_window_chain_blocks: int, model: dict, table_load_factor: float = 0.5,
-                 device: int = 0, stream=None, probe_mode: int = PS_PROBE_SEARCH):
+                 device: int = 0, stream=None, probe_mode: int = PS_PROBE_SEARCH, track_lru: bool = False,
+                 max_active_requests: int = 0):
         self.I = int(num_instances)
         self._cap = np.ascontiguousarray(cap_blocks, dtype=np.uint64)
         cfg = PsConfig()
@@ -185,6 +194,8 @@ class Scheduler:
         cfg.table_load_factor = float(table_load_factor)
         cfg.model = make_model(model)
         cfg.probe_mode = int(probe_mode)
+        cfg.track_lru = 1 if track_lru else 0
+        cfg.max_active_requests = int(max_active_requests)
         self.probe_mode = int(probe_mode)
         h = ctypes.c_void_p()
         s = lib().ps_create(ctypes.byref(cfg), ctypes.byref(h))
@@ -262,6 +273,17 @@ class Scheduler:
         self._check(lib().ps_cached_blocks(self._h, out.ctypes.data, self.I))
         return out
 
+    def load_requests(self, req: dict):
+        """Requests in flight (streaming): inst, state (0 queued FIFO / 1 decoding), L, out, rem."""
+        a = [np.ascontiguousarray(req[k], dtype=d) for k, d in
+             (("inst", np.uint32), ("state", np.uint32), ("L", np.uint32), ("out", np.uint32), ("rem", np.uint64))]
+        n = a[0].shape[0]
+        self._check(lib().ps_load_requests(self._h, n, *[x.ctypes.data if n else None for x in a]))
+
+    def advance_window(self, window_ms: float = 20.0, prefill_tokens: int = 1000, evict: bool = True):
+        p = PsAdvanceParams(float(window_ms), int(prefill_tokens), 1 if evict else 0)
+        self._check(lib().ps_advance_window(self._h, ctypes.byref(p)))
+
     def timings(self) -> dict:
         ms = np.zeros(4, np.float32)
         self._check(lib().ps_last_timings(self._h, ms.ctypes.data, 4))
@@ -274,14 +296,14 @@ class Scheduler:
         w = PsWindow()
         arrs = [(window.chain_off, np.uint64), (window.chain_hash, np.uint64),
                 (window.prompt_tokens, np.uint32), (window.ttft_target, np.float32),
-                (window.tpot_target, np.float32)]
+                (window.tpot_target, np.float32), (getattr(window, "out_tokens", None), np.uint32)]
         ptrs = [_ptr(a, d) for a, d in arrs]
         dev = {p[1] for p in ptrs if p[1] is not None}
         if len(dev) > 1:
             raise ValueError("window arrays must all be host or all be device")
         n_off = window.chain_off.numel() if _is_torch(window.chain_off) else window.chain_off.shape[0]
         w.R = int(n_off) - 1
-        w.chain_off, w.chain_hash, w.prompt_tokens, w.ttft_target, w.tpot_target = (p[0] for p in ptrs)
+        w.chain_off, w.chain_hash, w.prompt_tokens, w.ttft_target, w.tpot_target, w.out_tokens = (p[0] for p in ptrs)
         w.inputs_on_device = 1 if dev == {True} else 0
         return w
 
@@ -340,13 +362,14 @@ class Scheduler:
 
 def scheduler_for(workload, max_window_chain_blocks: int | None = None, device: int = 0, stream=None,
                   model: dict | None = None, load: bool = True,
-                  probe_mode: int = PS_PROBE_SEARCH) -> Scheduler:
+                  probe_mode: int = PS_PROBE_SEARCH, track_lru: bool = False,
+                  max_active_requests: int = 0, max_window_requests: int | None = None) -> Scheduler:
     """A context sized for a workload.Workload, optionally seeded with its instances."""
     win, ins = workload.window, workload.instances
     mb = max_window_chain_blocks or max(1, int(win.chain_off[-1]))
-    s = Scheduler(ins.I, ins.cap_blocks, max(1, win.R), mb, model or workload.model,
+    s = Scheduler(ins.I, ins.cap_blocks, max(1, max_window_requests or win.R), mb, model or workload.model,
                   table_load_factor=workload.table_load_factor, device=device, stream=stream,
-                  probe_mode=probe_mode)
+                  probe_mode=probe_mode, track_lru=track_lru, max_active_requests=max_active_requests)
     if load:
         s.load_workload_instances(ins)
     return s

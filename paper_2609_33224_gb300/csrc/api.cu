@@ -69,6 +69,13 @@ struct ps_ctx {
   bool ev_used[kNumEv / 2] = {};
   bool pending = false;
   psk::WindowDev pend_win{};
+  const uint32_t* pend_out = nullptr;
+  // streaming: per-block LRU metadata, request store, capacities on the device
+  bool lru = false;
+  psk::LruMeta meta{nullptr, nullptr, nullptr};
+  psk::ReqStore rq{};
+  uint64_t* d_cap = nullptr;
+  uint32_t* d_outtok = nullptr;
   std::vector<void*> allocs;
   std::string err;
 };
@@ -143,7 +150,11 @@ ps_status device_errors(ps_ctx* c) {
   if (e & psk::kErrParentMissing)
     return fail(c, PS_ERR_INVALID, "a chain's parent_hash is not cached (PS_PROBE_SEARCH needs prefix-closed caches)");
   if (e & psk::kErrDeltaFull) return fail(c, PS_ERR_TABLE_FULL, "window delta table full");
-  if (e & psk::kErrTimeout) return fail(c, PS_ERR_TIMEOUT, "a bounded wait for a shared-memory bulk copy gave up");
+  if (e & psk::kErrTimeout) return fail(c, PS_ERR_TIMEOUT, "a bounded device-side wait gave up");
+  if (e & psk::kErrRequestsFull)
+    return fail(c, PS_ERR_CAPACITY, "an instance has more requests in flight than max_active_requests");
+  if (e & psk::kErrLeavesFull)
+    return fail(c, PS_ERR_TABLE_FULL, "an instance has more leaf blocks than the eviction buffer (4096)");
   if (e & psk::kErrTableFull) return fail(c, PS_ERR_TABLE_FULL, "instance hash table full");
   return fail(c, PS_ERR_CUDA, "unknown device error");
 }
@@ -180,7 +191,9 @@ ps_status stage_window(ps_ctx* c, const ps_window* w, psk::WindowDev* out) {
   if (!w->chain_off || (w->R > 0 && (!w->prompt_tokens || !w->ttft_target || !w->tpot_target)))
     return fail(c, PS_ERR_INVALID, "window array is NULL");
   out->R = w->R;
+  c->pend_out = nullptr;
   if (w->inputs_on_device) {
+    c->pend_out = w->out_tokens;
     out->off = w->chain_off;
     out->hash = w->chain_hash;
     out->L = w->prompt_tokens;
@@ -213,6 +226,11 @@ ps_status stage_window(ps_ctx* c, const ps_window* w, psk::WindowDev* out) {
     PS_TRY_CUDA(c, cudaMemcpyAsync(c->d_L, w->prompt_tokens, w->R * sizeof(uint32_t), cudaMemcpyHostToDevice, c->stream));
     PS_TRY_CUDA(c, cudaMemcpyAsync(c->d_ttft, w->ttft_target, w->R * sizeof(float), cudaMemcpyHostToDevice, c->stream));
     PS_TRY_CUDA(c, cudaMemcpyAsync(c->d_tpot, w->tpot_target, w->R * sizeof(float), cudaMemcpyHostToDevice, c->stream));
+    if (w->out_tokens) {
+      PS_TRY_CUDA(c, cudaMemcpyAsync(c->d_outtok, w->out_tokens, w->R * sizeof(uint32_t), cudaMemcpyHostToDevice,
+                                     c->stream));
+      c->pend_out = c->d_outtok;
+    }
   }
   out->off = c->d_off;
   out->hash = c->d_hash;
@@ -291,6 +309,10 @@ ps_status ps_create(const ps_config* cfg, ps_ctx** out) {
   if (check_model(c, cfg->model) != PS_OK) return bail(PS_ERR_INVALID);
   if (cfg->probe_mode != PS_PROBE_LINEAR && cfg->probe_mode != PS_PROBE_SEARCH) return bail(PS_ERR_INVALID);
   c->search = cfg->probe_mode == PS_PROBE_SEARCH ? 1 : 0;
+  if (cfg->track_lru != 0 && cfg->track_lru != 1) return bail(PS_ERR_INVALID);
+  if (cfg->max_active_requests > (1u << 16)) return bail(PS_ERR_INVALID);
+  c->lru = cfg->track_lru == 1;
+  c->rq.M = cfg->max_active_requests;
   c->device = cfg->device;
   c->I = cfg->num_instances;
   c->Rmax = cfg->max_window_requests;
@@ -345,7 +367,20 @@ ps_status ps_create(const ps_config* cfg, ps_ctx** out) {
        dalloc(c, &c->d_ttft_o, RI) == cudaSuccess && dalloc(c, &c->d_cls, RI) == cudaSuccess &&
        dalloc(c, &c->d_best, c->Rmax) == cudaSuccess && dalloc(c, &c->d_path, c->Rmax) == cudaSuccess &&
        dalloc(c, &c->d_assign, c->Rmax) == cudaSuccess && dalloc(c, &c->d_dpath, c->Rmax) == cudaSuccess &&
-       dalloc(c, &c->d_hchosen, c->Rmax) == cudaSuccess && dalloc(c, &c->d_err, 1) == cudaSuccess;
+       dalloc(c, &c->d_hchosen, c->Rmax) == cudaSuccess && dalloc(c, &c->d_err, 1) == cudaSuccess &&
+       dalloc(c, &c->d_cap, I) == cudaSuccess && dalloc(c, &c->d_outtok, c->Rmax) == cudaSuccess;
+  if (ok && c->lru)
+    ok = dalloc(c, &c->meta.last_use, c->total_slots) == cudaSuccess &&
+         dalloc(c, &c->meta.children, c->total_slots) == cudaSuccess &&
+         dalloc(c, &c->meta.parent, c->total_slots) == cudaSuccess;
+  if (ok && c->rq.M) {
+    const size_t IM = I * (size_t)c->rq.M;
+    ok = dalloc(c, &c->rq.q_head, I) == cudaSuccess && dalloc(c, &c->rq.q_len, I) == cudaSuccess &&
+         dalloc(c, &c->rq.q_L, IM) == cudaSuccess && dalloc(c, &c->rq.q_out, IM) == cudaSuccess &&
+         dalloc(c, &c->rq.q_rem, IM) == cudaSuccess && dalloc(c, &c->rq.d_len, I) == cudaSuccess &&
+         dalloc(c, &c->rq.d_L, IM) == cudaSuccess && dalloc(c, &c->rq.d_out, IM) == cudaSuccess &&
+         dalloc(c, &c->rq.d_rem, IM) == cudaSuccess;
+  }
   if (!ok) {
     cudaGetLastError();
     return bail(PS_ERR_OOM);
@@ -370,6 +405,16 @@ ps_status ps_create(const ps_config* cfg, ps_ctx** out) {
           cudaMemsetAsync(s->M, 0, I * 8, c->stream) == cudaSuccess &&
           cudaMemsetAsync(s->Bmax, 0, I * 4, c->stream) == cudaSuccess;
   }
+  set = set && cudaMemcpyAsync(c->d_cap, c->cap.data(), I * sizeof(uint64_t), cudaMemcpyHostToDevice, c->stream) ==
+                   cudaSuccess;
+  if (c->lru)
+    set = set && cudaMemsetAsync(c->meta.last_use, 0, c->total_slots * 4, c->stream) == cudaSuccess &&
+          cudaMemsetAsync(c->meta.children, 0, c->total_slots * 4, c->stream) == cudaSuccess &&
+          cudaMemsetAsync(c->meta.parent, 0, c->total_slots * 8, c->stream) == cudaSuccess;
+  if (c->rq.M)
+    set = set && cudaMemsetAsync(c->rq.q_head, 0, I * 4, c->stream) == cudaSuccess &&
+          cudaMemsetAsync(c->rq.q_len, 0, I * 4, c->stream) == cudaSuccess &&
+          cudaMemsetAsync(c->rq.d_len, 0, I * 4, c->stream) == cudaSuccess;
   if (!set || cudaStreamSynchronize(c->stream) != cudaSuccess) return bail(PS_ERR_CUDA);
   c->probe_grid = pskl::probe_max_grid(c->I, c->num_sms);
   if (cudaGetLastError() != cudaSuccess) return bail(PS_ERR_CUDA);
@@ -452,8 +497,6 @@ ps_status ps_get_pending_instances(ps_ctx* c, ps_instance_state* out, uint32_t n
 
 ps_status ps_insert_chains(ps_ctx* c, uint64_t nchains, const uint32_t* inst, const uint64_t* off,
                            const uint64_t* hash, const uint64_t* parent, uint32_t last_use, int32_t on_device) {
-  (void)parent;
-  (void)last_use;
   if (!c) return PS_ERR_INVALID;
   if (nchains == 0) return PS_OK;
   if (!inst || !off || !parent || (on_device != 0 && on_device != 1))
@@ -495,7 +538,8 @@ ps_status ps_insert_chains(ps_ctx* c, uint64_t nchains, const uint32_t* inst, co
     PS_TRY_CUDA(c, cudaMemcpy(&total, off + nchains, 8, cudaMemcpyDeviceToHost));
   }
   cudaError_t e = pskl::launch_insert_chains(c->d_slots, c->d_ovf, c->d_tdesc, c->I, c->d_count, nchains, d_inst, d_off,
-                                             d_hash, total, c->d_err, c->num_sms, c->stream);
+                                             d_hash, d_parent, total, c->meta, last_use, c->d_err, c->num_sms,
+                                             c->stream);
   if (e == cudaSuccess && c->search)
     e = pskl::launch_check_parents(c->d_slots, c->d_ovf, c->d_tdesc, c->I, nchains, d_inst, d_parent, c->d_err, c->num_sms,
                                    c->stream);
@@ -572,13 +616,15 @@ ps_status ps_schedule_window(ps_ctx* c, const ps_window* w, ps_decisions* out, p
 }
 
 ps_status ps_commit_window(ps_ctx* c, uint32_t last_use) {
-  (void)last_use;
   if (!c) return PS_ERR_INVALID;
   if (!c->pending) return fail(c, PS_ERR_STATE, "no pending window");
+  if (c->rq.M && c->pend_win.R && !c->pend_out)
+    return fail(c, PS_ERR_INVALID, "request tracking needs the window's out_tokens");
   DeviceGuard g(c->device);
   record(c, kEvCommit0);
   PS_TRY_CUDA(c, pskl::launch_commit(c->d_slots, c->d_ovf, c->d_tdesc, c->I, c->d_count, c->pend_win, c->d_assign,
-                                     c->d_hchosen, c->d_err, c->num_sms, c->stream));
+                                     c->d_hchosen, c->meta, last_use, c->rq, c->pend_out, c->d_err, c->num_sms,
+                                     c->stream));
   const size_t I = c->I;
   PS_TRY_CUDA(c, cudaMemcpyAsync(c->st.b, c->pend.b, I * 4, cudaMemcpyDeviceToDevice, c->stream));
   PS_TRY_CUDA(c, cudaMemcpyAsync(c->st.qr, c->pend.qr, I * 4, cudaMemcpyDeviceToDevice, c->stream));
@@ -589,6 +635,69 @@ ps_status ps_commit_window(ps_ctx* c, uint32_t last_use) {
   record(c, kEvCommit1);
   c->ev_used[3] = true;
   c->pending = false;
+  return finish(c);
+}
+
+ps_status ps_load_requests(ps_ctx* c, uint64_t n, const uint32_t* inst, const uint32_t* state, const uint32_t* L,
+                           const uint32_t* out, const uint64_t* rem) {
+  if (!c) return PS_ERR_INVALID;
+  if (!c->rq.M) return fail(c, PS_ERR_STATE, "context has no request tracking (max_active_requests = 0)");
+  if (n && (!inst || !state || !L || !out || !rem)) return fail(c, PS_ERR_INVALID, "request array is NULL");
+  const uint32_t I = c->I, M = c->rq.M;
+  const size_t IM = (size_t)I * M;
+  std::vector<uint32_t> qlen(I, 0), dlen(I, 0), qL(IM), qo(IM), dL(IM), dO(IM), dR(IM);
+  std::vector<uint64_t> qR(IM);
+  std::vector<int32_t> b(I, 0), qr(I, 0);
+  std::vector<int64_t> q(I, 0), S(I, 0);
+  for (uint64_t k = 0; k < n; ++k) {
+    const uint32_t i = inst[k];
+    if (i >= I || state[k] > 1) return fail(c, PS_ERR_INVALID, "request " + std::to_string(k) + ": bad instance or state");
+    if (state[k] == 0) {
+      if (qlen[i] >= M) return fail(c, PS_ERR_CAPACITY, "too many queued requests on instance " + std::to_string(i));
+      const size_t at = (size_t)i * M + qlen[i]++;
+      qL[at] = L[k]; qo[at] = out[k]; qR[at] = rem[k];
+      qr[i] += 1; q[i] += (int64_t)rem[k]; S[i] += L[k];
+    } else {
+      if (rem[k] < 1 || rem[k] > out[k]) return fail(c, PS_ERR_INVALID, "decoding request needs 1 <= rem <= out");
+      if (dlen[i] >= M) return fail(c, PS_ERR_CAPACITY, "too many decoding requests on instance " + std::to_string(i));
+      const size_t at = (size_t)i * M + dlen[i]++;
+      dL[at] = L[k]; dO[at] = out[k]; dR[at] = (uint32_t)rem[k];
+      b[i] += 1; S[i] += (int64_t)L[k] + (int64_t)(out[k] - (uint32_t)rem[k]);
+    }
+  }
+  DeviceGuard g(c->device);
+  c->pending = false;
+  std::vector<uint32_t> zero(I, 0);
+  PS_TRY_CUDA(c, cudaMemcpyAsync(c->rq.q_head, zero.data(), I * 4, cudaMemcpyHostToDevice, c->stream));
+  PS_TRY_CUDA(c, cudaMemcpyAsync(c->rq.q_len, qlen.data(), I * 4, cudaMemcpyHostToDevice, c->stream));
+  PS_TRY_CUDA(c, cudaMemcpyAsync(c->rq.d_len, dlen.data(), I * 4, cudaMemcpyHostToDevice, c->stream));
+  PS_TRY_CUDA(c, cudaMemcpyAsync(c->rq.q_L, qL.data(), IM * 4, cudaMemcpyHostToDevice, c->stream));
+  PS_TRY_CUDA(c, cudaMemcpyAsync(c->rq.q_out, qo.data(), IM * 4, cudaMemcpyHostToDevice, c->stream));
+  PS_TRY_CUDA(c, cudaMemcpyAsync(c->rq.q_rem, qR.data(), IM * 8, cudaMemcpyHostToDevice, c->stream));
+  PS_TRY_CUDA(c, cudaMemcpyAsync(c->rq.d_L, dL.data(), IM * 4, cudaMemcpyHostToDevice, c->stream));
+  PS_TRY_CUDA(c, cudaMemcpyAsync(c->rq.d_out, dO.data(), IM * 4, cudaMemcpyHostToDevice, c->stream));
+  PS_TRY_CUDA(c, cudaMemcpyAsync(c->rq.d_rem, dR.data(), IM * 4, cudaMemcpyHostToDevice, c->stream));
+  PS_TRY_CUDA(c, cudaMemcpyAsync(c->st.b, b.data(), I * 4, cudaMemcpyHostToDevice, c->stream));
+  PS_TRY_CUDA(c, cudaMemcpyAsync(c->st.qr, qr.data(), I * 4, cudaMemcpyHostToDevice, c->stream));
+  PS_TRY_CUDA(c, cudaMemcpyAsync(c->st.q, q.data(), I * 8, cudaMemcpyHostToDevice, c->stream));
+  PS_TRY_CUDA(c, cudaMemcpyAsync(c->st.S, S.data(), I * 8, cudaMemcpyHostToDevice, c->stream));
+  PS_TRY_CUDA(c, cudaStreamSynchronize(c->stream));
+  return PS_OK;
+}
+
+ps_status ps_advance_window(ps_ctx* c, const ps_advance_params* p) {
+  if (!c) return PS_ERR_INVALID;
+  if (!p || !(p->window_ms > 0.0f) || !std::isfinite(p->window_ms) || (p->evict != 0 && p->evict != 1))
+    return fail(c, PS_ERR_INVALID, "advance params: window_ms > 0, evict 0 or 1");
+  if (c->pending) return fail(c, PS_ERR_STATE, "commit the pending window before advancing");
+  if (!c->rq.M) return fail(c, PS_ERR_STATE, "context has no request tracking (max_active_requests = 0)");
+  if (p->evict && !c->lru) return fail(c, PS_ERR_STATE, "eviction needs track_lru");
+  DeviceGuard g(c->device);
+  PS_TRY_CUDA(c, pskl::launch_advance(c->st, c->I, c->rq, c->model, p->window_ms, p->prefill_tokens, c->d_err,
+                                      c->stream));
+  if (p->evict)
+    PS_TRY_CUDA(c, pskl::launch_evict(c->d_slots, c->d_ovf, c->d_tdesc, c->I, c->d_count, c->d_cap, c->meta,
+                                      c->d_err, c->stream));
   return finish(c);
 }
 

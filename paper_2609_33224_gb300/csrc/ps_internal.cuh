@@ -39,6 +39,8 @@ enum : uint32_t {
   kErrBadInstance = 16u,
   kErrParentMissing = 32u,
   kErrTimeout = 64u,
+  kErrRequestsFull = 128u,
+  kErrLeavesFull = 256u,
 };
 
 struct TableDesc {
@@ -130,43 +132,124 @@ __device__ __forceinline__ bool main_contains(const uint64_t* __restrict__ slots
   return false;
 }
 
-// Warp-cooperative insert of one key by the instance's only writer warp (all 32 lanes call it with
-// the same key).  Lanes 0-7 read bucket b1, lanes 8-15 bucket b2; the key goes to the emptier one.
-// Returns 1 if inserted, 0 if already present, -1 if the table is full.
-__device__ __forceinline__ int warp_insert(uint64_t* slots, uint64_t* ovf, const TableDesc d, uint64_t key) {
-  const int lane = threadIdx.x & 31;
-  if (main_contains<false>(slots, ovf, d, key)) return 0;
+// Global slot index of key in an instance's main table, or ~0 if absent (L2-coherent reads; used
+// by the table writers).
+__device__ __forceinline__ uint64_t main_find(const uint64_t* slots, const uint64_t* ovf, const TableDesc d,
+                                              uint64_t key) {
+  if (key == kEmpty || key == kTomb) return ~0ull;
   const uint32_t b1 = fastrange32(key, d.nbkt);
   const uint32_t b2 = fastrange32(remix(key), d.nbkt);
-  uint64_t* p = nullptr;
-  if (lane < 8) p = slots + d.base + (uint64_t)b1 * kBucketSlots + lane;
-  else if (lane < 16) p = slots + d.base + (uint64_t)b2 * kBucketSlots + (lane - 8);
-  const uint64_t v = p ? __ldcg(reinterpret_cast<const unsigned long long*>(p)) : ~0ull;
-  const unsigned empty = __ballot_sync(0xffffffffu, p != nullptr && v == kEmpty);
+  const uint64_t s1 = d.base + (uint64_t)b1 * kBucketSlots, s2 = d.base + (uint64_t)b2 * kBucketSlots;
+  ulonglong2 v[8];
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    v[k] = __ldcg(reinterpret_cast<const ulonglong2*>(slots + s1) + k);
+    v[4 + k] = __ldcg(reinterpret_cast<const ulonglong2*>(slots + s2) + k);
+  }
+  const uint64_t ow = __ldcg(ovf + d.ovf + (b1 >> 6));
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    if (v[k].x == key) return s1 + 2 * k;
+    if (v[k].y == key) return s1 + 2 * k + 1;
+    if (v[4 + k].x == key) return s2 + 2 * k;
+    if (v[4 + k].y == key) return s2 + 2 * k + 1;
+  }
+  if (!((ow >> (b1 & 63)) & 1ull)) return ~0ull;
+  uint32_t b = b1;
+  for (uint32_t p = 1; p < d.nbkt; ++p) {
+    b = (b + 1 == d.nbkt) ? 0u : b + 1;
+    const uint64_t sb = d.base + (uint64_t)b * kBucketSlots;
+    for (int k = 0; k < kBucketSlots; ++k)
+      if (__ldcg(reinterpret_cast<const unsigned long long*>(slots + sb + k)) == key) return sb + k;
+    if (!((__ldcg(ovf + d.ovf + (b >> 6)) >> (b & 63)) & 1ull)) return ~0ull;
+  }
+  return ~0ull;
+}
+
+// Per-block LRU metadata, parallel to the slot array (streaming caches only).
+struct LruMeta {
+  uint32_t* last_use;
+  uint32_t* children;
+  uint64_t* parent;
+};
+
+// Requests in flight per instance (streaming only): a FIFO ring of queued requests and an array of
+// decoding ones, each of capacity M per instance.
+struct ReqStore {
+  uint32_t M;
+  uint32_t* q_head;   // [I] ring start
+  uint32_t* q_len;    // [I]
+  uint32_t* q_L;      // [I*M]
+  uint32_t* q_out;    // [I*M]
+  uint64_t* q_rem;    // [I*M] remaining prefill tokens
+  uint32_t* d_len;    // [I]
+  uint32_t* d_L;      // [I*M]
+  uint32_t* d_out;    // [I*M]
+  uint32_t* d_rem;    // [I*M] remaining output tokens
+};
+
+// Warp-cooperative insert of one key by the instance's only writer warp (all 32 lanes call it with
+// the same arguments).  Lanes 0-7 read bucket b1, lanes 8-15 bucket b2; the key goes to the emptier
+// one.  With LRU metadata (meta.last_use != nullptr) a new block records (last_use, 0 children,
+// parent) and its cached parent gains a child; an existing block only has its last_use raised.
+// parent_slot, if not ~0, is the parent's known slot (saves a lookup).  Returns the key's slot, or
+// ~0 if the table is full; *inserted tells whether the key is new.
+__device__ __forceinline__ uint64_t warp_insert(uint64_t* slots, uint64_t* ovf, const TableDesc d, uint64_t key,
+                                                bool* inserted, LruMeta meta = LruMeta{nullptr, nullptr, nullptr},
+                                                uint64_t parent = 0, uint32_t last_use = 0,
+                                                uint64_t parent_slot = ~0ull) {
+  const int lane = threadIdx.x & 31;
+  *inserted = false;
+  const uint64_t found = main_find(slots, ovf, d, key);
+  if (found != ~0ull) {
+    if (meta.last_use && lane == 0 && meta.last_use[found] < last_use) meta.last_use[found] = last_use;
+    __syncwarp();
+    return found;
+  }
+  const uint32_t b1 = fastrange32(key, d.nbkt);
+  const uint32_t b2 = fastrange32(remix(key), d.nbkt);
+  uint64_t idx = ~0ull;
+  if (lane < 8) idx = d.base + (uint64_t)b1 * kBucketSlots + lane;
+  else if (lane < 16) idx = d.base + (uint64_t)b2 * kBucketSlots + (lane - 8);
+  const uint64_t v = idx != ~0ull ? __ldcg(reinterpret_cast<const unsigned long long*>(slots + idx)) : ~0ull;
+  const unsigned empty = __ballot_sync(0xffffffffu, idx != ~0ull && v == kEmpty);
   const unsigned e1 = empty & 0xFFu, e2 = empty & 0xFF00u;
-  int target = -1;  // lane whose slot receives the key
+  int target = -1;
   if (e1 || e2) {
     // emptier bucket (more empty slots), b1 on ties
     target = (__popc(e1) >= __popc(e2)) ? __ffs(e1) - 1 : __ffs(e2) - 1;
-    if (lane == target) *p = key;
-    __syncwarp();
-    return 1;
+  } else {
+    // both full: first non-full bucket after b1; mark b1 and every full bucket passed
+    uint32_t b = b1;
+    for (uint32_t step = 0; step < d.nbkt && target < 0; ++step) {
+      if (lane == 0) atomicOr(reinterpret_cast<unsigned long long*>(ovf + d.ovf + (b >> 6)), 1ull << (b & 63));
+      b = (b + 1 == d.nbkt) ? 0u : b + 1;
+      const uint64_t q = d.base + (uint64_t)b * kBucketSlots + (lane & 7);
+      const uint64_t w = lane < 8 ? __ldcg(reinterpret_cast<const unsigned long long*>(slots + q)) : ~0ull;
+      const unsigned em = __ballot_sync(0xffffffffu, lane < 8 && w == kEmpty);
+      if (em) {
+        target = __ffs(em) - 1;
+        idx = q;
+      }
+    }
+    if (target < 0) return ~0ull;
   }
-  // both full: first non-full bucket after b1; mark b1 and every full bucket passed
-  uint32_t b = b1;
-  for (uint32_t step = 0; step < d.nbkt; ++step) {
-    if (lane == 0) atomicOr(reinterpret_cast<unsigned long long*>(ovf + d.ovf + (b >> 6)), 1ull << (b & 63));
-    b = (b + 1 == d.nbkt) ? 0u : b + 1;
-    uint64_t* q = slots + d.base + (uint64_t)b * kBucketSlots + (lane & 7);
-    const uint64_t w = lane < 8 ? __ldcg(reinterpret_cast<const unsigned long long*>(q)) : ~0ull;
-    const unsigned em = __ballot_sync(0xffffffffu, lane < 8 && w == kEmpty);
-    if (em) {
-      if (lane == __ffs(em) - 1) *q = key;
-      __syncwarp();
-      return 1;
+  const uint64_t slot = __shfl_sync(0xffffffffu, idx, target);
+  if (lane == target) {
+    slots[slot] = key;
+    if (meta.last_use) {
+      meta.last_use[slot] = last_use;
+      meta.children[slot] = 0;
+      meta.parent[slot] = parent;
     }
   }
-  return -1;
+  if (meta.last_use && parent != kEmpty) {
+    const uint64_t ps = parent_slot != ~0ull ? parent_slot : main_find(slots, ovf, d, parent);
+    if (ps != ~0ull && lane == 0) meta.children[ps] += 1;
+  }
+  __syncwarp();
+  *inserted = true;
+  return slot;
 }
 
 __device__ __forceinline__ uint32_t delta_home(uint64_t key, uint32_t inst, uint32_t nbkt) {
@@ -548,11 +631,19 @@ cudaError_t launch_greedy(const uint64_t* slots, const uint64_t* ovf, const psk:
 cudaError_t launch_delta_clear(psk::DeltaSlot* delta, uint64_t nslots, cudaStream_t s);
 cudaError_t launch_insert_chains(uint64_t* slots, uint64_t* ovf, const psk::TableDesc* tdesc, uint32_t I,
                                  unsigned long long* count, uint64_t nchains, const uint32_t* inst,
-                                 const uint64_t* off, const uint64_t* hash, uint64_t total,
-                                 uint32_t* err, int num_sms, cudaStream_t s);
+                                 const uint64_t* off, const uint64_t* hash, const uint64_t* parent,
+                                 uint64_t total, psk::LruMeta meta, uint32_t last_use, uint32_t* err,
+                                 int num_sms, cudaStream_t s);
 cudaError_t launch_commit(uint64_t* slots, uint64_t* ovf, const psk::TableDesc* tdesc, uint32_t I,
                           unsigned long long* count, const psk::WindowDev& w, const int32_t* assign,
-                          const uint32_t* hit_chosen, uint32_t* err, int num_sms, cudaStream_t s);
+                          const uint32_t* hit_chosen, psk::LruMeta meta, uint32_t last_use,
+                          const psk::ReqStore& rq, const uint32_t* out_tokens, uint32_t* err, int num_sms,
+                          cudaStream_t s);
+cudaError_t launch_advance(psk::StateSoA st, uint32_t I, const psk::ReqStore& rq, const psk::DevModel& m,
+                           float window_ms, uint64_t prefill_tokens, uint32_t* err, cudaStream_t s);
+cudaError_t launch_evict(uint64_t* slots, uint64_t* ovf, const psk::TableDesc* tdesc, uint32_t I,
+                         unsigned long long* count, const uint64_t* cap, psk::LruMeta meta, uint32_t* err,
+                         cudaStream_t s);
 cudaError_t launch_check_parents(const uint64_t* slots, const uint64_t* ovf, const psk::TableDesc* tdesc, uint32_t I,
                                  uint64_t nchains, const uint32_t* inst, const uint64_t* parent,
                                  uint32_t* err, int num_sms, cudaStream_t s);

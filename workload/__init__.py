@@ -87,6 +87,8 @@ def _lib():
         lib.ws_free.argtypes = [ctypes.c_void_p]
         lib.ws_chain_from_tokens.restype = ctypes.c_uint64
         lib.ws_chain_from_tokens.argtypes = [ctypes.c_void_p, ctypes.c_uint64, ctypes.c_void_p]
+        lib.ws_initial_requests.restype = ctypes.c_uint64
+        lib.ws_initial_requests.argtypes = [ctypes.c_void_p] * 6
         lib.ws_det_exp.restype = ctypes.c_double
         lib.ws_det_exp.argtypes = [ctypes.c_double]
         lib.ws_det_log.restype = ctypes.c_double
@@ -131,11 +133,14 @@ CONFIGS = {
             ctx_min=131072, ctx_start_hi=524288, ctx_max=1048576, sys_tokens=32768, zipf_s=1.1,
             fork_every=10, hist_hi=20, cap_blocks=1 << 20, b_hi=128, q_hi=32768, b_max=256,
             tpot_target_ms=30.0, ttft_target_ms=3000.0, table_load_factor=0.5),
-    # streaming: 1024 instances, 1000 windows of 1000 requests, state carried across windows
+    # streaming: 1024 instances, 1000 windows of 1000 requests, state carried across windows.
+    # A commit merges a window's blocks before eviction runs; the capacity guard bounds an
+    # instance's admitted blocks per window by its KV capacity (= cap blocks), so tables get
+    # 2 x cap slots.
     4: dict(_COMMON, seed=4, num_instances=1024, window_requests=1000, num_sessions=8192,
             ctx_min=4096, ctx_start_hi=65536, ctx_max=131072, sys_tokens=4096, zipf_s=1.1,
             cap_blocks=200000, b_hi=128, q_hi=32768, b_max=256, tpot_target_ms=50.0,
-            ttft_target_ms=3000.0, table_load_factor=0.85),
+            ttft_target_ms=3000.0, table_load_factor=0.5),
 }
 
 
@@ -191,6 +196,18 @@ class Workload:
         lib.ws_next_window(self._handle, int(self.params["window_requests"] if R is None else R))
         self.window = _copy_window(self._handle)
         return self.window
+
+    def initial_requests(self) -> dict:
+        """Requests in flight at the start of a stream (see ws_initial_requests in gen.cpp):
+        inst, state (0 queued in FIFO order, 1 decoding), L, out, rem."""
+        lib = _lib()
+        n = int(lib.ws_initial_requests(self._handle, None, None, None, None, None))
+        r = dict(inst=np.zeros(n, np.uint32), state=np.zeros(n, np.uint32), L=np.zeros(n, np.uint32),
+                 out=np.zeros(n, np.uint32), rem=np.zeros(n, np.uint64))
+        if n:
+            lib.ws_initial_requests(self._handle, _p(r["inst"]), _p(r["state"]), _p(r["L"]), _p(r["out"]),
+                                    _p(r["rem"]))
+        return r
 
     def close(self):
         if self._handle is not None:

@@ -42,7 +42,7 @@ inline uint64_t splitmix64(uint64_t x) { return sm_finalise(x + kGolden); }
 enum Purpose : uint64_t {
   kPurposeSession = 1, kPurposePlace = 2, kPurposeHome = 3, kPurposePick = 4, kPurposeState = 5,
   kPurposeFill = 6, kPurposeFillTarget = 7, kPurposeBranchKey = 8, kPurposeSysKey = 9,
-  kPurposeOutput = 10,
+  kPurposeOutput = 10, kPurposeRequests = 11,
 };
 
 struct Rng {
@@ -420,6 +420,35 @@ void ws_copy_seed_chains(void* h, uint32_t* inst, uint64_t* off, uint64_t* hash,
   }
   std::memcpy(off, g->c_off.data(), (n + 1) * 8);
   if (!g->c_hash.empty()) std::memcpy(hash, g->c_hash.data(), g->c_hash.size() * 8);
+}
+
+// Requests in flight at the start of a stream, consistent with the instance state's counts: per
+// instance, b decoding requests (prompt U{1024..16384} tokens, output U{16..1024}, remaining output
+// U{1..output}) and qr queued ones holding the queued prefill tokens q in FIFO chunks of 4096 (the
+// remainder last), each with a prompt of its chunk plus U{0..8192} cached tokens.  With inst == NULL
+// only the count is returned.
+uint64_t ws_initial_requests(void* h, uint32_t* inst, uint32_t* state, uint32_t* L, uint32_t* out,
+                             uint64_t* rem) {
+  Gen* g = static_cast<Gen*>(h);
+  uint64_t n = 0;
+  for (uint32_t i = 0; i < g->p.num_instances; ++i) {
+    Rng rr(g->p.seed, kPurposeRequests, i);
+    for (int32_t k = 0; k < g->s_b[i]; ++k, ++n) {
+      const uint32_t l = (uint32_t)rr.range(1024, 16384);
+      const uint32_t o = (uint32_t)rr.range(16, 1024);
+      const uint32_t left = (uint32_t)rr.range(1, o);
+      if (inst) { inst[n] = i; state[n] = 1; L[n] = l; out[n] = o; rem[n] = left; }
+    }
+    int64_t q = g->s_q[i];
+    for (int32_t k = 0; k < g->s_qr[i]; ++k, ++n) {
+      const int64_t chunk = k + 1 < g->s_qr[i] ? 4096 : q;
+      q -= chunk;
+      const uint32_t l = (uint32_t)(chunk + rr.range(0, 8192));
+      const uint32_t o = (uint32_t)rr.range(16, 1024);
+      if (inst) { inst[n] = i; state[n] = 0; L[n] = l; out[n] = o; rem[n] = (uint64_t)chunk; }
+    }
+  }
+  return n;
 }
 
 // Drop the instance seed chains (they can be large) once the caller has copied them.
