@@ -3,7 +3,7 @@
  * packing for agentic LLM serving, arXiv 2609.33224).
  *
  * For a window of requests against every serving instance the library computes, on one GPU:
- *   1. the KV-cache prefix-hit length of each (request, instance) pair (Section 6: the scheduler's
+ *   1. the KV-cache prefix-hit length of each (request, instance) pair (Section 7: the scheduler's
  *      prefix tree of cached prefixes, here per-instance hash tables of chained block hashes);
  *   2. predicted TTFT and TPOT from the white-box prefill/decode model (Eq. 4-7, Eq. 9);
  *   3. the capacity guard, the normalised recompute filter (Eq. 8) and the SLO admission test
@@ -67,7 +67,7 @@ enum { PS_MAX_EMA_SEGMENTS = 16, PS_BLOCK_TOKENS = 16 };
  * TTFT (Eq. 4, overhead neglected): T_pf(n, c) + (a0*qr + a1*q_tokens).
  * eta: recompute budget of Eq. 8 (>= 0; the paper's default is 0.5).
  * ttft_filter: 1 adds "TTFT <= max(ttft_target, T_pf(L, 0))" to the TPOT admission test of
- * Algorithm 1 (the TTFT SLO of Section 7.1 Metrics); 0 applies Algorithm 1 exactly.
+ * Algorithm 1 (the TTFT SLO of Section 8.1 Metrics); 0 applies Algorithm 1 exactly.
  * All coefficients must be finite with magnitude <= 1e9; EMA factors finite and > 0. */
 typedef struct {
   float a0, a1, a2, a3, a4, a5;
@@ -98,7 +98,7 @@ typedef struct {
  *     PS_PROBE_LINEAR  (0) walk the chain 32 blocks per warp step until the first block that is
  *                          not cached; exact for any cache contents.
  *     PS_PROBE_SEARCH  (1) the caches must be prefix-closed (every cached block's parent is
- *                          cached, as in the paper's Section 6 prefix tree).  Then "block k is
+ *                          cached, as in the paper's Section 7 prefix tree).  Then "block k is
  *                          cached" is monotone along a chain and a warp finds the first miss by a
  *                          32-ary search (32 evenly spaced probes per step, at most 4 steps for
  *                          65536 blocks).  ps_insert_* checks the closure: a chain whose parent_hash
@@ -125,7 +125,7 @@ typedef struct {
   uint32_t max_active_requests;
 } ps_config;
 
-/* Scheduler-tracked state of one instance (Section 4 Metadata service; Section 5.5):
+/* Scheduler-tracked state of one instance (Section 4 Metadata service; Section 6.2):
  * b decoding requests, qr queued (not yet decoding) requests, q_tokens queued uncached prefill
  * tokens, S_tokens KV tokens held by the active requests, M_KV_tokens KV capacity, B_max decode-slot
  * limit.  Capacity guard of Algorithm 1: b + qr + 1 <= B_max and S_tokens + L <= M_KV_tokens.

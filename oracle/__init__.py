@@ -8,7 +8,7 @@ Parity status of each oracle function (what pins it, in ``tests/test_oracle_pins
   * hit length           -- brute-force token longest-common-prefix on explicit token lists.
   * T_pf / W / Z / rho   -- closed forms under the workload coefficients, fp64 cross-check.
   * TPOT / TTFT          -- hand-computed literals (golden hand example), fp64 cross-check.
-  * filters and picks    -- special cases of Section 5.4/5.5 (eta = 0, Z = 0, T empty, A empty),
+  * filters and picks    -- special cases of Sections 6.1/6.2 (eta = 0, Z = 0, T empty, A empty),
                             exhaustive brute force over tiny instance sets.
   * greedy               -- hand-traced tiny windows; replay invariant (each decision equals the
                             single-request rule on the state left by the earlier decisions).

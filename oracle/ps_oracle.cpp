@@ -7,7 +7,7 @@
 // service": state tracked along request paths).
 //
 // Data structures: one std::unordered_set<uint64_t> of cached block hashes per instance (the
-// paper's Section 6 prefix tree, flattened: a block hash covers its whole prefix, so "prefix
+// paper's Section 7 prefix tree, flattened: a block hash covers its whole prefix, so "prefix
 // cached" == "block hash present").  Hit length = a linear walk along the request's chain until
 // the first hash that is not in the set (exact whether or not the set is prefix-closed).
 //
@@ -25,10 +25,10 @@
 //    f = EMA factor of B's decode-batch segment (Section 5.3).  Paper form (Eq. 9):
 //    ((b0 + b1 B) + b2 S') f + [b + qr > 0] T_pf(n,c) / max(1, L_out).
 //  * TTFT (Eq. 4): T_pf(n,c) + (a0 qr + a1 q), overhead neglected; the budget is
-//    max(target, T_pf(L,0)) (Section 7.1 Metrics); TTFT uses <=, TPOT uses strict < (Alg. 1).
-//  * Packing key D-C-Q (Section 5.5, Table 4): more decoding b, then more cached blocks h, then
+//    max(target, T_pf(L,0)) (Section 8.1 Metrics); TTFT uses <=, TPOT uses strict < (Alg. 1).
+//  * Packing key D-C-Q (Section 6.2, Table 4): more decoding b, then more cached blocks h, then
 //    fewer queued requests qr, then the lowest instance id.  Fallback CacheAwareLB = LMetric
-//    (Section 6, Section 7.1 Baselines): min over C of (q + n)(b + qr + 1), lowest id on ties.
+//    (Section 6, Section 8.1 Baselines): min over C of (q + n)(b + qr + 1), lowest id on ties.
 //  * Streaming windows (the paper leaves engine progress to the serving engine; these are the
 //    simulation rules of the streaming workload).  Each instance keeps a FIFO queue of admitted
 //    requests (remaining uncached prefill tokens) and a set of decoding requests (remaining output
@@ -101,7 +101,7 @@ float t_pf(const orc_model& m, float N, float C) {
   return t;
 }
 
-// Hit length: cached prefix blocks of the chain on instance i (Section 6 prefix-tree lookup).
+// Hit length: cached prefix blocks of the chain on instance i (Section 7 prefix-tree lookup).
 uint64_t hit_len(const Oracle& o, uint32_t i, const uint64_t* chain, uint64_t nb) {
   uint64_t h = 0;
   while (h < nb && o.cache[i].count(chain[h])) ++h;
@@ -133,7 +133,7 @@ void decide(const Oracle& o, const uint64_t* chain, uint64_t nb, uint32_t L, flo
   const float Lf = (float)L;
   const float t_cached = t_pf(m, 0.0f, Lf);       // fully cached input
   const float t_cold = t_pf(m, Lf, 0.0f);         // fully uncached input
-  const float Z = t_cold - t_cached;              // CacheBenefit (Alg. 1, Section 5.4)
+  const float Z = t_cold - t_cached;              // CacheBenefit (Alg. 1, Section 6.1)
   const float etaZ = m.eta * Z;
   const float ttft_budget = t_cold > ttft_target ? t_cold : ttft_target;
   std::vector<float> W(I, 0.f), tpf(I, 0.f);
@@ -141,7 +141,7 @@ void decide(const Oracle& o, const uint64_t* chain, uint64_t nb, uint32_t L, flo
   std::vector<char> inA(I, 0);
   bool anyA = false;
   float Wmin = 0.f;
-  // Capacity guard + RecomputeCost (Alg. 1, KVC-first filtering; Section 5.4).
+  // Capacity guard + RecomputeCost (Alg. 1, KVC-first filtering; Section 6.1).
   for (uint32_t i = 0; i < I; ++i) {
     const orc_inst& s = o.st[i];
     uint64_t h = hit_len(o, i, chain, nb);

@@ -9,6 +9,8 @@
 #include <string>
 #include <vector>
 
+#include <algorithm>
+
 #include "packserve.h"
 #include "ps_internal.cuh"
 
@@ -47,7 +49,11 @@ struct ps_ctx {
   psk::TableDesc* d_tdesc = nullptr;
   unsigned long long* d_count = nullptr;
   psk::DeltaSlot* d_delta = nullptr;
-  uint32_t delta_nbkt = 0;
+  uint64_t delta_nslots = 0;
+  psk::GreedySync gsync{nullptr, nullptr, nullptr};
+  psk::RowPre* d_rows = nullptr;      // per-request constants and relations (search mode greedy)
+  psk::LastSlot* d_lastslot = nullptr;
+  uint32_t lastslot_n = 0;
   psk::StateSoA st{}, pend{};
   uint64_t* d_off = nullptr;
   uint64_t* d_hash = nullptr;
@@ -347,14 +353,17 @@ ps_status ps_create(const ps_config* cfg, ps_ctx** out) {
   }
   c->total_slots = base;
   c->total_ovf = obase;
-  const uint64_t dn = (2 * c->max_blocks + psk::kDeltaSlots - 1) / psk::kDeltaSlots;
-  if (dn >= (1ull << 32)) return bail(PS_ERR_INVALID);
-  c->delta_nbkt = (uint32_t)dn;
+  const uint64_t dn = std::max<uint64_t>(16, 2 * c->max_blocks);  // delta slots: twice a window's blocks
+  c->delta_nslots = dn;
+  c->lastslot_n = 64;
+  while (c->lastslot_n < 2 * c->Rmax) c->lastslot_n <<= 1;
   const size_t RI = (size_t)c->Rmax * c->I;
   const size_t I = c->I;
   bool ok = dalloc(c, &c->d_slots, c->total_slots) == cudaSuccess && dalloc(c, &c->d_ovf, c->total_ovf) == cudaSuccess &&
             dalloc(c, &c->d_tdesc, I) == cudaSuccess && dalloc(c, &c->d_count, I) == cudaSuccess &&
-            dalloc(c, &c->d_delta, (size_t)dn * psk::kDeltaSlots) == cudaSuccess;
+            dalloc(c, &c->d_delta, (size_t)dn) == cudaSuccess && dalloc(c, &c->gsync.jobs, c->Rmax) == cudaSuccess &&
+            dalloc(c, &c->gsync.done, c->Rmax) == cudaSuccess && dalloc(c, &c->gsync.pub, 1) == cudaSuccess &&
+            dalloc(c, &c->d_rows, c->Rmax) == cudaSuccess && dalloc(c, &c->d_lastslot, c->lastslot_n) == cudaSuccess;
   for (psk::StateSoA* s : {&c->st, &c->pend}) {
     ok = ok && dalloc(c, &s->b, I) == cudaSuccess && dalloc(c, &s->qr, I) == cudaSuccess &&
          dalloc(c, &s->q, I) == cudaSuccess && dalloc(c, &s->S, I) == cudaSuccess &&
@@ -394,7 +403,7 @@ ps_status ps_create(const ps_config* cfg, ps_ctx** out) {
              cudaMemcpyAsync(c->d_tdesc, td.data(), I * sizeof(psk::TableDesc), cudaMemcpyHostToDevice,
                              c->stream) == cudaSuccess &&
              cudaMemsetAsync(c->d_count, 0, I * sizeof(unsigned long long), c->stream) == cudaSuccess &&
-             cudaMemsetAsync(c->d_delta, 0, (size_t)dn * psk::kDeltaSlots * sizeof(psk::DeltaSlot), c->stream) ==
+             cudaMemsetAsync(c->d_delta, 0, (size_t)dn * sizeof(psk::DeltaSlot), c->stream) ==
                  cudaSuccess &&
              cudaMemsetAsync(c->d_err, 0, sizeof(uint32_t), c->stream) == cudaSuccess;
   for (psk::StateSoA* s : {&c->st, &c->pend}) {
@@ -597,12 +606,19 @@ ps_status ps_schedule_window(ps_ctx* c, const ps_window* w, ps_decisions* out, p
   s = run_probe_and_score(c, wd, opt_scores, &hit0);
   if (s != PS_OK) return s;
   record(c, kEvGreedy0);
-  PS_TRY_CUDA(c, pskl::launch_greedy(c->d_slots, c->d_ovf, c->d_tdesc, c->I, wd, hit0, c->st, c->pend, c->model, c->d_delta,
-                                     c->delta_nbkt, c->d_assign, c->d_dpath, c->d_hchosen,
-                                     c->d_err, c->search, c->stream));
+  if (c->search) {
+    PS_TRY_CUDA(c, pskl::launch_relations(wd, c->model, c->d_lastslot, c->lastslot_n, c->d_rows, c->num_sms, c->stream));
+    PS_TRY_CUDA(c, pskl::launch_greedy_search(c->d_rows, wd, c->I, hit0, c->st, c->pend, c->model, c->d_delta,
+                                              c->delta_nslots, c->d_assign, c->d_dpath, c->d_hchosen, c->d_err,
+                                              c->gsync, c->stream));
+  } else {
+    PS_TRY_CUDA(c, pskl::launch_greedy(c->d_slots, c->d_ovf, c->d_tdesc, c->I, wd, hit0, c->st, c->pend, c->model,
+                                       c->d_delta, c->delta_nslots, c->d_assign, c->d_dpath, c->d_hchosen, c->d_err,
+                                       0, c->stream));
+  }
   record(c, kEvGreedy1);
   c->ev_used[2] = true;
-  PS_TRY_CUDA(c, pskl::launch_delta_clear(c->d_delta, (uint64_t)c->delta_nbkt * psk::kDeltaSlots, c->stream));
+  PS_TRY_CUDA(c, pskl::launch_delta_clear(c->d_delta, c->delta_nslots, c->stream));
   if (out) {
     PS_TRY_CUDA(c, deliver(c, out->assign, c->d_assign, wd.R, out->outputs_on_device));
     PS_TRY_CUDA(c, deliver(c, out->path, c->d_dpath, wd.R, out->outputs_on_device));

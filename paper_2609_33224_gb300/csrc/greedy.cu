@@ -61,7 +61,7 @@ __global__ void __launch_bounds__(1024, 1)
 greedy_kernel(const uint64_t* __restrict__ slots, const uint64_t* __restrict__ ovf,
               const psk::TableDesc* __restrict__ tdesc, uint32_t I,
               psk::WindowDev w, const uint32_t* __restrict__ hit0, psk::StateSoA committed,
-              psk::StateSoA pending, psk::DevModel m, psk::DeltaSlot* delta, uint32_t delta_nbkt,
+              psk::StateSoA pending, psk::DevModel m, psk::DeltaSlot* delta, uint64_t delta_nslots,
               int32_t* __restrict__ assign, uint8_t* __restrict__ path, uint32_t* __restrict__ hit_chosen,
               uint32_t* err) {
   extern __shared__ unsigned long long smem_raw[];
@@ -123,7 +123,7 @@ greedy_kernel(const uint64_t* __restrict__ slots, const uint64_t* __restrict__ o
       const uint32_t i = t + k * NT;
       hc[k] = hn[k];
       if (i < I) {
-        if (s_touched[i] && hc[k] < nb && psk::delta_contains(delta, delta_nbkt, i, cn[k])) {
+        if (s_touched[i] && hc[k] < nb && psk::delta_contains(delta, delta_nslots, i, cn[k])) {
           const uint32_t at = atomicAdd(&s_nwalk, 1u);
           s_walk[at] = i;
         }
@@ -150,7 +150,7 @@ greedy_kernel(const uint64_t* __restrict__ slots, const uint64_t* __restrict__ o
         // the search only consults the delta; the linear walk checks both.
         auto cached = [&](uint64_t k) {
           const uint64_t key = w.hash[o + k];
-          return psk::delta_contains(delta, delta_nbkt, i, key) ||
+          return psk::delta_contains(delta, delta_nslots, i, key) ||
                  (!SEARCH && psk::main_contains(slots, ovf, d, key));
         };
         // Likely answer: where the last request assigned to i in this window ended (the same
@@ -236,7 +236,7 @@ greedy_kernel(const uint64_t* __restrict__ slots, const uint64_t* __restrict__ o
     }
     if (pick) {
       for (uint64_t k = (uint64_t)hj + t; k < nb; k += NT)
-        if (!psk::delta_insert(delta, delta_nbkt, j, w.hash[o + k])) atomicOr(err, psk::kErrDeltaFull);
+        if (!psk::delta_insert(delta, delta_nslots, j, w.hash[o + k])) atomicOr(err, psk::kErrDeltaFull);
     }
     __syncthreads();  // (E) state, delta and walk counter ready for the next request
   }
@@ -258,15 +258,440 @@ template <int IPT, bool SEARCH>
 cudaError_t greedy_launch(const uint64_t* slots, const uint64_t* ovf, const psk::TableDesc* tdesc, uint32_t I,
                           const psk::WindowDev& w, const uint32_t* hit0, psk::StateSoA committed,
                           psk::StateSoA pending, const psk::DevModel& m, psk::DeltaSlot* delta,
-                          uint32_t delta_nbkt, int32_t* assign, uint8_t* path, uint32_t* hit_chosen,
+                          uint64_t delta_nslots, int32_t* assign, uint8_t* path, uint32_t* hit_chosen,
                           uint32_t* err, uint32_t nt, cudaStream_t s) {
   const size_t smem = greedy_smem(I);
   cudaError_t e = cudaFuncSetAttribute(greedy_kernel<IPT, SEARCH>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)smem);
   if (e != cudaSuccess) return e;
   greedy_kernel<IPT, SEARCH><<<1, nt, smem, s>>>(slots, ovf, tdesc, I, w, hit0, committed, pending, m, delta,
-                                                 delta_nbkt, assign, path, hit_chosen, err);
+                                                 delta_nslots, assign, path, hit_chosen, err);
   return cudaGetLastError();
+}
+
+
+// ----------------------------------------------------------------------------------------------
+// Prefix-closed caches (the probe's search mode): a software-pipelined greedy pass.
+//
+// On a prefix-closed cache the hit of a request is the first chain position not cached, and the
+// union of prefix-closed sets has as first miss the largest of the sets' first misses.  The
+// cached set of instance i while request s is decided is main_i plus the chains of the window's
+// earlier requests assigned to i, so
+//     hit(s, i) = max( first miss of main_i + delta_i(<= s - 5),
+//                      lcp(s, s - d) for each d = 1..4 such that request s - d went to i )
+// where delta_i(<= s - 5) holds the blocks inserted for requests up to s - 5 and lcp(s, s - d) is
+// the common chain prefix (from the relations pass).  The first term is probed ahead of time, while
+// earlier requests are still being decided, so no table access is on the per-request critical
+// path.  The probe position is hit0, raised to the end of the request's parent (the deepest earlier
+// request whose chain is a prefix of this one) on the instance that took the parent; a probe that
+// finds the block cached hands the instance to a warp search.  Probes may also see inserts of
+// requests s - 4 .. s - 1 (they land while the probe runs): any snapshot between delta(<= s - 5)
+// and delta(<= s - 1) gives a first miss between the two, and the max with the lcp terms is then
+// exact all the same.
+//
+// Block 0 decides.  Per step r it evaluates row r (two block reductions: W_min, then the argmin)
+// and besides:  loads hit0 of row r + 3;  places row r + 2's probe and loads the chain block there
+// (instances with window inserts only);  issues row r + 1's probe (consumed after the first
+// barrier);  publishes request r's pick as an insert job.  Blocks 1..kHelpers insert each job's
+// chain blocks chain[h, nb) into delta_j and count themselves done; block 0 waits (bounded) for job
+// r - 3 before its row r + 2 probes go out; a dedicated signalling thread (the block's last warp
+// owns no instances) publishes the jobs and does that wait, so the release and acquire orderings
+// never hold up a thread with loads in flight.  Instance state lives in shared memory and is
+// written only by the thread that owns the instance.
+
+constexpr uint32_t kHelpers = 8;              // insert blocks beside the deciding block
+constexpr uint32_t kLag = 5;                  // a probe for row s sees every insert of requests <= s - kLag
+constexpr uint64_t kWaitNs = 1000000000ull;   // bound on any cross-block wait
+constexpr unsigned long long kAbortJob = ~0ull;
+
+struct PickKey {  // lexicographic (class, value, instance) element carrying the pair's hit
+  uint32_t ci;
+  uint32_t h;
+  uint64_t v;
+};
+
+__device__ __forceinline__ bool pick_less(const PickKey& a, const PickKey& z) {
+  return psk::key_less(psk::ArgKey{a.ci, a.v}, psk::ArgKey{z.ci, z.v});
+}
+
+__device__ __forceinline__ PickKey warp_pick(PickKey k) {
+#pragma unroll
+  for (int s = 16; s > 0; s >>= 1) {
+    PickKey o;
+    o.ci = __shfl_xor_sync(0xffffffffu, k.ci, s);
+    o.h = __shfl_xor_sync(0xffffffffu, k.h, s);
+    o.v = __shfl_xor_sync(0xffffffffu, k.v, s);
+    if (pick_less(o, k)) k = o;
+  }
+  return k;
+}
+
+__device__ __forceinline__ psk::RowConst row_of(const psk::RowPre& x) {
+  psk::RowConst rc;
+  rc.t_cached = x.t_cached;
+  rc.Z = x.Z;
+  rc.etaZ = x.etaZ;
+  rc.ttft_budget = x.ttft_budget;
+  rc.tpot_target = x.tpot_target;
+  rc.L = x.L;
+  return rc;
+}
+
+// Blocks 1..kHelpers: insert every published pick's chain tail, in request order.
+__device__ void insert_helper(const psk::RowPre* __restrict__ rows, const uint64_t* __restrict__ hash, uint32_t R,
+                              psk::DeltaSlot* delta, uint64_t nslots, uint32_t* err, const psk::GreedySync& sync) {
+  __shared__ unsigned long long s_job;
+  const uint32_t t = threadIdx.x;
+  const uint64_t stride = (uint64_t)kHelpers * blockDim.x;
+  const uint64_t first = (uint64_t)(blockIdx.x - 1) * blockDim.x + t;
+  for (uint32_t job = 0; job < R; ++job) {
+    if (t == 0) {
+      const uint64_t t0 = psk::globaltimer_ns();
+      unsigned long long jb = kAbortJob;
+      for (;;) {
+        if (psk::ld_acquire_u32(sync.pub) > job) {
+          jb = __ldcg(sync.jobs + job);
+          break;
+        }
+        if (psk::globaltimer_ns() - t0 > kWaitNs) {
+          atomicOr(err, psk::kErrTimeout);
+          break;
+        }
+        __nanosleep(100);
+      }
+      s_job = jb;
+    }
+    __syncthreads();
+    const unsigned long long jb = s_job;
+    if (jb == kAbortJob) return;  // block-uniform
+    const uint32_t j = (uint32_t)jb;
+    const uint32_t hj = (uint32_t)(jb >> 32);
+    // rows >= job + kLag are the only ones that read this job's inserts
+    if (j != 0xFFFFFFFFu && job + kLag < R) {
+      const uint64_t off = __ldg(&rows[job].off);
+      const uint32_t nb = __ldg(&rows[job].nb);
+      for (uint64_t p = hj + first; p < nb; p += stride)
+        if (!psk::delta_insert(delta, nslots, j, __ldg(hash + off + p))) atomicOr(err, psk::kErrDeltaFull);
+    }
+    __syncthreads();
+    if (t == 0) {
+      __threadfence();  // release every thread's inserts before the count
+      atomicAdd(sync.done + job, 1u);
+    }
+  }
+}
+
+template <int IPT>
+__global__ void __launch_bounds__(544, 1)
+greedy_search_kernel(const psk::RowPre* __restrict__ rows, const uint64_t* __restrict__ hash, uint32_t R, uint32_t I,
+                     const uint32_t* __restrict__ hit0, psk::StateSoA committed, psk::StateSoA pending,
+                     psk::DevModel m, psk::DeltaSlot* delta, uint64_t nslots, int32_t* assign,
+                     uint8_t* __restrict__ path, uint32_t* __restrict__ hit_chosen, uint32_t* err,
+                     psk::GreedySync sync) {
+  if (blockIdx.x > 0) {
+    insert_helper(rows, hash, R, delta, nslots, err, sync);
+    return;
+  }
+  extern __shared__ unsigned long long smem_raw[];
+  int64_t* s_q = reinterpret_cast<int64_t*>(smem_raw);
+  int64_t* s_S = s_q + I;
+  int64_t* s_M = s_S + I;
+  int32_t* s_b = reinterpret_cast<int32_t*>(s_M + I);
+  int32_t* s_qr = s_b + I;
+  int32_t* s_Bmax = s_qr + I;
+  uint32_t* s_end = reinterpret_cast<uint32_t*>(s_Bmax + I);  // chain end of the last request on i
+  uint32_t* s_wres = s_end + I;                                // search start / result per instance
+  uint32_t* s_walk = s_wres + I;                               // instances handed to a warp search
+  psk::InstTerms* s_it = reinterpret_cast<psk::InstTerms*>(s_walk + I);
+  uint8_t* s_touched = reinterpret_cast<uint8_t*>(s_it + I);
+  __shared__ psk::RowPre s_row[8];  // rows r .. r + 4 (a ring of 8 so no reader is overtaken)
+  __shared__ float s_red_w[32];
+  __shared__ int s_red_a[32];
+  __shared__ PickKey s_red_k[32];
+  __shared__ uint32_t s_nwalk[2];
+
+  const int t = threadIdx.x;
+  const int NT = blockDim.x;
+  const int NTI = NT - 32;  // threads owning instances; the last warp signals
+  const bool sig = t == NTI;
+  const int lane = t & 31;
+  const int warp = t >> 5;
+  const int NW = NT >> 5;
+  // instance k of this thread (out of range for the signalling warp)
+  auto own = [&](int k) -> uint32_t { return t < NTI ? (uint32_t)(t + k * NTI) : 0xFFFFFFFFu; };
+
+  for (uint32_t i = t; i < I; i += NT) {
+    s_b[i] = committed.b[i];
+    s_qr[i] = committed.qr[i];
+    s_q[i] = committed.q[i];
+    s_S[i] = committed.S[i];
+    s_M[i] = committed.M[i];
+    s_Bmax[i] = committed.Bmax[i];
+    s_end[i] = 0;
+    s_touched[i] = 0;
+    s_it[i] = psk::inst_terms(m, s_b[i], s_qr[i], s_q[i], s_Bmax[i]);
+  }
+  if (t < 16) {
+    const uint32_t rr = (uint32_t)(t >> 2);
+    if (rr < R) reinterpret_cast<uint4*>(&s_row[rr])[t & 3] = __ldg(reinterpret_cast<const uint4*>(rows + rr) + (t & 3));
+  }
+  if (t < 2) s_nwalk[t] = 0;
+
+  uint32_t hr[IPT], h1[IPT], h2[IPT];
+  uint64_t key1[IPT];
+  bool need1[IPT];
+#pragma unroll
+  for (int k = 0; k < IPT; ++k) {
+    const uint32_t i = own(k);
+    hr[k] = (i < I && R > 0) ? __ldg(hit0 + i) : 0u;
+    h1[k] = (i < I && R > 1) ? __ldg(hit0 + (uint64_t)I + i) : 0u;
+    h2[k] = (i < I && R > 2) ? __ldg(hit0 + 2ull * I + i) : 0u;
+    key1[k] = 0;
+    need1[k] = false;
+  }
+  int32_t jm1 = -1, jm2 = -1, jm3 = -1, jm4 = -1;  // picks of requests r - 1 .. r - 4
+  int32_t jp_pre = -1;                             // pick of row r + 2's parent, loaded one step ahead
+  bool timed_out = false;
+  __syncthreads();
+
+  for (uint32_t r = 0; r < R; ++r) {
+    const psk::RowPre& cur = s_row[r & 7];
+    const uint32_t nb = cur.nb;
+    // ---- P0: ring refill, stages A-C, corrections and row evaluation -----------------------------
+    if (t < 4 && r + 4 < R) {
+      psk::cp_async16(reinterpret_cast<uint4*>(&s_row[(r + 4) & 7]) + t, reinterpret_cast<const uint4*>(rows + r + 4) + t);
+      psk::cp_async_commit();
+    }
+    // the parent's pick for row r + 3 when it is old enough to be in global memory
+    int32_t jp_next = -1;
+    if (r + 3 < R) {
+      const int32_t par3 = s_row[(r + 3) & 7].par;
+      if (par3 >= 0 && (int64_t)par3 <= (int64_t)r - 4) jp_next = __ldcg(assign + par3);
+    }
+    uint32_t h3[IPT];
+#pragma unroll
+    for (int k = 0; k < IPT; ++k) {
+      const uint32_t i = own(k);
+      h3[k] = (i < I && r + 3 < R) ? __ldg(hit0 + (uint64_t)(r + 3) * I + i) : 0u;
+    }
+    uint64_t key2[IPT];
+    bool need2[IPT];
+    if (r + 2 < R) {
+      const psk::RowPre& x2 = s_row[(r + 2) & 7];
+      // the parent counts only if its inserts are in every probe snapshot: par <= (r + 2) - kLag
+      const int64_t par = x2.par;
+      int32_t jp = -1;
+      if (par >= 0) {
+        if (par == (int64_t)r - 3) jp = jm3;
+        else if (par == (int64_t)r - 4) jp = jm4;
+        else if (par <= (int64_t)r - 5) jp = jp_pre;
+      }
+#pragma unroll
+      for (int k = 0; k < IPT; ++k) {
+        const uint32_t i = own(k);
+        uint32_t pos = h2[k];
+        if ((int32_t)i == jp && x2.par_nb > pos) pos = x2.par_nb;
+        need2[k] = i < I && s_touched[i] && pos < x2.nb;
+        key2[k] = need2[k] ? __ldg(hash + x2.off + pos) : 0ull;
+        h2[k] = pos;
+      }
+    } else {
+#pragma unroll
+      for (int k = 0; k < IPT; ++k) {
+        need2[k] = false;
+        key2[k] = 0;
+      }
+    }
+    ulonglong2 pv0[IPT], pv1[IPT];
+    uint64_t home1[IPT];
+#pragma unroll
+    for (int k = 0; k < IPT; ++k) {
+      const uint32_t i = own(k);
+      if (need1[k]) {
+        home1[k] = psk::delta_home(key1[k], nslots);
+        pv0[k] = __ldcg(reinterpret_cast<const ulonglong2*>(delta + home1[k]));
+        pv1[k] = __ldcg(reinterpret_cast<const ulonglong2*>(delta + psk::delta_next(home1[k], nslots)));
+      } else {
+        home1[k] = 0;
+        pv0[k] = make_ulonglong2(0ull, 0ull);
+        pv1[k] = make_ulonglong2(0ull, 0ull);
+      }
+    }
+
+    const psk::RowConst rc = row_of(cur);
+    psk::PairEval ev[IPT];
+    float wmin = INFINITY;
+    bool anyA = false;
+#pragma unroll
+    for (int k = 0; k < IPT; ++k) {
+      const uint32_t i = own(k);
+      if (i < I) {
+        uint32_t h = hr[k];
+        if ((int32_t)i == jm1 && cur.lcp[0] > h) h = cur.lcp[0];
+        if ((int32_t)i == jm2 && cur.lcp[1] > h) h = cur.lcp[1];
+        if ((int32_t)i == jm3 && cur.lcp[2] > h) h = cur.lcp[2];
+        if ((int32_t)i == jm4 && cur.lcp[3] > h) h = cur.lcp[3];
+        hr[k] = h;
+        ev[k] = psk::eval_pair_terms(m, rc, h, s_it[i], s_q[i], s_S[i], s_M[i]);
+        if (ev[k].inA) {
+          wmin = fminf(wmin, ev[k].W);
+          anyA = true;
+        }
+      } else {
+        ev[k].inA = false;
+      }
+    }
+    wmin = psk::warp_fmin(wmin);
+    anyA = __any_sync(0xffffffffu, anyA);
+    if (lane == 0) {
+      s_red_w[warp] = wmin;
+      s_red_a[warp] = anyA ? 1 : 0;
+    }
+    __syncthreads();  // (C)
+
+    // ---- P1: W_min, admission classes, argmin; row r + 1's probes; wait for job r - 3 -------------
+    {
+      const float v = lane < NW ? s_red_w[lane] : INFINITY;
+      const bool a = lane < NW ? (s_red_a[lane] != 0) : false;
+      wmin = psk::warp_fmin(v);
+      anyA = __any_sync(0xffffffffu, a);
+    }
+    PickKey best{psk::kNoKeyCi, 0u, ~0ull};
+#pragma unroll
+    for (int k = 0; k < IPT; ++k) {
+      const uint32_t i = own(k);
+      if (i < I && ev[k].inA) {
+        const uint32_t cls = psk::pair_class(m, rc, ev[k], wmin);
+        if (cls <= 1u) {
+          const PickKey kk{(cls << 28) | i, hr[k], psk::pair_value(cls, hr[k], s_b[i], s_qr[i], s_q[i], ev[k].n)};
+          if (pick_less(kk, best)) best = kk;
+        }
+      }
+    }
+    best = warp_pick(best);
+    if (lane == 0) s_red_k[warp] = best;
+    bool walked[IPT];
+#pragma unroll
+    for (int k = 0; k < IPT; ++k) {
+      const uint32_t i = own(k);
+      walked[k] = false;
+      if (need1[k]) {
+        int v = psk::delta_slot_verdict(pv0[k], key1[k], i + 1);
+        if (v < 0) v = psk::delta_slot_verdict(pv1[k], key1[k], i + 1);
+        const bool present = v >= 0 ? v == 1
+                                    : psk::delta_contains_from(delta, nslots, i, key1[k],
+                                                               psk::delta_next(psk::delta_next(home1[k], nslots), nslots));
+        if (present) {
+          const uint32_t x = atomicAdd(&s_nwalk[(r + 1) & 1], 1u);
+          s_walk[x] = i;
+          s_wres[i] = h1[k];
+          walked[k] = true;
+        }
+      }
+    }
+    if (t < 4) psk::cp_async_wait_all();
+    // Row r + 2's probes (issued in the next step) need every insert of requests <= r - 3.
+    if (sig && r >= 3 && !timed_out) {
+      const uint64_t t0 = psk::globaltimer_ns();
+      while (psk::ld_acquire_u32(sync.done + (r - 3)) < kHelpers) {
+        if (psk::globaltimer_ns() - t0 > kWaitNs) {
+          atomicOr(err, psk::kErrTimeout);
+          timed_out = true;
+          break;
+        }
+      }
+    }
+    __syncthreads();  // (D)
+
+    // ---- P2: the pick, its state, its insert job; searches for row r + 1 --------------------------
+    {
+      const PickKey o = lane < NW ? s_red_k[lane] : PickKey{psk::kNoKeyCi, 0u, ~0ull};
+      best = warp_pick(o);
+    }
+    const bool pick = anyA && best.ci != psk::kNoKeyCi;
+    const uint32_t j = best.ci & 0x0FFFFFFFu;
+    const uint32_t hj = pick ? best.h : 0u;
+    if (sig) {
+      assign[r] = pick ? (int32_t)j : -1;
+      path[r] = pick ? (uint8_t)(best.ci >> 28) : (uint8_t)2;
+      hit_chosen[r] = hj;
+      s_nwalk[r & 1] = 0;
+      sync.jobs[r] = ((unsigned long long)hj << 32) | (pick ? j : 0xFFFFFFFFu);
+      psk::st_release_u32(sync.pub, r + 1);
+    }
+    if (pick && (j % (uint32_t)NTI) == (uint32_t)t) {
+      s_qr[j] += 1;
+      s_q[j] += (int64_t)rc.L - 16 * (int64_t)hj;
+      s_S[j] += (int64_t)rc.L;
+      s_end[j] = nb;
+      s_touched[j] = 1;
+      s_it[j] = psk::inst_terms(m, s_b[j], s_qr[j], s_q[j], s_Bmax[j]);
+    }
+    const uint32_t nwalk = r + 1 < R ? s_nwalk[(r + 1) & 1] : 0u;
+    if (nwalk) {
+      const psk::RowPre& x1 = s_row[(r + 1) & 7];
+      const uint64_t xoff = x1.off, xnb = x1.nb;
+      for (uint32_t x = warp; x < nwalk; x += NW) {
+        const uint32_t i = s_walk[x];
+        auto cached = [&](uint64_t k) {
+          return k < xnb && psk::delta_contains(delta, nslots, i, __ldg(hash + xoff + k));
+        };
+        const uint64_t hnew = psk::warp_first_miss_search_hint((uint64_t)s_wres[i] + 1, xnb, s_end[i], cached);
+        __syncwarp();
+        if (lane == 0) s_wres[i] = (uint32_t)hnew;
+      }
+      __syncthreads();  // (E) search results visible to the owners
+#pragma unroll
+      for (int k = 0; k < IPT; ++k)
+        if (walked[k]) h1[k] = s_wres[own(k)];
+    }
+#pragma unroll
+    for (int k = 0; k < IPT; ++k) {
+      hr[k] = h1[k];
+      h1[k] = h2[k];
+      key1[k] = key2[k];
+      need1[k] = need2[k];
+      h2[k] = h3[k];
+    }
+    jm4 = jm3;
+    jm3 = jm2;
+    jm2 = jm1;
+    jm1 = pick ? (int32_t)j : -1;
+    jp_pre = jp_next;
+  }
+  for (uint32_t i = t; i < I; i += NT) {
+    pending.b[i] = s_b[i];
+    pending.qr[i] = s_qr[i];
+    pending.q[i] = s_q[i];
+    pending.S[i] = s_S[i];
+    pending.M[i] = s_M[i];
+    pending.Bmax[i] = s_Bmax[i];
+  }
+}
+
+size_t greedy_search_smem(uint32_t I) {
+  return (size_t)I * (3 * sizeof(int64_t) + 3 * sizeof(int32_t) + 3 * sizeof(uint32_t) + sizeof(psk::InstTerms) + 1) + 16;
+}
+
+template <int IPT>
+cudaError_t greedy_search_launch(const psk::RowPre* rows, const psk::WindowDev& w, uint32_t I, const uint32_t* hit0,
+                                 psk::StateSoA committed, psk::StateSoA pending, const psk::DevModel& m,
+                                 psk::DeltaSlot* delta, uint64_t nslots, int32_t* assign, uint8_t* path,
+                                 uint32_t* hit_chosen, uint32_t* err, const psk::GreedySync& sync, uint32_t nt,
+                                 cudaStream_t s) {
+  const size_t smem = greedy_search_smem(I);
+  cudaError_t e = cudaFuncSetAttribute(greedy_search_kernel<IPT>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
+  const uint64_t* hash = w.hash;
+  uint32_t R = w.R;
+  psk::StateSoA c = committed, p = pending;
+  psk::DevModel mm = m;
+  psk::GreedySync sy = sync;
+  void* args[] = {(void*)&rows, (void*)&hash, (void*)&R, (void*)&I, (void*)&hit0, (void*)&c, (void*)&p,
+                  (void*)&mm, (void*)&delta, (void*)&nslots, (void*)&assign, (void*)&path, (void*)&hit_chosen,
+                  (void*)&err, (void*)&sy};
+  // all 1 + kHelpers blocks must be resident at once: they wait on one another
+  return cudaLaunchCooperativeKernel((const void*)greedy_search_kernel<IPT>, dim3(1 + kHelpers), dim3(nt), args, smem, s);
 }
 
 }  // namespace
@@ -276,20 +701,41 @@ namespace pskl {
 cudaError_t launch_greedy(const uint64_t* slots, const uint64_t* ovf, const psk::TableDesc* tdesc, uint32_t I,
                           const psk::WindowDev& w, const uint32_t* hit0, psk::StateSoA committed,
                           psk::StateSoA pending, const psk::DevModel& m, psk::DeltaSlot* delta,
-                          uint32_t delta_nbkt, int32_t* assign, uint8_t* path, uint32_t* hit_chosen,
+                          uint64_t delta_nslots, int32_t* assign, uint8_t* path, uint32_t* hit_chosen,
                           uint32_t* err, int search, cudaStream_t s) {
   uint32_t nt = (I + 31) / 32 * 32;
   if (nt > 1024) nt = 1024;
   const uint32_t ipt = (I + nt - 1) / nt;
 #define PS_GREEDY(IPT)                                                                                         \
   return search ? greedy_launch<IPT, true>(slots, ovf, tdesc, I, w, hit0, committed, pending, m, delta,        \
-                                           delta_nbkt, assign, path, hit_chosen, err, nt, s)                   \
+                                           delta_nslots, assign, path, hit_chosen, err, nt, s)                   \
                 : greedy_launch<IPT, false>(slots, ovf, tdesc, I, w, hit0, committed, pending, m, delta,       \
-                                            delta_nbkt, assign, path, hit_chosen, err, nt, s)
+                                            delta_nslots, assign, path, hit_chosen, err, nt, s)
   if (ipt <= 1) PS_GREEDY(1);
   if (ipt <= 2) PS_GREEDY(2);
   if (ipt <= 4) PS_GREEDY(4);
 #undef PS_GREEDY
+  return cudaErrorInvalidValue;
+}
+
+cudaError_t launch_greedy_search(const psk::RowPre* rows, const psk::WindowDev& w, uint32_t I, const uint32_t* hit0,
+                                 psk::StateSoA committed, psk::StateSoA pending, const psk::DevModel& m,
+                                 psk::DeltaSlot* delta, uint64_t delta_nslots, int32_t* assign, uint8_t* path,
+                                 uint32_t* hit_chosen, uint32_t* err, const psk::GreedySync& sync, cudaStream_t s) {
+  cudaError_t e = w.R ? cudaMemsetAsync(sync.done, 0, (size_t)w.R * sizeof(uint32_t), s) : cudaSuccess;
+  if (e == cudaSuccess) e = cudaMemsetAsync(sync.pub, 0, sizeof(uint32_t), s);
+  if (e != cudaSuccess) return e;
+  // up to 512 threads each owning IPT instances (IPT = 1, 2 or 4 for I up to 2048), plus one
+  // signalling warp
+  const uint32_t ipt = I <= 512 ? 1u : (I <= 1024 ? 2u : 4u);
+  const uint32_t nt = ((I + ipt - 1) / ipt + 31) / 32 * 32 + 32;
+#define PS_GREEDY_S(IPT)                                                                                        \
+  return greedy_search_launch<IPT>(rows, w, I, hit0, committed, pending, m, delta, delta_nslots, assign, path,  \
+                                   hit_chosen, err, sync, nt, s)
+  if (ipt == 1) PS_GREEDY_S(1);
+  if (ipt == 2) PS_GREEDY_S(2);
+  if (ipt == 4 && I <= 2048) PS_GREEDY_S(4);
+#undef PS_GREEDY_S
   return cudaErrorInvalidValue;
 }
 

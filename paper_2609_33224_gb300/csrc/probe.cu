@@ -2,7 +2,7 @@
 //
 // hit(r, i) = the first chain position k whose block hash is not cached on instance i (= the
 // chain length if every block is cached): the cached prefix of the request on that instance, the
-// quantity the paper's scheduler reads from its prefix tree (Section 6) to estimate KVC reuse.
+// quantity the paper's scheduler reads from its prefix tree (Section 7) to estimate KVC reuse.
 //
 // One thread block per request (grid-stride over requests).  The request's chain is staged in
 // shared memory once (coalesced 8-byte loads) and reused by every instance's probe; positions past

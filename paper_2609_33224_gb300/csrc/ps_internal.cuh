@@ -27,7 +27,6 @@ namespace psk {
 constexpr uint64_t kEmpty = 0ull;
 constexpr uint64_t kTomb = ~0ull;
 constexpr int kBucketSlots = 8;    // main table: 8 x 8 B = 64 B
-constexpr int kDeltaSlots = 8;     // delta table: 8 x 16 B
 constexpr uint32_t kDeltaNoInst = 0xFFFFFFFFu;
 
 // Device error bits, OR-ed into one word per context and turned into a ps_status on the host.
@@ -50,9 +49,46 @@ struct TableDesc {
   uint32_t pad;
 };
 
+// One key of the window's delta table with up to two of the instances it was inserted for
+// (instance id + 1 in ia, then ib; 0 = free).  A key with more instances continues in a later slot.
 struct DeltaSlot {
   unsigned long long hash;
-  unsigned int inst1;  // instance id + 1; 0 while the slot is being claimed (never matches)
+  unsigned int ia;
+  unsigned int ib;
+};
+
+// Per-request constants of one window, computed in parallel before the greedy pass: the request's
+// chain range, the Algorithm 1 / Eq. 8 row constants, and its relations to earlier requests of the
+// window (longest common chain prefix with each of the four requests before it; the deepest earlier
+// request whose whole chain is a prefix of this one).
+struct __align__(16) RowPre {
+  uint64_t off;
+  uint32_t nb;
+  uint32_t L;
+  float t_cached;     // T_pf(0, L)
+  float Z;            // T_pf(L, 0) - T_pf(0, L)
+  float etaZ;         // eta * Z
+  float ttft_budget;  // max(target, T_pf(L, 0))
+  float tpot_target;
+  uint32_t lcp[4];    // common chain prefix with requests r - 1 .. r - 4 (blocks)
+  int32_t par;        // deepest earlier request whose chain is a prefix of r's, -1 if none
+  uint32_t par_nb;    // its chain length
+  uint32_t pad;
+};
+static_assert(sizeof(RowPre) == 64, "RowPre is one 64-byte record");
+
+// Hand-off between the greedy block and the blocks that insert its picks' chains into the delta
+// table (one cooperative launch).
+struct GreedySync {
+  unsigned long long* jobs;  // per request: hit of the pick << 32 | pick (0xFFFFFFFF = rejected)
+  uint32_t* done;            // per request: insert blocks that have finished its blocks
+  uint32_t* pub;             // number of requests published so far
+};
+
+// Window table from a chain's last block hash to the earliest request ending there.
+struct LastSlot {
+  unsigned long long key;
+  unsigned int neg_idx;  // 0xFFFFFFFF - request index (atomicMax keeps the earliest)
   unsigned int pad;
 };
 
@@ -252,52 +288,92 @@ __device__ __forceinline__ uint64_t warp_insert(uint64_t* slots, uint64_t* ovf, 
   return slot;
 }
 
-__device__ __forceinline__ uint32_t delta_home(uint64_t key, uint32_t inst, uint32_t nbkt) {
-  return fastrange32(key ^ ((uint64_t)(inst + 1) * 0x9E3779B97F4A7C15ull), nbkt);
+// The window's delta table: open addressing with linear probing over 16-byte slots, the home slot
+// a function of the block hash alone, so lookups of one block for many instances read one line.
+__device__ __forceinline__ uint64_t delta_home(uint64_t key, uint64_t nslots) { return __umul64hi(key, nslots); }
+
+__device__ __forceinline__ uint64_t delta_next(uint64_t slot, uint64_t nslots) {
+  return slot + 1 == nslots ? 0ull : slot + 1;
 }
 
-// Membership of (inst, key) in the delta table.  The delta table is written by the same thread
-// block between reads (separated by __syncthreads), so it is read through the coherent path.
-__device__ __forceinline__ bool delta_contains(const DeltaSlot* delta, uint32_t nbkt, uint32_t inst,
-                                               uint64_t key) {
+// Verdict of one slot for (key, tag = inst + 1): 1 present, 0 absent, -1 look at the next slot.
+// Slots fill as an unbroken run from a key's home (inserts only claim empty slots and nothing is
+// removed while a window runs), instances fill ia then ib, and a key moves on to a later slot only
+// once both are taken; so an empty slot, or an entry of the key with a free instance field, ends
+// the search.
+__device__ __forceinline__ int delta_slot_verdict(const ulonglong2& v, uint64_t key, uint32_t tag) {
+  if (v.x == key) {
+    const uint32_t ia = (uint32_t)v.y, ib = (uint32_t)(v.y >> 32);
+    if (ia == tag || ib == tag) return 1;
+    return (ia == 0u || ib == 0u) ? 0 : -1;
+  }
+  return v.x == kEmpty ? 0 : -1;
+}
+
+// Membership of (inst, key) from a given slot on, read through L2 (other blocks may be inserting).
+__device__ __forceinline__ bool delta_contains_from(const DeltaSlot* delta, uint64_t nslots, uint32_t inst,
+                                                    uint64_t key, uint64_t slot) {
+  for (uint64_t p = 0; p < nslots; ++p) {
+    const int v = delta_slot_verdict(__ldcg(reinterpret_cast<const ulonglong2*>(delta + slot)), key, inst + 1);
+    if (v >= 0) return v == 1;
+    slot = delta_next(slot, nslots);
+  }
+  return false;
+}
+
+__device__ __forceinline__ bool delta_contains(const DeltaSlot* delta, uint64_t nslots, uint32_t inst, uint64_t key) {
   if (key == kEmpty || key == kTomb) return false;
-  uint32_t b = delta_home(key, inst, nbkt);
-  for (uint32_t p = 0; p < nbkt; ++p) {
-    const ulonglong2* line = reinterpret_cast<const ulonglong2*>(delta + (uint64_t)b * kDeltaSlots);
-#pragma unroll
-    for (int k = 0; k < kDeltaSlots; ++k) {
-      const ulonglong2 v = __ldcg(line + k);
-      if (v.x == key && (uint32_t)v.y == inst + 1) return true;
-      if (v.x == kEmpty) return false;
+  return delta_contains_from(delta, nslots, inst, key, delta_home(key, nslots));
+}
+
+// Insert (inst, key): from the home slot, the first slot that is empty (claimed by compare-and-swap
+// on the hash) or already holds the key takes the instance in its first free field.  A lookup
+// racing with the insert sees the key without this instance, which only under-reports; a duplicate
+// entry is harmless.  The table has twice as many slots as a window has chain blocks, so it cannot
+// fill; false reports a full table anyway.
+__device__ __forceinline__ bool delta_insert(DeltaSlot* delta, uint64_t nslots, uint32_t inst, uint64_t key) {
+  if (key == kEmpty || key == kTomb) return true;
+  const uint32_t tag = inst + 1;
+  uint64_t slot = delta_home(key, nslots);
+  for (uint64_t p = 0; p < nslots; ++p) {
+    const unsigned long long old = atomicCAS(&delta[slot].hash, kEmpty, (unsigned long long)key);
+    if (old == kEmpty || old == key) {
+      const unsigned int a = atomicCAS(&delta[slot].ia, 0u, tag);
+      if (a == 0u || a == tag) return true;
+      const unsigned int b = atomicCAS(&delta[slot].ib, 0u, tag);
+      if (b == 0u || b == tag) return true;
     }
-    b = (b + 1 == nbkt) ? 0u : b + 1;
+    slot = delta_next(slot, nslots);
   }
   return false;
 }
 
-// Insert (inst, key) into the delta table.  All concurrent inserts come from one greedy step and
-// target one instance.  The key is CAS-ed into the first free slot of its home bucket (the table is
-// sized at twice the window's blocks, so the first attempt nearly always succeeds), then the slot's
-// instance field is written.  A lookup that races with the insert sees either an empty slot or a
-// slot whose instance field is still 0, which matches no instance: it never reports a block that is
-// not in that instance's delta.  A duplicate (inst, key) entry is harmless for lookups.  Returns
-// false if the table is full.
-__device__ __forceinline__ bool delta_insert(DeltaSlot* delta, uint32_t nbkt, uint32_t inst, uint64_t key) {
-  if (key == kEmpty || key == kTomb) return true;
-  uint32_t b = delta_home(key, inst, nbkt);
-  for (uint32_t p = 0; p < nbkt; ++p) {
-    DeltaSlot* line = delta + (uint64_t)b * kDeltaSlots;
-    for (int k = 0; k < kDeltaSlots; ++k) {
-      const unsigned long long old = atomicCAS(&line[k].hash, kEmpty, (unsigned long long)key);
-      if (old == kEmpty) {
-        line[k].inst1 = inst + 1;
-        return true;
-      }
-    }
-    b = (b + 1 == nbkt) ? 0u : b + 1;
-  }
-  return false;
+// ------------------------------------------------------------------ cross-block signalling (sm_90+) --
+__device__ __forceinline__ uint32_t ld_acquire_u32(const uint32_t* p) {
+  uint32_t v;
+  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
 }
+
+__device__ __forceinline__ void st_release_u32(uint32_t* p, uint32_t v) {
+  asm volatile("st.release.gpu.global.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+
+__device__ __forceinline__ uint64_t globaltimer_ns() {
+  uint64_t x;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(x));
+  return x;
+}
+
+// 16-byte asynchronous global -> shared copy (completes at cp_async_wait_all of the same thread).
+__device__ __forceinline__ void cp_async16(void* smem, const void* gmem) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"((uint32_t)__cvta_generic_to_shared(smem)), "l"(gmem)
+               : "memory");
+}
+
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+
+__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_all;" ::: "memory"); }
 
 // ------------------------------------------------------------------------------- first-miss walks --
 // All 32 lanes of a warp call these with the same arguments; present(k) is evaluated per lane.
@@ -385,7 +461,12 @@ __device__ __forceinline__ uint64_t warp_first_miss_search_hint(uint64_t lo, uin
   const uint64_t new_hi = warp_min_u64(pr ? ~0ull : p);
   const uint64_t last_present = warp_max_u64(pr ? p + 1 : 0ull);
   const uint64_t hi = new_hi == ~0ull ? nb : new_hi;
-  const uint64_t lo2 = last_present > lo ? last_present : lo;
+  uint64_t lo2 = last_present > lo ? last_present : lo;
+  // A table read while inserts land need not look monotone: a present position may lie above an
+  // absent one.  Every present answer is cached in the final set and every absent answer is not
+  // cached in the set the inserts started from, so any point between them keeps the result between
+  // the two sets' first misses; clamping also keeps the remaining range well formed.
+  if (lo2 > hi) lo2 = hi;
   return warp_search_range(lo2, hi, present);
 }
 
@@ -570,7 +651,7 @@ __device__ __forceinline__ uint32_t pair_class(const DevModel& m, const RowConst
   return ok ? 0u : 1u;
 }
 
-// Ordering value inside a class.  Class 0 (Section 5.5, D-C-Q): more decoding requests, then more
+// Ordering value inside a class.  Class 0 (Section 6.2, D-C-Q): more decoding requests, then more
 // cached blocks, then fewer queued requests: (2^18-1-b) | (2^26-1-h) | qr in 18/26/18 bits.
 // Class 1 (CacheAwareLB = LMetric): (q + n) * (b + qr + 1) as an unsigned 64-bit product.
 __device__ __forceinline__ uint64_t pair_value(uint32_t cls, uint32_t h, int32_t b, int32_t qr, int64_t q,
@@ -626,9 +707,15 @@ cudaError_t launch_score(const uint32_t* hits, psk::StateSoA st, uint32_t I, con
 cudaError_t launch_greedy(const uint64_t* slots, const uint64_t* ovf, const psk::TableDesc* tdesc, uint32_t I,
                           const psk::WindowDev& w, const uint32_t* hit0, psk::StateSoA committed,
                           psk::StateSoA pending, const psk::DevModel& m, psk::DeltaSlot* delta,
-                          uint32_t delta_nbkt, int32_t* assign, uint8_t* path, uint32_t* hit_chosen,
+                          uint64_t delta_nslots, int32_t* assign, uint8_t* path, uint32_t* hit_chosen,
                           uint32_t* err, int search, cudaStream_t s);
 cudaError_t launch_delta_clear(psk::DeltaSlot* delta, uint64_t nslots, cudaStream_t s);
+cudaError_t launch_relations(const psk::WindowDev& w, const psk::DevModel& m, psk::LastSlot* tab, uint32_t tab_n,
+                             psk::RowPre* rows, int num_sms, cudaStream_t s);
+cudaError_t launch_greedy_search(const psk::RowPre* rows, const psk::WindowDev& w, uint32_t I, const uint32_t* hit0,
+                                 psk::StateSoA committed, psk::StateSoA pending, const psk::DevModel& m,
+                                 psk::DeltaSlot* delta, uint64_t delta_nslots, int32_t* assign, uint8_t* path,
+                                 uint32_t* hit_chosen, uint32_t* err, const psk::GreedySync& sync, cudaStream_t s);
 cudaError_t launch_insert_chains(uint64_t* slots, uint64_t* ovf, const psk::TableDesc* tdesc, uint32_t I,
                                  unsigned long long* count, uint64_t nchains, const uint32_t* inst,
                                  const uint64_t* off, const uint64_t* hash, const uint64_t* parent,

@@ -1,0 +1,132 @@
+// Per-request window constants for the greedy pass, computed for all requests in parallel.
+//
+// Besides the Algorithm 1 / Eq. 8 row constants (T_pf(0, L), CacheBenefit Z, eta * Z, the TTFT
+// budget), each request gets its chain relations to earlier requests of the same window:
+//   * lcp[d - 1]: the common chain prefix with the request d places before it (d = 1..4).  Chained
+//     block hashes (Section 7's prefix tree) make "block k equal" imply "blocks 0..k equal", so the
+//     common prefix is found with the 32-ary first-miss search.
+//   * par: the deepest earlier request whose whole chain is a prefix of this one (an agentic
+//     session's previous step, Section 3).  Its chain end is where this request's hit on the
+//     instance that took the parent most likely ends.
+// The greedy pass uses these only to place probes and to account for the four most recent
+// decisions; every hit it derives is still exact.
+#include <algorithm>
+
+#include "ps_internal.cuh"
+
+namespace {
+
+constexpr uint32_t kParentScan = 4096;  // chain positions scanned back from the end for a parent
+
+__device__ __forceinline__ uint32_t tab_home(uint64_t key, uint32_t n) {  // n is a power of two
+  return (uint32_t)((key * 0x9E3779B97F4A7C15ull) >> 32) & (n - 1);
+}
+
+// Table of last-block hashes: each key keeps the earliest request whose chain ends with it.
+__global__ void lastblock_build_kernel(psk::WindowDev w, psk::LastSlot* tab, uint32_t n) {
+  for (uint32_t r = blockIdx.x * blockDim.x + threadIdx.x; r < w.R; r += gridDim.x * blockDim.x) {
+    const uint64_t o = w.off[r], nb = w.off[r + 1] - o;
+    if (nb == 0) continue;
+    const unsigned long long key = w.hash[o + nb - 1];
+    if (key == psk::kEmpty || key == psk::kTomb) continue;
+    uint32_t b = tab_home(key, n);
+    for (uint32_t p = 0; p < n; ++p) {
+      const unsigned long long old = atomicCAS(&tab[b].key, (unsigned long long)psk::kEmpty, key);
+      if (old == psk::kEmpty || old == key) {
+        atomicMax(&tab[b].neg_idx, 0xFFFFFFFFu - r);
+        break;
+      }
+      b = (b + 1) & (n - 1);
+    }
+  }
+}
+
+__device__ __forceinline__ int32_t tab_find(const psk::LastSlot* tab, uint32_t n, uint64_t key) {
+  if (key == psk::kEmpty || key == psk::kTomb) return -1;
+  uint32_t b = tab_home(key, n);
+  for (uint32_t p = 0; p < n; ++p) {
+    const ulonglong2 v = __ldg(reinterpret_cast<const ulonglong2*>(tab + b));
+    if (v.x == key) return (int32_t)(0xFFFFFFFFu - (uint32_t)v.y);
+    if (v.x == psk::kEmpty) return -1;
+    b = (b + 1) & (n - 1);
+  }
+  return -1;
+}
+
+// One warp per request.
+__global__ void relations_kernel(psk::WindowDev w, psk::DevModel m, const psk::LastSlot* tab, uint32_t n,
+                                 psk::RowPre* rows) {
+  const int lane = threadIdx.x & 31;
+  const uint32_t wpb = blockDim.x >> 5;
+  for (uint32_t r = blockIdx.x * wpb + (threadIdx.x >> 5); r < w.R; r += gridDim.x * wpb) {
+    const uint64_t o = w.off[r];
+    const uint64_t nb = w.off[r + 1] - o;
+    const uint64_t* a = w.hash + o;
+    auto lcp_with = [&](uint32_t q) -> uint32_t {
+      const uint64_t oq = w.off[q];
+      const uint64_t nq = w.off[q + 1] - oq;
+      const uint64_t* bq = w.hash + oq;
+      return (uint32_t)psk::warp_search_range(0, nb < nq ? nb : nq, [&](uint64_t k) { return a[k] == bq[k]; });
+    };
+    uint32_t lcp[4];
+#pragma unroll
+    for (uint32_t d = 1; d <= 4; ++d) lcp[d - 1] = r >= d ? lcp_with(r - d) : 0u;
+    int32_t par = -1;
+    uint32_t par_nb = 0;
+    const uint64_t stop = nb > kParentScan ? nb - kParentScan : 0;
+    uint64_t top = nb;
+    while (top > stop && par < 0) {
+      const uint64_t lo = top - stop > 32 ? top - 32 : stop;  // positions [lo, top), lane 0 the deepest
+      const uint64_t k = top - 1 - (uint64_t)lane;
+      int32_t cand = -1;
+      if ((uint64_t)lane < top - lo) {
+        const int32_t q = tab_find(tab, n, a[k]);
+        if (q >= 0 && (uint32_t)q < r && w.off[q + 1] - w.off[q] == k + 1) cand = q;
+      }
+      const unsigned ok = __ballot_sync(0xffffffffu, cand >= 0);
+      if (ok) {
+        const int src = __ffs(ok) - 1;
+        par = __shfl_sync(0xffffffffu, cand, src);
+        par_nb = (uint32_t)(top - (uint64_t)src);
+      }
+      top = lo;
+    }
+    if (lane == 0) {
+      const psk::RowConst rc = psk::row_const(m, w.L[r], w.ttft_t[r], w.tpot_t[r]);
+      psk::RowPre x{};
+      x.off = o;
+      x.nb = (uint32_t)nb;
+      x.L = rc.L;
+      x.t_cached = rc.t_cached;
+      x.Z = rc.Z;
+      x.etaZ = rc.etaZ;
+      x.ttft_budget = rc.ttft_budget;
+      x.tpot_target = rc.tpot_target;
+#pragma unroll
+      for (int d = 0; d < 4; ++d) x.lcp[d] = lcp[d];
+      x.par = par;
+      x.par_nb = par_nb;
+      rows[r] = x;
+    }
+  }
+}
+
+}  // namespace
+
+namespace pskl {
+
+cudaError_t launch_relations(const psk::WindowDev& w, const psk::DevModel& m, psk::LastSlot* tab, uint32_t tab_n,
+                             psk::RowPre* rows, int num_sms, cudaStream_t s) {
+  if (w.R == 0) return cudaSuccess;
+  cudaError_t e = cudaMemsetAsync(tab, 0, (size_t)tab_n * sizeof(psk::LastSlot), s);
+  if (e != cudaSuccess) return e;
+  const int g1 = (int)std::min<uint64_t>((w.R + 255) / 256, (uint64_t)num_sms * 8);
+  lastblock_build_kernel<<<g1, 256, 0, s>>>(w, tab, tab_n);
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  const int g2 = (int)std::min<uint64_t>((w.R + 7) / 8, (uint64_t)num_sms * 8);
+  relations_kernel<<<g2, 256, 0, s>>>(w, m, tab, tab_n, rows);
+  return cudaGetLastError();
+}
+
+}  // namespace pskl

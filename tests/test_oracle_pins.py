@@ -1,10 +1,10 @@
 """Pins for the oracle: facts fixed by the paper or by mathematics, not by the oracle itself.
 
-  * hit length   -- brute-force token longest-common-prefix (Section 6 prefix tree) and the
+  * hit length   -- brute-force token longest-common-prefix (Section 7 prefix tree) and the
                     "longest fully cached prefix" definition on non-closed sets;
   * latencies    -- hand-worked literals (tests/golden/hand_example.json), closed forms under the
                     workload coefficients (Eq. 6: W = n(a1 + a2 L), Z = L(a1 + a2 L));
-  * filters      -- Section 5.4 special cases (eta = 0, Z = 0), Alg. 1 reject and fallback rules;
+  * filters      -- Section 6.1 special cases (eta = 0, Z = 0), Alg. 1 reject and fallback rules;
   * selection    -- D-C-Q order and LMetric fallback through the hand example, invariants;
   * greedy       -- hand-traced window, replay invariant.
 """
@@ -220,7 +220,7 @@ def _graded_oracle(model, I=6, **kw):
 
 
 def test_eta_zero_keeps_only_min_cost():
-    """Section 5.4: eta = 0 retains only the minimum-cost candidates."""
+    """Section 6.1: eta = 0 retains only the minimum-cost candidates."""
     o = _graded_oracle(dict(W.MODEL_DEFAULT, eta=0.0))
     out = o.score_rows(make_window([(seq_tokens("A", 1600), 3000.0, 50.0)]))
     assert out["cls"][0].tolist() == [2, 2, 2, 2, 2, 0]
@@ -234,7 +234,7 @@ def test_eta_large_keeps_all_of_A():
 
 
 def test_zero_cache_benefit_keeps_all_of_A():
-    """Section 5.4: if Z_r = 0 all capacity-eligible candidates remain (prefill cost flat)."""
+    """Section 6.1: if Z_r = 0 all capacity-eligible candidates remain (prefill cost flat)."""
     m = dict(W.MODEL_DEFAULT, a1=0.0, a2=0.0, a3=0.0, eta=0.0)
     o = _graded_oracle(m)
     out = o.score_rows(make_window([(seq_tokens("A", 1600), 3000.0, 50.0)]))
@@ -267,7 +267,7 @@ def test_fallback_when_T_empty_prefers_cache_under_equal_load():
 
 
 def test_decode_batch_dominates_cache_in_T():
-    """D before C (Section 5.5): a packed pick never has fewer decoding requests than any
+    """D before C (Section 6.2): a packed pick never has fewer decoding requests than any
     instance of T, and among equal decode batches never fewer cached blocks."""
     wl = W.generate(0)
     o = _oracle(wl.model, wl.instances)

@@ -8,7 +8,7 @@ Model coefficients are the synthetic white-box fits every configuration shares: 
 ``5 + 0.02*new + 1e-6*new*ctx`` ms with ``ctx = cached + new`` (paper Eq. 6 with
 alpha0=5, alpha1=0.02, alpha2=alpha3=1e-6), decode ``8 + 0.15*batch + 2e-5*kv_tokens`` ms (Eq. 7)
 and ``0.004`` ms of TPOT per queued prefill token.  eta = 0.5 is the paper's default recompute
-budget (Section 7.1 setup).
+budget (Section 8.1 setup).
 
 KV tokens held (S): config 0 uses the sum of the instance's cached session lengths, as that
 configuration states.  The larger configurations cache far more session tokens than an instance's
