@@ -226,6 +226,8 @@ def main():
     ap.add_argument("--cpu-seconds", type=float, default=20.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--probe-mode", type=int, default=1, choices=[0, 1])
+    ap.add_argument("--window-requests", type=int, default=None,
+                    help="smaller window of the same workload (profiler captures only; not a bench line)")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
@@ -244,6 +246,8 @@ def main():
     P.build()
     W.build()
     over = {} if args.tpot is None else {"tpot_target_ms": args.tpot}
+    if args.window_requests:
+        over["window_requests"] = args.window_requests
     seed = W.CONFIGS[args.config]["seed"] + rank
     wl = W.generate(args.config, seed=seed, **over)
     win, ins = wl.window, wl.instances
@@ -343,7 +347,8 @@ def main():
             "roofline": roof,
             "e2e": {"value": world * R * I / (e2e_ms / 1000), "unit": "scorings/s", "ms_per_step": e2e_ms,
                     "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
-            "gpu_launches": 5 * args.steps,
+            # per step: window validation, probe, score, last-block table, relations, greedy
+            "gpu_launches": (6 if args.probe_mode == 1 else 4) * args.steps,
             "clocks": clk.summary()}
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         import oracle
