@@ -260,7 +260,10 @@ ps_status run_probe_and_score(ps_ctx* c, const psk::WindowDev& wd, ps_scores* ou
   const int dev_out = out ? out->outputs_on_device : 0;
   uint32_t* hits = (out && out->hits && dev_out) ? out->hits : c->d_hits;
   record(c, kEvProbe0);
-  PS_TRY_CUDA(c, pskl::launch_probe(c->d_slots, c->d_ovf, c->d_tdesc, c->I, wd, hits, c->probe_grid, c->search, c->stream));
+  // window relations first: the probe derives the rows of requests that extend an earlier request
+  PS_TRY_CUDA(c, pskl::launch_relations(wd, c->model, c->d_lastslot, c->lastslot_n, c->d_rows, c->num_sms, c->stream));
+  PS_TRY_CUDA(c, pskl::launch_probe(c->d_slots, c->d_ovf, c->d_tdesc, c->I, wd, c->d_rows, hits, c->probe_grid,
+                                    c->search, c->stream));
   record(c, kEvProbe1);
   c->ev_used[0] = true;
   *hits_used = hits;
@@ -607,7 +610,6 @@ ps_status ps_schedule_window(ps_ctx* c, const ps_window* w, ps_decisions* out, p
   if (s != PS_OK) return s;
   record(c, kEvGreedy0);
   if (c->search) {
-    PS_TRY_CUDA(c, pskl::launch_relations(wd, c->model, c->d_lastslot, c->lastslot_n, c->d_rows, c->num_sms, c->stream));
     PS_TRY_CUDA(c, pskl::launch_greedy_search(c->d_rows, wd, c->I, hit0, c->st, c->pend, c->model, c->d_delta,
                                               c->delta_nslots, c->d_assign, c->d_dpath, c->d_hchosen, c->d_err,
                                               c->gsync, c->stream));

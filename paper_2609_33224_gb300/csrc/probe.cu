@@ -13,6 +13,13 @@
 //     lane binary-searches its own instance.  All instances of a row share the chain length, so the
 //     32 lanes of a warp run the same number of steps in lock-step with 32 independent lookups in
 //     flight, and a pair costs about log2(nb) probes.
+//
+// Rows whose chain starts with the whole chain of an earlier request of the window (its base, from
+// the relations pass) are derived in a second pass instead: the two chains agree block by block up
+// to the base's length nb_b, so on any cache hit(r, i) = hit(base, i) when that is below nb_b, and
+// otherwise the first miss lies in [nb_b, nb_r) with everything below known cached.  Only those
+// instances (the ones caching the base in full) are searched, by a warp each.  Agentic sessions
+// resend their history with each step (Section 3), so most rows of a window are derived.
 #include "ps_internal.cuh"
 
 namespace {
@@ -24,11 +31,12 @@ __global__ void __launch_bounds__(WARPS * 32)
 probe_hits_kernel(const uint64_t* __restrict__ slots, const uint64_t* __restrict__ ovf,
                   const psk::TableDesc* __restrict__ tdesc,
                   uint32_t I, const uint64_t* __restrict__ off, const uint64_t* __restrict__ hash,
-                  uint32_t R, uint32_t* __restrict__ hits) {
+                  uint32_t R, const psk::RowPre* __restrict__ rows, uint32_t* __restrict__ hits) {
   extern __shared__ uint64_t s_chain[];
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
   for (uint32_t r = blockIdx.x; r < R; r += gridDim.x) {
+    if (rows && __ldg(&rows[r].base) >= 0) continue;  // derived in the second pass
     const uint64_t o = off[r];
     const uint64_t nb = off[r + 1] - o;
     const uint64_t ns = nb < kStageBlocks ? nb : kStageBlocks;
@@ -57,6 +65,45 @@ probe_hits_kernel(const uint64_t* __restrict__ slots, const uint64_t* __restrict
   }
 }
 
+// Second pass: rows with a base.  One block per row; threads copy the base's hits and collect the
+// instances that cache the base in full, then warps search those past the base's end.
+template <int WARPS, bool SEARCH>
+__global__ void __launch_bounds__(WARPS * 32)
+probe_derived_kernel(const uint64_t* __restrict__ slots, const uint64_t* __restrict__ ovf,
+                     const psk::TableDesc* __restrict__ tdesc, uint32_t I, const uint64_t* __restrict__ hash,
+                     uint32_t R, const psk::RowPre* __restrict__ rows, uint32_t* __restrict__ hits) {
+  extern __shared__ uint32_t s_list[];  // I entries
+  __shared__ uint32_t s_n;
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  for (uint32_t r = blockIdx.x; r < R; r += gridDim.x) {
+    const int32_t b = __ldg(&rows[r].base);
+    if (b < 0) continue;  // block-uniform
+    if (threadIdx.x == 0) s_n = 0;
+    __syncthreads();
+    const uint64_t nbb = __ldg(&rows[b].nb);
+    const uint64_t nbr = __ldg(&rows[r].nb);
+    const uint64_t o = __ldg(&rows[r].off);
+    const uint32_t* hb_row = hits + (uint64_t)(uint32_t)b * I;
+    uint32_t* h_row = hits + (uint64_t)r * I;
+    for (uint32_t i = threadIdx.x; i < I; i += WARPS * 32) {
+      const uint32_t hb = hb_row[i];
+      if (hb < nbb || nbb >= nbr) h_row[i] = hb;
+      else s_list[atomicAdd(&s_n, 1u)] = i;
+    }
+    __syncthreads();
+    const uint32_t n = s_n;
+    for (uint32_t x = warp; x < n; x += WARPS) {
+      const uint32_t i = s_list[x];
+      const psk::TableDesc d = tdesc[i];
+      auto cached = [&](uint64_t k) { return psk::main_contains(slots, ovf, d, __ldg(hash + o + k)); };
+      const uint64_t h = SEARCH ? psk::warp_search_range(nbb, nbr, cached) : psk::warp_first_miss_linear(nbb, nbr, cached);
+      if (lane == 0) h_row[i] = (uint32_t)h;
+    }
+    __syncthreads();
+  }
+}
+
 template <int WARPS>
 int max_grid(int num_sms) {
   int per_sm = 0, per_sm2 = 0;
@@ -79,22 +126,27 @@ int probe_max_grid(uint32_t I, int num_sms) {
 }
 
 cudaError_t launch_probe(const uint64_t* slots, const uint64_t* ovf, const psk::TableDesc* tdesc, uint32_t I,
-                         const psk::WindowDev& w, uint32_t* hits, int grid, int search, cudaStream_t s) {
+                         const psk::WindowDev& w, const psk::RowPre* rows, uint32_t* hits, int grid, int search,
+                         cudaStream_t s) {
   if (w.R == 0) return cudaSuccess;
   const int g = (int)((uint32_t)grid < w.R ? (uint32_t)grid : w.R);
   const size_t smem = kStageBlocks * sizeof(uint64_t);
+  const size_t smem2 = (size_t)I * sizeof(uint32_t);
+#define PS_PROBE(W, S)                                                                                      \
+  do {                                                                                                      \
+    probe_hits_kernel<W, S><<<g, W * 32, smem, s>>>(slots, ovf, tdesc, I, w.off, w.hash, w.R, rows, hits);  \
+    cudaError_t e = cudaGetLastError();                                                                     \
+    if (e != cudaSuccess || !rows) return e;                                                                \
+    probe_derived_kernel<W, S><<<g, W * 32, smem2, s>>>(slots, ovf, tdesc, I, w.hash, w.R, rows, hits);     \
+    return cudaGetLastError();                                                                              \
+  } while (0)
   if (I >= 64) {
-    if (search)
-      probe_hits_kernel<8, true><<<g, 8 * 32, smem, s>>>(slots, ovf, tdesc, I, w.off, w.hash, w.R, hits);
-    else
-      probe_hits_kernel<8, false><<<g, 8 * 32, smem, s>>>(slots, ovf, tdesc, I, w.off, w.hash, w.R, hits);
-  } else {
-    if (search)
-      probe_hits_kernel<4, true><<<g, 4 * 32, smem, s>>>(slots, ovf, tdesc, I, w.off, w.hash, w.R, hits);
-    else
-      probe_hits_kernel<4, false><<<g, 4 * 32, smem, s>>>(slots, ovf, tdesc, I, w.off, w.hash, w.R, hits);
+    if (search) PS_PROBE(8, true);
+    PS_PROBE(8, false);
   }
-  return cudaGetLastError();
+  if (search) PS_PROBE(4, true);
+  PS_PROBE(4, false);
+#undef PS_PROBE
 }
 
 }  // namespace pskl

@@ -73,7 +73,7 @@ struct __align__(16) RowPre {
   uint32_t lcp[4];    // common chain prefix with requests r - 1 .. r - 4 (blocks)
   int32_t par;        // deepest earlier request whose chain is a prefix of r's, -1 if none
   uint32_t par_nb;    // its chain length
-  uint32_t pad;
+  int32_t base;       // the topmost request of r's parent links (r's chain starts with its chain), -1 if none
 };
 static_assert(sizeof(RowPre) == 64, "RowPre is one 64-byte record");
 
@@ -698,8 +698,10 @@ constexpr uint32_t kNoKeyCi = 0xFFFFFFFFu;  // class 15: worse than any real pai
 
 // Kernel launchers (one translation unit each).
 namespace pskl {
+// rows (from launch_relations, or nullptr to probe every request from scratch)
 cudaError_t launch_probe(const uint64_t* slots, const uint64_t* ovf, const psk::TableDesc* tdesc, uint32_t I,
-                         const psk::WindowDev& w, uint32_t* hits, int grid, int search, cudaStream_t s);
+                         const psk::WindowDev& w, const psk::RowPre* rows, uint32_t* hits, int grid, int search,
+                         cudaStream_t s);
 int probe_max_grid(uint32_t I, int num_sms);
 cudaError_t launch_score(const uint32_t* hits, psk::StateSoA st, uint32_t I, const psk::WindowDev& w,
                          const psk::DevModel& m, float* tpot, float* ttft, uint8_t* cls, int32_t* best,

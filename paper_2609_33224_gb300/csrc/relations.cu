@@ -6,10 +6,12 @@
 //     block hashes (Section 7's prefix tree) make "block k equal" imply "blocks 0..k equal", so the
 //     common prefix is found with the 32-ary first-miss search.
 //   * par: the deepest earlier request whose whole chain is a prefix of this one (an agentic
-//     session's previous step, Section 3).  Its chain end is where this request's hit on the
-//     instance that took the parent most likely ends.
-// The greedy pass uses these only to place probes and to account for the four most recent
-// decisions; every hit it derives is still exact.
+//     session's previous step, Section 3), checked block by block.  Its chain end is where this
+//     request's hit on the instance that took the parent most likely ends.
+//   * base: the topmost request reached through par links.  This request's chain starts with the
+//     base's whole chain, so on any cache its hit equals the base's hit unless the base is cached
+//     in full; the probe derives such rows from the base's row.
+// Every hit derived from these relations is exact: they only say which chain blocks are equal.
 #include <algorithm>
 
 #include "ps_internal.cuh"
@@ -83,11 +85,23 @@ __global__ void relations_kernel(psk::WindowDev w, psk::DevModel m, const psk::L
         const int32_t q = tab_find(tab, n, a[k]);
         if (q >= 0 && (uint32_t)q < r && w.off[q + 1] - w.off[q] == k + 1) cand = q;
       }
-      const unsigned ok = __ballot_sync(0xffffffffu, cand >= 0);
-      if (ok) {
+      unsigned ok = __ballot_sync(0xffffffffu, cand >= 0);
+      while (ok && par < 0) {
+        // deepest candidate first; it is the parent if its chain matches this one block by block
         const int src = __ffs(ok) - 1;
-        par = __shfl_sync(0xffffffffu, cand, src);
-        par_nb = (uint32_t)(top - (uint64_t)src);
+        const int32_t q = __shfl_sync(0xffffffffu, cand, src);
+        const uint64_t nq = top - (uint64_t)src;
+        const uint64_t* bq = w.hash + w.off[q];
+        bool same = true;
+        for (uint64_t k0 = 0; k0 < nq && same; k0 += 32) {
+          const uint64_t k = k0 + lane;
+          same = __all_sync(0xffffffffu, k >= nq || a[k] == bq[k]);
+        }
+        if (same) {
+          par = q;
+          par_nb = (uint32_t)nq;
+        }
+        ok &= ok - 1;
       }
       top = lo;
     }
@@ -106,8 +120,19 @@ __global__ void relations_kernel(psk::WindowDev w, psk::DevModel m, const psk::L
       for (int d = 0; d < 4; ++d) x.lcp[d] = lcp[d];
       x.par = par;
       x.par_nb = par_nb;
+      x.base = -1;
       rows[r] = x;
     }
+  }
+}
+
+// base of each request: follow the parent links to the top (parents come earlier, so it ends).
+__global__ void base_kernel(uint32_t R, psk::RowPre* rows) {
+  for (uint32_t r = blockIdx.x * blockDim.x + threadIdx.x; r < R; r += gridDim.x * blockDim.x) {
+    int32_t a = rows[r].par;
+    if (a >= 0)
+      for (int32_t p = rows[a].par; p >= 0; p = rows[a].par) a = p;
+    rows[r].base = a;
   }
 }
 
@@ -126,6 +151,9 @@ cudaError_t launch_relations(const psk::WindowDev& w, const psk::DevModel& m, ps
   if (e != cudaSuccess) return e;
   const int g2 = (int)std::min<uint64_t>((w.R + 7) / 8, (uint64_t)num_sms * 8);
   relations_kernel<<<g2, 256, 0, s>>>(w, m, tab, tab_n, rows);
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  base_kernel<<<g1, 256, 0, s>>>(w.R, rows);
   return cudaGetLastError();
 }
 
