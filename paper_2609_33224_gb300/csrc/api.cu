@@ -61,6 +61,7 @@ struct ps_ctx {
   float* d_ttft = nullptr;
   float* d_tpot = nullptr;
   uint32_t* d_hits = nullptr;
+  float* d_tpf = nullptr;  // T_pf at each pair's hit, from the probe, for the greedy pass
   float* d_tpot_o = nullptr;
   float* d_ttft_o = nullptr;
   uint8_t* d_cls = nullptr;
@@ -262,8 +263,8 @@ ps_status run_probe_and_score(ps_ctx* c, const psk::WindowDev& wd, ps_scores* ou
   record(c, kEvProbe0);
   // window relations first: the probe derives the rows of requests that extend an earlier request
   PS_TRY_CUDA(c, pskl::launch_relations(wd, c->model, c->d_lastslot, c->lastslot_n, c->d_rows, c->num_sms, c->stream));
-  PS_TRY_CUDA(c, pskl::launch_probe(c->d_slots, c->d_ovf, c->d_tdesc, c->I, wd, c->d_rows, hits, c->probe_grid,
-                                    c->search, c->stream));
+  PS_TRY_CUDA(c, pskl::launch_probe(c->d_slots, c->d_ovf, c->d_tdesc, c->I, wd, c->d_rows, hits, c->d_tpf,
+                                    c->model, c->probe_grid, c->search, c->stream));
   record(c, kEvProbe1);
   c->ev_used[0] = true;
   *hits_used = hits;
@@ -375,7 +376,7 @@ ps_status ps_create(const ps_config* cfg, ps_ctx** out) {
   ok = ok && dalloc(c, &c->d_off, (size_t)c->Rmax + 1) == cudaSuccess &&
        dalloc(c, &c->d_hash, c->max_blocks) == cudaSuccess && dalloc(c, &c->d_L, c->Rmax) == cudaSuccess &&
        dalloc(c, &c->d_ttft, c->Rmax) == cudaSuccess && dalloc(c, &c->d_tpot, c->Rmax) == cudaSuccess &&
-       dalloc(c, &c->d_hits, RI) == cudaSuccess && dalloc(c, &c->d_tpot_o, RI) == cudaSuccess &&
+       dalloc(c, &c->d_hits, RI) == cudaSuccess && dalloc(c, &c->d_tpf, RI) == cudaSuccess && dalloc(c, &c->d_tpot_o, RI) == cudaSuccess &&
        dalloc(c, &c->d_ttft_o, RI) == cudaSuccess && dalloc(c, &c->d_cls, RI) == cudaSuccess &&
        dalloc(c, &c->d_best, c->Rmax) == cudaSuccess && dalloc(c, &c->d_path, c->Rmax) == cudaSuccess &&
        dalloc(c, &c->d_assign, c->Rmax) == cudaSuccess && dalloc(c, &c->d_dpath, c->Rmax) == cudaSuccess &&
@@ -610,7 +611,7 @@ ps_status ps_schedule_window(ps_ctx* c, const ps_window* w, ps_decisions* out, p
   if (s != PS_OK) return s;
   record(c, kEvGreedy0);
   if (c->search) {
-    PS_TRY_CUDA(c, pskl::launch_greedy_search(c->d_rows, wd, c->I, hit0, c->st, c->pend, c->model, c->d_delta,
+    PS_TRY_CUDA(c, pskl::launch_greedy_search(c->d_rows, wd, c->I, hit0, c->d_tpf, c->st, c->pend, c->model, c->d_delta,
                                               c->delta_nslots, c->d_assign, c->d_dpath, c->d_hchosen, c->d_err,
                                               c->gsync, c->stream));
   } else {

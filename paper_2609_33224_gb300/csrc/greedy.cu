@@ -384,7 +384,7 @@ __device__ void insert_helper(const psk::RowPre* __restrict__ rows, const uint64
 template <int IPT>
 __global__ void __launch_bounds__(544, 1)
 greedy_search_kernel(const psk::RowPre* __restrict__ rows, const uint64_t* __restrict__ hash, uint32_t R, uint32_t I,
-                     const uint32_t* __restrict__ hit0, psk::StateSoA committed, psk::StateSoA pending,
+                     const uint32_t* __restrict__ hit0, const float* __restrict__ tpf0, psk::StateSoA committed, psk::StateSoA pending,
                      psk::DevModel m, psk::DeltaSlot* delta, uint64_t nslots, int32_t* assign,
                      uint8_t* __restrict__ path, uint32_t* __restrict__ hit_chosen, uint32_t* err,
                      psk::GreedySync sync) {
@@ -431,13 +431,16 @@ greedy_search_kernel(const psk::RowPre* __restrict__ rows, const uint64_t* __res
     s_touched[i] = 0;
     s_it[i] = psk::inst_terms(m, s_b[i], s_qr[i], s_q[i], s_Bmax[i]);
   }
-  if (t < 16) {
-    const uint32_t rr = (uint32_t)(t >> 2);
-    if (rr < R) reinterpret_cast<uint4*>(&s_row[rr])[t & 3] = __ldg(reinterpret_cast<const uint4*>(rows + rr) + (t & 3));
+  if (t < 20) {  // rows 0 .. 3, five 16-byte words each
+    const uint32_t rr = (uint32_t)(t / 5);
+    if (rr < R) reinterpret_cast<uint4*>(&s_row[rr])[t % 5] = __ldg(reinterpret_cast<const uint4*>(rows + rr) + (t % 5));
   }
   if (t < 2) s_nwalk[t] = 0;
 
+  // hit and T_pf at that hit of rows r .. r + 2 (T_pf from the probe; kNoTpfBits once the greedy
+  // changed the hit)
   uint32_t hr[IPT], h1[IPT], h2[IPT];
+  float tr[IPT], t1[IPT], t2[IPT];
   uint64_t key1[IPT];
   bool need1[IPT];
 #pragma unroll
@@ -446,11 +449,14 @@ greedy_search_kernel(const psk::RowPre* __restrict__ rows, const uint64_t* __res
     hr[k] = (i < I && R > 0) ? __ldg(hit0 + i) : 0u;
     h1[k] = (i < I && R > 1) ? __ldg(hit0 + (uint64_t)I + i) : 0u;
     h2[k] = (i < I && R > 2) ? __ldg(hit0 + 2ull * I + i) : 0u;
+    tr[k] = (i < I && R > 0) ? __ldg(tpf0 + i) : 0.0f;
+    t1[k] = (i < I && R > 1) ? __ldg(tpf0 + (uint64_t)I + i) : 0.0f;
+    t2[k] = (i < I && R > 2) ? __ldg(tpf0 + 2ull * I + i) : 0.0f;
     key1[k] = 0;
     need1[k] = false;
   }
   int32_t jm1 = -1, jm2 = -1, jm3 = -1, jm4 = -1;  // picks of requests r - 1 .. r - 4
-  int32_t jp_pre = -1;                             // pick of row r + 2's parent, loaded one step ahead
+  int32_t jp_pre[3] = {-1, -1, -1};  // picks of row r + 2's parent and two next ancestors, loaded a step ahead
   bool timed_out = false;
   __syncthreads();
 
@@ -458,41 +464,57 @@ greedy_search_kernel(const psk::RowPre* __restrict__ rows, const uint64_t* __res
     const psk::RowPre& cur = s_row[r & 7];
     const uint32_t nb = cur.nb;
     // ---- P0: ring refill, stages A-C, corrections and row evaluation -----------------------------
-    if (t < 4 && r + 4 < R) {
+    if (t < 5 && r + 4 < R) {
       psk::cp_async16(reinterpret_cast<uint4*>(&s_row[(r + 4) & 7]) + t, reinterpret_cast<const uint4*>(rows + r + 4) + t);
       psk::cp_async_commit();
     }
-    // the parent's pick for row r + 3 when it is old enough to be in global memory
-    int32_t jp_next = -1;
-    if (r + 3 < R) {
-      const int32_t par3 = s_row[(r + 3) & 7].par;
-      if (par3 >= 0 && (int64_t)par3 <= (int64_t)r - 4) jp_next = __ldcg(assign + par3);
+    // picks of row r + 3's ancestors when they are old enough to be in global memory (instance
+    // threads only: the signalling thread keeps no loads in flight)
+    int32_t jp_next[3] = {-1, -1, -1};
+    if (t < NTI && r + 3 < R) {
+      const psk::RowPre& x3 = s_row[(r + 3) & 7];
+      const int32_t a3[3] = {x3.par, x3.anc[0], x3.anc[1]};
+#pragma unroll
+      for (int q = 0; q < 3; ++q)
+        if (a3[q] >= 0 && (int64_t)a3[q] <= (int64_t)r - 4) jp_next[q] = __ldcg(assign + a3[q]);
     }
     uint32_t h3[IPT];
+    float t3[IPT];
 #pragma unroll
     for (int k = 0; k < IPT; ++k) {
       const uint32_t i = own(k);
       h3[k] = (i < I && r + 3 < R) ? __ldg(hit0 + (uint64_t)(r + 3) * I + i) : 0u;
+      t3[k] = (i < I && r + 3 < R) ? __ldg(tpf0 + (uint64_t)(r + 3) * I + i) : 0.0f;
     }
     uint64_t key2[IPT];
     bool need2[IPT];
     if (r + 2 < R) {
       const psk::RowPre& x2 = s_row[(r + 2) & 7];
-      // the parent counts only if its inserts are in every probe snapshot: par <= (r + 2) - kLag
-      const int64_t par = x2.par;
-      int32_t jp = -1;
-      if (par >= 0) {
-        if (par == (int64_t)r - 3) jp = jm3;
-        else if (par == (int64_t)r - 4) jp = jm4;
-        else if (par <= (int64_t)r - 5) jp = jp_pre;
+      // An ancestor's chain is a prefix of this one; on the instance that took it, the probe goes
+      // to its end.  It counts only if its inserts are in every probe snapshot: a <= (r + 2) - kLag.
+      const int32_t a2[3] = {x2.par, x2.anc[0], x2.anc[1]};
+      const uint32_t a2nb[3] = {x2.par_nb, x2.anc_nb[0], x2.anc_nb[1]};
+      int32_t jp[3];
+#pragma unroll
+      for (int q = 0; q < 3; ++q) {
+        const int64_t a = a2[q];
+        jp[q] = -1;
+        if (a >= 0) {
+          if (a == (int64_t)r - 3) jp[q] = jm3;
+          else if (a == (int64_t)r - 4) jp[q] = jm4;
+          else if (a <= (int64_t)r - 5) jp[q] = jp_pre[q];
+        }
       }
 #pragma unroll
       for (int k = 0; k < IPT; ++k) {
         const uint32_t i = own(k);
         uint32_t pos = h2[k];
-        if ((int32_t)i == jp && x2.par_nb > pos) pos = x2.par_nb;
+#pragma unroll
+        for (int q = 0; q < 3; ++q)
+          if ((int32_t)i == jp[q] && a2nb[q] > pos) pos = a2nb[q];
         need2[k] = i < I && s_touched[i] && pos < x2.nb;
         key2[k] = need2[k] ? __ldg(hash + x2.off + pos) : 0ull;
+        if (pos != h2[k]) t2[k] = __uint_as_float(psk::kNoTpfBits);
         h2[k] = pos;
       }
     } else {
@@ -531,8 +553,9 @@ greedy_search_kernel(const psk::RowPre* __restrict__ rows, const uint64_t* __res
         if ((int32_t)i == jm2 && cur.lcp[1] > h) h = cur.lcp[1];
         if ((int32_t)i == jm3 && cur.lcp[2] > h) h = cur.lcp[2];
         if ((int32_t)i == jm4 && cur.lcp[3] > h) h = cur.lcp[3];
+        const float tp = h == hr[k] ? tr[k] : __uint_as_float(psk::kNoTpfBits);
         hr[k] = h;
-        ev[k] = psk::eval_pair_terms(m, rc, h, s_it[i], s_q[i], s_S[i], s_M[i]);
+        ev[k] = psk::eval_pair_tpf(m, rc, h, tp, s_it[i], s_q[i], s_S[i], s_M[i]);
         if (ev[k].inA) {
           wmin = fminf(wmin, ev[k].W);
           anyA = true;
@@ -589,7 +612,7 @@ greedy_search_kernel(const psk::RowPre* __restrict__ rows, const uint64_t* __res
         }
       }
     }
-    if (t < 4) psk::cp_async_wait_all();
+    if (t < 5) psk::cp_async_wait_all();
     // Row r + 2's probes (issued in the next step) need every insert of requests <= r - 3.
     if (sig && r >= 3 && !timed_out) {
       const uint64_t t0 = psk::globaltimer_ns();
@@ -643,10 +666,16 @@ greedy_search_kernel(const psk::RowPre* __restrict__ rows, const uint64_t* __res
       __syncthreads();  // (E) search results visible to the owners
 #pragma unroll
       for (int k = 0; k < IPT; ++k)
-        if (walked[k]) h1[k] = s_wres[own(k)];
+        if (walked[k]) {
+          h1[k] = s_wres[own(k)];
+          t1[k] = __uint_as_float(psk::kNoTpfBits);
+        }
     }
 #pragma unroll
     for (int k = 0; k < IPT; ++k) {
+      tr[k] = t1[k];
+      t1[k] = t2[k];
+      t2[k] = t3[k];
       hr[k] = h1[k];
       h1[k] = h2[k];
       key1[k] = key2[k];
@@ -657,7 +686,8 @@ greedy_search_kernel(const psk::RowPre* __restrict__ rows, const uint64_t* __res
     jm3 = jm2;
     jm2 = jm1;
     jm1 = pick ? (int32_t)j : -1;
-    jp_pre = jp_next;
+#pragma unroll
+    for (int q = 0; q < 3; ++q) jp_pre[q] = jp_next[q];
   }
   for (uint32_t i = t; i < I; i += NT) {
     pending.b[i] = s_b[i];
@@ -675,7 +705,7 @@ size_t greedy_search_smem(uint32_t I) {
 
 template <int IPT>
 cudaError_t greedy_search_launch(const psk::RowPre* rows, const psk::WindowDev& w, uint32_t I, const uint32_t* hit0,
-                                 psk::StateSoA committed, psk::StateSoA pending, const psk::DevModel& m,
+                                 const float* tpf0, psk::StateSoA committed, psk::StateSoA pending, const psk::DevModel& m,
                                  psk::DeltaSlot* delta, uint64_t nslots, int32_t* assign, uint8_t* path,
                                  uint32_t* hit_chosen, uint32_t* err, const psk::GreedySync& sync, uint32_t nt,
                                  cudaStream_t s) {
@@ -687,7 +717,7 @@ cudaError_t greedy_search_launch(const psk::RowPre* rows, const psk::WindowDev& 
   psk::StateSoA c = committed, p = pending;
   psk::DevModel mm = m;
   psk::GreedySync sy = sync;
-  void* args[] = {(void*)&rows, (void*)&hash, (void*)&R, (void*)&I, (void*)&hit0, (void*)&c, (void*)&p,
+  void* args[] = {(void*)&rows, (void*)&hash, (void*)&R, (void*)&I, (void*)&hit0, (void*)&tpf0, (void*)&c, (void*)&p,
                   (void*)&mm, (void*)&delta, (void*)&nslots, (void*)&assign, (void*)&path, (void*)&hit_chosen,
                   (void*)&err, (void*)&sy};
   // all 1 + kHelpers blocks must be resident at once: they wait on one another
@@ -719,7 +749,7 @@ cudaError_t launch_greedy(const uint64_t* slots, const uint64_t* ovf, const psk:
 }
 
 cudaError_t launch_greedy_search(const psk::RowPre* rows, const psk::WindowDev& w, uint32_t I, const uint32_t* hit0,
-                                 psk::StateSoA committed, psk::StateSoA pending, const psk::DevModel& m,
+                                 const float* tpf0, psk::StateSoA committed, psk::StateSoA pending, const psk::DevModel& m,
                                  psk::DeltaSlot* delta, uint64_t delta_nslots, int32_t* assign, uint8_t* path,
                                  uint32_t* hit_chosen, uint32_t* err, const psk::GreedySync& sync, cudaStream_t s) {
   cudaError_t e = w.R ? cudaMemsetAsync(sync.done, 0, (size_t)w.R * sizeof(uint32_t), s) : cudaSuccess;
@@ -730,7 +760,7 @@ cudaError_t launch_greedy_search(const psk::RowPre* rows, const psk::WindowDev& 
   const uint32_t ipt = I <= 512 ? 1u : (I <= 1024 ? 2u : 4u);
   const uint32_t nt = ((I + ipt - 1) / ipt + 31) / 32 * 32 + 32;
 #define PS_GREEDY_S(IPT)                                                                                        \
-  return greedy_search_launch<IPT>(rows, w, I, hit0, committed, pending, m, delta, delta_nslots, assign, path,  \
+  return greedy_search_launch<IPT>(rows, w, I, hit0, tpf0, committed, pending, m, delta, delta_nslots, assign, path,  \
                                    hit_chosen, err, sync, nt, s)
   if (ipt == 1) PS_GREEDY_S(1);
   if (ipt == 2) PS_GREEDY_S(2);

@@ -26,12 +26,25 @@ namespace {
 
 constexpr uint32_t kStageBlocks = 4096;  // 32 KB of staged chain per thread block
 
+// Where a pair's result goes: its hit and, when requested, T_pf at that hit (the greedy pass reads
+// it instead of recomputing it for pairs whose hit does not change).
+struct PairOut {
+  uint32_t* hits;
+  float* tpf;
+  const uint32_t* L;
+  psk::DevModel m;
+  __device__ __forceinline__ void put(uint32_t r, uint32_t I, uint32_t i, uint32_t h, uint32_t Lr) const {
+    hits[(uint64_t)r * I + i] = h;
+    if (tpf) tpf[(uint64_t)r * I + i] = psk::t_pf_of_hit(m, Lr, h);
+  }
+};
+
 template <int WARPS, bool SEARCH>
 __global__ void __launch_bounds__(WARPS * 32)
 probe_hits_kernel(const uint64_t* __restrict__ slots, const uint64_t* __restrict__ ovf,
                   const psk::TableDesc* __restrict__ tdesc,
                   uint32_t I, const uint64_t* __restrict__ off, const uint64_t* __restrict__ hash,
-                  uint32_t R, const psk::RowPre* __restrict__ rows, uint32_t* __restrict__ hits) {
+                  uint32_t R, const psk::RowPre* __restrict__ rows, PairOut out) {
   extern __shared__ uint64_t s_chain[];
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -39,6 +52,7 @@ probe_hits_kernel(const uint64_t* __restrict__ slots, const uint64_t* __restrict
     if (rows && __ldg(&rows[r].base) >= 0) continue;  // derived in the second pass
     const uint64_t o = off[r];
     const uint64_t nb = off[r + 1] - o;
+    const uint32_t Lr = out.tpf ? __ldg(out.L + r) : 0u;
     const uint64_t ns = nb < kStageBlocks ? nb : kStageBlocks;
     for (uint64_t k = threadIdx.x; k < ns; k += WARPS * 32) s_chain[k] = __ldg(hash + o + k);
     __syncthreads();
@@ -51,14 +65,14 @@ probe_hits_kernel(const uint64_t* __restrict__ slots, const uint64_t* __restrict
           const uint64_t mid = (lo + hi) >> 1;
           if (psk::main_contains(slots, ovf, d, chain(mid))) lo = mid + 1; else hi = mid;
         }
-        hits[(uint64_t)r * I + i] = (uint32_t)lo;
+        out.put(r, I, i, (uint32_t)lo, Lr);
       }
     } else {
       for (uint32_t i = warp; i < I; i += WARPS) {
         const psk::TableDesc d = tdesc[i];
         auto cached = [&](uint64_t k) { return psk::main_contains(slots, ovf, d, chain(k)); };
         const uint64_t h = psk::warp_first_miss_linear(0, nb, cached);
-        if (lane == 0) hits[(uint64_t)r * I + i] = (uint32_t)h;
+        if (lane == 0) out.put(r, I, i, (uint32_t)h, Lr);
       }
     }
     __syncthreads();
@@ -71,7 +85,7 @@ template <int WARPS, bool SEARCH>
 __global__ void __launch_bounds__(WARPS * 32)
 probe_derived_kernel(const uint64_t* __restrict__ slots, const uint64_t* __restrict__ ovf,
                      const psk::TableDesc* __restrict__ tdesc, uint32_t I, const uint64_t* __restrict__ hash,
-                     uint32_t R, const psk::RowPre* __restrict__ rows, uint32_t* __restrict__ hits) {
+                     uint32_t R, const psk::RowPre* __restrict__ rows, PairOut out) {
   extern __shared__ uint32_t s_list[];  // I entries
   __shared__ uint32_t s_n;
   const int warp = threadIdx.x >> 5;
@@ -84,11 +98,11 @@ probe_derived_kernel(const uint64_t* __restrict__ slots, const uint64_t* __restr
     const uint64_t nbb = __ldg(&rows[b].nb);
     const uint64_t nbr = __ldg(&rows[r].nb);
     const uint64_t o = __ldg(&rows[r].off);
-    const uint32_t* hb_row = hits + (uint64_t)(uint32_t)b * I;
-    uint32_t* h_row = hits + (uint64_t)r * I;
+    const uint32_t Lr = __ldg(&rows[r].L);
+    const uint32_t* hb_row = out.hits + (uint64_t)(uint32_t)b * I;
     for (uint32_t i = threadIdx.x; i < I; i += WARPS * 32) {
       const uint32_t hb = hb_row[i];
-      if (hb < nbb || nbb >= nbr) h_row[i] = hb;
+      if (hb < nbb || nbb >= nbr) out.put(r, I, i, hb, Lr);
       else s_list[atomicAdd(&s_n, 1u)] = i;
     }
     __syncthreads();
@@ -98,7 +112,7 @@ probe_derived_kernel(const uint64_t* __restrict__ slots, const uint64_t* __restr
       const psk::TableDesc d = tdesc[i];
       auto cached = [&](uint64_t k) { return psk::main_contains(slots, ovf, d, __ldg(hash + o + k)); };
       const uint64_t h = SEARCH ? psk::warp_search_range(nbb, nbr, cached) : psk::warp_first_miss_linear(nbb, nbr, cached);
-      if (lane == 0) h_row[i] = (uint32_t)h;
+      if (lane == 0) out.put(r, I, i, (uint32_t)h, Lr);
     }
     __syncthreads();
   }
@@ -126,18 +140,19 @@ int probe_max_grid(uint32_t I, int num_sms) {
 }
 
 cudaError_t launch_probe(const uint64_t* slots, const uint64_t* ovf, const psk::TableDesc* tdesc, uint32_t I,
-                         const psk::WindowDev& w, const psk::RowPre* rows, uint32_t* hits, int grid, int search,
-                         cudaStream_t s) {
+                         const psk::WindowDev& w, const psk::RowPre* rows, uint32_t* hits, float* tpf,
+                         const psk::DevModel& m, int grid, int search, cudaStream_t s) {
   if (w.R == 0) return cudaSuccess;
+  const PairOut out{hits, tpf, w.L, m};
   const int g = (int)((uint32_t)grid < w.R ? (uint32_t)grid : w.R);
   const size_t smem = kStageBlocks * sizeof(uint64_t);
   const size_t smem2 = (size_t)I * sizeof(uint32_t);
 #define PS_PROBE(W, S)                                                                                      \
   do {                                                                                                      \
-    probe_hits_kernel<W, S><<<g, W * 32, smem, s>>>(slots, ovf, tdesc, I, w.off, w.hash, w.R, rows, hits);  \
+    probe_hits_kernel<W, S><<<g, W * 32, smem, s>>>(slots, ovf, tdesc, I, w.off, w.hash, w.R, rows, out);    \
     cudaError_t e = cudaGetLastError();                                                                     \
     if (e != cudaSuccess || !rows) return e;                                                                \
-    probe_derived_kernel<W, S><<<g, W * 32, smem2, s>>>(slots, ovf, tdesc, I, w.hash, w.R, rows, hits);     \
+    probe_derived_kernel<W, S><<<g, W * 32, smem2, s>>>(slots, ovf, tdesc, I, w.hash, w.R, rows, out);       \
     return cudaGetLastError();                                                                              \
   } while (0)
   if (I >= 64) {

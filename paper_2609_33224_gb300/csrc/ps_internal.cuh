@@ -50,11 +50,13 @@ struct TableDesc {
 };
 
 // One key of the window's delta table with up to two of the instances it was inserted for
-// (instance id + 1 in ia, then ib; 0 = free).  A key with more instances continues in a later slot.
+// (instance id + 1, filled in order; 0 = free).  A key with more instances continues in a later
+// slot.  (Four 16-bit fields would resolve more keys in one slot, but 16-bit compare-and-swap made
+// the inserts markedly slower.)
+constexpr int kDeltaTags = 2;
 struct DeltaSlot {
   unsigned long long hash;
-  unsigned int ia;
-  unsigned int ib;
+  unsigned int tag[kDeltaTags];
 };
 
 // Per-request constants of one window, computed in parallel before the greedy pass: the request's
@@ -74,8 +76,10 @@ struct __align__(16) RowPre {
   int32_t par;        // deepest earlier request whose chain is a prefix of r's, -1 if none
   uint32_t par_nb;    // its chain length
   int32_t base;       // the topmost request of r's parent links (r's chain starts with its chain), -1 if none
+  int32_t anc[2];     // the parent's parent and its parent (-1 if none): their chains are prefixes too
+  uint32_t anc_nb[2]; // their chain lengths
 };
-static_assert(sizeof(RowPre) == 64, "RowPre is one 64-byte record");
+static_assert(sizeof(RowPre) == 80, "RowPre is five 16-byte words");
 
 // Hand-off between the greedy block and the blocks that insert its picks' chains into the delta
 // table (one cooperative launch).
@@ -298,14 +302,19 @@ __device__ __forceinline__ uint64_t delta_next(uint64_t slot, uint64_t nslots) {
 
 // Verdict of one slot for (key, tag = inst + 1): 1 present, 0 absent, -1 look at the next slot.
 // Slots fill as an unbroken run from a key's home (inserts only claim empty slots and nothing is
-// removed while a window runs), instances fill ia then ib, and a key moves on to a later slot only
-// once both are taken; so an empty slot, or an entry of the key with a free instance field, ends
-// the search.
+// removed while a window runs), a key's instance fields fill in order, and a key moves on to a
+// later slot only once all its fields are taken; so an empty slot, or an entry of the key with a
+// free field, ends the search.
 __device__ __forceinline__ int delta_slot_verdict(const ulonglong2& v, uint64_t key, uint32_t tag) {
   if (v.x == key) {
-    const uint32_t ia = (uint32_t)v.y, ib = (uint32_t)(v.y >> 32);
-    if (ia == tag || ib == tag) return 1;
-    return (ia == 0u || ib == 0u) ? 0 : -1;
+    bool full = true;
+#pragma unroll
+    for (int f = 0; f < kDeltaTags; ++f) {
+      const uint32_t x = (uint32_t)(v.y >> (32 * f));
+      if (x == tag) return 1;
+      full = full && x != 0u;
+    }
+    return full ? -1 : 0;
   }
   return v.x == kEmpty ? 0 : -1;
 }
@@ -338,10 +347,11 @@ __device__ __forceinline__ bool delta_insert(DeltaSlot* delta, uint64_t nslots, 
   for (uint64_t p = 0; p < nslots; ++p) {
     const unsigned long long old = atomicCAS(&delta[slot].hash, kEmpty, (unsigned long long)key);
     if (old == kEmpty || old == key) {
-      const unsigned int a = atomicCAS(&delta[slot].ia, 0u, tag);
-      if (a == 0u || a == tag) return true;
-      const unsigned int b = atomicCAS(&delta[slot].ib, 0u, tag);
-      if (b == 0u || b == tag) return true;
+#pragma unroll
+      for (int f = 0; f < kDeltaTags; ++f) {
+        const unsigned int x = atomicCAS(&delta[slot].tag[f], 0u, tag);
+        if (x == 0 || x == tag) return true;
+      }
     }
     slot = delta_next(slot, nslots);
   }
@@ -616,13 +626,22 @@ __device__ __forceinline__ InstTerms inst_terms(const DevModel& m, int32_t b, in
   return x;
 }
 
-// eval_pair with the instance terms precomputed.
-__device__ __forceinline__ PairEval eval_pair_terms(const DevModel& m, const RowConst& rc, uint32_t h,
-                                                    const InstTerms& it, int64_t q, int64_t S, int64_t M) {
+// T_pf of a pair from its hit h: n = L - 16 h uncached tokens, c = 16 h cached.
+__device__ __forceinline__ float t_pf_of_hit(const DevModel& m, uint32_t L, uint32_t h) {
+  const int64_t c = 16 * (int64_t)h;
+  return t_pf(m, __ll2float_rn((int64_t)L - c), __ll2float_rn(c));
+}
+
+// Marks a precomputed T_pf as not available (a NaN pattern T_pf never produces).
+constexpr uint32_t kNoTpfBits = 0xFFFFFFFFu;
+
+// eval_pair with the instance terms precomputed, and T_pf given unless it carries kNoTpfBits.
+__device__ __forceinline__ PairEval eval_pair_tpf(const DevModel& m, const RowConst& rc, uint32_t h, float tpf_in,
+                                                  const InstTerms& it, int64_t q, int64_t S, int64_t M) {
   PairEval e;
   const int64_t c = 16 * (int64_t)h;
   const int64_t n = (int64_t)rc.L - c;
-  const float tpf = t_pf(m, __ll2float_rn(n), __ll2float_rn(c));
+  const float tpf = __float_as_uint(tpf_in) == kNoTpfBits ? t_pf(m, __ll2float_rn(n), __ll2float_rn(c)) : tpf_in;
   e.n = n;
   e.W = __fsub_rn(tpf, rc.t_cached);
   const int64_t Sp = S + (int64_t)rc.L;
@@ -638,6 +657,11 @@ __device__ __forceinline__ PairEval eval_pair_terms(const DevModel& m, const Row
   }
   e.ttft = __fadd_rn(tpf, it.tq);
   return e;
+}
+
+__device__ __forceinline__ PairEval eval_pair_terms(const DevModel& m, const RowConst& rc, uint32_t h,
+                                                    const InstTerms& it, int64_t q, int64_t S, int64_t M) {
+  return eval_pair_tpf(m, rc, h, __uint_as_float(kNoTpfBits), it, q, S, M);
 }
 
 // Class of a capacity-eligible pair once W_min is known (Eq. 8, Alg. 1 TPOT filter + TTFT budget):
@@ -698,10 +722,11 @@ constexpr uint32_t kNoKeyCi = 0xFFFFFFFFu;  // class 15: worse than any real pai
 
 // Kernel launchers (one translation unit each).
 namespace pskl {
-// rows (from launch_relations, or nullptr to probe every request from scratch)
+// rows (from launch_relations, or nullptr to probe every request from scratch); tpf (nullable)
+// receives T_pf of every pair's hit.
 cudaError_t launch_probe(const uint64_t* slots, const uint64_t* ovf, const psk::TableDesc* tdesc, uint32_t I,
-                         const psk::WindowDev& w, const psk::RowPre* rows, uint32_t* hits, int grid, int search,
-                         cudaStream_t s);
+                         const psk::WindowDev& w, const psk::RowPre* rows, uint32_t* hits, float* tpf,
+                         const psk::DevModel& m, int grid, int search, cudaStream_t s);
 int probe_max_grid(uint32_t I, int num_sms);
 cudaError_t launch_score(const uint32_t* hits, psk::StateSoA st, uint32_t I, const psk::WindowDev& w,
                          const psk::DevModel& m, float* tpot, float* ttft, uint8_t* cls, int32_t* best,
@@ -715,7 +740,7 @@ cudaError_t launch_delta_clear(psk::DeltaSlot* delta, uint64_t nslots, cudaStrea
 cudaError_t launch_relations(const psk::WindowDev& w, const psk::DevModel& m, psk::LastSlot* tab, uint32_t tab_n,
                              psk::RowPre* rows, int num_sms, cudaStream_t s);
 cudaError_t launch_greedy_search(const psk::RowPre* rows, const psk::WindowDev& w, uint32_t I, const uint32_t* hit0,
-                                 psk::StateSoA committed, psk::StateSoA pending, const psk::DevModel& m,
+                                 const float* tpf0, psk::StateSoA committed, psk::StateSoA pending, const psk::DevModel& m,
                                  psk::DeltaSlot* delta, uint64_t delta_nslots, int32_t* assign, uint8_t* path,
                                  uint32_t* hit_chosen, uint32_t* err, const psk::GreedySync& sync, cudaStream_t s);
 cudaError_t launch_insert_chains(uint64_t* slots, uint64_t* ovf, const psk::TableDesc* tdesc, uint32_t I,

@@ -8,6 +8,7 @@
 //   * par: the deepest earlier request whose whole chain is a prefix of this one (an agentic
 //     session's previous step, Section 3), checked block by block.  Its chain end is where this
 //     request's hit on the instance that took the parent most likely ends.
+//   * anc: the parent's parent and its parent, for the greedy's probe placement.
 //   * base: the topmost request reached through par links.  This request's chain starts with the
 //     base's whole chain, so on any cache its hit equals the base's hit unless the base is cached
 //     in full; the probe derives such rows from the base's row.
@@ -126,13 +127,27 @@ __global__ void relations_kernel(psk::WindowDev w, psk::DevModel m, const psk::L
   }
 }
 
-// base of each request: follow the parent links to the top (parents come earlier, so it ends).
+// base and the two next ancestors of each request: follow the parent links (parents come
+// earlier, so the walk ends).
 __global__ void base_kernel(uint32_t R, psk::RowPre* rows) {
   for (uint32_t r = blockIdx.x * blockDim.x + threadIdx.x; r < R; r += gridDim.x * blockDim.x) {
     int32_t a = rows[r].par;
-    if (a >= 0)
+    int32_t anc[2] = {-1, -1};
+    uint32_t anc_nb[2] = {0u, 0u};
+    if (a >= 0) {
+      anc[0] = rows[a].par;
+      if (anc[0] >= 0) {
+        anc_nb[0] = rows[a].par_nb;
+        anc[1] = rows[anc[0]].par;
+        if (anc[1] >= 0) anc_nb[1] = rows[anc[0]].par_nb;
+      }
       for (int32_t p = rows[a].par; p >= 0; p = rows[a].par) a = p;
+    }
     rows[r].base = a;
+    rows[r].anc[0] = anc[0];
+    rows[r].anc[1] = anc[1];
+    rows[r].anc_nb[0] = anc_nb[0];
+    rows[r].anc_nb[1] = anc_nb[1];
   }
 }
 
