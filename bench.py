@@ -112,34 +112,17 @@ class ClockSampler:
                 "samples": len(sm)}
 
 
-def search_probe_count(h: np.ndarray, nb: np.ndarray) -> np.ndarray:
-    """Probes the per-lane binary search makes for hit h on a chain of nb blocks: one per step of
-    lo, hi = 0, nb; while lo < hi: mid = (lo + hi) // 2; lo = mid + 1 if mid < h else hi = mid."""
-    h = h.astype(np.int64)
-    lo = np.zeros_like(h)
-    hi = np.broadcast_to(nb, h.shape).astype(np.int64).copy()
-    cnt = np.zeros_like(h)
-    while True:
-        live = lo < hi
-        if not live.any():
-            return cnt
-        mid = (lo + hi) >> 1
-        cnt += live
-        up = live & (mid < h)
-        lo = np.where(up, mid + 1, lo)
-        hi = np.where(live & ~up, mid, hi)
-
-
-def probe_algorithmic_bytes(hits: np.ndarray, nb: np.ndarray, search: bool) -> int:
-    """Bytes the probe kernel's algorithm must move per launch: one 32-byte sector per probed
-    position (linear walk: positions 0..h capped at the chain length; search: the search's own probe
-    count), the chain read once per request, the u32 hit written per pair."""
-    if search:
-        probes = int(sum(search_probe_count(hits[r0:r0 + 512], nb[r0:r0 + 512, None]).sum()
-                         for r0 in range(0, hits.shape[0], 512)))
-    else:
-        probes = int(np.minimum(hits.astype(np.int64) + 1, nb[:, None]).sum())
-    return int(32 * probes + 8 * nb.sum() + 4 * hits.size), probes
+def probe_algorithmic_bytes(st: dict, I: int, with_tpf: bool) -> tuple[int, int]:
+    """Bytes the two probe kernels' algorithm must move in one launch, from the library's own
+    counters of that launch (ps_last_probe_stats): one 32-byte sector per table lookup (the least a
+    random lookup can move), the staged chain blocks of the rows searched from scratch (8 B each),
+    the key of every lookup of a derived row (8 B, read from the chain), the earlier row's hits a
+    derived row starts from (4 B per instance), and per pair the u32 hit and, when the greedy pass
+    follows, the f32 T_pf written."""
+    out_b = (4 + (4 if with_tpf else 0)) * I
+    scratch = 32 * st["lookups_scratch"] + 8 * st["staged_blocks"] + out_b * st["rows_scratch"]
+    derived = (32 + 8) * st["lookups_derived"] + (4 * I + out_b) * st["rows_derived"]
+    return int(scratch + derived), int(st["lookups_scratch"] + st["lookups_derived"])
 
 
 def oracle_sample(wl, seconds: float, max_rows: int | None = None):
@@ -268,14 +251,14 @@ def main():
 
     for _ in range(args.warmup):
         step()
-    hits = sched.score_window(win, want=("hits",))["hits"]
-    probe_bytes, n_probes = probe_algorithmic_bytes(hits, nb, args.probe_mode == 1)
+    pstats = sched.probe_stats()  # the probe phase of the last schedule step (same window every step)
+    probe_bytes, n_probes = probe_algorithmic_bytes(pstats, I, with_tpf=args.probe_mode == 1)
     dist_on = world > 1
     if dist_on:
         import torch.distributed as dist
         dist.barrier()
     torch.cuda.synchronize()
-    kern = {"probe": [], "score": [], "greedy": []}
+    kern = {"probe": [], "score": [], "greedy": [], "relations": [], "probe_scratch": [], "probe_derived": []}
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     with ClockSampler(local) as clk:
         e0.record(stream)
@@ -317,12 +300,14 @@ def main():
     d2h = int(R * (4 + 1 + 4) + R * (4 + 1))
 
     km = {k: float(np.mean(v)) for k, v in kern.items()}
-    dominant = max(km, key=km.get)
+    phases = {k: km[k] for k in ("probe", "score", "greedy")}
+    dominant = max(phases, key=phases.get)
     peak, peak_src = _peaks()
+    probe_ms = km["probe_scratch"] + max(0.0, km["probe_derived"])
     if dominant == "probe":
-        achieved = probe_bytes / (km["probe"] / 1000) / 1e9
-        roof = {"bound": "hbm", "kernel": "probe_hits", "achieved": achieved, "peak": peak, "unit": "GB/s",
-                "frac": achieved / peak, "traffic": None, "peak_source": peak_src,
+        achieved = probe_bytes / (probe_ms / 1000) / 1e9
+        roof = {"bound": "hbm", "kernel": "probe_hits_kernel + probe_derived_kernel", "achieved": achieved,
+                "peak": peak, "unit": "GB/s", "frac": achieved / peak, "traffic": None, "peak_source": peak_src,
                 "algorithmic_bytes_per_launch": probe_bytes}
     else:
         greedy_bytes = int(4 * R * I + 24 * R + 16 * I * 6)
@@ -331,7 +316,7 @@ def main():
                 "unit": "GB/s", "frac": achieved / peak, "traffic": None, "peak_source": peak_src,
                 "algorithmic_bytes_per_launch": greedy_bytes,
                 "note": "serial per-request dependency chain: latency-bound, not bandwidth-bound"}
-    probe_achieved = probe_bytes / (km["probe"] / 1000) / 1e9
+    probe_achieved = probe_bytes / (probe_ms / 1000) / 1e9
     line = {"metric": METRIC, "value": world * R * I / (ms / 1000), "unit": "scorings/s", "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f32+u64", "data": "synthetic (seeded generator)",
@@ -342,8 +327,10 @@ def main():
                                  else "linear 32-wide warp walk"), "probes_per_window": n_probes,
                        "l2": "inputs larger than L2 (no flush)", "path_counts": path_counts},
             "kernel_ms": km,
-            "probe_roofline": {"achieved": probe_achieved, "peak": peak, "frac": probe_achieved / peak,
-                               "frac_vs_8tbs": probe_achieved / 8000.0},
+            "probe_roofline": {"kernels": "probe_hits_kernel + probe_derived_kernel", "achieved": probe_achieved,
+                               "unit": "GB/s", "peak": peak, "frac": probe_achieved / peak,
+                               "frac_vs_8tbs": probe_achieved / 8000.0, "ms": probe_ms,
+                               "algorithmic_bytes_per_launch": probe_bytes, "stats": pstats},
             "roofline": roof,
             "e2e": {"value": world * R * I / (e2e_ms / 1000), "unit": "scorings/s", "ms_per_step": e2e_ms,
                     "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},

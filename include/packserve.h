@@ -99,10 +99,13 @@ typedef struct {
  *                          not cached; exact for any cache contents.
  *     PS_PROBE_SEARCH  (1) the caches must be prefix-closed (every cached block's parent is
  *                          cached, as in the paper's Section 7 prefix tree).  Then "block k is
- *                          cached" is monotone along a chain and a warp finds the first miss by a
- *                          32-ary search (32 evenly spaced probes per step, at most 4 steps for
- *                          65536 blocks).  ps_insert_* checks the closure: a chain whose parent_hash
- *                          is neither 0 nor cached after the call fails with PS_ERR_INVALID.
+ *                          cached" is monotone along a chain, so the first miss is found by search:
+ *                          each lane binary-searches one instance (about log2(chain length)
+ *                          lookups per pair), and the continuation of a chain past an earlier
+ *                          request's end is found by a warp's 32-ary search (32 evenly spaced
+ *                          lookups per step).  ps_insert_* checks the closure: a chain whose
+ *                          parent_hash is neither 0 nor cached after the call fails with
+ *                          PS_ERR_INVALID.
  *   track_lru             1: keep per-block (last_use, child count, parent) metadata so that
  *                         ps_advance_window can evict leaf-first LRU; 0: no eviction.
  *   max_active_requests   0: no request tracking.  > 0: each instance keeps up to this many queued
@@ -289,9 +292,22 @@ typedef struct {
 PS_API ps_status ps_advance_window(ps_ctx* ctx, const ps_advance_params* p);
 
 /* Device time in ms (CUDA events recorded on the context's stream around each kernel) of the last
- * ps_score_window / ps_schedule_window call and of the commit after it: ms[0] probe, ms[1] fused
- * score, ms[2] greedy, ms[3] commit; -1 where that kernel did not run.  n must be >= 4. */
+ * ps_score_window / ps_schedule_window call and of the commit after it: ms[0] probe phase (relations
+ * + both probe kernels), ms[1] fused score, ms[2] greedy, ms[3] commit; with n >= 7 also the probe
+ * phase's parts: ms[4] relations kernel, ms[5] probe of the rows searched from scratch, ms[6] probe
+ * of the derived rows.  -1 where that kernel did not run.  n must be >= 4; entries past 7 are left
+ * untouched. */
 PS_API ps_status ps_last_timings(ps_ctx* ctx, float* ms, uint32_t n);
+
+/* Counters of the last probe phase (ps_score_window / ps_schedule_window), for roofline accounting
+ * (host array of n >= 6 entries):
+ *   out[0] rows searched from scratch        out[1] rows derived from an earlier request's row
+ *   out[2] table lookups in scratch rows     out[3] table lookups in derived rows
+ *   out[4] chain blocks staged in shared memory (scratch rows)
+ *   out[5] (row, instance) pairs searched past the earlier request's chain (derived rows)
+ * A table lookup reads the key's two candidate buckets (2 x 64 bytes) and one overflow word.
+ * All zero if no probe phase ran.  Synchronises the context's stream. */
+PS_API ps_status ps_last_probe_stats(ps_ctx* ctx, uint64_t* out, uint32_t n);
 
 /* ---- Scoring without device allocation ------------------------------------------------------
  * The paper has no counterpart to this call; it exists for callers that cannot allocate device

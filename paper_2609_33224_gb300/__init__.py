@@ -24,7 +24,7 @@ STATUS_NAMES = {0: "PS_OK", 1: "PS_ERR_INVALID", 2: "PS_ERR_CUDA", 3: "PS_ERR_OO
 
 ABI_FUNCTIONS = ("ps_create", "ps_load_instances", "ps_get_instances", "ps_get_pending_instances",
                  "ps_insert_blocks", "ps_insert_chains", "ps_cached_blocks", "ps_score_window",
-                 "ps_schedule_window", "ps_commit_window", "ps_last_timings", "ps_last_error",
+                 "ps_schedule_window", "ps_commit_window", "ps_last_timings", "ps_last_probe_stats", "ps_last_error",
                  "ps_destroy", "ps_score_window_noalloc", "ps_load_requests", "ps_advance_window")
 
 
@@ -113,6 +113,7 @@ def lib() -> ctypes.CDLL:
                                    ctypes.POINTER(PsScores)],
             "ps_commit_window": [vp, u32],
             "ps_last_timings": [vp, vp, u32],
+            "ps_last_probe_stats": [vp, vp, u32],
             "ps_load_requests": [vp, u64, vp, vp, vp, vp, vp],
             "ps_advance_window": [vp, ctypes.POINTER(PsAdvanceParams)],
             "ps_score_window_noalloc": [vp, vp, vp, u32, ctypes.POINTER(PsStateArrays), ctypes.POINTER(PsWindow),
@@ -285,9 +286,20 @@ class Scheduler:
         self._check(lib().ps_advance_window(self._h, ctypes.byref(p)))
 
     def timings(self) -> dict:
-        ms = np.zeros(4, np.float32)
-        self._check(lib().ps_last_timings(self._h, ms.ctypes.data, 4))
-        return dict(zip(("probe", "score", "greedy", "commit"), (float(x) for x in ms)))
+        """Device ms of the last call's kernels: probe phase, score, greedy, commit, and the probe
+        phase's parts (relations, probe_scratch, probe_derived); -1 where a kernel did not run."""
+        ms = np.zeros(7, np.float32)
+        self._check(lib().ps_last_timings(self._h, ms.ctypes.data, 7))
+        names = ("probe", "score", "greedy", "commit", "relations", "probe_scratch", "probe_derived")
+        return dict(zip(names, (float(x) for x in ms)))
+
+    def probe_stats(self) -> dict:
+        """Counters of the last probe phase (see ps_last_probe_stats)."""
+        v = np.zeros(6, np.uint64)
+        self._check(lib().ps_last_probe_stats(self._h, v.ctypes.data, 6))
+        names = ("rows_scratch", "rows_derived", "lookups_scratch", "lookups_derived", "staged_blocks",
+                 "pairs_derived")
+        return dict(zip(names, (int(x) for x in v)))
 
     # ------------------------------------------------------------------------------------------
     @staticmethod

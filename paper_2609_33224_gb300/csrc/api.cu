@@ -16,7 +16,12 @@
 
 namespace {
 
-enum Ev { kEvProbe0, kEvProbe1, kEvScore0, kEvScore1, kEvGreedy0, kEvGreedy1, kEvCommit0, kEvCommit1, kNumEv };
+// Events on the context's stream: four timed phases (start/end pairs), then the two split points of
+// the probe phase (after the relations kernel, between the two probe kernels).
+enum Ev { kEvProbe0, kEvProbe1, kEvScore0, kEvScore1, kEvGreedy0, kEvGreedy1, kEvCommit0, kEvCommit1, kEvRelDone,
+          kEvProbeMid, kNumEv };
+constexpr int kNumPhases = 4;
+constexpr int kNumStats = 6;
 
 struct DeviceGuard {
   int prev = -1;
@@ -73,7 +78,9 @@ struct ps_ctx {
   uint32_t* d_err = nullptr;
   uint32_t* h_err = nullptr;
   cudaEvent_t ev[kNumEv] = {};
-  bool ev_used[kNumEv / 2] = {};
+  bool ev_used[kNumPhases] = {};
+  bool probe_split = false;            // kEvRelDone / kEvProbeMid recorded in the last probe phase
+  unsigned long long* d_stats = nullptr;  // probe launch counters (ps_last_probe_stats)
   bool pending = false;
   psk::WindowDev pend_win{};
   const uint32_t* pend_out = nullptr;
@@ -260,13 +267,16 @@ void record(ps_ctx* c, int ev) { cudaEventRecord(c->ev[ev], c->stream); }
 ps_status run_probe_and_score(ps_ctx* c, const psk::WindowDev& wd, ps_scores* out, uint32_t** hits_used) {
   const int dev_out = out ? out->outputs_on_device : 0;
   uint32_t* hits = (out && out->hits && dev_out) ? out->hits : c->d_hits;
+  PS_TRY_CUDA(c, cudaMemsetAsync(c->d_stats, 0, kNumStats * sizeof(unsigned long long), c->stream));
   record(c, kEvProbe0);
   // window relations first: the probe derives the rows of requests that extend an earlier request
   PS_TRY_CUDA(c, pskl::launch_relations(wd, c->model, c->d_lastslot, c->lastslot_n, c->d_rows, c->num_sms, c->stream));
+  record(c, kEvRelDone);
   PS_TRY_CUDA(c, pskl::launch_probe(c->d_slots, c->d_ovf, c->d_tdesc, c->I, wd, c->d_rows, hits, c->d_tpf,
-                                    c->model, c->probe_grid, c->search, c->stream));
+                                    c->model, c->probe_grid, c->search, c->d_stats, c->ev[kEvProbeMid], c->stream));
   record(c, kEvProbe1);
   c->ev_used[0] = true;
+  c->probe_split = wd.R > 0;
   *hits_used = hits;
   if (!out) return PS_OK;
   const size_t RI = (size_t)wd.R * c->I;
@@ -296,6 +306,7 @@ ps_status run_probe_and_score(ps_ctx* c, const psk::WindowDev& wd, ps_scores* ou
 
 void reset_timers(ps_ctx* c) {
   for (bool& u : c->ev_used) u = false;
+  c->probe_split = false;
 }
 
 }  // namespace
@@ -381,6 +392,7 @@ ps_status ps_create(const ps_config* cfg, ps_ctx** out) {
        dalloc(c, &c->d_best, c->Rmax) == cudaSuccess && dalloc(c, &c->d_path, c->Rmax) == cudaSuccess &&
        dalloc(c, &c->d_assign, c->Rmax) == cudaSuccess && dalloc(c, &c->d_dpath, c->Rmax) == cudaSuccess &&
        dalloc(c, &c->d_hchosen, c->Rmax) == cudaSuccess && dalloc(c, &c->d_err, 1) == cudaSuccess &&
+       dalloc(c, &c->d_stats, kNumStats) == cudaSuccess &&
        dalloc(c, &c->d_cap, I) == cudaSuccess && dalloc(c, &c->d_outtok, c->Rmax) == cudaSuccess;
   if (ok && c->lru)
     ok = dalloc(c, &c->meta.last_use, c->total_slots) == cudaSuccess &&
@@ -409,7 +421,8 @@ ps_status ps_create(const ps_config* cfg, ps_ctx** out) {
              cudaMemsetAsync(c->d_count, 0, I * sizeof(unsigned long long), c->stream) == cudaSuccess &&
              cudaMemsetAsync(c->d_delta, 0, (size_t)dn * sizeof(psk::DeltaSlot), c->stream) ==
                  cudaSuccess &&
-             cudaMemsetAsync(c->d_err, 0, sizeof(uint32_t), c->stream) == cudaSuccess;
+             cudaMemsetAsync(c->d_err, 0, sizeof(uint32_t), c->stream) == cudaSuccess &&
+             cudaMemsetAsync(c->d_stats, 0, kNumStats * sizeof(unsigned long long), c->stream) == cudaSuccess;
   for (psk::StateSoA* s : {&c->st, &c->pend}) {
     set = set && cudaMemsetAsync(s->b, 0, I * 4, c->stream) == cudaSuccess &&
           cudaMemsetAsync(s->qr, 0, I * 4, c->stream) == cudaSuccess &&
@@ -724,13 +737,27 @@ ps_status ps_last_timings(ps_ctx* c, float* ms, uint32_t n) {
   if (!c) return PS_ERR_INVALID;
   if (!ms || n < 4) return fail(c, PS_ERR_INVALID, "need 4 entries");
   DeviceGuard g(c->device);
-  for (int k = 0; k < 4; ++k) {
-    ms[k] = -1.0f;
-    if (c->ev_used[k]) {
-      float t = 0.0f;
-      if (cudaEventElapsedTime(&t, c->ev[2 * k], c->ev[2 * k + 1]) == cudaSuccess) ms[k] = t;
-    }
+  auto span = [&](int a, int b) {
+    float t = 0.0f;
+    return cudaEventElapsedTime(&t, c->ev[a], c->ev[b]) == cudaSuccess ? t : -1.0f;
+  };
+  for (int k = 0; k < kNumPhases; ++k) ms[k] = c->ev_used[k] ? span(2 * k, 2 * k + 1) : -1.0f;
+  const int split[3][2] = {{kEvProbe0, kEvRelDone}, {kEvRelDone, kEvProbeMid}, {kEvProbeMid, kEvProbe1}};
+  for (uint32_t k = 0; k < 3 && 4 + k < n; ++k)
+    ms[4 + k] = (c->ev_used[0] && c->probe_split) ? span(split[k][0], split[k][1]) : -1.0f;
+  return PS_OK;
+}
+
+ps_status ps_last_probe_stats(ps_ctx* c, uint64_t* out, uint32_t n) {
+  if (!c) return PS_ERR_INVALID;
+  if (!out || n < (uint32_t)kNumStats) return fail(c, PS_ERR_INVALID, "need 6 entries");
+  DeviceGuard g(c->device);
+  unsigned long long v[kNumStats] = {};
+  if (c->ev_used[0]) {
+    PS_TRY_CUDA(c, cudaMemcpyAsync(v, c->d_stats, sizeof(v), cudaMemcpyDeviceToHost, c->stream));
+    PS_TRY_CUDA(c, cudaStreamSynchronize(c->stream));
   }
+  for (int k = 0; k < kNumStats; ++k) out[k] = v[k];
   return PS_OK;
 }
 

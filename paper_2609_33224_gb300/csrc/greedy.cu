@@ -1,7 +1,7 @@
 // Greedy in-window assignment (Algorithm 1 applied to the window's requests in arrival order).
 //
 // The paper's gateway decides each request online and updates the instance records along the
-// request path before the next decision (Section 4, Metadata service; Section 6).  This kernel
+// request path before the next decision (Section 4, Metadata service; Section 7).  This kernel
 // replays that sequence for a whole window on the GPU: one persistent thread block whose threads
 // each own up to IPT instances.  Per request r:
 //   1. hit of r on instance i = hit0[r][i] (the probe kernel's result on the committed tables)
@@ -277,30 +277,31 @@ cudaError_t greedy_launch(const uint64_t* slots, const uint64_t* ovf, const psk:
 // union of prefix-closed sets has as first miss the largest of the sets' first misses.  The
 // cached set of instance i while request s is decided is main_i plus the chains of the window's
 // earlier requests assigned to i, so
-//     hit(s, i) = max( first miss of main_i + delta_i(<= s - 5),
-//                      lcp(s, s - d) for each d = 1..4 such that request s - d went to i )
-// where delta_i(<= s - 5) holds the blocks inserted for requests up to s - 5 and lcp(s, s - d) is
+//     hit(s, i) = max( first miss of main_i + delta_i(<= s - kLag),
+//                      lcp(s, s - d) for each d = 1..kLag-1 such that request s - d went to i )
+// where delta_i(<= s - kLag) holds the blocks inserted for requests up to s - kLag and lcp(s, s - d) is
 // the common chain prefix (from the relations pass).  The first term is probed ahead of time, while
 // earlier requests are still being decided, so no table access is on the per-request critical
 // path.  The probe position is hit0, raised to the end of the request's parent (the deepest earlier
 // request whose chain is a prefix of this one) on the instance that took the parent; a probe that
 // finds the block cached hands the instance to a warp search.  Probes may also see inserts of
-// requests s - 4 .. s - 1 (they land while the probe runs): any snapshot between delta(<= s - 5)
-// and delta(<= s - 1) gives a first miss between the two, and the max with the lcp terms is then
-// exact all the same.
+// requests s - kLag + 1 .. s - 1 (they land while the probe runs, in any order): any snapshot
+// between delta(<= s - kLag) and delta(<= s - 1) gives a first miss between the two, and the max
+// with the lcp terms is then exact all the same.
 //
 // Block 0 decides.  Per step r it evaluates row r (two block reductions: W_min, then the argmin)
 // and besides:  loads hit0 of row r + 3;  places row r + 2's probe and loads the chain block there
 // (instances with window inserts only);  issues row r + 1's probe (consumed after the first
-// barrier);  publishes request r's pick as an insert job.  Blocks 1..kHelpers insert each job's
-// chain blocks chain[h, nb) into delta_j and count themselves done; block 0 waits (bounded) for job
-// r - 3 before its row r + 2 probes go out; a dedicated signalling thread (the block's last warp
+// barrier);  publishes request r's pick as an insert job.  Blocks 1..kHelpers take the jobs
+// round-robin (up to kHelpers jobs in flight), insert each job's chain blocks chain[h, nb) into
+// delta_j and release the job's done flag; block 0 waits (bounded) for job r - (kLag - 2) before its
+// row r + 2 probes go out; a dedicated signalling thread (the block's last warp
 // owns no instances) publishes the jobs and does that wait, so the release and acquire orderings
 // never hold up a thread with loads in flight.  Instance state lives in shared memory and is
 // written only by the thread that owns the instance.
 
 constexpr uint32_t kHelpers = 8;              // insert blocks beside the deciding block
-constexpr uint32_t kLag = 5;                  // a probe for row s sees every insert of requests <= s - kLag
+constexpr uint32_t kRingAhead = 6;            // row constants are copied into the ring this many rows ahead
 constexpr uint64_t kWaitNs = 1000000000ull;   // bound on any cross-block wait
 constexpr unsigned long long kAbortJob = ~0ull;
 
@@ -337,14 +338,13 @@ __device__ __forceinline__ psk::RowConst row_of(const psk::RowPre& x) {
   return rc;
 }
 
-// Blocks 1..kHelpers: insert every published pick's chain tail, in request order.
+// Blocks 1..kHelpers: block b inserts the chain tails of jobs b - 1, b - 1 + kHelpers, ... and
+// releases each job's done flag once all its blocks are in.
 __device__ void insert_helper(const psk::RowPre* __restrict__ rows, const uint64_t* __restrict__ hash, uint32_t R,
                               psk::DeltaSlot* delta, uint64_t nslots, uint32_t* err, const psk::GreedySync& sync) {
   __shared__ unsigned long long s_job;
   const uint32_t t = threadIdx.x;
-  const uint64_t stride = (uint64_t)kHelpers * blockDim.x;
-  const uint64_t first = (uint64_t)(blockIdx.x - 1) * blockDim.x + t;
-  for (uint32_t job = 0; job < R; ++job) {
+  for (uint32_t job = blockIdx.x - 1; job < R; job += kHelpers) {
     if (t == 0) {
       const uint64_t t0 = psk::globaltimer_ns();
       unsigned long long jb = kAbortJob;
@@ -357,7 +357,7 @@ __device__ void insert_helper(const psk::RowPre* __restrict__ rows, const uint64
           atomicOr(err, psk::kErrTimeout);
           break;
         }
-        __nanosleep(100);
+        __nanosleep(32);
       }
       s_job = jb;
     }
@@ -367,16 +367,16 @@ __device__ void insert_helper(const psk::RowPre* __restrict__ rows, const uint64
     const uint32_t j = (uint32_t)jb;
     const uint32_t hj = (uint32_t)(jb >> 32);
     // rows >= job + kLag are the only ones that read this job's inserts
-    if (j != 0xFFFFFFFFu && job + kLag < R) {
+    if (j != 0xFFFFFFFFu && job + psk::kLag < R) {
       const uint64_t off = __ldg(&rows[job].off);
       const uint32_t nb = __ldg(&rows[job].nb);
-      for (uint64_t p = hj + first; p < nb; p += stride)
+      for (uint64_t p = hj + t; p < nb; p += blockDim.x)
         if (!psk::delta_insert(delta, nslots, j, __ldg(hash + off + p))) atomicOr(err, psk::kErrDeltaFull);
     }
     __syncthreads();
     if (t == 0) {
-      __threadfence();  // release every thread's inserts before the count
-      atomicAdd(sync.done + job, 1u);
+      __threadfence();  // every thread's inserts before the flag
+      psk::st_release_u32(sync.done + job, 1u);
     }
   }
 }
@@ -404,7 +404,7 @@ greedy_search_kernel(const psk::RowPre* __restrict__ rows, const uint64_t* __res
   uint32_t* s_walk = s_wres + I;                               // instances handed to a warp search
   psk::InstTerms* s_it = reinterpret_cast<psk::InstTerms*>(s_walk + I);
   uint8_t* s_touched = reinterpret_cast<uint8_t*>(s_it + I);
-  __shared__ psk::RowPre s_row[8];  // rows r .. r + 4 (a ring of 8 so no reader is overtaken)
+  __shared__ psk::RowPre s_row[8];  // rows r .. r + kRingAhead (a ring of 8 so no reader is overtaken)
   __shared__ float s_red_w[32];
   __shared__ int s_red_a[32];
   __shared__ PickKey s_red_k[32];
@@ -431,9 +431,11 @@ greedy_search_kernel(const psk::RowPre* __restrict__ rows, const uint64_t* __res
     s_touched[i] = 0;
     s_it[i] = psk::inst_terms(m, s_b[i], s_qr[i], s_q[i], s_Bmax[i]);
   }
-  if (t < 20) {  // rows 0 .. 3, five 16-byte words each
-    const uint32_t rr = (uint32_t)(t / 5);
-    if (rr < R) reinterpret_cast<uint4*>(&s_row[rr])[t % 5] = __ldg(reinterpret_cast<const uint4*>(rows + rr) + (t % 5));
+  if (t < kRingAhead * psk::kRowWords) {  // rows 0 .. kRingAhead - 1
+    const uint32_t rr = (uint32_t)(t / psk::kRowWords);
+    if (rr < R)
+      reinterpret_cast<uint4*>(&s_row[rr])[t % psk::kRowWords] =
+          __ldg(reinterpret_cast<const uint4*>(rows + rr) + (t % psk::kRowWords));
   }
   if (t < 2) s_nwalk[t] = 0;
 
@@ -455,7 +457,9 @@ greedy_search_kernel(const psk::RowPre* __restrict__ rows, const uint64_t* __res
     key1[k] = 0;
     need1[k] = false;
   }
-  int32_t jm1 = -1, jm2 = -1, jm3 = -1, jm4 = -1;  // picks of requests r - 1 .. r - 4
+  int32_t jm[psk::kLcpBack];  // jm[d] = pick of request r - 1 - d
+#pragma unroll
+  for (int d = 0; d < psk::kLcpBack; ++d) jm[d] = -1;
   int32_t jp_pre[3] = {-1, -1, -1};  // picks of row r + 2's parent and two next ancestors, loaded a step ahead
   bool timed_out = false;
   __syncthreads();
@@ -464,10 +468,18 @@ greedy_search_kernel(const psk::RowPre* __restrict__ rows, const uint64_t* __res
     const psk::RowPre& cur = s_row[r & 7];
     const uint32_t nb = cur.nb;
     // ---- P0: ring refill, stages A-C, corrections and row evaluation -----------------------------
-    if (t < 5 && r + 4 < R) {
-      psk::cp_async16(reinterpret_cast<uint4*>(&s_row[(r + 4) & 7]) + t, reinterpret_cast<const uint4*>(rows + r + 4) + t);
+    // Refill the ring kRingAhead rows ahead: one copy group per step (empty past the window's end),
+    // waited for two steps later, so the copy's latency stays off the step.
+    if (t < psk::kRowWords) {
+      if (r + kRingAhead < R)
+        psk::cp_async16(reinterpret_cast<uint4*>(&s_row[(r + kRingAhead) & 7]) + t,
+                        reinterpret_cast<const uint4*>(rows + r + kRingAhead) + t);
       psk::cp_async_commit();
     }
+    // The signalling thread starts reading job r - (kLag - 2)'s done flag now; it is checked before
+    // the second barrier.
+    uint32_t done_seen = 1u;
+    if (sig && r >= psk::kLag - 2 && !timed_out) done_seen = psk::ld_acquire_u32(sync.done + (r - (psk::kLag - 2)));
     // picks of row r + 3's ancestors when they are old enough to be in global memory (instance
     // threads only: the signalling thread keeps no loads in flight)
     int32_t jp_next[3] = {-1, -1, -1};
@@ -476,7 +488,7 @@ greedy_search_kernel(const psk::RowPre* __restrict__ rows, const uint64_t* __res
       const int32_t a3[3] = {x3.par, x3.anc[0], x3.anc[1]};
 #pragma unroll
       for (int q = 0; q < 3; ++q)
-        if (a3[q] >= 0 && (int64_t)a3[q] <= (int64_t)r - 4) jp_next[q] = __ldcg(assign + a3[q]);
+        if (a3[q] >= 0 && (int64_t)a3[q] <= (int64_t)r - (psk::kLag - 1)) jp_next[q] = __ldcg(assign + a3[q]);
     }
     uint32_t h3[IPT];
     float t3[IPT];
@@ -491,7 +503,9 @@ greedy_search_kernel(const psk::RowPre* __restrict__ rows, const uint64_t* __res
     if (r + 2 < R) {
       const psk::RowPre& x2 = s_row[(r + 2) & 7];
       // An ancestor's chain is a prefix of this one; on the instance that took it, the probe goes
-      // to its end.  It counts only if its inserts are in every probe snapshot: a <= (r + 2) - kLag.
+      // to its end.  It counts only if its inserts are in every probe snapshot: a <= (r + 2) - kLag,
+      // i.e. its distance d = r + 2 - a is at least kLag; its pick is jm[d - 3] while that is still
+      // in registers, else the one loaded from global memory a step ahead.
       const int32_t a2[3] = {x2.par, x2.anc[0], x2.anc[1]};
       const uint32_t a2nb[3] = {x2.par_nb, x2.anc_nb[0], x2.anc_nb[1]};
       int32_t jp[3];
@@ -500,9 +514,10 @@ greedy_search_kernel(const psk::RowPre* __restrict__ rows, const uint64_t* __res
         const int64_t a = a2[q];
         jp[q] = -1;
         if (a >= 0) {
-          if (a == (int64_t)r - 3) jp[q] = jm3;
-          else if (a == (int64_t)r - 4) jp[q] = jm4;
-          else if (a <= (int64_t)r - 5) jp[q] = jp_pre[q];
+          const int64_t d = (int64_t)r + 2 - a;
+          if (d == psk::kLag) jp[q] = jm[psk::kLag - 3];
+          else if (d == psk::kLag + 1) jp[q] = jm[psk::kLag - 2];
+          else if (d >= psk::kLag + 2) jp[q] = jp_pre[q];
         }
       }
 #pragma unroll
@@ -540,8 +555,9 @@ greedy_search_kernel(const psk::RowPre* __restrict__ rows, const uint64_t* __res
       }
     }
 
+    // Pass 1: hit corrections, W and the capacity guard; W_min over A.
     const psk::RowConst rc = row_of(cur);
-    psk::PairEval ev[IPT];
+    psk::PairW ev[IPT];
     float wmin = INFINITY;
     bool anyA = false;
 #pragma unroll
@@ -549,13 +565,12 @@ greedy_search_kernel(const psk::RowPre* __restrict__ rows, const uint64_t* __res
       const uint32_t i = own(k);
       if (i < I) {
         uint32_t h = hr[k];
-        if ((int32_t)i == jm1 && cur.lcp[0] > h) h = cur.lcp[0];
-        if ((int32_t)i == jm2 && cur.lcp[1] > h) h = cur.lcp[1];
-        if ((int32_t)i == jm3 && cur.lcp[2] > h) h = cur.lcp[2];
-        if ((int32_t)i == jm4 && cur.lcp[3] > h) h = cur.lcp[3];
+#pragma unroll
+        for (int d = 0; d < psk::kLcpBack; ++d)
+          if ((int32_t)i == jm[d] && cur.lcp[d] > h) h = cur.lcp[d];
         const float tp = h == hr[k] ? tr[k] : __uint_as_float(psk::kNoTpfBits);
         hr[k] = h;
-        ev[k] = psk::eval_pair_tpf(m, rc, h, tp, s_it[i], s_q[i], s_S[i], s_M[i]);
+        ev[k] = psk::pair_w(m, rc, h, tp, s_it[i], s_S[i], s_M[i]);
         if (ev[k].inA) {
           wmin = fminf(wmin, ev[k].W);
           anyA = true;
@@ -579,16 +594,18 @@ greedy_search_kernel(const psk::RowPre* __restrict__ rows, const uint64_t* __res
       wmin = psk::warp_fmin(v);
       anyA = __any_sync(0xffffffffu, a);
     }
+    // Pass 2: latencies and the admission class of the pairs in C only; the argmin key.
     PickKey best{psk::kNoKeyCi, 0u, ~0ull};
 #pragma unroll
     for (int k = 0; k < IPT; ++k) {
       const uint32_t i = own(k);
-      if (i < I && ev[k].inA) {
-        const uint32_t cls = psk::pair_class(m, rc, ev[k], wmin);
-        if (cls <= 1u) {
-          const PickKey kk{(cls << 28) | i, hr[k], psk::pair_value(cls, hr[k], s_b[i], s_qr[i], s_q[i], ev[k].n)};
-          if (pick_less(kk, best)) best = kk;
-        }
+      if (i < I && ev[k].inA && psk::pair_in_c(rc, ev[k].W, wmin)) {
+        const int64_t q = s_q[i];
+        float tpot, ttft;
+        psk::pair_lat(m, rc, ev[k], s_it[i], q, s_S[i], &tpot, &ttft);
+        const uint32_t cls = psk::pair_admitted(m, rc, tpot, ttft) ? 0u : 1u;
+        const PickKey kk{(cls << 28) | i, hr[k], psk::pair_value(cls, hr[k], s_b[i], s_qr[i], q, ev[k].n)};
+        if (pick_less(kk, best)) best = kk;
       }
     }
     best = warp_pick(best);
@@ -612,11 +629,13 @@ greedy_search_kernel(const psk::RowPre* __restrict__ rows, const uint64_t* __res
         }
       }
     }
-    if (t < 5) psk::cp_async_wait_all();
-    // Row r + 2's probes (issued in the next step) need every insert of requests <= r - 3.
-    if (sig && r >= 3 && !timed_out) {
+    // rows <= r + kRingAhead - 2 are in (the next step reads row r + 4)
+    if (t < psk::kRowWords) psk::cp_async_wait_group<2>();
+    // Row r + 2's probes (issued in the next step) need every insert of requests <= r + 2 - kLag;
+    // the earlier jobs were waited for in earlier steps.
+    if (sig && done_seen == 0u) {
       const uint64_t t0 = psk::globaltimer_ns();
-      while (psk::ld_acquire_u32(sync.done + (r - 3)) < kHelpers) {
+      while (psk::ld_acquire_u32(sync.done + (r - (psk::kLag - 2))) == 0u) {
         if (psk::globaltimer_ns() - t0 > kWaitNs) {
           atomicOr(err, psk::kErrTimeout);
           timed_out = true;
@@ -682,10 +701,9 @@ greedy_search_kernel(const psk::RowPre* __restrict__ rows, const uint64_t* __res
       need1[k] = need2[k];
       h2[k] = h3[k];
     }
-    jm4 = jm3;
-    jm3 = jm2;
-    jm2 = jm1;
-    jm1 = pick ? (int32_t)j : -1;
+#pragma unroll
+    for (int d = psk::kLcpBack - 1; d > 0; --d) jm[d] = jm[d - 1];
+    jm[0] = pick ? (int32_t)j : -1;
 #pragma unroll
     for (int q = 0; q < 3; ++q) jp_pre[q] = jp_next[q];
   }

@@ -26,6 +26,16 @@ namespace {
 
 constexpr uint32_t kStageBlocks = 4096;  // 32 KB of staged chain per thread block
 
+// Launch statistics (ps_last_probe_stats): each warp adds its threads' counts once, at the end.
+enum { kStatRowsScratch = 0, kStatRowsDerived, kStatLookupsScratch, kStatLookupsDerived, kStatStagedBlocks,
+       kStatPairsDerived };
+
+__device__ __forceinline__ void add_stat(unsigned long long* p, uint64_t v) {
+#pragma unroll
+  for (int s = 16; s > 0; s >>= 1) v += __shfl_xor_sync(0xffffffffu, v, s);
+  if ((threadIdx.x & 31) == 0 && v) atomicAdd(p, (unsigned long long)v);
+}
+
 // Where a pair's result goes: its hit and, when requested, T_pf at that hit (the greedy pass reads
 // it instead of recomputing it for pairs whose hit does not change).
 struct PairOut {
@@ -44,16 +54,22 @@ __global__ void __launch_bounds__(WARPS * 32)
 probe_hits_kernel(const uint64_t* __restrict__ slots, const uint64_t* __restrict__ ovf,
                   const psk::TableDesc* __restrict__ tdesc,
                   uint32_t I, const uint64_t* __restrict__ off, const uint64_t* __restrict__ hash,
-                  uint32_t R, const psk::RowPre* __restrict__ rows, PairOut out) {
+                  uint32_t R, const psk::RowPre* __restrict__ rows, PairOut out,
+                  unsigned long long* __restrict__ stats) {
   extern __shared__ uint64_t s_chain[];
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
+  uint64_t n_look = 0, n_rows = 0, n_staged = 0;  // this thread's share of the launch statistics
   for (uint32_t r = blockIdx.x; r < R; r += gridDim.x) {
     if (rows && __ldg(&rows[r].base) >= 0) continue;  // derived in the second pass
     const uint64_t o = off[r];
     const uint64_t nb = off[r + 1] - o;
     const uint32_t Lr = out.tpf ? __ldg(out.L + r) : 0u;
     const uint64_t ns = nb < kStageBlocks ? nb : kStageBlocks;
+    if (threadIdx.x == 0) {
+      n_rows += 1;
+      n_staged += ns;
+    }
     for (uint64_t k = threadIdx.x; k < ns; k += WARPS * 32) s_chain[k] = __ldg(hash + o + k);
     __syncthreads();
     auto chain = [&](uint64_t k) { return k < ns ? s_chain[k] : __ldg(hash + o + k); };
@@ -63,6 +79,7 @@ probe_hits_kernel(const uint64_t* __restrict__ slots, const uint64_t* __restrict
         uint64_t lo = 0, hi = nb;  // first miss in [lo, hi]
         while (lo < hi) {
           const uint64_t mid = (lo + hi) >> 1;
+          ++n_look;
           if (psk::main_contains(slots, ovf, d, chain(mid))) lo = mid + 1; else hi = mid;
         }
         out.put(r, I, i, (uint32_t)lo, Lr);
@@ -70,12 +87,20 @@ probe_hits_kernel(const uint64_t* __restrict__ slots, const uint64_t* __restrict
     } else {
       for (uint32_t i = warp; i < I; i += WARPS) {
         const psk::TableDesc d = tdesc[i];
-        auto cached = [&](uint64_t k) { return psk::main_contains(slots, ovf, d, chain(k)); };
+        auto cached = [&](uint64_t k) {
+          ++n_look;
+          return psk::main_contains(slots, ovf, d, chain(k));
+        };
         const uint64_t h = psk::warp_first_miss_linear(0, nb, cached);
         if (lane == 0) out.put(r, I, i, (uint32_t)h, Lr);
       }
     }
     __syncthreads();
+  }
+  if (stats) {
+    add_stat(stats + kStatRowsScratch, n_rows);
+    add_stat(stats + kStatLookupsScratch, n_look);
+    add_stat(stats + kStatStagedBlocks, n_staged);
   }
 }
 
@@ -85,11 +110,13 @@ template <int WARPS, bool SEARCH>
 __global__ void __launch_bounds__(WARPS * 32)
 probe_derived_kernel(const uint64_t* __restrict__ slots, const uint64_t* __restrict__ ovf,
                      const psk::TableDesc* __restrict__ tdesc, uint32_t I, const uint64_t* __restrict__ hash,
-                     uint32_t R, const psk::RowPre* __restrict__ rows, PairOut out) {
+                     uint32_t R, const psk::RowPre* __restrict__ rows, PairOut out,
+                     unsigned long long* __restrict__ stats) {
   extern __shared__ uint32_t s_list[];  // I entries
   __shared__ uint32_t s_n;
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
+  uint64_t n_look = 0, n_rows = 0, n_pairs = 0;
   for (uint32_t r = blockIdx.x; r < R; r += gridDim.x) {
     const int32_t b = __ldg(&rows[r].base);
     if (b < 0) continue;  // block-uniform
@@ -107,14 +134,26 @@ probe_derived_kernel(const uint64_t* __restrict__ slots, const uint64_t* __restr
     }
     __syncthreads();
     const uint32_t n = s_n;
+    if (threadIdx.x == 0) {
+      n_rows += 1;
+      n_pairs += n;
+    }
     for (uint32_t x = warp; x < n; x += WARPS) {
       const uint32_t i = s_list[x];
       const psk::TableDesc d = tdesc[i];
-      auto cached = [&](uint64_t k) { return psk::main_contains(slots, ovf, d, __ldg(hash + o + k)); };
+      auto cached = [&](uint64_t k) {
+        ++n_look;
+        return psk::main_contains(slots, ovf, d, __ldg(hash + o + k));
+      };
       const uint64_t h = SEARCH ? psk::warp_search_range(nbb, nbr, cached) : psk::warp_first_miss_linear(nbb, nbr, cached);
       if (lane == 0) out.put(r, I, i, (uint32_t)h, Lr);
     }
     __syncthreads();
+  }
+  if (stats) {
+    add_stat(stats + kStatRowsDerived, n_rows);
+    add_stat(stats + kStatLookupsDerived, n_look);
+    add_stat(stats + kStatPairsDerived, n_pairs);
   }
 }
 
@@ -141,7 +180,8 @@ int probe_max_grid(uint32_t I, int num_sms) {
 
 cudaError_t launch_probe(const uint64_t* slots, const uint64_t* ovf, const psk::TableDesc* tdesc, uint32_t I,
                          const psk::WindowDev& w, const psk::RowPre* rows, uint32_t* hits, float* tpf,
-                         const psk::DevModel& m, int grid, int search, cudaStream_t s) {
+                         const psk::DevModel& m, int grid, int search, unsigned long long* stats,
+                         cudaEvent_t ev_mid, cudaStream_t s) {
   if (w.R == 0) return cudaSuccess;
   const PairOut out{hits, tpf, w.L, m};
   const int g = (int)((uint32_t)grid < w.R ? (uint32_t)grid : w.R);
@@ -149,10 +189,13 @@ cudaError_t launch_probe(const uint64_t* slots, const uint64_t* ovf, const psk::
   const size_t smem2 = (size_t)I * sizeof(uint32_t);
 #define PS_PROBE(W, S)                                                                                      \
   do {                                                                                                      \
-    probe_hits_kernel<W, S><<<g, W * 32, smem, s>>>(slots, ovf, tdesc, I, w.off, w.hash, w.R, rows, out);    \
+    probe_hits_kernel<W, S><<<g, W * 32, smem, s>>>(slots, ovf, tdesc, I, w.off, w.hash, w.R, rows, out,    \
+                                                   stats);                                                  \
     cudaError_t e = cudaGetLastError();                                                                     \
     if (e != cudaSuccess || !rows) return e;                                                                \
-    probe_derived_kernel<W, S><<<g, W * 32, smem2, s>>>(slots, ovf, tdesc, I, w.hash, w.R, rows, out);       \
+    if (ev_mid) cudaEventRecord(ev_mid, s);                                                                 \
+    probe_derived_kernel<W, S><<<g, W * 32, smem2, s>>>(slots, ovf, tdesc, I, w.hash, w.R, rows, out,       \
+                                                        stats);                                             \
     return cudaGetLastError();                                                                              \
   } while (0)
   if (I >= 64) {

@@ -12,9 +12,9 @@
 //                 path.  Slot value 0 = empty.  Each table has a single writer (one warp per
 //                 instance), so placement needs no atomics and a key is never stored twice.
 //   delta table   window-scoped set of (instance, block) pairs cached by the window's own earlier
-//                 decisions: 16-byte slots {hash, instance}, 8 per 128-byte bucket, linear probing,
-//                 sized at twice the window's block bound so it can never fill.  Cleared (through its
-//                 insert log) after each window.
+//                 decisions: one 16-byte slot {hash, instance + 1} per pair, linear probing from the
+//                 hash's home slot, sized at twice the window's block bound so it can never fill.
+//                 Cleared after each window.
 //   state         structure of arrays per instance (b, qr, q, S, M_KV, B_max).
 //   hits          u32 [R x I], request-major.
 #pragma once
@@ -49,15 +49,21 @@ struct TableDesc {
   uint32_t pad;
 };
 
-// One key of the window's delta table with up to two of the instances it was inserted for
-// (instance id + 1, filled in order; 0 = free).  A key with more instances continues in a later
-// slot.  (Four 16-bit fields would resolve more keys in one slot, but 16-bit compare-and-swap made
-// the inserts markedly slower.)
-constexpr int kDeltaTags = 2;
+// One (block, instance) pair of the window's delta table: the block hash and instance id + 1 (0 while
+// the claiming thread has not yet written it).  Within one window each pair is inserted at most once:
+// a request inserts chain[h, nb) on its pick with h the exact first miss there, so none of those
+// blocks is cached on that instance yet (a block hash fixes its whole prefix, so an earlier insert of
+// the same block would have cached chain[0, that position] and moved the first miss past it).
 struct DeltaSlot {
   unsigned long long hash;
-  unsigned int tag[kDeltaTags];
+  unsigned int tag;
+  unsigned int pad;
 };
+
+// Greedy pipeline depth: a probe for request s sees every delta insert of requests <= s - kLag, and
+// the requests s - 1 .. s - (kLag - 1) are covered by their common chain prefix with s (RowPre::lcp).
+constexpr int kLag = 9;
+constexpr int kLcpBack = kLag - 1;
 
 // Per-request constants of one window, computed in parallel before the greedy pass: the request's
 // chain range, the Algorithm 1 / Eq. 8 row constants, and its relations to earlier requests of the
@@ -72,20 +78,21 @@ struct __align__(16) RowPre {
   float etaZ;         // eta * Z
   float ttft_budget;  // max(target, T_pf(L, 0))
   float tpot_target;
-  uint32_t lcp[4];    // common chain prefix with requests r - 1 .. r - 4 (blocks)
   int32_t par;        // deepest earlier request whose chain is a prefix of r's, -1 if none
   uint32_t par_nb;    // its chain length
   int32_t base;       // the topmost request of r's parent links (r's chain starts with its chain), -1 if none
   int32_t anc[2];     // the parent's parent and its parent (-1 if none): their chains are prefixes too
   uint32_t anc_nb[2]; // their chain lengths
+  uint32_t lcp[kLcpBack];  // common chain prefix with requests r - 1 .. r - kLcpBack (blocks)
 };
-static_assert(sizeof(RowPre) == 80, "RowPre is five 16-byte words");
+constexpr int kRowWords = (int)(sizeof(RowPre) / 16);
+static_assert(sizeof(RowPre) % 16 == 0 && kRowWords == 6, "RowPre is six 16-byte words");
 
 // Hand-off between the greedy block and the blocks that insert its picks' chains into the delta
 // table (one cooperative launch).
 struct GreedySync {
   unsigned long long* jobs;  // per request: hit of the pick << 32 | pick (0xFFFFFFFF = rejected)
-  uint32_t* done;            // per request: insert blocks that have finished its blocks
+  uint32_t* done;            // per request: 1 once its insert block has finished its blocks
   uint32_t* pub;             // number of requests published so far
 };
 
@@ -302,20 +309,10 @@ __device__ __forceinline__ uint64_t delta_next(uint64_t slot, uint64_t nslots) {
 
 // Verdict of one slot for (key, tag = inst + 1): 1 present, 0 absent, -1 look at the next slot.
 // Slots fill as an unbroken run from a key's home (inserts only claim empty slots and nothing is
-// removed while a window runs), a key's instance fields fill in order, and a key moves on to a
-// later slot only once all its fields are taken; so an empty slot, or an entry of the key with a
-// free field, ends the search.
+// removed while a window runs), so an empty slot ends the search.  A slot of the key whose tag is
+// not (yet) this instance's sends the search on: the pair is stored once, in its own slot.
 __device__ __forceinline__ int delta_slot_verdict(const ulonglong2& v, uint64_t key, uint32_t tag) {
-  if (v.x == key) {
-    bool full = true;
-#pragma unroll
-    for (int f = 0; f < kDeltaTags; ++f) {
-      const uint32_t x = (uint32_t)(v.y >> (32 * f));
-      if (x == tag) return 1;
-      full = full && x != 0u;
-    }
-    return full ? -1 : 0;
-  }
+  if (v.x == key) return (uint32_t)v.y == tag ? 1 : -1;
   return v.x == kEmpty ? 0 : -1;
 }
 
@@ -335,23 +332,18 @@ __device__ __forceinline__ bool delta_contains(const DeltaSlot* delta, uint64_t 
   return delta_contains_from(delta, nslots, inst, key, delta_home(key, nslots));
 }
 
-// Insert (inst, key): from the home slot, the first slot that is empty (claimed by compare-and-swap
-// on the hash) or already holds the key takes the instance in its first free field.  A lookup
-// racing with the insert sees the key without this instance, which only under-reports; a duplicate
-// entry is harmless.  The table has twice as many slots as a window has chain blocks, so it cannot
-// fill; false reports a full table anyway.
+// Insert (inst, key): the first empty slot from the key's home is claimed by compare-and-swap on
+// the hash, then the tag is stored (one round trip).  A lookup racing with the insert may see the
+// slot without its tag and report the pair absent, which only under-reports; it is visible to every
+// reader once the inserting block has released its done flag.  The table has twice as many slots as
+// a window has chain blocks, so it cannot fill; false reports a full table anyway.
 __device__ __forceinline__ bool delta_insert(DeltaSlot* delta, uint64_t nslots, uint32_t inst, uint64_t key) {
   if (key == kEmpty || key == kTomb) return true;
-  const uint32_t tag = inst + 1;
   uint64_t slot = delta_home(key, nslots);
   for (uint64_t p = 0; p < nslots; ++p) {
-    const unsigned long long old = atomicCAS(&delta[slot].hash, kEmpty, (unsigned long long)key);
-    if (old == kEmpty || old == key) {
-#pragma unroll
-      for (int f = 0; f < kDeltaTags; ++f) {
-        const unsigned int x = atomicCAS(&delta[slot].tag[f], 0u, tag);
-        if (x == 0 || x == tag) return true;
-      }
+    if (atomicCAS(&delta[slot].hash, kEmpty, (unsigned long long)key) == kEmpty) {
+      __stcg(&delta[slot].tag, inst + 1);
+      return true;
     }
     slot = delta_next(slot, nslots);
   }
@@ -384,6 +376,10 @@ __device__ __forceinline__ void cp_async16(void* smem, const void* gmem) {
 __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
 
 __device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_all;" ::: "memory"); }
+
+// Wait until at most N of this thread's most recent copy groups are still pending.
+template <int N>
+__device__ __forceinline__ void cp_async_wait_group() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
 
 // ------------------------------------------------------------------------------- first-miss walks --
 // All 32 lanes of a warp call these with the same arguments; present(k) is evaluated per lane.
@@ -635,28 +631,67 @@ __device__ __forceinline__ float t_pf_of_hit(const DevModel& m, uint32_t L, uint
 // Marks a precomputed T_pf as not available (a NaN pattern T_pf never produces).
 constexpr uint32_t kNoTpfBits = 0xFFFFFFFFu;
 
-// eval_pair with the instance terms precomputed, and T_pf given unless it carries kNoTpfBits.
-__device__ __forceinline__ PairEval eval_pair_tpf(const DevModel& m, const RowConst& rc, uint32_t h, float tpf_in,
-                                                  const InstTerms& it, int64_t q, int64_t S, int64_t M) {
-  PairEval e;
+// The two halves of eval_pair with the instance terms precomputed (the greedy evaluates the
+// latencies only for pairs that pass the capacity guard and the recompute filter).  Together they
+// perform exactly eval_pair's rounded operations.
+//   pair_w:   T_pf at the hit (given unless tpf_in carries kNoTpfBits), W = T_pf(n, c) - T_pf(0, L),
+//             n, and the capacity guard (Algorithm 1 CapacityCandidates).
+//   pair_lat: TPOT (Eq. 5 / Eq. 9) and TTFT (Eq. 4) of the pair.
+struct PairW {
+  float W, tpf;
+  int64_t n;
+  bool inA;
+};
+
+__device__ __forceinline__ PairW pair_w(const DevModel& m, const RowConst& rc, uint32_t h, float tpf_in,
+                                        const InstTerms& it, int64_t S, int64_t M) {
+  PairW x;
   const int64_t c = 16 * (int64_t)h;
-  const int64_t n = (int64_t)rc.L - c;
-  const float tpf = __float_as_uint(tpf_in) == kNoTpfBits ? t_pf(m, __ll2float_rn(n), __ll2float_rn(c)) : tpf_in;
-  e.n = n;
-  e.W = __fsub_rn(tpf, rc.t_cached);
+  x.n = (int64_t)rc.L - c;
+  x.tpf = __float_as_uint(tpf_in) == kNoTpfBits ? t_pf(m, __ll2float_rn(x.n), __ll2float_rn(c)) : tpf_in;
+  x.W = __fsub_rn(x.tpf, rc.t_cached);
+  x.inA = it.okB && (S + (int64_t)rc.L <= M);
+  return x;
+}
+
+__device__ __forceinline__ void pair_lat(const DevModel& m, const RowConst& rc, const PairW& x, const InstTerms& it,
+                                         int64_t q, int64_t S, float* tpot, float* ttft) {
   const int64_t Sp = S + (int64_t)rc.L;
-  e.inA = it.okB && (Sp <= M);
   float dec = __fadd_rn(it.dec0, __fmul_rn(m.b2, __ll2float_rn(Sp)));
   dec = __fmul_rn(dec, it.f);
   if (m.interference_mode == 0) {
-    e.tpot = __fadd_rn(dec, __fmul_rn(m.g_q, __ll2float_rn(q + n)));
+    *tpot = __fadd_rn(dec, __fmul_rn(m.g_q, __ll2float_rn(q + x.n)));
   } else {
     const float den = m.lout > 1.0f ? m.lout : 1.0f;
-    const float interf = (it.Bp > 1) ? __fdiv_rn(tpf, den) : 0.0f;
-    e.tpot = __fadd_rn(dec, interf);
+    const float interf = (it.Bp > 1) ? __fdiv_rn(x.tpf, den) : 0.0f;
+    *tpot = __fadd_rn(dec, interf);
   }
-  e.ttft = __fadd_rn(tpf, it.tq);
+  *ttft = __fadd_rn(x.tpf, it.tq);
+}
+
+// eval_pair with the instance terms precomputed, and T_pf given unless it carries kNoTpfBits.
+__device__ __forceinline__ PairEval eval_pair_tpf(const DevModel& m, const RowConst& rc, uint32_t h, float tpf_in,
+                                                  const InstTerms& it, int64_t q, int64_t S, int64_t M) {
+  const PairW x = pair_w(m, rc, h, tpf_in, it, S, M);
+  PairEval e;
+  e.n = x.n;
+  e.W = x.W;
+  e.inA = x.inA;
+  pair_lat(m, rc, x, it, q, S, &e.tpot, &e.ttft);
   return e;
+}
+
+// Recompute filter (Eq. 8) of a capacity-eligible pair once W_min is known: W - W_min <= eta Z,
+// every pair of A when Z <= 0.
+__device__ __forceinline__ bool pair_in_c(const RowConst& rc, float W, float Wmin) {
+  return (rc.Z > 0.0f) ? (__fsub_rn(W, Wmin) <= rc.etaZ) : true;
+}
+
+// Admission of a pair of C (Algorithm 1 TPOT filter, plus the TTFT budget when enabled).
+__device__ __forceinline__ bool pair_admitted(const DevModel& m, const RowConst& rc, float tpot, float ttft) {
+  bool ok = tpot < rc.tpot_target;
+  if (m.ttft_filter) ok = ok && (ttft <= rc.ttft_budget);
+  return ok;
 }
 
 __device__ __forceinline__ PairEval eval_pair_terms(const DevModel& m, const RowConst& rc, uint32_t h,
@@ -668,11 +703,8 @@ __device__ __forceinline__ PairEval eval_pair_terms(const DevModel& m, const Row
 // 0 in T, 1 in C \ T, 2 filtered by the recompute budget.
 __device__ __forceinline__ uint32_t pair_class(const DevModel& m, const RowConst& rc, const PairEval& e,
                                                float Wmin) {
-  const bool inC = (rc.Z > 0.0f) ? (__fsub_rn(e.W, Wmin) <= rc.etaZ) : true;
-  if (!inC) return 2u;
-  bool ok = e.tpot < rc.tpot_target;
-  if (m.ttft_filter) ok = ok && (e.ttft <= rc.ttft_budget);
-  return ok ? 0u : 1u;
+  if (!pair_in_c(rc, e.W, Wmin)) return 2u;
+  return pair_admitted(m, rc, e.tpot, e.ttft) ? 0u : 1u;
 }
 
 // Ordering value inside a class.  Class 0 (Section 6.2, D-C-Q): more decoding requests, then more
@@ -723,10 +755,12 @@ constexpr uint32_t kNoKeyCi = 0xFFFFFFFFu;  // class 15: worse than any real pai
 // Kernel launchers (one translation unit each).
 namespace pskl {
 // rows (from launch_relations, or nullptr to probe every request from scratch); tpf (nullable)
-// receives T_pf of every pair's hit.
+// receives T_pf of every pair's hit; stats (nullable) accumulates the six launch counters of
+// ps_last_probe_stats; ev_mid (nullable) is recorded between the two probe kernels.
 cudaError_t launch_probe(const uint64_t* slots, const uint64_t* ovf, const psk::TableDesc* tdesc, uint32_t I,
                          const psk::WindowDev& w, const psk::RowPre* rows, uint32_t* hits, float* tpf,
-                         const psk::DevModel& m, int grid, int search, cudaStream_t s);
+                         const psk::DevModel& m, int grid, int search, unsigned long long* stats,
+                         cudaEvent_t ev_mid, cudaStream_t s);
 int probe_max_grid(uint32_t I, int num_sms);
 cudaError_t launch_score(const uint32_t* hits, psk::StateSoA st, uint32_t I, const psk::WindowDev& w,
                          const psk::DevModel& m, float* tpot, float* ttft, uint8_t* cls, int32_t* best,

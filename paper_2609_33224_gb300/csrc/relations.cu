@@ -2,7 +2,7 @@
 //
 // Besides the Algorithm 1 / Eq. 8 row constants (T_pf(0, L), CacheBenefit Z, eta * Z, the TTFT
 // budget), each request gets its chain relations to earlier requests of the same window:
-//   * lcp[d - 1]: the common chain prefix with the request d places before it (d = 1..4).  Chained
+//   * lcp[d - 1]: the common chain prefix with the request d places before it (d = 1..kLcpBack).  Chained
 //     block hashes (Section 7's prefix tree) make "block k equal" imply "blocks 0..k equal", so the
 //     common prefix is found with the 32-ary first-miss search.
 //   * par: the deepest earlier request whose whole chain is a prefix of this one (an agentic
@@ -71,9 +71,9 @@ __global__ void relations_kernel(psk::WindowDev w, psk::DevModel m, const psk::L
       const uint64_t* bq = w.hash + oq;
       return (uint32_t)psk::warp_search_range(0, nb < nq ? nb : nq, [&](uint64_t k) { return a[k] == bq[k]; });
     };
-    uint32_t lcp[4];
+    uint32_t lcp[psk::kLcpBack];
 #pragma unroll
-    for (uint32_t d = 1; d <= 4; ++d) lcp[d - 1] = r >= d ? lcp_with(r - d) : 0u;
+    for (uint32_t d = 1; d <= (uint32_t)psk::kLcpBack; ++d) lcp[d - 1] = r >= d ? lcp_with(r - d) : 0u;
     int32_t par = -1;
     uint32_t par_nb = 0;
     const uint64_t stop = nb > kParentScan ? nb - kParentScan : 0;
@@ -118,7 +118,7 @@ __global__ void relations_kernel(psk::WindowDev w, psk::DevModel m, const psk::L
       x.ttft_budget = rc.ttft_budget;
       x.tpot_target = rc.tpot_target;
 #pragma unroll
-      for (int d = 0; d < 4; ++d) x.lcp[d] = lcp[d];
+      for (int d = 0; d < psk::kLcpBack; ++d) x.lcp[d] = lcp[d];
       x.par = par;
       x.par_nb = par_nb;
       x.base = -1;
