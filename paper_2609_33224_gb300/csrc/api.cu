@@ -55,7 +55,7 @@ struct ps_ctx {
   unsigned long long* d_count = nullptr;
   psk::DeltaSlot* d_delta = nullptr;
   uint64_t delta_nslots = 0;
-  psk::GreedySync gsync{nullptr, nullptr, nullptr};
+  psk::GreedySync gsync{nullptr, nullptr, nullptr, nullptr, nullptr, 0u};
   psk::RowPre* d_rows = nullptr;      // per-request constants and relations (search mode greedy)
   psk::LastSlot* d_lastslot = nullptr;
   uint32_t lastslot_n = 0;
@@ -374,10 +374,13 @@ ps_status ps_create(const ps_config* cfg, ps_ctx** out) {
   while (c->lastslot_n < 2 * c->Rmax) c->lastslot_n <<= 1;
   const size_t RI = (size_t)c->Rmax * c->I;
   const size_t I = c->I;
+  c->gsync.ring_stride = (c->I + 3u) / 4u * 4u;
   bool ok = dalloc(c, &c->d_slots, c->total_slots) == cudaSuccess && dalloc(c, &c->d_ovf, c->total_ovf) == cudaSuccess &&
             dalloc(c, &c->d_tdesc, I) == cudaSuccess && dalloc(c, &c->d_count, I) == cudaSuccess &&
             dalloc(c, &c->d_delta, (size_t)dn) == cudaSuccess && dalloc(c, &c->gsync.jobs, c->Rmax) == cudaSuccess &&
-            dalloc(c, &c->gsync.done, c->Rmax) == cudaSuccess && dalloc(c, &c->gsync.pub, 1) == cudaSuccess &&
+            dalloc(c, &c->gsync.done, c->Rmax) == cudaSuccess && dalloc(c, &c->gsync.ready, c->Rmax) == cudaSuccess &&
+            dalloc(c, &c->gsync.hitring, (size_t)psk::kHitSlots * c->gsync.ring_stride) == cudaSuccess &&
+            dalloc(c, &c->gsync.tpfring, (size_t)psk::kHitSlots * c->gsync.ring_stride) == cudaSuccess &&
             dalloc(c, &c->d_rows, c->Rmax) == cudaSuccess && dalloc(c, &c->d_lastslot, c->lastslot_n) == cudaSuccess;
   for (psk::StateSoA* s : {&c->st, &c->pend}) {
     ok = ok && dalloc(c, &s->b, I) == cudaSuccess && dalloc(c, &s->qr, I) == cudaSuccess &&

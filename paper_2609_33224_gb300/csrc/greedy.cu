@@ -271,7 +271,8 @@ cudaError_t greedy_launch(const uint64_t* slots, const uint64_t* ovf, const psk:
 
 
 // ----------------------------------------------------------------------------------------------
-// Prefix-closed caches (the probe's search mode): a software-pipelined greedy pass.
+// Prefix-closed caches (the probe's search mode): a pipelined greedy pass over three kinds of
+// thread block in one cooperative launch.
 //
 // On a prefix-closed cache the hit of a request is the first chain position not cached, and the
 // union of prefix-closed sets has as first miss the largest of the sets' first misses.  The
@@ -280,52 +281,35 @@ cudaError_t greedy_launch(const uint64_t* slots, const uint64_t* ovf, const psk:
 //     hit(s, i) = max( first miss of main_i + delta_i(<= s - kLag),
 //                      lcp(s, s - d) for each d = 1..kLag-1 such that request s - d went to i )
 // where delta_i(<= s - kLag) holds the blocks inserted for requests up to s - kLag and lcp(s, s - d) is
-// the common chain prefix (from the relations pass).  The first term is probed ahead of time, while
-// earlier requests are still being decided, so no table access is on the per-request critical
-// path.  The probe position is hit0, raised to the end of the request's parent (the deepest earlier
-// request whose chain is a prefix of this one) on the instance that took the parent; a probe that
-// finds the block cached hands the instance to a warp search.  Probes may also see inserts of
-// requests s - kLag + 1 .. s - 1 (they land while the probe runs, in any order): any snapshot
-// between delta(<= s - kLag) and delta(<= s - 1) gives a first miss between the two, and the max
-// with the lcp terms is then exact all the same.
+// the common chain prefix (from the relations pass).
 //
-// Block 0 decides.  Per step r it evaluates row r (two block reductions: W_min, then the argmin)
-// and besides:  loads hit0 of row r + 3;  places row r + 2's probe and loads the chain block there
-// (instances with window inserts only);  issues row r + 1's probe (consumed after the first
-// barrier);  publishes request r's pick as an insert job.  Blocks 1..kHelpers take the jobs
-// round-robin (up to kHelpers jobs in flight), insert each job's chain blocks chain[h, nb) into
-// delta_j and release the job's done flag; block 0 waits (bounded) for job r - (kLag - 2) before its
-// row r + 2 probes go out; a dedicated signalling thread (the block's last warp
-// owns no instances) publishes the jobs and does that wait, so the release and acquire orderings
-// never hold up a thread with loads in flight.  Instance state lives in shared memory and is
-// written only by the thread that owns the instance.
+//   Deciding block (block 0).  Per request r: reads row r's probed hits (first term above) from a
+//   shared-memory ring that was filled by asynchronous copies two steps earlier, raises the hits of
+//   the instances that took requests r - 1 .. r - kLag + 1 to the common prefix, evaluates the row
+//   (capacity guard and W, block reduction to W_min; recompute filter, latencies, admission class
+//   and key of the pairs in C, block reduction to the pick), updates the pick's state and publishes
+//   the decision as an insert job.  No table access is on its per-request path.
+//   Insert blocks.  Take the jobs round-robin (up to kInsertBlocks in flight), insert each job's
+//   chain blocks chain[h, nb) into delta_j and release the job's done flag.
+//   Probe blocks.  Take the rows round-robin.  For row s they wait until the jobs <= s - kLag are
+//   done, replay those jobs (which instances have window inserts, where their last chain ended,
+//   which instances took s's ancestors), then per instance start from hit0, raise the position to
+//   the end of an ancestor's chain on the instance that took it (its chain is a prefix of s's, and
+//   its inserts are in), probe the delta table there when the instance has window inserts, hand the
+//   instances whose block is present to a warp search over the delta, and release the row's ready
+//   flag.  The main table is never probed here: positions past hit0 are absent from a
+//   prefix-closed main table.  Inserts of requests s - kLag + 1 .. s - 1 may land while a probe
+//   runs, in any order: any snapshot between delta(<= s - kLag) and delta(<= s - 1) gives a first
+//   miss between the two sets' first misses, and the max with the lcp terms is exact all the same.
+// Every cross-block wait is bounded (kWaitNs); on expiry the waiter records PS_ERR_TIMEOUT and
+// stops waiting, so the launch always ends.  Instance state lives in the deciding block's shared
+// memory and is written only by the thread that owns the instance.
 
-constexpr uint32_t kHelpers = 8;              // insert blocks beside the deciding block
+constexpr uint32_t kInsertBlocks = 8;         // insert blocks
+constexpr uint32_t kProbeBlocks = 16;         // probe blocks
 constexpr uint32_t kRingAhead = 6;            // row constants are copied into the ring this many rows ahead
 constexpr uint64_t kWaitNs = 1000000000ull;   // bound on any cross-block wait
-constexpr unsigned long long kAbortJob = ~0ull;
-
-struct PickKey {  // lexicographic (class, value, instance) element carrying the pair's hit
-  uint32_t ci;
-  uint32_t h;
-  uint64_t v;
-};
-
-__device__ __forceinline__ bool pick_less(const PickKey& a, const PickKey& z) {
-  return psk::key_less(psk::ArgKey{a.ci, a.v}, psk::ArgKey{z.ci, z.v});
-}
-
-__device__ __forceinline__ PickKey warp_pick(PickKey k) {
-#pragma unroll
-  for (int s = 16; s > 0; s >>= 1) {
-    PickKey o;
-    o.ci = __shfl_xor_sync(0xffffffffu, k.ci, s);
-    o.h = __shfl_xor_sync(0xffffffffu, k.h, s);
-    o.v = __shfl_xor_sync(0xffffffffu, k.v, s);
-    if (pick_less(o, k)) k = o;
-  }
-  return k;
-}
+constexpr unsigned long long kJobValid = 1ull << 63;  // a published job word (0 = not yet published)
 
 __device__ __forceinline__ psk::RowConst row_of(const psk::RowPre& x) {
   psk::RowConst rc;
@@ -338,34 +322,52 @@ __device__ __forceinline__ psk::RowConst row_of(const psk::RowPre& x) {
   return rc;
 }
 
-// Blocks 1..kHelpers: block b inserts the chain tails of jobs b - 1, b - 1 + kHelpers, ... and
+// Bounded spin until *flag != 0 (acquire).  false on timeout (and the error bit is set).
+__device__ __forceinline__ bool wait_flag(const uint32_t* flag, uint32_t* err) {
+  if (psk::ld_acquire_u32(flag) != 0u) return true;
+  const uint64_t t0 = psk::globaltimer_ns();
+  while (psk::ld_acquire_u32(flag) == 0u) {
+    if (psk::globaltimer_ns() - t0 > kWaitNs) {
+      atomicOr(err, psk::kErrTimeout);
+      return false;
+    }
+    __nanosleep(32);
+  }
+  return true;
+}
+
+// Bounded wait for a published job word; 0 on timeout (and the error bit is set).
+__device__ __forceinline__ unsigned long long wait_job(const unsigned long long* job, uint32_t* err) {
+  unsigned long long v = psk::ld_relaxed_u64(job);
+  if (v & kJobValid) return v;
+  const uint64_t t0 = psk::globaltimer_ns();
+  for (;;) {
+    v = psk::ld_relaxed_u64(job);
+    if (v & kJobValid) return v;
+    if (psk::globaltimer_ns() - t0 > kWaitNs) {
+      atomicOr(err, psk::kErrTimeout);
+      return 0ull;
+    }
+    __nanosleep(32);
+  }
+}
+
+__device__ __forceinline__ uint32_t job_pick(unsigned long long jb) { return (uint32_t)jb; }
+__device__ __forceinline__ uint32_t job_hit(unsigned long long jb) { return (uint32_t)(jb >> 32) & 0x7FFFFFFFu; }
+
+// Insert blocks: block b inserts the chain tails of jobs b - 1, b - 1 + kInsertBlocks, ... and
 // releases each job's done flag once all its blocks are in.
-__device__ void insert_helper(const psk::RowPre* __restrict__ rows, const uint64_t* __restrict__ hash, uint32_t R,
+__device__ void insert_blocks(const psk::RowPre* __restrict__ rows, const uint64_t* __restrict__ hash, uint32_t R,
                               psk::DeltaSlot* delta, uint64_t nslots, uint32_t* err, const psk::GreedySync& sync) {
   __shared__ unsigned long long s_job;
   const uint32_t t = threadIdx.x;
-  for (uint32_t job = blockIdx.x - 1; job < R; job += kHelpers) {
-    if (t == 0) {
-      const uint64_t t0 = psk::globaltimer_ns();
-      unsigned long long jb = kAbortJob;
-      for (;;) {
-        if (psk::ld_acquire_u32(sync.pub) > job) {
-          jb = __ldcg(sync.jobs + job);
-          break;
-        }
-        if (psk::globaltimer_ns() - t0 > kWaitNs) {
-          atomicOr(err, psk::kErrTimeout);
-          break;
-        }
-        __nanosleep(32);
-      }
-      s_job = jb;
-    }
+  for (uint32_t job = blockIdx.x - 1; job < R; job += kInsertBlocks) {
+    if (t == 0) s_job = wait_job(sync.jobs + job, err);
     __syncthreads();
     const unsigned long long jb = s_job;
-    if (jb == kAbortJob) return;  // block-uniform
-    const uint32_t j = (uint32_t)jb;
-    const uint32_t hj = (uint32_t)(jb >> 32);
+    if (jb == 0ull) return;  // block-uniform: timed out
+    const uint32_t j = job_pick(jb);
+    const uint32_t hj = job_hit(jb);
     // rows >= job + kLag are the only ones that read this job's inserts
     if (j != 0xFFFFFFFFu && job + psk::kLag < R) {
       const uint64_t off = __ldg(&rows[job].off);
@@ -381,44 +383,181 @@ __device__ void insert_helper(const psk::RowPre* __restrict__ rows, const uint64
   }
 }
 
+// Probe blocks: block p probes rows p, p + kProbeBlocks, ... in order (see the section comment).
+// Shared memory: touched flags and last chain end per instance, the walk list.
 template <int IPT>
-__global__ void __launch_bounds__(544, 1)
-greedy_search_kernel(const psk::RowPre* __restrict__ rows, const uint64_t* __restrict__ hash, uint32_t R, uint32_t I,
-                     const uint32_t* __restrict__ hit0, const float* __restrict__ tpf0, psk::StateSoA committed, psk::StateSoA pending,
-                     psk::DevModel m, psk::DeltaSlot* delta, uint64_t nslots, int32_t* assign,
-                     uint8_t* __restrict__ path, uint32_t* __restrict__ hit_chosen, uint32_t* err,
-                     psk::GreedySync sync) {
-  if (blockIdx.x > 0) {
-    insert_helper(rows, hash, R, delta, nslots, err, sync);
-    return;
+__device__ void probe_rows(const psk::RowPre* __restrict__ rows, const uint64_t* __restrict__ hash, uint32_t R,
+                           uint32_t I, const uint32_t* __restrict__ hit0, const float* __restrict__ tpf0,
+                           const psk::DeltaSlot* delta, uint64_t nslots, uint32_t* err, const psk::GreedySync& sync,
+                           unsigned long long* smem_raw) {
+  uint32_t* s_end = reinterpret_cast<uint32_t*>(smem_raw);  // chain end of the last job on i (0 = none)
+  uint32_t* s_res = s_end + I;                               // search start / result per instance
+  uint32_t* s_walk = s_res + I;                              // instances handed to a warp search
+  __shared__ uint32_t s_nwalk;
+  __shared__ int32_t s_ja[3];       // picks of the row's ancestors old enough to count (-1: none)
+  __shared__ uint32_t s_jnb[3];     // their chain lengths
+  __shared__ uint32_t s_frontier;   // jobs [0, frontier) are done and replayed
+  __shared__ int s_abort;
+  const uint32_t t = threadIdx.x;
+  const uint32_t NT = blockDim.x;
+  const int lane = t & 31, warp = t >> 5, NW = NT >> 5;
+  for (uint32_t i = t; i < I; i += NT) s_end[i] = 0u;
+  if (t == 0) {
+    s_frontier = 0;
+    s_nwalk = 0;
+    s_abort = 0;
   }
-  extern __shared__ unsigned long long smem_raw[];
-  int64_t* s_q = reinterpret_cast<int64_t*>(smem_raw);
+  __syncthreads();
+  for (uint32_t s = blockIdx.x - 1 - kInsertBlocks; s < R; s += kProbeBlocks) {
+    const uint64_t off = __ldg(&rows[s].off);
+    const uint32_t nb = __ldg(&rows[s].nb);
+    if (warp == 0) {
+      // Jobs <= s - kLag must be in the delta table.  Replay them in order, 32 at a time: the
+      // leading run of done flags among the next 32 jobs is taken, and for each instance the latest
+      // of those jobs sets its chain end.
+      const int64_t need = (int64_t)s - psk::kLag + 1;
+      uint32_t f = s_frontier;
+      bool abort = false;
+      while ((int64_t)f < need && !abort) {
+        const uint32_t x = f + (uint32_t)lane;
+        const bool in = (int64_t)x < need;
+        const bool ok = in && psk::ld_acquire_u32(sync.done + x) != 0u;
+        const unsigned okm = __ballot_sync(0xffffffffu, ok);
+        const uint32_t nok = (okm == 0xffffffffu) ? 32u : (uint32_t)(__ffs(~okm) - 1);
+        if (nok == 0u) {  // the next job is not done yet: wait for it
+          bool got = true;
+          if (lane == 0) got = wait_flag(sync.done + f, err);
+          abort = !__shfl_sync(0xffffffffu, got, 0);
+          continue;
+        }
+        const bool mine = (uint32_t)lane < nok;
+        unsigned long long jb = 0ull;
+        if (mine) jb = wait_job(sync.jobs + x, err);
+        abort = __any_sync(0xffffffffu, mine && jb == 0ull);
+        if (abort) break;
+        const uint32_t j = mine ? job_pick(jb) : 0xFFFFFFFFu;
+        const uint32_t nbx = mine ? __ldg(&rows[x].nb) : 0u;
+        // the highest lane of each group of equal picks holds the latest job on that instance
+        const unsigned same = __match_any_sync(0xffffffffu, j);
+        if (mine && j < I && (31 - __clz(same)) == lane) s_end[j] = nbx;
+        f += nok;
+      }
+      if (lane == 0) {
+        s_frontier = f;
+        s_abort = abort ? 1 : 0;
+        const int32_t a[3] = {__ldg(&rows[s].par), __ldg(&rows[s].anc[0]), __ldg(&rows[s].anc[1])};
+        const uint32_t anb[3] = {__ldg(&rows[s].par_nb), __ldg(&rows[s].anc_nb[0]), __ldg(&rows[s].anc_nb[1])};
+#pragma unroll
+        for (int q = 0; q < 3; ++q) {
+          s_ja[q] = -1;
+          s_jnb[q] = anb[q];
+          if (!abort && a[q] >= 0 && (int64_t)a[q] < need) {
+            const uint32_t j = job_pick(psk::ld_relaxed_u64(sync.jobs + a[q]));
+            if (j < I) s_ja[q] = (int32_t)j;
+          }
+        }
+      }
+    }
+    __syncthreads();
+    if (s_abort) return;  // block-uniform
+    const int32_t ja0 = s_ja[0], ja1 = s_ja[1], ja2 = s_ja[2];
+    const uint32_t jn0 = s_jnb[0], jn1 = s_jnb[1], jn2 = s_jnb[2];
+    uint32_t h0[IPT], pos[IPT];
+    float tp0[IPT];
+    bool walk[IPT];
+#pragma unroll
+    for (int k = 0; k < IPT; ++k) {
+      const uint32_t i = t + k * NT;
+      walk[k] = false;
+      if (i < I) {
+        h0[k] = __ldg(hit0 + (uint64_t)s * I + i);
+        tp0[k] = __ldg(tpf0 + (uint64_t)s * I + i);
+        uint32_t p = h0[k];
+        if ((int32_t)i == ja0 && jn0 > p) p = jn0;
+        if ((int32_t)i == ja1 && jn1 > p) p = jn1;
+        if ((int32_t)i == ja2 && jn2 > p) p = jn2;
+        pos[k] = p;
+        // s_end[i] != 0: the instance has window inserts visible to this row
+        if (s_end[i] != 0u && p < nb && psk::delta_contains(delta, nslots, i, __ldg(hash + off + p))) {
+          walk[k] = true;
+          s_res[i] = p;
+          s_walk[atomicAdd(&s_nwalk, 1u)] = i;
+        }
+      }
+    }
+    __syncthreads();
+    const uint32_t nwalk = s_nwalk;
+    if (nwalk) {
+      for (uint32_t x = warp; x < nwalk; x += NW) {
+        const uint32_t i = s_walk[x];
+        auto cached = [&](uint64_t k) { return k < nb && psk::delta_contains(delta, nslots, i, __ldg(hash + off + k)); };
+        const uint64_t hnew = psk::warp_first_miss_search_hint((uint64_t)s_res[i] + 1, nb, s_end[i], cached);
+        __syncwarp();
+        if (lane == 0) s_res[i] = (uint32_t)hnew;
+      }
+      __syncthreads();
+    }
+    const uint32_t slot = s % psk::kHitSlots;
+#pragma unroll
+    for (int k = 0; k < IPT; ++k) {
+      const uint32_t i = t + k * NT;
+      if (i < I) {
+        const uint32_t h = walk[k] ? s_res[i] : pos[k];
+        sync.hitring[(uint64_t)slot * sync.ring_stride + i] = h;
+        sync.tpfring[(uint64_t)slot * sync.ring_stride + i] = h == h0[k] ? tp0[k] : __uint_as_float(psk::kNoTpfBits);
+      }
+    }
+    __syncthreads();
+    if (t == 0) {
+      s_nwalk = 0;
+      __threadfence();  // the row's hits before its flag
+      psk::st_release_u32(sync.ready + s, 1u);
+    }
+  }
+}
+
+// Deciding block.  Thread t < NTI owns instances t * IPT .. t * IPT + IPT - 1; thread NTI (first
+// lane of the last warp) signals.  Block reductions: each warp reduces its lanes with
+// single-instruction warp reductions, writes one partial, and after the barrier every warp reduces
+// the partials itself (no second barrier).
+template <int IPT>
+__device__ void decide_rows(const psk::RowPre* __restrict__ rows, uint32_t R, uint32_t I, psk::StateSoA committed,
+                            psk::StateSoA pending, const psk::DevModel& m, int32_t* assign, uint8_t* __restrict__ path,
+                            uint32_t* __restrict__ hit_chosen, uint32_t* err, const psk::GreedySync& sync,
+                            unsigned long long* smem_raw) {
+  const uint32_t Ip = sync.ring_stride;  // I rounded up to a multiple of 4
+  // Ip is a multiple of 4, so every array below starts 16-byte aligned or at its own alignment.
+  uint32_t* s_hit = reinterpret_cast<uint32_t*>(smem_raw);        // [4][Ip] probed hits of rows r .. r + 3
+  float* s_tpf = reinterpret_cast<float*>(s_hit + 4 * Ip);        // [4][Ip] T_pf at those hits
+  uint32_t* s_ovr = reinterpret_cast<uint32_t*>(s_tpf + 4 * Ip);  // [2][Ip] lcp raises for the next row
+  int64_t* s_q = reinterpret_cast<int64_t*>(s_ovr + 2 * Ip);
   int64_t* s_S = s_q + I;
   int64_t* s_M = s_S + I;
-  int32_t* s_b = reinterpret_cast<int32_t*>(s_M + I);
+  uint64_t* s_key0 = reinterpret_cast<uint64_t*>(s_M + I);        // class-0 key bits of (b, qr)
+  psk::InstTerms* s_it = reinterpret_cast<psk::InstTerms*>(s_key0 + I);
+  int32_t* s_b = reinterpret_cast<int32_t*>(s_it + I);
   int32_t* s_qr = s_b + I;
   int32_t* s_Bmax = s_qr + I;
-  uint32_t* s_end = reinterpret_cast<uint32_t*>(s_Bmax + I);  // chain end of the last request on i
-  uint32_t* s_wres = s_end + I;                                // search start / result per instance
-  uint32_t* s_walk = s_wres + I;                               // instances handed to a warp search
-  psk::InstTerms* s_it = reinterpret_cast<psk::InstTerms*>(s_walk + I);
-  uint8_t* s_touched = reinterpret_cast<uint8_t*>(s_it + I);
+  int32_t* s_room = s_Bmax + I;                                    // kv_room(S, M_KV)
   __shared__ psk::RowPre s_row[8];  // rows r .. r + kRingAhead (a ring of 8 so no reader is overtaken)
-  __shared__ float s_red_w[32];
-  __shared__ int s_red_a[32];
-  __shared__ PickKey s_red_k[32];
-  __shared__ uint32_t s_nwalk[2];
+  __shared__ int32_t s_jm[8];       // pick of request x in s_jm[x & 7] (-1: rejected)
+  __shared__ uint32_t s_red_w[32];  // per-warp W_min (order-preserving bits), 0 = no pair in A
+  __shared__ uint64_t s_red_key[32];
+  __shared__ uint32_t s_red_i[32];
+  __shared__ uint32_t s_red_h[32];
 
   const int t = threadIdx.x;
   const int NT = blockDim.x;
-  const int NTI = NT - 32;  // threads owning instances; the last warp signals
+  const int NTI = NT - 32;
   const bool sig = t == NTI;
   const int lane = t & 31;
   const int warp = t >> 5;
   const int NW = NT >> 5;
-  // instance k of this thread (out of range for the signalling warp)
-  auto own = [&](int k) -> uint32_t { return t < NTI ? (uint32_t)(t + k * NTI) : 0xFFFFFFFFu; };
+  const uint32_t i0 = (uint32_t)t * IPT;  // first owned instance (>= I for the signalling warp)
+  const bool owner = t < NTI;
+  auto key0_bits = [](int32_t b, int32_t qr) -> uint64_t {
+    return ((uint64_t)((1u << 18) - 1u - (uint32_t)b) << 44) | (uint64_t)(uint32_t)qr;
+  };
 
   for (uint32_t i = t; i < I; i += NT) {
     s_b[i] = committed.b[i];
@@ -427,286 +566,165 @@ greedy_search_kernel(const psk::RowPre* __restrict__ rows, const uint64_t* __res
     s_S[i] = committed.S[i];
     s_M[i] = committed.M[i];
     s_Bmax[i] = committed.Bmax[i];
-    s_end[i] = 0;
-    s_touched[i] = 0;
     s_it[i] = psk::inst_terms(m, s_b[i], s_qr[i], s_q[i], s_Bmax[i]);
+    s_room[i] = psk::kv_room(s_S[i], s_M[i]);
+    s_key0[i] = key0_bits(s_b[i], s_qr[i]);
   }
+  for (uint32_t i = t; i < 2 * Ip; i += NT) s_ovr[i] = 0u;
+  if (t < 8) s_jm[t] = -1;
   if (t < kRingAhead * psk::kRowWords) {  // rows 0 .. kRingAhead - 1
     const uint32_t rr = (uint32_t)(t / psk::kRowWords);
     if (rr < R)
       reinterpret_cast<uint4*>(&s_row[rr])[t % psk::kRowWords] =
           __ldg(reinterpret_cast<const uint4*>(rows + rr) + (t % psk::kRowWords));
   }
-  if (t < 2) s_nwalk[t] = 0;
-
-  // hit and T_pf at that hit of rows r .. r + 2 (T_pf from the probe; kNoTpfBits once the greedy
-  // changed the hit)
-  uint32_t hr[IPT], h1[IPT], h2[IPT];
-  float tr[IPT], t1[IPT], t2[IPT];
-  uint64_t key1[IPT];
-  bool need1[IPT];
-#pragma unroll
-  for (int k = 0; k < IPT; ++k) {
-    const uint32_t i = own(k);
-    hr[k] = (i < I && R > 0) ? __ldg(hit0 + i) : 0u;
-    h1[k] = (i < I && R > 1) ? __ldg(hit0 + (uint64_t)I + i) : 0u;
-    h2[k] = (i < I && R > 2) ? __ldg(hit0 + 2ull * I + i) : 0u;
-    tr[k] = (i < I && R > 0) ? __ldg(tpf0 + i) : 0.0f;
-    t1[k] = (i < I && R > 1) ? __ldg(tpf0 + (uint64_t)I + i) : 0.0f;
-    t2[k] = (i < I && R > 2) ? __ldg(tpf0 + 2ull * I + i) : 0.0f;
-    key1[k] = 0;
-    need1[k] = false;
-  }
-  int32_t jm[psk::kLcpBack];  // jm[d] = pick of request r - 1 - d
-#pragma unroll
-  for (int d = 0; d < psk::kLcpBack; ++d) jm[d] = -1;
-  int32_t jp_pre[3] = {-1, -1, -1};  // picks of row r + 2's parent and two next ancestors, loaded a step ahead
   bool timed_out = false;
+  if (sig) {
+    for (uint32_t x = 0; x < 2 && x < R && !timed_out; ++x) timed_out = !wait_flag(sync.ready + x, err);
+  }
   __syncthreads();
+  // hits of rows 0 and 1, one copy group each (each thread copies and later reads only its own)
+  static_assert(IPT == 1 || IPT == 2 || IPT == 4, "one 4-, 8- or 16-byte copy per array and row");
+  auto copy_row = [&](uint32_t x) {
+    if (owner && i0 < I) {
+      const uint64_t src = (uint64_t)(x % psk::kHitSlots) * Ip + i0;
+      const uint32_t dst = (x & 3u) * Ip + i0;
+      psk::cp_async_bytes<4 * IPT>(s_hit + dst, sync.hitring + src);
+      psk::cp_async_bytes<4 * IPT>(s_tpf + dst, sync.tpfring + src);
+    }
+  };
+  if (R > 0) copy_row(0);
+  psk::cp_async_commit();
+  if (R > 1) copy_row(1);
+  psk::cp_async_commit();
+
+  int32_t jprev = -1;  // pick of request r - 1
+  uint32_t hr[IPT];
 
   for (uint32_t r = 0; r < R; ++r) {
     const psk::RowPre& cur = s_row[r & 7];
-    const uint32_t nb = cur.nb;
-    // ---- P0: ring refill, stages A-C, corrections and row evaluation -----------------------------
-    // Refill the ring kRingAhead rows ahead: one copy group per step (empty past the window's end),
-    // waited for two steps later, so the copy's latency stays off the step.
-    if (t < psk::kRowWords) {
-      if (r + kRingAhead < R)
-        psk::cp_async16(reinterpret_cast<uint4*>(&s_row[(r + kRingAhead) & 7]) + t,
-                        reinterpret_cast<const uint4*>(rows + r + kRingAhead) + t);
-      psk::cp_async_commit();
-    }
-    // The signalling thread starts reading job r - (kLag - 2)'s done flag now; it is checked before
-    // the second barrier.
-    uint32_t done_seen = 1u;
-    if (sig && r >= psk::kLag - 2 && !timed_out) done_seen = psk::ld_acquire_u32(sync.done + (r - (psk::kLag - 2)));
-    // picks of row r + 3's ancestors when they are old enough to be in global memory (instance
-    // threads only: the signalling thread keeps no loads in flight)
-    int32_t jp_next[3] = {-1, -1, -1};
-    if (t < NTI && r + 3 < R) {
-      const psk::RowPre& x3 = s_row[(r + 3) & 7];
-      const int32_t a3[3] = {x3.par, x3.anc[0], x3.anc[1]};
-#pragma unroll
-      for (int q = 0; q < 3; ++q)
-        if (a3[q] >= 0 && (int64_t)a3[q] <= (int64_t)r - (psk::kLag - 1)) jp_next[q] = __ldcg(assign + a3[q]);
-    }
-    uint32_t h3[IPT];
-    float t3[IPT];
-#pragma unroll
-    for (int k = 0; k < IPT; ++k) {
-      const uint32_t i = own(k);
-      h3[k] = (i < I && r + 3 < R) ? __ldg(hit0 + (uint64_t)(r + 3) * I + i) : 0u;
-      t3[k] = (i < I && r + 3 < R) ? __ldg(tpf0 + (uint64_t)(r + 3) * I + i) : 0.0f;
-    }
-    uint64_t key2[IPT];
-    bool need2[IPT];
-    if (r + 2 < R) {
-      const psk::RowPre& x2 = s_row[(r + 2) & 7];
-      // An ancestor's chain is a prefix of this one; on the instance that took it, the probe goes
-      // to its end.  It counts only if its inserts are in every probe snapshot: a <= (r + 2) - kLag,
-      // i.e. its distance d = r + 2 - a is at least kLag; its pick is jm[d - 3] while that is still
-      // in registers, else the one loaded from global memory a step ahead.
-      const int32_t a2[3] = {x2.par, x2.anc[0], x2.anc[1]};
-      const uint32_t a2nb[3] = {x2.par_nb, x2.anc_nb[0], x2.anc_nb[1]};
-      int32_t jp[3];
-#pragma unroll
-      for (int q = 0; q < 3; ++q) {
-        const int64_t a = a2[q];
-        jp[q] = -1;
-        if (a >= 0) {
-          const int64_t d = (int64_t)r + 2 - a;
-          if (d == psk::kLag) jp[q] = jm[psk::kLag - 3];
-          else if (d == psk::kLag + 1) jp[q] = jm[psk::kLag - 2];
-          else if (d >= psk::kLag + 2) jp[q] = jp_pre[q];
-        }
-      }
-#pragma unroll
-      for (int k = 0; k < IPT; ++k) {
-        const uint32_t i = own(k);
-        uint32_t pos = h2[k];
-#pragma unroll
-        for (int q = 0; q < 3; ++q)
-          if ((int32_t)i == jp[q] && a2nb[q] > pos) pos = a2nb[q];
-        need2[k] = i < I && s_touched[i] && pos < x2.nb;
-        key2[k] = need2[k] ? __ldg(hash + x2.off + pos) : 0ull;
-        if (pos != h2[k]) t2[k] = __uint_as_float(psk::kNoTpfBits);
-        h2[k] = pos;
-      }
-    } else {
-#pragma unroll
-      for (int k = 0; k < IPT; ++k) {
-        need2[k] = false;
-        key2[k] = 0;
-      }
-    }
-    ulonglong2 pv0[IPT], pv1[IPT];
-    uint64_t home1[IPT];
-#pragma unroll
-    for (int k = 0; k < IPT; ++k) {
-      const uint32_t i = own(k);
-      if (need1[k]) {
-        home1[k] = psk::delta_home(key1[k], nslots);
-        pv0[k] = __ldcg(reinterpret_cast<const ulonglong2*>(delta + home1[k]));
-        pv1[k] = __ldcg(reinterpret_cast<const ulonglong2*>(delta + psk::delta_next(home1[k], nslots)));
-      } else {
-        home1[k] = 0;
-        pv0[k] = make_ulonglong2(0ull, 0ull);
-        pv1[k] = make_ulonglong2(0ull, 0ull);
-      }
-    }
-
-    // Pass 1: hit corrections, W and the capacity guard; W_min over A.
+    // ---- P0: row-constant refill, row r's hits, pass 1 ------------------------------------------
+    if (t < psk::kRowWords && r + kRingAhead < R)
+      psk::cp_async16(reinterpret_cast<uint4*>(&s_row[(r + kRingAhead) & 7]) + t,
+                      reinterpret_cast<const uint4*>(rows + r + kRingAhead) + t);
+    uint32_t ready_seen = 1u;
+    if (sig && r + 2 < R && !timed_out) ready_seen = psk::ld_acquire_u32(sync.ready + r + 2);
+    psk::cp_async_wait_group<1>();  // this thread's copies of row r (and row constants <= r + 4)
     const psk::RowConst rc = row_of(cur);
-    psk::PairW ev[IPT];
-    float wmin = INFINITY;
-    bool anyA = false;
+    const uint32_t lcp0 = cur.lcp[0];
+    const uint32_t* hrow = s_hit + (r & 3u) * Ip;
+    const float* trow = s_tpf + (r & 3u) * Ip;
+    uint32_t* orow = s_ovr + (r & 1u) * Ip;
+    float Wk[IPT], tpk[IPT];
+    bool inA[IPT];
+    uint32_t wbest = 0xFFFFFFFFu;  // order-preserving bits of this thread's W_min over A
 #pragma unroll
     for (int k = 0; k < IPT; ++k) {
-      const uint32_t i = own(k);
-      if (i < I) {
-        uint32_t h = hr[k];
-#pragma unroll
-        for (int d = 0; d < psk::kLcpBack; ++d)
-          if ((int32_t)i == jm[d] && cur.lcp[d] > h) h = cur.lcp[d];
-        const float tp = h == hr[k] ? tr[k] : __uint_as_float(psk::kNoTpfBits);
-        hr[k] = h;
-        ev[k] = psk::pair_w(m, rc, h, tp, s_it[i], s_S[i], s_M[i]);
-        if (ev[k].inA) {
-          wmin = fminf(wmin, ev[k].W);
-          anyA = true;
+      const uint32_t i = i0 + k;
+      inA[k] = false;
+      if (owner && i < I) {
+        const uint32_t hb = hrow[i];
+        uint32_t h = hb;
+        const uint32_t ov = orow[i];
+        if (ov) {
+          orow[i] = 0u;
+          if (ov > h) h = ov;
         }
-      } else {
-        ev[k].inA = false;
+        if ((int32_t)i == jprev && lcp0 > h) h = lcp0;
+        hr[k] = h;
+        // T_pf at the hit: the ring's value unless it is marked unknown (the probe blocks raised the
+        // hit) or the hit was raised here; W = T_pf(n, c) - T_pf(0, L)
+        const float tb = trow[i];
+        tpk[k] = (h == hb && __float_as_uint(tb) != psk::kNoTpfBits) ? tb : psk::t_pf_of_hit(m, rc.L, h);
+        Wk[k] = __fsub_rn(tpk[k], rc.t_cached);
+        const psk::InstTerms& it = s_it[i];
+        inA[k] = it.okB && (int32_t)rc.L <= s_room[i];
+        if (inA[k]) wbest = min(wbest, psk::f2ord(Wk[k]));
       }
     }
-    wmin = psk::warp_fmin(wmin);
-    anyA = __any_sync(0xffffffffu, anyA);
-    if (lane == 0) {
-      s_red_w[warp] = wmin;
-      s_red_a[warp] = anyA ? 1 : 0;
-    }
+    wbest = __reduce_min_sync(0xffffffffu, wbest);
+    if (lane == 0) s_red_w[warp] = wbest;
     __syncthreads();  // (C)
 
-    // ---- P1: W_min, admission classes, argmin; row r + 1's probes; wait for job r - 3 -------------
-    {
-      const float v = lane < NW ? s_red_w[lane] : INFINITY;
-      const bool a = lane < NW ? (s_red_a[lane] != 0) : false;
-      wmin = psk::warp_fmin(v);
-      anyA = __any_sync(0xffffffffu, a);
-    }
-    // Pass 2: latencies and the admission class of the pairs in C only; the argmin key.
-    PickKey best{psk::kNoKeyCi, 0u, ~0ull};
+    // ---- P1: W_min, pass 2, the row's argmin; lcp raises for row r + 1; row r + 2 ready ----------
+    const uint32_t wmin_o = __reduce_min_sync(0xffffffffu, lane < NW ? s_red_w[lane] : 0xFFFFFFFFu);
+    const bool anyA = wmin_o != 0xFFFFFFFFu;  // a W of a pair in A never maps to all ones (not NaN)
+    const float wmin = psk::ord2f(wmin_o);
+    uint64_t bkey = psk::kNoKey;
+    uint32_t binst = 0xFFFFFFFFu, bh = 0u;
 #pragma unroll
     for (int k = 0; k < IPT; ++k) {
-      const uint32_t i = own(k);
-      if (i < I && ev[k].inA && psk::pair_in_c(rc, ev[k].W, wmin)) {
+      const uint32_t i = i0 + k;
+      if (owner && i < I && inA[k] && psk::pair_in_c(rc, Wk[k], wmin)) {
+        const psk::InstTerms it = s_it[i];
         const int64_t q = s_q[i];
+        const int64_t S = s_S[i];
+        psk::PairW x;
+        x.W = Wk[k];
+        x.tpf = tpk[k];
+        x.n = (int64_t)rc.L - 16 * (int64_t)hr[k];
+        x.inA = true;
         float tpot, ttft;
-        psk::pair_lat(m, rc, ev[k], s_it[i], q, s_S[i], &tpot, &ttft);
-        const uint32_t cls = psk::pair_admitted(m, rc, tpot, ttft) ? 0u : 1u;
-        const PickKey kk{(cls << 28) | i, hr[k], psk::pair_value(cls, hr[k], s_b[i], s_qr[i], q, ev[k].n)};
-        if (pick_less(kk, best)) best = kk;
-      }
-    }
-    best = warp_pick(best);
-    if (lane == 0) s_red_k[warp] = best;
-    bool walked[IPT];
-#pragma unroll
-    for (int k = 0; k < IPT; ++k) {
-      const uint32_t i = own(k);
-      walked[k] = false;
-      if (need1[k]) {
-        int v = psk::delta_slot_verdict(pv0[k], key1[k], i + 1);
-        if (v < 0) v = psk::delta_slot_verdict(pv1[k], key1[k], i + 1);
-        const bool present = v >= 0 ? v == 1
-                                    : psk::delta_contains_from(delta, nslots, i, key1[k],
-                                                               psk::delta_next(psk::delta_next(home1[k], nslots), nslots));
-        if (present) {
-          const uint32_t x = atomicAdd(&s_nwalk[(r + 1) & 1], 1u);
-          s_walk[x] = i;
-          s_wres[i] = h1[k];
-          walked[k] = true;
+        psk::pair_lat(m, rc, x, it, q, S, &tpot, &ttft);
+        const uint64_t key = psk::pair_admitted(m, rc, tpot, ttft)
+                                 ? psk::packed_key(0u, s_key0[i] | ((uint64_t)((1u << 26) - 1u - hr[k]) << 18))
+                                 : psk::packed_key(1u, (uint64_t)(q + x.n) * (uint64_t)(uint32_t)it.Bp);
+        if (key < bkey) {  // instances ascend within a thread, so ties keep the lowest
+          bkey = key;
+          binst = i;
+          bh = hr[k];
         }
       }
     }
-    // rows <= r + kRingAhead - 2 are in (the next step reads row r + 4)
-    if (t < psk::kRowWords) psk::cp_async_wait_group<2>();
-    // Row r + 2's probes (issued in the next step) need every insert of requests <= r + 2 - kLag;
-    // the earlier jobs were waited for in earlier steps.
-    if (sig && done_seen == 0u) {
-      const uint64_t t0 = psk::globaltimer_ns();
-      while (psk::ld_acquire_u32(sync.done + (r - (psk::kLag - 2))) == 0u) {
-        if (psk::globaltimer_ns() - t0 > kWaitNs) {
-          atomicOr(err, psk::kErrTimeout);
-          timed_out = true;
-          break;
-        }
+    {
+      uint64_t wk;
+      uint32_t wi, wh;
+      psk::warp_pick_min(bkey, binst, bh, &wk, &wi, &wh);
+      if (lane == 0) {
+        s_red_key[warp] = wk;
+        s_red_i[warp] = wi;
+        s_red_h[warp] = wh;
       }
     }
+    // Row r + 1's raises from requests r - 1 .. r - kLag + 1 (thread d - 1 takes request r - d); the
+    // raise from request r itself is applied in registers next step.
+    if (t < psk::kLcpBack - 1 && r + 1 < R) {
+      const uint32_t d = (uint32_t)t + 1u;
+      const int32_t jd = r >= d ? s_jm[(r - d) & 7u] : -1;
+      const uint32_t v = s_row[(r + 1) & 7].lcp[d];
+      if (jd >= 0 && v > 0u) atomicMax(s_ovr + ((r + 1) & 1u) * Ip + (uint32_t)jd, v);
+    }
+    if (sig && ready_seen == 0u) timed_out = !wait_flag(sync.ready + r + 2, err);
     __syncthreads();  // (D)
 
-    // ---- P2: the pick, its state, its insert job; searches for row r + 1 --------------------------
-    {
-      const PickKey o = lane < NW ? s_red_k[lane] : PickKey{psk::kNoKeyCi, 0u, ~0ull};
-      best = warp_pick(o);
-    }
-    const bool pick = anyA && best.ci != psk::kNoKeyCi;
-    const uint32_t j = best.ci & 0x0FFFFFFFu;
-    const uint32_t hj = pick ? best.h : 0u;
+    // ---- P2: the pick, its state, its insert job; copies of row r + 2 ----------------------------
+    uint64_t key;
+    uint32_t j, hj;
+    psk::warp_pick_min(lane < NW ? s_red_key[lane] : psk::kNoKey, lane < NW ? s_red_i[lane] : 0xFFFFFFFFu,
+                       lane < NW ? s_red_h[lane] : 0u, &key, &j, &hj);
+    const bool pick = anyA && key != psk::kNoKey;
+    if (!pick) hj = 0u;
     if (sig) {
       assign[r] = pick ? (int32_t)j : -1;
-      path[r] = pick ? (uint8_t)(best.ci >> 28) : (uint8_t)2;
+      path[r] = pick ? (uint8_t)(key >> 62) : (uint8_t)2;
       hit_chosen[r] = hj;
-      s_nwalk[r & 1] = 0;
-      sync.jobs[r] = ((unsigned long long)hj << 32) | (pick ? j : 0xFFFFFFFFu);
-      psk::st_release_u32(sync.pub, r + 1);
+      s_jm[r & 7u] = pick ? (int32_t)j : -1;
+      psk::st_relaxed_u64(sync.jobs + r, kJobValid | ((unsigned long long)hj << 32) | (pick ? j : 0xFFFFFFFFu));
     }
-    if (pick && (j % (uint32_t)NTI) == (uint32_t)t) {
+    if (pick && owner && j >= i0 && j < i0 + IPT) {
       s_qr[j] += 1;
       s_q[j] += (int64_t)rc.L - 16 * (int64_t)hj;
       s_S[j] += (int64_t)rc.L;
-      s_end[j] = nb;
-      s_touched[j] = 1;
       s_it[j] = psk::inst_terms(m, s_b[j], s_qr[j], s_q[j], s_Bmax[j]);
+      s_room[j] = psk::kv_room(s_S[j], s_M[j]);
+      s_key0[j] = key0_bits(s_b[j], s_qr[j]);
     }
-    const uint32_t nwalk = r + 1 < R ? s_nwalk[(r + 1) & 1] : 0u;
-    if (nwalk) {
-      const psk::RowPre& x1 = s_row[(r + 1) & 7];
-      const uint64_t xoff = x1.off, xnb = x1.nb;
-      for (uint32_t x = warp; x < nwalk; x += NW) {
-        const uint32_t i = s_walk[x];
-        auto cached = [&](uint64_t k) {
-          return k < xnb && psk::delta_contains(delta, nslots, i, __ldg(hash + xoff + k));
-        };
-        const uint64_t hnew = psk::warp_first_miss_search_hint((uint64_t)s_wres[i] + 1, xnb, s_end[i], cached);
-        __syncwarp();
-        if (lane == 0) s_wres[i] = (uint32_t)hnew;
-      }
-      __syncthreads();  // (E) search results visible to the owners
-#pragma unroll
-      for (int k = 0; k < IPT; ++k)
-        if (walked[k]) {
-          h1[k] = s_wres[own(k)];
-          t1[k] = __uint_as_float(psk::kNoTpfBits);
-        }
-    }
-#pragma unroll
-    for (int k = 0; k < IPT; ++k) {
-      tr[k] = t1[k];
-      t1[k] = t2[k];
-      t2[k] = t3[k];
-      hr[k] = h1[k];
-      h1[k] = h2[k];
-      key1[k] = key2[k];
-      need1[k] = need2[k];
-      h2[k] = h3[k];
-    }
-#pragma unroll
-    for (int d = psk::kLcpBack - 1; d > 0; --d) jm[d] = jm[d - 1];
-    jm[0] = pick ? (int32_t)j : -1;
-#pragma unroll
-    for (int q = 0; q < 3; ++q) jp_pre[q] = jp_next[q];
+    if (r + 2 < R && !timed_out) copy_row(r + 2);
+    psk::cp_async_commit();
+    jprev = pick ? (int32_t)j : -1;
   }
+  psk::cp_async_wait_all();
+  __syncthreads();
   for (uint32_t i = t; i < I; i += NT) {
     pending.b[i] = s_b[i];
     pending.qr[i] = s_qr[i];
@@ -717,18 +735,37 @@ greedy_search_kernel(const psk::RowPre* __restrict__ rows, const uint64_t* __res
   }
 }
 
-size_t greedy_search_smem(uint32_t I) {
-  return (size_t)I * (3 * sizeof(int64_t) + 3 * sizeof(int32_t) + 3 * sizeof(uint32_t) + sizeof(psk::InstTerms) + 1) + 16;
+template <int IPT>
+__global__ void __launch_bounds__(544, 1)
+greedy_pipe_kernel(const psk::RowPre* __restrict__ rows, const uint64_t* __restrict__ hash, uint32_t R, uint32_t I,
+                   const uint32_t* __restrict__ hit0, const float* __restrict__ tpf0, psk::StateSoA committed,
+                   psk::StateSoA pending, psk::DevModel m, psk::DeltaSlot* delta, uint64_t nslots, int32_t* assign,
+                   uint8_t* __restrict__ path, uint32_t* __restrict__ hit_chosen, uint32_t* err, psk::GreedySync sync) {
+  extern __shared__ unsigned long long smem_raw[];
+  if (blockIdx.x == 0) {
+    decide_rows<IPT>(rows, R, I, committed, pending, m, assign, path, hit_chosen, err, sync, smem_raw);
+  } else if (blockIdx.x <= kInsertBlocks) {
+    insert_blocks(rows, hash, R, delta, nslots, err, sync);
+  } else {
+    probe_rows<IPT>(rows, hash, R, I, hit0, tpf0, delta, nslots, err, sync, smem_raw);
+  }
+}
+
+size_t greedy_pipe_smem(uint32_t I, uint32_t Ip) {
+  const size_t decide = (size_t)I * (4 * sizeof(int64_t) + sizeof(psk::InstTerms) + 4 * sizeof(int32_t)) +
+                        (size_t)Ip * (2 + 4 + 4) * sizeof(uint32_t);
+  const size_t probe = (size_t)I * 3 * sizeof(uint32_t);
+  return decide > probe ? decide : probe;
 }
 
 template <int IPT>
-cudaError_t greedy_search_launch(const psk::RowPre* rows, const psk::WindowDev& w, uint32_t I, const uint32_t* hit0,
-                                 const float* tpf0, psk::StateSoA committed, psk::StateSoA pending, const psk::DevModel& m,
-                                 psk::DeltaSlot* delta, uint64_t nslots, int32_t* assign, uint8_t* path,
-                                 uint32_t* hit_chosen, uint32_t* err, const psk::GreedySync& sync, uint32_t nt,
-                                 cudaStream_t s) {
-  const size_t smem = greedy_search_smem(I);
-  cudaError_t e = cudaFuncSetAttribute(greedy_search_kernel<IPT>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+cudaError_t greedy_pipe_launch(const psk::RowPre* rows, const psk::WindowDev& w, uint32_t I, const uint32_t* hit0,
+                               const float* tpf0, psk::StateSoA committed, psk::StateSoA pending, const psk::DevModel& m,
+                               psk::DeltaSlot* delta, uint64_t nslots, int32_t* assign, uint8_t* path,
+                               uint32_t* hit_chosen, uint32_t* err, const psk::GreedySync& sync, uint32_t nt,
+                               cudaStream_t s) {
+  const size_t smem = greedy_pipe_smem(I, sync.ring_stride);
+  cudaError_t e = cudaFuncSetAttribute(greedy_pipe_kernel<IPT>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   const uint64_t* hash = w.hash;
   uint32_t R = w.R;
@@ -738,8 +775,9 @@ cudaError_t greedy_search_launch(const psk::RowPre* rows, const psk::WindowDev& 
   void* args[] = {(void*)&rows, (void*)&hash, (void*)&R, (void*)&I, (void*)&hit0, (void*)&tpf0, (void*)&c, (void*)&p,
                   (void*)&mm, (void*)&delta, (void*)&nslots, (void*)&assign, (void*)&path, (void*)&hit_chosen,
                   (void*)&err, (void*)&sy};
-  // all 1 + kHelpers blocks must be resident at once: they wait on one another
-  return cudaLaunchCooperativeKernel((const void*)greedy_search_kernel<IPT>, dim3(1 + kHelpers), dim3(nt), args, smem, s);
+  // all blocks must be resident at once: they wait on one another
+  return cudaLaunchCooperativeKernel((const void*)greedy_pipe_kernel<IPT>, dim3(1 + kInsertBlocks + kProbeBlocks),
+                                     dim3(nt), args, smem, s);
 }
 
 }  // namespace
@@ -770,20 +808,22 @@ cudaError_t launch_greedy_search(const psk::RowPre* rows, const psk::WindowDev& 
                                  const float* tpf0, psk::StateSoA committed, psk::StateSoA pending, const psk::DevModel& m,
                                  psk::DeltaSlot* delta, uint64_t delta_nslots, int32_t* assign, uint8_t* path,
                                  uint32_t* hit_chosen, uint32_t* err, const psk::GreedySync& sync, cudaStream_t s) {
-  cudaError_t e = w.R ? cudaMemsetAsync(sync.done, 0, (size_t)w.R * sizeof(uint32_t), s) : cudaSuccess;
-  if (e == cudaSuccess) e = cudaMemsetAsync(sync.pub, 0, sizeof(uint32_t), s);
+  if (w.R == 0) return cudaSuccess;
+  cudaError_t e = cudaMemsetAsync(sync.done, 0, (size_t)w.R * sizeof(uint32_t), s);
+  if (e == cudaSuccess) e = cudaMemsetAsync(sync.ready, 0, (size_t)w.R * sizeof(uint32_t), s);
+  if (e == cudaSuccess) e = cudaMemsetAsync(sync.jobs, 0, (size_t)w.R * sizeof(unsigned long long), s);
   if (e != cudaSuccess) return e;
-  // up to 512 threads each owning IPT instances (IPT = 1, 2 or 4 for I up to 2048), plus one
-  // signalling warp
+  // up to 512 threads each owning IPT consecutive instances (IPT = 1, 2 or 4 for I up to 2048),
+  // plus one signalling warp
   const uint32_t ipt = I <= 512 ? 1u : (I <= 1024 ? 2u : 4u);
   const uint32_t nt = ((I + ipt - 1) / ipt + 31) / 32 * 32 + 32;
-#define PS_GREEDY_S(IPT)                                                                                        \
-  return greedy_search_launch<IPT>(rows, w, I, hit0, tpf0, committed, pending, m, delta, delta_nslots, assign, path,  \
-                                   hit_chosen, err, sync, nt, s)
-  if (ipt == 1) PS_GREEDY_S(1);
-  if (ipt == 2) PS_GREEDY_S(2);
-  if (ipt == 4 && I <= 2048) PS_GREEDY_S(4);
-#undef PS_GREEDY_S
+#define PS_GREEDY_P(IPT)                                                                                      \
+  return greedy_pipe_launch<IPT>(rows, w, I, hit0, tpf0, committed, pending, m, delta, delta_nslots, assign, path, \
+                                 hit_chosen, err, sync, nt, s)
+  if (ipt == 1) PS_GREEDY_P(1);
+  if (ipt == 2) PS_GREEDY_P(2);
+  if (ipt == 4 && I <= 2048) PS_GREEDY_P(4);
+#undef PS_GREEDY_P
   return cudaErrorInvalidValue;
 }
 

@@ -88,12 +88,17 @@ struct __align__(16) RowPre {
 constexpr int kRowWords = (int)(sizeof(RowPre) / 16);
 static_assert(sizeof(RowPre) % 16 == 0 && kRowWords == 6, "RowPre is six 16-byte words");
 
-// Hand-off between the greedy block and the blocks that insert its picks' chains into the delta
-// table (one cooperative launch).
+// Hand-offs between the blocks of the pipelined greedy (one cooperative launch): the deciding
+// block publishes each decision as a job, insert blocks put the job's chain blocks into the delta
+// table, probe blocks turn hit0 rows into the hits the deciding block reads.
+constexpr uint32_t kHitSlots = 64;  // rows of probed hits in flight (a ring; more than kLag + 2)
 struct GreedySync {
-  unsigned long long* jobs;  // per request: hit of the pick << 32 | pick (0xFFFFFFFF = rejected)
-  uint32_t* done;            // per request: 1 once its insert block has finished its blocks
-  uint32_t* pub;             // number of requests published so far
+  unsigned long long* jobs;  // [R] 1 << 63 | hit of the pick << 32 | pick (0xFFFFFFFF = rejected); 0 = unpublished
+  uint32_t* done;            // [R] 1 once the job's blocks are in the delta table
+  uint32_t* ready;           // [R] 1 once the row's probed hits are in the ring
+  uint32_t* hitring;         // [kHitSlots][ring_stride] probed hits (row s in slot s % kHitSlots)
+  float* tpfring;            // [kHitSlots][ring_stride] T_pf at those hits (kNoTpfBits where it changed)
+  uint32_t ring_stride;      // I rounded up to a multiple of 4
 };
 
 // Window table from a chain's last block hash to the earliest request ending there.
@@ -361,6 +366,16 @@ __device__ __forceinline__ void st_release_u32(uint32_t* p, uint32_t v) {
   asm volatile("st.release.gpu.global.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
 }
 
+__device__ __forceinline__ unsigned long long ld_relaxed_u64(const unsigned long long* p) {
+  unsigned long long v;
+  asm volatile("ld.relaxed.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
+  return v;
+}
+
+__device__ __forceinline__ void st_relaxed_u64(unsigned long long* p, unsigned long long v) {
+  asm volatile("st.relaxed.gpu.global.u64 [%0], %1;" ::"l"(p), "l"(v) : "memory");
+}
+
 __device__ __forceinline__ uint64_t globaltimer_ns() {
   uint64_t x;
   asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(x));
@@ -371,6 +386,19 @@ __device__ __forceinline__ uint64_t globaltimer_ns() {
 __device__ __forceinline__ void cp_async16(void* smem, const void* gmem) {
   asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"((uint32_t)__cvta_generic_to_shared(smem)), "l"(gmem)
                : "memory");
+}
+
+// 4-, 8- or 16-byte asynchronous global -> shared copy (both addresses aligned to the size).
+template <int BYTES>
+__device__ __forceinline__ void cp_async_bytes(void* smem, const void* gmem) {
+  static_assert(BYTES == 4 || BYTES == 8 || BYTES == 16, "cp.async copies 4, 8 or 16 bytes");
+  if (BYTES == 16) {
+    cp_async16(smem, gmem);
+  } else {
+    asm volatile("cp.async.ca.shared.global [%0], [%1], %2;" ::"r"((uint32_t)__cvta_generic_to_shared(smem)),
+                 "l"(gmem), "n"(BYTES)
+                 : "memory");
+  }
 }
 
 __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
@@ -526,6 +554,11 @@ __device__ __forceinline__ bool mbar_wait_bounded(uint64_t* mbar, uint32_t parit
 // Every operation is an explicitly rounded fp32 intrinsic in the order the header documents, so
 // nothing is fused or reassociated.
 
+// int64 -> fp32, round to nearest: the 32-bit conversion when the value fits (the same result).
+__device__ __forceinline__ float i64_to_f32(int64_t v) {
+  return v == (int64_t)(int32_t)v ? __int2float_rn((int32_t)v) : __ll2float_rn(v);
+}
+
 // Eq. 6 with the Section 5.3 empirical C and C^2 terms.
 __device__ __forceinline__ float t_pf(const DevModel& m, float N, float C) {
   float t = __fadd_rn(m.a0, __fmul_rn(m.a1, N));
@@ -611,6 +644,13 @@ struct InstTerms {
   int32_t okB;  // B <= B_max
 };
 
+// Free KV room M_KV - S of an instance clamped to [-1, 2^31 - 1]: for 0 <= L < 2^30 the capacity
+// test S + L <= M_KV is L <= room.
+__device__ __forceinline__ int32_t kv_room(int64_t S, int64_t M) {
+  const int64_t d = M - S;
+  return d < 0 ? -1 : (d > 0x7FFFFFFFll ? 0x7FFFFFFF : (int32_t)d);
+}
+
 __device__ __forceinline__ InstTerms inst_terms(const DevModel& m, int32_t b, int32_t qr, int64_t q, int32_t Bmax) {
   InstTerms x;
   const int64_t Bp = (int64_t)b + qr + 1;
@@ -625,7 +665,7 @@ __device__ __forceinline__ InstTerms inst_terms(const DevModel& m, int32_t b, in
 // T_pf of a pair from its hit h: n = L - 16 h uncached tokens, c = 16 h cached.
 __device__ __forceinline__ float t_pf_of_hit(const DevModel& m, uint32_t L, uint32_t h) {
   const int64_t c = 16 * (int64_t)h;
-  return t_pf(m, __ll2float_rn((int64_t)L - c), __ll2float_rn(c));
+  return t_pf(m, i64_to_f32((int64_t)L - c), i64_to_f32(c));
 }
 
 // Marks a precomputed T_pf as not available (a NaN pattern T_pf never produces).
@@ -648,7 +688,7 @@ __device__ __forceinline__ PairW pair_w(const DevModel& m, const RowConst& rc, u
   PairW x;
   const int64_t c = 16 * (int64_t)h;
   x.n = (int64_t)rc.L - c;
-  x.tpf = __float_as_uint(tpf_in) == kNoTpfBits ? t_pf(m, __ll2float_rn(x.n), __ll2float_rn(c)) : tpf_in;
+  x.tpf = __float_as_uint(tpf_in) == kNoTpfBits ? t_pf(m, i64_to_f32(x.n), i64_to_f32(c)) : tpf_in;
   x.W = __fsub_rn(x.tpf, rc.t_cached);
   x.inA = it.okB && (S + (int64_t)rc.L <= M);
   return x;
@@ -657,10 +697,10 @@ __device__ __forceinline__ PairW pair_w(const DevModel& m, const RowConst& rc, u
 __device__ __forceinline__ void pair_lat(const DevModel& m, const RowConst& rc, const PairW& x, const InstTerms& it,
                                          int64_t q, int64_t S, float* tpot, float* ttft) {
   const int64_t Sp = S + (int64_t)rc.L;
-  float dec = __fadd_rn(it.dec0, __fmul_rn(m.b2, __ll2float_rn(Sp)));
+  float dec = __fadd_rn(it.dec0, __fmul_rn(m.b2, i64_to_f32(Sp)));
   dec = __fmul_rn(dec, it.f);
   if (m.interference_mode == 0) {
-    *tpot = __fadd_rn(dec, __fmul_rn(m.g_q, __ll2float_rn(q + x.n)));
+    *tpot = __fadd_rn(dec, __fmul_rn(m.g_q, i64_to_f32(q + x.n)));
   } else {
     const float den = m.lout > 1.0f ? m.lout : 1.0f;
     const float interf = (it.Bp > 1) ? __fdiv_rn(x.tpf, den) : 0.0f;
@@ -749,6 +789,37 @@ __device__ __forceinline__ float warp_fmin(float x) {
 }
 
 constexpr uint32_t kNoKeyCi = 0xFFFFFFFFu;  // class 15: worse than any real pair
+
+// (class, value) of a pair of C as one 64-bit key, class in the top two bits: class-0 values are
+// below 2^62 and class-1 values below 2^59 ((q + n) < 2^41 times (b + qr + 1) < 2^18), so the
+// unsigned order of the packed key is the lexicographic order of (class, value).
+__device__ __forceinline__ uint64_t packed_key(uint32_t cls, uint64_t v) { return ((uint64_t)cls << 62) | v; }
+constexpr uint64_t kNoKey = ~0ull;
+
+// Order-preserving map of a non-NaN float to an unsigned integer (for integer warp reductions).
+__device__ __forceinline__ uint32_t f2ord(float x) {
+  const uint32_t u = __float_as_uint(x);
+  return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+__device__ __forceinline__ float ord2f(uint32_t o) {
+  return __uint_as_float((o & 0x80000000u) ? (o & 0x7FFFFFFFu) : ~o);
+}
+
+// Warp argmin of (key, instance) with single-instruction reductions; every lane receives the
+// minimum and the winning lane's h.  Lanes without a pair pass (kNoKey, 0xFFFFFFFF).
+__device__ __forceinline__ void warp_pick_min(uint64_t key, uint32_t inst, uint32_t h, uint64_t* kout,
+                                              uint32_t* iout, uint32_t* hout) {
+  const uint32_t hi = (uint32_t)(key >> 32);
+  const uint32_t mhi = __reduce_min_sync(0xffffffffu, hi);
+  const uint32_t lo = hi == mhi ? (uint32_t)key : 0xFFFFFFFFu;
+  const uint32_t mlo = __reduce_min_sync(0xffffffffu, lo);
+  const bool eq = hi == mhi && (uint32_t)key == mlo;
+  const uint32_t mi = __reduce_min_sync(0xffffffffu, eq ? inst : 0xFFFFFFFFu);
+  const unsigned win = __ballot_sync(0xffffffffu, eq && inst == mi);
+  *hout = __shfl_sync(0xffffffffu, h, __ffs(win) - 1);
+  *kout = ((uint64_t)mhi << 32) | mlo;
+  *iout = mi;
+}
 
 }  // namespace psk
 
