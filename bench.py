@@ -115,14 +115,14 @@ class ClockSampler:
 def probe_algorithmic_bytes(st: dict, I: int, with_tpf: bool) -> tuple[int, int]:
     """Bytes the two probe kernels' algorithm must move in one launch, from the library's own
     counters of that launch (ps_last_probe_stats): one 32-byte sector per table lookup (the least a
-    random lookup can move), the staged chain blocks of the rows searched from scratch (8 B each),
-    the key of every lookup of a derived row (8 B, read from the chain), the earlier row's hits a
-    derived row starts from (4 B per instance), and per pair the u32 hit and, when the greedy pass
-    follows, the f32 T_pf written."""
+    random lookup can move), 8 B per chain block read (the key of a lookup, or a staged block), the
+    earlier row's hits a derived row starts from (4 B per instance), and per pair the u32 hit and,
+    when the greedy pass follows, the f32 T_pf written."""
     out_b = (4 + (4 if with_tpf else 0)) * I
-    scratch = 32 * st["lookups_scratch"] + 8 * st["staged_blocks"] + out_b * st["rows_scratch"]
-    derived = (32 + 8) * st["lookups_derived"] + (4 * I + out_b) * st["rows_derived"]
-    return int(scratch + derived), int(st["lookups_scratch"] + st["lookups_derived"])
+    lookups = st["lookups_scratch"] + st["lookups_derived"]
+    nbytes = (32 * lookups + 8 * st["chain_reads"] + out_b * (st["rows_scratch"] + st["rows_derived"])
+              + 4 * I * st["rows_derived"])
+    return int(nbytes), int(lookups)
 
 
 def oracle_sample(wl, seconds: float, max_rows: int | None = None):

@@ -303,7 +303,7 @@ PS_API ps_status ps_last_timings(ps_ctx* ctx, float* ms, uint32_t n);
  * (host array of n >= 6 entries):
  *   out[0] rows searched from scratch        out[1] rows derived from an earlier request's row
  *   out[2] table lookups in scratch rows     out[3] table lookups in derived rows
- *   out[4] chain blocks staged in shared memory (scratch rows)
+ *   out[4] chain blocks read from global memory (a lookup's key, or a block staged in shared memory)
  *   out[5] (row, instance) pairs searched past the earlier request's chain (derived rows)
  * A table lookup reads the key's two candidate buckets (2 x 64 bytes) and one overflow word.
  * All zero if no probe phase ran.  Synchronises the context's stream. */

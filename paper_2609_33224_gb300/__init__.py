@@ -297,7 +297,7 @@ class Scheduler:
         """Counters of the last probe phase (see ps_last_probe_stats)."""
         v = np.zeros(6, np.uint64)
         self._check(lib().ps_last_probe_stats(self._h, v.ctypes.data, 6))
-        names = ("rows_scratch", "rows_derived", "lookups_scratch", "lookups_derived", "staged_blocks",
+        names = ("rows_scratch", "rows_derived", "lookups_scratch", "lookups_derived", "chain_reads",
                  "pairs_derived")
         return dict(zip(names, (int(x) for x in v)))
 

@@ -58,6 +58,7 @@ struct ps_ctx {
   psk::GreedySync gsync{nullptr, nullptr, nullptr, nullptr, nullptr, 0u};
   psk::RowPre* d_rows = nullptr;      // per-request constants and relations (search mode greedy)
   psk::LastSlot* d_lastslot = nullptr;
+  psk::RowList scratch{nullptr, nullptr};  // rows the probe searches from scratch
   uint32_t lastslot_n = 0;
   psk::StateSoA st{}, pend{};
   uint64_t* d_off = nullptr;
@@ -270,9 +271,10 @@ ps_status run_probe_and_score(ps_ctx* c, const psk::WindowDev& wd, ps_scores* ou
   PS_TRY_CUDA(c, cudaMemsetAsync(c->d_stats, 0, kNumStats * sizeof(unsigned long long), c->stream));
   record(c, kEvProbe0);
   // window relations first: the probe derives the rows of requests that extend an earlier request
-  PS_TRY_CUDA(c, pskl::launch_relations(wd, c->model, c->d_lastslot, c->lastslot_n, c->d_rows, c->num_sms, c->stream));
+  PS_TRY_CUDA(c, pskl::launch_relations(wd, c->model, c->d_lastslot, c->lastslot_n, c->d_rows, c->scratch, c->num_sms,
+                                        c->stream));
   record(c, kEvRelDone);
-  PS_TRY_CUDA(c, pskl::launch_probe(c->d_slots, c->d_ovf, c->d_tdesc, c->I, wd, c->d_rows, hits, c->d_tpf,
+  PS_TRY_CUDA(c, pskl::launch_probe(c->d_slots, c->d_ovf, c->d_tdesc, c->I, wd, c->d_rows, c->scratch, hits, c->d_tpf,
                                     c->model, c->probe_grid, c->search, c->d_stats, c->ev[kEvProbeMid], c->stream));
   record(c, kEvProbe1);
   c->ev_used[0] = true;
@@ -381,7 +383,8 @@ ps_status ps_create(const ps_config* cfg, ps_ctx** out) {
             dalloc(c, &c->gsync.done, c->Rmax) == cudaSuccess && dalloc(c, &c->gsync.ready, c->Rmax) == cudaSuccess &&
             dalloc(c, &c->gsync.hitring, (size_t)psk::kHitSlots * c->gsync.ring_stride) == cudaSuccess &&
             dalloc(c, &c->gsync.tpfring, (size_t)psk::kHitSlots * c->gsync.ring_stride) == cudaSuccess &&
-            dalloc(c, &c->d_rows, c->Rmax) == cudaSuccess && dalloc(c, &c->d_lastslot, c->lastslot_n) == cudaSuccess;
+            dalloc(c, &c->d_rows, c->Rmax) == cudaSuccess && dalloc(c, &c->d_lastslot, c->lastslot_n) == cudaSuccess &&
+            dalloc(c, &c->scratch.rows, c->Rmax) == cudaSuccess && dalloc(c, &c->scratch.count, 1) == cudaSuccess;
   for (psk::StateSoA* s : {&c->st, &c->pend}) {
     ok = ok && dalloc(c, &s->b, I) == cudaSuccess && dalloc(c, &s->qr, I) == cudaSuccess &&
          dalloc(c, &s->q, I) == cudaSuccess && dalloc(c, &s->S, I) == cudaSuccess &&

@@ -124,7 +124,7 @@ ps_status ps_score_window_noalloc(const uint64_t* slots, const uint64_t* overflo
   const psk::TableDesc* td = reinterpret_cast<const psk::TableDesc*>(tables);
   const int grid = num_instances >= 64 ? d->probe_grid_large : d->probe_grid_small;
   const psk::DevModel dm = dev_model(*model);
-  if (pskl::launch_probe(slots, overflow_bits, td, num_instances, wd, nullptr, hits, nullptr, dm, grid,
+  if (pskl::launch_probe(slots, overflow_bits, td, num_instances, wd, nullptr, psk::RowList{nullptr, nullptr}, hits, nullptr, dm, grid,
                          probe_mode == PS_PROBE_SEARCH, nullptr, nullptr, s) != cudaSuccess)
     return PS_ERR_CUDA;
   const psk::StateSoA soa{const_cast<int32_t*>(state->b), const_cast<int32_t*>(state->qr),

@@ -9,10 +9,13 @@
 // the staging capacity are read from global memory (L1/L2-resident: the same block re-reads them).
 //   linear mode (any cache): each warp walks one instance at a time, 32 consecutive chain positions
 //     per step, __ballot_sync collecting the misses and __ffs finding the first.
-//   search mode (prefix-closed caches, where "block k cached" is monotone along the chain): each
-//     lane binary-searches its own instance.  All instances of a row share the chain length, so the
-//     32 lanes of a warp run the same number of steps in lock-step with 32 independent lookups in
-//     flight, and a pair costs about log2(nb) probes.
+//   search mode (prefix-closed caches, where "block k cached" is monotone along the chain): the
+//     rows without an earlier prefix in the window come as a list from the relations pass; a work
+//     item is (row, chunk of 256 instances), one lane per instance.  A lane first looks up the
+//     row's hint position and the one before it together: the hint is the shortest common prefix
+//     with the previous requests of the window, which on most instances is exactly the cached
+//     prefix (typically a shared system prompt), so most pairs end after one round trip; the
+//     others binary-search the rest of their range.
 //
 // Rows whose chain starts with the whole chain of an earlier request of the window (its base, from
 // the relations pass) are derived in a second pass instead: the two chains agree block by block up
@@ -27,7 +30,7 @@ namespace {
 constexpr uint32_t kStageBlocks = 4096;  // 32 KB of staged chain per thread block
 
 // Launch statistics (ps_last_probe_stats): each warp adds its threads' counts once, at the end.
-enum { kStatRowsScratch = 0, kStatRowsDerived, kStatLookupsScratch, kStatLookupsDerived, kStatStagedBlocks,
+enum { kStatRowsScratch = 0, kStatRowsDerived, kStatLookupsScratch, kStatLookupsDerived, kStatChainReads,
        kStatPairsDerived };
 
 __device__ __forceinline__ void add_stat(unsigned long long* p, uint64_t v) {
@@ -100,7 +103,73 @@ probe_hits_kernel(const uint64_t* __restrict__ slots, const uint64_t* __restrict
   if (stats) {
     add_stat(stats + kStatRowsScratch, n_rows);
     add_stat(stats + kStatLookupsScratch, n_look);
-    add_stat(stats + kStatStagedBlocks, n_staged);
+    add_stat(stats + kStatChainReads, n_staged);
+  }
+}
+
+// Hint of a row for the search: the shortest common chain prefix with the previous requests of
+// the window (0 if there are none).
+__device__ __forceinline__ uint32_t row_hint(const psk::RowPre* __restrict__ rows, uint32_t r) {
+  uint32_t hint = 0xFFFFFFFFu;
+#pragma unroll
+  for (int d = 0; d < psk::kLcpBack; ++d)
+    if ((uint32_t)d < r) hint = min(hint, __ldg(&rows[r].lcp[d]));
+  return hint == 0xFFFFFFFFu ? 0u : hint;
+}
+
+// Search mode, rows from the list: see the file comment.
+template <int WARPS>
+__global__ void __launch_bounds__(WARPS * 32)
+probe_search_kernel(const uint64_t* __restrict__ slots, const uint64_t* __restrict__ ovf,
+                    const psk::TableDesc* __restrict__ tdesc, uint32_t I, const uint64_t* __restrict__ off,
+                    const uint64_t* __restrict__ hash, const psk::RowPre* __restrict__ rows, psk::RowList list,
+                    PairOut out, unsigned long long* __restrict__ stats) {
+  constexpr uint32_t kChunk = WARPS * 32;
+  const uint32_t nchunk = (I + kChunk - 1) / kChunk;
+  const uint64_t items = (uint64_t)__ldg(list.count) * nchunk;
+  uint64_t n_look = 0, n_rows = 0;
+  for (uint64_t item = blockIdx.x; item < items; item += gridDim.x) {
+    const uint32_t r = __ldg(list.rows + item / nchunk);
+    const uint32_t chunk = (uint32_t)(item % nchunk);
+    if (threadIdx.x == 0 && chunk == 0) n_rows += 1;
+    const uint32_t i = chunk * kChunk + threadIdx.x;
+    if (i >= I) continue;
+    const uint64_t o = __ldg(off + r);
+    const uint64_t nb = __ldg(off + r + 1) - o;
+    const uint64_t* chain = hash + o;
+    const psk::TableDesc d = tdesc[i];
+    uint64_t lo = 0, hi = nb;  // the first miss lies in [lo, hi]
+    if (nb > 0) {
+      const uint64_t hint = row_hint(rows, r);
+      if (hint == 0 || hint >= nb) {
+        const uint64_t p = hint == 0 ? 0 : nb - 1;
+        n_look += 1;
+        const bool pr = psk::main_contains(slots, ovf, d, __ldg(chain + p));
+        if (pr) lo = p + 1; else hi = p;
+      } else {
+        const uint64_t k1 = __ldg(chain + hint - 1), k2 = __ldg(chain + hint);
+        psk::Lookup L1, L2;
+        psk::lookup_issue(slots, ovf, d, k1, L1);
+        psk::lookup_issue(slots, ovf, d, k2, L2);
+        n_look += 2;
+        const bool p1 = psk::lookup_finish(slots, ovf, d, k1, L1);
+        const bool p2 = psk::lookup_finish(slots, ovf, d, k2, L2);
+        if (!p1) hi = hint - 1;
+        else if (p2) lo = hint + 1;
+        else lo = hi = hint;
+      }
+    }
+    while (lo < hi) {
+      const uint64_t mid = (lo + hi) >> 1;
+      ++n_look;
+      if (psk::main_contains(slots, ovf, d, __ldg(chain + mid))) lo = mid + 1; else hi = mid;
+    }
+    out.put(r, I, i, (uint32_t)lo, out.tpf ? __ldg(out.L + r) : 0u);
+  }
+  if (stats) {
+    add_stat(stats + kStatRowsScratch, n_rows);
+    add_stat(stats + kStatLookupsScratch, n_look);
+    add_stat(stats + kStatChainReads, n_look);
   }
 }
 
@@ -153,6 +222,7 @@ probe_derived_kernel(const uint64_t* __restrict__ slots, const uint64_t* __restr
   if (stats) {
     add_stat(stats + kStatRowsDerived, n_rows);
     add_stat(stats + kStatLookupsDerived, n_look);
+    add_stat(stats + kStatChainReads, n_look);
     add_stat(stats + kStatPairsDerived, n_pairs);
   }
 }
@@ -166,6 +236,9 @@ int max_grid(int num_sms) {
   cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, probe_hits_kernel<WARPS, false>, WARPS * 32, smem);
   cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm2, probe_hits_kernel<WARPS, true>, WARPS * 32, smem);
   if (per_sm2 < per_sm) per_sm = per_sm2;
+  int per_sm3 = 0;
+  cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm3, probe_search_kernel<WARPS>, WARPS * 32, 0);
+  if (per_sm3 < per_sm) per_sm = per_sm3;
   if (per_sm < 1) per_sm = 1;
   return per_sm * num_sms;
 }
@@ -179,8 +252,8 @@ int probe_max_grid(uint32_t I, int num_sms) {
 }
 
 cudaError_t launch_probe(const uint64_t* slots, const uint64_t* ovf, const psk::TableDesc* tdesc, uint32_t I,
-                         const psk::WindowDev& w, const psk::RowPre* rows, uint32_t* hits, float* tpf,
-                         const psk::DevModel& m, int grid, int search, unsigned long long* stats,
+                         const psk::WindowDev& w, const psk::RowPre* rows, psk::RowList list, uint32_t* hits,
+                         float* tpf, const psk::DevModel& m, int grid, int search, unsigned long long* stats,
                          cudaEvent_t ev_mid, cudaStream_t s) {
   if (w.R == 0) return cudaSuccess;
   const PairOut out{hits, tpf, w.L, m};
@@ -189,8 +262,12 @@ cudaError_t launch_probe(const uint64_t* slots, const uint64_t* ovf, const psk::
   const size_t smem2 = (size_t)I * sizeof(uint32_t);
 #define PS_PROBE(W, S)                                                                                      \
   do {                                                                                                      \
-    probe_hits_kernel<W, S><<<g, W * 32, smem, s>>>(slots, ovf, tdesc, I, w.off, w.hash, w.R, rows, out,    \
-                                                   stats);                                                  \
+    if (S && rows && list.rows)                                                                             \
+      probe_search_kernel<W><<<grid, W * 32, 0, s>>>(slots, ovf, tdesc, I, w.off, w.hash, rows, list, out,   \
+                                                     stats);                                                \
+    else                                                                                                    \
+      probe_hits_kernel<W, S><<<g, W * 32, smem, s>>>(slots, ovf, tdesc, I, w.off, w.hash, w.R, rows, out,  \
+                                                     stats);                                                \
     cudaError_t e = cudaGetLastError();                                                                     \
     if (e != cudaSuccess || !rows) return e;                                                                \
     if (ev_mid) cudaEventRecord(ev_mid, s);                                                                 \

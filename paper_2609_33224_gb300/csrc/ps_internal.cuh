@@ -92,6 +92,13 @@ static_assert(sizeof(RowPre) % 16 == 0 && kRowWords == 6, "RowPre is six 16-byte
 // block publishes each decision as a job, insert blocks put the job's chain blocks into the delta
 // table, probe blocks turn hit0 rows into the hits the deciding block reads.
 constexpr uint32_t kHitSlots = 64;  // rows of probed hits in flight (a ring; more than kLag + 2)
+// Rows of a window whose hits are searched from scratch (no earlier request of the window is a
+// prefix of theirs), in no particular order: filled by the relations pass, read by the probe.
+struct RowList {
+  uint32_t* rows;   // [R]
+  uint32_t* count;  // [1]
+};
+
 struct GreedySync {
   unsigned long long* jobs;  // [R] 1 << 63 | hit of the pick << 32 | pick (0xFFFFFFFF = rejected); 0 = unpublished
   uint32_t* done;            // [R] 1 once the job's blocks are in the delta table
@@ -145,31 +152,43 @@ __device__ __forceinline__ bool ovf_bit(const uint64_t* ovf, const TableDesc& d,
   return (ovf[d.ovf + (b >> 6)] >> (b & 63)) & 1ull;
 }
 
-// Membership in an instance's main table.  Both candidate buckets (2 x 4 x 16-byte loads) and the
-// overflow word are requested before any comparison.  LOAD selects the read path: the read-only
-// path for kernels that never write the tables, the L2-coherent path for the table writers.
-template <bool RO = true>
-__device__ __forceinline__ bool main_contains(const uint64_t* __restrict__ slots, const uint64_t* __restrict__ ovf,
-                                              const TableDesc d, uint64_t key) {
-  if (key == kEmpty || key == kTomb) return false;
-  const uint32_t b1 = fastrange32(key, d.nbkt);
-  const uint32_t b2 = fastrange32(remix(key), d.nbkt);
-  const ulonglong2* l1 = reinterpret_cast<const ulonglong2*>(slots + d.base + (uint64_t)b1 * kBucketSlots);
-  const ulonglong2* l2 = reinterpret_cast<const ulonglong2*>(slots + d.base + (uint64_t)b2 * kBucketSlots);
+// Membership in an instance's main table, in two parts so that several lookups can have their
+// loads in flight together: lookup_issue requests both candidate buckets (2 x 4 x 16-byte loads)
+// and the overflow word, lookup_finish compares (and, rarely, follows the overflow run after b1).
+// RO selects the read path: the read-only path for kernels that never write the tables, the
+// L2-coherent path for the table writers.
+struct Lookup {
   ulonglong2 v[8];
+  uint64_t ow;
+  uint32_t b1;
+};
+
+template <bool RO = true>
+__device__ __forceinline__ void lookup_issue(const uint64_t* __restrict__ slots, const uint64_t* __restrict__ ovf,
+                                             const TableDesc& d, uint64_t key, Lookup& L) {
+  L.b1 = fastrange32(key, d.nbkt);
+  const uint32_t b2 = fastrange32(remix(key), d.nbkt);
+  const ulonglong2* l1 = reinterpret_cast<const ulonglong2*>(slots + d.base + (uint64_t)L.b1 * kBucketSlots);
+  const ulonglong2* l2 = reinterpret_cast<const ulonglong2*>(slots + d.base + (uint64_t)b2 * kBucketSlots);
 #pragma unroll
   for (int k = 0; k < 4; ++k) {
-    v[k] = RO ? __ldg(l1 + k) : __ldcg(l1 + k);
-    v[4 + k] = RO ? __ldg(l2 + k) : __ldcg(l2 + k);
+    L.v[k] = RO ? __ldg(l1 + k) : __ldcg(l1 + k);
+    L.v[4 + k] = RO ? __ldg(l2 + k) : __ldcg(l2 + k);
   }
-  const uint64_t* ow_p = ovf + d.ovf + (b1 >> 6);
-  const uint64_t ow = RO ? __ldg(ow_p) : __ldcg(ow_p);
+  const uint64_t* ow_p = ovf + d.ovf + (L.b1 >> 6);
+  L.ow = RO ? __ldg(ow_p) : __ldcg(ow_p);
+}
+
+template <bool RO = true>
+__device__ __forceinline__ bool lookup_finish(const uint64_t* __restrict__ slots, const uint64_t* __restrict__ ovf,
+                                              const TableDesc& d, uint64_t key, const Lookup& L) {
+  if (key == kEmpty || key == kTomb) return false;
   bool hit = false;
 #pragma unroll
-  for (int k = 0; k < 8; ++k) hit |= (v[k].x == key) | (v[k].y == key);
+  for (int k = 0; k < 8; ++k) hit |= (L.v[k].x == key) | (L.v[k].y == key);
   if (hit) return true;
-  if (!((ow >> (b1 & 63)) & 1ull)) return false;
-  uint32_t b = b1;  // rare: follow the overflow run after b1
+  if (!((L.ow >> (L.b1 & 63)) & 1ull)) return false;
+  uint32_t b = L.b1;  // rare: follow the overflow run after b1
   for (uint32_t p = 1; p < d.nbkt; ++p) {
     b = (b + 1 == d.nbkt) ? 0u : b + 1;
     const ulonglong2* l = reinterpret_cast<const ulonglong2*>(slots + d.base + (uint64_t)b * kBucketSlots);
@@ -182,6 +201,15 @@ __device__ __forceinline__ bool main_contains(const uint64_t* __restrict__ slots
     if (!(((RO ? __ldg(q) : __ldcg(q)) >> (b & 63)) & 1ull)) return false;
   }
   return false;
+}
+
+template <bool RO = true>
+__device__ __forceinline__ bool main_contains(const uint64_t* __restrict__ slots, const uint64_t* __restrict__ ovf,
+                                              const TableDesc d, uint64_t key) {
+  if (key == kEmpty || key == kTomb) return false;
+  Lookup L;
+  lookup_issue<RO>(slots, ovf, d, key, L);
+  return lookup_finish<RO>(slots, ovf, d, key, L);
 }
 
 // Global slot index of key in an instance's main table, or ~0 if absent (L2-coherent reads; used
@@ -829,8 +857,8 @@ namespace pskl {
 // receives T_pf of every pair's hit; stats (nullable) accumulates the six launch counters of
 // ps_last_probe_stats; ev_mid (nullable) is recorded between the two probe kernels.
 cudaError_t launch_probe(const uint64_t* slots, const uint64_t* ovf, const psk::TableDesc* tdesc, uint32_t I,
-                         const psk::WindowDev& w, const psk::RowPre* rows, uint32_t* hits, float* tpf,
-                         const psk::DevModel& m, int grid, int search, unsigned long long* stats,
+                         const psk::WindowDev& w, const psk::RowPre* rows, psk::RowList list, uint32_t* hits,
+                         float* tpf, const psk::DevModel& m, int grid, int search, unsigned long long* stats,
                          cudaEvent_t ev_mid, cudaStream_t s);
 int probe_max_grid(uint32_t I, int num_sms);
 cudaError_t launch_score(const uint32_t* hits, psk::StateSoA st, uint32_t I, const psk::WindowDev& w,
@@ -843,7 +871,7 @@ cudaError_t launch_greedy(const uint64_t* slots, const uint64_t* ovf, const psk:
                           uint32_t* err, int search, cudaStream_t s);
 cudaError_t launch_delta_clear(psk::DeltaSlot* delta, uint64_t nslots, cudaStream_t s);
 cudaError_t launch_relations(const psk::WindowDev& w, const psk::DevModel& m, psk::LastSlot* tab, uint32_t tab_n,
-                             psk::RowPre* rows, int num_sms, cudaStream_t s);
+                             psk::RowPre* rows, psk::RowList list, int num_sms, cudaStream_t s);
 cudaError_t launch_greedy_search(const psk::RowPre* rows, const psk::WindowDev& w, uint32_t I, const uint32_t* hit0,
                                  const float* tpf0, psk::StateSoA committed, psk::StateSoA pending, const psk::DevModel& m,
                                  psk::DeltaSlot* delta, uint64_t delta_nslots, int32_t* assign, uint8_t* path,

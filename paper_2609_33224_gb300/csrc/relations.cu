@@ -128,10 +128,12 @@ __global__ void relations_kernel(psk::WindowDev w, psk::DevModel m, const psk::L
 }
 
 // base and the two next ancestors of each request: follow the parent links (parents come
-// earlier, so the walk ends).
-__global__ void base_kernel(uint32_t R, psk::RowPre* rows) {
+// earlier, so the walk ends).  Requests without a parent go to the list of rows the probe
+// searches from scratch.
+__global__ void base_kernel(uint32_t R, psk::RowPre* rows, psk::RowList list) {
   for (uint32_t r = blockIdx.x * blockDim.x + threadIdx.x; r < R; r += gridDim.x * blockDim.x) {
     int32_t a = rows[r].par;
+    if (a < 0) list.rows[atomicAdd(list.count, 1u)] = r;  // searched from scratch
     int32_t anc[2] = {-1, -1};
     uint32_t anc_nb[2] = {0u, 0u};
     if (a >= 0) {
@@ -156,9 +158,10 @@ __global__ void base_kernel(uint32_t R, psk::RowPre* rows) {
 namespace pskl {
 
 cudaError_t launch_relations(const psk::WindowDev& w, const psk::DevModel& m, psk::LastSlot* tab, uint32_t tab_n,
-                             psk::RowPre* rows, int num_sms, cudaStream_t s) {
-  if (w.R == 0) return cudaSuccess;
-  cudaError_t e = cudaMemsetAsync(tab, 0, (size_t)tab_n * sizeof(psk::LastSlot), s);
+                             psk::RowPre* rows, psk::RowList list, int num_sms, cudaStream_t s) {
+  cudaError_t e = cudaMemsetAsync(list.count, 0, sizeof(uint32_t), s);
+  if (e != cudaSuccess || w.R == 0) return e;
+  e = cudaMemsetAsync(tab, 0, (size_t)tab_n * sizeof(psk::LastSlot), s);
   if (e != cudaSuccess) return e;
   const int g1 = (int)std::min<uint64_t>((w.R + 255) / 256, (uint64_t)num_sms * 8);
   lastblock_build_kernel<<<g1, 256, 0, s>>>(w, tab, tab_n);
@@ -168,7 +171,7 @@ cudaError_t launch_relations(const psk::WindowDev& w, const psk::DevModel& m, ps
   relations_kernel<<<g2, 256, 0, s>>>(w, m, tab, tab_n, rows);
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  base_kernel<<<g1, 256, 0, s>>>(w.R, rows);
+  base_kernel<<<g1, 256, 0, s>>>(w.R, rows, list);
   return cudaGetLastError();
 }
 
