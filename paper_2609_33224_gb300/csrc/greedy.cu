@@ -384,7 +384,11 @@ __device__ void insert_blocks(const psk::RowPre* __restrict__ rows, const uint64
 }
 
 // Probe blocks: block p probes rows p, p + kProbeBlocks, ... in order (see the section comment).
-// Shared memory: touched flags and last chain end per instance, the walk list.
+// Per row, everything that does not need the window's inserts comes first: replaying the published
+// jobs <= s - kLag (which instances have window inserts, their last chain end, the picks of the
+// row's ancestors), the hit0 row, the probe positions and the chain blocks there.  Only then does the
+// block wait until those jobs' inserts are done, so after the wait one delta lookup per instance
+// (and, rarely, a warp search) is left before the row is released.
 template <int IPT>
 __device__ void probe_rows(const psk::RowPre* __restrict__ rows, const uint64_t* __restrict__ hash, uint32_t R,
                            uint32_t I, const uint32_t* __restrict__ hit0, const float* __restrict__ tpf0,
@@ -396,14 +400,16 @@ __device__ void probe_rows(const psk::RowPre* __restrict__ rows, const uint64_t*
   __shared__ uint32_t s_nwalk;
   __shared__ int32_t s_ja[3];       // picks of the row's ancestors old enough to count (-1: none)
   __shared__ uint32_t s_jnb[3];     // their chain lengths
-  __shared__ uint32_t s_frontier;   // jobs [0, frontier) are done and replayed
+  __shared__ uint32_t s_replayed;   // jobs [0, s_replayed) are published and replayed
+  __shared__ uint32_t s_done;       // jobs [0, s_done) have their inserts in the delta table
   __shared__ int s_abort;
   const uint32_t t = threadIdx.x;
   const uint32_t NT = blockDim.x;
   const int lane = t & 31, warp = t >> 5, NW = NT >> 5;
   for (uint32_t i = t; i < I; i += NT) s_end[i] = 0u;
   if (t == 0) {
-    s_frontier = 0;
+    s_replayed = 0;
+    s_done = 0;
     s_nwalk = 0;
     s_abort = 0;
   }
@@ -411,39 +417,28 @@ __device__ void probe_rows(const psk::RowPre* __restrict__ rows, const uint64_t*
   for (uint32_t s = blockIdx.x - 1 - kInsertBlocks; s < R; s += kProbeBlocks) {
     const uint64_t off = __ldg(&rows[s].off);
     const uint32_t nb = __ldg(&rows[s].nb);
+    const int64_t need = (int64_t)s - psk::kLag + 1;  // jobs [0, need) count for this row
     if (warp == 0) {
-      // Jobs <= s - kLag must be in the delta table.  Replay them in order, 32 at a time: the
-      // leading run of done flags among the next 32 jobs is taken, and for each instance the latest
-      // of those jobs sets its chain end.
-      const int64_t need = (int64_t)s - psk::kLag + 1;
-      uint32_t f = s_frontier;
+      // Replay the published jobs [replayed, need), 32 at a time; for each instance the latest of
+      // them sets its chain end.
+      uint32_t f = s_replayed;
       bool abort = false;
       while ((int64_t)f < need && !abort) {
         const uint32_t x = f + (uint32_t)lane;
-        const bool in = (int64_t)x < need;
-        const bool ok = in && psk::ld_acquire_u32(sync.done + x) != 0u;
-        const unsigned okm = __ballot_sync(0xffffffffu, ok);
-        const uint32_t nok = (okm == 0xffffffffu) ? 32u : (uint32_t)(__ffs(~okm) - 1);
-        if (nok == 0u) {  // the next job is not done yet: wait for it
-          bool got = true;
-          if (lane == 0) got = wait_flag(sync.done + f, err);
-          abort = !__shfl_sync(0xffffffffu, got, 0);
-          continue;
-        }
-        const bool mine = (uint32_t)lane < nok;
+        const bool mine = (int64_t)x < need;
         unsigned long long jb = 0ull;
         if (mine) jb = wait_job(sync.jobs + x, err);
         abort = __any_sync(0xffffffffu, mine && jb == 0ull);
         if (abort) break;
         const uint32_t j = mine ? job_pick(jb) : 0xFFFFFFFFu;
         const uint32_t nbx = mine ? __ldg(&rows[x].nb) : 0u;
-        // the highest lane of each group of equal picks holds the latest job on that instance
         const unsigned same = __match_any_sync(0xffffffffu, j);
         if (mine && j < I && (31 - __clz(same)) == lane) s_end[j] = nbx;
-        f += nok;
+        const uint32_t n = (int64_t)f + 32 <= need ? 32u : (uint32_t)(need - (int64_t)f);
+        f += n;
       }
       if (lane == 0) {
-        s_frontier = f;
+        s_replayed = f;
         s_abort = abort ? 1 : 0;
         const int32_t a[3] = {__ldg(&rows[s].par), __ldg(&rows[s].anc[0]), __ldg(&rows[s].anc[1])};
         const uint32_t anb[3] = {__ldg(&rows[s].par_nb), __ldg(&rows[s].anc_nb[0]), __ldg(&rows[s].anc_nb[1])};
@@ -464,10 +459,12 @@ __device__ void probe_rows(const psk::RowPre* __restrict__ rows, const uint64_t*
     const uint32_t jn0 = s_jnb[0], jn1 = s_jnb[1], jn2 = s_jnb[2];
     uint32_t h0[IPT], pos[IPT];
     float tp0[IPT];
-    bool walk[IPT];
+    uint64_t key[IPT];
+    bool probe[IPT], walk[IPT];
 #pragma unroll
     for (int k = 0; k < IPT; ++k) {
       const uint32_t i = t + k * NT;
+      probe[k] = false;
       walk[k] = false;
       if (i < I) {
         h0[k] = __ldg(hit0 + (uint64_t)s * I + i);
@@ -478,11 +475,42 @@ __device__ void probe_rows(const psk::RowPre* __restrict__ rows, const uint64_t*
         if ((int32_t)i == ja2 && jn2 > p) p = jn2;
         pos[k] = p;
         // s_end[i] != 0: the instance has window inserts visible to this row
-        if (s_end[i] != 0u && p < nb && psk::delta_contains(delta, nslots, i, __ldg(hash + off + p))) {
-          walk[k] = true;
-          s_res[i] = p;
-          s_walk[atomicAdd(&s_nwalk, 1u)] = i;
+        probe[k] = s_end[i] != 0u && p < nb;
+        key[k] = probe[k] ? __ldg(hash + off + p) : 0ull;
+      }
+    }
+    if (warp == 0) {
+      // Wait until the inserts of jobs [done, need) are in: the leading run of done flags among the
+      // next 32 is taken, and the first one not yet done is waited for.
+      uint32_t f = s_done;
+      bool abort = false;
+      while ((int64_t)f < need && !abort) {
+        const uint32_t x = f + (uint32_t)lane;
+        const bool ok = (int64_t)x < need && psk::ld_acquire_u32(sync.done + x) != 0u;
+        const unsigned okm = __ballot_sync(0xffffffffu, ok);
+        const uint32_t nok = (okm == 0xffffffffu) ? 32u : (uint32_t)(__ffs(~okm) - 1);
+        if (nok == 0u) {
+          bool got = true;
+          if (lane == 0) got = wait_flag(sync.done + f, err);
+          abort = !__shfl_sync(0xffffffffu, got, 0);
+          continue;
         }
+        f += nok;
+      }
+      if (lane == 0) {
+        s_done = f;
+        s_abort = abort ? 1 : 0;
+      }
+    }
+    __syncthreads();
+    if (s_abort) return;  // block-uniform
+#pragma unroll
+    for (int k = 0; k < IPT; ++k) {
+      const uint32_t i = t + k * NT;
+      if (probe[k] && psk::delta_contains(delta, nslots, i, key[k])) {
+        walk[k] = true;
+        s_res[i] = pos[k];
+        s_walk[atomicAdd(&s_nwalk, 1u)] = i;
       }
     }
     __syncthreads();
@@ -516,10 +544,11 @@ __device__ void probe_rows(const psk::RowPre* __restrict__ rows, const uint64_t*
   }
 }
 
-// Deciding block.  Thread t < NTI owns instances t * IPT .. t * IPT + IPT - 1; thread NTI (first
-// lane of the last warp) signals.  Block reductions: each warp reduces its lanes with
-// single-instruction warp reductions, writes one partial, and after the barrier every warp reduces
-// the partials itself (no second barrier).
+// Deciding block.  Thread t < NTI owns instances t * IPT .. t * IPT + IPT - 1; thread 0 publishes
+// the decisions.  The last warp only waits for the probe blocks' ready flags (thread NTI): an
+// acquire load holds up its thread's later memory accesses, so that warp does nothing else.  Block
+// reductions: each instance warp reduces its lanes with single-instruction warp reductions, writes
+// one partial, and after the barrier every instance warp reduces the partials itself.
 template <int IPT>
 __device__ void decide_rows(const psk::RowPre* __restrict__ rows, uint32_t R, uint32_t I, psk::StateSoA committed,
                             psk::StateSoA pending, const psk::DevModel& m, int32_t* assign, uint8_t* __restrict__ path,
@@ -540,7 +569,7 @@ __device__ void decide_rows(const psk::RowPre* __restrict__ rows, uint32_t R, ui
   int32_t* s_Bmax = s_qr + I;
   int32_t* s_room = s_Bmax + I;                                    // kv_room(S, M_KV)
   __shared__ psk::RowPre s_row[8];  // rows r .. r + kRingAhead (a ring of 8 so no reader is overtaken)
-  __shared__ int32_t s_jm[8];       // pick of request x in s_jm[x & 7] (-1: rejected)
+  __shared__ int32_t s_jm[16];      // pick of request x in s_jm[x & 15] (-1: rejected)
   __shared__ uint32_t s_red_w[32];  // per-warp W_min (order-preserving bits), 0 = no pair in A
   __shared__ uint64_t s_red_key[32];
   __shared__ uint32_t s_red_i[32];
@@ -552,9 +581,9 @@ __device__ void decide_rows(const psk::RowPre* __restrict__ rows, uint32_t R, ui
   const bool sig = t == NTI;
   const int lane = t & 31;
   const int warp = t >> 5;
-  const int NW = NT >> 5;
+  const int NWI = NTI >> 5;               // instance warps
   const uint32_t i0 = (uint32_t)t * IPT;  // first owned instance (>= I for the signalling warp)
-  const bool owner = t < NTI;
+  const bool owner = t < NTI;             // false for the whole signalling warp
   auto key0_bits = [](int32_t b, int32_t qr) -> uint64_t {
     return ((uint64_t)((1u << 18) - 1u - (uint32_t)b) << 44) | (uint64_t)(uint32_t)qr;
   };
@@ -571,7 +600,7 @@ __device__ void decide_rows(const psk::RowPre* __restrict__ rows, uint32_t R, ui
     s_key0[i] = key0_bits(s_b[i], s_qr[i]);
   }
   for (uint32_t i = t; i < 2 * Ip; i += NT) s_ovr[i] = 0u;
-  if (t < 8) s_jm[t] = -1;
+  if (t < 16) s_jm[t] = -1;
   if (t < kRingAhead * psk::kRowWords) {  // rows 0 .. kRingAhead - 1
     const uint32_t rr = (uint32_t)(t / psk::kRowWords);
     if (rr < R)
@@ -602,13 +631,19 @@ __device__ void decide_rows(const psk::RowPre* __restrict__ rows, uint32_t R, ui
   uint32_t hr[IPT];
 
   for (uint32_t r = 0; r < R; ++r) {
+    if (!owner) {  // the signalling warp: row r + 2's ready flag, then the step's two barriers
+      uint32_t ready_seen = 1u;
+      if (sig && r + 2 < R && !timed_out) ready_seen = psk::ld_acquire_u32(sync.ready + r + 2);
+      __syncthreads();  // (C)
+      if (sig && ready_seen == 0u) timed_out = !wait_flag(sync.ready + r + 2, err);
+      __syncthreads();  // (D)
+      continue;
+    }
     const psk::RowPre& cur = s_row[r & 7];
     // ---- P0: row-constant refill, row r's hits, pass 1 ------------------------------------------
     if (t < psk::kRowWords && r + kRingAhead < R)
       psk::cp_async16(reinterpret_cast<uint4*>(&s_row[(r + kRingAhead) & 7]) + t,
                       reinterpret_cast<const uint4*>(rows + r + kRingAhead) + t);
-    uint32_t ready_seen = 1u;
-    if (sig && r + 2 < R && !timed_out) ready_seen = psk::ld_acquire_u32(sync.ready + r + 2);
     psk::cp_async_wait_group<1>();  // this thread's copies of row r (and row constants <= r + 4)
     const psk::RowConst rc = row_of(cur);
     const uint32_t lcp0 = cur.lcp[0];
@@ -622,7 +657,7 @@ __device__ void decide_rows(const psk::RowPre* __restrict__ rows, uint32_t R, ui
     for (int k = 0; k < IPT; ++k) {
       const uint32_t i = i0 + k;
       inA[k] = false;
-      if (owner && i < I) {
+      if (i < I) {
         const uint32_t hb = hrow[i];
         uint32_t h = hb;
         const uint32_t ov = orow[i];
@@ -637,8 +672,7 @@ __device__ void decide_rows(const psk::RowPre* __restrict__ rows, uint32_t R, ui
         const float tb = trow[i];
         tpk[k] = (h == hb && __float_as_uint(tb) != psk::kNoTpfBits) ? tb : psk::t_pf_of_hit(m, rc.L, h);
         Wk[k] = __fsub_rn(tpk[k], rc.t_cached);
-        const psk::InstTerms& it = s_it[i];
-        inA[k] = it.okB && (int32_t)rc.L <= s_room[i];
+        inA[k] = s_it[i].okB && (int32_t)rc.L <= s_room[i];
         if (inA[k]) wbest = min(wbest, psk::f2ord(Wk[k]));
       }
     }
@@ -646,8 +680,8 @@ __device__ void decide_rows(const psk::RowPre* __restrict__ rows, uint32_t R, ui
     if (lane == 0) s_red_w[warp] = wbest;
     __syncthreads();  // (C)
 
-    // ---- P1: W_min, pass 2, the row's argmin; lcp raises for row r + 1; row r + 2 ready ----------
-    const uint32_t wmin_o = __reduce_min_sync(0xffffffffu, lane < NW ? s_red_w[lane] : 0xFFFFFFFFu);
+    // ---- P1: W_min, pass 2, the row's argmin; lcp raises for row r + 1 --------------------------
+    const uint32_t wmin_o = __reduce_min_sync(0xffffffffu, lane < NWI ? s_red_w[lane] : 0xFFFFFFFFu);
     const bool anyA = wmin_o != 0xFFFFFFFFu;  // a W of a pair in A never maps to all ones (not NaN)
     const float wmin = psk::ord2f(wmin_o);
     uint64_t bkey = psk::kNoKey;
@@ -655,7 +689,7 @@ __device__ void decide_rows(const psk::RowPre* __restrict__ rows, uint32_t R, ui
 #pragma unroll
     for (int k = 0; k < IPT; ++k) {
       const uint32_t i = i0 + k;
-      if (owner && i < I && inA[k] && psk::pair_in_c(rc, Wk[k], wmin)) {
+      if (i < I && inA[k] && psk::pair_in_c(rc, Wk[k], wmin)) {
         const psk::InstTerms it = s_it[i];
         const int64_t q = s_q[i];
         const int64_t S = s_S[i];
@@ -690,28 +724,27 @@ __device__ void decide_rows(const psk::RowPre* __restrict__ rows, uint32_t R, ui
     // raise from request r itself is applied in registers next step.
     if (t < psk::kLcpBack - 1 && r + 1 < R) {
       const uint32_t d = (uint32_t)t + 1u;
-      const int32_t jd = r >= d ? s_jm[(r - d) & 7u] : -1;
+      const int32_t jd = r >= d ? s_jm[(r - d) & 15u] : -1;
       const uint32_t v = s_row[(r + 1) & 7].lcp[d];
       if (jd >= 0 && v > 0u) atomicMax(s_ovr + ((r + 1) & 1u) * Ip + (uint32_t)jd, v);
     }
-    if (sig && ready_seen == 0u) timed_out = !wait_flag(sync.ready + r + 2, err);
     __syncthreads();  // (D)
 
     // ---- P2: the pick, its state, its insert job; copies of row r + 2 ----------------------------
     uint64_t key;
     uint32_t j, hj;
-    psk::warp_pick_min(lane < NW ? s_red_key[lane] : psk::kNoKey, lane < NW ? s_red_i[lane] : 0xFFFFFFFFu,
-                       lane < NW ? s_red_h[lane] : 0u, &key, &j, &hj);
+    psk::warp_pick_min(lane < NWI ? s_red_key[lane] : psk::kNoKey, lane < NWI ? s_red_i[lane] : 0xFFFFFFFFu,
+                       lane < NWI ? s_red_h[lane] : 0u, &key, &j, &hj);
     const bool pick = anyA && key != psk::kNoKey;
     if (!pick) hj = 0u;
-    if (sig) {
+    if (t == 0) {
       assign[r] = pick ? (int32_t)j : -1;
       path[r] = pick ? (uint8_t)(key >> 62) : (uint8_t)2;
       hit_chosen[r] = hj;
-      s_jm[r & 7u] = pick ? (int32_t)j : -1;
+      s_jm[r & 15u] = pick ? (int32_t)j : -1;
       psk::st_relaxed_u64(sync.jobs + r, kJobValid | ((unsigned long long)hj << 32) | (pick ? j : 0xFFFFFFFFu));
     }
-    if (pick && owner && j >= i0 && j < i0 + IPT) {
+    if (pick && j >= i0 && j < i0 + IPT) {
       s_qr[j] += 1;
       s_q[j] += (int64_t)rc.L - 16 * (int64_t)hj;
       s_S[j] += (int64_t)rc.L;
@@ -719,7 +752,7 @@ __device__ void decide_rows(const psk::RowPre* __restrict__ rows, uint32_t R, ui
       s_room[j] = psk::kv_room(s_S[j], s_M[j]);
       s_key0[j] = key0_bits(s_b[j], s_qr[j]);
     }
-    if (r + 2 < R && !timed_out) copy_row(r + 2);
+    if (r + 2 < R) copy_row(r + 2);
     psk::cp_async_commit();
     jprev = pick ? (int32_t)j : -1;
   }

@@ -62,7 +62,7 @@ struct DeltaSlot {
 
 // Greedy pipeline depth: a probe for request s sees every delta insert of requests <= s - kLag, and
 // the requests s - 1 .. s - (kLag - 1) are covered by their common chain prefix with s (RowPre::lcp).
-constexpr int kLag = 9;
+constexpr int kLag = 13;
 constexpr int kLcpBack = kLag - 1;
 
 // Per-request constants of one window, computed in parallel before the greedy pass: the request's
@@ -86,7 +86,7 @@ struct __align__(16) RowPre {
   uint32_t lcp[kLcpBack];  // common chain prefix with requests r - 1 .. r - kLcpBack (blocks)
 };
 constexpr int kRowWords = (int)(sizeof(RowPre) / 16);
-static_assert(sizeof(RowPre) % 16 == 0 && kRowWords == 6, "RowPre is six 16-byte words");
+static_assert(sizeof(RowPre) % 16 == 0 && kRowWords == 7, "RowPre is seven 16-byte words");
 
 // Hand-offs between the blocks of the pipelined greedy (one cooperative launch): the deciding
 // block publishes each decision as a job, insert blocks put the job's chain blocks into the delta
