@@ -125,6 +125,18 @@ def probe_algorithmic_bytes(st: dict, I: int, with_tpf: bool) -> tuple[int, int]
     return int(nbytes), int(lookups)
 
 
+def profile_figure(name: str, label: str):
+    """A per-unit DRAM figure ("<label>: <number>") from a committed ncu summary under profiles/, or
+    None when the summary is absent."""
+    path = os.path.join(ROOT, "profiles", name)
+    if not os.path.exists(path):
+        return None
+    for line in open(path):
+        if line.startswith(label + ":"):
+            return float(line.split(":", 1)[1])
+    return None
+
+
 def oracle_sample(wl, seconds: float, max_rows: int | None = None):
     """Oracle greedy over successive prefixes of the window until ~`seconds` of CPU time."""
     import workload as W
@@ -304,18 +316,25 @@ def main():
     dominant = max(phases, key=phases.get)
     peak, peak_src = _peaks()
     probe_ms = km["probe_scratch"] + max(0.0, km["probe_derived"])
+    greedy_traffic = profile_figure("greedy_pipe_production_window_1024x2048.md", "DRAM bytes per request")
+    probe_traffic = profile_figure("probe_search_production_window_1024x2048.md", "DRAM bytes per lookup")
     if dominant == "probe":
         achieved = probe_bytes / (probe_ms / 1000) / 1e9
-        roof = {"bound": "hbm", "kernel": "probe_hits_kernel + probe_derived_kernel", "achieved": achieved,
-                "peak": peak, "unit": "GB/s", "frac": achieved / peak, "traffic": None, "peak_source": peak_src,
-                "algorithmic_bytes_per_launch": probe_bytes}
+        roof = {"bound": "hbm", "kernel": "probe_search_kernel + probe_derived_kernel", "achieved": achieved,
+                "peak": peak, "unit": "GB/s", "frac": achieved / peak,
+                "traffic": None if probe_traffic is None else probe_traffic * n_probes,
+                "peak_source": peak_src, "algorithmic_bytes_per_launch": probe_bytes}
     else:
-        greedy_bytes = int(4 * R * I + 24 * R + 16 * I * 6)
+        # per decision: the request's hit and T_pf rows (8 B per instance) and its decision outputs
+        greedy_bytes = int(R * (8 * I + 16))
         achieved = greedy_bytes / (km[dominant] / 1000) / 1e9
-        roof = {"bound": "hbm", "kernel": f"{dominant}_kernel", "achieved": achieved, "peak": peak,
-                "unit": "GB/s", "frac": achieved / peak, "traffic": None, "peak_source": peak_src,
-                "algorithmic_bytes_per_launch": greedy_bytes,
-                "note": "serial per-request dependency chain: latency-bound, not bandwidth-bound"}
+        roof = {"bound": "hbm", "kernel": "greedy_pipe_kernel" if args.probe_mode == 1 else "greedy_kernel",
+                "achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak,
+                "traffic": (None if greedy_traffic is None or args.probe_mode != 1 else greedy_traffic * R),
+                "peak_source": peak_src, "algorithmic_bytes_per_launch": greedy_bytes,
+                "ns_per_decision": 1e6 * km[dominant] / R,
+                "note": "serial per-request dependency chain decided on one SM: latency-bound, not "
+                        "bandwidth-bound; traffic scaled by request count from the 2048-request ncu capture"}
     probe_achieved = probe_bytes / (probe_ms / 1000) / 1e9
     line = {"metric": METRIC, "value": world * R * I / (ms / 1000), "unit": "scorings/s", "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
@@ -323,19 +342,21 @@ def main():
             "decisions_per_s": world * R / (ms / 1000),
             "config": {"workload": WORKLOADS.get(args.config, str(args.config)), "instances": I,
                        "window_requests": R, "window_chain_blocks": int(nb.sum()),
-                       "tpot_target_ms": float(win.tpot_target[0]), "probe": ("per-lane binary first-miss search (prefix-closed caches)" if args.probe_mode == 1
-                                 else "linear 32-wide warp walk"), "probes_per_window": n_probes,
+                       "tpot_target_ms": float(win.tpot_target[0]), "probe": ("hinted per-lane search of rows without an earlier prefix in the window, the rest derived"
+                                 if args.probe_mode == 1 else "linear 32-wide warp walk"), "probes_per_window": n_probes,
                        "l2": "inputs larger than L2 (no flush)", "path_counts": path_counts},
             "kernel_ms": km,
-            "probe_roofline": {"kernels": "probe_hits_kernel + probe_derived_kernel", "achieved": probe_achieved,
+            "probe_roofline": {"kernels": "probe_search_kernel + probe_derived_kernel", "achieved": probe_achieved,
                                "unit": "GB/s", "peak": peak, "frac": probe_achieved / peak,
                                "frac_vs_8tbs": probe_achieved / 8000.0, "ms": probe_ms,
-                               "algorithmic_bytes_per_launch": probe_bytes, "stats": pstats},
+                               "algorithmic_bytes_per_launch": probe_bytes, "stats": pstats,
+                               "traffic": None if probe_traffic is None else probe_traffic * n_probes},
             "roofline": roof,
             "e2e": {"value": world * R * I / (e2e_ms / 1000), "unit": "scorings/s", "ms_per_step": e2e_ms,
                     "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
-            # per step: window validation, probe, score, last-block table, relations, greedy
-            "gpu_launches": (6 if args.probe_mode == 1 else 4) * args.steps,
+            # per step: window validation, last-block table, relations, base, probe (scratch rows),
+            # probe (derived rows), score, greedy
+            "gpu_launches": 8 * args.steps,
             "clocks": clk.summary()}
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         import oracle
