@@ -549,31 +549,74 @@ __device__ void probe_rows(const psk::RowPre* __restrict__ rows, const uint64_t*
 // acquire load holds up its thread's later memory accesses, so that warp does nothing else.  Block
 // reductions: each instance warp reduces its lanes with single-instruction warp reductions, writes
 // one partial, and after the barrier every instance warp reduces the partials itself.
+// Instance state is kept as padded structure-of-arrays in shared memory, so a thread reads its IPT
+// consecutive instances' values of one field with one vector load; the capacity guard is one
+// compare against the free KV room, stored as -1 where the decode-slot guard fails.
+template <int N>
+__device__ __forceinline__ void ld_u32v(const void* p, uint32_t (&v)[N]) {
+  static_assert(N == 1 || N == 2 || N == 4, "vector of 1, 2 or 4");
+  if (N == 1) {
+    v[0] = *reinterpret_cast<const uint32_t*>(p);
+  } else if (N == 2) {
+    const uint2 x = *reinterpret_cast<const uint2*>(p);
+    v[0] = x.x;
+    v[N > 1 ? 1 : 0] = x.y;
+  } else {
+    const uint4 x = *reinterpret_cast<const uint4*>(p);
+    v[0] = x.x;
+    v[N > 1 ? 1 : 0] = x.y;
+    v[N > 2 ? 2 : 0] = x.z;
+    v[N > 3 ? 3 : 0] = x.w;
+  }
+}
+
+template <int N>
+__device__ __forceinline__ void st_zero_u32v(void* p) {
+  if (N == 1) *reinterpret_cast<uint32_t*>(p) = 0u;
+  else if (N == 2) *reinterpret_cast<uint2*>(p) = make_uint2(0u, 0u);
+  else *reinterpret_cast<uint4*>(p) = make_uint4(0u, 0u, 0u, 0u);
+}
+
+template <int N>
+__device__ __forceinline__ void ld_u64v(const void* p, uint64_t (&v)[N]) {
+  if (N == 1) {
+    v[0] = *reinterpret_cast<const unsigned long long*>(p);
+  } else {
+#pragma unroll
+    for (int k = 0; k < N; k += 2) {
+      const ulonglong2 x = reinterpret_cast<const ulonglong2*>(p)[k / 2];
+      v[k] = x.x;
+      v[k + 1 < N ? k + 1 : k] = x.y;
+    }
+  }
+}
+
 template <int IPT>
 __device__ void decide_rows(const psk::RowPre* __restrict__ rows, uint32_t R, uint32_t I, psk::StateSoA committed,
                             psk::StateSoA pending, const psk::DevModel& m, int32_t* assign, uint8_t* __restrict__ path,
                             uint32_t* __restrict__ hit_chosen, uint32_t* err, const psk::GreedySync& sync,
                             unsigned long long* smem_raw) {
   const uint32_t Ip = sync.ring_stride;  // I rounded up to a multiple of 4
-  // Ip is a multiple of 4, so every array below starts 16-byte aligned or at its own alignment.
-  uint32_t* s_hit = reinterpret_cast<uint32_t*>(smem_raw);        // [4][Ip] probed hits of rows r .. r + 3
-  float* s_tpf = reinterpret_cast<float*>(s_hit + 4 * Ip);        // [4][Ip] T_pf at those hits
-  uint32_t* s_ovr = reinterpret_cast<uint32_t*>(s_tpf + 4 * Ip);  // [2][Ip] lcp raises for the next row
-  int64_t* s_q = reinterpret_cast<int64_t*>(s_ovr + 2 * Ip);
-  int64_t* s_S = s_q + I;
-  int64_t* s_M = s_S + I;
-  uint64_t* s_key0 = reinterpret_cast<uint64_t*>(s_M + I);        // class-0 key bits of (b, qr)
-  psk::InstTerms* s_it = reinterpret_cast<psk::InstTerms*>(s_key0 + I);
-  int32_t* s_b = reinterpret_cast<int32_t*>(s_it + I);
-  int32_t* s_qr = s_b + I;
-  int32_t* s_Bmax = s_qr + I;
-  int32_t* s_room = s_Bmax + I;                                    // kv_room(S, M_KV)
+  // Every [Ip] array starts 16-byte aligned (Ip is a multiple of 4); the 8-byte arrays come first.
+  int64_t* s_q = reinterpret_cast<int64_t*>(smem_raw);    // [Ip] queued prefill tokens
+  int64_t* s_S = s_q + Ip;                                // [Ip] KV tokens held
+  uint64_t* s_key0 = reinterpret_cast<uint64_t*>(s_S + Ip);  // [Ip] class-0 key bits of (b, qr)
+  int64_t* s_M = reinterpret_cast<int64_t*>(s_key0 + Ip);    // [Ip] KV capacity
+  uint32_t* s_hit = reinterpret_cast<uint32_t*>(s_M + Ip);   // [4][Ip] probed hits of rows r .. r + 3
+  uint32_t* s_tpf = s_hit + 4 * Ip;                          // [4][Ip] T_pf at those hits (bits)
+  uint32_t* s_ovr = s_tpf + 4 * Ip;                          // [2][Ip] lcp raises for the next row
+  int32_t* s_room = reinterpret_cast<int32_t*>(s_ovr + 2 * Ip);  // [Ip] free KV room, -1 if no slot
+  float* s_dec0 = reinterpret_cast<float*>(s_room + Ip);     // [Ip] InstTerms, field by field
+  float* s_f = s_dec0 + Ip;
+  float* s_tq = s_f + Ip;
+  int32_t* s_Bp = reinterpret_cast<int32_t*>(s_tq + Ip);
+  int32_t* s_b = s_Bp + Ip;                                  // [Ip] decoding requests
+  int32_t* s_qr = s_b + Ip;                                  // [Ip] queued requests
+  int32_t* s_Bmax = s_qr + Ip;                               // [Ip] decode-slot limit
   __shared__ psk::RowPre s_row[8];  // rows r .. r + kRingAhead (a ring of 8 so no reader is overtaken)
   __shared__ int32_t s_jm[16];      // pick of request x in s_jm[x & 15] (-1: rejected)
-  __shared__ uint32_t s_red_w[32];  // per-warp W_min (order-preserving bits), 0 = no pair in A
-  __shared__ uint64_t s_red_key[32];
-  __shared__ uint32_t s_red_i[32];
-  __shared__ uint32_t s_red_h[32];
+  __shared__ uint32_t s_red_w[32];  // per-warp W_min (order-preserving bits)
+  __shared__ uint4 s_red_k[32];     // per-warp pick: key (x, y), instance (z), hit (w)
 
   const int t = threadIdx.x;
   const int NT = blockDim.x;
@@ -584,20 +627,33 @@ __device__ void decide_rows(const psk::RowPre* __restrict__ rows, uint32_t R, ui
   const int NWI = NTI >> 5;               // instance warps
   const uint32_t i0 = (uint32_t)t * IPT;  // first owned instance (>= I for the signalling warp)
   const bool owner = t < NTI;             // false for the whole signalling warp
+  const bool has = owner && i0 < I;       // the thread owns instances (then i0 + IPT <= Ip)
   auto key0_bits = [](int32_t b, int32_t qr) -> uint64_t {
     return ((uint64_t)((1u << 18) - 1u - (uint32_t)b) << 44) | (uint64_t)(uint32_t)qr;
   };
-
-  for (uint32_t i = t; i < I; i += NT) {
-    s_b[i] = committed.b[i];
-    s_qr[i] = committed.qr[i];
-    s_q[i] = committed.q[i];
-    s_S[i] = committed.S[i];
-    s_M[i] = committed.M[i];
-    s_Bmax[i] = committed.Bmax[i];
-    s_it[i] = psk::inst_terms(m, s_b[i], s_qr[i], s_q[i], s_Bmax[i]);
-    s_room[i] = psk::kv_room(s_S[i], s_M[i]);
+  // instance terms of i after a state change (decode-slot guard folded into the KV room)
+  auto set_terms = [&](uint32_t i) {
+    const psk::InstTerms it = psk::inst_terms(m, s_b[i], s_qr[i], s_q[i], s_Bmax[i]);
+    s_dec0[i] = it.dec0;
+    s_f[i] = it.f;
+    s_tq[i] = it.tq;
+    s_Bp[i] = it.Bp;
+    s_room[i] = it.okB ? psk::kv_room(s_S[i], s_M[i]) : -1;
     s_key0[i] = key0_bits(s_b[i], s_qr[i]);
+  };
+
+  for (uint32_t i = t; i < Ip; i += NT) {
+    if (i < I) {
+      s_b[i] = committed.b[i];
+      s_qr[i] = committed.qr[i];
+      s_q[i] = committed.q[i];
+      s_S[i] = committed.S[i];
+      s_M[i] = committed.M[i];
+      s_Bmax[i] = committed.Bmax[i];
+      set_terms(i);
+    } else {
+      s_room[i] = -1;  // padding: never capacity-eligible
+    }
   }
   for (uint32_t i = t; i < 2 * Ip; i += NT) s_ovr[i] = 0u;
   if (t < 16) s_jm[t] = -1;
@@ -615,7 +671,7 @@ __device__ void decide_rows(const psk::RowPre* __restrict__ rows, uint32_t R, ui
   // hits of rows 0 and 1, one copy group each (each thread copies and later reads only its own)
   static_assert(IPT == 1 || IPT == 2 || IPT == 4, "one 4-, 8- or 16-byte copy per array and row");
   auto copy_row = [&](uint32_t x) {
-    if (owner && i0 < I) {
+    if (has) {
       const uint64_t src = (uint64_t)(x % psk::kHitSlots) * Ip + i0;
       const uint32_t dst = (x & 3u) * Ip + i0;
       psk::cp_async_bytes<4 * IPT>(s_hit + dst, sync.hitring + src);
@@ -647,34 +703,35 @@ __device__ void decide_rows(const psk::RowPre* __restrict__ rows, uint32_t R, ui
     psk::cp_async_wait_group<1>();  // this thread's copies of row r (and row constants <= r + 4)
     const psk::RowConst rc = row_of(cur);
     const uint32_t lcp0 = cur.lcp[0];
-    const uint32_t* hrow = s_hit + (r & 3u) * Ip;
-    const float* trow = s_tpf + (r & 3u) * Ip;
-    uint32_t* orow = s_ovr + (r & 1u) * Ip;
     float Wk[IPT], tpk[IPT];
     bool inA[IPT];
     uint32_t wbest = 0xFFFFFFFFu;  // order-preserving bits of this thread's W_min over A
+    if (has) {
+      uint32_t hb[IPT], ov[IPT], tb[IPT], rm[IPT];
+      ld_u32v<IPT>(s_hit + (r & 3u) * Ip + i0, hb);
+      ld_u32v<IPT>(s_tpf + (r & 3u) * Ip + i0, tb);
+      uint32_t* op = s_ovr + (r & 1u) * Ip + i0;
+      ld_u32v<IPT>(op, ov);
+      ld_u32v<IPT>(s_room + i0, rm);
+      uint32_t anyov = 0u;
 #pragma unroll
-    for (int k = 0; k < IPT; ++k) {
-      const uint32_t i = i0 + k;
-      inA[k] = false;
-      if (i < I) {
-        const uint32_t hb = hrow[i];
-        uint32_t h = hb;
-        const uint32_t ov = orow[i];
-        if (ov) {
-          orow[i] = 0u;
-          if (ov > h) h = ov;
-        }
-        if ((int32_t)i == jprev && lcp0 > h) h = lcp0;
+      for (int k = 0; k < IPT; ++k) anyov |= ov[k];
+      if (anyov) st_zero_u32v<IPT>(op);
+#pragma unroll
+      for (int k = 0; k < IPT; ++k) {
+        uint32_t h = hb[k] > ov[k] ? hb[k] : ov[k];
+        if ((int32_t)(i0 + k) == jprev && lcp0 > h) h = lcp0;
         hr[k] = h;
         // T_pf at the hit: the ring's value unless it is marked unknown (the probe blocks raised the
         // hit) or the hit was raised here; W = T_pf(n, c) - T_pf(0, L)
-        const float tb = trow[i];
-        tpk[k] = (h == hb && __float_as_uint(tb) != psk::kNoTpfBits) ? tb : psk::t_pf_of_hit(m, rc.L, h);
+        tpk[k] = (h == hb[k] && tb[k] != psk::kNoTpfBits) ? __uint_as_float(tb[k]) : psk::t_pf_of_hit(m, rc.L, h);
         Wk[k] = __fsub_rn(tpk[k], rc.t_cached);
-        inA[k] = s_it[i].okB && (int32_t)rc.L <= s_room[i];
+        inA[k] = (int32_t)rc.L <= (int32_t)rm[k];
         if (inA[k]) wbest = min(wbest, psk::f2ord(Wk[k]));
       }
+    } else {
+#pragma unroll
+      for (int k = 0; k < IPT; ++k) inA[k] = false;
     }
     wbest = __reduce_min_sync(0xffffffffu, wbest);
     if (lane == 0) s_red_w[warp] = wbest;
@@ -686,26 +743,45 @@ __device__ void decide_rows(const psk::RowPre* __restrict__ rows, uint32_t R, ui
     const float wmin = psk::ord2f(wmin_o);
     uint64_t bkey = psk::kNoKey;
     uint32_t binst = 0xFFFFFFFFu, bh = 0u;
+    bool inC[IPT];
+    bool anyC = false;
 #pragma unroll
     for (int k = 0; k < IPT; ++k) {
-      const uint32_t i = i0 + k;
-      if (i < I && inA[k] && psk::pair_in_c(rc, Wk[k], wmin)) {
-        const psk::InstTerms it = s_it[i];
-        const int64_t q = s_q[i];
-        const int64_t S = s_S[i];
+      inC[k] = inA[k] && psk::pair_in_c(rc, Wk[k], wmin);
+      anyC |= inC[k];
+    }
+    if (anyC) {
+      uint32_t dec0[IPT], fe[IPT], tq[IPT], Bp[IPT];
+      uint64_t q[IPT], S[IPT], k0[IPT];
+      ld_u32v<IPT>(s_dec0 + i0, dec0);
+      ld_u32v<IPT>(s_f + i0, fe);
+      ld_u32v<IPT>(s_tq + i0, tq);
+      ld_u32v<IPT>(s_Bp + i0, Bp);
+      ld_u64v<IPT>(s_q + i0, q);
+      ld_u64v<IPT>(s_S + i0, S);
+      ld_u64v<IPT>(s_key0 + i0, k0);
+#pragma unroll
+      for (int k = 0; k < IPT; ++k) {
+        if (!inC[k]) continue;
+        psk::InstTerms it;
+        it.dec0 = __uint_as_float(dec0[k]);
+        it.f = __uint_as_float(fe[k]);
+        it.tq = __uint_as_float(tq[k]);
+        it.Bp = (int32_t)Bp[k];
+        it.okB = 1;
         psk::PairW x;
         x.W = Wk[k];
         x.tpf = tpk[k];
         x.n = (int64_t)rc.L - 16 * (int64_t)hr[k];
         x.inA = true;
         float tpot, ttft;
-        psk::pair_lat(m, rc, x, it, q, S, &tpot, &ttft);
+        psk::pair_lat(m, rc, x, it, (int64_t)q[k], (int64_t)S[k], &tpot, &ttft);
         const uint64_t key = psk::pair_admitted(m, rc, tpot, ttft)
-                                 ? psk::packed_key(0u, s_key0[i] | ((uint64_t)((1u << 26) - 1u - hr[k]) << 18))
-                                 : psk::packed_key(1u, (uint64_t)(q + x.n) * (uint64_t)(uint32_t)it.Bp);
+                                 ? psk::packed_key(0u, k0[k] | ((uint64_t)((1u << 26) - 1u - hr[k]) << 18))
+                                 : psk::packed_key(1u, ((uint64_t)q[k] + (uint64_t)x.n) * (uint64_t)Bp[k]);
         if (key < bkey) {  // instances ascend within a thread, so ties keep the lowest
           bkey = key;
-          binst = i;
+          binst = i0 + k;
           bh = hr[k];
         }
       }
@@ -714,11 +790,7 @@ __device__ void decide_rows(const psk::RowPre* __restrict__ rows, uint32_t R, ui
       uint64_t wk;
       uint32_t wi, wh;
       psk::warp_pick_min(bkey, binst, bh, &wk, &wi, &wh);
-      if (lane == 0) {
-        s_red_key[warp] = wk;
-        s_red_i[warp] = wi;
-        s_red_h[warp] = wh;
-      }
+      if (lane == 0) s_red_k[warp] = make_uint4((uint32_t)wk, (uint32_t)(wk >> 32), wi, wh);
     }
     // Row r + 1's raises from requests r - 1 .. r - kLag + 1 (thread d - 1 takes request r - d); the
     // raise from request r itself is applied in registers next step.
@@ -733,8 +805,10 @@ __device__ void decide_rows(const psk::RowPre* __restrict__ rows, uint32_t R, ui
     // ---- P2: the pick, its state, its insert job; copies of row r + 2 ----------------------------
     uint64_t key;
     uint32_t j, hj;
-    psk::warp_pick_min(lane < NWI ? s_red_key[lane] : psk::kNoKey, lane < NWI ? s_red_i[lane] : 0xFFFFFFFFu,
-                       lane < NWI ? s_red_h[lane] : 0u, &key, &j, &hj);
+    {
+      const uint4 pk = lane < NWI ? s_red_k[lane] : make_uint4(0xFFFFFFFFu, 0xFFFFFFFFu, 0xFFFFFFFFu, 0u);
+      psk::warp_pick_min(((uint64_t)pk.y << 32) | pk.x, pk.z, pk.w, &key, &j, &hj);
+    }
     const bool pick = anyA && key != psk::kNoKey;
     if (!pick) hj = 0u;
     if (t == 0) {
@@ -748,9 +822,7 @@ __device__ void decide_rows(const psk::RowPre* __restrict__ rows, uint32_t R, ui
       s_qr[j] += 1;
       s_q[j] += (int64_t)rc.L - 16 * (int64_t)hj;
       s_S[j] += (int64_t)rc.L;
-      s_it[j] = psk::inst_terms(m, s_b[j], s_qr[j], s_q[j], s_Bmax[j]);
-      s_room[j] = psk::kv_room(s_S[j], s_M[j]);
-      s_key0[j] = key0_bits(s_b[j], s_qr[j]);
+      set_terms(j);
     }
     if (r + 2 < R) copy_row(r + 2);
     psk::cp_async_commit();
@@ -785,8 +857,9 @@ greedy_pipe_kernel(const psk::RowPre* __restrict__ rows, const uint64_t* __restr
 }
 
 size_t greedy_pipe_smem(uint32_t I, uint32_t Ip) {
-  const size_t decide = (size_t)I * (4 * sizeof(int64_t) + sizeof(psk::InstTerms) + 4 * sizeof(int32_t)) +
-                        (size_t)Ip * (2 + 4 + 4) * sizeof(uint32_t);
+  // 4 eight-byte and 18 four-byte [Ip] arrays (q, S, key0, M; hit and T_pf rings, raises, room,
+  // dec0, f, tq, Bp, b, qr, B_max)
+  const size_t decide = (size_t)Ip * (4 * sizeof(int64_t) + 18 * sizeof(uint32_t));
   const size_t probe = (size_t)I * 3 * sizeof(uint32_t);
   return decide > probe ? decide : probe;
 }
