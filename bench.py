@@ -47,6 +47,30 @@ def _env_rank():
             int(os.environ.get("LOCAL_RANK", "0")))
 
 
+def rank_seed(config: int, rank: int) -> int:
+    """Seed of a rank's instance pool and window: each rank schedules an independent problem."""
+    import workload as W
+    return int(W.CONFIGS[config]["seed"]) + rank
+
+
+def max_over_ranks(value: float, device) -> float:
+    """The largest value over all ranks (the job is as slow as its slowest rank); identity when
+    torch.distributed is not initialised."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return float(value)
+    t = torch.tensor([float(value)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_rate(world: int, units_per_rank: int, ms_per_step: float) -> float:
+    """Whole-job throughput (weak scaling): every rank processes units_per_rank per step and the
+    step time is the slowest rank's."""
+    return world * units_per_rank / (ms_per_step / 1000.0)
+
+
 def _peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(p):
@@ -243,8 +267,7 @@ def main():
     over = {} if args.tpot is None else {"tpot_target_ms": args.tpot}
     if args.window_requests:
         over["window_requests"] = args.window_requests
-    seed = W.CONFIGS[args.config]["seed"] + rank
-    wl = W.generate(args.config, seed=seed, **over)
+    wl = W.generate(args.config, seed=rank_seed(args.config, rank), **over)
     win, ins = wl.window, wl.instances
     I, R = ins.I, win.R
     nb = np.diff(win.chain_off).astype(np.int64)
@@ -283,11 +306,7 @@ def main():
         torch.cuda.synchronize()
     if dist_on:
         dist.barrier()
-    ms = e0.elapsed_time(e1) / args.steps
-    if dist_on:
-        tt = torch.tensor([ms], device=f"cuda:{local}")
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        ms = float(tt.item())
+    ms = max_over_ranks(e0.elapsed_time(e1) / args.steps, f"cuda:{local}")
     path_counts = np.bincount(out["path"].cpu().numpy().astype(np.int64), minlength=3).tolist()
 
     # e2e: same step through the C ABI with page-locked host inputs and host outputs
@@ -303,11 +322,7 @@ def main():
     for _ in range(args.steps):
         sched.schedule_window(hwin, scores=("best", "path"))
     torch.cuda.synchronize()
-    e2e_ms = 1000 * (time.perf_counter() - t0) / args.steps
-    if dist_on:
-        tt = torch.tensor([e2e_ms], device=f"cuda:{local}")
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        e2e_ms = float(tt.item())
+    e2e_ms = max_over_ranks(1000 * (time.perf_counter() - t0) / args.steps, f"cuda:{local}")
     h2d = int(8 * (R + 1) + 8 * nb.sum() + 12 * R)
     d2h = int(R * (4 + 1 + 4) + R * (4 + 1))
 
@@ -336,10 +351,10 @@ def main():
                 "note": "serial per-request dependency chain decided on one SM: latency-bound, not "
                         "bandwidth-bound; traffic scaled by request count from the 2048-request ncu capture"}
     probe_achieved = probe_bytes / (probe_ms / 1000) / 1e9
-    line = {"metric": METRIC, "value": world * R * I / (ms / 1000), "unit": "scorings/s", "n_gpus": world,
+    line = {"metric": METRIC, "value": job_rate(world, R * I, ms), "unit": "scorings/s", "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f32+u64", "data": "synthetic (seeded generator)",
-            "decisions_per_s": world * R / (ms / 1000),
+            "decisions_per_s": job_rate(world, R, ms),
             "config": {"workload": WORKLOADS.get(args.config, str(args.config)), "instances": I,
                        "window_requests": R, "window_chain_blocks": int(nb.sum()),
                        "tpot_target_ms": float(win.tpot_target[0]), "probe": ("hinted per-lane search of rows without an earlier prefix in the window, the rest derived"
@@ -352,7 +367,7 @@ def main():
                                "algorithmic_bytes_per_launch": probe_bytes, "stats": pstats,
                                "traffic": None if probe_traffic is None else probe_traffic * n_probes},
             "roofline": roof,
-            "e2e": {"value": world * R * I / (e2e_ms / 1000), "unit": "scorings/s", "ms_per_step": e2e_ms,
+            "e2e": {"value": job_rate(world, R * I, e2e_ms), "unit": "scorings/s", "ms_per_step": e2e_ms,
                     "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
             # per step: window validation, last-block table, relations, base, probe (scratch rows),
             # probe (derived rows), score, greedy
