@@ -107,7 +107,8 @@ typedef struct {
  *                          parent_hash is neither 0 nor cached after the call fails with
  *                          PS_ERR_INVALID.
  *   track_lru             1: keep per-block (last_use, child count, parent) metadata so that
- *                         ps_advance_window can evict leaf-first LRU; 0: no eviction.
+ *                         ps_advance_window can evict leaf-first LRU (the tables must then hold fewer
+ *                         than 2^32 slots in total); 0: no eviction.
  *   max_active_requests   0: no request tracking.  > 0: each instance keeps up to this many queued
  *                         and this many decoding requests for ps_advance_window (streaming windows);
  *                         committed windows then need ps_window.out_tokens. */

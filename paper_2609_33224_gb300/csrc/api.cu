@@ -77,7 +77,8 @@ struct ps_ctx {
   uint8_t* d_dpath = nullptr;
   uint32_t* d_hchosen = nullptr;
   uint32_t* d_err = nullptr;
-  uint32_t* h_err = nullptr;
+  uint32_t* h_err = nullptr;   // pinned: the device error word, read at the end of each call
+  uint32_t* h_more = nullptr;  // pinned: "another eviction round" flag
   cudaEvent_t ev[kNumEv] = {};
   bool ev_used[kNumPhases] = {};
   bool probe_split = false;            // kEvRelDone / kEvProbeMid recorded in the last probe phase
@@ -85,9 +86,13 @@ struct ps_ctx {
   bool pending = false;
   psk::WindowDev pend_win{};
   const uint32_t* pend_out = nullptr;
-  // streaming: per-block LRU metadata, request store, capacities on the device
+  // streaming: per-block LRU metadata, request store, capacities on the device, eviction buffers
   bool lru = false;
   psk::LruMeta meta{nullptr, nullptr, nullptr};
+  void* d_leafbuf = nullptr;
+  uint32_t* d_nleaf = nullptr;
+  uint32_t* d_more = nullptr;
+  uint64_t max_instance_slots = 0;
   psk::ReqStore rq{};
   uint64_t* d_cap = nullptr;
   uint32_t* d_outtok = nullptr;
@@ -369,6 +374,10 @@ ps_status ps_create(const ps_config* cfg, ps_ctx** out) {
     obase += (nbkt + 63) / 64;
   }
   c->total_slots = base;
+  if (c->lru && c->total_slots >= (1ull << 32)) {
+    c->err = "track_lru needs fewer than 2^32 table slots in total (eviction keeps 32-bit slot indices)";
+    return bail(PS_ERR_INVALID);
+  }
   c->total_ovf = obase;
   const uint64_t dn = std::max<uint64_t>(16, 2 * c->max_blocks);  // delta slots: twice a window's blocks
   c->delta_nslots = dn;
@@ -400,6 +409,14 @@ ps_status ps_create(const ps_config* cfg, ps_ctx** out) {
        dalloc(c, &c->d_hchosen, c->Rmax) == cudaSuccess && dalloc(c, &c->d_err, 1) == cudaSuccess &&
        dalloc(c, &c->d_stats, kNumStats) == cudaSuccess &&
        dalloc(c, &c->d_cap, I) == cudaSuccess && dalloc(c, &c->d_outtok, c->Rmax) == cudaSuccess;
+  if (ok && c->lru) {
+    for (uint32_t i = 0; i < I; ++i)
+      c->max_instance_slots = std::max<uint64_t>(c->max_instance_slots, (uint64_t)td[i].nbkt * psk::kBucketSlots);
+    unsigned char* lb = nullptr;
+    ok = dalloc(c, &lb, pskl::evict_leafbuf_bytes(c->I)) == cudaSuccess && dalloc(c, &c->d_nleaf, I) == cudaSuccess &&
+         dalloc(c, &c->d_more, 1) == cudaSuccess;
+    c->d_leafbuf = lb;
+  }
   if (ok && c->lru)
     ok = dalloc(c, &c->meta.last_use, c->total_slots) == cudaSuccess &&
          dalloc(c, &c->meta.children, c->total_slots) == cudaSuccess &&
@@ -418,6 +435,8 @@ ps_status ps_create(const ps_config* cfg, ps_ctx** out) {
   }
   if (cudaMallocHost(&c->h_err, sizeof(uint32_t)) != cudaSuccess) return bail(PS_ERR_OOM);
   *c->h_err = 0;
+  if (cudaMallocHost(&c->h_more, sizeof(uint32_t)) != cudaSuccess) return bail(PS_ERR_OOM);
+  *c->h_more = 0;
   for (int e = 0; e < kNumEv; ++e)
     if (cudaEventCreate(&c->ev[e]) != cudaSuccess) return bail(PS_ERR_CUDA);
   bool set = cudaMemsetAsync(c->d_slots, 0, c->total_slots * sizeof(uint64_t), c->stream) == cudaSuccess &&
@@ -442,7 +461,7 @@ ps_status ps_create(const ps_config* cfg, ps_ctx** out) {
   if (c->lru)
     set = set && cudaMemsetAsync(c->meta.last_use, 0, c->total_slots * 4, c->stream) == cudaSuccess &&
           cudaMemsetAsync(c->meta.children, 0, c->total_slots * 4, c->stream) == cudaSuccess &&
-          cudaMemsetAsync(c->meta.parent, 0, c->total_slots * 8, c->stream) == cudaSuccess;
+          cudaMemsetAsync(c->meta.parent, 0xFF, c->total_slots * 8, c->stream) == cudaSuccess;  // kNoParent
   if (c->rq.M)
     set = set && cudaMemsetAsync(c->rq.q_head, 0, I * 4, c->stream) == cudaSuccess &&
           cudaMemsetAsync(c->rq.q_len, 0, I * 4, c->stream) == cudaSuccess &&
@@ -461,6 +480,7 @@ void ps_destroy(ps_ctx* c) {
     if (c->stream) cudaStreamSynchronize(c->stream);
     for (void* p : c->allocs) cudaFree(p);
     if (c->h_err) cudaFreeHost(c->h_err);
+    if (c->h_more) cudaFreeHost(c->h_more);
     for (cudaEvent_t e : c->ev)
       if (e) cudaEventDestroy(e);
     if (c->own_stream && c->stream) cudaStreamDestroy(c->stream);
@@ -734,8 +754,8 @@ ps_status ps_advance_window(ps_ctx* c, const ps_advance_params* p) {
   PS_TRY_CUDA(c, pskl::launch_advance(c->st, c->I, c->rq, c->model, p->window_ms, p->prefill_tokens, c->d_err,
                                       c->stream));
   if (p->evict)
-    PS_TRY_CUDA(c, pskl::launch_evict(c->d_slots, c->d_ovf, c->d_tdesc, c->I, c->d_count, c->d_cap, c->meta,
-                                      c->d_err, c->stream));
+    PS_TRY_CUDA(c, pskl::launch_evict(c->d_slots, c->d_tdesc, c->I, c->d_count, c->d_cap, c->meta, c->d_leafbuf,
+                                      c->d_nleaf, c->d_more, c->h_more, c->max_instance_slots, c->d_err, c->stream));
   return finish(c);
 }
 

@@ -246,7 +246,12 @@ __device__ __forceinline__ uint64_t main_find(const uint64_t* slots, const uint6
   return ~0ull;
 }
 
-// Per-block LRU metadata, parallel to the slot array (streaming caches only).
+// Per-block LRU metadata, parallel to the slot array (streaming caches only): the block's last use,
+// its number of cached children, and its parent's slot (kNoParent for a chain root or a parent that
+// was not cached when the block was inserted).  A slot is stable while its block is cached and a
+// parent outlives its children (eviction is leaf-first), so a cached block's parent slot stays valid.
+constexpr uint64_t kNoParent = ~0ull;
+constexpr uint64_t kLinkPending = ~1ull;  // inserted by a commit whose linking pass has not run yet
 struct LruMeta {
   uint32_t* last_use;
   uint32_t* children;
@@ -271,9 +276,9 @@ struct ReqStore {
 // Warp-cooperative insert of one key by the instance's only writer warp (all 32 lanes call it with
 // the same arguments).  Lanes 0-7 read bucket b1, lanes 8-15 bucket b2; the key goes to the emptier
 // one.  With LRU metadata (meta.last_use != nullptr) a new block records (last_use, 0 children,
-// parent) and its cached parent gains a child; an existing block only has its last_use raised.
-// parent_slot, if not ~0, is the parent's known slot (saves a lookup).  Returns the key's slot, or
-// ~0 if the table is full; *inserted tells whether the key is new.
+// its parent's slot) and its cached parent gains a child; an existing block only has its last_use
+// raised.  parent_slot, if not ~0, is the parent's known slot (saves a lookup).  Returns the key's
+// slot, or ~0 if the table is full; *inserted tells whether the key is new.
 __device__ __forceinline__ uint64_t warp_insert(uint64_t* slots, uint64_t* ovf, const TableDesc d, uint64_t key,
                                                 bool* inserted, LruMeta meta = LruMeta{nullptr, nullptr, nullptr},
                                                 uint64_t parent = 0, uint32_t last_use = 0,
@@ -315,21 +320,82 @@ __device__ __forceinline__ uint64_t warp_insert(uint64_t* slots, uint64_t* ovf, 
     if (target < 0) return ~0ull;
   }
   const uint64_t slot = __shfl_sync(0xffffffffu, idx, target);
+  uint64_t ps = kNoParent;
+  if (meta.last_use && parent != kEmpty) ps = parent_slot != ~0ull ? parent_slot : main_find(slots, ovf, d, parent);
   if (lane == target) {
     slots[slot] = key;
     if (meta.last_use) {
       meta.last_use[slot] = last_use;
       meta.children[slot] = 0;
-      meta.parent[slot] = parent;
+      meta.parent[slot] = ps;
     }
   }
-  if (meta.last_use && parent != kEmpty) {
-    const uint64_t ps = parent_slot != ~0ull ? parent_slot : main_find(slots, ovf, d, parent);
-    if (ps != ~0ull && lane == 0) meta.children[ps] += 1;
-  }
+  if (ps != kNoParent && lane == 0) meta.children[ps] += 1;
   __syncwarp();
   *inserted = true;
   return slot;
+}
+
+// Insert of one key by one thread while other threads insert other keys into the same table (each
+// key by one thread only; a key cached before the batch is found and left in place): both
+// candidate buckets are read, the emptier one (b1 on ties) is tried first, a slot is claimed by
+// compare-and-swap from empty, and if both buckets are full the key goes to the first bucket after
+// b1 with a free slot, setting the overflow bit of b1 and of every full bucket passed (the layout
+// lookups expect).  Placement can differ from a one-at-a-time build, the set of keys cannot.
+// Returns the key's slot (~0: the table is full); *inserted tells whether this thread stored it.
+__device__ __forceinline__ uint64_t thread_insert(uint64_t* slots, uint64_t* ovf, const TableDesc d, uint64_t key,
+                                                  bool* inserted) {
+  *inserted = false;
+  const uint64_t found = main_find(slots, ovf, d, key);  // already cached before this batch of inserts
+  if (found != ~0ull) return found;
+  const uint32_t b1 = fastrange32(key, d.nbkt);
+  const uint32_t b2 = fastrange32(remix(key), d.nbkt);
+  auto try_bucket = [&](uint32_t b, uint64_t* out) -> int {  // 1 claimed, 0 full, -1 key found
+    unsigned long long* base = reinterpret_cast<unsigned long long*>(slots + d.base + (uint64_t)b * kBucketSlots);
+#pragma unroll 1
+    for (int k = 0; k < kBucketSlots; ++k) {
+      const unsigned long long v = __ldcg(base + k);
+      if (v == key) {
+        *out = d.base + (uint64_t)b * kBucketSlots + k;
+        return -1;
+      }
+      if (v != kEmpty) continue;
+      const unsigned long long old = atomicCAS(base + k, kEmpty, (unsigned long long)key);
+      if (old == kEmpty || old == key) {
+        *out = d.base + (uint64_t)b * kBucketSlots + k;
+        return old == kEmpty ? 1 : -1;
+      }
+    }
+    return 0;
+  };
+  auto empties = [&](uint32_t b) {
+    const unsigned long long* base = reinterpret_cast<const unsigned long long*>(slots + d.base + (uint64_t)b * kBucketSlots);
+    int n = 0;
+#pragma unroll
+    for (int k = 0; k < kBucketSlots; ++k) n += __ldcg(base + k) == kEmpty;
+    return n;
+  };
+  uint64_t slot = ~0ull;
+  const bool first_b1 = empties(b1) >= empties(b2);
+  const uint32_t order[2] = {first_b1 ? b1 : b2, first_b1 ? b2 : b1};
+  for (int c = 0; c < 2; ++c) {
+    const int v = try_bucket(order[c], &slot);
+    if (v != 0) {
+      *inserted = v == 1;
+      return slot;
+    }
+  }
+  uint32_t b = b1;
+  for (uint32_t step = 0; step < d.nbkt; ++step) {
+    atomicOr(reinterpret_cast<unsigned long long*>(ovf + d.ovf + (b >> 6)), 1ull << (b & 63));
+    b = (b + 1 == d.nbkt) ? 0u : b + 1;
+    const int v = try_bucket(b, &slot);
+    if (v != 0) {
+      *inserted = v == 1;
+      return slot;
+    }
+  }
+  return ~0ull;
 }
 
 // The window's delta table: open addressing with linear probing over 16-byte slots, the home slot
@@ -888,9 +954,13 @@ cudaError_t launch_commit(uint64_t* slots, uint64_t* ovf, const psk::TableDesc* 
                           cudaStream_t s);
 cudaError_t launch_advance(psk::StateSoA st, uint32_t I, const psk::ReqStore& rq, const psk::DevModel& m,
                            float window_ms, uint64_t prefill_tokens, uint32_t* err, cudaStream_t s);
-cudaError_t launch_evict(uint64_t* slots, uint64_t* ovf, const psk::TableDesc* tdesc, uint32_t I,
-                         unsigned long long* count, const uint64_t* cap, psk::LruMeta meta, uint32_t* err,
-                         cudaStream_t s);
+// Leaf-first LRU eviction of every instance over capacity (rounds until none is; synchronises the
+// stream between rounds).  leafbuf holds evict_leafbuf_bytes(I) bytes; nleaf [I], more [1] device
+// words; more_host one pinned word; max_instance_slots the largest table (slots) of an instance.
+cudaError_t launch_evict(uint64_t* slots, const psk::TableDesc* tdesc, uint32_t I, unsigned long long* count,
+                         const uint64_t* cap, psk::LruMeta meta, void* leafbuf, uint32_t* nleaf, uint32_t* more,
+                         uint32_t* more_host, uint64_t max_instance_slots, uint32_t* err, cudaStream_t s);
+size_t evict_leafbuf_bytes(uint32_t I);
 cudaError_t launch_check_parents(const uint64_t* slots, const uint64_t* ovf, const psk::TableDesc* tdesc, uint32_t I,
                                  uint64_t nchains, const uint32_t* inst, const uint64_t* parent,
                                  uint32_t* err, int num_sms, cudaStream_t s);

@@ -60,53 +60,117 @@ __global__ void check_instances_kernel(uint32_t I, uint64_t nchains, const uint3
     if (inst[c] >= I) atomicOr(err, psk::kErrBadInstance);
 }
 
-// Commit: one warp per instance applies that instance's admitted requests in arrival order: the
-// cached prefix chain[0..h) is stamped last_use (lanes in parallel), the uncached blocks
-// chain[h..nb) are cached (stamped, parents linked), and with request tracking the request joins
-// the instance's FIFO queue with its uncached tokens as remaining prefill.
-__global__ void commit_kernel(uint64_t* slots, uint64_t* ovf, const psk::TableDesc* __restrict__ tdesc, uint32_t I,
-                              unsigned long long* count, psk::WindowDev w, const int32_t* __restrict__ assign,
-                              const uint32_t* __restrict__ hit_chosen, psk::LruMeta meta, uint32_t last_use,
-                              psk::ReqStore rq, const uint32_t* __restrict__ out_tokens, uint32_t* err) {
+// Commit of a scheduled window, in four passes so that every admitted request's blocks are handled
+// in parallel (within a window each (block, instance) pair is inserted at most once: a request
+// inserts chain[h, nb) on its pick with h the exact first miss there, so none of those blocks is
+// cached on that instance yet, neither by the committed caches nor by an earlier request):
+//   stamp   the cached prefix chain[0, h) gets last_use (every stamp writes the same value, so
+//           their order does not matter);
+//   insert  the uncached blocks chain[h, nb) are cached, stamped, with 0 children and their parent
+//           link pending;
+//   link    each new block records its parent's slot and the parent gains a child;
+//   queue   with request tracking, each instance appends its admitted requests to its FIFO queue
+//           in arrival order (one warp per instance).
+// One warp per request for the first three, lanes over the request's blocks.
+__global__ void commit_stamp_kernel(const uint64_t* slots, const uint64_t* ovf, const psk::TableDesc* __restrict__ tdesc,
+                                    psk::WindowDev w, const int32_t* __restrict__ assign,
+                                    const uint32_t* __restrict__ hit_chosen, psk::LruMeta meta, uint32_t last_use) {
+  const int lane = threadIdx.x & 31;
+  const uint32_t warps_total = (gridDim.x * blockDim.x) >> 5;
+  for (uint32_t r = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; r < w.R; r += warps_total) {
+    const int32_t j = assign[r];
+    if (j < 0) continue;
+    const psk::TableDesc d = tdesc[j];
+    const uint64_t o = w.off[r];
+    const uint64_t h = hit_chosen[r];
+    for (uint64_t k = lane; k < h; k += 32) {
+      const uint64_t s = psk::main_find(slots, ovf, d, w.hash[o + k]);
+      if (s != ~0ull && meta.last_use[s] < last_use) meta.last_use[s] = last_use;
+    }
+  }
+}
+
+__global__ void commit_insert_kernel(uint64_t* slots, uint64_t* ovf, const psk::TableDesc* __restrict__ tdesc,
+                                     unsigned long long* count, psk::WindowDev w, const int32_t* __restrict__ assign,
+                                     const uint32_t* __restrict__ hit_chosen, psk::LruMeta meta, uint32_t last_use,
+                                     uint32_t* err) {
+  const int lane = threadIdx.x & 31;
+  const uint32_t warps_total = (gridDim.x * blockDim.x) >> 5;
+  for (uint32_t r = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; r < w.R; r += warps_total) {
+    const int32_t j = assign[r];
+    if (j < 0) continue;
+    const psk::TableDesc d = tdesc[j];
+    const uint64_t o = w.off[r];
+    const uint64_t nb = w.off[r + 1] - o;
+    const uint64_t h = hit_chosen[r];
+    uint32_t added = 0;
+    bool full = false;
+    for (uint64_t k = h + lane; k < nb; k += 32) {
+      const uint64_t key = w.hash[o + k];
+      if (key == psk::kEmpty || key == psk::kTomb) continue;
+      bool ins = false;
+      const uint64_t slot = psk::thread_insert(slots, ovf, d, key, &ins);
+      if (slot == ~0ull) {
+        full = true;
+        continue;
+      }
+      if (ins) {
+        ++added;
+        if (meta.last_use) {
+          meta.last_use[slot] = last_use;
+          meta.children[slot] = 0;
+          meta.parent[slot] = psk::kLinkPending;
+        }
+      } else if (meta.last_use && meta.last_use[slot] < last_use) {
+        meta.last_use[slot] = last_use;
+      }
+    }
+#pragma unroll
+    for (int s = 16; s > 0; s >>= 1) added += __shfl_xor_sync(0xffffffffu, added, s);
+    full = __any_sync(0xffffffffu, full);
+    if (lane == 0) {
+      if (added) atomicAdd(count + j, (unsigned long long)added);
+      if (full) atomicOr(err, psk::kErrTableFull);
+    }
+  }
+}
+
+__global__ void commit_link_kernel(const uint64_t* slots, const uint64_t* ovf, const psk::TableDesc* __restrict__ tdesc,
+                                   psk::WindowDev w, const int32_t* __restrict__ assign,
+                                   const uint32_t* __restrict__ hit_chosen, psk::LruMeta meta) {
+  const int lane = threadIdx.x & 31;
+  const uint32_t warps_total = (gridDim.x * blockDim.x) >> 5;
+  for (uint32_t r = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; r < w.R; r += warps_total) {
+    const int32_t j = assign[r];
+    if (j < 0) continue;
+    const psk::TableDesc d = tdesc[j];
+    const uint64_t o = w.off[r];
+    const uint64_t nb = w.off[r + 1] - o;
+    const uint64_t h = hit_chosen[r];
+    for (uint64_t k = h + lane; k < nb; k += 32) {
+      const uint64_t s = psk::main_find(slots, ovf, d, w.hash[o + k]);
+      if (s == ~0ull || meta.parent[s] != psk::kLinkPending) continue;  // not inserted by this commit
+      const uint64_t ps = k > 0 ? psk::main_find(slots, ovf, d, w.hash[o + k - 1]) : ~0ull;
+      meta.parent[s] = ps == ~0ull ? psk::kNoParent : ps;
+      if (ps != ~0ull) atomicAdd(meta.children + ps, 1u);
+    }
+  }
+}
+
+__global__ void commit_queue_kernel(uint32_t I, psk::WindowDev w, const int32_t* __restrict__ assign,
+                                    const uint32_t* __restrict__ hit_chosen, psk::ReqStore rq,
+                                    const uint32_t* __restrict__ out_tokens, uint32_t* err) {
   const int lane = threadIdx.x & 31;
   const uint32_t warps_total = (gridDim.x * blockDim.x) >> 5;
   for (uint32_t i = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; i < I; i += warps_total) {
-    const psk::TableDesc d = tdesc[i];
-    unsigned long long added = 0;
-    bool full = false, overflow = false;
+    bool overflow = false;
     for (uint32_t r0 = 0; r0 < w.R; r0 += 32) {
       const uint32_t r = r0 + lane;
       unsigned mine = __ballot_sync(0xffffffffu, r < w.R && assign[r] == (int32_t)i);
-      while (mine) {
-        const int l = __ffs(mine) - 1;
+      while (mine) {  // in arrival order
+        const uint32_t rr = r0 + (uint32_t)(__ffs(mine) - 1);
         mine &= mine - 1;
-        const uint32_t rr = r0 + l;
-        const uint64_t o = w.off[rr];
-        const uint64_t nb = w.off[rr + 1] - o;
-        const uint64_t h = hit_chosen[rr];
-        if (meta.last_use) {
-          for (uint64_t k = lane; k < h; k += 32) {
-            const uint64_t s = psk::main_find(slots, ovf, d, w.hash[o + k]);
-            if (s != ~0ull && meta.last_use[s] < last_use) meta.last_use[s] = last_use;
-          }
-          __syncwarp();
-        }
-        uint64_t prev_key = h ? w.hash[o + h - 1] : psk::kEmpty, prev_slot = ~0ull;
-        for (uint64_t k = h; k < nb && !full; ++k) {
-          const uint64_t key = w.hash[o + k];
-          if (key == psk::kEmpty || key == psk::kTomb) {
-            prev_key = key;
-            prev_slot = ~0ull;
-            continue;
-          }
-          bool ins = false;
-          const uint64_t slot = psk::warp_insert(slots, ovf, d, key, &ins, meta, prev_key, last_use, prev_slot);
-          if (slot == ~0ull) full = true;
-          if (ins) ++added;
-          prev_key = key;
-          prev_slot = slot;
-        }
-        if (rq.M && lane == 0) {
+        if (lane == 0) {
           const uint32_t len = rq.q_len[i];
           if (len >= rq.M) {
             overflow = true;
@@ -114,18 +178,14 @@ __global__ void commit_kernel(uint64_t* slots, uint64_t* ovf, const psk::TableDe
             const uint64_t at = (uint64_t)i * rq.M + (rq.q_head[i] + len) % rq.M;
             rq.q_L[at] = w.L[rr];
             rq.q_out[at] = out_tokens ? out_tokens[rr] : 0u;
-            rq.q_rem[at] = (uint64_t)((int64_t)w.L[rr] - 16 * (int64_t)h);
+            rq.q_rem[at] = (uint64_t)((int64_t)w.L[rr] - 16 * (int64_t)hit_chosen[rr]);
             rq.q_len[i] = len + 1;
           }
         }
         __syncwarp();
       }
     }
-    if (lane == 0) {
-      count[i] += added;
-      if (full) atomicOr(err, psk::kErrTableFull);
-      if (overflow) atomicOr(err, psk::kErrRequestsFull);
-    }
+    if (lane == 0 && overflow) atomicOr(err, psk::kErrRequestsFull);
   }
 }
 
@@ -226,23 +286,27 @@ __global__ void advance_kernel(psk::StateSoA st, uint32_t I, psk::ReqStore rq, p
   }
 }
 
-// Leaf-first LRU eviction, one thread block per instance over capacity.  Per round: collect the
-// instance's leaves (cached blocks with no cached child) into shared memory, sort them by
-// (last_use, hash), then thread 0 evicts in order, taking the smaller of the next sorted leaf and the
-// smallest parent that became a leaf (a small heap).  Every evicted block only ever makes its parent
-// a leaf, and a leaf outside the first E sorted ones can never be among E evictions, so a round of
-// at most kHeapMax evictions reproduces the one-at-a-time rule exactly; rounds repeat until the
-// instance is at capacity.
+// Leaf-first LRU eviction of the instances over capacity, in rounds of two kernels:
+//   collect  all SMs scan the over-capacity instances' slots (coalesced) and append each leaf (a
+//            cached block with no cached child) to its instance's leaf buffer;
+//   evict    one thread block per over-capacity instance sorts its leaves by (last_use, hash), then
+//            thread 0 evicts in order, taking the smaller of the next sorted leaf and the smallest
+//            parent that became a leaf (a small heap); the parent is reached through its stored slot.
+// Every evicted block only ever makes its parent a leaf, and a leaf outside the first E sorted ones
+// can never be among E evictions, so a round of at most kHeapMax evictions reproduces the
+// one-at-a-time rule exactly; the host repeats rounds while an instance is still over capacity.
 constexpr int kLeafMax = 4096;
 constexpr int kHeapMax = 2048;
 constexpr int kEvictThreads = 256;
+constexpr int kCollectThreads = 256;
+constexpr uint32_t kCollectSlotsPerThread = 8;
 
 struct Leaf {
   uint32_t last_use;
-  uint32_t pad;
+  uint32_t slot;
   uint64_t hash;
-  uint64_t slot;
 };
+static_assert(sizeof(Leaf) == 16, "a leaf is one 16-byte word");
 
 __device__ __forceinline__ bool leaf_less(const Leaf& a, const Leaf& b) {
   return a.last_use != b.last_use ? a.last_use < b.last_use : a.hash < b.hash;
@@ -279,93 +343,84 @@ __device__ __forceinline__ Leaf heap_pop(Leaf* h, int& n) {
   return top;
 }
 
+// grid: (slot chunks, instances)
+__global__ void __launch_bounds__(kCollectThreads)
+leaf_collect_kernel(const uint64_t* __restrict__ slots, const psk::TableDesc* __restrict__ tdesc,
+                    const unsigned long long* __restrict__ count, const uint64_t* __restrict__ cap, psk::LruMeta meta,
+                    Leaf* __restrict__ leafbuf, uint32_t* __restrict__ nleaf) {
+  const uint32_t i = blockIdx.y;
+  if (count[i] <= cap[i]) return;  // block-uniform
+  const psk::TableDesc d = tdesc[i];
+  const uint64_t nslots = (uint64_t)d.nbkt * psk::kBucketSlots;
+  const uint64_t stride = (uint64_t)gridDim.x * kCollectThreads;
+  for (uint64_t x = (uint64_t)blockIdx.x * kCollectThreads + threadIdx.x; x < nslots; x += stride) {
+    const uint64_t s = d.base + x;
+    const uint64_t key = __ldcs(slots + s);
+    if (key == psk::kEmpty || key == psk::kTomb || meta.children[s] != 0u) continue;
+    const uint32_t at = atomicAdd(nleaf + i, 1u);
+    if (at < (uint32_t)kLeafMax) leafbuf[(uint64_t)i * kLeafMax + at] = Leaf{meta.last_use[s], (uint32_t)s, key};
+  }
+}
+
 __global__ void __launch_bounds__(kEvictThreads)
-evict_kernel(uint64_t* slots, uint64_t* ovf, const psk::TableDesc* __restrict__ tdesc, uint32_t I,
-             unsigned long long* count, const uint64_t* __restrict__ cap, psk::LruMeta meta, uint32_t* err) {
+evict_kernel(uint64_t* slots, unsigned long long* count, const uint64_t* __restrict__ cap, psk::LruMeta meta,
+             const Leaf* __restrict__ leafbuf, const uint32_t* __restrict__ nleaf, uint32_t* more, uint32_t* err) {
   extern __shared__ unsigned long long ev_smem[];
   Leaf* leaves = reinterpret_cast<Leaf*>(ev_smem);
   Leaf* heap = leaves + kLeafMax;
-  __shared__ uint32_t s_nleaf;
-  __shared__ int s_stop;
-  for (uint32_t i = blockIdx.x; i < I; i += gridDim.x) {
-    const psk::TableDesc d = tdesc[i];
-    const uint64_t nslots = (uint64_t)d.nbkt * psk::kBucketSlots;
-    for (;;) {
-      const unsigned long long cnt = count[i];
-      if (cnt <= cap[i]) break;
-      const uint64_t E = cnt - cap[i];
-      if (threadIdx.x == 0) {
-        s_nleaf = 0;
-        s_stop = 0;
-      }
-      __syncthreads();
-      for (uint64_t x = threadIdx.x; x < nslots; x += kEvictThreads) {
-        const uint64_t s = d.base + x;
-        const uint64_t key = slots[s];
-        if (key != psk::kEmpty && meta.children[s] == 0) {
-          const uint32_t at = atomicAdd(&s_nleaf, 1u);
-          if (at < kLeafMax) leaves[at] = Leaf{meta.last_use[s], 0u, key, s};
-        }
-      }
-      __syncthreads();
-      const uint32_t nleaf = s_nleaf;
-      if (nleaf > kLeafMax || nleaf == 0) {
-        if (threadIdx.x == 0) atomicOr(err, psk::kErrLeavesFull);
-        break;
-      }
-      // bitonic sort of the leaves (padded to a power of two with +infinity)
-      uint32_t np2 = 1;
-      while (np2 < nleaf) np2 <<= 1;
-      for (uint32_t x = nleaf + threadIdx.x; x < np2; x += kEvictThreads)
-        leaves[x] = Leaf{0xFFFFFFFFu, 0u, ~0ull, ~0ull};
-      __syncthreads();
-      for (uint32_t size = 2; size <= np2; size <<= 1) {
-        for (uint32_t stride = size >> 1; stride > 0; stride >>= 1) {
-          for (uint32_t x = threadIdx.x; x < np2; x += kEvictThreads) {
-            const uint32_t y = x ^ stride;
-            if (y > x) {
-              const bool up = (x & size) == 0;
-              const Leaf a = leaves[x], b = leaves[y];
-              if (leaf_less(b, a) == up) {
-                leaves[x] = b;
-                leaves[y] = a;
-              }
-            }
-          }
-          __syncthreads();
-        }
-      }
-      if (threadIdx.x == 0) {
-        const uint64_t todo = E < (uint64_t)kHeapMax ? E : (uint64_t)kHeapMax;
-        uint32_t ptr = 0;
-        int hn = 0;
-        uint64_t evicted = 0;
-        while (evicted < todo) {
-          const bool from_sorted = ptr < nleaf && (hn == 0 || leaf_less(leaves[ptr], heap[0]));
-          if (!from_sorted && hn == 0) break;
-          const Leaf v = from_sorted ? leaves[ptr++] : heap_pop(heap, hn);
-          const uint64_t parent = meta.parent[v.slot];
-          slots[v.slot] = psk::kEmpty;
-          meta.last_use[v.slot] = 0;
-          meta.children[v.slot] = 0;
-          meta.parent[v.slot] = 0;
-          ++evicted;
-          if (parent != psk::kEmpty) {
-            const uint64_t ps = psk::main_find(slots, ovf, d, parent);
-            if (ps != ~0ull) {
-              const uint32_t c = meta.children[ps] - 1;
-              meta.children[ps] = c;
-              if (c == 0) heap_push(heap, hn, Leaf{meta.last_use[ps], 0u, parent, ps});
-            }
+  const uint32_t i = blockIdx.x;
+  const unsigned long long cnt = count[i];
+  if (cnt <= cap[i]) return;  // block-uniform
+  const uint32_t n = nleaf[i];
+  if (n > (uint32_t)kLeafMax || n == 0) {
+    if (threadIdx.x == 0) atomicOr(err, psk::kErrLeavesFull);
+    return;
+  }
+  uint32_t np2 = 1;
+  while (np2 < n) np2 <<= 1;
+  for (uint32_t x = threadIdx.x; x < np2; x += kEvictThreads)
+    leaves[x] = x < n ? leafbuf[(uint64_t)i * kLeafMax + x] : Leaf{0xFFFFFFFFu, 0xFFFFFFFFu, ~0ull};
+  __syncthreads();
+  for (uint32_t size = 2; size <= np2; size <<= 1) {  // bitonic sort by (last_use, hash)
+    for (uint32_t stride = size >> 1; stride > 0; stride >>= 1) {
+      for (uint32_t x = threadIdx.x; x < np2; x += kEvictThreads) {
+        const uint32_t y = x ^ stride;
+        if (y > x) {
+          const bool up = (x & size) == 0;
+          const Leaf a = leaves[x], b = leaves[y];
+          if (leaf_less(b, a) == up) {
+            leaves[x] = b;
+            leaves[y] = a;
           }
         }
-        count[i] = cnt - evicted;
-        if (evicted == 0) s_stop = 1;
       }
       __syncthreads();
-      if (s_stop) break;
     }
-    __syncthreads();
+  }
+  if (threadIdx.x == 0) {
+    const uint64_t E = cnt - cap[i];
+    const uint64_t todo = E < (uint64_t)kHeapMax ? E : (uint64_t)kHeapMax;
+    uint32_t ptr = 0;
+    int hn = 0;
+    uint64_t evicted = 0;
+    while (evicted < todo) {
+      const bool from_sorted = ptr < n && (hn == 0 || leaf_less(leaves[ptr], heap[0]));
+      if (!from_sorted && hn == 0) break;
+      const Leaf v = from_sorted ? leaves[ptr++] : heap_pop(heap, hn);
+      const uint64_t ps = meta.parent[v.slot];
+      slots[v.slot] = psk::kEmpty;
+      meta.last_use[v.slot] = 0;
+      meta.children[v.slot] = 0;
+      meta.parent[v.slot] = psk::kNoParent;
+      ++evicted;
+      if (ps != psk::kNoParent && ps != psk::kLinkPending) {
+        const uint32_t c = meta.children[ps] - 1;
+        meta.children[ps] = c;
+        if (c == 0) heap_push(heap, hn, Leaf{meta.last_use[ps], (uint32_t)ps, slots[ps]});
+      }
+    }
+    count[i] = cnt - evicted;
+    if (evicted > 0 && cnt - evicted > cap[i]) atomicOr(more, 1u);
   }
 }
 
@@ -417,12 +472,29 @@ cudaError_t launch_commit(uint64_t* slots, uint64_t* ovf, const psk::TableDesc* 
                           const uint32_t* hit_chosen, psk::LruMeta meta, uint32_t last_use,
                           const psk::ReqStore& rq, const uint32_t* out_tokens, uint32_t* err, int num_sms,
                           cudaStream_t s) {
-  (void)num_sms;
   if (w.R == 0) return cudaSuccess;
-  const uint32_t warps_per_block = 4;
-  commit_kernel<<<(I + warps_per_block - 1) / warps_per_block, 32 * warps_per_block, 0, s>>>(
-      slots, ovf, tdesc, I, count, w, assign, hit_chosen, meta, last_use, rq, out_tokens, err);
-  return cudaGetLastError();
+  uint32_t g = (w.R + 7) / 8;  // one warp per request, 8 per block
+  if (g > (uint32_t)num_sms * 16) g = (uint32_t)num_sms * 16;
+  if (meta.last_use) {
+    commit_stamp_kernel<<<g, 256, 0, s>>>(slots, ovf, tdesc, w, assign, hit_chosen, meta, last_use);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+  }
+  commit_insert_kernel<<<g, 256, 0, s>>>(slots, ovf, tdesc, count, w, assign, hit_chosen, meta, last_use, err);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  if (meta.last_use) {
+    commit_link_kernel<<<g, 256, 0, s>>>(slots, ovf, tdesc, w, assign, hit_chosen, meta);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+  }
+  if (rq.M) {
+    const uint32_t warps_per_block = 4;
+    commit_queue_kernel<<<(I + warps_per_block - 1) / warps_per_block, 32 * warps_per_block, 0, s>>>(
+        I, w, assign, hit_chosen, rq, out_tokens, err);
+    e = cudaGetLastError();
+  }
+  return e;
 }
 
 cudaError_t launch_advance(psk::StateSoA st, uint32_t I, const psk::ReqStore& rq, const psk::DevModel& m,
@@ -433,15 +505,31 @@ cudaError_t launch_advance(psk::StateSoA st, uint32_t I, const psk::ReqStore& rq
   return cudaGetLastError();
 }
 
-cudaError_t launch_evict(uint64_t* slots, uint64_t* ovf, const psk::TableDesc* tdesc, uint32_t I,
-                         unsigned long long* count, const uint64_t* cap, psk::LruMeta meta, uint32_t* err,
-                         cudaStream_t s) {
+cudaError_t launch_evict(uint64_t* slots, const psk::TableDesc* tdesc, uint32_t I, unsigned long long* count,
+                         const uint64_t* cap, psk::LruMeta meta, void* leafbuf, uint32_t* nleaf, uint32_t* more,
+                         uint32_t* more_host, uint64_t max_instance_slots, uint32_t* err, cudaStream_t s) {
   const size_t smem = (size_t)(kLeafMax + kHeapMax) * sizeof(Leaf);
   cudaError_t e = cudaFuncSetAttribute(evict_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
-  evict_kernel<<<I, kEvictThreads, smem, s>>>(slots, ovf, tdesc, I, count, cap, meta, err);
-  return cudaGetLastError();
+  const uint64_t per_block = (uint64_t)kCollectThreads * kCollectSlotsPerThread;
+  const unsigned gx = (unsigned)((max_instance_slots + per_block - 1) / per_block);
+  for (int round = 0; round < 4096; ++round) {
+    if ((e = cudaMemsetAsync(nleaf, 0, (size_t)I * sizeof(uint32_t), s)) != cudaSuccess) return e;
+    if ((e = cudaMemsetAsync(more, 0, sizeof(uint32_t), s)) != cudaSuccess) return e;
+    leaf_collect_kernel<<<dim3(gx ? gx : 1u, I), kCollectThreads, 0, s>>>(slots, tdesc, count, cap, meta,
+                                                                           static_cast<Leaf*>(leafbuf), nleaf);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    evict_kernel<<<I, kEvictThreads, smem, s>>>(slots, count, cap, meta, static_cast<const Leaf*>(leafbuf), nleaf,
+                                                more, err);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    if ((e = cudaMemcpyAsync(more_host, more, sizeof(uint32_t), cudaMemcpyDeviceToHost, s)) != cudaSuccess) return e;
+    if ((e = cudaStreamSynchronize(s)) != cudaSuccess) return e;
+    if (*more_host == 0u) break;
+  }
+  return cudaSuccess;
 }
+
+size_t evict_leafbuf_bytes(uint32_t I) { return (size_t)I * kLeafMax * sizeof(Leaf); }
 
 cudaError_t launch_check_parents(const uint64_t* slots, const uint64_t* ovf, const psk::TableDesc* tdesc, uint32_t I,
                                  uint64_t nchains, const uint32_t* inst, const uint64_t* parent,
