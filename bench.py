@@ -149,6 +149,15 @@ def probe_algorithmic_bytes(st: dict, I: int, with_tpf: bool) -> tuple[int, int]
     return int(nbytes), int(lookups)
 
 
+def score_algorithmic_bytes(R: int, I: int, per_pair_outputs: bool) -> int:
+    """Bytes the fused score kernel must move in one launch: the u32 hit of every pair read; with
+    per-pair outputs the f32 TPOT, f32 TTFT and u8 class of every pair written; per request its
+    prompt length and two targets read and its pick (i32) and path (u8) written; per instance its
+    state (b, qr, B_max as i32; q, S, M_KV as i64) read."""
+    per_pair = 4 + ((4 + 4 + 1) if per_pair_outputs else 0)
+    return int(R * I * per_pair + R * (12 + 5) + I * 36)
+
+
 def profile_figure(name: str, label: str):
     """A per-unit DRAM figure ("<label>: <number>") from a committed ncu summary under profiles/, or
     None when the summary is absent."""
@@ -404,6 +413,26 @@ def main():
     h2d = int(8 * (R + 1) + 8 * nb.sum() + 12 * R)
     d2h = int(R * (4 + 1 + 4) + R * (4 + 1))
 
+    # The scoring call alone (ps_score_window, rows A1-A6): every per-pair output (hits, TPOT, TTFT,
+    # class) and the per-request pick written to device buffers, timed the same way.
+    want = ("hits", "tpot", "ttft", "cls", "best", "path")
+    for _ in range(args.warmup):
+        sched.score_window(dwin, want=want, device_outputs=True)
+    skern = {"probe": [], "score": [], "relations": [], "probe_scratch": [], "probe_derived": []}
+    torch.cuda.synchronize()
+    e0.record(stream)
+    for _ in range(args.steps):
+        sched.score_window(dwin, want=want, device_outputs=True)
+        t = sched.timings()
+        for k in skern:
+            skern[k].append(t[k])
+    e1.record(stream)
+    torch.cuda.synchronize()
+    score_call_ms = max_over_ranks(e0.elapsed_time(e1) / args.steps, f"cuda:{local}")
+    skm = {k: float(np.mean(v)) for k, v in skern.items()}
+    score_bytes = score_algorithmic_bytes(R, I, per_pair_outputs=True)
+    score_achieved = score_bytes / (skm["score"] / 1000) / 1e9
+
     km = {k: float(np.mean(v)) for k, v in kern.items()}
     phases = {k: km[k] for k in ("probe", "score", "greedy")}
     dominant = max(phases, key=phases.get)
@@ -411,6 +440,7 @@ def main():
     probe_ms = km["probe_scratch"] + max(0.0, km["probe_derived"])
     greedy_traffic = profile_figure("greedy_pipe_production_window_1024x2048.md", "DRAM bytes per request")
     probe_traffic = profile_figure("probe_search_production_window_1024x2048.md", "DRAM bytes per lookup")
+    score_traffic = profile_figure("score_rows_production_window_1024x8192.md", "DRAM bytes per request")
     if dominant == "probe":
         achieved = probe_bytes / (probe_ms / 1000) / 1e9
         roof = {"bound": "hbm", "kernel": "probe_search_kernel + probe_derived_kernel", "achieved": achieved,
@@ -445,6 +475,16 @@ def main():
                                "algorithmic_bytes_per_launch": probe_bytes, "stats": pstats,
                                "traffic": None if probe_traffic is None else probe_traffic * n_probes},
             "roofline": roof,
+            "scoring_call": {"what": "ps_score_window with hits, TPOT, TTFT and class of every pair and the "
+                                     "per-request pick written to device buffers",
+                             "ms": score_call_ms, "scorings_per_s": job_rate(world, R * I, score_call_ms),
+                             "kernel_ms": skm,
+                             "score_roofline": {"bound": "hbm", "kernel": "score_rows_kernel",
+                                                "achieved": score_achieved, "peak": peak, "unit": "GB/s",
+                                                "frac": score_achieved / peak, "peak_source": peak_src,
+                                                "algorithmic_bytes_per_launch": score_bytes,
+                                                "traffic": (None if score_traffic is None
+                                                            else score_traffic * R)}},
             "e2e": {"value": job_rate(world, R * I, e2e_ms), "unit": "scorings/s", "ms_per_step": e2e_ms,
                     "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
             # per step: window validation, last-block table, relations, base, probe (scratch rows),

@@ -648,9 +648,12 @@ __device__ __forceinline__ bool mbar_wait_bounded(uint64_t* mbar, uint32_t parit
 // Every operation is an explicitly rounded fp32 intrinsic in the order the header documents, so
 // nothing is fused or reassociated.
 
-// int64 -> fp32, round to nearest: the 32-bit conversion when the value fits (the same result).
+// int64 -> fp32, round to nearest: the 32-bit conversion when the value fits (the same result).  The
+// 64-bit conversion is kept out of line, so values that fit (all token counts here) never issue it.
+static __device__ __noinline__ float i64_to_f32_wide(int64_t v) { return __ll2float_rn(v); }
 __device__ __forceinline__ float i64_to_f32(int64_t v) {
-  return v == (int64_t)(int32_t)v ? __int2float_rn((int32_t)v) : __ll2float_rn(v);
+  if (v == (int64_t)(int32_t)v) return __int2float_rn((int32_t)v);
+  return i64_to_f32_wide(v);
 }
 
 // Eq. 6 with the Section 5.3 empirical C and C^2 terms.
@@ -706,23 +709,23 @@ __device__ __forceinline__ PairEval eval_pair(const DevModel& m, const RowConst&
   PairEval e;
   const int64_t c = 16 * (int64_t)h;
   const int64_t n = (int64_t)rc.L - c;
-  const float tpf = t_pf(m, __ll2float_rn(n), __ll2float_rn(c));
+  const float tpf = t_pf(m, i64_to_f32(n), i64_to_f32(c));
   e.n = n;
   e.W = __fsub_rn(tpf, rc.t_cached);
   const int64_t Bp = (int64_t)b + qr + 1;
   const int64_t Sp = S + (int64_t)rc.L;
   e.inA = (Bp <= (int64_t)Bmax) && (Sp <= M);
-  float dec = __fadd_rn(m.b0, __fmul_rn(m.b1, __ll2float_rn(Bp)));
-  dec = __fadd_rn(dec, __fmul_rn(m.b2, __ll2float_rn(Sp)));
+  float dec = __fadd_rn(m.b0, __fmul_rn(m.b1, i64_to_f32(Bp)));
+  dec = __fadd_rn(dec, __fmul_rn(m.b2, i64_to_f32(Sp)));
   dec = __fmul_rn(dec, ema_factor(m, Bp));
   if (m.interference_mode == 0) {
-    e.tpot = __fadd_rn(dec, __fmul_rn(m.g_q, __ll2float_rn(q + n)));
+    e.tpot = __fadd_rn(dec, __fmul_rn(m.g_q, i64_to_f32(q + n)));
   } else {
     const float den = m.lout > 1.0f ? m.lout : 1.0f;
     const float interf = ((int64_t)b + qr > 0) ? __fdiv_rn(tpf, den) : 0.0f;
     e.tpot = __fadd_rn(dec, interf);
   }
-  const float tq = __fadd_rn(__fmul_rn(m.a0, __int2float_rn(qr)), __fmul_rn(m.a1, __ll2float_rn(q)));
+  const float tq = __fadd_rn(__fmul_rn(m.a0, __int2float_rn(qr)), __fmul_rn(m.a1, i64_to_f32(q)));
   e.ttft = __fadd_rn(tpf, tq);
   return e;
 }
@@ -748,9 +751,9 @@ __device__ __forceinline__ int32_t kv_room(int64_t S, int64_t M) {
 __device__ __forceinline__ InstTerms inst_terms(const DevModel& m, int32_t b, int32_t qr, int64_t q, int32_t Bmax) {
   InstTerms x;
   const int64_t Bp = (int64_t)b + qr + 1;
-  x.dec0 = __fadd_rn(m.b0, __fmul_rn(m.b1, __ll2float_rn(Bp)));
+  x.dec0 = __fadd_rn(m.b0, __fmul_rn(m.b1, i64_to_f32(Bp)));
   x.f = ema_factor(m, Bp);
-  x.tq = __fadd_rn(__fmul_rn(m.a0, __int2float_rn(qr)), __fmul_rn(m.a1, __ll2float_rn(q)));
+  x.tq = __fadd_rn(__fmul_rn(m.a0, __int2float_rn(qr)), __fmul_rn(m.a1, i64_to_f32(q)));
   x.Bp = (int32_t)Bp;
   x.okB = Bp <= (int64_t)Bmax;
   return x;

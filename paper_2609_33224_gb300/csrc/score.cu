@@ -1,62 +1,304 @@
 // Fused score kernel: hit lengths + instance state -> predicted latencies, Algorithm 1's admission
 // sets and the per-request pick, each request independently against the same state.
 //
-// One warp per request (grid-stride).  Lane l handles instances l, l+32, ...  Pass 1 evaluates the
-// capacity guard and the recompute cost W (Alg. 1 KVC-first filtering) and reduces W_min over A with
-// warp shuffles; pass 2 classifies each pair (Eq. 8 filter, TPOT and TTFT admission), writes the
-// optional per-pair outputs, and reduces the lexicographic (class, value, instance) key to the
-// pick: D-C-Q inside T, the LMetric product inside C when T is empty, Reject when A is empty.
+// The instance terms that do not depend on the request (InstTerms, the free KV room with the
+// decode-slot guard folded in, q, S and the class-0 key bits of (b, qr)) are computed once per
+// thread block into shared memory as padded structure-of-arrays.  One warp then takes one request
+// at a time: lane l owns the instances 128 v + 4 l .. 128 v + 4 l + 3 of each 128-instance chunk v,
+// so a row of hits is read with one 16-byte load per lane and chunk, and the per-pair outputs
+// (TPOT, TTFT as float4, the classes as one 32-bit word) are written with one store per lane and
+// chunk.  Pass 1 evaluates the capacity guard and the recompute cost W (Alg. 1 KVC-first filtering)
+// and reduces W_min over A; pass 2 classifies each pair (Eq. 8 filter, TPOT and TTFT admission)
+// and reduces the packed (class, value) key to the pick: D-C-Q inside T, the LMetric product inside
+// C when T is empty, Reject when A is empty.  Pass 2 takes the hits from registers; rows of more
+// than 128 NV instances are taken in pieces of NV chunks, each read again for pass 2.
 #include "ps_internal.cuh"
 
 namespace {
 
-__global__ void __launch_bounds__(256)
+constexpr int kScoreThreads = 256;
+
+// Shared-memory instance arrays, each [Ip] (I rounded up to a multiple of 4), 8-byte arrays first.
+struct ScoreSmem {
+  int64_t* q;
+  int64_t* S;
+  uint64_t* k0;    // class-0 key bits of (b, qr)
+  int32_t* room;   // free KV room M_KV - S, -1 when the decode-slot guard fails or past I
+  float* dec0;
+  float* f;
+  float* tq;
+  int32_t* Bp;
+};
+
+__device__ __forceinline__ ScoreSmem score_smem(unsigned long long* raw, uint32_t Ip) {
+  ScoreSmem s;
+  s.q = reinterpret_cast<int64_t*>(raw);
+  s.S = s.q + Ip;
+  s.k0 = reinterpret_cast<uint64_t*>(s.S + Ip);
+  s.room = reinterpret_cast<int32_t*>(s.k0 + Ip);
+  s.dec0 = reinterpret_cast<float*>(s.room + Ip);
+  s.f = s.dec0 + Ip;
+  s.tq = s.f + Ip;
+  s.Bp = reinterpret_cast<int32_t*>(s.tq + Ip);
+  return s;
+}
+
+// Four consecutive shared-memory elements (16-byte aligned) with 16-byte loads.
+__device__ __forceinline__ void lds4(const float* p, float (&v)[4]) {
+  const float4 x = *reinterpret_cast<const float4*>(p);
+  v[0] = x.x;
+  v[1] = x.y;
+  v[2] = x.z;
+  v[3] = x.w;
+}
+__device__ __forceinline__ void lds4(const int32_t* p, int32_t (&v)[4]) {
+  const int4 x = *reinterpret_cast<const int4*>(p);
+  v[0] = x.x;
+  v[1] = x.y;
+  v[2] = x.z;
+  v[3] = x.w;
+}
+__device__ __forceinline__ void lds4(const int64_t* p, int64_t (&v)[4]) {
+  const longlong2 x = reinterpret_cast<const longlong2*>(p)[0];
+  const longlong2 y = reinterpret_cast<const longlong2*>(p)[1];
+  v[0] = x.x;
+  v[1] = x.y;
+  v[2] = y.x;
+  v[3] = y.y;
+}
+__device__ __forceinline__ void lds4(const uint64_t* p, uint64_t (&v)[4]) {
+  const ulonglong2 x = reinterpret_cast<const ulonglong2*>(p)[0];
+  const ulonglong2 y = reinterpret_cast<const ulonglong2*>(p)[1];
+  v[0] = x.x;
+  v[1] = x.y;
+  v[2] = y.x;
+  v[3] = y.y;
+}
+
+// One piece of a row: NV chunks of 128 instances starting at instance i_lo.
+template <int NV>
+struct Piece {
+  uint32_t h[NV][4];
+  uint32_t amask;  // bit 4 v + k: the pair is in A
+};
+
+// Loads a piece's hits and evaluates pass 1: the capacity guard and, for pairs in A, T_pf at the hit
+// and W = T_pf(n, c) - T_pf(0, L).  Returns the order-preserving bits of the lane's W_min over A (all ones if none).
+template <int NV, bool VEC>
+__device__ __forceinline__ uint32_t piece_pass1(const uint32_t* __restrict__ hrow, uint32_t I, uint32_t i_lo,
+                                                const ScoreSmem& s, const psk::DevModel& m, const psk::RowConst& rc,
+                                                Piece<NV>& p) {
+  const int lane = threadIdx.x & 31;
+#pragma unroll
+  for (int v = 0; v < NV; ++v) {
+    const uint32_t i = i_lo + 128u * v + 4u * lane;
+    if (VEC) {
+      uint4 x = make_uint4(0u, 0u, 0u, 0u);
+      if (i < I) x = __ldg(reinterpret_cast<const uint4*>(hrow + i));
+      p.h[v][0] = x.x;
+      p.h[v][1] = x.y;
+      p.h[v][2] = x.z;
+      p.h[v][3] = x.w;
+    } else {
+#pragma unroll
+      for (int k = 0; k < 4; ++k) p.h[v][k] = (i + k < I) ? __ldg(hrow + i + k) : 0u;
+    }
+  }
+  p.amask = 0u;
+  uint32_t wbest = 0xFFFFFFFFu;
+#pragma unroll
+  for (int v = 0; v < NV; ++v) {
+    const uint32_t i = i_lo + 128u * v + 4u * lane;
+    int32_t rm[4] = {-1, -1, -1, -1};
+    if (i < I) lds4(s.room + i, rm);  // padding past I holds -1
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      if ((int32_t)rc.L <= rm[k]) {
+        p.amask |= 1u << (4 * v + k);
+        wbest = min(wbest, psk::f2ord(__fsub_rn(psk::t_pf_of_hit(m, rc.L, p.h[v][k]), rc.t_cached)));
+      }
+    }
+  }
+  return wbest;
+}
+
+// Pass 2 of a piece: classes, optional per-pair outputs, and the lane's best (key, instance, hit).
+// T_pf is evaluated again (the same rounded operations) rather than held in registers.
+template <int NV, bool VEC>
+__device__ __forceinline__ void piece_pass2(uint32_t I, uint32_t i_lo, uint64_t x0, const ScoreSmem& s,
+                                            const psk::DevModel& m, const psk::RowConst& rc, float wmin,
+                                            const Piece<NV>& p, float* __restrict__ tpot_out,
+                                            float* __restrict__ ttft_out, uint8_t* __restrict__ cls_out,
+                                            uint64_t& bkey, uint32_t& binst, uint32_t& bh) {
+  const int lane = threadIdx.x & 31;
+  const bool all_pairs = tpot_out || ttft_out || cls_out;
+#pragma unroll
+  for (int v = 0; v < NV; ++v) {
+    const uint32_t i = i_lo + 128u * v + 4u * lane;
+    if (i >= I) continue;
+    const uint32_t am = (p.amask >> (4 * v)) & 0xFu;
+    bool inC[4];
+    float tpf[4];
+    bool anyC = false;
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      tpf[k] = (all_pairs || ((am >> k) & 1u)) ? psk::t_pf_of_hit(m, rc.L, p.h[v][k]) : 0.0f;
+      inC[k] = ((am >> k) & 1u) && psk::pair_in_c(rc, __fsub_rn(tpf[k], rc.t_cached), wmin);
+      anyC |= inC[k];
+    }
+    if (!anyC && !all_pairs) continue;
+    float dec0[4], fe[4], tq[4];
+    int32_t Bp[4];
+    int64_t q[4], S[4];
+    uint64_t k0[4];
+    lds4(s.dec0 + i, dec0);
+    lds4(s.f + i, fe);
+    lds4(s.tq + i, tq);
+    lds4(s.Bp + i, Bp);
+    lds4(s.q + i, q);
+    lds4(s.S + i, S);
+    lds4(s.k0 + i, k0);
+    float tp[4], tt[4];
+    uint32_t cw = 0u;
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      psk::InstTerms it;
+      it.dec0 = dec0[k];
+      it.f = fe[k];
+      it.tq = tq[k];
+      it.Bp = Bp[k];
+      it.okB = 1;
+      psk::PairW x;
+      x.tpf = tpf[k];
+      x.W = __fsub_rn(x.tpf, rc.t_cached);
+      x.n = (int64_t)rc.L - 16 * (int64_t)p.h[v][k];
+      x.inA = true;
+      uint32_t cls = 3u;
+      if (all_pairs || inC[k]) {
+        psk::pair_lat(m, rc, x, it, q[k], S[k], &tp[k], &tt[k]);
+        if ((am >> k) & 1u) cls = inC[k] ? (psk::pair_admitted(m, rc, tp[k], tt[k]) ? 0u : 1u) : 2u;
+      }
+      cw |= cls << (8 * k);
+      if (cls <= 1u) {
+        const uint64_t key =
+            cls == 0u ? psk::packed_key(0u, k0[k] | ((uint64_t)((1u << 26) - 1u - p.h[v][k]) << 18))
+                      : psk::packed_key(1u, ((uint64_t)q[k] + (uint64_t)x.n) * (uint64_t)(uint32_t)Bp[k]);
+        if (key < bkey) {  // a lane's instances ascend, so ties keep the lowest
+          bkey = key;
+          binst = i + k;
+          bh = p.h[v][k];
+        }
+      }
+    }
+    if (!all_pairs) continue;
+    const uint64_t x = x0 + i;
+    if (VEC) {
+      if (tpot_out) __stcs(reinterpret_cast<float4*>(tpot_out + x), make_float4(tp[0], tp[1], tp[2], tp[3]));
+      if (ttft_out) __stcs(reinterpret_cast<float4*>(ttft_out + x), make_float4(tt[0], tt[1], tt[2], tt[3]));
+      if (cls_out) __stcs(reinterpret_cast<uint32_t*>(cls_out + x), cw);
+    } else {
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        if (i + k >= I) break;
+        if (tpot_out) tpot_out[x + k] = tp[k];
+        if (ttft_out) ttft_out[x + k] = tt[k];
+        if (cls_out) cls_out[x + k] = (uint8_t)(cw >> (8 * k));
+      }
+    }
+  }
+}
+
+template <int NV, bool VEC>
+__global__ void __launch_bounds__(kScoreThreads, 2)
 score_rows_kernel(const uint32_t* __restrict__ hits, psk::StateSoA st, uint32_t I, psk::WindowDev w,
                   psk::DevModel m, float* __restrict__ tpot_out, float* __restrict__ ttft_out,
                   uint8_t* __restrict__ cls_out, int32_t* __restrict__ best_out,
                   uint8_t* __restrict__ path_out) {
-  const int lane = threadIdx.x & 31;
-  const uint32_t warps_total = (gridDim.x * blockDim.x) >> 5;
-  for (uint32_t r = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; r < w.R; r += warps_total) {
-    const psk::RowConst rc = psk::row_const(m, w.L[r], w.ttft_t[r], w.tpot_t[r]);
-    const uint32_t* hrow = hits + (uint64_t)r * I;
-    float wmin = INFINITY;
-    bool anyA = false;
-    for (uint32_t i = lane; i < I; i += 32) {
-      const psk::PairEval e = psk::eval_pair(m, rc, __ldg(hrow + i), __ldg(st.b + i), __ldg(st.qr + i),
-                                             __ldg(st.q + i), __ldg(st.S + i), __ldg(st.M + i),
-                                             __ldg(st.Bmax + i));
-      if (e.inA) {
-        wmin = fminf(wmin, e.W);
-        anyA = true;
-      }
-    }
-    anyA = __any_sync(0xffffffffu, anyA);
-    wmin = psk::warp_fmin(wmin);
-    psk::ArgKey best{psk::kNoKeyCi, ~0ull};
-    for (uint32_t i = lane; i < I; i += 32) {
-      const uint32_t h = __ldg(hrow + i);
-      const int32_t b = __ldg(st.b + i), qr = __ldg(st.qr + i);
-      const int64_t q = __ldg(st.q + i);
-      const psk::PairEval e = psk::eval_pair(m, rc, h, b, qr, q, __ldg(st.S + i), __ldg(st.M + i),
-                                             __ldg(st.Bmax + i));
-      const uint32_t cls = e.inA ? psk::pair_class(m, rc, e, wmin) : 3u;
-      const uint64_t x = (uint64_t)r * I + i;
-      if (tpot_out) tpot_out[x] = e.tpot;
-      if (ttft_out) ttft_out[x] = e.ttft;
-      if (cls_out) cls_out[x] = (uint8_t)cls;
-      if (cls <= 1u) {
-        const psk::ArgKey k{(cls << 28) | i, psk::pair_value(cls, h, b, qr, q, e.n)};
-        if (psk::key_less(k, best)) best = k;
-      }
-    }
-    best = psk::warp_argmin(best);
-    if (lane == 0) {
-      const bool pick = anyA && best.ci != psk::kNoKeyCi;
-      if (best_out) best_out[r] = pick ? (int32_t)(best.ci & 0x0FFFFFFFu) : -1;
-      if (path_out) path_out[r] = pick ? (uint8_t)(best.ci >> 28) : (uint8_t)2;
+  extern __shared__ __align__(16) unsigned long long smem_raw[];
+  const uint32_t Ip = (I + 3u) & ~3u;
+  const ScoreSmem s = score_smem(smem_raw, Ip);
+  for (uint32_t i = threadIdx.x; i < Ip; i += blockDim.x) {
+    if (i < I) {
+      const int32_t b = __ldg(st.b + i), qr = __ldg(st.qr + i), Bmax = __ldg(st.Bmax + i);
+      const int64_t q = __ldg(st.q + i), S = __ldg(st.S + i), M = __ldg(st.M + i);
+      const psk::InstTerms it = psk::inst_terms(m, b, qr, q, Bmax);
+      s.q[i] = q;
+      s.S[i] = S;
+      s.k0[i] = ((uint64_t)((1u << 18) - 1u - (uint32_t)b) << 44) | (uint64_t)(uint32_t)qr;
+      s.room[i] = it.okB ? psk::kv_room(S, M) : -1;
+      s.dec0[i] = it.dec0;
+      s.f[i] = it.f;
+      s.tq[i] = it.tq;
+      s.Bp[i] = it.Bp;
+    } else {
+      s.q[i] = 0;
+      s.S[i] = 0;
+      s.k0[i] = 0;
+      s.room[i] = -1;
+      s.dec0[i] = 0.0f;
+      s.f[i] = 0.0f;
+      s.tq[i] = 0.0f;
+      s.Bp[i] = 1;
     }
   }
+  __syncthreads();
+  const int lane = threadIdx.x & 31;
+  const uint32_t warps_total = (gridDim.x * blockDim.x) >> 5;
+  constexpr uint32_t kPiece = 128u * NV;
+  const bool one_piece = I <= kPiece;
+  for (uint32_t r = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; r < w.R; r += warps_total) {
+    const psk::RowConst rc = psk::row_const(m, __ldg(w.L + r), __ldg(w.ttft_t + r), __ldg(w.tpot_t + r));
+    const uint64_t x0 = (uint64_t)r * I;
+    const uint32_t* hrow = hits + x0;
+    Piece<NV> p;
+    uint32_t wbest = piece_pass1<NV, VEC>(hrow, I, 0u, s, m, rc, p);
+    for (uint32_t lo = kPiece; lo < I; lo += kPiece) {
+      Piece<NV> p2;
+      wbest = min(wbest, piece_pass1<NV, VEC>(hrow, I, lo, s, m, rc, p2));
+    }
+    wbest = __reduce_min_sync(0xffffffffu, wbest);
+    const bool anyA = wbest != 0xFFFFFFFFu;  // a W of a pair in A is never NaN, so never all ones
+    const float wmin = psk::ord2f(wbest);
+    uint64_t bkey = psk::kNoKey;
+    uint32_t binst = 0xFFFFFFFFu, bh = 0u;
+    if (one_piece) {
+      piece_pass2<NV, VEC>(I, 0u, x0, s, m, rc, wmin, p, tpot_out, ttft_out, cls_out, bkey, binst, bh);
+    } else {
+      for (uint32_t lo = 0; lo < I; lo += kPiece) {
+        piece_pass1<NV, VEC>(hrow, I, lo, s, m, rc, p);
+        piece_pass2<NV, VEC>(I, lo, x0, s, m, rc, wmin, p, tpot_out, ttft_out, cls_out, bkey, binst, bh);
+      }
+    }
+    uint64_t key;
+    uint32_t j, hj;
+    psk::warp_pick_min(bkey, binst, bh, &key, &j, &hj);
+    if (lane == 0) {
+      const bool pick = anyA && key != psk::kNoKey;
+      if (best_out) best_out[r] = pick ? (int32_t)j : -1;
+      if (path_out) path_out[r] = pick ? (uint8_t)(key >> 62) : (uint8_t)2;
+    }
+  }
+}
+
+template <int NV>
+cudaError_t score_launch(const uint32_t* hits, psk::StateSoA st, uint32_t I, const psk::WindowDev& w,
+                         const psk::DevModel& m, float* tpot, float* ttft, uint8_t* cls, int32_t* best,
+                         uint8_t* path, int num_sms, cudaStream_t s) {
+  const uint32_t Ip = (I + 3u) & ~3u;
+  const size_t smem = (size_t)Ip * (3 * sizeof(int64_t) + 5 * sizeof(uint32_t));
+  // 16-byte loads of hit rows and stores of TPOT / TTFT rows, 4-byte stores of class rows
+  const bool vec = (I & 3u) == 0u && (reinterpret_cast<uintptr_t>(hits) & 15u) == 0u &&
+                   (reinterpret_cast<uintptr_t>(tpot) & 15u) == 0u && (reinterpret_cast<uintptr_t>(ttft) & 15u) == 0u &&
+                   (reinterpret_cast<uintptr_t>(cls) & 3u) == 0u;
+  auto kern = vec ? score_rows_kernel<NV, true> : score_rows_kernel<NV, false>;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
+  const uint32_t rows_per_block = kScoreThreads / 32;
+  uint32_t grid = (w.R + rows_per_block - 1) / rows_per_block;
+  const uint32_t cap = (uint32_t)num_sms * 2u;
+  if (grid > cap) grid = cap;
+  kern<<<grid, kScoreThreads, smem, s>>>(hits, st, I, w, m, tpot, ttft, cls, best, path);
+  return cudaGetLastError();
 }
 
 }  // namespace
@@ -67,12 +309,10 @@ cudaError_t launch_score(const uint32_t* hits, psk::StateSoA st, uint32_t I, con
                          const psk::DevModel& m, float* tpot, float* ttft, uint8_t* cls, int32_t* best,
                          uint8_t* path, int num_sms, cudaStream_t s) {
   if (w.R == 0) return cudaSuccess;
-  const uint32_t rows_per_block = 8;
-  uint32_t grid = (w.R + rows_per_block - 1) / rows_per_block;
-  const uint32_t cap = (uint32_t)num_sms * 8u;
-  if (grid > cap) grid = cap;
-  score_rows_kernel<<<grid, 256, 0, s>>>(hits, st, I, w, m, tpot, ttft, cls, best, path);
-  return cudaGetLastError();
+  if (I <= 128u) return score_launch<1>(hits, st, I, w, m, tpot, ttft, cls, best, path, num_sms, s);
+  if (I <= 256u) return score_launch<2>(hits, st, I, w, m, tpot, ttft, cls, best, path, num_sms, s);
+  if (I <= 512u) return score_launch<4>(hits, st, I, w, m, tpot, ttft, cls, best, path, num_sms, s);
+  return score_launch<8>(hits, st, I, w, m, tpot, ttft, cls, best, path, num_sms, s);
 }
 
 }  // namespace pskl
