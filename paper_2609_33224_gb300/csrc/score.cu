@@ -19,6 +19,8 @@ namespace {
 constexpr int kScoreThreads = 256;
 
 // Shared-memory instance arrays, each [Ip] (I rounded up to a multiple of 4), 8-byte arrays first.
+// q32 / S32 are 32-bit copies of q / S, used when every instance of the block has both in
+// [0, 2^30): then S + L and q + n (L, n < 2^30) are exact in 32 bits.
 struct ScoreSmem {
   int64_t* q;
   int64_t* S;
@@ -28,6 +30,8 @@ struct ScoreSmem {
   float* f;
   float* tq;
   int32_t* Bp;
+  int32_t* q32;
+  int32_t* S32;
 };
 
 __device__ __forceinline__ ScoreSmem score_smem(unsigned long long* raw, uint32_t Ip) {
@@ -40,6 +44,8 @@ __device__ __forceinline__ ScoreSmem score_smem(unsigned long long* raw, uint32_
   s.f = s.dec0 + Ip;
   s.tq = s.f + Ip;
   s.Bp = reinterpret_cast<int32_t*>(s.tq + Ip);
+  s.q32 = s.Bp + Ip;
+  s.S32 = s.q32 + Ip;
   return s;
 }
 
@@ -73,6 +79,28 @@ __device__ __forceinline__ void lds4(const uint64_t* p, uint64_t (&v)[4]) {
   v[1] = x.y;
   v[2] = y.x;
   v[3] = y.y;
+}
+
+// T_pf at hit h of a request of L tokens, in 32-bit integers: c = 16 h and n = L - c are below 2^30
+// in magnitude (L < 2^30, h <= L / 16), so their conversions equal the 64-bit ones.
+__device__ __forceinline__ float t_pf32(const psk::DevModel& m, uint32_t L, uint32_t h) {
+  const int32_t c = (int32_t)(h << 4);
+  return psk::t_pf(m, __int2float_rn((int32_t)L - c), __int2float_rn(c));
+}
+
+// TPOT and TTFT of a pair (pair_lat's rounded operations) with S + L and q + n formed in 32 bits.
+__device__ __forceinline__ void pair_lat32(const psk::DevModel& m, const psk::RowConst& rc, float tpf, int32_t n,
+                                           float dec0, float f, float tq, int32_t Bp, int32_t q32, int32_t S32,
+                                           float* tpot, float* ttft) {
+  float dec = __fadd_rn(dec0, __fmul_rn(m.b2, __int2float_rn(S32 + (int32_t)rc.L)));
+  dec = __fmul_rn(dec, f);
+  if (m.interference_mode == 0) {
+    *tpot = __fadd_rn(dec, __fmul_rn(m.g_q, __int2float_rn(q32 + n)));
+  } else {
+    const float den = m.lout > 1.0f ? m.lout : 1.0f;
+    *tpot = __fadd_rn(dec, Bp > 1 ? __fdiv_rn(tpf, den) : 0.0f);
+  }
+  *ttft = __fadd_rn(tpf, tq);
 }
 
 // One piece of a row: NV chunks of 128 instances starting at instance i_lo.
@@ -115,7 +143,7 @@ __device__ __forceinline__ uint32_t piece_pass1(const uint32_t* __restrict__ hro
     for (int k = 0; k < 4; ++k) {
       if ((int32_t)rc.L <= rm[k]) {
         p.amask |= 1u << (4 * v + k);
-        wbest = min(wbest, psk::f2ord(__fsub_rn(psk::t_pf_of_hit(m, rc.L, p.h[v][k]), rc.t_cached)));
+        wbest = min(wbest, psk::f2ord(__fsub_rn(t_pf32(m, rc.L, p.h[v][k]), rc.t_cached)));
       }
     }
   }
@@ -124,7 +152,7 @@ __device__ __forceinline__ uint32_t piece_pass1(const uint32_t* __restrict__ hro
 
 // Pass 2 of a piece: classes, optional per-pair outputs, and the lane's best (key, instance, hit).
 // T_pf is evaluated again (the same rounded operations) rather than held in registers.
-template <int NV, bool VEC>
+template <int NV, bool VEC, bool NARROW>
 __device__ __forceinline__ void piece_pass2(uint32_t I, uint32_t i_lo, uint64_t x0, const ScoreSmem& s,
                                             const psk::DevModel& m, const psk::RowConst& rc, float wmin,
                                             const Piece<NV>& p, float* __restrict__ tpot_out,
@@ -142,47 +170,58 @@ __device__ __forceinline__ void piece_pass2(uint32_t I, uint32_t i_lo, uint64_t 
     bool anyC = false;
 #pragma unroll
     for (int k = 0; k < 4; ++k) {
-      tpf[k] = (all_pairs || ((am >> k) & 1u)) ? psk::t_pf_of_hit(m, rc.L, p.h[v][k]) : 0.0f;
+      tpf[k] = (all_pairs || ((am >> k) & 1u)) ? t_pf32(m, rc.L, p.h[v][k]) : 0.0f;
       inC[k] = ((am >> k) & 1u) && psk::pair_in_c(rc, __fsub_rn(tpf[k], rc.t_cached), wmin);
       anyC |= inC[k];
     }
     if (!anyC && !all_pairs) continue;
     float dec0[4], fe[4], tq[4];
     int32_t Bp[4];
-    int64_t q[4], S[4];
     uint64_t k0[4];
     lds4(s.dec0 + i, dec0);
     lds4(s.f + i, fe);
     lds4(s.tq + i, tq);
     lds4(s.Bp + i, Bp);
-    lds4(s.q + i, q);
-    lds4(s.S + i, S);
     lds4(s.k0 + i, k0);
+    int32_t q32[4], S32[4];
+    int64_t q[4], S[4];
+    if (NARROW) {
+      lds4(s.q32 + i, q32);
+      lds4(s.S32 + i, S32);
+    } else {
+      lds4(s.q + i, q);
+      lds4(s.S + i, S);
+    }
     float tp[4], tt[4];
     uint32_t cw = 0u;
 #pragma unroll
     for (int k = 0; k < 4; ++k) {
-      psk::InstTerms it;
-      it.dec0 = dec0[k];
-      it.f = fe[k];
-      it.tq = tq[k];
-      it.Bp = Bp[k];
-      it.okB = 1;
-      psk::PairW x;
-      x.tpf = tpf[k];
-      x.W = __fsub_rn(x.tpf, rc.t_cached);
-      x.n = (int64_t)rc.L - 16 * (int64_t)p.h[v][k];
-      x.inA = true;
+      const int32_t n = (int32_t)rc.L - (int32_t)(p.h[v][k] << 4);
       uint32_t cls = 3u;
       if (all_pairs || inC[k]) {
-        psk::pair_lat(m, rc, x, it, q[k], S[k], &tp[k], &tt[k]);
+        if (NARROW) {
+          pair_lat32(m, rc, tpf[k], n, dec0[k], fe[k], tq[k], Bp[k], q32[k], S32[k], &tp[k], &tt[k]);
+        } else {
+          psk::InstTerms it;
+          it.dec0 = dec0[k];
+          it.f = fe[k];
+          it.tq = tq[k];
+          it.Bp = Bp[k];
+          it.okB = 1;
+          psk::PairW x;
+          x.tpf = tpf[k];
+          x.W = __fsub_rn(x.tpf, rc.t_cached);
+          x.n = n;
+          x.inA = true;
+          psk::pair_lat(m, rc, x, it, q[k], S[k], &tp[k], &tt[k]);
+        }
         if ((am >> k) & 1u) cls = inC[k] ? (psk::pair_admitted(m, rc, tp[k], tt[k]) ? 0u : 1u) : 2u;
       }
       cw |= cls << (8 * k);
       if (cls <= 1u) {
-        const uint64_t key =
-            cls == 0u ? psk::packed_key(0u, k0[k] | ((uint64_t)((1u << 26) - 1u - p.h[v][k]) << 18))
-                      : psk::packed_key(1u, ((uint64_t)q[k] + (uint64_t)x.n) * (uint64_t)(uint32_t)Bp[k]);
+        const uint64_t qn = NARROW ? (uint64_t)(uint32_t)(q32[k] + n) : (uint64_t)q[k] + (uint64_t)(int64_t)n;
+        const uint64_t key = cls == 0u ? psk::packed_key(0u, k0[k] | ((uint64_t)((1u << 26) - 1u - p.h[v][k]) << 18))
+                                       : psk::packed_key(1u, qn * (uint64_t)(uint32_t)Bp[k]);
         if (key < bkey) {  // a lane's instances ascend, so ties keep the lowest
           bkey = key;
           binst = i + k;
@@ -217,6 +256,7 @@ score_rows_kernel(const uint32_t* __restrict__ hits, psk::StateSoA st, uint32_t 
   extern __shared__ __align__(16) unsigned long long smem_raw[];
   const uint32_t Ip = (I + 3u) & ~3u;
   const ScoreSmem s = score_smem(smem_raw, Ip);
+  bool wide = false;  // some instance's q or S is outside [0, 2^30)
   for (uint32_t i = threadIdx.x; i < Ip; i += blockDim.x) {
     if (i < I) {
       const int32_t b = __ldg(st.b + i), qr = __ldg(st.qr + i), Bmax = __ldg(st.Bmax + i);
@@ -230,6 +270,9 @@ score_rows_kernel(const uint32_t* __restrict__ hits, psk::StateSoA st, uint32_t 
       s.f[i] = it.f;
       s.tq[i] = it.tq;
       s.Bp[i] = it.Bp;
+      wide |= !(q >= 0 && q < (1ll << 30) && S >= 0 && S < (1ll << 30));
+      s.q32[i] = (int32_t)q;
+      s.S32[i] = (int32_t)S;
     } else {
       s.q[i] = 0;
       s.S[i] = 0;
@@ -239,9 +282,11 @@ score_rows_kernel(const uint32_t* __restrict__ hits, psk::StateSoA st, uint32_t 
       s.f[i] = 0.0f;
       s.tq[i] = 0.0f;
       s.Bp[i] = 1;
+      s.q32[i] = 0;
+      s.S32[i] = 0;
     }
   }
-  __syncthreads();
+  const bool narrow = __syncthreads_or(wide ? 1 : 0) == 0;
   const int lane = threadIdx.x & 31;
   const uint32_t warps_total = (gridDim.x * blockDim.x) >> 5;
   constexpr uint32_t kPiece = 128u * NV;
@@ -262,11 +307,17 @@ score_rows_kernel(const uint32_t* __restrict__ hits, psk::StateSoA st, uint32_t 
     uint64_t bkey = psk::kNoKey;
     uint32_t binst = 0xFFFFFFFFu, bh = 0u;
     if (one_piece) {
-      piece_pass2<NV, VEC>(I, 0u, x0, s, m, rc, wmin, p, tpot_out, ttft_out, cls_out, bkey, binst, bh);
+      if (narrow)
+        piece_pass2<NV, VEC, true>(I, 0u, x0, s, m, rc, wmin, p, tpot_out, ttft_out, cls_out, bkey, binst, bh);
+      else
+        piece_pass2<NV, VEC, false>(I, 0u, x0, s, m, rc, wmin, p, tpot_out, ttft_out, cls_out, bkey, binst, bh);
     } else {
       for (uint32_t lo = 0; lo < I; lo += kPiece) {
         piece_pass1<NV, VEC>(hrow, I, lo, s, m, rc, p);
-        piece_pass2<NV, VEC>(I, lo, x0, s, m, rc, wmin, p, tpot_out, ttft_out, cls_out, bkey, binst, bh);
+        if (narrow)
+          piece_pass2<NV, VEC, true>(I, lo, x0, s, m, rc, wmin, p, tpot_out, ttft_out, cls_out, bkey, binst, bh);
+        else
+          piece_pass2<NV, VEC, false>(I, lo, x0, s, m, rc, wmin, p, tpot_out, ttft_out, cls_out, bkey, binst, bh);
       }
     }
     uint64_t key;
@@ -285,7 +336,7 @@ cudaError_t score_launch(const uint32_t* hits, psk::StateSoA st, uint32_t I, con
                          const psk::DevModel& m, float* tpot, float* ttft, uint8_t* cls, int32_t* best,
                          uint8_t* path, int num_sms, cudaStream_t s) {
   const uint32_t Ip = (I + 3u) & ~3u;
-  const size_t smem = (size_t)Ip * (3 * sizeof(int64_t) + 5 * sizeof(uint32_t));
+  const size_t smem = (size_t)Ip * (3 * sizeof(int64_t) + 7 * sizeof(uint32_t));
   // 16-byte loads of hit rows and stores of TPOT / TTFT rows, 4-byte stores of class rows
   const bool vec = (I & 3u) == 0u && (reinterpret_cast<uintptr_t>(hits) & 15u) == 0u &&
                    (reinterpret_cast<uintptr_t>(tpot) & 15u) == 0u && (reinterpret_cast<uintptr_t>(ttft) & 15u) == 0u &&
@@ -311,8 +362,7 @@ cudaError_t launch_score(const uint32_t* hits, psk::StateSoA st, uint32_t I, con
   if (w.R == 0) return cudaSuccess;
   if (I <= 128u) return score_launch<1>(hits, st, I, w, m, tpot, ttft, cls, best, path, num_sms, s);
   if (I <= 256u) return score_launch<2>(hits, st, I, w, m, tpot, ttft, cls, best, path, num_sms, s);
-  if (I <= 512u) return score_launch<4>(hits, st, I, w, m, tpot, ttft, cls, best, path, num_sms, s);
-  return score_launch<8>(hits, st, I, w, m, tpot, ttft, cls, best, path, num_sms, s);
+  return score_launch<4>(hits, st, I, w, m, tpot, ttft, cls, best, path, num_sms, s);
 }
 
 }  // namespace pskl
