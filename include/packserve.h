@@ -108,7 +108,7 @@ typedef struct {
  *                          PS_ERR_INVALID.
  *   track_lru             1: keep per-block (last_use, child count, parent) metadata so that
  *                         ps_advance_window can evict leaf-first LRU (the tables must then hold fewer
- *                         than 2^32 slots in total); 0: no eviction.
+ *                         than 2^32 - 2 slots in total); 0: no eviction.
  *   max_active_requests   0: no request tracking.  > 0: each instance keeps up to this many queued
  *                         and this many decoding requests for ps_advance_window (streaming windows);
  *                         committed windows then need ps_window.out_tokens. */

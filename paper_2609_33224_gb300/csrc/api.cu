@@ -90,6 +90,7 @@ struct ps_ctx {
   bool lru = false;
   psk::LruMeta meta{nullptr, nullptr, nullptr};
   void* d_leafbuf = nullptr;
+  unsigned long long* d_cprefix = nullptr;  // [2 (Rmax + 1)] commit item prefixes
   uint32_t* d_nleaf = nullptr;
   uint32_t* d_more = nullptr;
   uint64_t max_instance_slots = 0;
@@ -374,8 +375,8 @@ ps_status ps_create(const ps_config* cfg, ps_ctx** out) {
     obase += (nbkt + 63) / 64;
   }
   c->total_slots = base;
-  if (c->lru && c->total_slots >= (1ull << 32)) {
-    c->err = "track_lru needs fewer than 2^32 table slots in total (eviction keeps 32-bit slot indices)";
+  if (c->lru && c->total_slots >= (1ull << 32) - 2) {
+    c->err = "track_lru needs fewer than 2^32 - 2 table slots in total (eviction keeps 32-bit slot indices)";
     return bail(PS_ERR_INVALID);
   }
   c->total_ovf = obase;
@@ -393,7 +394,8 @@ ps_status ps_create(const ps_config* cfg, ps_ctx** out) {
             dalloc(c, &c->gsync.hitring, (size_t)psk::kHitSlots * c->gsync.ring_stride) == cudaSuccess &&
             dalloc(c, &c->gsync.tpfring, (size_t)psk::kHitSlots * c->gsync.ring_stride) == cudaSuccess &&
             dalloc(c, &c->d_rows, c->Rmax) == cudaSuccess && dalloc(c, &c->d_lastslot, c->lastslot_n) == cudaSuccess &&
-            dalloc(c, &c->scratch.rows, c->Rmax) == cudaSuccess && dalloc(c, &c->scratch.count, 1) == cudaSuccess;
+            dalloc(c, &c->scratch.rows, c->Rmax) == cudaSuccess && dalloc(c, &c->scratch.count, 1) == cudaSuccess &&
+            dalloc(c, &c->d_cprefix, 2 * ((size_t)c->Rmax + 1)) == cudaSuccess;
   for (psk::StateSoA* s : {&c->st, &c->pend}) {
     ok = ok && dalloc(c, &s->b, I) == cudaSuccess && dalloc(c, &s->qr, I) == cudaSuccess &&
          dalloc(c, &s->q, I) == cudaSuccess && dalloc(c, &s->S, I) == cudaSuccess &&
@@ -681,8 +683,8 @@ ps_status ps_commit_window(ps_ctx* c, uint32_t last_use) {
   DeviceGuard g(c->device);
   record(c, kEvCommit0);
   PS_TRY_CUDA(c, pskl::launch_commit(c->d_slots, c->d_ovf, c->d_tdesc, c->I, c->d_count, c->pend_win, c->d_assign,
-                                     c->d_hchosen, c->meta, last_use, c->rq, c->pend_out, c->d_err, c->num_sms,
-                                     c->stream));
+                                     c->d_hchosen, c->meta, last_use, c->rq, c->pend_out, c->d_cprefix, c->d_err,
+                                     c->num_sms, c->stream));
   const size_t I = c->I;
   PS_TRY_CUDA(c, cudaMemcpyAsync(c->st.b, c->pend.b, I * 4, cudaMemcpyDeviceToDevice, c->stream));
   PS_TRY_CUDA(c, cudaMemcpyAsync(c->st.qr, c->pend.qr, I * 4, cudaMemcpyDeviceToDevice, c->stream));

@@ -696,6 +696,7 @@ struct PairEval {
 };
 
 __device__ __forceinline__ float ema_factor(const DevModel& m, int64_t B) {
+  if (m.nseg == 1) return m.ema[0];
   int s = 0;
   for (int k = 0; k < m.nseg; ++k)
     if ((int64_t)m.seg_lo[k] <= B) s = k;
@@ -763,6 +764,29 @@ __device__ __forceinline__ InstTerms inst_terms(const DevModel& m, int32_t b, in
 __device__ __forceinline__ float t_pf_of_hit(const DevModel& m, uint32_t L, uint32_t h) {
   const int64_t c = 16 * (int64_t)h;
   return t_pf(m, i64_to_f32((int64_t)L - c), i64_to_f32(c));
+}
+
+// T_pf at hit h of a request of L tokens, in 32-bit integers: c = 16 h and n = L - c are below 2^30
+// in magnitude (L < 2^30, h <= L / 16), so their conversions equal the 64-bit ones.
+__device__ __forceinline__ float t_pf32(const DevModel& m, uint32_t L, uint32_t h) {
+  const int32_t c = (int32_t)(h << 4);
+  return t_pf(m, __int2float_rn((int32_t)L - c), __int2float_rn(c));
+}
+
+// TPOT and TTFT of a pair (pair_lat's rounded operations) with S + L and q + n formed in 32 bits, for
+// instances whose q and S lie in [0, 2^30) (n = L - 16 h, L < 2^30).
+__device__ __forceinline__ void pair_lat32(const DevModel& m, const RowConst& rc, float tpf, int32_t n, float dec0,
+                                           float f, float tq, int32_t Bp, int32_t q32, int32_t S32, float* tpot,
+                                           float* ttft) {
+  float dec = __fadd_rn(dec0, __fmul_rn(m.b2, __int2float_rn(S32 + (int32_t)rc.L)));
+  dec = __fmul_rn(dec, f);
+  if (m.interference_mode == 0) {
+    *tpot = __fadd_rn(dec, __fmul_rn(m.g_q, __int2float_rn(q32 + n)));
+  } else {
+    const float den = m.lout > 1.0f ? m.lout : 1.0f;
+    *tpot = __fadd_rn(dec, Bp > 1 ? __fdiv_rn(tpf, den) : 0.0f);
+  }
+  *ttft = __fadd_rn(tpf, tq);
 }
 
 // Marks a precomputed T_pf as not available (a NaN pattern T_pf never produces).
@@ -950,11 +974,12 @@ cudaError_t launch_insert_chains(uint64_t* slots, uint64_t* ovf, const psk::Tabl
                                  const uint64_t* off, const uint64_t* hash, const uint64_t* parent,
                                  uint64_t total, psk::LruMeta meta, uint32_t last_use, uint32_t* err,
                                  int num_sms, cudaStream_t s);
+// prefix: device scratch of 2 (R + 1) words.
 cudaError_t launch_commit(uint64_t* slots, uint64_t* ovf, const psk::TableDesc* tdesc, uint32_t I,
                           unsigned long long* count, const psk::WindowDev& w, const int32_t* assign,
                           const uint32_t* hit_chosen, psk::LruMeta meta, uint32_t last_use,
-                          const psk::ReqStore& rq, const uint32_t* out_tokens, uint32_t* err, int num_sms,
-                          cudaStream_t s);
+                          const psk::ReqStore& rq, const uint32_t* out_tokens, unsigned long long* prefix,
+                          uint32_t* err, int num_sms, cudaStream_t s);
 cudaError_t launch_advance(psk::StateSoA st, uint32_t I, const psk::ReqStore& rq, const psk::DevModel& m,
                            float window_ms, uint64_t prefill_tokens, uint32_t* err, cudaStream_t s);
 // Leaf-first LRU eviction of every instance over capacity (rounds until none is; synchronises the

@@ -81,27 +81,8 @@ __device__ __forceinline__ void lds4(const uint64_t* p, uint64_t (&v)[4]) {
   v[3] = y.y;
 }
 
-// T_pf at hit h of a request of L tokens, in 32-bit integers: c = 16 h and n = L - c are below 2^30
-// in magnitude (L < 2^30, h <= L / 16), so their conversions equal the 64-bit ones.
-__device__ __forceinline__ float t_pf32(const psk::DevModel& m, uint32_t L, uint32_t h) {
-  const int32_t c = (int32_t)(h << 4);
-  return psk::t_pf(m, __int2float_rn((int32_t)L - c), __int2float_rn(c));
-}
-
-// TPOT and TTFT of a pair (pair_lat's rounded operations) with S + L and q + n formed in 32 bits.
-__device__ __forceinline__ void pair_lat32(const psk::DevModel& m, const psk::RowConst& rc, float tpf, int32_t n,
-                                           float dec0, float f, float tq, int32_t Bp, int32_t q32, int32_t S32,
-                                           float* tpot, float* ttft) {
-  float dec = __fadd_rn(dec0, __fmul_rn(m.b2, __int2float_rn(S32 + (int32_t)rc.L)));
-  dec = __fmul_rn(dec, f);
-  if (m.interference_mode == 0) {
-    *tpot = __fadd_rn(dec, __fmul_rn(m.g_q, __int2float_rn(q32 + n)));
-  } else {
-    const float den = m.lout > 1.0f ? m.lout : 1.0f;
-    *tpot = __fadd_rn(dec, Bp > 1 ? __fdiv_rn(tpf, den) : 0.0f);
-  }
-  *ttft = __fadd_rn(tpf, tq);
-}
+using psk::pair_lat32;
+using psk::t_pf32;
 
 // One piece of a row: NV chunks of 128 instances starting at instance i_lo.
 template <int NV>

@@ -60,10 +60,10 @@ __global__ void check_instances_kernel(uint32_t I, uint64_t nchains, const uint3
     if (inst[c] >= I) atomicOr(err, psk::kErrBadInstance);
 }
 
-// Commit of a scheduled window, in four passes so that every admitted request's blocks are handled
-// in parallel (within a window each (block, instance) pair is inserted at most once: a request
-// inserts chain[h, nb) on its pick with h the exact first miss there, so none of those blocks is
-// cached on that instance yet, neither by the committed caches nor by an earlier request):
+// Commit of a scheduled window, in four passes over every admitted request's blocks (within a window
+// each (block, instance) pair is inserted at most once: a request inserts chain[h, nb) on its pick
+// with h the exact first miss there, so none of those blocks is cached on that instance yet, neither
+// by the committed caches nor by an earlier request):
 //   stamp   the cached prefix chain[0, h) gets last_use (every stamp writes the same value, so
 //           their order does not matter);
 //   insert  the uncached blocks chain[h, nb) are cached, stamped, with 0 children and their parent
@@ -71,89 +71,157 @@ __global__ void check_instances_kernel(uint32_t I, uint64_t nchains, const uint3
 //   link    each new block records its parent's slot and the parent gains a child;
 //   queue   with request tracking, each instance appends its admitted requests to its FIFO queue
 //           in arrival order (one warp per instance).
-// One warp per request for the first three, lanes over the request's blocks.
+// The first three run over one flat index space of (request, block) items, so a long chain is
+// spread over the whole grid: a prefix pass gives each admitted request its first item, and an item
+// finds its request by binary search.
+
+// Exclusive prefix sums over the window's requests of the items of the stamp pass (h) and of the
+// insert and link passes (nb - h); rejected requests have none.  One block; pre_s and pre_i hold
+// R + 1 entries each.
+__global__ void __launch_bounds__(1024)
+commit_prefix_kernel(psk::WindowDev w, const int32_t* __restrict__ assign, const uint32_t* __restrict__ hit_chosen,
+                     unsigned long long* pre_s, unsigned long long* pre_i) {
+  __shared__ unsigned long long s_ws[32], s_wi[32];
+  __shared__ unsigned long long s_carry_s, s_carry_i;
+  const uint32_t t = threadIdx.x, lane = t & 31u, warp = t >> 5;
+  if (t == 0) {
+    s_carry_s = 0ull;
+    s_carry_i = 0ull;
+  }
+  __syncthreads();
+  for (uint32_t r0 = 0; r0 < w.R; r0 += blockDim.x) {
+    const uint32_t r = r0 + t;
+    unsigned long long cs = 0ull, ci = 0ull;
+    if (r < w.R && assign[r] >= 0) {
+      const uint64_t h = hit_chosen[r];
+      const uint64_t nb = w.off[r + 1] - w.off[r];
+      cs = h;
+      ci = nb > h ? nb - h : 0ull;
+    }
+    unsigned long long xs = cs, xi = ci;  // inclusive warp scans
+#pragma unroll
+    for (int d = 1; d < 32; d <<= 1) {
+      const unsigned long long ys = __shfl_up_sync(0xffffffffu, xs, d), yi = __shfl_up_sync(0xffffffffu, xi, d);
+      if ((int)lane >= d) {
+        xs += ys;
+        xi += yi;
+      }
+    }
+    if (lane == 31u) {
+      s_ws[warp] = xs;
+      s_wi[warp] = xi;
+    }
+    __syncthreads();
+    if (warp == 0) {
+      const uint32_t nw = blockDim.x >> 5;
+      unsigned long long vs = lane < nw ? s_ws[lane] : 0ull, vi = lane < nw ? s_wi[lane] : 0ull;
+#pragma unroll
+      for (int d = 1; d < 32; d <<= 1) {
+        const unsigned long long ys = __shfl_up_sync(0xffffffffu, vs, d), yi = __shfl_up_sync(0xffffffffu, vi, d);
+        if ((int)lane >= d) {
+          vs += ys;
+          vi += yi;
+        }
+      }
+      // exclusive warp offsets from the inclusive ones
+      const unsigned long long es = __shfl_up_sync(0xffffffffu, vs, 1), ei = __shfl_up_sync(0xffffffffu, vi, 1);
+      if (lane < nw) {
+        s_ws[lane] = lane == 0 ? 0ull : es;
+        s_wi[lane] = lane == 0 ? 0ull : ei;
+      }
+    }
+    __syncthreads();
+    if (r < w.R) {
+      pre_s[r] = s_carry_s + s_ws[warp] + xs - cs;
+      pre_i[r] = s_carry_i + s_wi[warp] + xi - ci;
+    }
+    __syncthreads();
+    if (t == blockDim.x - 1u) {  // the chunk's total carries into the next chunk
+      s_carry_s += s_ws[warp] + xs;
+      s_carry_i += s_wi[warp] + xi;
+    }
+    __syncthreads();
+  }
+  if (t == 0) {
+    pre_s[w.R] = s_carry_s;
+    pre_i[w.R] = s_carry_i;
+  }
+}
+
+// The request of flat item x: the last r with pre[r] <= x (pre ascending, pre[0] = 0, x < pre[R]).
+__device__ __forceinline__ uint32_t item_request(const unsigned long long* __restrict__ pre, uint32_t R,
+                                                 unsigned long long x) {
+  uint32_t lo = 0, hi = R;  // pre[lo] <= x < pre[hi]
+  while (hi - lo > 1u) {
+    const uint32_t mid = (lo + hi) >> 1;
+    if (__ldg(pre + mid) <= x) lo = mid;
+    else hi = mid;
+  }
+  return lo;
+}
+
 __global__ void commit_stamp_kernel(const uint64_t* slots, const uint64_t* ovf, const psk::TableDesc* __restrict__ tdesc,
                                     psk::WindowDev w, const int32_t* __restrict__ assign,
-                                    const uint32_t* __restrict__ hit_chosen, psk::LruMeta meta, uint32_t last_use) {
-  const int lane = threadIdx.x & 31;
-  const uint32_t warps_total = (gridDim.x * blockDim.x) >> 5;
-  for (uint32_t r = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; r < w.R; r += warps_total) {
-    const int32_t j = assign[r];
-    if (j < 0) continue;
-    const psk::TableDesc d = tdesc[j];
-    const uint64_t o = w.off[r];
-    const uint64_t h = hit_chosen[r];
-    for (uint64_t k = lane; k < h; k += 32) {
-      const uint64_t s = psk::main_find(slots, ovf, d, w.hash[o + k]);
-      if (s != ~0ull && meta.last_use[s] < last_use) meta.last_use[s] = last_use;
-    }
+                                    const unsigned long long* __restrict__ pre_s, psk::LruMeta meta, uint32_t last_use) {
+  const unsigned long long total = pre_s[w.R];
+  for (unsigned long long x = blockIdx.x * (unsigned long long)blockDim.x + threadIdx.x; x < total;
+       x += (unsigned long long)gridDim.x * blockDim.x) {
+    const uint32_t r = item_request(pre_s, w.R, x);
+    const uint64_t k = x - pre_s[r];
+    const uint64_t s = psk::main_find(slots, ovf, tdesc[assign[r]], w.hash[w.off[r] + k]);
+    if (s != ~0ull && meta.last_use[s] < last_use) meta.last_use[s] = last_use;
   }
 }
 
 __global__ void commit_insert_kernel(uint64_t* slots, uint64_t* ovf, const psk::TableDesc* __restrict__ tdesc,
                                      unsigned long long* count, psk::WindowDev w, const int32_t* __restrict__ assign,
-                                     const uint32_t* __restrict__ hit_chosen, psk::LruMeta meta, uint32_t last_use,
-                                     uint32_t* err) {
-  const int lane = threadIdx.x & 31;
-  const uint32_t warps_total = (gridDim.x * blockDim.x) >> 5;
-  for (uint32_t r = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; r < w.R; r += warps_total) {
+                                     const uint32_t* __restrict__ hit_chosen, const unsigned long long* __restrict__ pre_i,
+                                     psk::LruMeta meta, uint32_t last_use, uint32_t* err) {
+  const unsigned long long total = pre_i[w.R];
+  for (unsigned long long x = blockIdx.x * (unsigned long long)blockDim.x + threadIdx.x; x < total;
+       x += (unsigned long long)gridDim.x * blockDim.x) {
+    const uint32_t r = item_request(pre_i, w.R, x);
     const int32_t j = assign[r];
-    if (j < 0) continue;
-    const psk::TableDesc d = tdesc[j];
-    const uint64_t o = w.off[r];
-    const uint64_t nb = w.off[r + 1] - o;
-    const uint64_t h = hit_chosen[r];
-    uint32_t added = 0;
-    bool full = false;
-    for (uint64_t k = h + lane; k < nb; k += 32) {
-      const uint64_t key = w.hash[o + k];
-      if (key == psk::kEmpty || key == psk::kTomb) continue;
-      bool ins = false;
-      const uint64_t slot = psk::thread_insert(slots, ovf, d, key, &ins);
-      if (slot == ~0ull) {
-        full = true;
-        continue;
-      }
-      if (ins) {
-        ++added;
-        if (meta.last_use) {
-          meta.last_use[slot] = last_use;
-          meta.children[slot] = 0;
-          meta.parent[slot] = psk::kLinkPending;
-        }
-      } else if (meta.last_use && meta.last_use[slot] < last_use) {
-        meta.last_use[slot] = last_use;
-      }
+    const uint64_t k = hit_chosen[r] + (x - pre_i[r]);
+    const uint64_t key = w.hash[w.off[r] + k];
+    if (key == psk::kEmpty || key == psk::kTomb) continue;
+    bool ins = false;
+    const uint64_t slot = psk::thread_insert(slots, ovf, tdesc[j], key, &ins);
+    if (slot == ~0ull) {
+      atomicOr(err, psk::kErrTableFull);
+      continue;
     }
-#pragma unroll
-    for (int s = 16; s > 0; s >>= 1) added += __shfl_xor_sync(0xffffffffu, added, s);
-    full = __any_sync(0xffffffffu, full);
-    if (lane == 0) {
-      if (added) atomicAdd(count + j, (unsigned long long)added);
-      if (full) atomicOr(err, psk::kErrTableFull);
+    if (ins) {
+      atomicAdd(count + j, 1ull);
+      if (meta.last_use) {
+        meta.last_use[slot] = last_use;
+        meta.children[slot] = 0;
+        meta.parent[slot] = psk::kLinkPending;
+      }
+    } else if (meta.last_use && meta.last_use[slot] < last_use) {
+      meta.last_use[slot] = last_use;
     }
   }
 }
 
 __global__ void commit_link_kernel(const uint64_t* slots, const uint64_t* ovf, const psk::TableDesc* __restrict__ tdesc,
                                    psk::WindowDev w, const int32_t* __restrict__ assign,
-                                   const uint32_t* __restrict__ hit_chosen, psk::LruMeta meta) {
-  const int lane = threadIdx.x & 31;
-  const uint32_t warps_total = (gridDim.x * blockDim.x) >> 5;
-  for (uint32_t r = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; r < w.R; r += warps_total) {
-    const int32_t j = assign[r];
-    if (j < 0) continue;
-    const psk::TableDesc d = tdesc[j];
+                                   const uint32_t* __restrict__ hit_chosen, const unsigned long long* __restrict__ pre_i,
+                                   psk::LruMeta meta) {
+  const unsigned long long total = pre_i[w.R];
+  for (unsigned long long x = blockIdx.x * (unsigned long long)blockDim.x + threadIdx.x; x < total;
+       x += (unsigned long long)gridDim.x * blockDim.x) {
+    const uint32_t r = item_request(pre_i, w.R, x);
+    const psk::TableDesc d = tdesc[assign[r]];
     const uint64_t o = w.off[r];
-    const uint64_t nb = w.off[r + 1] - o;
-    const uint64_t h = hit_chosen[r];
-    for (uint64_t k = h + lane; k < nb; k += 32) {
-      const uint64_t s = psk::main_find(slots, ovf, d, w.hash[o + k]);
-      if (s == ~0ull || meta.parent[s] != psk::kLinkPending) continue;  // not inserted by this commit
-      const uint64_t ps = k > 0 ? psk::main_find(slots, ovf, d, w.hash[o + k - 1]) : ~0ull;
-      meta.parent[s] = ps == ~0ull ? psk::kNoParent : ps;
-      if (ps != ~0ull) atomicAdd(meta.children + ps, 1u);
-    }
+    const uint64_t k = hit_chosen[r] + (x - pre_i[r]);
+    const uint64_t key = w.hash[o + k];
+    const uint64_t pkey = k > 0 ? w.hash[o + k - 1] : psk::kEmpty;
+    const uint64_t s = psk::main_find(slots, ovf, d, key);
+    if (s == ~0ull || meta.parent[s] != psk::kLinkPending) continue;  // not inserted by this commit
+    const uint64_t ps = k > 0 ? psk::main_find(slots, ovf, d, pkey) : ~0ull;
+    meta.parent[s] = ps == ~0ull ? psk::kNoParent : ps;
+    if (ps != ~0ull) atomicAdd(meta.children + ps, 1u);
   }
 }
 
@@ -296,20 +364,33 @@ __global__ void advance_kernel(psk::StateSoA st, uint32_t I, psk::ReqStore rq, p
 // can never be among E evictions, so a round of at most kHeapMax evictions reproduces the
 // one-at-a-time rule exactly; the host repeats rounds while an instance is still over capacity.
 constexpr int kLeafMax = 4096;
-constexpr int kHeapMax = 2048;
+constexpr int kHeapMax = 1536;  // with kLeafMax, two eviction blocks fit on an SM
 constexpr int kEvictThreads = 256;
 constexpr int kCollectThreads = 256;
 constexpr uint32_t kCollectSlotsPerThread = 8;
 
+// A leaf candidate with its parent's slot (kLeafNoParent for none), so that evicting it needs no
+// dependent load before the parent's metadata can be read.  Five 32-bit words (the hash split).
 struct Leaf {
   uint32_t last_use;
   uint32_t slot;
-  uint64_t hash;
+  uint32_t hash_lo, hash_hi;
+  uint32_t parent;
 };
-static_assert(sizeof(Leaf) == 16, "a leaf is one 16-byte word");
+static_assert(sizeof(Leaf) == 20, "a leaf is five 32-bit words");
+constexpr uint32_t kLeafNoParent = 0xFFFFFFFFu;
+
+__device__ __forceinline__ uint32_t parent32(uint64_t p) {
+  return (p == psk::kNoParent || p == psk::kLinkPending) ? kLeafNoParent : (uint32_t)p;
+}
+
+__device__ __forceinline__ Leaf make_leaf(uint32_t last_use, uint32_t slot, uint64_t hash, uint64_t parent) {
+  return Leaf{last_use, slot, (uint32_t)hash, (uint32_t)(hash >> 32), parent32(parent)};
+}
 
 __device__ __forceinline__ bool leaf_less(const Leaf& a, const Leaf& b) {
-  return a.last_use != b.last_use ? a.last_use < b.last_use : a.hash < b.hash;
+  if (a.last_use != b.last_use) return a.last_use < b.last_use;
+  return a.hash_hi != b.hash_hi ? a.hash_hi < b.hash_hi : a.hash_lo < b.hash_lo;
 }
 
 __device__ __forceinline__ void heap_push(Leaf* h, int& n, const Leaf& x) {
@@ -358,7 +439,8 @@ leaf_collect_kernel(const uint64_t* __restrict__ slots, const psk::TableDesc* __
     const uint64_t key = __ldcs(slots + s);
     if (key == psk::kEmpty || key == psk::kTomb || meta.children[s] != 0u) continue;
     const uint32_t at = atomicAdd(nleaf + i, 1u);
-    if (at < (uint32_t)kLeafMax) leafbuf[(uint64_t)i * kLeafMax + at] = Leaf{meta.last_use[s], (uint32_t)s, key};
+    if (at < (uint32_t)kLeafMax)
+      leafbuf[(uint64_t)i * kLeafMax + at] = make_leaf(meta.last_use[s], (uint32_t)s, key, meta.parent[s]);
   }
 }
 
@@ -379,7 +461,8 @@ evict_kernel(uint64_t* slots, unsigned long long* count, const uint64_t* __restr
   uint32_t np2 = 1;
   while (np2 < n) np2 <<= 1;
   for (uint32_t x = threadIdx.x; x < np2; x += kEvictThreads)
-    leaves[x] = x < n ? leafbuf[(uint64_t)i * kLeafMax + x] : Leaf{0xFFFFFFFFu, 0xFFFFFFFFu, ~0ull};
+    leaves[x] = x < n ? leafbuf[(uint64_t)i * kLeafMax + x]
+                      : Leaf{0xFFFFFFFFu, 0xFFFFFFFFu, 0xFFFFFFFFu, 0xFFFFFFFFu, kLeafNoParent};
   __syncthreads();
   for (uint32_t size = 2; size <= np2; size <<= 1) {  // bitonic sort by (last_use, hash)
     for (uint32_t stride = size >> 1; stride > 0; stride >>= 1) {
@@ -407,16 +490,25 @@ evict_kernel(uint64_t* slots, unsigned long long* count, const uint64_t* __restr
       const bool from_sorted = ptr < n && (hn == 0 || leaf_less(leaves[ptr], heap[0]));
       if (!from_sorted && hn == 0) break;
       const Leaf v = from_sorted ? leaves[ptr++] : heap_pop(heap, hn);
-      const uint64_t ps = meta.parent[v.slot];
+      const uint32_t ps = v.parent;
+      // the parent's metadata, all four words requested together
+      uint32_t pc = 0u, plu = 0u;
+      uint64_t ph = 0ull, pp = psk::kNoParent;
+      if (ps != kLeafNoParent) {
+        pc = meta.children[ps];
+        plu = meta.last_use[ps];
+        ph = slots[ps];
+        pp = meta.parent[ps];
+      }
       slots[v.slot] = psk::kEmpty;
       meta.last_use[v.slot] = 0;
       meta.children[v.slot] = 0;
       meta.parent[v.slot] = psk::kNoParent;
       ++evicted;
-      if (ps != psk::kNoParent && ps != psk::kLinkPending) {
-        const uint32_t c = meta.children[ps] - 1;
+      if (ps != kLeafNoParent) {
+        const uint32_t c = pc - 1;
         meta.children[ps] = c;
-        if (c == 0) heap_push(heap, hn, Leaf{meta.last_use[ps], (uint32_t)ps, slots[ps]});
+        if (c == 0) heap_push(heap, hn, make_leaf(plu, ps, ph, pp));
       }
     }
     count[i] = cnt - evicted;
@@ -470,21 +562,25 @@ cudaError_t launch_insert_chains(uint64_t* slots, uint64_t* ovf, const psk::Tabl
 cudaError_t launch_commit(uint64_t* slots, uint64_t* ovf, const psk::TableDesc* tdesc, uint32_t I,
                           unsigned long long* count, const psk::WindowDev& w, const int32_t* assign,
                           const uint32_t* hit_chosen, psk::LruMeta meta, uint32_t last_use,
-                          const psk::ReqStore& rq, const uint32_t* out_tokens, uint32_t* err, int num_sms,
-                          cudaStream_t s) {
+                          const psk::ReqStore& rq, const uint32_t* out_tokens, unsigned long long* prefix,
+                          uint32_t* err, int num_sms, cudaStream_t s) {
   if (w.R == 0) return cudaSuccess;
-  uint32_t g = (w.R + 7) / 8;  // one warp per request, 8 per block
-  if (g > (uint32_t)num_sms * 16) g = (uint32_t)num_sms * 16;
-  if (meta.last_use) {
-    commit_stamp_kernel<<<g, 256, 0, s>>>(slots, ovf, tdesc, w, assign, hit_chosen, meta, last_use);
-    cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
-  }
-  commit_insert_kernel<<<g, 256, 0, s>>>(slots, ovf, tdesc, count, w, assign, hit_chosen, meta, last_use, err);
+  unsigned long long* pre_s = prefix;          // [R + 1]
+  unsigned long long* pre_i = prefix + w.R + 1;  // [R + 1]
+  commit_prefix_kernel<<<1, 1024, 0, s>>>(w, assign, hit_chosen, pre_s, pre_i);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
+  const uint32_t g = (uint32_t)num_sms * 8u;  // flat items, grid-stride
   if (meta.last_use) {
-    commit_link_kernel<<<g, 256, 0, s>>>(slots, ovf, tdesc, w, assign, hit_chosen, meta);
+    commit_stamp_kernel<<<g, 256, 0, s>>>(slots, ovf, tdesc, w, assign, pre_s, meta, last_use);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+  }
+  commit_insert_kernel<<<g, 256, 0, s>>>(slots, ovf, tdesc, count, w, assign, hit_chosen, pre_i, meta, last_use, err);
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  if (meta.last_use) {
+    commit_link_kernel<<<g, 256, 0, s>>>(slots, ovf, tdesc, w, assign, hit_chosen, pre_i, meta);
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
   }
