@@ -438,8 +438,8 @@ def main():
     dominant = max(phases, key=phases.get)
     peak, peak_src = _peaks()
     probe_ms = km["probe_scratch"] + max(0.0, km["probe_derived"])
-    greedy_traffic = profile_figure("greedy_pipe_production_window_1024x2048.md", "DRAM bytes per request")
-    probe_traffic = profile_figure("probe_search_production_window_1024x2048.md", "DRAM bytes per lookup")
+    greedy_traffic = profile_figure("step_kernels_production_window_1024x8192.md", "DRAM bytes per request")
+    probe_traffic = profile_figure("step_kernels_production_window_1024x8192.md", "DRAM bytes per lookup")
     score_traffic = profile_figure("score_rows_production_window_1024x8192.md", "DRAM bytes per request")
     if dominant == "probe":
         achieved = probe_bytes / (probe_ms / 1000) / 1e9
@@ -457,7 +457,7 @@ def main():
                 "peak_source": peak_src, "algorithmic_bytes_per_launch": greedy_bytes,
                 "ns_per_decision": 1e6 * km[dominant] / R,
                 "note": "serial per-request dependency chain decided on one SM: latency-bound, not "
-                        "bandwidth-bound; traffic scaled by request count from the 2048-request ncu capture"}
+                        "bandwidth-bound; traffic scaled by request count from the 8192-request ncu capture"}
     probe_achieved = probe_bytes / (probe_ms / 1000) / 1e9
     line = {"metric": METRIC, "value": job_rate(world, R * I, ms), "unit": "scorings/s", "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
