@@ -591,6 +591,11 @@ __device__ __forceinline__ void ld_u64v(const void* p, uint64_t (&v)[N]) {
   }
 }
 
+// q and S within [0, 2^30): with L, n < 2^30 the sums S + L and q + n are exact in 32 bits.
+__device__ __forceinline__ bool narrow_qs(int64_t q, int64_t S) {
+  return q >= 0 && q < (1ll << 30) && S >= 0 && S < (1ll << 30);
+}
+
 template <int IPT>
 __device__ void decide_rows(const psk::RowPre* __restrict__ rows, uint32_t R, uint32_t I, psk::StateSoA committed,
                             psk::StateSoA pending, const psk::DevModel& m, int32_t* assign, uint8_t* __restrict__ path,
@@ -614,6 +619,7 @@ __device__ void decide_rows(const psk::RowPre* __restrict__ rows, uint32_t R, ui
   int32_t* s_qr = s_b + Ip;                                  // [Ip] queued requests
   int32_t* s_Bmax = s_qr + Ip;                               // [Ip] decode-slot limit
   __shared__ psk::RowPre s_row[8];  // rows r .. r + kRingAhead (a ring of 8 so no reader is overtaken)
+  __shared__ int s_wide;            // some instance's q or S left [0, 2^30): 64-bit token sums from then on
   __shared__ int32_t s_jm[16];      // pick of request x in s_jm[x & 15] (-1: rejected)
   __shared__ uint32_t s_red_w[32];  // per-warp W_min (order-preserving bits)
   __shared__ uint4 s_red_k[32];     // per-warp pick: key (x, y), instance (z), hit (w)
@@ -642,6 +648,8 @@ __device__ void decide_rows(const psk::RowPre* __restrict__ rows, uint32_t R, ui
     s_key0[i] = key0_bits(s_b[i], s_qr[i]);
   };
 
+  if (t == 0) s_wide = 0;
+  __syncthreads();
   for (uint32_t i = t; i < Ip; i += NT) {
     if (i < I) {
       s_b[i] = committed.b[i];
@@ -651,6 +659,7 @@ __device__ void decide_rows(const psk::RowPre* __restrict__ rows, uint32_t R, ui
       s_M[i] = committed.M[i];
       s_Bmax[i] = committed.Bmax[i];
       set_terms(i);
+      if (!narrow_qs(s_q[i], s_S[i])) s_wide = 1;
     } else {
       s_room[i] = -1;  // padding: never capacity-eligible
     }
@@ -702,6 +711,7 @@ __device__ void decide_rows(const psk::RowPre* __restrict__ rows, uint32_t R, ui
                       reinterpret_cast<const uint4*>(rows + r + kRingAhead) + t);
     psk::cp_async_wait_group<1>();  // this thread's copies of row r (and row constants <= r + 4)
     const psk::RowConst rc = row_of(cur);
+    const bool narrow = s_wide == 0;  // a thread owning an instance that left the range set the flag itself
     const uint32_t lcp0 = cur.lcp[0];
     float Wk[IPT], tpk[IPT];
     bool inA[IPT];
@@ -724,7 +734,7 @@ __device__ void decide_rows(const psk::RowPre* __restrict__ rows, uint32_t R, ui
         hr[k] = h;
         // T_pf at the hit: the ring's value unless it is marked unknown (the probe blocks raised the
         // hit) or the hit was raised here; W = T_pf(n, c) - T_pf(0, L)
-        tpk[k] = (h == hb[k] && tb[k] != psk::kNoTpfBits) ? __uint_as_float(tb[k]) : psk::t_pf_of_hit(m, rc.L, h);
+        tpk[k] = (h == hb[k] && tb[k] != psk::kNoTpfBits) ? __uint_as_float(tb[k]) : psk::t_pf32(m, rc.L, h);
         Wk[k] = __fsub_rn(tpk[k], rc.t_cached);
         inA[k] = (int32_t)rc.L <= (int32_t)rm[k];
         if (inA[k]) wbest = min(wbest, psk::f2ord(Wk[k]));
@@ -775,7 +785,11 @@ __device__ void decide_rows(const psk::RowPre* __restrict__ rows, uint32_t R, ui
         x.n = (int64_t)rc.L - 16 * (int64_t)hr[k];
         x.inA = true;
         float tpot, ttft;
-        psk::pair_lat(m, rc, x, it, (int64_t)q[k], (int64_t)S[k], &tpot, &ttft);
+        if (narrow)
+          psk::pair_lat32(m, rc, x.tpf, (int32_t)x.n, it.dec0, it.f, it.tq, it.Bp, (int32_t)q[k], (int32_t)S[k], &tpot,
+                          &ttft);
+        else
+          psk::pair_lat(m, rc, x, it, (int64_t)q[k], (int64_t)S[k], &tpot, &ttft);
         const uint64_t key = psk::pair_admitted(m, rc, tpot, ttft)
                                  ? psk::packed_key(0u, k0[k] | ((uint64_t)((1u << 26) - 1u - hr[k]) << 18))
                                  : psk::packed_key(1u, ((uint64_t)q[k] + (uint64_t)x.n) * (uint64_t)Bp[k]);
@@ -823,6 +837,7 @@ __device__ void decide_rows(const psk::RowPre* __restrict__ rows, uint32_t R, ui
       s_q[j] += (int64_t)rc.L - 16 * (int64_t)hj;
       s_S[j] += (int64_t)rc.L;
       set_terms(j);
+      if (!narrow_qs(s_q[j], s_S[j])) s_wide = 1;  // seen from the next step on (after its barriers)
     }
     if (r + 2 < R) copy_row(r + 2);
     psk::cp_async_commit();
