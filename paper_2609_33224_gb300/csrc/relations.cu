@@ -21,7 +21,7 @@
 
 namespace {
 
-constexpr uint32_t kParentScan = 4096;  // chain positions scanned back from the end for a parent
+constexpr uint32_t kParentScan = 1024;  // chain positions scanned back from the end for a parent (16K tokens)
 
 __device__ __forceinline__ uint32_t tab_home(uint64_t key, uint32_t n) {  // n is a power of two
   return (uint32_t)((key * 0x9E3779B97F4A7C15ull) >> 32) & (n - 1);
