@@ -92,7 +92,8 @@ struct Piece {
 };
 
 // Loads a piece's hits and evaluates pass 1: the capacity guard and, for pairs in A, T_pf at the hit
-// and W = T_pf(n, c) - T_pf(0, L).  Returns the order-preserving bits of the lane's W_min over A (all ones if none).
+// and W = T_pf(n, c) - T_pf(0, L).  Returns the order-preserving bits of the lane's W_min over A
+// (all ones if none).
 template <int NV, bool VEC>
 __device__ __forceinline__ uint32_t piece_pass1(const uint32_t* __restrict__ hrow, uint32_t I, uint32_t i_lo,
                                                 const ScoreSmem& s, const psk::DevModel& m, const psk::RowConst& rc,
