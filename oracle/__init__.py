@@ -12,6 +12,10 @@ Parity status of each oracle function (what pins it, in ``tests/test_oracle_pins
                             exhaustive brute force over tiny instance sets.
   * greedy               -- hand-traced tiny windows; replay invariant (each decision equals the
                             single-request rule on the state left by the earlier decisions).
+  * policy variants      -- Table 3 ablations and Table 4 selectors on a hand-worked request
+                            (``tests/test_oracle_policies.py``).
+  * eviction             -- hand traces, and the evicted set against the subtree-maximum order on
+                            random branching caches (``tests/test_oracle_eviction_order.py``).
 No oracle function is left "parity unpinned".
 """
 from __future__ import annotations
@@ -37,7 +41,15 @@ class OrcModel(ctypes.Structure):
     _fields_ = [(k, ctypes.c_float) for k in
                 ("a0", "a1", "a2", "a3", "a4", "a5", "b0", "b1", "b2", "g_q", "eta", "lout_median")] + [
         ("interference_mode", ctypes.c_int32), ("ttft_filter", ctypes.c_int32),
-        ("nseg", ctypes.c_int32), ("seg_lo", ctypes.c_int32 * 16), ("ema_factor", ctypes.c_float * 16)]
+        ("nseg", ctypes.c_int32), ("seg_lo", ctypes.c_int32 * 16), ("ema_factor", ctypes.c_float * 16),
+        ("cache_filter", ctypes.c_int32), ("slo_filter", ctypes.c_int32), ("fallback", ctypes.c_int32),
+        ("selector", ctypes.c_int32)]
+
+# Instance orders inside T (Table 4) and the ablation configurations (Table 3) as model keys.
+SELECTORS = {"D-C-Q": 0, "D": 1, "D-Q": 2, "D-C": 3, "D-Q-C": 4, "H-C-Q": 5}
+ABLATIONS = {"G": dict(cache_filter=0, slo_filter=0, fallback=1), "C": dict(cache_filter=1, slo_filter=0, fallback=1),
+             "T": dict(cache_filter=0, slo_filter=1, fallback=1), "CT": dict(cache_filter=1, slo_filter=1, fallback=1),
+             "F": dict(cache_filter=1, slo_filter=1, fallback=0)}
 
 
 def build(force: bool = False) -> str:
@@ -103,6 +115,12 @@ def make_model(model: dict) -> OrcModel:
     for k, (lo, f) in enumerate(zip(seg_lo, ema)):
         m.seg_lo[k] = int(lo)
         m.ema_factor[k] = float(f)
+    m.cache_filter = int(model.get("cache_filter", 1))
+    m.slo_filter = int(model.get("slo_filter", 1))
+    m.fallback = int(model.get("fallback", 0))
+    m.selector = int(model.get("selector", 0))
+    if m.fallback not in (0, 1) or not 0 <= m.selector <= 5:
+        raise ValueError("fallback 0 (LMetric) or 1 (D-C-Q); selector 0..5")
     return m
 
 

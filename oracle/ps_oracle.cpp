@@ -26,6 +26,11 @@
 //    ((b0 + b1 B) + b2 S') f + [b + qr > 0] T_pf(n,c) / max(1, L_out).
 //  * TTFT (Eq. 4): T_pf(n,c) + (a0 qr + a1 q), overhead neglected; the budget is
 //    max(target, T_pf(L,0)) (Section 8.1 Metrics); TTFT uses <=, TPOT uses strict < (Alg. 1).
+//  * Policy variants of the evaluation (Section 8.3; off by default): Table 3's admission
+//    ablations switch the KVC-first filter (C = A when off) and the SLO admission (T = C when off;
+//    the TTFT test goes with the TPOT test) and replace the LMetric fallback by the D-C-Q order
+//    over C; Table 4's selectors order T by D, D-Q, D-C, D-Q-C or H-C-Q, H being the predicted TPOT
+//    headroom target - TPOT (fp32), smallest first.  Every order ends with the lowest id.
 //  * Packing key D-C-Q (Section 6.2, Table 4): more decoding b, then more cached blocks h, then
 //    fewer queued requests qr, then the lowest instance id.  Fallback CacheAwareLB = LMetric
 //    (Section 6, Section 8.1 Baselines): min over C of (q + n)(b + qr + 1), lowest id on ties.
@@ -63,6 +68,12 @@ typedef struct {
   int32_t nseg;                    // decode-batch segments of the EMA factor table
   int32_t seg_lo[16];              // segment s covers B >= seg_lo[s] (ascending)
   float ema_factor[16];
+  // Policy variants of the evaluation's ablations (Section 8.3, Table 3 and Table 4); the defaults
+  // (1, 1, 0, 0) are Algorithm 1 as above.
+  int32_t cache_filter;            // 1: KVC-first filter (Eq. 8); 0: C = A
+  int32_t slo_filter;              // 1: TPOT (and TTFT) admission; 0: T = C
+  int32_t fallback;                // with T empty: 0 LMetric over C, 1 the D-C-Q order over C
+  int32_t selector;                // order inside T: 0 D-C-Q, 1 D, 2 D-Q, 3 D-C, 4 D-Q-C, 5 H-C-Q
 } orc_model;
 
 typedef struct { int32_t b, qr; int64_t q, S, M_KV; int32_t B_max; } orc_inst;
@@ -181,27 +192,51 @@ void decide(const Oracle& o, const uint64_t* chain, uint64_t nb, uint32_t L, flo
   for (uint32_t i = 0; i < I; ++i) {
     if (!inA[i]) continue;
     bool inC = (Z > 0.0f) ? ((W[i] - Wmin) <= etaZ) : true;
+    if (!m.cache_filter) inC = true;
     if (!inC) { row.cls[i] = 2; continue; }
     bool ok = row.tpot[i] < tpot_target;
     if (m.ttft_filter) ok = ok && (row.ttft[i] <= ttft_budget);
+    if (!m.slo_filter) ok = true;
     row.cls[i] = ok ? 0 : 1;
     anyT = anyT || ok;
   }
+  // Instance order (Section 6.2, Table 4): D more decoding requests, C more cached blocks, Q fewer
+  // queued requests, H smaller predicted TPOT headroom (target - TPOT); the lowest id last.
+  auto before = [&](uint32_t i, uint32_t z, int32_t sel) -> bool {
+    const orc_inst& a = o.st[i];
+    const orc_inst& y = o.st[z];
+    if (sel == 5) {
+      const float ha = tpot_target - row.tpot[i], hy = tpot_target - row.tpot[z];
+      if (ha != hy) return ha < hy;
+      if (row.hit[i] != row.hit[z]) return row.hit[i] > row.hit[z];
+      return a.qr < y.qr;
+    }
+    if (a.b != y.b) return a.b > y.b;
+    const bool useC = sel == 0 || sel == 3 || sel == 4, useQ = sel == 0 || sel == 2 || sel == 4;
+    const bool c_first = sel != 4;
+    if (c_first) {
+      if (useC && row.hit[i] != row.hit[z]) return row.hit[i] > row.hit[z];
+      if (useQ && a.qr != y.qr) return a.qr < y.qr;
+    } else {
+      if (useQ && a.qr != y.qr) return a.qr < y.qr;
+      if (useC && row.hit[i] != row.hit[z]) return row.hit[i] > row.hit[z];
+    }
+    return false;  // equal: the lower id, visited first, stays
+  };
   int32_t best = -1;
   if (anyT) {
-    // Decode-batch-size-centric key: more decoding, more cached, fewer queued, lowest id.
     for (uint32_t i = 0; i < I; ++i) {
       if (row.cls[i] != 0) continue;
-      if (best < 0) { best = (int32_t)i; continue; }
-      const orc_inst& a = o.st[i];
-      const orc_inst& z = o.st[best];
-      bool better;
-      if (a.b != z.b) better = a.b > z.b;
-      else if (row.hit[i] != row.hit[best]) better = row.hit[i] > row.hit[best];
-      else better = a.qr < z.qr;
-      if (better) best = (int32_t)i;
+      if (best < 0 || before(i, (uint32_t)best, m.selector)) best = (int32_t)i;
     }
     row.pick = best; row.path = 0;
+  } else if (m.fallback == 1) {
+    // The ablations' D-C-Q fallback over C (Table 3, configurations T and CT).
+    for (uint32_t i = 0; i < I; ++i) {
+      if (row.cls[i] != 1) continue;
+      if (best < 0 || before(i, (uint32_t)best, 0)) best = (int32_t)i;
+    }
+    row.pick = best; row.path = best >= 0 ? 1 : 2;
   } else {
     // CacheAwareLB = LMetric over C: pending uncached prefill tokens x active requests,
     // both including the arriving request.
