@@ -14,6 +14,8 @@ Parity status of each oracle function (what pins it, in ``tests/test_oracle_pins
                             single-request rule on the state left by the earlier decisions).
   * policy variants      -- Table 3 ablations and Table 4 selectors on a hand-worked request
                             (``tests/test_oracle_policies.py``).
+  * online calibration   -- hand trace, closed form of a constant ratio, bounds
+                            (``tests/test_oracle_calibration.py``).
   * eviction             -- hand traces, and the evicted set against the subtree-maximum order on
                             random branching caches (``tests/test_oracle_eviction_order.py``).
 No oracle function is left "parity unpinned".
@@ -93,6 +95,8 @@ def _lib():
         lib.orc_advance.argtypes = [vp, ctypes.c_float, u64, i32]
         lib.orc_last_use.restype = u32
         lib.orc_last_use.argtypes = [vp, u32, u64]
+        lib.orc_calibrate.argtypes = [vp, u64, vp, vp, vp, ctypes.c_float]
+        lib.orc_ema_factors.argtypes = [vp, vp]
         _LIB = lib
     return _LIB
 
@@ -246,3 +250,18 @@ class Oracle:
 
     def last_use(self, inst: int, block: int) -> int:
         return int(_lib().orc_last_use(self._h, int(inst), int(block)))
+
+    # -- online calibration (Section 5.3) --------------------------------------------------------
+    def calibrate(self, batch, ctx_tokens, measured_ms, weight: float = 0.02):
+        """Feed pure-decode samples (batch size, total context tokens, measured ms), in order."""
+        b = _c(batch, np.int32)
+        c = _c(ctx_tokens, np.int64)
+        t = _c(measured_ms, np.float32)
+        if not (b.shape == c.shape == t.shape):
+            raise ValueError("one batch size, context and duration per sample")
+        _lib().orc_calibrate(self._h, b.shape[0], _p(b), _p(c), _p(t), float(weight))
+
+    def ema_factors(self) -> np.ndarray:
+        out = np.zeros(16, np.float32)
+        _lib().orc_ema_factors(self._h, _p(out))
+        return out[: self._m.nseg].copy()

@@ -511,4 +511,36 @@ uint32_t orc_last_use(void* h, uint32_t inst, uint64_t block) {
   return it == o->meta[inst].end() ? 0 : it->second.last_use;
 }
 
+// Online calibration (Section 5.3): per decode-batch segment a multiplicative EMA factor of the
+// decode term.  Each pure-decode feedback sample (measured batch size B, total context S, measured
+// forward duration) is taken in order: the base model's prediction at the same B and S is
+// (b0 + b1 B) + b2 S, the measured-to-predicted ratio is clipped to [0.5, 2], the factor of B's
+// segment moves by the update weight towards it, f <- f + weight (ratio - f), and is clipped to
+// [1, 2].  Factors start at 1 (the model's table as given).
+void orc_calibrate(void* h, uint64_t n, const int32_t* batch, const int64_t* ctx_tokens, const float* measured_ms,
+                   float weight) {
+  Oracle* o = static_cast<Oracle*>(h);
+  orc_model& m = o->m;
+  for (uint64_t k = 0; k < n; ++k) {
+    const int64_t B = batch[k];
+    float base = m.b0 + m.b1 * (float)B;
+    base = base + m.b2 * (float)ctx_tokens[k];
+    float ratio = measured_ms[k] / base;
+    if (ratio < 0.5f) ratio = 0.5f;
+    if (ratio > 2.0f) ratio = 2.0f;
+    int s = 0;
+    for (int q = 0; q < m.nseg; ++q)
+      if ((int64_t)m.seg_lo[q] <= B) s = q;
+    float f = m.ema_factor[s] + weight * (ratio - m.ema_factor[s]);
+    if (f < 1.0f) f = 1.0f;
+    if (f > 2.0f) f = 2.0f;
+    m.ema_factor[s] = f;
+  }
+}
+
+void orc_ema_factors(void* h, float* out) {
+  const Oracle* o = static_cast<const Oracle*>(h);
+  for (int s = 0; s < 16; ++s) out[s] = o->m.ema_factor[s];
+}
+
 }  // extern "C"
