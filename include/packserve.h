@@ -207,6 +207,22 @@ PS_API ps_status ps_load_instances(ps_ctx* ctx, const ps_instance_state* s, uint
 /* Read the committed state (host array of n = num_instances entries). */
 PS_API ps_status ps_get_instances(ps_ctx* ctx, ps_instance_state* out, uint32_t n);
 
+/* Online calibration of the decode model (Section 5.3, "Online calibration"): feed n pure-decode
+ * feedback samples, in order (host arrays): batch[k] the measured decode batch size, ctx_tokens[k]
+ * the total context tokens of the batch, measured_ms[k] the forward's duration.  For each, the base
+ * prediction (b0 + b1 B) + b2 S at the same B and S gives the measured-to-predicted ratio, clipped
+ * to [0.5, 2]; the EMA factor of B's decode-batch segment (ps_model.seg_lo) moves towards it by
+ * `weight` (the paper uses 0.02), f <- f + weight (ratio - f), and is clipped to [1, 2].  The
+ * factors scale the decode term of every later TPOT prediction of the context.  Host-side only (no
+ * device work, no synchronisation).  PS_ERR_INVALID for n > 0 with a NULL array, a batch size below
+ * 0, a context below 0, a non-finite or non-positive duration, or a weight outside (0, 1]. */
+PS_API ps_status ps_calibrate(ps_ctx* ctx, uint32_t n, const int32_t* batch, const int64_t* ctx_tokens,
+                              const float* measured_ms, float weight);
+
+/* The current EMA factors, one per decode-batch segment (host array of n >= ps_model.nseg
+ * entries; entries past nseg are left untouched). */
+PS_API ps_status ps_get_ema_factors(ps_ctx* ctx, float* out, uint32_t n);
+
 /* Read the state a pending window would commit (the committed state updated by each of the
  * window's admitted requests: qr += 1, q_tokens += n, S_tokens += L).  PS_ERR_STATE if none. */
 PS_API ps_status ps_get_pending_instances(ps_ctx* ctx, ps_instance_state* out, uint32_t n);

@@ -23,6 +23,7 @@ STATUS_NAMES = {0: "PS_OK", 1: "PS_ERR_INVALID", 2: "PS_ERR_CUDA", 3: "PS_ERR_OO
                 4: "PS_ERR_TABLE_FULL", 5: "PS_ERR_TIMEOUT", 6: "PS_ERR_CAPACITY", 7: "PS_ERR_STATE"}
 
 ABI_FUNCTIONS = ("ps_create", "ps_load_instances", "ps_get_instances", "ps_get_pending_instances",
+                 "ps_calibrate", "ps_get_ema_factors",
                  "ps_insert_blocks", "ps_insert_chains", "ps_cached_blocks", "ps_score_window",
                  "ps_schedule_window", "ps_commit_window", "ps_last_timings", "ps_last_probe_stats", "ps_last_error",
                  "ps_destroy", "ps_score_window_noalloc", "ps_load_requests", "ps_advance_window")
@@ -114,6 +115,8 @@ def lib() -> ctypes.CDLL:
             "ps_commit_window": [vp, u32],
             "ps_last_timings": [vp, vp, u32],
             "ps_last_probe_stats": [vp, vp, u32],
+            "ps_calibrate": [vp, u32, vp, vp, vp, ctypes.c_float],
+            "ps_get_ema_factors": [vp, vp, u32],
             "ps_load_requests": [vp, u64, vp, vp, vp, vp, vp],
             "ps_advance_window": [vp, ctypes.POINTER(PsAdvanceParams)],
             "ps_score_window_noalloc": [vp, vp, vp, u32, ctypes.POINTER(PsStateArrays), ctypes.POINTER(PsWindow),
@@ -292,6 +295,22 @@ class Scheduler:
         self._check(lib().ps_last_timings(self._h, ms.ctypes.data, 7))
         names = ("probe", "score", "greedy", "commit", "relations", "probe_scratch", "probe_derived")
         return dict(zip(names, (float(x) for x in ms)))
+
+    def calibrate(self, batch, ctx_tokens, measured_ms, weight: float = 0.02):
+        """Online calibration (ps_calibrate): pure-decode samples, in order."""
+        b = np.ascontiguousarray(batch, np.int32)
+        c = np.ascontiguousarray(ctx_tokens, np.int64)
+        t = np.ascontiguousarray(measured_ms, np.float32)
+        if not (b.shape == c.shape == t.shape):
+            raise ValueError("one batch size, context and duration per sample")
+        n = b.shape[0]
+        self._check(lib().ps_calibrate(self._h, n, b.ctypes.data if n else None, c.ctypes.data if n else None,
+                                       t.ctypes.data if n else None, float(weight)))
+
+    def ema_factors(self) -> np.ndarray:
+        out = np.zeros(16, np.float32)
+        self._check(lib().ps_get_ema_factors(self._h, out.ctypes.data, 16))
+        return out
 
     def probe_stats(self) -> dict:
         """Counters of the last probe phase (see ps_last_probe_stats)."""

@@ -18,7 +18,9 @@ BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(BUILD, "libpackserve.so")
 SOURCES = ["api.cu", "probe.cu", "score.cu", "greedy.cu", "relations.cu", "table.cu", "noalloc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
+# host code is compiled without floating-point contraction (calibrate.h is exact fp32, op by op)
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-fvisibility=hidden",
+         "-Xcompiler", "-ffp-contract=off",
          "--expt-relaxed-constexpr"]
 
 
@@ -39,7 +41,8 @@ def _stale(out: str, deps) -> bool:
 def build(force: bool = False, verbose: bool = False) -> str:
     os.makedirs(BUILD, exist_ok=True)
     nvcc = _nvcc()
-    headers = [os.path.join(CSRC, "ps_internal.cuh"), os.path.join(ROOT, "include", "packserve.h")]
+    headers = [os.path.join(CSRC, "ps_internal.cuh"), os.path.join(CSRC, "calibrate.h"),
+               os.path.join(ROOT, "include", "packserve.h")]
     jobs = []
     for src in SOURCES:
         s = os.path.join(CSRC, src)

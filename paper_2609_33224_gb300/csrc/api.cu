@@ -12,6 +12,7 @@
 #include <algorithm>
 
 #include "packserve.h"
+#include "calibrate.h"
 #include "ps_internal.cuh"
 
 namespace {
@@ -541,6 +542,28 @@ static ps_status read_state(ps_ctx* c, const psk::StateSoA& st, ps_instance_stat
 ps_status ps_get_instances(ps_ctx* c, ps_instance_state* out, uint32_t n) {
   if (!c) return PS_ERR_INVALID;
   return read_state(c, c->st, out, n);
+}
+
+ps_status ps_calibrate(ps_ctx* c, uint32_t n, const int32_t* batch, const int64_t* ctx_tokens,
+                       const float* measured_ms, float weight) {
+  if (!c) return PS_ERR_INVALID;
+  if (!(weight > 0.0f && weight <= 1.0f)) return fail(c, PS_ERR_INVALID, "calibration weight must be in (0, 1]");
+  if (n == 0) return PS_OK;
+  if (!batch || !ctx_tokens || !measured_ms) return fail(c, PS_ERR_INVALID, "NULL calibration sample array");
+  for (uint32_t k = 0; k < n; ++k)
+    if (batch[k] < 0 || ctx_tokens[k] < 0 || !std::isfinite(measured_ms[k]) || !(measured_ms[k] > 0.0f))
+      return fail(c, PS_ERR_INVALID, "calibration sample " + std::to_string(k) +
+                                         ": batch and context >= 0, duration finite and > 0");
+  psk::DevModel& m = c->model;
+  pscal::ema_update(m.b0, m.b1, m.b2, m.nseg, m.seg_lo, m.ema, n, batch, ctx_tokens, measured_ms, weight);
+  return PS_OK;
+}
+
+ps_status ps_get_ema_factors(ps_ctx* c, float* out, uint32_t n) {
+  if (!c) return PS_ERR_INVALID;
+  if (!out || n < (uint32_t)c->model.nseg) return fail(c, PS_ERR_INVALID, "need nseg entries");
+  for (int s = 0; s < c->model.nseg; ++s) out[s] = c->model.ema[s];
+  return PS_OK;
 }
 
 ps_status ps_get_pending_instances(ps_ctx* c, ps_instance_state* out, uint32_t n) {
