@@ -83,3 +83,33 @@ def test_default_policy_is_algorithm_1():
     """The defaults are the F configuration with the D-C-Q order."""
     assert _pick(50.0)[:2] == _pick(50.0, **ABLATIONS["F"], selector=SELECTORS["D-C-Q"])[:2]
     assert _pick(5.0)[:2] == _pick(5.0, **ABLATIONS["F"])[:2]
+
+
+@pytest.mark.parametrize("policy", [dict(ABLATIONS["G"]), dict(ABLATIONS["T"]), dict(ABLATIONS["CT"]),
+                                    dict(selector=SELECTORS["H-C-Q"]), dict(selector=SELECTORS["D-Q-C"])])
+def test_greedy_replay_under_policy_variants(policy):
+    """Under every variant, each greedy decision equals the single-request rule on the state left by
+    the earlier decisions (the greedy applies the variant, not the default)."""
+    wl = W.generate(0)
+    win, ins = wl.window, wl.instances
+    model = dict(wl.model, **policy)
+    sched = Oracle(ins.I, model).load(ins).schedule(win)
+    replay = Oracle(ins.I, model).load(ins)
+    for r in range(win.R):
+        one = replay.score_rows(win, rows=[r])
+        assert one["best"][0] == sched["assign"][r] and one["path"][0] == sched["path"][r]
+        j = int(one["best"][0])
+        if j < 0:
+            continue
+        h = int(one["hits"][0, j])
+        st = replay.get_state()
+        L = int(win.prompt_tokens[r])
+        st["qr"][j] += 1
+        st["q"][j] += L - 16 * h
+        st["S"][j] += L
+        replay.set_state(st["b"], st["qr"], st["q"], st["S"], st["M_KV"], st["B_max"])
+        ch = win.chain_hash[win.chain_off[r]:win.chain_off[r + 1]]
+        replay.insert_chain(j, ch[h:], parent=int(ch[h - 1]) if h else 0)
+    if policy in (dict(ABLATIONS["G"]), dict(ABLATIONS["T"])):  # these admit other instances here
+        default = Oracle(ins.I, wl.model).load(ins).schedule(win)
+        assert not np.array_equal(sched["assign"], default["assign"])
