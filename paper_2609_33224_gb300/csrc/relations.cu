@@ -70,8 +70,9 @@ static_assert(psk::kLcpBack % kLcpGroup == 0, "whole groups of searches");
 // earlier request is a 32-ary first-miss search, and an earlier request whose last block equals
 // this chain's block at its own length is a prefix of this chain.
 //   lcp: the kLcpBack searches advance kLcpGroup at a time, one 32-ary step of each per round.
-//   par: positions are scanned back from the chain's end, 256 per warp step; the deepest position
-//        whose block ends an earlier request of exactly that length gives the parent.
+//   par: the last kParentScan positions are scanned back from the chain's end, 256 per warp step;
+//        the deepest position whose block ends an earlier request of exactly that length gives the
+//        parent.  A request whose parent lies further back is searched from scratch (exact).
 __global__ void __launch_bounds__(256, 3)
 relations_kernel(psk::WindowDev w, psk::DevModel m, const psk::LastSlot* tab, uint32_t n, psk::RowPre* rows) {
   const int lane = threadIdx.x & 31;
