@@ -223,6 +223,15 @@ PS_API ps_status ps_calibrate(ps_ctx* ctx, uint32_t n, const int32_t* batch, con
  * entries; entries past nseg are left untouched). */
 PS_API ps_status ps_get_ema_factors(ps_ctx* ctx, float* out, uint32_t n);
 
+/* Replace the performance model (Section 5 coefficients, eta of Eq. 8, the TTFT filter, the EMA
+ * segments and factors) with the same checks as ps_create.  The new model's EMA factors replace
+ * what ps_calibrate has learned.  Takes effect at the next ps_score_window, ps_schedule_window or
+ * ps_advance_window; a pending window keeps the decisions it was made with.  Host-side only (no
+ * device work).  Used, for instance, to sweep the recompute budget eta over one window (the
+ * sensitivity study of Section 8) without rebuilding the tables.
+ * Errors: PS_ERR_INVALID (NULL model or a field out of range; the previous model stays). */
+PS_API ps_status ps_set_model(ps_ctx* ctx, const ps_model* model);
+
 /* Read the state a pending window would commit (the committed state updated by each of the
  * window's admitted requests: qr += 1, q_tokens += n, S_tokens += L).  PS_ERR_STATE if none. */
 PS_API ps_status ps_get_pending_instances(ps_ctx* ctx, ps_instance_state* out, uint32_t n);

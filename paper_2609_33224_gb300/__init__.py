@@ -23,7 +23,7 @@ STATUS_NAMES = {0: "PS_OK", 1: "PS_ERR_INVALID", 2: "PS_ERR_CUDA", 3: "PS_ERR_OO
                 4: "PS_ERR_TABLE_FULL", 5: "PS_ERR_TIMEOUT", 6: "PS_ERR_CAPACITY", 7: "PS_ERR_STATE"}
 
 ABI_FUNCTIONS = ("ps_create", "ps_load_instances", "ps_get_instances", "ps_get_pending_instances",
-                 "ps_calibrate", "ps_get_ema_factors",
+                 "ps_calibrate", "ps_get_ema_factors", "ps_set_model",
                  "ps_insert_blocks", "ps_insert_chains", "ps_cached_blocks", "ps_score_window",
                  "ps_schedule_window", "ps_commit_window", "ps_last_timings", "ps_last_probe_stats", "ps_last_error",
                  "ps_destroy", "ps_score_window_noalloc", "ps_load_requests", "ps_advance_window")
@@ -117,6 +117,7 @@ def lib() -> ctypes.CDLL:
             "ps_last_probe_stats": [vp, vp, u32],
             "ps_calibrate": [vp, u32, vp, vp, vp, ctypes.c_float],
             "ps_get_ema_factors": [vp, vp, u32],
+            "ps_set_model": [vp, ctypes.POINTER(PsModel)],
             "ps_load_requests": [vp, u64, vp, vp, vp, vp, vp],
             "ps_advance_window": [vp, ctypes.POINTER(PsAdvanceParams)],
             "ps_score_window_noalloc": [vp, vp, vp, u32, ctypes.POINTER(PsStateArrays), ctypes.POINTER(PsWindow),
@@ -311,6 +312,11 @@ class Scheduler:
         out = np.zeros(16, np.float32)
         self._check(lib().ps_get_ema_factors(self._h, out.ctypes.data, 16))
         return out
+
+    def set_model(self, model: dict):
+        """Replace the performance model (ps_set_model); the EMA factors become the model's."""
+        m = make_model(model)
+        self._check(lib().ps_set_model(self._h, ctypes.byref(m)))
 
     def probe_stats(self) -> dict:
         """Counters of the last probe phase (see ps_last_probe_stats)."""

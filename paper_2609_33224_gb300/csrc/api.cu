@@ -566,6 +566,14 @@ ps_status ps_get_ema_factors(ps_ctx* c, float* out, uint32_t n) {
   return PS_OK;
 }
 
+ps_status ps_set_model(ps_ctx* c, const ps_model* m) {
+  if (!c) return PS_ERR_INVALID;
+  if (!m) return fail(c, PS_ERR_INVALID, "NULL model");
+  if (check_model(c, *m) != PS_OK) return PS_ERR_INVALID;
+  c->model = to_dev(*m);
+  return PS_OK;
+}
+
 ps_status ps_get_pending_instances(ps_ctx* c, ps_instance_state* out, uint32_t n) {
   if (!c) return PS_ERR_INVALID;
   if (!c->pending) return fail(c, PS_ERR_STATE, "no pending window");
