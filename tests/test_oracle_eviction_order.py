@@ -89,3 +89,37 @@ def test_eviction_set_matches_subtree_maximum_order(seed):
         for ch, _ in chains:
             for h in (int(x) for x in ch):
                 assert o.contains(0, h) == (h in keep), (seed, E, h)
+
+
+def test_streaming_stamps_are_monotone_and_eviction_takes_whole_windows():
+    """Under the streaming rules a commit stamps the whole chain of an admitted request on its
+    instance (cached prefix and new blocks) with the window, so along every cached chain a block's
+    last_use is at least its child's; with the subtree-maximum order above, eviction then takes
+    blocks oldest window first: no evicted block is newer than a surviving one."""
+    wl = W.generate(0, seed=5)
+    ins = wl.instances
+    o = Oracle(ins.I, wl.model, track_lru=True).load(ins)
+    o.set_capacity(np.full(ins.I, 1500, np.uint64))  # below the seeded caches: every window evicts
+    o.load_requests(dict(inst=[], state=[], L=[], out=[], rem=[]))  # nothing in flight: requests admitted
+    tracked = []  # chains of every window so far
+    evicted_any = False
+    for w in range(4):
+        win = wl.window if w == 0 else wl.next_window(24)
+        o.schedule(win, window_id=w + 1, streaming=True)
+        tracked += [win.chain_hash[win.chain_off[r]:win.chain_off[r + 1]] for r in range(win.R)]
+        blocks = {int(h) for ch in tracked for h in ch}
+        before = {(i, h): o.last_use(i, h) for i in range(ins.I) for h in blocks if o.contains(i, h)}
+        for i in range(ins.I):
+            for ch in tracked:
+                for k in range(1, len(ch)):
+                    if o.contains(i, int(ch[k])):
+                        assert o.contains(i, int(ch[k - 1]))
+                        assert o.last_use(i, int(ch[k - 1])) >= o.last_use(i, int(ch[k])), (w, i, k)
+        o.advance(20.0, 1000)
+        for i in range(ins.I):
+            gone = [lu for (j, h), lu in before.items() if j == i and not o.contains(i, h)]
+            kept = [lu for (j, h), lu in before.items() if j == i and o.contains(i, h)]
+            if gone and kept:
+                evicted_any = True
+                assert max(gone) <= min(kept), (w, i, max(gone), min(kept))
+    assert evicted_any
