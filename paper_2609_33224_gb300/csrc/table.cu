@@ -257,7 +257,7 @@ __global__ void commit_queue_kernel(uint32_t I, psk::WindowDev w, const int32_t*
   }
 }
 
-// Engine progress of one streaming window, one warp per instance (the rules the oracle states):
+// Engine progress of one streaming window, one warp per instance (the serving engine's rules):
 // every decoding request emits k = max(1, floor(window_ms / ((b0 + b1 b) + b2 S))) tokens (fp32,
 // state at the window start), finished requests leave (b -= 1, S -= L + out), then the FIFO queue
 // drains prefill_tokens tokens and requests whose prefill completes start decoding.
