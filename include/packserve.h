@@ -49,7 +49,7 @@ typedef enum {
   PS_ERR_CUDA = 2,       /* a CUDA runtime call failed (message in ps_last_error) */
   PS_ERR_OOM = 3,        /* device or pinned allocation failed in ps_create */
   PS_ERR_TABLE_FULL = 4, /* a hash table has no free slot left for an insert */
-  PS_ERR_TIMEOUT = 5,    /* a bounded device-side wait gave up (reserved; no kernel waits today) */
+  PS_ERR_TIMEOUT = 5,    /* a bounded device-side wait of the greedy pass gave up (ps_set_wait_limit) */
   PS_ERR_CAPACITY = 6,   /* an instance holds more blocks than its cache capacity */
   PS_ERR_STATE = 7       /* call out of order (e.g. commit with no pending window) */
 } ps_status;
@@ -68,7 +68,21 @@ enum { PS_MAX_EMA_SEGMENTS = 16, PS_BLOCK_TOKENS = 16 };
  * eta: recompute budget of Eq. 8 (>= 0; the paper's default is 0.5).
  * ttft_filter: 1 adds "TTFT <= max(ttft_target, T_pf(L, 0))" to the TPOT admission test of
  * Algorithm 1 (the TTFT SLO of Section 8.1 Metrics); 0 applies Algorithm 1 exactly.
- * All coefficients must be finite with magnitude <= 1e9; EMA factors finite and > 0. */
+ * All coefficients must be finite with magnitude <= 1e9; EMA factors finite and > 0.
+ *
+ * Policy variants of the evaluation (Section 8.3; all zero = Algorithm 1 as above):
+ *   cache_filter_off  1: no KVC-first filter, C = A (Table 3 configurations G and T).
+ *   slo_filter_off    1: no SLO admission, T = C (Table 3 G and C; the TTFT test goes with it).
+ *   fallback_dcq      1: with T empty, pick over C by the D-C-Q order instead of the LMetric product
+ *                     (Table 3 T and CT; path 1 as for the LMetric fallback).
+ *   selector          order inside T (Table 4): PS_SELECT_DCQ (0, Section 6.2: more decoding
+ *                     requests, then more cached blocks, then fewer queued requests), PS_SELECT_D,
+ *                     PS_SELECT_DQ, PS_SELECT_DC, PS_SELECT_DQC, PS_SELECT_HCQ (smallest predicted
+ *                     TPOT headroom tpot_target - TPOT in fp32 first, then more cached blocks, then
+ *                     fewer queued requests).  Every order ends with the lowest instance id. */
+enum { PS_SELECT_DCQ = 0, PS_SELECT_D = 1, PS_SELECT_DQ = 2, PS_SELECT_DC = 3, PS_SELECT_DQC = 4,
+       PS_SELECT_HCQ = 5 };
+
 typedef struct {
   float a0, a1, a2, a3, a4, a5;
   float b0, b1, b2;
@@ -80,18 +94,23 @@ typedef struct {
   int32_t nseg;
   int32_t seg_lo[PS_MAX_EMA_SEGMENTS];
   float ema_factor[PS_MAX_EMA_SEGMENTS];
+  int32_t cache_filter_off;
+  int32_t slo_filter_off;
+  int32_t fallback_dcq;
+  int32_t selector;
 } ps_model;
 
 /* Context configuration (ps_create).
  *   device, cuda_stream   CUDA device ordinal and the cudaStream_t to launch on (NULL: the
  *                         library creates and owns a non-blocking stream).
- *   num_instances         1..2048 (the greedy kernel keeps ~85 bytes of shared memory per instance).
+ *   num_instances         1..2048 (the greedy pass keeps every instance's state in the shared memory
+ *                         of one SM, about 100 bytes per instance).
  *   max_window_requests   largest R a window may have (1..131072).
  *   max_window_chain_blocks  largest total chain length (sum over requests) of a window.
  *   block_tokens          must be 16 (PS_BLOCK_TOKENS).
  *   cap_blocks            host array [num_instances]: cache capacity of each instance in blocks.
  *   table_load_factor     slots of instance i = ceil(cap_blocks[i] / table_load_factor), rounded
- *                         up to 16-slot buckets; (0, 0.95].
+ *                         up to whole 8-slot (64-byte) buckets; (0, 0.95].
  *   model                 the performance model above.
  *   probe_mode            how hit lengths are found (both give the same hits on the caches they
  *                         accept):
@@ -194,17 +213,23 @@ typedef struct {
   int32_t outputs_on_device;
 } ps_decisions;
 
-/* Create a context: allocates every table and buffer up front (instance hash tables sized by
- * cap_blocks / table_load_factor, a window-scoped delta table of 2 * max_window_chain_blocks
- * slots, window staging and score scratch).  Instances start empty with zero state.
+/* Create a context: the scheduler of Section 4 (System overview) with the per-instance prefix caches
+ * of Section 7 (Implementation: the scheduler's prefix tree of cached prefixes, here one hash table of
+ * chained block hashes per instance) and the performance model of Section 5.  Allocates every table
+ * and buffer up front (instance hash tables sized by cap_blocks / table_load_factor, a window-scoped
+ * delta table of 2 * max_window_chain_blocks slots, window staging and score scratch).  Instances
+ * start empty with zero state.  cfg is read during the call only.
  * Errors: PS_ERR_INVALID (config), PS_ERR_CUDA, PS_ERR_OOM.  *out is NULL on failure. */
 PS_API ps_status ps_create(const ps_config* cfg, ps_ctx** out);
 
-/* Replace the committed state of all instances (host array of n = num_instances entries).
- * Discards any pending window.  Errors: PS_ERR_INVALID (n or a field out of range). */
+/* Replace the committed state of all instances (host array of n = num_instances entries): the
+ * per-instance records the paper's metadata service keeps (Section 4, "Metadata service": running
+ * decode batch, queued requests and prefill tokens, KV usage and capacity).  Discards any pending
+ * window.  Errors: PS_ERR_INVALID (n or a field out of range); the state is unchanged then. */
 PS_API ps_status ps_load_instances(ps_ctx* ctx, const ps_instance_state* s, uint32_t n);
 
-/* Read the committed state (host array of n = num_instances entries). */
+/* Read the committed state (host array of n = num_instances entries): the Section 4 metadata-service
+ * records as the library holds them after the last commit or load. */
 PS_API ps_status ps_get_instances(ps_ctx* ctx, ps_instance_state* out, uint32_t n);
 
 /* Online calibration of the decode model (Section 5.3, "Online calibration"): feed n pure-decode
@@ -219,8 +244,8 @@ PS_API ps_status ps_get_instances(ps_ctx* ctx, ps_instance_state* out, uint32_t 
 PS_API ps_status ps_calibrate(ps_ctx* ctx, uint32_t n, const int32_t* batch, const int64_t* ctx_tokens,
                               const float* measured_ms, float weight);
 
-/* The current EMA factors, one per decode-batch segment (host array of n >= ps_model.nseg
- * entries; entries past nseg are left untouched). */
+/* The current EMA factors of Section 5.3's online calibration, one per decode-batch segment (host
+ * array of n >= ps_model.nseg entries; entries past nseg are left untouched). */
 PS_API ps_status ps_get_ema_factors(ps_ctx* ctx, float* out, uint32_t n);
 
 /* Replace the performance model (Section 5 coefficients, eta of Eq. 8, the TTFT filter, the EMA
@@ -232,12 +257,23 @@ PS_API ps_status ps_get_ema_factors(ps_ctx* ctx, float* out, uint32_t n);
  * Errors: PS_ERR_INVALID (NULL model or a field out of range; the previous model stays). */
 PS_API ps_status ps_set_model(ps_ctx* ctx, const ps_model* model);
 
+/* Bound on every cross-block wait of the greedy pass (ns; 0 restores the default of 1 s; at most
+ * 60 s).  The greedy's thread blocks hand decisions, inserts and probed hits to one another through
+ * flags in device memory (Section 4's per-request state tracking, run as a pipeline); a block that
+ * waits longer than this records the failure and returns, so a launch always ends, and the call
+ * returns PS_ERR_TIMEOUT with the window's outputs undefined and no pending window.  The context
+ * stays usable: the next call starts from the committed state.  Host-side only.
+ * Errors: PS_ERR_INVALID (ns above 60 s). */
+PS_API ps_status ps_set_wait_limit(ps_ctx* ctx, uint64_t ns);
+
 /* Read the state a pending window would commit (the committed state updated by each of the
- * window's admitted requests: qr += 1, q_tokens += n, S_tokens += L).  PS_ERR_STATE if none. */
+ * window's admitted requests: qr += 1, q_tokens += n, S_tokens += L, the per-decision state update
+ * of Section 4's request-path tracking).  PS_ERR_STATE if none. */
 PS_API ps_status ps_get_pending_instances(ps_ctx* ctx, ps_instance_state* out, uint32_t n);
 
-/* Cache a chain of n blocks on instance inst (host array): block 0 continues parent_hash (0 = the
- * chain starts at the root), block k continues block k-1.  Blocks already cached are skipped.
+/* Cache a chain of n blocks on instance inst (host array): a path of the instance's prefix tree
+ * (Section 7, Implementation), block 0 continuing parent_hash (0 = the chain starts at the root) and
+ * block k continuing block k-1.  Blocks already cached are skipped.
  * last_use stamps the blocks for LRU bookkeeping.
  * Errors: PS_ERR_INVALID (inst, reserved hash, or in PS_PROBE_SEARCH mode a parent_hash that is not
  * cached once the call's blocks are in), PS_ERR_TABLE_FULL (no slot left), PS_ERR_CAPACITY (the
@@ -246,17 +282,20 @@ PS_API ps_status ps_get_pending_instances(ps_ctx* ctx, ps_instance_state* out, u
 PS_API ps_status ps_insert_blocks(ps_ctx* ctx, uint32_t inst, const uint64_t* chain, uint64_t n,
                            uint64_t parent_hash, uint32_t last_use);
 
-/* Bulk form of ps_insert_blocks over nchains chains in CSR form: chain c goes to instance inst[c],
+/* Bulk form of ps_insert_blocks (Section 7 prefix-tree paths) over nchains chains in CSR form: chain c goes to instance inst[c],
  * its blocks are hash[off[c] .. off[c+1]) and its first block continues parent[c].  on_device
  * selects host (0) or device (1) arrays.  Same errors as ps_insert_blocks. */
 PS_API ps_status ps_insert_chains(ps_ctx* ctx, uint64_t nchains, const uint32_t* inst, const uint64_t* off,
                            const uint64_t* hash, const uint64_t* parent, uint32_t last_use,
                            int32_t on_device);
 
-/* Number of blocks cached on each instance (host array [n = num_instances]). */
+/* Number of blocks cached on each instance's prefix cache (Section 7; host array
+ * [n = num_instances]). */
 PS_API ps_status ps_cached_blocks(ps_ctx* ctx, uint64_t* out, uint32_t n);
 
-/* Score a window: every request independently against the committed state (no state change).
+/* Score a window: Algorithm 1 (Section 6) for every request independently against the committed
+ * state (no state change), with the hit lengths of Section 7's prefix caches and the latencies of
+ * Eq. 4-9.
  * Runs the probe kernel (hit lengths of all R x I pairs) and the fused score kernel (latencies,
  * filters, packing key and per-request argmin).  Errors: PS_ERR_INVALID (window layout, R too
  * large, chain length != L/16, total blocks too large), PS_ERR_CUDA. */
@@ -273,7 +312,8 @@ PS_API ps_status ps_score_window(ps_ctx* ctx, const ps_window* w, ps_scores* out
 PS_API ps_status ps_schedule_window(ps_ctx* ctx, const ps_window* w, ps_decisions* out,
                              ps_scores* opt_scores);
 
-/* Commit the pending window: the pending state becomes the committed state and each admitted
+/* Commit the pending window (Section 4: the gateway updates the instance records along the
+ * request path): the pending state becomes the committed state and each admitted
  * request's uncached blocks are cached on its instance.  With track_lru every block of an admitted
  * request's chain on its instance (cached prefix and new blocks) gets last_use; with request
  * tracking each admitted request joins its instance's FIFO queue (remaining prefill = its uncached
@@ -295,7 +335,8 @@ PS_API ps_status ps_commit_window(ps_ctx* ctx, uint32_t last_use);
  *   3. with evict = 1 (needs track_lru): while an instance holds more blocks than its capacity,
  *      its leaf block (no cached child) with the smallest (last_use, hash) is evicted. */
 
-/* Requests in flight at the start of a stream (context created with max_active_requests > 0),
+/* Requests in flight at the start of a stream (Section 4's request-path tracking; context created
+ * with max_active_requests > 0),
  * host arrays of n entries: instance, state (0 queued, in FIFO order per instance; 1 decoding),
  * prompt tokens L, output tokens out, rem (queued: remaining prefill tokens; decoding: remaining
  * output tokens, 1..out).  Replaces all tracked requests; the committed state's b, qr, q_tokens
@@ -311,13 +352,15 @@ typedef struct {
   int32_t evict;            /* 1: evict to capacity (needs track_lru) */
 } ps_advance_params;
 
-/* Advance every instance by one window (rules above).  Errors: PS_ERR_STATE (a scheduled window
+/* Advance every instance by one window (rules above: Section 4's response-path updates, with the
+ * engine's progress simulated).  Errors: PS_ERR_STATE (a scheduled window
  * is still pending, or no request tracking), PS_ERR_INVALID (params), PS_ERR_CAPACITY (a decoding
  * list is full), PS_ERR_TABLE_FULL (an instance has more leaves than the eviction buffer holds,
  * 4096; its eviction stops). */
 PS_API ps_status ps_advance_window(ps_ctx* ctx, const ps_advance_params* p);
 
-/* Device time in ms (CUDA events recorded on the context's stream around each kernel) of the last
+/* Scheduling overhead, the quantity Section 8.3.3 reports as arrival-to-decision latency: device
+ * time in ms (CUDA events recorded on the context's stream around each kernel) of the last
  * ps_score_window / ps_schedule_window call and of the commit after it: ms[0] probe phase (relations
  * + both probe kernels), ms[1] fused score, ms[2] greedy, ms[3] commit; with n >= 7 also the probe
  * phase's parts: ms[4] relations kernel, ms[5] probe of the rows searched from scratch, ms[6] probe
@@ -325,7 +368,8 @@ PS_API ps_status ps_advance_window(ps_ctx* ctx, const ps_advance_params* p);
  * untouched. */
 PS_API ps_status ps_last_timings(ps_ctx* ctx, float* ms, uint32_t n);
 
-/* Counters of the last probe phase (ps_score_window / ps_schedule_window), for roofline accounting
+/* Counters of the last probe phase (the Section 7 prefix-cache lookups of ps_score_window /
+ * ps_schedule_window), for roofline accounting
  * (host array of n >= 6 entries):
  *   out[0] rows searched from scratch        out[1] rows derived from an earlier request's row
  *   out[2] table lookups in scratch rows     out[3] table lookups in derived rows
@@ -345,11 +389,16 @@ PS_API ps_status ps_last_probe_stats(ps_ctx* ctx, uint64_t* out, uint32_t n);
  *
  * It computes what ps_score_window computes (probe kernel + fused score kernel, same results) for
  * caches laid out the way the library lays them out:
- *   slots    device u64 array holding every instance's table; value 0 = empty slot.
- *   overflow_bits  device u64 array of overflow bitmaps, one bit per bucket.
- *   tables   device array [num_instances] of ps_table_desc: instance i's table is num_buckets
- *            buckets of 8 slots starting at slot `base`, and its overflow bitmap starts at word
- *            `overflow_base` of overflow_bits (bit b of the bitmap = word b / 64, bit b % 64).
+ *   slots    device u64 array holding every instance's table, 16-byte aligned; value 0 = empty
+ *            slot.  0 and 0xFFFFFFFFFFFFFFFF are reserved key values: a request block with either
+ *            value never counts as cached (its hit ends there), so a block hash must avoid both.
+ *   overflow_bits  device u64 array of overflow bitmaps, one bit per bucket (8-byte aligned).
+ *   tables   device array [num_instances] of ps_table_desc (8-byte aligned): instance i's table is
+ *            num_buckets >= 1 buckets of 8 slots starting at slot `base`, a multiple of 8 (whole
+ *            buckets), and its overflow bitmap starts at word `overflow_base` of overflow_bits (bit b
+ *            of the bitmap = word b / 64, bit b % 64).  Every table and bitmap must lie inside the
+ *            caller's arrays (the library cannot see their sizes); a descriptor with num_buckets 0 or
+ *            a base that is not a multiple of 8 is rejected (PS_ERR_INVALID) before any lookup.
  *            A block hash h has two candidate buckets, b1 = (h * num_buckets) >> 64 and
  *            b2 = (g * num_buckets) >> 64 with g = (h ^ (h >> 31)) * 0x7FB5D329728EA185 mod 2^64
  *            (high 64 bits of the 128-bit products), and is stored in one of them; if both were
@@ -366,8 +415,9 @@ PS_API ps_status ps_last_probe_stats(ps_ctx* ctx, uint64_t* out, uint32_t n);
  * any stream capture.  All calls share the one array: calls that overlap on the GPU (other threads
  * or streams) race and must be serialised by the caller.  The call allocates nothing (no
  * cudaMalloc, cudaFree or allocating library routine).
- * Errors: PS_ERR_INVALID (NULL or host buffers, sizes beyond the limit, bad window layout or model),
- * PS_ERR_CUDA.  No context exists, so there is no message for ps_last_error. */
+ * Errors: PS_ERR_INVALID (NULL or host buffers, misaligned arrays, a bad table descriptor, sizes
+ * beyond the limit, bad window layout or model), PS_ERR_CUDA.  No context exists, so there is no
+ * message for ps_last_error. */
 #define PS_NOALLOC_MAX_PAIRS 2097152u
 
 typedef struct {
@@ -392,10 +442,13 @@ PS_API ps_status ps_score_window_noalloc(const uint64_t* slots, const uint64_t* 
                                          const ps_window* window, const ps_model* model,
                                          int32_t probe_mode, ps_scores* out, void* cuda_stream);
 
-/* Text of the last error on this context ("" if none).  Valid until the next call. */
+/* Text of the last error on this context ("" if none).  Valid until the next call.  Error
+ * reporting only: the paper has no counterpart. */
 PS_API const char* ps_last_error(const ps_ctx* ctx);
 
-/* Release every resource of the context.  NULL is accepted. */
+/* Release every resource of the context (its prefix-cache tables of Section 7 and the scheduler
+ * state of Section 4): waits for the context's stream, then frees every allocation.  NULL is
+ * accepted.  The context pointer is invalid afterwards. */
 PS_API void ps_destroy(ps_ctx* ctx);
 
 #ifdef __cplusplus

@@ -23,7 +23,7 @@ STATUS_NAMES = {0: "PS_OK", 1: "PS_ERR_INVALID", 2: "PS_ERR_CUDA", 3: "PS_ERR_OO
                 4: "PS_ERR_TABLE_FULL", 5: "PS_ERR_TIMEOUT", 6: "PS_ERR_CAPACITY", 7: "PS_ERR_STATE"}
 
 ABI_FUNCTIONS = ("ps_create", "ps_load_instances", "ps_get_instances", "ps_get_pending_instances",
-                 "ps_calibrate", "ps_get_ema_factors", "ps_set_model",
+                 "ps_calibrate", "ps_get_ema_factors", "ps_set_model", "ps_set_wait_limit",
                  "ps_insert_blocks", "ps_insert_chains", "ps_cached_blocks", "ps_score_window",
                  "ps_schedule_window", "ps_commit_window", "ps_last_timings", "ps_last_probe_stats", "ps_last_error",
                  "ps_destroy", "ps_score_window_noalloc", "ps_load_requests", "ps_advance_window")
@@ -33,7 +33,18 @@ class PsModel(ctypes.Structure):
     _fields_ = [(k, ctypes.c_float) for k in
                 ("a0", "a1", "a2", "a3", "a4", "a5", "b0", "b1", "b2", "g_q", "eta", "lout_median")] + [
         ("interference_mode", ctypes.c_int32), ("ttft_filter", ctypes.c_int32), ("nseg", ctypes.c_int32),
-        ("seg_lo", ctypes.c_int32 * 16), ("ema_factor", ctypes.c_float * 16)]
+        ("seg_lo", ctypes.c_int32 * 16), ("ema_factor", ctypes.c_float * 16),
+        ("cache_filter_off", ctypes.c_int32), ("slo_filter_off", ctypes.c_int32), ("fallback_dcq", ctypes.c_int32),
+        ("selector", ctypes.c_int32)]
+
+
+# Table 4 instance orders (ps_model.selector) and Table 3 admission ablations (ps_model switches).
+SELECTORS = {"D-C-Q": 0, "D": 1, "D-Q": 2, "D-C": 3, "D-Q-C": 4, "H-C-Q": 5}
+ABLATIONS = {"G": dict(cache_filter_off=1, slo_filter_off=1, fallback_dcq=1),
+             "C": dict(cache_filter_off=0, slo_filter_off=1, fallback_dcq=1),
+             "T": dict(cache_filter_off=1, slo_filter_off=0, fallback_dcq=1),
+             "CT": dict(cache_filter_off=0, slo_filter_off=0, fallback_dcq=1),
+             "F": dict(cache_filter_off=0, slo_filter_off=0, fallback_dcq=0)}
 
 
 class PsConfig(ctypes.Structure):
@@ -118,6 +129,7 @@ def lib() -> ctypes.CDLL:
             "ps_calibrate": [vp, u32, vp, vp, vp, ctypes.c_float],
             "ps_get_ema_factors": [vp, vp, u32],
             "ps_set_model": [vp, ctypes.POINTER(PsModel)],
+            "ps_set_wait_limit": [vp, u64],
             "ps_load_requests": [vp, u64, vp, vp, vp, vp, vp],
             "ps_advance_window": [vp, ctypes.POINTER(PsAdvanceParams)],
             "ps_score_window_noalloc": [vp, vp, vp, u32, ctypes.POINTER(PsStateArrays), ctypes.POINTER(PsWindow),
@@ -159,6 +171,8 @@ def make_model(model: dict) -> PsModel:
     for k, (lo, f) in enumerate(zip(seg_lo, ema)):
         m.seg_lo[k] = int(lo)
         m.ema_factor[k] = float(f)
+    for k in ("cache_filter_off", "slo_filter_off", "fallback_dcq", "selector"):
+        setattr(m, k, int(model.get(k, 0)))
     return m
 
 
@@ -317,6 +331,10 @@ class Scheduler:
         """Replace the performance model (ps_set_model); the EMA factors become the model's."""
         m = make_model(model)
         self._check(lib().ps_set_model(self._h, ctypes.byref(m)))
+
+    def set_wait_limit(self, ns: int = 0):
+        """Bound on the greedy pass's cross-block waits (ps_set_wait_limit; 0 = the 1-s default)."""
+        self._check(lib().ps_set_wait_limit(self._h, int(ns)))
 
     def probe_stats(self) -> dict:
         """Counters of the last probe phase (see ps_last_probe_stats)."""

@@ -23,6 +23,7 @@ enum Ev { kEvProbe0, kEvProbe1, kEvScore0, kEvScore1, kEvGreedy0, kEvGreedy1, kE
           kEvProbeMid, kNumEv };
 constexpr int kNumPhases = 4;
 constexpr int kNumStats = 6;
+constexpr uint64_t kDefaultWaitNs = 1000000000ull;  // 1 s: bound on a cross-block wait of the greedy
 
 struct DeviceGuard {
   int prev = -1;
@@ -56,7 +57,7 @@ struct ps_ctx {
   unsigned long long* d_count = nullptr;
   psk::DeltaSlot* d_delta = nullptr;
   uint64_t delta_nslots = 0;
-  psk::GreedySync gsync{nullptr, nullptr, nullptr, nullptr, nullptr, 0u};
+  psk::GreedySync gsync{nullptr, nullptr, nullptr, nullptr, nullptr, 0u, kDefaultWaitNs};
   psk::RowPre* d_rows = nullptr;      // per-request constants and relations (search mode greedy)
   psk::LastSlot* d_lastslot = nullptr;
   psk::RowList scratch{nullptr, nullptr};  // rows the probe searches from scratch
@@ -144,6 +145,9 @@ ps_status check_model(ps_ctx* c, const ps_model& m) {
     if (s > 0 && m.seg_lo[s] <= m.seg_lo[s - 1]) return fail(c, PS_ERR_INVALID, "seg_lo must ascend");
   }
   if (m.seg_lo[0] > 1) return fail(c, PS_ERR_INVALID, "seg_lo[0] must be <= 1");
+  if ((m.cache_filter_off | m.slo_filter_off | m.fallback_dcq) & ~1)
+    return fail(c, PS_ERR_INVALID, "cache_filter_off, slo_filter_off and fallback_dcq must be 0 or 1");
+  if (m.selector < PS_SELECT_DCQ || m.selector > PS_SELECT_HCQ) return fail(c, PS_ERR_INVALID, "selector must be 0..5");
   return PS_OK;
 }
 
@@ -158,6 +162,10 @@ psk::DevModel to_dev(const ps_model& m) {
     d.seg_lo[s] = m.seg_lo[s];
     d.ema[s] = m.ema_factor[s];
   }
+  d.cache_off = m.cache_filter_off;
+  d.slo_off = m.slo_filter_off;
+  d.fb_dcq = m.fallback_dcq;
+  d.sel = m.selector;
   return d;
 }
 
@@ -571,6 +579,13 @@ ps_status ps_set_model(ps_ctx* c, const ps_model* m) {
   if (!m) return fail(c, PS_ERR_INVALID, "NULL model");
   if (check_model(c, *m) != PS_OK) return PS_ERR_INVALID;
   c->model = to_dev(*m);
+  return PS_OK;
+}
+
+ps_status ps_set_wait_limit(ps_ctx* c, uint64_t ns) {
+  if (!c) return PS_ERR_INVALID;
+  if (ns > 60ull * kDefaultWaitNs) return fail(c, PS_ERR_INVALID, "wait limit above 60 s");
+  c->gsync.wait_ns = ns == 0 ? kDefaultWaitNs : ns;
   return PS_OK;
 }
 

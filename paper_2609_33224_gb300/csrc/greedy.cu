@@ -50,10 +50,12 @@ __device__ __forceinline__ void cross_warp_min_any(const float* s_w, const int* 
   anyA = __any_sync(0xffffffffu, a);
 }
 
-__device__ __forceinline__ psk::ArgKey cross_warp_argmin(const psk::ArgKey* s_k, int nw) {
+// Per-warp (key, tie) partials -> the block's minimum, reduced by every warp.
+__device__ __forceinline__ void cross_warp_pick(const uint4* s_k, int nw, uint64_t* key, uint32_t* tie) {
   const int lane = threadIdx.x & 31;
-  psk::ArgKey k = lane < nw ? s_k[lane] : psk::ArgKey{psk::kNoKeyCi, ~0ull};
-  return psk::warp_argmin(k);
+  const uint4 pk = lane < nw ? s_k[lane] : make_uint4(0xFFFFFFFFu, 0xFFFFFFFFu, 0xFFFFFFFFu, 0u);
+  uint32_t h;
+  psk::warp_pick_min(((uint64_t)pk.y << 32) | pk.x, pk.z, pk.w, key, tie, &h);
 }
 
 template <int IPT, bool SEARCH>
@@ -78,7 +80,7 @@ greedy_kernel(const uint64_t* __restrict__ slots, const uint64_t* __restrict__ o
   uint8_t* s_touched = reinterpret_cast<uint8_t*>(s_it + I);
   __shared__ float s_red_w[32];
   __shared__ int s_red_a[32];
-  __shared__ psk::ArgKey s_red_k[32];
+  __shared__ uint4 s_red_k[32];
   __shared__ uint32_t s_nwalk;
 
   const int t = threadIdx.x;
@@ -200,29 +202,49 @@ greedy_kernel(const uint64_t* __restrict__ slots, const uint64_t* __restrict__ o
         if (i < I && hn[k] < nx.nb) cn[k] = w.hash[nx.o + hn[k]];
       }
     }
-    // Pass 2: admission classes and the lexicographic argmin.
-    psk::ArgKey best{psk::kNoKeyCi, ~0ull};
+    // Pass 2: admission classes and the packed (class, value) key with its tie word.
+    uint64_t bkey = psk::kNoKey;
+    uint32_t btie = 0xFFFFFFFFu;
 #pragma unroll
     for (int k = 0; k < IPT; ++k) {
       const uint32_t i = t + k * NT;
       if (i < I && ev[k].inA) {
         const uint32_t cls = psk::pair_class(m, rc, ev[k], wmin);
         if (cls <= 1u) {
-          const psk::ArgKey kk{(cls << 28) | i, psk::pair_value(cls, hc[k], s_b[i], s_qr[i], s_q[i], ev[k].n)};
-          if (psk::key_less(kk, best)) best = kk;
+          uint64_t key;
+          uint32_t tie = i;
+          if (cls == 0u) {
+            key = psk::packed_key(0u, psk::value_in_t(m, psk::key0_bits(m, s_b[i], s_qr[i]), hc[k], ev[k].tpot,
+                                                      rc.tpot_target));
+            tie = psk::tie_in_t(m, i, s_qr[i]);
+          } else {
+            const int32_t Bp = s_b[i] + s_qr[i] + 1;
+            key = psk::packed_key(1u, psk::value_fallback(m, (uint64_t)(s_q[i] + ev[k].n), (uint32_t)Bp,
+                                                          psk::dcq_key0(s_b[i], s_qr[i]), hc[k]));
+          }
+          if (key < bkey || (key == bkey && tie < btie)) {
+            bkey = key;
+            btie = tie;
+          }
         }
       }
     }
-    best = psk::warp_argmin(best);
-    if (lane == 0) s_red_k[warp] = best;
+    {
+      uint64_t wk;
+      uint32_t wt, wh;
+      psk::warp_pick_min(bkey, btie, 0u, &wk, &wt, &wh);
+      if (lane == 0) s_red_k[warp] = make_uint4((uint32_t)wk, (uint32_t)(wk >> 32), wt, 0u);
+    }
     __syncthreads();  // (D)
-    best = cross_warp_argmin(s_red_k, NW);
-    const bool pick = anyA && best.ci != psk::kNoKeyCi;
-    const uint32_t j = best.ci & 0x0FFFFFFFu;
+    uint64_t bk;
+    uint32_t bt;
+    cross_warp_pick(s_red_k, NW, &bk, &bt);
+    const bool pick = anyA && bk != psk::kNoKey;
+    const uint32_t j = bt & psk::kTieInstMask;
     const uint32_t hj = pick ? s_h[j] : 0u;
     if (t == 0) {
       assign[r] = pick ? (int32_t)j : -1;
-      path[r] = pick ? (uint8_t)(best.ci >> 28) : (uint8_t)2;
+      path[r] = pick ? (uint8_t)(bk >> 62) : (uint8_t)2;
       hit_chosen[r] = hj;
       if (pick) {
         s_qr[j] += 1;
@@ -301,14 +323,13 @@ cudaError_t greedy_launch(const uint64_t* slots, const uint64_t* ovf, const psk:
 //   prefix-closed main table.  Inserts of requests s - kLag + 1 .. s - 1 may land while a probe
 //   runs, in any order: any snapshot between delta(<= s - kLag) and delta(<= s - 1) gives a first
 //   miss between the two sets' first misses, and the max with the lcp terms is exact all the same.
-// Every cross-block wait is bounded (kWaitNs); on expiry the waiter records PS_ERR_TIMEOUT and
-// stops waiting, so the launch always ends.  Instance state lives in the deciding block's shared
+// Every cross-block wait is bounded (GreedySync::wait_ns, 1 s unless the caller set another limit);
+// on expiry the waiter records PS_ERR_TIMEOUT and stops waiting, so the launch always ends.  Instance state lives in the deciding block's shared
 // memory and is written only by the thread that owns the instance.
 
 constexpr uint32_t kInsertBlocks = 8;         // insert blocks
 constexpr uint32_t kProbeBlocks = 16;         // probe blocks
 constexpr uint32_t kRingAhead = 6;            // row constants are copied into the ring this many rows ahead
-constexpr uint64_t kWaitNs = 1000000000ull;   // bound on any cross-block wait
 constexpr unsigned long long kJobValid = 1ull << 63;  // a published job word (0 = not yet published)
 
 __device__ __forceinline__ psk::RowConst row_of(const psk::RowPre& x) {
@@ -322,12 +343,12 @@ __device__ __forceinline__ psk::RowConst row_of(const psk::RowPre& x) {
   return rc;
 }
 
-// Bounded spin until *flag != 0 (acquire).  false on timeout (and the error bit is set).
-__device__ __forceinline__ bool wait_flag(const uint32_t* flag, uint32_t* err) {
+// Bounded spin until *flag != 0 (acquire).  false after limit_ns (and the error bit is set).
+__device__ __forceinline__ bool wait_flag(const uint32_t* flag, uint32_t* err, uint64_t limit_ns) {
   if (psk::ld_acquire_u32(flag) != 0u) return true;
   const uint64_t t0 = psk::globaltimer_ns();
   while (psk::ld_acquire_u32(flag) == 0u) {
-    if (psk::globaltimer_ns() - t0 > kWaitNs) {
+    if (psk::globaltimer_ns() - t0 > limit_ns) {
       atomicOr(err, psk::kErrTimeout);
       return false;
     }
@@ -336,15 +357,16 @@ __device__ __forceinline__ bool wait_flag(const uint32_t* flag, uint32_t* err) {
   return true;
 }
 
-// Bounded wait for a published job word; 0 on timeout (and the error bit is set).
-__device__ __forceinline__ unsigned long long wait_job(const unsigned long long* job, uint32_t* err) {
+// Bounded wait for a published job word; 0 after limit_ns (and the error bit is set).
+__device__ __forceinline__ unsigned long long wait_job(const unsigned long long* job, uint32_t* err,
+                                                       uint64_t limit_ns) {
   unsigned long long v = psk::ld_relaxed_u64(job);
   if (v & kJobValid) return v;
   const uint64_t t0 = psk::globaltimer_ns();
   for (;;) {
     v = psk::ld_relaxed_u64(job);
     if (v & kJobValid) return v;
-    if (psk::globaltimer_ns() - t0 > kWaitNs) {
+    if (psk::globaltimer_ns() - t0 > limit_ns) {
       atomicOr(err, psk::kErrTimeout);
       return 0ull;
     }
@@ -362,7 +384,7 @@ __device__ void insert_blocks(const psk::RowPre* __restrict__ rows, const uint64
   __shared__ unsigned long long s_job;
   const uint32_t t = threadIdx.x;
   for (uint32_t job = blockIdx.x - 1; job < R; job += kInsertBlocks) {
-    if (t == 0) s_job = wait_job(sync.jobs + job, err);
+    if (t == 0) s_job = wait_job(sync.jobs + job, err, sync.wait_ns);
     __syncthreads();
     const unsigned long long jb = s_job;
     if (jb == 0ull) return;  // block-uniform: timed out
@@ -427,7 +449,7 @@ __device__ void probe_rows(const psk::RowPre* __restrict__ rows, const uint64_t*
         const uint32_t x = f + (uint32_t)lane;
         const bool mine = (int64_t)x < need;
         unsigned long long jb = 0ull;
-        if (mine) jb = wait_job(sync.jobs + x, err);
+        if (mine) jb = wait_job(sync.jobs + x, err, sync.wait_ns);
         abort = __any_sync(0xffffffffu, mine && jb == 0ull);
         if (abort) break;
         const uint32_t j = mine ? job_pick(jb) : 0xFFFFFFFFu;
@@ -491,7 +513,7 @@ __device__ void probe_rows(const psk::RowPre* __restrict__ rows, const uint64_t*
         const uint32_t nok = (okm == 0xffffffffu) ? 32u : (uint32_t)(__ffs(~okm) - 1);
         if (nok == 0u) {
           bool got = true;
-          if (lane == 0) got = wait_flag(sync.done + f, err);
+          if (lane == 0) got = wait_flag(sync.done + f, err, sync.wait_ns);
           abort = !__shfl_sync(0xffffffffu, got, 0);
           continue;
         }
@@ -605,7 +627,7 @@ __device__ void decide_rows(const psk::RowPre* __restrict__ rows, uint32_t R, ui
   // Every [Ip] array starts 16-byte aligned (Ip is a multiple of 4); the 8-byte arrays come first.
   int64_t* s_q = reinterpret_cast<int64_t*>(smem_raw);    // [Ip] queued prefill tokens
   int64_t* s_S = s_q + Ip;                                // [Ip] KV tokens held
-  uint64_t* s_key0 = reinterpret_cast<uint64_t*>(s_S + Ip);  // [Ip] class-0 key bits of (b, qr)
+  uint64_t* s_key0 = reinterpret_cast<uint64_t*>(s_S + Ip);  // [Ip] D-C-Q key bits of (b, qr) (psk::dcq_key0)
   int64_t* s_M = reinterpret_cast<int64_t*>(s_key0 + Ip);    // [Ip] KV capacity
   uint32_t* s_hit = reinterpret_cast<uint32_t*>(s_M + Ip);   // [4][Ip] probed hits of rows r .. r + 3
   uint32_t* s_tpf = s_hit + 4 * Ip;                          // [4][Ip] T_pf at those hits (bits)
@@ -634,9 +656,6 @@ __device__ void decide_rows(const psk::RowPre* __restrict__ rows, uint32_t R, ui
   const uint32_t i0 = (uint32_t)t * IPT;  // first owned instance (>= I for the signalling warp)
   const bool owner = t < NTI;             // false for the whole signalling warp
   const bool has = owner && i0 < I;       // the thread owns instances (then i0 + IPT <= Ip)
-  auto key0_bits = [](int32_t b, int32_t qr) -> uint64_t {
-    return ((uint64_t)((1u << 18) - 1u - (uint32_t)b) << 44) | (uint64_t)(uint32_t)qr;
-  };
   // instance terms of i after a state change (decode-slot guard folded into the KV room)
   auto set_terms = [&](uint32_t i) {
     const psk::InstTerms it = psk::inst_terms(m, s_b[i], s_qr[i], s_q[i], s_Bmax[i]);
@@ -645,7 +664,7 @@ __device__ void decide_rows(const psk::RowPre* __restrict__ rows, uint32_t R, ui
     s_tq[i] = it.tq;
     s_Bp[i] = it.Bp;
     s_room[i] = it.okB ? psk::kv_room(s_S[i], s_M[i]) : -1;
-    s_key0[i] = key0_bits(s_b[i], s_qr[i]);
+    s_key0[i] = psk::dcq_key0(s_b[i], s_qr[i]);
   };
 
   if (t == 0) s_wide = 0;
@@ -674,7 +693,7 @@ __device__ void decide_rows(const psk::RowPre* __restrict__ rows, uint32_t R, ui
   }
   bool timed_out = false;
   if (sig) {
-    for (uint32_t x = 0; x < 2 && x < R && !timed_out; ++x) timed_out = !wait_flag(sync.ready + x, err);
+    for (uint32_t x = 0; x < 2 && x < R && !timed_out; ++x) timed_out = !wait_flag(sync.ready + x, err, sync.wait_ns);
   }
   __syncthreads();
   // hits of rows 0 and 1, one copy group each (each thread copies and later reads only its own)
@@ -700,7 +719,7 @@ __device__ void decide_rows(const psk::RowPre* __restrict__ rows, uint32_t R, ui
       uint32_t ready_seen = 1u;
       if (sig && r + 2 < R && !timed_out) ready_seen = psk::ld_acquire_u32(sync.ready + r + 2);
       __syncthreads();  // (C)
-      if (sig && ready_seen == 0u) timed_out = !wait_flag(sync.ready + r + 2, err);
+      if (sig && ready_seen == 0u) timed_out = !wait_flag(sync.ready + r + 2, err, sync.wait_ns);
       __syncthreads();  // (D)
       continue;
     }
@@ -752,7 +771,7 @@ __device__ void decide_rows(const psk::RowPre* __restrict__ rows, uint32_t R, ui
     const bool anyA = wmin_o != 0xFFFFFFFFu;  // a W of a pair in A never maps to all ones (not NaN)
     const float wmin = psk::ord2f(wmin_o);
     uint64_t bkey = psk::kNoKey;
-    uint32_t binst = 0xFFFFFFFFu, bh = 0u;
+    uint32_t btie = 0xFFFFFFFFu, bh = 0u;
     bool inC[IPT];
     bool anyC = false;
 #pragma unroll
@@ -790,12 +809,17 @@ __device__ void decide_rows(const psk::RowPre* __restrict__ rows, uint32_t R, ui
                           &ttft);
         else
           psk::pair_lat(m, rc, x, it, (int64_t)q[k], (int64_t)S[k], &tpot, &ttft);
-        const uint64_t key = psk::pair_admitted(m, rc, tpot, ttft)
-                                 ? psk::packed_key(0u, k0[k] | ((uint64_t)((1u << 26) - 1u - hr[k]) << 18))
-                                 : psk::packed_key(1u, ((uint64_t)q[k] + (uint64_t)x.n) * (uint64_t)Bp[k]);
-        if (key < bkey) {  // instances ascend within a thread, so ties keep the lowest
+        uint64_t key;
+        uint32_t tie = i0 + k;
+        if (psk::pair_admitted(m, rc, tpot, ttft)) {
+          key = psk::packed_key(0u, psk::value_in_t(m, psk::key0_from_dcq(m, k0[k]), hr[k], tpot, rc.tpot_target));
+          if (m.sel == psk::kSelHCQ) tie = psk::tie_in_t(m, i0 + k, (int32_t)(k0[k] & 0x3FFFFull));
+        } else {
+          key = psk::packed_key(1u, psk::value_fallback(m, (uint64_t)q[k] + (uint64_t)x.n, (uint32_t)Bp[k], k0[k], hr[k]));
+        }
+        if (key < bkey || (key == bkey && tie < btie)) {
           bkey = key;
-          binst = i0 + k;
+          btie = tie;
           bh = hr[k];
         }
       }
@@ -803,7 +827,7 @@ __device__ void decide_rows(const psk::RowPre* __restrict__ rows, uint32_t R, ui
     {
       uint64_t wk;
       uint32_t wi, wh;
-      psk::warp_pick_min(bkey, binst, bh, &wk, &wi, &wh);
+      psk::warp_pick_min(bkey, btie, bh, &wk, &wi, &wh);
       if (lane == 0) s_red_k[warp] = make_uint4((uint32_t)wk, (uint32_t)(wk >> 32), wi, wh);
     }
     // Row r + 1's raises from requests r - 1 .. r - kLag + 1 (thread d - 1 takes request r - d); the
@@ -822,6 +846,7 @@ __device__ void decide_rows(const psk::RowPre* __restrict__ rows, uint32_t R, ui
     {
       const uint4 pk = lane < NWI ? s_red_k[lane] : make_uint4(0xFFFFFFFFu, 0xFFFFFFFFu, 0xFFFFFFFFu, 0u);
       psk::warp_pick_min(((uint64_t)pk.y << 32) | pk.x, pk.z, pk.w, &key, &j, &hj);
+      j &= psk::kTieInstMask;
     }
     const bool pick = anyA && key != psk::kNoKey;
     if (!pick) hj = 0u;

@@ -64,7 +64,8 @@ bool model_ok(const ps_model& m) {
     if (!(m.ema_factor[s] > 0.0f && m.ema_factor[s] <= 1e9f)) return false;
     if (s > 0 && m.seg_lo[s] <= m.seg_lo[s - 1]) return false;
   }
-  return true;
+  if ((m.cache_filter_off | m.slo_filter_off | m.fallback_dcq) & ~1) return false;
+  return m.selector >= PS_SELECT_DCQ && m.selector <= PS_SELECT_HCQ;
 }
 
 psk::DevModel dev_model(const ps_model& m) {
@@ -78,10 +79,25 @@ psk::DevModel dev_model(const ps_model& m) {
     d.seg_lo[s] = m.seg_lo[s];
     d.ema[s] = m.ema_factor[s];
   }
+  d.cache_off = m.cache_filter_off;
+  d.slo_off = m.slo_filter_off;
+  d.fb_dcq = m.fallback_dcq;
+  d.sel = m.selector;
   return d;
 }
 
 static_assert(sizeof(ps_table_desc) == sizeof(psk::TableDesc), "ps_table_desc layout");
+
+// The caller's table descriptors live in device memory: before any lookup reads a table, check that
+// each starts on a whole bucket (the probe reads a bucket as four 16-byte loads) and has at least
+// one bucket.  A bad descriptor sets the error word, so the call returns PS_ERR_INVALID instead of
+// reading misaligned or absent slots.
+__global__ void check_tables_kernel(const psk::TableDesc* __restrict__ td, uint32_t I, uint32_t* err) {
+  for (uint32_t i = blockIdx.x * blockDim.x + threadIdx.x; i < I; i += gridDim.x * blockDim.x) {
+    const psk::TableDesc d = td[i];
+    if (d.nbkt == 0u || (d.base % psk::kBucketSlots) != 0u) atomicOr(err, psk::kErrTableLayout);
+  }
+}
 
 }  // namespace
 
@@ -92,6 +108,10 @@ ps_status ps_score_window_noalloc(const uint64_t* slots, const uint64_t* overflo
                                   const ps_state_arrays* state, const ps_window* w, const ps_model* model,
                                   int32_t probe_mode, ps_scores* out, void* cuda_stream) {
   if (!slots || !overflow_bits || !tables || !state || !w || !model || !out) return PS_ERR_INVALID;
+  // buckets are read with 16-byte loads; overflow words and descriptors are 8-byte words
+  if ((reinterpret_cast<uintptr_t>(slots) & 15u) || (reinterpret_cast<uintptr_t>(overflow_bits) & 7u) ||
+      (reinterpret_cast<uintptr_t>(tables) & 7u))
+    return PS_ERR_INVALID;
   if (num_instances < 1 || num_instances > 4096) return PS_ERR_INVALID;
   if (w->inputs_on_device != 1 || out->outputs_on_device != 1) return PS_ERR_INVALID;
   if (probe_mode != PS_PROBE_LINEAR && probe_mode != PS_PROBE_SEARCH) return PS_ERR_INVALID;
@@ -114,6 +134,9 @@ ps_status ps_score_window_noalloc(const uint64_t* slots, const uint64_t* overflo
   if (cudaMemsetAsync(err, 0, sizeof(uint32_t), s) != cudaSuccess) return PS_ERR_CUDA;
   const psk::WindowDev wd{w->chain_off, w->chain_hash, w->prompt_tokens, w->ttft_target, w->tpot_target, w->R};
   if (pskl::launch_validate_window(wd, ~0ull, err, s) != cudaSuccess) return PS_ERR_CUDA;
+  const psk::TableDesc* td = reinterpret_cast<const psk::TableDesc*>(tables);
+  check_tables_kernel<<<(num_instances + 255) / 256, 256, 0, s>>>(td, num_instances, err);
+  if (cudaGetLastError() != cudaSuccess) return PS_ERR_CUDA;
   uint32_t herr = 0;
   uint64_t nblk = 0;
   if (cudaMemcpyAsync(&herr, err, sizeof(uint32_t), cudaMemcpyDeviceToHost, s) != cudaSuccess ||
@@ -121,7 +144,6 @@ ps_status ps_score_window_noalloc(const uint64_t* slots, const uint64_t* overflo
       cudaStreamSynchronize(s) != cudaSuccess)
     return PS_ERR_CUDA;
   if (herr != 0 || (nblk > 0 && !w->chain_hash)) return PS_ERR_INVALID;
-  const psk::TableDesc* td = reinterpret_cast<const psk::TableDesc*>(tables);
   const int grid = num_instances >= 64 ? d->probe_grid_large : d->probe_grid_small;
   const psk::DevModel dm = dev_model(*model);
   if (pskl::launch_probe(slots, overflow_bits, td, num_instances, wd, nullptr, psk::RowList{nullptr, nullptr}, hits, nullptr, dm, grid,

@@ -40,6 +40,7 @@ enum : uint32_t {
   kErrTimeout = 64u,
   kErrRequestsFull = 128u,
   kErrLeavesFull = 256u,
+  kErrTableLayout = 512u,
 };
 
 struct TableDesc {
@@ -106,6 +107,7 @@ struct GreedySync {
   uint32_t* hitring;         // [kHitSlots][ring_stride] probed hits (row s in slot s % kHitSlots)
   float* tpfring;            // [kHitSlots][ring_stride] T_pf at those hits (kNoTpfBits where it changed)
   uint32_t ring_stride;      // I rounded up to a multiple of 4
+  uint64_t wait_ns;          // bound on any cross-block wait (ns); a waiter that gives up sets kErrTimeout
 };
 
 // Window table from a chain's last block hash to the earliest request ending there.
@@ -115,11 +117,20 @@ struct LastSlot {
   unsigned int pad;
 };
 
+// Instance orders inside T (Table 4), as ps_model.selector.
+enum : int32_t { kSelDCQ = 0, kSelD = 1, kSelDQ = 2, kSelDC = 3, kSelDQC = 4, kSelHCQ = 5 };
+
 struct DevModel {
   float a0, a1, a2, a3, a4, a5, b0, b1, b2, g_q, eta, lout;
   int32_t interference_mode, ttft_filter, nseg;
   int32_t seg_lo[16];
   float ema[16];
+  // policy variants of the evaluation (Table 3 admission ablations, Table 4 selectors); all zero is
+  // Algorithm 1
+  int32_t cache_off;  // 1: C = A (no KVC-first filter)
+  int32_t slo_off;    // 1: T = C (no SLO admission)
+  int32_t fb_dcq;     // 1: with T empty, the D-C-Q order over C instead of the LMetric product
+  int32_t sel;        // order inside T (kSel*)
 };
 
 struct StateSoA {
@@ -598,52 +609,6 @@ __device__ __forceinline__ uint64_t warp_first_miss_search_hint(uint64_t lo, uin
   return warp_search_range(lo2, hi, present);
 }
 
-// --------------------------------------------------------------------- bulk copies (TMA, sm_90+) --
-__device__ __forceinline__ uint32_t smem_u32(const void* p) {
-  return (uint32_t)__cvta_generic_to_shared(p);
-}
-
-__device__ __forceinline__ void mbar_init(uint64_t* mbar, uint32_t count) {
-  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(mbar)), "r"(count) : "memory");
-}
-
-__device__ __forceinline__ void fence_mbar_init() {
-  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-}
-
-__device__ __forceinline__ void fence_proxy_async_smem() {
-  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-}
-
-// Arm the barrier for `bytes` of transaction count (one arrival) and start a global -> shared bulk
-// copy that completes against it.  dst, src 16-byte aligned, bytes a multiple of 16.
-__device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t bytes, uint64_t* mbar) {
-  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(mbar)), "r"(bytes)
-               : "memory");
-  asm volatile(
-      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
-          smem_u32(dst)),
-      "l"(src), "r"(bytes), "r"(smem_u32(mbar))
-      : "memory");
-}
-
-__device__ __forceinline__ bool mbar_try_wait(uint64_t* mbar, uint32_t parity) {
-  uint32_t ok;
-  asm volatile(
-      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}"
-      : "=r"(ok)
-      : "r"(smem_u32(mbar)), "r"(parity)
-      : "memory");
-  return ok != 0;
-}
-
-// Bounded wait for the barrier phase with the given parity; false after max_iter unsuccessful tries.
-__device__ __forceinline__ bool mbar_wait_bounded(uint64_t* mbar, uint32_t parity, uint32_t max_iter) {
-  for (uint32_t it = 0; it < max_iter; ++it)
-    if (mbar_try_wait(mbar, parity)) return true;
-  return false;
-}
-
 // ---------------------------------------------------------------------------- performance model --
 // Every operation is an explicitly rounded fp32 intrinsic in the order the header documents, so
 // nothing is fused or reassociated.
@@ -676,12 +641,16 @@ struct RowConst {
   uint32_t L;
 };
 
+// Z of a row as the recompute filter uses it: without the KVC-first filter (Table 3) every pair of A
+// is in C, which the filter's own rule gives for Z <= 0.
+__device__ __forceinline__ float filter_z(const DevModel& m, float Z) { return m.cache_off ? 0.0f : Z; }
+
 __device__ __forceinline__ RowConst row_const(const DevModel& m, uint32_t L, float ttft_t, float tpot_t) {
   RowConst rc;
   const float Lf = __uint2float_rn(L);
   rc.t_cached = t_pf(m, 0.0f, Lf);
   const float t_cold = t_pf(m, Lf, 0.0f);
-  rc.Z = __fsub_rn(t_cold, rc.t_cached);
+  rc.Z = filter_z(m, __fsub_rn(t_cold, rc.t_cached));
   rc.etaZ = __fmul_rn(m.eta, rc.Z);
   rc.ttft_budget = t_cold > ttft_t ? t_cold : ttft_t;
   rc.tpot_target = tpot_t;
@@ -848,8 +817,10 @@ __device__ __forceinline__ bool pair_in_c(const RowConst& rc, float W, float Wmi
   return (rc.Z > 0.0f) ? (__fsub_rn(W, Wmin) <= rc.etaZ) : true;
 }
 
-// Admission of a pair of C (Algorithm 1 TPOT filter, plus the TTFT budget when enabled).
+// Admission of a pair of C (Algorithm 1 TPOT filter, plus the TTFT budget when enabled; every pair
+// of C without the SLO admission, Table 3).
 __device__ __forceinline__ bool pair_admitted(const DevModel& m, const RowConst& rc, float tpot, float ttft) {
+  if (m.slo_off) return true;
   bool ok = tpot < rc.tpot_target;
   if (m.ttft_filter) ok = ok && (ttft <= rc.ttft_budget);
   return ok;
@@ -868,55 +839,6 @@ __device__ __forceinline__ uint32_t pair_class(const DevModel& m, const RowConst
   return pair_admitted(m, rc, e.tpot, e.ttft) ? 0u : 1u;
 }
 
-// Ordering value inside a class.  Class 0 (Section 6.2, D-C-Q): more decoding requests, then more
-// cached blocks, then fewer queued requests: (2^18-1-b) | (2^26-1-h) | qr in 18/26/18 bits.
-// Class 1 (CacheAwareLB = LMetric): (q + n) * (b + qr + 1) as an unsigned 64-bit product.
-__device__ __forceinline__ uint64_t pair_value(uint32_t cls, uint32_t h, int32_t b, int32_t qr, int64_t q,
-                                               int64_t n) {
-  if (cls == 0u)
-    return ((uint64_t)((1u << 18) - 1u - (uint32_t)b) << 44) |
-           ((uint64_t)((1u << 26) - 1u - h) << 18) | (uint64_t)(uint32_t)qr;
-  return (uint64_t)(q + n) * (uint64_t)((int64_t)b + qr + 1);
-}
-
-// Lexicographic (class, value, instance) argmin element; ci packs class << 28 | instance.
-struct ArgKey {
-  uint32_t ci;
-  uint64_t v;
-};
-
-__device__ __forceinline__ bool key_less(const ArgKey& a, const ArgKey& z) {
-  const uint32_t ca = a.ci >> 28, cz = z.ci >> 28;
-  if (ca != cz) return ca < cz;
-  if (a.v != z.v) return a.v < z.v;
-  return (a.ci & 0x0FFFFFFFu) < (z.ci & 0x0FFFFFFFu);
-}
-
-__device__ __forceinline__ ArgKey warp_argmin(ArgKey k) {
-#pragma unroll
-  for (int s = 16; s > 0; s >>= 1) {
-    ArgKey o;
-    o.ci = __shfl_xor_sync(0xffffffffu, k.ci, s);
-    o.v = __shfl_xor_sync(0xffffffffu, k.v, s);
-    if (key_less(o, k)) k = o;
-  }
-  return k;
-}
-
-__device__ __forceinline__ float warp_fmin(float x) {
-#pragma unroll
-  for (int s = 16; s > 0; s >>= 1) x = fminf(x, __shfl_xor_sync(0xffffffffu, x, s));
-  return x;
-}
-
-constexpr uint32_t kNoKeyCi = 0xFFFFFFFFu;  // class 15: worse than any real pair
-
-// (class, value) of a pair of C as one 64-bit key, class in the top two bits: class-0 values are
-// below 2^62 and class-1 values below 2^59 ((q + n) < 2^41 times (b + qr + 1) < 2^18), so the
-// unsigned order of the packed key is the lexicographic order of (class, value).
-__device__ __forceinline__ uint64_t packed_key(uint32_t cls, uint64_t v) { return ((uint64_t)cls << 62) | v; }
-constexpr uint64_t kNoKey = ~0ull;
-
 // Order-preserving map of a non-NaN float to an unsigned integer (for integer warp reductions).
 __device__ __forceinline__ uint32_t f2ord(float x) {
   const uint32_t u = __float_as_uint(x);
@@ -925,6 +847,74 @@ __device__ __forceinline__ uint32_t f2ord(float x) {
 __device__ __forceinline__ float ord2f(uint32_t o) {
   return __uint_as_float((o & 0x80000000u) ? (o & 0x7FFFFFFFu) : ~o);
 }
+
+// ---- packing keys under the policy variants ---------------------------------------------------
+// Class-0 value fields: D = 2^18-1-b (18 bits), C = 2^26-1-h (26 bits), Q = qr (18 bits), so a
+// smaller value means more decoding requests, more cached blocks, fewer queued requests.
+//   D-C-Q  D << 44 | C << 18 | Q        D    D << 44             D-Q  D << 44 | Q
+//   D-C    D << 44 | C << 18            D-Q-C  D << 44 | Q << 26 | C
+//   H-C-Q  ord(tpot_target - TPOT) << 26 | C, with Q carried in the tie word (qr << 12 | instance)
+// The instance-only fields (D, Q) are kept per instance (key0_bits); a pair adds its hit field.
+__device__ __forceinline__ uint64_t dcq_key0(int32_t b, int32_t qr) {
+  return ((uint64_t)((1u << 18) - 1u - (uint32_t)b) << 44) | (uint64_t)(uint32_t)qr;
+}
+
+__device__ __forceinline__ uint64_t key0_bits(const DevModel& m, int32_t b, int32_t qr) {
+  const uint64_t D = (uint64_t)((1u << 18) - 1u - (uint32_t)b) << 44;
+  switch (m.sel) {
+    case kSelDCQ:
+    case kSelDQ: return D | (uint64_t)(uint32_t)qr;
+    case kSelDQC: return D | ((uint64_t)(uint32_t)qr << 26);
+    case kSelHCQ: return 0ull;
+    default: return D;
+  }
+}
+
+__device__ __forceinline__ uint64_t hit_bits(const DevModel& m, uint32_t h) {
+  const uint64_t C = (uint64_t)((1u << 26) - 1u - h);
+  if (m.sel == kSelDCQ || m.sel == kSelDC) return C << 18;
+  if (m.sel == kSelDQC || m.sel == kSelHCQ) return C;
+  return 0ull;
+}
+
+// key0_bits from the D-C-Q bits of (b, qr) (dcq_key0), which is what kernels keep per instance.
+__device__ __forceinline__ uint64_t key0_from_dcq(const DevModel& m, uint64_t kd) {
+  if (m.sel == kSelDCQ) return kd;
+  return key0_bits(m, (int32_t)((1u << 18) - 1u - (uint32_t)(kd >> 44)), (int32_t)(kd & 0x3FFFFull));
+}
+
+// Value of a pair of T (class 0) from its instance's key0_bits, hit and predicted TPOT.
+__device__ __forceinline__ uint64_t value_in_t(const DevModel& m, uint64_t k0, uint32_t h, float tpot, float target) {
+  uint64_t v = k0 | hit_bits(m, h);
+  if (m.sel == kSelHCQ) v |= (uint64_t)f2ord(__fsub_rn(target, tpot)) << 26;
+  return v;
+}
+
+// Tie word of a pair of T: the instance id, or qr << 12 | id under H-C-Q (ids < 4096).
+__device__ __forceinline__ uint32_t tie_in_t(const DevModel& m, uint32_t i, int32_t qr) {
+  return m.sel == kSelHCQ ? (((uint32_t)qr << 12) | i) : i;
+}
+constexpr uint32_t kTieInstMask = 0xFFFu;
+
+// Value of a pair of C \ T (class 1): the LMetric product (q + n)(b + qr + 1), or the D-C-Q value
+// under the ablations' D-C-Q fallback (kd = dcq_key0(b, qr)).
+__device__ __forceinline__ uint64_t value_fallback(const DevModel& m, uint64_t qn, uint32_t Bp, uint64_t kd,
+                                                   uint32_t h) {
+  if (m.fb_dcq) return kd | ((uint64_t)((1u << 26) - 1u - h) << 18);
+  return qn * (uint64_t)Bp;
+}
+
+__device__ __forceinline__ float warp_fmin(float x) {
+#pragma unroll
+  for (int s = 16; s > 0; s >>= 1) x = fminf(x, __shfl_xor_sync(0xffffffffu, x, s));
+  return x;
+}
+
+// (class, value) of a pair of C as one 64-bit key, class in the top two bits: class-0 values are
+// below 2^62 and class-1 values below 2^59 ((q + n) < 2^41 times (b + qr + 1) < 2^18), so the
+// unsigned order of the packed key is the lexicographic order of (class, value).
+__device__ __forceinline__ uint64_t packed_key(uint32_t cls, uint64_t v) { return ((uint64_t)cls << 62) | v; }
+constexpr uint64_t kNoKey = ~0ull;
 
 // Warp argmin of (key, instance) with single-instruction reductions; every lane receives the
 // minimum and the winning lane's h.  Lanes without a pair pass (kNoKey, 0xFFFFFFFF).

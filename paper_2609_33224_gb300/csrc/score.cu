@@ -10,8 +10,9 @@
 // chunk.  Pass 1 evaluates the capacity guard and the recompute cost W (Alg. 1 KVC-first filtering)
 // and reduces W_min over A; pass 2 classifies each pair (Eq. 8 filter, TPOT and TTFT admission)
 // and reduces the packed (class, value) key to the pick: D-C-Q inside T, the LMetric product inside
-// C when T is empty, Reject when A is empty.  Pass 2 takes the hits from registers; rows of more
-// than 128 NV instances are taken in pieces of NV chunks, each read again for pass 2.
+// C when T is empty, Reject when A is empty (or the model's policy variant of Table 3 / Table 4).
+// Pass 2 takes the hits from registers; rows of more than 128 NV instances are taken in pieces of
+// NV chunks, each read again for pass 2.
 #include "ps_internal.cuh"
 
 namespace {
@@ -24,7 +25,7 @@ constexpr int kScoreThreads = 256;
 struct ScoreSmem {
   int64_t* q;
   int64_t* S;
-  uint64_t* k0;    // class-0 key bits of (b, qr)
+  uint64_t* k0;    // D-C-Q key bits of (b, qr) (psk::dcq_key0; other orders derive theirs)
   int32_t* room;   // free KV room M_KV - S, -1 when the decode-slot guard fails or past I
   float* dec0;
   float* f;
@@ -139,7 +140,7 @@ __device__ __forceinline__ void piece_pass2(uint32_t I, uint32_t i_lo, uint64_t 
                                             const psk::DevModel& m, const psk::RowConst& rc, float wmin,
                                             const Piece<NV>& p, float* __restrict__ tpot_out,
                                             float* __restrict__ ttft_out, uint8_t* __restrict__ cls_out,
-                                            uint64_t& bkey, uint32_t& binst, uint32_t& bh) {
+                                            uint64_t& bkey, uint32_t& btie, uint32_t& bh) {
   const int lane = threadIdx.x & 31;
   const bool all_pairs = tpot_out || ttft_out || cls_out;
 #pragma unroll
@@ -202,12 +203,19 @@ __device__ __forceinline__ void piece_pass2(uint32_t I, uint32_t i_lo, uint64_t 
       cw |= cls << (8 * k);
       if (cls <= 1u) {
         const uint64_t qn = NARROW ? (uint64_t)(uint32_t)(q32[k] + n) : (uint64_t)q[k] + (uint64_t)(int64_t)n;
-        const uint64_t key = cls == 0u ? psk::packed_key(0u, k0[k] | ((uint64_t)((1u << 26) - 1u - p.h[v][k]) << 18))
-                                       : psk::packed_key(1u, qn * (uint64_t)(uint32_t)Bp[k]);
-        if (key < bkey) {  // a lane's instances ascend, so ties keep the lowest
+        const uint32_t h = p.h[v][k];
+        uint64_t key;
+        uint32_t tie = i + k;
+        if (cls == 0u) {
+          key = psk::packed_key(0u, psk::value_in_t(m, psk::key0_from_dcq(m, k0[k]), h, tp[k], rc.tpot_target));
+          if (m.sel == psk::kSelHCQ) tie |= (uint32_t)(k0[k] & 0x3FFFFull) << 12;
+        } else {
+          key = psk::packed_key(1u, psk::value_fallback(m, qn, (uint32_t)Bp[k], k0[k], h));
+        }
+        if (key < bkey || (key == bkey && tie < btie)) {
           bkey = key;
-          binst = i + k;
-          bh = p.h[v][k];
+          btie = tie;
+          bh = h;
         }
       }
     }
@@ -246,7 +254,7 @@ score_rows_kernel(const uint32_t* __restrict__ hits, psk::StateSoA st, uint32_t 
       const psk::InstTerms it = psk::inst_terms(m, b, qr, q, Bmax);
       s.q[i] = q;
       s.S[i] = S;
-      s.k0[i] = ((uint64_t)((1u << 18) - 1u - (uint32_t)b) << 44) | (uint64_t)(uint32_t)qr;
+      s.k0[i] = psk::dcq_key0(b, qr);
       s.room[i] = it.okB ? psk::kv_room(S, M) : -1;
       s.dec0[i] = it.dec0;
       s.f[i] = it.f;
@@ -287,27 +295,27 @@ score_rows_kernel(const uint32_t* __restrict__ hits, psk::StateSoA st, uint32_t 
     const bool anyA = wbest != 0xFFFFFFFFu;  // a W of a pair in A is never NaN, so never all ones
     const float wmin = psk::ord2f(wbest);
     uint64_t bkey = psk::kNoKey;
-    uint32_t binst = 0xFFFFFFFFu, bh = 0u;
+    uint32_t btie = 0xFFFFFFFFu, bh = 0u;
     if (one_piece) {
       if (narrow)
-        piece_pass2<NV, VEC, true>(I, 0u, x0, s, m, rc, wmin, p, tpot_out, ttft_out, cls_out, bkey, binst, bh);
+        piece_pass2<NV, VEC, true>(I, 0u, x0, s, m, rc, wmin, p, tpot_out, ttft_out, cls_out, bkey, btie, bh);
       else
-        piece_pass2<NV, VEC, false>(I, 0u, x0, s, m, rc, wmin, p, tpot_out, ttft_out, cls_out, bkey, binst, bh);
+        piece_pass2<NV, VEC, false>(I, 0u, x0, s, m, rc, wmin, p, tpot_out, ttft_out, cls_out, bkey, btie, bh);
     } else {
       for (uint32_t lo = 0; lo < I; lo += kPiece) {
         piece_pass1<NV, VEC>(hrow, I, lo, s, m, rc, p);
         if (narrow)
-          piece_pass2<NV, VEC, true>(I, lo, x0, s, m, rc, wmin, p, tpot_out, ttft_out, cls_out, bkey, binst, bh);
+          piece_pass2<NV, VEC, true>(I, lo, x0, s, m, rc, wmin, p, tpot_out, ttft_out, cls_out, bkey, btie, bh);
         else
-          piece_pass2<NV, VEC, false>(I, lo, x0, s, m, rc, wmin, p, tpot_out, ttft_out, cls_out, bkey, binst, bh);
+          piece_pass2<NV, VEC, false>(I, lo, x0, s, m, rc, wmin, p, tpot_out, ttft_out, cls_out, bkey, btie, bh);
       }
     }
     uint64_t key;
-    uint32_t j, hj;
-    psk::warp_pick_min(bkey, binst, bh, &key, &j, &hj);
+    uint32_t tie, hj;
+    psk::warp_pick_min(bkey, btie, bh, &key, &tie, &hj);
     if (lane == 0) {
       const bool pick = anyA && key != psk::kNoKey;
-      if (best_out) best_out[r] = pick ? (int32_t)j : -1;
+      if (best_out) best_out[r] = pick ? (int32_t)(tie & psk::kTieInstMask) : -1;
       if (path_out) path_out[r] = pick ? (uint8_t)(key >> 62) : (uint8_t)2;
     }
   }

@@ -53,6 +53,7 @@ int main(void) {
   O(ps_config, model) O(ps_config, table_load_factor) O(ps_config, cap_blocks)
   O(ps_model, seg_lo) O(ps_model, ema_factor) O(ps_instance_state, B_max)
   O(ps_window, inputs_on_device) O(ps_scores, outputs_on_device) O(ps_decisions, outputs_on_device)
+  O(ps_model, cache_filter_off) O(ps_model, selector)
   return 0;
 }
 """)
@@ -91,3 +92,28 @@ def test_graft_entry_build_runs_on_cpu():
     import __graft_entry__ as g
     g.build()
     assert os.path.exists(P._LIB_PATH)
+
+
+def test_every_declared_call_names_its_passage():
+    """Each exported call's comment block (the text between the previous declaration and this one)
+    names the passage of the paper that defines the operation (a section, equation, algorithm or
+    table), or says that the paper has no counterpart."""
+    cite = re.compile(r"Section \d|Eq\. ?\d|Algorithm \d|Table \d|no counterpart")
+    for h in glob.glob(os.path.join(ROOT, "include", "*.h")):
+        src = open(h).read()
+        prev = 0
+        for mt in re.finditer(r"^PS_API\s+[\w\s\*]+?\b(ps_\w+)\s*\([^;]*;", src, flags=re.M | re.S):
+            block = src[prev:mt.start()]
+            assert cite.search(block), f"{mt.group(1)}: its comment names no section, equation, algorithm or table"
+            prev = mt.end()
+
+
+def test_policy_switches_default_to_algorithm_1():
+    """A zero-initialised ps_model's policy fields select Algorithm 1: KVC-first filter and SLO
+    admission on, the LMetric fallback, the D-C-Q order; the binding's tables name Table 3 / Table 4."""
+    m = P.PsModel()
+    assert (m.cache_filter_off, m.slo_filter_off, m.fallback_dcq, m.selector) == (0, 0, 0, 0)
+    assert P.SELECTORS["D-C-Q"] == 0 and sorted(P.SELECTORS.values()) == list(range(6))
+    assert P.ABLATIONS["F"] == dict(cache_filter_off=0, slo_filter_off=0, fallback_dcq=0)
+    g = P.make_model(dict(__import__("workload").MODEL_DEFAULT, **P.ABLATIONS["G"], selector=5))
+    assert (g.cache_filter_off, g.slo_filter_off, g.fallback_dcq, g.selector) == (1, 1, 1, 5)
