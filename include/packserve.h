@@ -375,6 +375,9 @@ PS_API ps_status ps_last_timings(ps_ctx* ctx, float* ms, uint32_t n);
  *   out[2] table lookups in scratch rows     out[3] table lookups in derived rows
  *   out[4] chain blocks read from global memory (a lookup's key, or a block staged in shared memory)
  *   out[5] (row, instance) pairs searched past the earlier request's chain (derived rows)
+ * With n >= 8, of the last ps_schedule_window in PS_PROBE_SEARCH mode (else 0):
+ *   out[6] decisions taken from a row summary corrected for the recent picks
+ *   out[7] decisions that needed a full pass over the row
  * A table lookup reads the key's two candidate buckets (2 x 64 bytes) and one overflow word.
  * All zero if no probe phase ran.  Synchronises the context's stream. */
 PS_API ps_status ps_last_probe_stats(ps_ctx* ctx, uint64_t* out, uint32_t n);

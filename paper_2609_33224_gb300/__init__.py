@@ -338,10 +338,10 @@ class Scheduler:
 
     def probe_stats(self) -> dict:
         """Counters of the last probe phase (see ps_last_probe_stats)."""
-        v = np.zeros(6, np.uint64)
-        self._check(lib().ps_last_probe_stats(self._h, v.ctypes.data, 6))
+        v = np.zeros(8, np.uint64)
+        self._check(lib().ps_last_probe_stats(self._h, v.ctypes.data, 8))
         names = ("rows_scratch", "rows_derived", "lookups_scratch", "lookups_derived", "chain_reads",
-                 "pairs_derived")
+                 "pairs_derived", "greedy_fast", "greedy_full")
         return dict(zip(names, (int(x) for x in v)))
 
     # ------------------------------------------------------------------------------------------

@@ -57,7 +57,7 @@ struct ps_ctx {
   unsigned long long* d_count = nullptr;
   psk::DeltaSlot* d_delta = nullptr;
   uint64_t delta_nslots = 0;
-  psk::GreedySync gsync{nullptr, nullptr, nullptr, nullptr, nullptr, 0u, kDefaultWaitNs};
+  psk::GreedySync gsync{nullptr, nullptr, nullptr, nullptr, nullptr, 0u, kDefaultWaitNs, nullptr, nullptr, nullptr};
   psk::RowPre* d_rows = nullptr;      // per-request constants and relations (search mode greedy)
   psk::LastSlot* d_lastslot = nullptr;
   psk::RowList scratch{nullptr, nullptr};  // rows the probe searches from scratch
@@ -400,6 +400,8 @@ ps_status ps_create(const ps_config* cfg, ps_ctx** out) {
             dalloc(c, &c->d_tdesc, I) == cudaSuccess && dalloc(c, &c->d_count, I) == cudaSuccess &&
             dalloc(c, &c->d_delta, (size_t)dn) == cudaSuccess && dalloc(c, &c->gsync.jobs, c->Rmax) == cudaSuccess &&
             dalloc(c, &c->gsync.done, c->Rmax) == cudaSuccess && dalloc(c, &c->gsync.ready, c->Rmax) == cudaSuccess &&
+            dalloc(c, &c->gsync.sums, psk::kSumSlots) == cudaSuccess && dalloc(c, &c->gsync.sready, c->Rmax) == cudaSuccess &&
+            dalloc(c, &c->gsync.stats, 2) == cudaSuccess &&
             dalloc(c, &c->gsync.hitring, (size_t)psk::kHitSlots * c->gsync.ring_stride) == cudaSuccess &&
             dalloc(c, &c->gsync.tpfring, (size_t)psk::kHitSlots * c->gsync.ring_stride) == cudaSuccess &&
             dalloc(c, &c->d_rows, c->Rmax) == cudaSuccess && dalloc(c, &c->d_lastslot, c->lastslot_n) == cudaSuccess &&
@@ -827,11 +829,16 @@ ps_status ps_last_probe_stats(ps_ctx* c, uint64_t* out, uint32_t n) {
   if (!out || n < (uint32_t)kNumStats) return fail(c, PS_ERR_INVALID, "need 6 entries");
   DeviceGuard g(c->device);
   unsigned long long v[kNumStats] = {};
-  if (c->ev_used[0]) {
-    PS_TRY_CUDA(c, cudaMemcpyAsync(v, c->d_stats, sizeof(v), cudaMemcpyDeviceToHost, c->stream));
-    PS_TRY_CUDA(c, cudaStreamSynchronize(c->stream));
-  }
+  unsigned long long gs[2] = {};
+  if (c->ev_used[0]) PS_TRY_CUDA(c, cudaMemcpyAsync(v, c->d_stats, sizeof(v), cudaMemcpyDeviceToHost, c->stream));
+  if (c->ev_used[2] && c->search && n >= 8)
+    PS_TRY_CUDA(c, cudaMemcpyAsync(gs, c->gsync.stats, sizeof(gs), cudaMemcpyDeviceToHost, c->stream));
+  PS_TRY_CUDA(c, cudaStreamSynchronize(c->stream));
   for (int k = 0; k < kNumStats; ++k) out[k] = v[k];
+  if (n >= 8) {
+    out[6] = gs[0];
+    out[7] = gs[1];
+  }
   return PS_OK;
 }
 

@@ -293,7 +293,7 @@ cudaError_t greedy_launch(const uint64_t* slots, const uint64_t* ovf, const psk:
 
 
 // ----------------------------------------------------------------------------------------------
-// Prefix-closed caches (the probe's search mode): a pipelined greedy pass over three kinds of
+// Prefix-closed caches (the probe's search mode): a pipelined greedy pass over four kinds of
 // thread block in one cooperative launch.
 //
 // On a prefix-closed cache the hit of a request is the first chain position not cached, and the
@@ -305,14 +305,13 @@ cudaError_t greedy_launch(const uint64_t* slots, const uint64_t* ovf, const psk:
 // where delta_i(<= s - kLag) holds the blocks inserted for requests up to s - kLag and lcp(s, s - d) is
 // the common chain prefix (from the relations pass).
 //
-//   Deciding block (block 0).  Per request r: reads row r's probed hits (first term above) from a
-//   shared-memory ring that was filled by asynchronous copies two steps earlier, raises the hits of
-//   the instances that took requests r - 1 .. r - kLag + 1 to the common prefix, evaluates the row
-//   (capacity guard and W, block reduction to W_min; recompute filter, latencies, admission class
-//   and key of the pairs in C, block reduction to the pick), updates the pick's state and publishes
-//   the decision as an insert job.  No table access is on its per-request path.
-//   Insert blocks.  Take the jobs round-robin (up to kInsertBlocks in flight), insert each job's
-//   chain blocks chain[h, nb) into delta_j and release the job's done flag.
+//   Deciding block (block 0).  A feeder warp stages each row's summary, row constants and probed
+//   hits in shared memory; the deciding warp decides the requests in arrival order from the
+//   summaries, correcting them for the last kSpecLag picks (the lag-d speculation below), updates
+//   the pick's state and publishes each decision as an insert job.  No table access is on its
+//   per-request path.
+//   Insert blocks.  Groups of kInsertGroup blocks take the jobs round-robin; a group's members split
+//   each job's chain blocks chain[h, nb) between them, insert them into delta_j and count the job done.
 //   Probe blocks.  Take the rows round-robin.  For row s they wait until the jobs <= s - kLag are
 //   done, replay those jobs (which instances have window inserts, where their last chain ended,
 //   which instances took s's ancestors), then per instance start from hit0, raise the position to
@@ -323,13 +322,17 @@ cudaError_t greedy_launch(const uint64_t* slots, const uint64_t* ovf, const psk:
 //   prefix-closed main table.  Inserts of requests s - kLag + 1 .. s - 1 may land while a probe
 //   runs, in any order: any snapshot between delta(<= s - kLag) and delta(<= s - 1) gives a first
 //   miss between the two sets' first misses, and the max with the lcp terms is exact all the same.
+//   Summary blocks.  Take the rows round-robin; evaluate row s on every instance against the state
+//   before decision s - kSpecLag and publish its summary (below).
 // Every cross-block wait is bounded (GreedySync::wait_ns, 1 s unless the caller set another limit);
-// on expiry the waiter records PS_ERR_TIMEOUT and stops waiting, so the launch always ends.  Instance state lives in the deciding block's shared
-// memory and is written only by the thread that owns the instance.
+// on expiry the waiter records PS_ERR_TIMEOUT and stops waiting, so the launch always ends.  Each
+// role keeps the instance state it needs in its own shared memory.
 
-constexpr uint32_t kInsertBlocks = 8;         // insert blocks
-constexpr uint32_t kProbeBlocks = 16;         // probe blocks
-constexpr uint32_t kRingAhead = 6;            // row constants are copied into the ring this many rows ahead
+constexpr uint32_t kInsertBlocks = 16;   // insert blocks
+constexpr uint32_t kProbeBlocks = 16;    // probe blocks
+constexpr uint32_t kSummaryBlocks = 32;  // summary blocks (lag-d speculation, below)
+constexpr uint32_t kPipeThreads = 256;   // threads of every block of the launch
+constexpr uint32_t kFeedRing = 4;        // rows staged in the deciding block's shared memory
 constexpr unsigned long long kJobValid = 1ull << 63;  // a published job word (0 = not yet published)
 
 __device__ __forceinline__ psk::RowConst row_of(const psk::RowPre& x) {
@@ -348,6 +351,20 @@ __device__ __forceinline__ bool wait_flag(const uint32_t* flag, uint32_t* err, u
   if (psk::ld_acquire_u32(flag) != 0u) return true;
   const uint64_t t0 = psk::globaltimer_ns();
   while (psk::ld_acquire_u32(flag) == 0u) {
+    if (psk::globaltimer_ns() - t0 > limit_ns) {
+      atomicOr(err, psk::kErrTimeout);
+      return false;
+    }
+    __nanosleep(32);
+  }
+  return true;
+}
+
+// Bounded spin until *count >= want (acquire).  false after limit_ns (and the error bit is set).
+__device__ __forceinline__ bool wait_count(const uint32_t* count, uint32_t want, uint32_t* err, uint64_t limit_ns) {
+  if (psk::ld_acquire_u32(count) >= want) return true;
+  const uint64_t t0 = psk::globaltimer_ns();
+  while (psk::ld_acquire_u32(count) < want) {
     if (psk::globaltimer_ns() - t0 > limit_ns) {
       atomicOr(err, psk::kErrTimeout);
       return false;
@@ -377,13 +394,55 @@ __device__ __forceinline__ unsigned long long wait_job(const unsigned long long*
 __device__ __forceinline__ uint32_t job_pick(unsigned long long jb) { return (uint32_t)jb; }
 __device__ __forceinline__ uint32_t job_hit(unsigned long long jb) { return (uint32_t)(jb >> 32) & 0x7FFFFFFFu; }
 
-// Insert blocks: block b inserts the chain tails of jobs b - 1, b - 1 + kInsertBlocks, ... and
-// releases each job's done flag once all its blocks are in.
+// Insert blocks, in groups of kInsertGroup: group g inserts the chain tails of jobs g, g + the number
+// of groups, ...; the group's members split a tail by position (member m takes positions
+// h + m * 256 + t, stride kInsertGroup * 256) and each adds 1 to the job's done count once its
+// inserts are in, so the job's blocks are all in when the count reaches kInsertGroup.  A thread
+// claims the home slots of kInsertBatch keys at once (the claims are independent) and follows the
+// rare occupied home slot on its own.
+constexpr uint32_t kInsertGroup = 4;
+constexpr int kInsertBatch = 4;
+static_assert(kInsertBlocks % kInsertGroup == 0, "whole insert groups");
+
+__device__ __forceinline__ void insert_tail(psk::DeltaSlot* delta, uint64_t nslots, uint32_t j,
+                                            const uint64_t* __restrict__ chain, uint64_t first, uint64_t nb,
+                                            uint64_t stride, uint32_t* err) {
+  for (uint64_t p0 = first; p0 < nb; p0 += kInsertBatch * stride) {
+    uint64_t key[kInsertBatch], slot[kInsertBatch];
+    unsigned long long old[kInsertBatch];
+#pragma unroll
+    for (int q = 0; q < kInsertBatch; ++q) {
+      const uint64_t p = p0 + (uint64_t)q * stride;
+      key[q] = p < nb ? __ldg(chain + p) : psk::kEmpty;
+    }
+#pragma unroll
+    for (int q = 0; q < kInsertBatch; ++q) {
+      old[q] = ~0ull;
+      if (key[q] != psk::kEmpty && key[q] != psk::kTomb) {
+        slot[q] = psk::delta_home(key[q], nslots);
+        old[q] = atomicCAS(&delta[slot[q]].hash, psk::kEmpty, (unsigned long long)key[q]);
+      }
+    }
+#pragma unroll
+    for (int q = 0; q < kInsertBatch; ++q) {
+      if (key[q] == psk::kEmpty || key[q] == psk::kTomb) continue;
+      if (old[q] == psk::kEmpty) {
+        __stcg(&delta[slot[q]].tag, j + 1);
+      } else if (!psk::delta_insert_from(delta, nslots, j, key[q], psk::delta_next(slot[q], nslots))) {
+        atomicOr(err, psk::kErrDeltaFull);
+      }
+    }
+  }
+}
+
 __device__ void insert_blocks(const psk::RowPre* __restrict__ rows, const uint64_t* __restrict__ hash, uint32_t R,
                               psk::DeltaSlot* delta, uint64_t nslots, uint32_t* err, const psk::GreedySync& sync) {
   __shared__ unsigned long long s_job;
   const uint32_t t = threadIdx.x;
-  for (uint32_t job = blockIdx.x - 1; job < R; job += kInsertBlocks) {
+  const uint32_t ib = blockIdx.x - 1;
+  const uint32_t group = ib / kInsertGroup, member = ib % kInsertGroup;
+  constexpr uint32_t kGroups = kInsertBlocks / kInsertGroup;
+  for (uint32_t job = group; job < R; job += kGroups) {
     if (t == 0) s_job = wait_job(sync.jobs + job, err, sync.wait_ns);
     __syncthreads();
     const unsigned long long jb = s_job;
@@ -394,13 +453,13 @@ __device__ void insert_blocks(const psk::RowPre* __restrict__ rows, const uint64
     if (j != 0xFFFFFFFFu && job + psk::kLag < R) {
       const uint64_t off = __ldg(&rows[job].off);
       const uint32_t nb = __ldg(&rows[job].nb);
-      for (uint64_t p = hj + t; p < nb; p += blockDim.x)
-        if (!psk::delta_insert(delta, nslots, j, __ldg(hash + off + p))) atomicOr(err, psk::kErrDeltaFull);
+      insert_tail(delta, nslots, j, hash + off, (uint64_t)hj + member * blockDim.x + t, nb,
+                  (uint64_t)kInsertGroup * blockDim.x, err);
     }
     __syncthreads();
     if (t == 0) {
-      __threadfence();  // every thread's inserts before the flag
-      psk::st_release_u32(sync.done + job, 1u);
+      __threadfence();  // every thread's inserts before the count
+      atomicAdd(sync.done + job, 1u);
     }
   }
 }
@@ -508,12 +567,12 @@ __device__ void probe_rows(const psk::RowPre* __restrict__ rows, const uint64_t*
       bool abort = false;
       while ((int64_t)f < need && !abort) {
         const uint32_t x = f + (uint32_t)lane;
-        const bool ok = (int64_t)x < need && psk::ld_acquire_u32(sync.done + x) != 0u;
+        const bool ok = (int64_t)x < need && psk::ld_acquire_u32(sync.done + x) >= kInsertGroup;
         const unsigned okm = __ballot_sync(0xffffffffu, ok);
         const uint32_t nok = (okm == 0xffffffffu) ? 32u : (uint32_t)(__ffs(~okm) - 1);
         if (nok == 0u) {
           bool got = true;
-          if (lane == 0) got = wait_flag(sync.done + f, err, sync.wait_ns);
+          if (lane == 0) got = wait_count(sync.done + f, kInsertGroup, err, sync.wait_ns);
           abort = !__shfl_sync(0xffffffffu, got, 0);
           continue;
         }
@@ -566,340 +625,731 @@ __device__ void probe_rows(const psk::RowPre* __restrict__ rows, const uint64_t*
   }
 }
 
-// Deciding block.  Thread t < NTI owns instances t * IPT .. t * IPT + IPT - 1; thread 0 publishes
-// the decisions.  The last warp only waits for the probe blocks' ready flags (thread NTI): an
-// acquire load holds up its thread's later memory accesses, so that warp does nothing else.  Block
-// reductions: each instance warp reduces its lanes with single-instruction warp reductions, writes
-// one partial, and after the barrier every instance warp reduces the partials itself.
-// Instance state is kept as padded structure-of-arrays in shared memory, so a thread reads its IPT
-// consecutive instances' values of one field with one vector load; the capacity guard is one
-// compare against the free KV room, stored as -1 where the decode-slot guard fails.
-template <int N>
-__device__ __forceinline__ void ld_u32v(const void* p, uint32_t (&v)[N]) {
-  static_assert(N == 1 || N == 2 || N == 4, "vector of 1, 2 or 4");
-  if (N == 1) {
-    v[0] = *reinterpret_cast<const uint32_t*>(p);
-  } else if (N == 2) {
-    const uint2 x = *reinterpret_cast<const uint2*>(p);
-    v[0] = x.x;
-    v[N > 1 ? 1 : 0] = x.y;
-  } else {
-    const uint4 x = *reinterpret_cast<const uint4*>(p);
-    v[0] = x.x;
-    v[N > 1 ? 1 : 0] = x.y;
-    v[N > 2 ? 2 : 0] = x.z;
-    v[N > 3 ? 3 : 0] = x.w;
-  }
-}
-
-template <int N>
-__device__ __forceinline__ void st_zero_u32v(void* p) {
-  if (N == 1) *reinterpret_cast<uint32_t*>(p) = 0u;
-  else if (N == 2) *reinterpret_cast<uint2*>(p) = make_uint2(0u, 0u);
-  else *reinterpret_cast<uint4*>(p) = make_uint4(0u, 0u, 0u, 0u);
-}
-
-template <int N>
-__device__ __forceinline__ void ld_u64v(const void* p, uint64_t (&v)[N]) {
-  if (N == 1) {
-    v[0] = *reinterpret_cast<const unsigned long long*>(p);
-  } else {
-#pragma unroll
-    for (int k = 0; k < N; k += 2) {
-      const ulonglong2 x = reinterpret_cast<const ulonglong2*>(p)[k / 2];
-      v[k] = x.x;
-      v[k + 1 < N ? k + 1 : k] = x.y;
-    }
-  }
-}
-
 // q and S within [0, 2^30): with L, n < 2^30 the sums S + L and q + n are exact in 32 bits.
 __device__ __forceinline__ bool narrow_qs(int64_t q, int64_t S) {
   return q >= 0 && q < (1ll << 30) && S >= 0 && S < (1ll << 30);
 }
 
+// ---- lag-d speculation: summary blocks and the deciding warp ------------------------------------
+//
+// Row s's decision depends on the state left by decisions 0 .. s - 1.  Summary blocks evaluate row s
+// on every instance against the state before decision s - kSpecLag (replaying the published jobs
+// into their own copy of the state), and publish per warp the kKeysPerWarp smallest (packed key, tie)
+// pairs of C with their W and hit, and the kWPerWarp smallest W of A, with the bounds of what they
+// did not publish (RowSummary).  Only the instances picked by decisions s - kSpecLag .. s - 1 (the
+// touched ones) have changed since: their state, and their caches (each touched instance's hit on
+// row s rises to the common prefix with the requests it took).  Every other instance keeps its
+// capacity test, W and key.  So the deciding warp re-evaluates the touched instances only, and:
+//   * W_min over A is the smaller of the touched instances' W and the smallest published W of an
+//     untouched instance, known exactly when that W lies at or below the W bound;
+//   * in-window inserts only lengthen hits, so W_min can only fall unless an instance leaves A; if
+//     it rose above the summary's W_min, the summary's C may miss members (full pass);
+//   * with W_min at or below the summary's, C of the current state holds no untouched pair outside
+//     the summary's C, and a published untouched pair stays in C when W - W_min <= eta Z still holds;
+//   * the pick is the smallest (key, tie) over the surviving published pairs and the touched pairs
+//     in C; every unpublished pair has (key, tie) >= the key bound, so a pick below the bound is
+//     exact.
+// Otherwise (W_min unknown or risen, or no pick below the bound) the warp evaluates the whole row on
+// the current state.  Both ways give Algorithm 1's decision exactly.
+//
+// Deciding block: warp 0 decides, warp 1 (the feeder) copies each row's summary, row constants, hits
+// and T_pf into a shared-memory ring as soon as the summary is published; the two hand off through
+// shared-memory counters (the feeder's row count, the decider's consumed count), each wait bounded.
+
+static_assert(kPipeThreads == 32 * psk::kSumWarps, "a summary block is kSumWarps warps");
+
+// Instance state of the summary blocks and the deciding warp: padded structure-of-arrays in shared
+// memory, [Ip] each, 8-byte arrays first (64 bytes per instance).
+struct InstSmem {
+  int64_t* q;
+  int64_t* S;
+  int64_t* M;
+  uint64_t* kd;   // D-C-Q key bits of (b, qr) (psk::dcq_key0)
+  int32_t* room;  // free KV room, -1 when the decode-slot guard fails
+  float* dec0;
+  float* f;
+  float* tq;
+  int32_t* Bp;
+  int32_t* b;
+  int32_t* qr;
+  int32_t* Bmax;
+};
+constexpr size_t kInstSmemBytes = 4 * sizeof(int64_t) + 8 * sizeof(int32_t);
+
+__device__ __forceinline__ InstSmem inst_smem(unsigned long long* raw, uint32_t Ip) {
+  InstSmem a;
+  a.q = reinterpret_cast<int64_t*>(raw);
+  a.S = a.q + Ip;
+  a.M = a.S + Ip;
+  a.kd = reinterpret_cast<uint64_t*>(a.M + Ip);
+  a.room = reinterpret_cast<int32_t*>(a.kd + Ip);
+  a.dec0 = reinterpret_cast<float*>(a.room + Ip);
+  a.f = a.dec0 + Ip;
+  a.tq = a.f + Ip;
+  a.Bp = reinterpret_cast<int32_t*>(a.tq + Ip);
+  a.b = a.Bp + Ip;
+  a.qr = a.b + Ip;
+  a.Bmax = a.qr + Ip;
+  return a;
+}
+
+// Derived terms of instance i after a state change (the decode-slot guard folded into the KV room).
+__device__ __forceinline__ void inst_refresh(const InstSmem& a, const psk::DevModel& m, uint32_t i) {
+  const psk::InstTerms it = psk::inst_terms(m, a.b[i], a.qr[i], a.q[i], a.Bmax[i]);
+  a.dec0[i] = it.dec0;
+  a.f[i] = it.f;
+  a.tq[i] = it.tq;
+  a.Bp[i] = it.Bp;
+  a.room[i] = it.okB ? psk::kv_room(a.S[i], a.M[i]) : -1;
+  a.kd[i] = psk::dcq_key0(a.b[i], a.qr[i]);
+}
+
+__device__ __forceinline__ void inst_load(const InstSmem& a, const psk::StateSoA& st, const psk::DevModel& m,
+                                          uint32_t i) {
+  a.b[i] = st.b[i];
+  a.qr[i] = st.qr[i];
+  a.q[i] = st.q[i];
+  a.S[i] = st.S[i];
+  a.M[i] = st.M[i];
+  a.Bmax[i] = st.Bmax[i];
+  inst_refresh(a, m, i);
+}
+
+// The values of one instance's state a pair evaluation reads.
+struct InstVals {
+  int64_t q, S;
+  uint64_t kd;  // dcq_key0(b, qr)
+  int32_t room;
+  float dec0, f, tq;
+  int32_t Bp;
+};
+
+__device__ __forceinline__ InstVals inst_vals(const InstSmem& a, uint32_t i) {
+  InstVals v;
+  v.q = a.q[i];
+  v.S = a.S[i];
+  v.kd = a.kd[i];
+  v.room = a.room[i];
+  v.dec0 = a.dec0[i];
+  v.f = a.f[i];
+  v.tq = a.tq[i];
+  v.Bp = a.Bp[i];
+  return v;
+}
+
+// Instance i's state after it takes a request of L tokens at hit h (qr + 1, q + L - 16 h, S + L), as
+// the state update of a decision computes it.
+__device__ __forceinline__ InstVals inst_vals_after(const InstSmem& a, const psk::DevModel& m, uint32_t i, uint32_t L,
+                                                    uint32_t h, int32_t* qr_out) {
+  const int32_t qr = a.qr[i] + 1;
+  InstVals v;
+  v.q = a.q[i] + (int64_t)L - 16 * (int64_t)h;
+  v.S = a.S[i] + (int64_t)L;
+  const psk::InstTerms it = psk::inst_terms(m, a.b[i], qr, v.q, a.Bmax[i]);
+  v.dec0 = it.dec0;
+  v.f = it.f;
+  v.tq = it.tq;
+  v.Bp = it.Bp;
+  v.room = it.okB ? psk::kv_room(v.S, a.M[i]) : -1;
+  v.kd = psk::dcq_key0(a.b[i], qr);
+  *qr_out = qr;
+  return v;
+}
+
+__device__ __forceinline__ void inst_store(const InstSmem& a, uint32_t i, int32_t qr, const InstVals& v) {
+  a.qr[i] = qr;
+  a.q[i] = v.q;
+  a.S[i] = v.S;
+  a.kd[i] = v.kd;
+  a.room[i] = v.room;
+  a.dec0[i] = v.dec0;
+  a.f[i] = v.f;
+  a.tq[i] = v.tq;
+  a.Bp[i] = v.Bp;
+}
+
+// One pair (row, instance i at hit h) on state v: W, the capacity guard, and the packed key and tie
+// word the pair has in C (class 0 if the SLO admission passes, class 1 otherwise); key kNoKey
+// outside A.  tpf_bits: T_pf at h if known, else kNoTpfBits.
+struct PairKey {
+  float W;
+  uint64_t key;
+  uint32_t tie;
+  bool inA;
+};
+
+__device__ __forceinline__ PairKey pair_key_v(const psk::DevModel& m, const psk::RowConst& rc, const InstVals& v,
+                                              uint32_t i, uint32_t h, uint32_t tpf_bits) {
+  PairKey p;
+  const float tpf = tpf_bits != psk::kNoTpfBits ? __uint_as_float(tpf_bits) : psk::t_pf32(m, rc.L, h);
+  p.W = __fsub_rn(tpf, rc.t_cached);
+  p.inA = (int32_t)rc.L <= v.room;
+  p.key = psk::kNoKey;
+  p.tie = i;
+  if (p.inA) {
+    const int32_t n = (int32_t)rc.L - (int32_t)(h << 4);
+    float tpot, ttft;
+    if (narrow_qs(v.q, v.S)) {
+      psk::pair_lat32(m, rc, tpf, n, v.dec0, v.f, v.tq, v.Bp, (int32_t)v.q, (int32_t)v.S, &tpot, &ttft);
+    } else {
+      psk::InstTerms it;
+      it.dec0 = v.dec0;
+      it.f = v.f;
+      it.tq = v.tq;
+      it.Bp = v.Bp;
+      it.okB = 1;
+      psk::PairW x;
+      x.W = p.W;
+      x.tpf = tpf;
+      x.n = n;
+      x.inA = true;
+      psk::pair_lat(m, rc, x, it, v.q, v.S, &tpot, &ttft);
+    }
+    if (psk::pair_admitted(m, rc, tpot, ttft)) {
+      p.key = psk::packed_key(0u, psk::value_in_t(m, psk::key0_from_dcq(m, v.kd), h, tpot, rc.tpot_target));
+      if (m.sel == psk::kSelHCQ) p.tie |= (uint32_t)(v.kd & 0x3FFFFull) << 12;
+    } else {
+      p.key = psk::packed_key(1u, psk::value_fallback(m, (uint64_t)v.q + (uint64_t)n, (uint32_t)v.Bp, v.kd, h));
+    }
+  }
+  return p;
+}
+
+__device__ __forceinline__ PairKey pair_key_of(const psk::DevModel& m, const psk::RowConst& rc, const InstSmem& a,
+                                               uint32_t i, uint32_t h, uint32_t tpf_bits) {
+  return pair_key_v(m, rc, inst_vals(a, i), i, h, tpf_bits);
+}
+
+__device__ __forceinline__ bool kt_less(uint64_t k1, uint32_t t1, uint64_t k2, uint32_t t2) {
+  return k1 < k2 || (k1 == k2 && t1 < t2);
+}
+
+// Warp minimum of a 64-bit word with single-instruction reductions on each half.
+__device__ __forceinline__ unsigned long long warp_min_u64w(unsigned long long v) {
+  const uint32_t hi = (uint32_t)(v >> 32);
+  const uint32_t mhi = __reduce_min_sync(0xffffffffu, hi);
+  const uint32_t mlo = __reduce_min_sync(0xffffffffu, hi == mhi ? (uint32_t)v : 0xFFFFFFFFu);
+  return ((unsigned long long)mhi << 32) | mlo;
+}
+
+// Bounded spin on a shared-memory counter (acquire) until it reaches `want` or *abort is set; false
+// on timeout (error bit set) or abort.
+__device__ __forceinline__ bool wait_smem_at_least(const uint32_t* p, uint32_t want, const volatile int* abort,
+                                                   uint32_t* err, uint64_t limit_ns) {
+  if (psk::ld_acquire_cta_shared_u32(p) >= want) return true;
+  const uint64_t t0 = psk::globaltimer_ns();
+  for (;;) {
+    if (psk::ld_acquire_cta_shared_u32(p) >= want) return true;
+    if (*abort) return false;
+    if (psk::globaltimer_ns() - t0 > limit_ns) {
+      atomicOr(err, psk::kErrTimeout);
+      return false;
+    }
+    __nanosleep(20);
+  }
+}
+
+// Summary block sb: rows sb, sb + kSummaryBlocks, ...  Thread t holds instances t, t + 256, ...
 template <int IPT>
-__device__ void decide_rows(const psk::RowPre* __restrict__ rows, uint32_t R, uint32_t I, psk::StateSoA committed,
+__device__ void summary_rows(const psk::RowPre* __restrict__ rows, uint32_t R, uint32_t I, psk::StateSoA committed,
+                             const psk::DevModel& m, uint32_t* err, const psk::GreedySync& sync, uint32_t sb,
+                             unsigned long long* smem_raw) {
+  const uint32_t Ip = sync.ring_stride;
+  const InstSmem a = inst_smem(smem_raw, Ip);
+  __shared__ psk::RowPre s_row;
+  __shared__ int32_t s_jm[16];  // pick of request x in s_jm[x & 15] (-1: rejected)
+  __shared__ uint32_t s_wmin[psk::kSumWarps];
+  __shared__ uint32_t s_wb[psk::kSumWarps];
+  __shared__ unsigned long long s_kb[psk::kSumWarps];
+  __shared__ uint32_t s_tb[psk::kSumWarps];
+  __shared__ int s_abort;
+  const uint32_t t = threadIdx.x;
+  const int lane = (int)(t & 31u), warp = (int)(t >> 5);
+  for (uint32_t i = t; i < I; i += kPipeThreads) inst_load(a, committed, m, i);
+  if (t < 16) s_jm[t] = -1;
+  if (t == 0) s_abort = 0;
+  uint32_t applied = 0;  // decisions [0, applied) are in this block's state
+  __syncthreads();
+  for (uint32_t s = sb; s < R; s += kSummaryBlocks) {
+    const int64_t need = (int64_t)s - psk::kSpecLag;  // decisions [0, need) count for row s
+    if (warp == 0) {
+      // Replay decisions [applied, need), 32 at a time: the adds commute; the last lane of each
+      // instance refreshes its terms once every add is in.
+      bool abort = false;
+      while ((int64_t)applied < need && !abort) {
+        const uint32_t x = applied + (uint32_t)lane;
+        const bool mine = (int64_t)x < need;
+        unsigned long long jb = 0ull;
+        if (mine) jb = wait_job(sync.jobs + x, err, sync.wait_ns);
+        abort = __any_sync(0xffffffffu, mine && jb == 0ull);
+        if (abort) break;
+        const uint32_t j = mine ? job_pick(jb) : 0xFFFFFFFFu;
+        const bool upd = mine && j < I;
+        if (upd) {
+          const uint32_t L = __ldg(&rows[x].L);
+          const int64_t n = (int64_t)L - 16 * (int64_t)job_hit(jb);
+          atomicAdd(&a.qr[j], 1);
+          atomicAdd(reinterpret_cast<unsigned long long*>(&a.q[j]), (unsigned long long)n);
+          atomicAdd(reinterpret_cast<unsigned long long*>(&a.S[j]), (unsigned long long)(int64_t)L);
+        }
+        const uint32_t nbatch = (int64_t)applied + 32 <= need ? 32u : (uint32_t)(need - (int64_t)applied);
+        // the last 16 decisions of the batch take the ring slots (distinct within 16)
+        if (mine && x + 16u >= applied + nbatch) s_jm[x & 15u] = j < I ? (int32_t)j : -1;
+        const unsigned same = __match_any_sync(0xffffffffu, upd ? j : 0xFFFFFFFFu);
+        __syncwarp();
+        if (upd && (31 - __clz(same)) == lane) inst_refresh(a, m, j);
+        __syncwarp();
+        applied += nbatch;
+      }
+      if (lane == 0) {
+        if (abort) s_abort = 1;
+        else if (!wait_flag(sync.ready + s, err, sync.wait_ns)) s_abort = 1;  // the row's probed hits
+      }
+      if (lane < psk::kRowWords)
+        reinterpret_cast<uint4*>(&s_row)[lane] = __ldg(reinterpret_cast<const uint4*>(rows + s) + lane);
+    }
+    __syncthreads();
+    if (s_abort) return;  // block-uniform
+    const psk::RowConst rc = row_of(s_row);
+    const uint32_t slot = s % psk::kHitSlots;
+    // raises from the picks of requests s - kLcpBack .. s - kSpecLag - 1 (older than the lag)
+    constexpr int kNR = psk::kLcpBack - psk::kSpecLag;
+    int32_t rj[kNR > 0 ? kNR : 1];
+    uint32_t rl[kNR > 0 ? kNR : 1];
+#pragma unroll
+    for (int k2 = psk::kSpecLag; k2 < psk::kLcpBack; ++k2) {
+      const int64_t t2 = (int64_t)s - 1 - k2;
+      rj[k2 - psk::kSpecLag] = t2 >= 0 ? s_jm[(uint32_t)t2 & 15u] : -1;
+      rl[k2 - psk::kSpecLag] = s_row.lcp[k2];
+    }
+    // every pair: hit, W, capacity guard, key in C
+    PairKey pk[IPT];
+    uint32_t hk[IPT];
+    uint32_t wbest = 0xFFFFFFFFu;
+#pragma unroll
+    for (int k = 0; k < IPT; ++k) {
+      const uint32_t i = t + (uint32_t)k * kPipeThreads;
+      pk[k].inA = false;
+      pk[k].key = psk::kNoKey;
+      hk[k] = 0u;
+      if (i < I) {
+        const uint32_t h0 = __ldcg(sync.hitring + (uint64_t)slot * Ip + i);
+        const uint32_t tp0 = __float_as_uint(__ldcg(sync.tpfring + (uint64_t)slot * Ip + i));
+        uint32_t h = h0;
+#pragma unroll
+        for (int q = 0; q < kNR; ++q)
+          if (rj[q] == (int32_t)i && rl[q] > h) h = rl[q];
+        hk[k] = h;
+        pk[k] = pair_key_of(m, rc, a, i, h, h == h0 ? tp0 : psk::kNoTpfBits);
+        if (pk[k].inA) wbest = min(wbest, psk::f2ord(pk[k].W));
+      }
+    }
+    psk::RowSummary* out = sync.sums + (s % psk::kSumSlots);
+    // per warp: W_min over A, its kWPerWarp smallest (W, instance), the next one as its bound
+    {
+      const uint32_t wm = __reduce_min_sync(0xffffffffu, wbest);
+      if (lane == 0) s_wmin[warp] = wm;
+      uint32_t taken = 0u;
+#pragma unroll
+      for (int rnd = 0; rnd <= psk::kWPerWarp; ++rnd) {
+        unsigned long long mine = ~0ull;
+        int mk = -1;
+#pragma unroll
+        for (int k = 0; k < IPT; ++k) {
+          if (!pk[k].inA || ((taken >> k) & 1u)) continue;
+          const unsigned long long w = ((unsigned long long)psk::f2ord(pk[k].W) << 32) | (t + (uint32_t)k * kPipeThreads);
+          if (w < mine) {
+            mine = w;
+            mk = k;
+          }
+        }
+        const unsigned long long best = warp_min_u64w(mine);
+        if (mk >= 0 && mine == best) taken |= 1u << mk;
+        if (rnd < psk::kWPerWarp) {
+          if (lane == 0) out->w[warp * psk::kWPerWarp + rnd] = best;
+        } else if (lane == 0) {
+          s_wb[warp] = (uint32_t)(best >> 32);  // all ones when the warp has no more
+        }
+      }
+    }
+    __syncthreads();
+    uint32_t wmin_o = 0xFFFFFFFFu;
+#pragma unroll
+    for (int w = 0; w < psk::kSumWarps; ++w) wmin_o = min(wmin_o, s_wmin[w]);
+    const float wmin = psk::ord2f(wmin_o);
+    // per warp: the kKeysPerWarp smallest (key, tie) of C, the next one as its bound
+    {
+      bool inC[IPT];
+#pragma unroll
+      for (int k = 0; k < IPT; ++k) inC[k] = pk[k].inA && psk::pair_in_c(rc, pk[k].W, wmin);
+      uint32_t taken = 0u;
+#pragma unroll
+      for (int rnd = 0; rnd <= psk::kKeysPerWarp; ++rnd) {
+        uint64_t bk = psk::kNoKey;
+        uint32_t bt = 0xFFFFFFFFu, bh = 0u, bw = 0u;
+        int mk = -1;
+#pragma unroll
+        for (int k = 0; k < IPT; ++k) {
+          if (!inC[k] || ((taken >> k) & 1u)) continue;
+          if (kt_less(pk[k].key, pk[k].tie, bk, bt)) {
+            bk = pk[k].key;
+            bt = pk[k].tie;
+            bh = hk[k];
+            bw = psk::f2ord(pk[k].W);
+            mk = k;
+          }
+        }
+        uint64_t wk;
+        uint32_t wt, wh;
+        psk::warp_pick_min(bk, bt, bh, &wk, &wt, &wh);
+        const bool won = mk >= 0 && bk == wk && bt == wt;  // tie words are unique (instance in them)
+        if (won) taken |= 1u << mk;
+        const unsigned winm = __ballot_sync(0xffffffffu, won);
+        const uint32_t ww = __shfl_sync(0xffffffffu, bw, winm ? __ffs(winm) - 1 : 0);
+        if (rnd < psk::kKeysPerWarp) {
+          if (lane == 0) {
+            const int e = warp * psk::kKeysPerWarp + rnd;
+            out->key[e] = wk;
+            out->tie[e] = wt;
+            out->word[e] = ww;
+            out->hit[e] = wh;
+          }
+        } else if (lane == 0) {
+          s_kb[warp] = wk;
+          s_tb[warp] = wt;
+        }
+      }
+    }
+    __syncthreads();
+    if (t == 0) {
+      unsigned long long kb = psk::kNoKey;
+      uint32_t tb = 0xFFFFFFFFu, wb = 0xFFFFFFFFu;
+#pragma unroll
+      for (int w = 0; w < psk::kSumWarps; ++w) {
+        if (kt_less(s_kb[w], s_tb[w], kb, tb)) {
+          kb = s_kb[w];
+          tb = s_tb[w];
+        }
+        wb = min(wb, s_wb[w]);
+      }
+      out->key_bound = kb;
+      out->tie_bound = tb;
+      out->w_bound = wb;
+      out->wmin = wmin_o;
+      __threadfence();  // every warp's entries (written before the barrier) before the flag
+      psk::st_release_u32(sync.sready + s, 1u);
+    }
+    __syncthreads();  // the next row reuses the reduction slots
+  }
+}
+
+// Deciding block (warps 0 and 1; the block's other warps return at once).
+__device__ void decide_spec(const psk::RowPre* __restrict__ rows, uint32_t R, uint32_t I, psk::StateSoA committed,
                             psk::StateSoA pending, const psk::DevModel& m, int32_t* assign, uint8_t* __restrict__ path,
                             uint32_t* __restrict__ hit_chosen, uint32_t* err, const psk::GreedySync& sync,
                             unsigned long long* smem_raw) {
-  const uint32_t Ip = sync.ring_stride;  // I rounded up to a multiple of 4
-  // Every [Ip] array starts 16-byte aligned (Ip is a multiple of 4); the 8-byte arrays come first.
-  int64_t* s_q = reinterpret_cast<int64_t*>(smem_raw);    // [Ip] queued prefill tokens
-  int64_t* s_S = s_q + Ip;                                // [Ip] KV tokens held
-  uint64_t* s_key0 = reinterpret_cast<uint64_t*>(s_S + Ip);  // [Ip] D-C-Q key bits of (b, qr) (psk::dcq_key0)
-  int64_t* s_M = reinterpret_cast<int64_t*>(s_key0 + Ip);    // [Ip] KV capacity
-  uint32_t* s_hit = reinterpret_cast<uint32_t*>(s_M + Ip);   // [4][Ip] probed hits of rows r .. r + 3
-  uint32_t* s_tpf = s_hit + 4 * Ip;                          // [4][Ip] T_pf at those hits (bits)
-  uint32_t* s_ovr = s_tpf + 4 * Ip;                          // [2][Ip] lcp raises for the next row
-  int32_t* s_room = reinterpret_cast<int32_t*>(s_ovr + 2 * Ip);  // [Ip] free KV room, -1 if no slot
-  float* s_dec0 = reinterpret_cast<float*>(s_room + Ip);     // [Ip] InstTerms, field by field
-  float* s_f = s_dec0 + Ip;
-  float* s_tq = s_f + Ip;
-  int32_t* s_Bp = reinterpret_cast<int32_t*>(s_tq + Ip);
-  int32_t* s_b = s_Bp + Ip;                                  // [Ip] decoding requests
-  int32_t* s_qr = s_b + Ip;                                  // [Ip] queued requests
-  int32_t* s_Bmax = s_qr + Ip;                               // [Ip] decode-slot limit
-  __shared__ psk::RowPre s_row[8];  // rows r .. r + kRingAhead (a ring of 8 so no reader is overtaken)
-  __shared__ int s_wide;            // some instance's q or S left [0, 2^30): 64-bit token sums from then on
-  __shared__ int32_t s_jm[16];      // pick of request x in s_jm[x & 15] (-1: rejected)
-  __shared__ uint32_t s_red_w[32];  // per-warp W_min (order-preserving bits)
-  __shared__ uint4 s_red_k[32];     // per-warp pick: key (x, y), instance (z), hit (w)
-
-  const int t = threadIdx.x;
-  const int NT = blockDim.x;
-  const int NTI = NT - 32;
-  const bool sig = t == NTI;
-  const int lane = t & 31;
-  const int warp = t >> 5;
-  const int NWI = NTI >> 5;               // instance warps
-  const uint32_t i0 = (uint32_t)t * IPT;  // first owned instance (>= I for the signalling warp)
-  const bool owner = t < NTI;             // false for the whole signalling warp
-  const bool has = owner && i0 < I;       // the thread owns instances (then i0 + IPT <= Ip)
-  // instance terms of i after a state change (decode-slot guard folded into the KV room)
-  auto set_terms = [&](uint32_t i) {
-    const psk::InstTerms it = psk::inst_terms(m, s_b[i], s_qr[i], s_q[i], s_Bmax[i]);
-    s_dec0[i] = it.dec0;
-    s_f[i] = it.f;
-    s_tq[i] = it.tq;
-    s_Bp[i] = it.Bp;
-    s_room[i] = it.okB ? psk::kv_room(s_S[i], s_M[i]) : -1;
-    s_key0[i] = psk::dcq_key0(s_b[i], s_qr[i]);
-  };
-
-  if (t == 0) s_wide = 0;
-  __syncthreads();
-  for (uint32_t i = t; i < Ip; i += NT) {
-    if (i < I) {
-      s_b[i] = committed.b[i];
-      s_qr[i] = committed.qr[i];
-      s_q[i] = committed.q[i];
-      s_S[i] = committed.S[i];
-      s_M[i] = committed.M[i];
-      s_Bmax[i] = committed.Bmax[i];
-      set_terms(i);
-      if (!narrow_qs(s_q[i], s_S[i])) s_wide = 1;
-    } else {
-      s_room[i] = -1;  // padding: never capacity-eligible
-    }
+  if (threadIdx.x >= 64) return;
+  const uint32_t Ip = sync.ring_stride;
+  const InstSmem a = inst_smem(smem_raw, Ip);
+  uint32_t* s_hitr = reinterpret_cast<uint32_t*>(a.Bmax + Ip);  // [kFeedRing][Ip] probed hits
+  uint32_t* s_tpfr = s_hitr + kFeedRing * Ip;                   // [kFeedRing][Ip] T_pf at them (bits)
+  __shared__ psk::RowSummary s_sum[kFeedRing];
+  __shared__ psk::RowPre s_rowc[kFeedRing];
+  __shared__ uint32_t s_fed;       // rows [0, s_fed) are staged (release / acquire)
+  __shared__ uint32_t s_consumed;  // rows [0, s_consumed) are decided (release / acquire)
+  __shared__ volatile int s_stop;           // the feeder or the decider gave up
+  const uint32_t t = threadIdx.x;
+  const int lane = (int)(t & 31u);
+  const unsigned full = 0xffffffffu;
+  for (uint32_t i = t; i < I; i += 64) inst_load(a, committed, m, i);
+  if (t == 0) {
+    s_fed = 0u;
+    s_consumed = 0u;
+    s_stop = 0;
   }
-  for (uint32_t i = t; i < 2 * Ip; i += NT) s_ovr[i] = 0u;
-  if (t < 16) s_jm[t] = -1;
-  if (t < kRingAhead * psk::kRowWords) {  // rows 0 .. kRingAhead - 1
-    const uint32_t rr = (uint32_t)(t / psk::kRowWords);
-    if (rr < R)
-      reinterpret_cast<uint4*>(&s_row[rr])[t % psk::kRowWords] =
-          __ldg(reinterpret_cast<const uint4*>(rows + rr) + (t % psk::kRowWords));
-  }
-  bool timed_out = false;
-  if (sig) {
-    for (uint32_t x = 0; x < 2 && x < R && !timed_out; ++x) timed_out = !wait_flag(sync.ready + x, err, sync.wait_ns);
-  }
-  __syncthreads();
-  // hits of rows 0 and 1, one copy group each (each thread copies and later reads only its own)
-  static_assert(IPT == 1 || IPT == 2 || IPT == 4, "one 4-, 8- or 16-byte copy per array and row");
-  auto copy_row = [&](uint32_t x) {
-    if (has) {
-      const uint64_t src = (uint64_t)(x % psk::kHitSlots) * Ip + i0;
-      const uint32_t dst = (x & 3u) * Ip + i0;
-      psk::cp_async_bytes<4 * IPT>(s_hit + dst, sync.hitring + src);
-      psk::cp_async_bytes<4 * IPT>(s_tpf + dst, sync.tpfring + src);
-    }
-  };
-  if (R > 0) copy_row(0);
-  psk::cp_async_commit();
-  if (R > 1) copy_row(1);
-  psk::cp_async_commit();
+  asm volatile("bar.sync 1, 64;" ::: "memory");
 
-  int32_t jprev = -1;  // pick of request r - 1
-  uint32_t hr[IPT];
-
-  for (uint32_t r = 0; r < R; ++r) {
-    if (!owner) {  // the signalling warp: row r + 2's ready flag, then the step's two barriers
-      uint32_t ready_seen = 1u;
-      if (sig && r + 2 < R && !timed_out) ready_seen = psk::ld_acquire_u32(sync.ready + r + 2);
-      __syncthreads();  // (C)
-      if (sig && ready_seen == 0u) timed_out = !wait_flag(sync.ready + r + 2, err, sync.wait_ns);
-      __syncthreads();  // (D)
-      continue;
-    }
-    const psk::RowPre& cur = s_row[r & 7];
-    // ---- P0: row-constant refill, row r's hits, pass 1 ------------------------------------------
-    if (t < psk::kRowWords && r + kRingAhead < R)
-      psk::cp_async16(reinterpret_cast<uint4*>(&s_row[(r + kRingAhead) & 7]) + t,
-                      reinterpret_cast<const uint4*>(rows + r + kRingAhead) + t);
-    psk::cp_async_wait_group<1>();  // this thread's copies of row r (and row constants <= r + 4)
-    const psk::RowConst rc = row_of(cur);
-    const bool narrow = s_wide == 0;  // a thread owning an instance that left the range set the flag itself
-    const uint32_t lcp0 = cur.lcp[0];
-    float Wk[IPT], tpk[IPT];
-    bool inA[IPT];
-    uint32_t wbest = 0xFFFFFFFFu;  // order-preserving bits of this thread's W_min over A
-    if (has) {
-      uint32_t hb[IPT], ov[IPT], tb[IPT], rm[IPT];
-      ld_u32v<IPT>(s_hit + (r & 3u) * Ip + i0, hb);
-      ld_u32v<IPT>(s_tpf + (r & 3u) * Ip + i0, tb);
-      uint32_t* op = s_ovr + (r & 1u) * Ip + i0;
-      ld_u32v<IPT>(op, ov);
-      ld_u32v<IPT>(s_room + i0, rm);
-      uint32_t anyov = 0u;
-#pragma unroll
-      for (int k = 0; k < IPT; ++k) anyov |= ov[k];
-      if (anyov) st_zero_u32v<IPT>(op);
-#pragma unroll
-      for (int k = 0; k < IPT; ++k) {
-        uint32_t h = hb[k] > ov[k] ? hb[k] : ov[k];
-        if ((int32_t)(i0 + k) == jprev && lcp0 > h) h = lcp0;
-        hr[k] = h;
-        // T_pf at the hit: the ring's value unless it is marked unknown (the probe blocks raised the
-        // hit) or the hit was raised here; W = T_pf(n, c) - T_pf(0, L)
-        tpk[k] = (h == hb[k] && tb[k] != psk::kNoTpfBits) ? __uint_as_float(tb[k]) : psk::t_pf32(m, rc.L, h);
-        Wk[k] = __fsub_rn(tpk[k], rc.t_cached);
-        inA[k] = (int32_t)rc.L <= (int32_t)rm[k];
-        if (inA[k]) wbest = min(wbest, psk::f2ord(Wk[k]));
+  if (t >= 32) {
+    // ---- feeder -----------------------------------------------------------------------------------
+    for (uint32_t x = 0; x < R; ++x) {
+      const uint32_t slot = x % kFeedRing;
+      // lane 0 waits for the slot to be free and the row's summary to be published; the warp follows
+      bool ok = true;
+      if (lane == 0) {
+        if (x >= kFeedRing) ok = wait_smem_at_least(&s_consumed, x - kFeedRing + 1, &s_stop, err, sync.wait_ns);
+        if (ok) ok = wait_flag(sync.sready + x, err, sync.wait_ns);
+        if (!ok) s_stop = 1;
       }
-    } else {
-#pragma unroll
-      for (int k = 0; k < IPT; ++k) inA[k] = false;
+      ok = __shfl_sync(full, ok ? 1 : 0, 0) != 0;
+      __syncwarp();
+      if (!ok) break;  // warp-uniform
+      const uint4* src_sum = reinterpret_cast<const uint4*>(sync.sums + (x % psk::kSumSlots));
+      uint4* dst_sum = reinterpret_cast<uint4*>(&s_sum[slot]);
+      for (uint32_t w = (uint32_t)lane; w < sizeof(psk::RowSummary) / 16; w += 32) psk::cp_async16(dst_sum + w, src_sum + w);
+      if (lane < psk::kRowWords)
+        psk::cp_async16(reinterpret_cast<uint4*>(&s_rowc[slot]) + lane, reinterpret_cast<const uint4*>(rows + x) + lane);
+      const uint4* src_h = reinterpret_cast<const uint4*>(sync.hitring + (uint64_t)(x % psk::kHitSlots) * Ip);
+      const uint4* src_t = reinterpret_cast<const uint4*>(sync.tpfring + (uint64_t)(x % psk::kHitSlots) * Ip);
+      uint4* dst_h = reinterpret_cast<uint4*>(s_hitr + slot * Ip);
+      uint4* dst_t = reinterpret_cast<uint4*>(s_tpfr + slot * Ip);
+      for (uint32_t w = (uint32_t)lane; w < Ip / 4; w += 32) {
+        psk::cp_async16(dst_h + w, src_h + w);
+        psk::cp_async16(dst_t + w, src_t + w);
+      }
+      psk::cp_async_commit();
+      psk::cp_async_wait_all();
+      __syncwarp();
+      if (lane == 0) psk::st_release_cta_shared_u32(&s_fed, x + 1);
     }
-    wbest = __reduce_min_sync(0xffffffffu, wbest);
-    if (lane == 0) s_red_w[warp] = wbest;
-    __syncthreads();  // (C)
+    return;
+  }
 
-    // ---- P1: W_min, pass 2, the row's argmin; lcp raises for row r + 1 --------------------------
-    const uint32_t wmin_o = __reduce_min_sync(0xffffffffu, lane < NWI ? s_red_w[lane] : 0xFFFFFFFFu);
-    const bool anyA = wmin_o != 0xFFFFFFFFu;  // a W of a pair in A never maps to all ones (not NaN)
-    const float wmin = psk::ord2f(wmin_o);
-    uint64_t bkey = psk::kNoKey;
-    uint32_t btie = 0xFFFFFFFFu, bh = 0u;
-    bool inC[IPT];
-    bool anyC = false;
+  // ---- deciding warp --------------------------------------------------------------------------------
+  // Carried from step s to step s + 1 (software pipelining: what step s + 1 needs of its touched
+  // instances is computed in step s, beside step s's reductions):
+  //   pk          lane k < kLcpBack: the pick of request s - 1 - k (-1: none or rejected)
+  //   hist        the same picks in every lane
+  //   cor, chit   lane k < kSpecLag: that instance's pair (key, tie, W, capacity) and hit on row s on
+  //               the current state.  Lane 0's is the pick of request s - 1, which each candidate lane
+  //               of step s - 1 evaluated as if it were picked; lanes 1 .. kSpecLag - 1 evaluated
+  //               theirs on row s in step s - 1 (stale only when step s - 1 picked the same instance,
+  //               and then lane 0 holds it and the duplicate is dropped).
+  int32_t pk = -1;
+  int32_t hist[psk::kLcpBack];
 #pragma unroll
-    for (int k = 0; k < IPT; ++k) {
-      inC[k] = inA[k] && psk::pair_in_c(rc, Wk[k], wmin);
-      anyC |= inC[k];
+  for (int k = 0; k < psk::kLcpBack; ++k) hist[k] = -1;
+  PairKey cor;
+  cor.W = 0.0f;
+  cor.key = psk::kNoKey;
+  cor.tie = 0xFFFFFFFFu;
+  cor.inA = false;
+  uint32_t chit = 0u;
+  unsigned long long n_fast = 0, n_full = 0;
+  // hit of instance c on a row: its probed hit raised to the common prefix with each of the last
+  // kLcpBack requests that went to c; `self` raises by lcp[0] too (c taking the request just before)
+  auto raised_hit = [&](const psk::RowPre& rw, const uint32_t* hr, uint32_t c, bool self, int shift) {
+    const uint32_t hb = hr[c];
+    uint32_t h = hb;
+    if (self && rw.lcp[0] > h) h = rw.lcp[0];
+#pragma unroll
+    for (int k2 = 0; k2 < psk::kLcpBack; ++k2) {
+      // shift 0: lcp[k2] is with request s - 1 - k2 = hist[k2]; shift 1 (the next row): lcp[k2] is with
+      // request s - k2 = hist[k2 - 1]
+      const int kk = k2 - shift;
+      if (kk >= 0 && hist[kk < 0 ? 0 : kk] == (int32_t)c && rw.lcp[k2] > h) h = rw.lcp[k2];
     }
-    if (anyC) {
-      uint32_t dec0[IPT], fe[IPT], tq[IPT], Bp[IPT];
-      uint64_t q[IPT], S[IPT], k0[IPT];
-      ld_u32v<IPT>(s_dec0 + i0, dec0);
-      ld_u32v<IPT>(s_f + i0, fe);
-      ld_u32v<IPT>(s_tq + i0, tq);
-      ld_u32v<IPT>(s_Bp + i0, Bp);
-      ld_u64v<IPT>(s_q + i0, q);
-      ld_u64v<IPT>(s_S + i0, S);
-      ld_u64v<IPT>(s_key0 + i0, k0);
+    return h;
+  };
+  for (uint32_t s = 0; s < R; ++s) {
+    const uint32_t slot = s % kFeedRing;
+    const bool has_next = s + 1 < R;
+    bool ok = true;
+    if (lane == 0) {
+      ok = wait_smem_at_least(&s_fed, has_next ? s + 2 : s + 1, &s_stop, err, sync.wait_ns);
+      if (!ok) s_stop = 1;
+    }
+    ok = __shfl_sync(full, ok ? 1 : 0, 0) != 0;
+    __syncwarp();
+    if (!ok) break;  // warp-uniform
+    const psk::RowPre& row = s_rowc[slot];
+    const psk::RowSummary& sm = s_sum[slot];
+    const uint32_t* hrow = s_hitr + slot * Ip;
+    const uint32_t* trow = s_tpfr + slot * Ip;
+    const psk::RowConst rc = row_of(row);
+    auto touched = [&](uint32_t i) {
+      bool r = false;
 #pragma unroll
-      for (int k = 0; k < IPT; ++k) {
-        if (!inC[k]) continue;
-        psk::InstTerms it;
-        it.dec0 = __uint_as_float(dec0[k]);
-        it.f = __uint_as_float(fe[k]);
-        it.tq = __uint_as_float(tq[k]);
-        it.Bp = (int32_t)Bp[k];
-        it.okB = 1;
-        psk::PairW x;
-        x.W = Wk[k];
-        x.tpf = tpk[k];
-        x.n = (int64_t)rc.L - 16 * (int64_t)hr[k];
-        x.inA = true;
-        float tpot, ttft;
-        if (narrow)
-          psk::pair_lat32(m, rc, x.tpf, (int32_t)x.n, it.dec0, it.f, it.tq, it.Bp, (int32_t)q[k], (int32_t)S[k], &tpot,
-                          &ttft);
-        else
-          psk::pair_lat(m, rc, x, it, (int64_t)q[k], (int64_t)S[k], &tpot, &ttft);
-        uint64_t key;
-        uint32_t tie = i0 + k;
-        if (psk::pair_admitted(m, rc, tpot, ttft)) {
-          key = psk::packed_key(0u, psk::value_in_t(m, psk::key0_from_dcq(m, k0[k]), hr[k], tpot, rc.tpot_target));
-          if (m.sel == psk::kSelHCQ) tie = psk::tie_in_t(m, i0 + k, (int32_t)(k0[k] & 0x3FFFFull));
-        } else {
-          key = psk::packed_key(1u, psk::value_fallback(m, (uint64_t)q[k] + (uint64_t)x.n, (uint32_t)Bp[k], k0[k], hr[k]));
-        }
-        if (key < bkey || (key == bkey && tie < btie)) {
-          bkey = key;
-          btie = tie;
-          bh = hr[k];
-        }
+      for (int k = 0; k < psk::kSpecLag; ++k) r |= hist[k] == (int32_t)i;
+      return r;
+    };
+    // the touched instances, one lane each (the latest occurrence)
+    const int32_t tk = lane < psk::kSpecLag ? pk : -1;
+    const unsigned same = __match_any_sync(full, tk);
+    const bool corr = tk >= 0 && (__ffs(same) - 1) == lane;
+    // W_min of the current state
+    const unsigned long long wv = lane < psk::kSumWarps * psk::kWPerWarp ? sm.w[lane] : ~0ull;
+    const bool w_untouched = wv != ~0ull && !touched((uint32_t)wv);
+    const uint32_t mu = __reduce_min_sync(full, w_untouched ? (uint32_t)(wv >> 32) : 0xFFFFFFFFu);
+    const uint32_t mt = __reduce_min_sync(full, (corr && cor.inA) ? psk::f2ord(cor.W) : 0xFFFFFFFFu);
+    uint32_t wmin_o = min(mu, mt);
+    bool anyA = wmin_o != 0xFFFFFFFFu;
+    bool fast = sm.w_bound == 0xFFFFFFFFu || mu <= sm.w_bound;
+    if (fast && anyA && rc.Z > 0.0f && wmin_o > sm.wmin) fast = false;
+    // this lane's candidate: its summary entry or its touched instance, whichever is smaller
+    uint64_t bk = psk::kNoKey;
+    uint32_t bt = 0xFFFFFFFFu, bh = 0u;
+    if (fast && anyA) {
+      const float wmin = psk::ord2f(wmin_o);
+      const uint64_t ek = sm.key[lane];
+      const uint32_t et = sm.tie[lane];
+      if (ek != psk::kNoKey && !touched(et & psk::kTieInstMask) && psk::pair_in_c(rc, psk::ord2f(sm.word[lane]), wmin)) {
+        bk = ek;
+        bt = et;
+        bh = sm.hit[lane];
+      }
+      if (corr && cor.inA && psk::pair_in_c(rc, cor.W, wmin) && kt_less(cor.key, cor.tie, bk, bt)) {
+        bk = cor.key;
+        bt = cor.tie;
+        bh = chit;
       }
     }
-    {
-      uint64_t wk;
-      uint32_t wi, wh;
-      psk::warp_pick_min(bkey, btie, bh, &wk, &wi, &wh);
-      if (lane == 0) s_red_k[warp] = make_uint4((uint32_t)wk, (uint32_t)(wk >> 32), wi, wh);
+    // next row, computed beside this row's reductions: (a) this lane's candidate as the pick of
+    // request s (its state after the pick, its pair on row s + 1); (b) lanes 1 .. kSpecLag - 1: the
+    // instance picked by request s - lane, on row s + 1 with its current state
+    const uint32_t slot1 = (s + 1) % kFeedRing;
+    const psk::RowPre& row1 = s_rowc[slot1];
+    const uint32_t* hrow1 = s_hitr + slot1 * Ip;
+    const uint32_t* trow1 = s_tpfr + slot1 * Ip;
+    const int32_t u = __shfl_up_sync(full, pk, 1);  // lane k >= 1: the pick of request s - k
+    PairKey nx, nt;
+    nx.W = nt.W = 0.0f;
+    nx.key = nt.key = psk::kNoKey;
+    nx.tie = nt.tie = 0xFFFFFFFFu;
+    nx.inA = nt.inA = false;
+    uint32_t nxh = 0u, nth = 0u;
+    InstVals nv;
+    int32_t nqr = 0;
+    if (bk != psk::kNoKey) nv = inst_vals_after(a, m, bt & psk::kTieInstMask, rc.L, bh, &nqr);
+    if (has_next) {
+      const psk::RowConst rc1 = row_of(row1);
+      if (bk != psk::kNoKey) {
+        const uint32_t c = bt & psk::kTieInstMask;
+        nxh = raised_hit(row1, hrow1, c, true, 1);
+        nx = pair_key_v(m, rc1, nv, c, nxh, nxh == hrow1[c] ? trow1[c] : psk::kNoTpfBits);
+      }
+      if (lane >= 1 && lane < psk::kSpecLag && u >= 0) {
+        const uint32_t c = (uint32_t)u;
+        nth = raised_hit(row1, hrow1, c, false, 1);
+        nt = pair_key_of(m, rc1, a, c, nth, nth == hrow1[c] ? trow1[c] : psk::kNoTpfBits);
+      }
     }
-    // Row r + 1's raises from requests r - 1 .. r - kLag + 1 (thread d - 1 takes request r - d); the
-    // raise from request r itself is applied in registers next step.
-    if (t < psk::kLcpBack - 1 && r + 1 < R) {
-      const uint32_t d = (uint32_t)t + 1u;
-      const int32_t jd = r >= d ? s_jm[(r - d) & 15u] : -1;
-      const uint32_t v = s_row[(r + 1) & 7].lcp[d];
-      if (jd >= 0 && v > 0u) atomicMax(s_ovr + ((r + 1) & 1u) * Ip + (uint32_t)jd, v);
+    uint64_t K = psk::kNoKey;
+    uint32_t T = 0xFFFFFFFFu, H = 0u;
+    if (fast && anyA) {
+      psk::warp_pick_min(bk, bt, bh, &K, &T, &H);
+      fast = K != psk::kNoKey && (sm.key_bound == psk::kNoKey || kt_less(K, T, sm.key_bound, sm.tie_bound));
     }
-    __syncthreads();  // (D)
-
-    // ---- P2: the pick, its state, its insert job; copies of row r + 2 ----------------------------
-    uint64_t key;
-    uint32_t j, hj;
-    {
-      const uint4 pk = lane < NWI ? s_red_k[lane] : make_uint4(0xFFFFFFFFu, 0xFFFFFFFFu, 0xFFFFFFFFu, 0u);
-      psk::warp_pick_min(((uint64_t)pk.y << 32) | pk.x, pk.z, pk.w, &key, &j, &hj);
-      j &= psk::kTieInstMask;
+    const bool won = fast && bk != psk::kNoKey && bk == K && bt == T;  // one lane at most (tie words are unique)
+    if (fast) {
+      ++n_fast;
+    } else {
+      // full pass over the row on the current state
+      ++n_full;
+      uint32_t wo = 0xFFFFFFFFu;
+      for (uint32_t i = (uint32_t)lane; i < I; i += 32) {
+        if ((int32_t)rc.L <= a.room[i]) {
+          const uint32_t h = raised_hit(row, hrow, i, false, 0);
+          const float tpf = (h == hrow[i] && trow[i] != psk::kNoTpfBits) ? __uint_as_float(trow[i]) : psk::t_pf32(m, rc.L, h);
+          wo = min(wo, psk::f2ord(__fsub_rn(tpf, rc.t_cached)));
+        }
+      }
+      wmin_o = __reduce_min_sync(full, wo);
+      anyA = wmin_o != 0xFFFFFFFFu;
+      const float wmin = psk::ord2f(wmin_o);
+      uint64_t fk = psk::kNoKey;
+      uint32_t ft = 0xFFFFFFFFu, fh = 0u;
+      if (anyA) {
+        for (uint32_t i = (uint32_t)lane; i < I; i += 32) {
+          const uint32_t h = raised_hit(row, hrow, i, false, 0);
+          const PairKey p = pair_key_of(m, rc, a, i, h, h == hrow[i] ? trow[i] : psk::kNoTpfBits);
+          if (p.inA && psk::pair_in_c(rc, p.W, wmin) && kt_less(p.key, p.tie, fk, ft)) {
+            fk = p.key;
+            ft = p.tie;
+            fh = h;
+          }
+        }
+      }
+      psk::warp_pick_min(fk, ft, fh, &K, &T, &H);
     }
-    const bool pick = anyA && key != psk::kNoKey;
-    if (!pick) hj = 0u;
-    if (t == 0) {
-      assign[r] = pick ? (int32_t)j : -1;
-      path[r] = pick ? (uint8_t)(key >> 62) : (uint8_t)2;
-      hit_chosen[r] = hj;
-      s_jm[r & 15u] = pick ? (int32_t)j : -1;
-      psk::st_relaxed_u64(sync.jobs + r, kJobValid | ((unsigned long long)hj << 32) | (pick ? j : 0xFFFFFFFFu));
+    const bool pick = anyA && K != psk::kNoKey;
+    const uint32_t j = T & psk::kTieInstMask;
+    if (!pick) H = 0u;
+    __syncwarp();  // every lane's reads of this step are done before the pick's state changes
+    // the pick's state after the decision, and its pair on row s + 1 for lane 0 of the next step
+    PairKey pn;
+    uint32_t pnh = 0u;
+    const unsigned wm = __ballot_sync(full, won);
+    if (wm) {
+      const int wl = __ffs(wm) - 1;
+      if (won) inst_store(a, j, nqr, nv);
+      pn.W = __shfl_sync(full, nx.W, wl);
+      pn.key = ((uint64_t)__shfl_sync(full, (uint32_t)(nx.key >> 32), wl) << 32) | __shfl_sync(full, (uint32_t)nx.key, wl);
+      pn.tie = __shfl_sync(full, nx.tie, wl);
+      pn.inA = __shfl_sync(full, nx.inA ? 1 : 0, wl) != 0;
+      pnh = __shfl_sync(full, nxh, wl);
+    } else {
+      pn.W = 0.0f;
+      pn.key = psk::kNoKey;
+      pn.tie = 0xFFFFFFFFu;
+      pn.inA = false;
+      if (pick && lane == 0) {
+        int32_t qr2;
+        const InstVals v2 = inst_vals_after(a, m, j, rc.L, H, &qr2);
+        inst_store(a, j, qr2, v2);
+        if (has_next) {
+          pnh = raised_hit(row1, hrow1, j, true, 1);
+          pn = pair_key_v(m, row_of(row1), v2, j, pnh, pnh == hrow1[j] ? trow1[j] : psk::kNoTpfBits);
+        }
+      }
     }
-    if (pick && j >= i0 && j < i0 + IPT) {
-      s_qr[j] += 1;
-      s_q[j] += (int64_t)rc.L - 16 * (int64_t)hj;
-      s_S[j] += (int64_t)rc.L;
-      set_terms(j);
-      if (!narrow_qs(s_q[j], s_S[j])) s_wide = 1;  // seen from the next step on (after its barriers)
+    if (lane == 0) {
+      assign[s] = pick ? (int32_t)j : -1;
+      path[s] = pick ? (uint8_t)(K >> 62) : (uint8_t)2;
+      hit_chosen[s] = H;
+      psk::st_relaxed_u64(sync.jobs + s, kJobValid | ((unsigned long long)H << 32) | (pick ? j : 0xFFFFFFFFu));
+      psk::st_release_cta_shared_u32(&s_consumed, s + 1);
     }
-    if (r + 2 < R) copy_row(r + 2);
-    psk::cp_async_commit();
-    jprev = pick ? (int32_t)j : -1;
+    __syncwarp();
+    const int32_t pj = pick ? (int32_t)j : -1;
+    pk = __shfl_up_sync(full, pk, 1);
+    if (lane == 0) pk = pj;
+#pragma unroll
+    for (int k = psk::kLcpBack - 1; k > 0; --k) hist[k] = hist[k - 1];
+    hist[0] = pj;
+    if (lane == 0) {
+      cor = pn;
+      chit = pnh;
+    } else {
+      cor = nt;
+      chit = nth;
+    }
   }
-  psk::cp_async_wait_all();
-  __syncthreads();
-  for (uint32_t i = t; i < I; i += NT) {
-    pending.b[i] = s_b[i];
-    pending.qr[i] = s_qr[i];
-    pending.q[i] = s_q[i];
-    pending.S[i] = s_S[i];
-    pending.M[i] = s_M[i];
-    pending.Bmax[i] = s_Bmax[i];
+  if (lane == 0 && sync.stats) {
+    atomicAdd(sync.stats, n_fast);
+    atomicAdd(sync.stats + 1, n_full);
+  }
+  for (uint32_t i = (uint32_t)lane; i < I; i += 32) {
+    pending.b[i] = a.b[i];
+    pending.qr[i] = a.qr[i];
+    pending.q[i] = a.q[i];
+    pending.S[i] = a.S[i];
+    pending.M[i] = a.M[i];
+    pending.Bmax[i] = a.Bmax[i];
   }
 }
 
 template <int IPT>
-__global__ void __launch_bounds__(544, 1)
+__global__ void __launch_bounds__(kPipeThreads, 1)
 greedy_pipe_kernel(const psk::RowPre* __restrict__ rows, const uint64_t* __restrict__ hash, uint32_t R, uint32_t I,
                    const uint32_t* __restrict__ hit0, const float* __restrict__ tpf0, psk::StateSoA committed,
                    psk::StateSoA pending, psk::DevModel m, psk::DeltaSlot* delta, uint64_t nslots, int32_t* assign,
                    uint8_t* __restrict__ path, uint32_t* __restrict__ hit_chosen, uint32_t* err, psk::GreedySync sync) {
   extern __shared__ unsigned long long smem_raw[];
   if (blockIdx.x == 0) {
-    decide_rows<IPT>(rows, R, I, committed, pending, m, assign, path, hit_chosen, err, sync, smem_raw);
+    decide_spec(rows, R, I, committed, pending, m, assign, path, hit_chosen, err, sync, smem_raw);
   } else if (blockIdx.x <= kInsertBlocks) {
     insert_blocks(rows, hash, R, delta, nslots, err, sync);
-  } else {
+  } else if (blockIdx.x <= kInsertBlocks + kProbeBlocks) {
     probe_rows<IPT>(rows, hash, R, I, hit0, tpf0, delta, nslots, err, sync, smem_raw);
+  } else {
+    summary_rows<IPT>(rows, R, I, committed, m, err, sync, blockIdx.x - 1 - kInsertBlocks - kProbeBlocks, smem_raw);
   }
 }
 
 size_t greedy_pipe_smem(uint32_t I, uint32_t Ip) {
-  // 4 eight-byte and 18 four-byte [Ip] arrays (q, S, key0, M; hit and T_pf rings, raises, room,
-  // dec0, f, tq, Bp, b, qr, B_max)
-  const size_t decide = (size_t)Ip * (4 * sizeof(int64_t) + 18 * sizeof(uint32_t));
+  // deciding block: instance state, the hit and T_pf rows of kFeedRing rows; summary blocks: the
+  // instance state; probe blocks: three u32 arrays per instance
+  const size_t decide = (size_t)Ip * (kInstSmemBytes + 2 * kFeedRing * sizeof(uint32_t));
   const size_t probe = (size_t)I * 3 * sizeof(uint32_t);
   return decide > probe ? decide : probe;
 }
@@ -908,8 +1358,7 @@ template <int IPT>
 cudaError_t greedy_pipe_launch(const psk::RowPre* rows, const psk::WindowDev& w, uint32_t I, const uint32_t* hit0,
                                const float* tpf0, psk::StateSoA committed, psk::StateSoA pending, const psk::DevModel& m,
                                psk::DeltaSlot* delta, uint64_t nslots, int32_t* assign, uint8_t* path,
-                               uint32_t* hit_chosen, uint32_t* err, const psk::GreedySync& sync, uint32_t nt,
-                               cudaStream_t s) {
+                               uint32_t* hit_chosen, uint32_t* err, const psk::GreedySync& sync, cudaStream_t s) {
   const size_t smem = greedy_pipe_smem(I, sync.ring_stride);
   cudaError_t e = cudaFuncSetAttribute(greedy_pipe_kernel<IPT>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
@@ -922,8 +1371,9 @@ cudaError_t greedy_pipe_launch(const psk::RowPre* rows, const psk::WindowDev& w,
                   (void*)&mm, (void*)&delta, (void*)&nslots, (void*)&assign, (void*)&path, (void*)&hit_chosen,
                   (void*)&err, (void*)&sy};
   // all blocks must be resident at once: they wait on one another
-  return cudaLaunchCooperativeKernel((const void*)greedy_pipe_kernel<IPT>, dim3(1 + kInsertBlocks + kProbeBlocks),
-                                     dim3(nt), args, smem, s);
+  return cudaLaunchCooperativeKernel((const void*)greedy_pipe_kernel<IPT>,
+                                     dim3(1 + kInsertBlocks + kProbeBlocks + kSummaryBlocks), dim3(kPipeThreads), args,
+                                     smem, s);
 }
 
 }  // namespace
@@ -957,18 +1407,19 @@ cudaError_t launch_greedy_search(const psk::RowPre* rows, const psk::WindowDev& 
   if (w.R == 0) return cudaSuccess;
   cudaError_t e = cudaMemsetAsync(sync.done, 0, (size_t)w.R * sizeof(uint32_t), s);
   if (e == cudaSuccess) e = cudaMemsetAsync(sync.ready, 0, (size_t)w.R * sizeof(uint32_t), s);
+  if (e == cudaSuccess) e = cudaMemsetAsync(sync.sready, 0, (size_t)w.R * sizeof(uint32_t), s);
   if (e == cudaSuccess) e = cudaMemsetAsync(sync.jobs, 0, (size_t)w.R * sizeof(unsigned long long), s);
+  if (e == cudaSuccess && sync.stats) e = cudaMemsetAsync(sync.stats, 0, 2 * sizeof(unsigned long long), s);
   if (e != cudaSuccess) return e;
-  // up to 512 threads each owning IPT consecutive instances (IPT = 1, 2 or 4 for I up to 2048),
-  // plus one signalling warp
-  const uint32_t ipt = I <= 512 ? 1u : (I <= 1024 ? 2u : 4u);
-  const uint32_t nt = ((I + ipt - 1) / ipt + 31) / 32 * 32 + 32;
+  // every block has 256 threads; probe and summary threads hold IPT = ceil(I / 256) instances each
+  const uint32_t ipt = (I + kPipeThreads - 1) / kPipeThreads;
 #define PS_GREEDY_P(IPT)                                                                                      \
   return greedy_pipe_launch<IPT>(rows, w, I, hit0, tpf0, committed, pending, m, delta, delta_nslots, assign, path, \
-                                 hit_chosen, err, sync, nt, s)
-  if (ipt == 1) PS_GREEDY_P(1);
-  if (ipt == 2) PS_GREEDY_P(2);
-  if (ipt == 4 && I <= 2048) PS_GREEDY_P(4);
+                                 hit_chosen, err, sync, s)
+  if (ipt <= 1) PS_GREEDY_P(1);
+  if (ipt <= 2) PS_GREEDY_P(2);
+  if (ipt <= 4) PS_GREEDY_P(4);
+  if (ipt <= 8) PS_GREEDY_P(8);
 #undef PS_GREEDY_P
   return cudaErrorInvalidValue;
 }

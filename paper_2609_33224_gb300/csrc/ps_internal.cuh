@@ -100,14 +100,46 @@ struct RowList {
   uint32_t* count;  // [1]
 };
 
+// Lag-d speculation of the greedy pass: summary blocks evaluate row s in full on the state before
+// decision s - kSpecLag and publish a RowSummary; the deciding warp corrects it for the instances
+// picked by decisions s - kSpecLag .. s - 1 (kSpecLag <= kLcpBack, so their common chain prefixes
+// with request s are in RowPre::lcp).
+constexpr int kSpecLag = 8;
+constexpr int kSumWarps = 8;      // warps of a summary block (256 threads)
+constexpr int kKeysPerWarp = 4;   // smallest (key, tie) pairs of C a summary warp publishes
+constexpr int kWPerWarp = 2;      // smallest (W, instance) pairs of A a summary warp publishes
+constexpr uint32_t kSumSlots = 64;  // ring of published summaries (row s in slot s % kSumSlots)
+static_assert(kSpecLag <= kLcpBack, "the corrected picks need their common prefix with the row");
+
+// Summary of row s on the state before decision s - kSpecLag: for each of the kSumWarps warps its
+// kKeysPerWarp smallest packed keys of C (with tie word, W and hit) and its kWPerWarp smallest W of A;
+// every pair of C it does not publish has (key, tie) >= (key_bound, tie_bound), every W of A it does
+// not publish is >= the W bound.  W values travel as order-preserving bits (f2ord).
+struct __align__(16) RowSummary {
+  unsigned long long key[kSumWarps * kKeysPerWarp];  // packed (class, value) keys; kNoKey: none
+  uint32_t tie[kSumWarps * kKeysPerWarp];            // tie words (instance in the low 12 bits)
+  uint32_t word[kSumWarps * kKeysPerWarp];           // f2ord(W) of the pair
+  uint32_t hit[kSumWarps * kKeysPerWarp];            // its hit (blocks)
+  unsigned long long w[kSumWarps * kWPerWarp];       // f2ord(W) << 32 | instance over A; ~0: none
+  unsigned long long key_bound;                      // kNoKey: every pair of C is published
+  uint32_t tie_bound;
+  uint32_t w_bound;                                  // 0xFFFFFFFF: every W of A is published
+  uint32_t wmin;                                     // f2ord(W_min over A), 0xFFFFFFFF: A empty
+  uint32_t pad[3];
+};
+static_assert(sizeof(RowSummary) % 16 == 0, "summaries are copied in 16-byte pieces");
+
 struct GreedySync {
   unsigned long long* jobs;  // [R] 1 << 63 | hit of the pick << 32 | pick (0xFFFFFFFF = rejected); 0 = unpublished
-  uint32_t* done;            // [R] 1 once the job's blocks are in the delta table
+  uint32_t* done;            // [R] insert blocks done with the job (its blocks are all in at the group size)
   uint32_t* ready;           // [R] 1 once the row's probed hits are in the ring
   uint32_t* hitring;         // [kHitSlots][ring_stride] probed hits (row s in slot s % kHitSlots)
   float* tpfring;            // [kHitSlots][ring_stride] T_pf at those hits (kNoTpfBits where it changed)
   uint32_t ring_stride;      // I rounded up to a multiple of 4
   uint64_t wait_ns;          // bound on any cross-block wait (ns); a waiter that gives up sets kErrTimeout
+  RowSummary* sums;          // [kSumSlots] published row summaries
+  uint32_t* sready;          // [R] 1 once row s's summary is published
+  unsigned long long* stats; // [2] rows decided from the summary, rows decided by a full pass
 };
 
 // Window table from a chain's last block hash to the earliest request ending there.
@@ -442,6 +474,19 @@ __device__ __forceinline__ bool delta_contains(const DeltaSlot* delta, uint64_t 
   return delta_contains_from(delta, nslots, inst, key, delta_home(key, nslots));
 }
 
+// Insert (inst, key) at the first empty slot from `slot` on (see delta_insert).
+__device__ __forceinline__ bool delta_insert_from(DeltaSlot* delta, uint64_t nslots, uint32_t inst, uint64_t key,
+                                                  uint64_t slot) {
+  for (uint64_t p = 0; p < nslots; ++p) {
+    if (atomicCAS(&delta[slot].hash, kEmpty, (unsigned long long)key) == kEmpty) {
+      __stcg(&delta[slot].tag, inst + 1);
+      return true;
+    }
+    slot = delta_next(slot, nslots);
+  }
+  return false;
+}
+
 // Insert (inst, key): the first empty slot from the key's home is claimed by compare-and-swap on
 // the hash, then the tag is stored (one round trip).  A lookup racing with the insert may see the
 // slot without its tag and report the pair absent, which only under-reports; it is visible to every
@@ -479,6 +524,20 @@ __device__ __forceinline__ unsigned long long ld_relaxed_u64(const unsigned long
 
 __device__ __forceinline__ void st_relaxed_u64(unsigned long long* p, unsigned long long v) {
   asm volatile("st.relaxed.gpu.global.u64 [%0], %1;" ::"l"(p), "l"(v) : "memory");
+}
+
+// Shared-memory flags between the warps of one block: release store / acquire load at CTA scope
+// (orders this thread's earlier accesses / its later accesses, without waiting for global stores).
+__device__ __forceinline__ void st_release_cta_shared_u32(uint32_t* p, uint32_t v) {
+  asm volatile("st.release.cta.shared::cta.u32 [%0], %1;" ::"r"((uint32_t)__cvta_generic_to_shared(p)), "r"(v)
+               : "memory");
+}
+
+__device__ __forceinline__ uint32_t ld_acquire_cta_shared_u32(const uint32_t* p) {
+  uint32_t v;
+  asm volatile("ld.acquire.cta.shared::cta.u32 %0, [%1];" : "=r"(v) : "r"((uint32_t)__cvta_generic_to_shared(p))
+               : "memory");
+  return v;
 }
 
 __device__ __forceinline__ uint64_t globaltimer_ns() {

@@ -94,11 +94,12 @@ struct Piece {
 
 // Loads a piece's hits and evaluates pass 1: the capacity guard and, for pairs in A, T_pf at the hit
 // and W = T_pf(n, c) - T_pf(0, L).  Returns the order-preserving bits of the lane's W_min over A
-// (all ones if none).
+// (all ones if none).  With a stash (this warp's [Ip] scratch row in shared memory) T_pf of every
+// pair pass 2 will need (all pairs when every per-pair output is wanted, else the pairs in A) is
+// kept there, so pass 2 reads it instead of evaluating it again.
 template <int NV, bool VEC>
-__device__ __forceinline__ uint32_t piece_pass1(const uint32_t* __restrict__ hrow, uint32_t I, uint32_t i_lo,
-                                                const ScoreSmem& s, const psk::DevModel& m, const psk::RowConst& rc,
-                                                Piece<NV>& p) {
+__device__ __forceinline__ void piece_load(const uint32_t* __restrict__ hrow, uint32_t I, uint32_t i_lo,
+                                           const ScoreSmem& s, const psk::RowConst& rc, Piece<NV>& p) {
   const int lane = threadIdx.x & 31;
 #pragma unroll
   for (int v = 0; v < NV; ++v) {
@@ -116,29 +117,45 @@ __device__ __forceinline__ uint32_t piece_pass1(const uint32_t* __restrict__ hro
     }
   }
   p.amask = 0u;
-  uint32_t wbest = 0xFFFFFFFFu;
 #pragma unroll
   for (int v = 0; v < NV; ++v) {
     const uint32_t i = i_lo + 128u * v + 4u * lane;
     int32_t rm[4] = {-1, -1, -1, -1};
     if (i < I) lds4(s.room + i, rm);  // padding past I holds -1
 #pragma unroll
+    for (int k = 0; k < 4; ++k)
+      if ((int32_t)rc.L <= rm[k]) p.amask |= 1u << (4 * v + k);
+  }
+}
+
+template <int NV, bool VEC, bool STASH>
+__device__ __forceinline__ uint32_t piece_pass1(const uint32_t* __restrict__ hrow, uint32_t I, uint32_t i_lo,
+                                                const ScoreSmem& s, const psk::DevModel& m, const psk::RowConst& rc,
+                                                Piece<NV>& p, float* stash, bool all_pairs) {
+  const int lane = threadIdx.x & 31;
+  piece_load<NV, VEC>(hrow, I, i_lo, s, rc, p);
+  uint32_t wbest = 0xFFFFFFFFu;
+#pragma unroll
+  for (int v = 0; v < NV; ++v) {
+    const uint32_t i = i_lo + 128u * v + 4u * lane;
+    float tp[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+#pragma unroll
     for (int k = 0; k < 4; ++k) {
-      if ((int32_t)rc.L <= rm[k]) {
-        p.amask |= 1u << (4 * v + k);
-        wbest = min(wbest, psk::f2ord(__fsub_rn(t_pf32(m, rc.L, p.h[v][k]), rc.t_cached)));
-      }
+      const bool inA = (p.amask >> (4 * v + k)) & 1u;
+      if (inA || (STASH && all_pairs)) tp[k] = t_pf32(m, rc.L, p.h[v][k]);
+      if (inA) wbest = min(wbest, psk::f2ord(__fsub_rn(tp[k], rc.t_cached)));
     }
+    if (STASH && i < I) *reinterpret_cast<float4*>(stash + i) = make_float4(tp[0], tp[1], tp[2], tp[3]);
   }
   return wbest;
 }
 
 // Pass 2 of a piece: classes, optional per-pair outputs, and the lane's best (key, instance, hit).
 // T_pf is evaluated again (the same rounded operations) rather than held in registers.
-template <int NV, bool VEC, bool NARROW>
+template <int NV, bool VEC, bool NARROW, bool GEN, bool STASH>
 __device__ __forceinline__ void piece_pass2(uint32_t I, uint32_t i_lo, uint64_t x0, const ScoreSmem& s,
                                             const psk::DevModel& m, const psk::RowConst& rc, float wmin,
-                                            const Piece<NV>& p, float* __restrict__ tpot_out,
+                                            const Piece<NV>& p, const float* stash, float* __restrict__ tpot_out,
                                             float* __restrict__ ttft_out, uint8_t* __restrict__ cls_out,
                                             uint64_t& bkey, uint32_t& btie, uint32_t& bh) {
   const int lane = threadIdx.x & 31;
@@ -151,9 +168,16 @@ __device__ __forceinline__ void piece_pass2(uint32_t I, uint32_t i_lo, uint64_t 
     bool inC[4];
     float tpf[4];
     bool anyC = false;
+    if (STASH) {
+      const float4 x = *reinterpret_cast<const float4*>(stash + i);
+      tpf[0] = x.x;
+      tpf[1] = x.y;
+      tpf[2] = x.z;
+      tpf[3] = x.w;
+    }
 #pragma unroll
     for (int k = 0; k < 4; ++k) {
-      tpf[k] = (all_pairs || ((am >> k) & 1u)) ? t_pf32(m, rc.L, p.h[v][k]) : 0.0f;
+      if (!STASH) tpf[k] = (all_pairs || ((am >> k) & 1u)) ? t_pf32(m, rc.L, p.h[v][k]) : 0.0f;
       inC[k] = ((am >> k) & 1u) && psk::pair_in_c(rc, __fsub_rn(tpf[k], rc.t_cached), wmin);
       anyC |= inC[k];
     }
@@ -206,13 +230,17 @@ __device__ __forceinline__ void piece_pass2(uint32_t I, uint32_t i_lo, uint64_t 
         const uint32_t h = p.h[v][k];
         uint64_t key;
         uint32_t tie = i + k;
-        if (cls == 0u) {
+        if (!GEN) {  // Algorithm 1's order: D-C-Q in T, the LMetric product in C \ T
+          key = cls == 0u ? psk::packed_key(0u, k0[k] | ((uint64_t)((1u << 26) - 1u - h) << 18))
+                          : psk::packed_key(1u, qn * (uint64_t)(uint32_t)Bp[k]);
+        } else if (cls == 0u) {
           key = psk::packed_key(0u, psk::value_in_t(m, psk::key0_from_dcq(m, k0[k]), h, tp[k], rc.tpot_target));
           if (m.sel == psk::kSelHCQ) tie |= (uint32_t)(k0[k] & 0x3FFFFull) << 12;
         } else {
           key = psk::packed_key(1u, psk::value_fallback(m, qn, (uint32_t)Bp[k], k0[k], h));
         }
-        if (key < bkey || (key == bkey && tie < btie)) {
+        // a lane's instances ascend, so under the default order ties keep the lowest by themselves
+        if (key < bkey || (GEN && key == bkey && tie < btie)) {
           bkey = key;
           btie = tie;
           bh = h;
@@ -237,7 +265,9 @@ __device__ __forceinline__ void piece_pass2(uint32_t I, uint32_t i_lo, uint64_t 
   }
 }
 
-template <int NV, bool VEC>
+constexpr uint32_t kStashMax = 1024;  // rows of up to this many instances keep T_pf in shared memory
+
+template <int NV, bool VEC, bool GEN, bool STASH>
 __global__ void __launch_bounds__(kScoreThreads, 2)
 score_rows_kernel(const uint32_t* __restrict__ hits, psk::StateSoA st, uint32_t I, psk::WindowDev w,
                   psk::DevModel m, float* __restrict__ tpot_out, float* __restrict__ ttft_out,
@@ -246,6 +276,9 @@ score_rows_kernel(const uint32_t* __restrict__ hits, psk::StateSoA st, uint32_t 
   extern __shared__ __align__(16) unsigned long long smem_raw[];
   const uint32_t Ip = (I + 3u) & ~3u;
   const ScoreSmem s = score_smem(smem_raw, Ip);
+  // this warp's T_pf row (after the instance arrays), when rows are short enough
+  float* const stash = STASH ? reinterpret_cast<float*>(s.S32 + Ip) + (threadIdx.x >> 5) * Ip : nullptr;
+  const bool all_pairs = tpot_out || ttft_out || cls_out;
   bool wide = false;  // some instance's q or S is outside [0, 2^30)
   for (uint32_t i = threadIdx.x; i < Ip; i += blockDim.x) {
     if (i < I) {
@@ -286,11 +319,12 @@ score_rows_kernel(const uint32_t* __restrict__ hits, psk::StateSoA st, uint32_t 
     const uint64_t x0 = (uint64_t)r * I;
     const uint32_t* hrow = hits + x0;
     Piece<NV> p;
-    uint32_t wbest = piece_pass1<NV, VEC>(hrow, I, 0u, s, m, rc, p);
+    uint32_t wbest = piece_pass1<NV, VEC, STASH>(hrow, I, 0u, s, m, rc, p, stash, all_pairs);
     for (uint32_t lo = kPiece; lo < I; lo += kPiece) {
       Piece<NV> p2;
-      wbest = min(wbest, piece_pass1<NV, VEC>(hrow, I, lo, s, m, rc, p2));
+      wbest = min(wbest, piece_pass1<NV, VEC, STASH>(hrow, I, lo, s, m, rc, p2, stash, all_pairs));
     }
+    __syncwarp();  // the stash row is read back by other lanes of the warp
     wbest = __reduce_min_sync(0xffffffffu, wbest);
     const bool anyA = wbest != 0xFFFFFFFFu;  // a W of a pair in A is never NaN, so never all ones
     const float wmin = psk::ord2f(wbest);
@@ -298,18 +332,20 @@ score_rows_kernel(const uint32_t* __restrict__ hits, psk::StateSoA st, uint32_t 
     uint32_t btie = 0xFFFFFFFFu, bh = 0u;
     if (one_piece) {
       if (narrow)
-        piece_pass2<NV, VEC, true>(I, 0u, x0, s, m, rc, wmin, p, tpot_out, ttft_out, cls_out, bkey, btie, bh);
+        piece_pass2<NV, VEC, true, GEN, STASH>(I, 0u, x0, s, m, rc, wmin, p, stash, tpot_out, ttft_out, cls_out, bkey, btie, bh);
       else
-        piece_pass2<NV, VEC, false>(I, 0u, x0, s, m, rc, wmin, p, tpot_out, ttft_out, cls_out, bkey, btie, bh);
+        piece_pass2<NV, VEC, false, GEN, STASH>(I, 0u, x0, s, m, rc, wmin, p, stash, tpot_out, ttft_out, cls_out, bkey, btie, bh);
     } else {
       for (uint32_t lo = 0; lo < I; lo += kPiece) {
-        piece_pass1<NV, VEC>(hrow, I, lo, s, m, rc, p);
+        if (STASH) piece_load<NV, VEC>(hrow, I, lo, s, rc, p);
+        else piece_pass1<NV, VEC, false>(hrow, I, lo, s, m, rc, p, nullptr, all_pairs);
         if (narrow)
-          piece_pass2<NV, VEC, true>(I, lo, x0, s, m, rc, wmin, p, tpot_out, ttft_out, cls_out, bkey, btie, bh);
+          piece_pass2<NV, VEC, true, GEN, STASH>(I, lo, x0, s, m, rc, wmin, p, stash, tpot_out, ttft_out, cls_out, bkey, btie, bh);
         else
-          piece_pass2<NV, VEC, false>(I, lo, x0, s, m, rc, wmin, p, tpot_out, ttft_out, cls_out, bkey, btie, bh);
+          piece_pass2<NV, VEC, false, GEN, STASH>(I, lo, x0, s, m, rc, wmin, p, stash, tpot_out, ttft_out, cls_out, bkey, btie, bh);
       }
     }
+    __syncwarp();  // the next row rewrites the stash
     uint64_t key;
     uint32_t tie, hj;
     psk::warp_pick_min(bkey, btie, bh, &key, &tie, &hj);
@@ -326,12 +362,25 @@ cudaError_t score_launch(const uint32_t* hits, psk::StateSoA st, uint32_t I, con
                          const psk::DevModel& m, float* tpot, float* ttft, uint8_t* cls, int32_t* best,
                          uint8_t* path, int num_sms, cudaStream_t s) {
   const uint32_t Ip = (I + 3u) & ~3u;
-  const size_t smem = (size_t)Ip * (3 * sizeof(int64_t) + 7 * sizeof(uint32_t));
+  size_t smem = (size_t)Ip * (3 * sizeof(int64_t) + 7 * sizeof(uint32_t));
+  if (Ip <= kStashMax) smem += (size_t)(kScoreThreads / 32) * Ip * sizeof(float);
   // 16-byte loads of hit rows and stores of TPOT / TTFT rows, 4-byte stores of class rows
   const bool vec = (I & 3u) == 0u && (reinterpret_cast<uintptr_t>(hits) & 15u) == 0u &&
                    (reinterpret_cast<uintptr_t>(tpot) & 15u) == 0u && (reinterpret_cast<uintptr_t>(ttft) & 15u) == 0u &&
                    (reinterpret_cast<uintptr_t>(cls) & 3u) == 0u;
-  auto kern = vec ? score_rows_kernel<NV, true> : score_rows_kernel<NV, false>;
+  const bool gen = m.sel != psk::kSelDCQ || m.fb_dcq;  // not Algorithm 1's order (Table 4 / Table 3 variants)
+  // rows of up to kStashMax instances (every NV < 4 window) keep T_pf in shared memory
+  constexpr bool kCanSkipStash = NV == 4;
+  const bool stash = Ip <= kStashMax || !kCanSkipStash;
+  decltype(&score_rows_kernel<NV, true, true, true>) kern;
+  if (stash)
+    kern = vec ? (gen ? score_rows_kernel<NV, true, true, true> : score_rows_kernel<NV, true, false, true>)
+               : (gen ? score_rows_kernel<NV, false, true, true> : score_rows_kernel<NV, false, false, true>);
+  else
+    kern = vec ? (gen ? score_rows_kernel<NV, true, true, kCanSkipStash ? false : true>
+                      : score_rows_kernel<NV, true, false, kCanSkipStash ? false : true>)
+               : (gen ? score_rows_kernel<NV, false, true, kCanSkipStash ? false : true>
+                      : score_rows_kernel<NV, false, false, kCanSkipStash ? false : true>);
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   const uint32_t rows_per_block = kScoreThreads / 32;

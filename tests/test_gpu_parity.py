@@ -317,3 +317,17 @@ def test_config1_full_parity(P, tpot, mode):
     gd, od = _check_window(P, wl.model, wl.instances, wl.window, commit=(tpot == 50.0), mode=mode)
     counts = np.bincount(od["path"], minlength=3)
     print(f"config 1 tpot {tpot}: packed {counts[0]} fallback {counts[1]} reject {counts[2]}")
+
+
+@pytest.mark.parametrize("mode", MODES)
+@pytest.mark.parametrize("seed,I,R", [(9, 2048, 48), (10, 1537, 33), (11, 2047, 5)])
+def test_random_ragged_windows_at_the_instance_limit(P, seed, I, R, mode):
+    """The largest context ps_create accepts (2048 instances; probe and summary threads then hold 8
+    instances each), and ragged counts just below it."""
+    ins, win = _random_case(seed, I, R)
+    _check_window(P, dict(W.MODEL_DEFAULT), ins, win, mode=mode)
+
+
+def test_instance_limit_is_enforced(P):
+    with pytest.raises(P.PSError):
+        P.Scheduler(2049, np.full(2049, 64, np.uint64), 4, 64, dict(W.MODEL_DEFAULT))
