@@ -312,6 +312,44 @@ PS_API ps_status ps_score_window(ps_ctx* ctx, const ps_window* w, ps_scores* out
 PS_API ps_status ps_schedule_window(ps_ctx* ctx, const ps_window* w, ps_decisions* out,
                              ps_scores* opt_scores);
 
+/* ---- Column-block scoring (one instance pool split over several contexts) ---------------------
+ * Algorithm 1 (Section 6) maps every instance to a pair evaluation and then reduces each request's
+ * row twice: W_min over the capacity-eligible set A (the KVC-first filter's reference, Eq. 8), then
+ * the smallest packing key over C (Section 6.2's order inside T, the LMetric fallback over C when T
+ * is empty).  Both reductions are minima, so a pool whose instances are split into column blocks,
+ * one context each (for instance one per GPU), scores a window in two exchanges:
+ *   1. every block calls ps_shard_wmin; the caller takes the minimum of wmin_ord over the blocks
+ *      (an all-reduce MIN of u32 words);
+ *   2. every block calls ps_shard_pick with that minimum; the caller takes, per request, the
+ *      smallest key over the blocks and, among the blocks holding it, the smallest tie word (two
+ *      all-reduce MINs).  The request's pick is then the tie word's instance id (its low 12 bits
+ *      under PS_SELECT_HCQ, the whole word otherwise), Reject when the key is all ones or the pool's
+ *      W_min is all ones; its path is key >> 62.
+ * The result equals ps_score_window over the whole pool.  The greedy assignment does not split this
+ * way (each decision needs the previous one): ps_schedule_window runs on a context holding the whole
+ * pool.
+ *
+ * ps_shard_wmin: runs the probe phase of ps_score_window on this context's instances and writes, per
+ * request, W_min over this block's A as order-preserving bits (float bits b with the sign bit set ->
+ * ~b, else b | 0x80000000, so unsigned order = float order), 0xFFFFFFFF when the block's A is empty.
+ * wmin_ord [R] is host (on_device 0) or device (1) memory.  The window's hit lengths stay in the
+ * context for the ps_shard_pick that follows; a window with device inputs must stay unchanged until
+ * then.  Errors: as ps_score_window, PS_ERR_INVALID for a NULL wmin_ord. */
+PS_API ps_status ps_shard_wmin(ps_ctx* ctx, const ps_window* w, uint32_t* wmin_ord, int32_t on_device);
+
+/* ps_shard_pick: the second half of the last ps_shard_wmin's window.  wmin_ord [R] is the pool's
+ * W_min (the minimum over the blocks, same encoding); key [R] receives this block's smallest packed
+ * key over C under that W_min (all ones if none): class in the top two bits (0 in T, 1 in C \ T),
+ * then the order's fields, so the unsigned order of keys is Algorithm 1's order; tie [R] receives its
+ * tie word with the pool instance id id_base + local id (all ones if none).  wmin_ord, key and tie are
+ * host (on_device 0) or device (1) memory.  opt (may be NULL) receives this block's columns of
+ * ps_score_window's outputs under the pool's W_min (hits, tpot, ttft, cls; best is this block's own
+ * pick in local ids, path its path).  Must follow ps_shard_wmin with no call in between that scores
+ * or schedules a window or changes the context's state, caches or model (PS_ERR_STATE otherwise).  Errors: PS_ERR_INVALID (NULL arrays,
+ * id_base + num_instances above 2^31 - 1, or above 4096 under PS_SELECT_HCQ), PS_ERR_STATE. */
+PS_API ps_status ps_shard_pick(ps_ctx* ctx, const uint32_t* wmin_ord, uint32_t id_base, uint64_t* key, uint32_t* tie,
+                               int32_t on_device, ps_scores* opt);
+
 /* Commit the pending window (Section 4: the gateway updates the instance records along the
  * request path): the pending state becomes the committed state and each admitted
  * request's uncached blocks are cached on its instance.  With track_lru every block of an admitted
@@ -375,9 +413,14 @@ PS_API ps_status ps_last_timings(ps_ctx* ctx, float* ms, uint32_t n);
  *   out[2] table lookups in scratch rows     out[3] table lookups in derived rows
  *   out[4] chain blocks read from global memory (a lookup's key, or a block staged in shared memory)
  *   out[5] (row, instance) pairs searched past the earlier request's chain (derived rows)
- * With n >= 8, of the last ps_schedule_window in PS_PROBE_SEARCH mode (else 0):
+ * Of the last ps_schedule_window in PS_PROBE_SEARCH mode (else 0), where n reaches them:
  *   out[6] decisions taken from a row summary corrected for the recent picks
  *   out[7] decisions that needed a full pass over the row
+ *   out[8..15] SM clock cycles, summed over the thread blocks of each role of the greedy pass: the
+ *          deciding warp waiting for staged rows, the deciding warp in all, its feeder waiting for a
+ *          free staging slot, the feeder waiting for published row summaries, the summary blocks
+ *          waiting for published decisions, waiting for probed rows, and evaluating rows, the probe
+ *          blocks waiting for the inserts of earlier decisions
  * A table lookup reads the key's two candidate buckets (2 x 64 bytes) and one overflow word.
  * All zero if no probe phase ran.  Synchronises the context's stream. */
 PS_API ps_status ps_last_probe_stats(ps_ctx* ctx, uint64_t* out, uint32_t n);

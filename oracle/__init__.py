@@ -89,6 +89,7 @@ def _lib():
         lib.orc_hit.argtypes = [vp, u32, vp, u64]
         lib.orc_hit_pairs.argtypes = [vp, vp, vp, u64, vp, vp, vp]
         lib.orc_score_rows.argtypes = [vp] * 6 + [u64] + [vp] * 7
+        lib.orc_score_rows_block.argtypes = [vp] * 6 + [u64] + [vp] * 8
         lib.orc_schedule.argtypes = [vp, u32] + [vp] * 9 + [u32]
         lib.orc_set_capacity.argtypes = [vp, vp]
         lib.orc_load_requests.argtypes = [vp, u64, vp, vp, vp, vp, vp]
@@ -218,6 +219,25 @@ class Oracle:
                               _p(_c(window.tpot_target, np.float32)), n, _p(rows),
                               _p(out["hits"]), _p(out["tpot"]), _p(out["ttft"]), _p(out["cls"]),
                               _p(out["best"]), _p(out["path"]))
+        return out
+
+    def score_rows_block(self, window, wmin=None, rows=None) -> dict:
+        """Score mode when this oracle holds one column block of a larger instance pool: returns the
+        block's W_min over A ("wmin", valid where "anyA") and, with ``wmin`` given (the pool's W_min
+        per row), classes and the block's pick under that W_min (block-local ids)."""
+        rows = np.arange(window.R, dtype=np.uint32) if rows is None else _c(rows, np.uint32)
+        n = rows.shape[0]
+        win = None if wmin is None else _c(wmin, np.float32)
+        out = dict(wmin=np.zeros(n, np.float32), anyA=np.zeros(n, np.uint8),
+                   hits=np.zeros((n, self.I), np.uint32), cls=np.zeros((n, self.I), np.uint8),
+                   best=np.zeros(n, np.int32), path=np.zeros(n, np.uint8))
+        _lib().orc_score_rows_block(self._h, _p(_c(window.chain_off, np.uint64)),
+                                    _p(_c(window.chain_hash, np.uint64)),
+                                    _p(_c(window.prompt_tokens, np.uint32)),
+                                    _p(_c(window.ttft_target, np.float32)),
+                                    _p(_c(window.tpot_target, np.float32)), n, _p(rows), _p(win),
+                                    _p(out["wmin"]), _p(out["anyA"]), _p(out["hits"]), _p(out["cls"]),
+                                    _p(out["best"]), _p(out["path"]))
         return out
 
     def schedule(self, window, window_id: int = 0, streaming: bool = False) -> dict:

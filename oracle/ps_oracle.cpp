@@ -132,11 +132,18 @@ struct Row {
   std::vector<uint8_t> cls;    // 0: in T, 1: in C \ T, 2: in A \ C, 3: not in A
   int32_t pick = -1;
   uint8_t path = 2;            // 0 packed (from T), 1 fallback (LMetric over C), 2 reject
+  bool anyA = false;           // A is not empty (over this oracle's instances)
+  float Wmin = 0.f;            // min of W over A (over this oracle's instances), when anyA
 };
+
+// A W_min that replaces the one over this oracle's own instances: the oracle then holds one column
+// block of a larger instance pool, and W_min is the minimum over the whole pool's A (Algorithm 1
+// takes W_min over every capacity-eligible instance).
+struct WminOverride { bool given = false; float Wmin = 0.f; };
 
 // Algorithm 1 for one request against the current caches and state.
 void decide(const Oracle& o, const uint64_t* chain, uint64_t nb, uint32_t L, float ttft_target,
-            float tpot_target, Row& row) {
+            float tpot_target, Row& row, WminOverride ov = WminOverride()) {
   const orc_model& m = o.m;
   const uint32_t I = o.I;
   row.hit.assign(I, 0); row.tpot.assign(I, 0.f); row.ttft.assign(I, 0.f); row.cls.assign(I, 3);
@@ -186,7 +193,10 @@ void decide(const Oracle& o, const uint64_t* chain, uint64_t nb, uint32_t L, flo
     row.tpot[i] = tp;
     row.ttft[i] = tpf[i] + tq;
   }
+  row.anyA = anyA;
+  row.Wmin = Wmin;
   if (!anyA) return;  // Reject (Alg. 1: A empty)
+  if (ov.given) Wmin = ov.Wmin;
   // Normalised recompute filter, Eq. 8; SLO admission (Alg. 1 TPOT filter, plus TTFT budget).
   bool anyT = false;
   for (uint32_t i = 0; i < I; ++i) {
@@ -393,6 +403,33 @@ void orc_score_rows(void* h, const uint64_t* off, const uint64_t* hash, const ui
       if (tpot) tpot[x] = row.tpot[i];
       if (ttft) ttft[x] = row.ttft[i];
       if (cls) cls[x] = row.cls[i];
+    }
+    if (best) best[k] = row.pick;
+    if (path) path[k] = row.path;
+  }
+}
+
+// Score mode over one column block of an instance pool (the oracle holds the block's instances):
+// wmin_out / anyA_out (nullable) receive W_min over the block's A and whether A is not empty;
+// with wmin_in non-null, row k's recompute filter uses W_min = wmin_in[k] (the pool's W_min; not read
+// where the block's A is empty) instead of the block's own.  Other outputs as
+// orc_score_rows; best is the block's pick (a block-local id).
+void orc_score_rows_block(void* h, const uint64_t* off, const uint64_t* hash, const uint32_t* L,
+                          const float* ttft_target, const float* tpot_target, uint64_t nrows,
+                          const uint32_t* rows, const float* wmin_in, float* wmin_out, uint8_t* anyA_out,
+                          uint32_t* hits, uint8_t* cls, int32_t* best, uint8_t* path) {
+  Oracle* o = static_cast<Oracle*>(h);
+  Row row;
+  for (uint64_t k = 0; k < nrows; ++k) {
+    uint32_t r = rows[k];
+    WminOverride ov;
+    if (wmin_in) { ov.given = true; ov.Wmin = wmin_in[k]; }
+    decide(*o, hash + off[r], off[r + 1] - off[r], L[r], ttft_target[r], tpot_target[r], row, ov);
+    if (wmin_out) wmin_out[k] = row.Wmin;
+    if (anyA_out) anyA_out[k] = row.anyA ? 1 : 0;
+    for (uint32_t i = 0; i < o->I; ++i) {
+      if (hits) hits[(size_t)k * o->I + i] = (uint32_t)row.hit[i];
+      if (cls) cls[(size_t)k * o->I + i] = row.cls[i];
     }
     if (best) best[k] = row.pick;
     if (path) path[k] = row.path;

@@ -26,7 +26,8 @@ ABI_FUNCTIONS = ("ps_create", "ps_load_instances", "ps_get_instances", "ps_get_p
                  "ps_calibrate", "ps_get_ema_factors", "ps_set_model", "ps_set_wait_limit",
                  "ps_insert_blocks", "ps_insert_chains", "ps_cached_blocks", "ps_score_window",
                  "ps_schedule_window", "ps_commit_window", "ps_last_timings", "ps_last_probe_stats", "ps_last_error",
-                 "ps_destroy", "ps_score_window_noalloc", "ps_load_requests", "ps_advance_window")
+                 "ps_destroy", "ps_score_window_noalloc", "ps_load_requests", "ps_advance_window",
+                 "ps_shard_wmin", "ps_shard_pick")
 
 
 class PsModel(ctypes.Structure):
@@ -132,6 +133,8 @@ def lib() -> ctypes.CDLL:
             "ps_set_wait_limit": [vp, u64],
             "ps_load_requests": [vp, u64, vp, vp, vp, vp, vp],
             "ps_advance_window": [vp, ctypes.POINTER(PsAdvanceParams)],
+            "ps_shard_wmin": [vp, ctypes.POINTER(PsWindow), vp, i32],
+            "ps_shard_pick": [vp, vp, u32, vp, vp, i32, ctypes.POINTER(PsScores)],
             "ps_score_window_noalloc": [vp, vp, vp, u32, ctypes.POINTER(PsStateArrays), ctypes.POINTER(PsWindow),
                                         ctypes.POINTER(PsModel), i32, ctypes.POINTER(PsScores), vp],
         }
@@ -212,6 +215,7 @@ class Scheduler:
         cfg.cap_blocks = self._cap.ctypes.data
         cfg.table_load_factor = float(table_load_factor)
         cfg.model = make_model(model)
+        self.selector = int(cfg.model.selector)  # the instance order inside T (Table 4)
         cfg.probe_mode = int(probe_mode)
         cfg.track_lru = 1 if track_lru else 0
         cfg.max_active_requests = int(max_active_requests)
@@ -331,6 +335,7 @@ class Scheduler:
         """Replace the performance model (ps_set_model); the EMA factors become the model's."""
         m = make_model(model)
         self._check(lib().ps_set_model(self._h, ctypes.byref(m)))
+        self.selector = int(m.selector)
 
     def set_wait_limit(self, ns: int = 0):
         """Bound on the greedy pass's cross-block waits (ps_set_wait_limit; 0 = the 1-s default)."""
@@ -338,10 +343,12 @@ class Scheduler:
 
     def probe_stats(self) -> dict:
         """Counters of the last probe phase (see ps_last_probe_stats)."""
-        v = np.zeros(8, np.uint64)
-        self._check(lib().ps_last_probe_stats(self._h, v.ctypes.data, 8))
+        v = np.zeros(16, np.uint64)
+        self._check(lib().ps_last_probe_stats(self._h, v.ctypes.data, 16))
         names = ("rows_scratch", "rows_derived", "lookups_scratch", "lookups_derived", "chain_reads",
-                 "pairs_derived", "greedy_fast", "greedy_full")
+                 "pairs_derived", "greedy_fast", "greedy_full", "cyc_decide_wait", "cyc_decide_total",
+                 "cyc_feed_slot_wait", "cyc_feed_summary_wait", "cyc_summary_job_wait",
+                 "cyc_summary_ready_wait", "cyc_summary_eval", "cyc_probe_insert_wait")
         return dict(zip(names, (int(x) for x in v)))
 
     # ------------------------------------------------------------------------------------------
@@ -413,6 +420,38 @@ class Scheduler:
 
     def commit_window(self, last_use: int = 0):
         self._check(lib().ps_commit_window(self._h, int(last_use)))
+
+    # -- column-block scoring (see paper_2609_33224_gb300.shard) -------------------------------
+    def shard_wmin(self, window, device_outputs: bool = False):
+        """ps_shard_wmin: this context's W_min over A per request (order-preserving u32 bits)."""
+        w = self.make_window(window)
+        if device_outputs:
+            import torch
+            out = torch.empty(w.R, dtype=torch.int32, device=f"cuda:{self.device}")
+        else:
+            out = np.zeros(w.R, np.uint32)
+        self._check(lib().ps_shard_wmin(self._h, ctypes.byref(w), _ptr(out)[0], 1 if device_outputs else 0))
+        return out
+
+    def shard_pick(self, wmin_ord, id_base: int, scores=(), device_outputs: bool = False) -> dict:
+        """ps_shard_pick: {key (u64), tie (u32)} per request under the pool's W_min ``wmin_ord`` (host
+        u32 array, or a CUDA int32 tensor with device_outputs), plus this block's ``scores``."""
+        R = wmin_ord.numel() if _is_torch(wmin_ord) else len(wmin_ord)
+        if device_outputs:
+            import torch
+            key = torch.empty(R, dtype=torch.int64, device=f"cuda:{self.device}")
+            tie = torch.empty(R, dtype=torch.int32, device=f"cuda:{self.device}")
+        else:
+            wmin_ord = np.ascontiguousarray(wmin_ord, dtype=np.uint32)
+            key, tie = np.zeros(R, np.uint64), np.zeros(R, np.uint32)
+        so = self._outputs(R, tuple(scores), device_outputs) if scores else {}
+        sc = self._scores_struct(so, device_outputs) if scores else None
+        self._check(lib().ps_shard_pick(self._h, _ptr(wmin_ord)[0], int(id_base), _ptr(key)[0], _ptr(tie)[0],
+                                        1 if device_outputs else 0, ctypes.byref(sc) if sc is not None else None))
+        res = {"key": key, "tie": tie}
+        if scores:
+            res["scores"] = so
+        return res
 
 
 def scheduler_for(workload, max_window_chain_blocks: int | None = None, device: int = 0, stream=None,

@@ -87,6 +87,12 @@ struct ps_ctx {
   unsigned long long* d_stats = nullptr;  // probe launch counters (ps_last_probe_stats)
   bool pending = false;
   psk::WindowDev pend_win{};
+  // column-block scoring: the window of the last ps_shard_wmin, whose hits are in d_hits
+  bool shard_pending = false;
+  psk::WindowDev shard_win{};
+  uint32_t* d_shard_wmin = nullptr;
+  unsigned long long* d_shard_key = nullptr;
+  uint32_t* d_shard_tie = nullptr;
   const uint32_t* pend_out = nullptr;
   // streaming: per-block LRU metadata, request store, capacities on the device, eviction buffers
   bool lru = false;
@@ -324,6 +330,7 @@ ps_status run_probe_and_score(ps_ctx* c, const psk::WindowDev& wd, ps_scores* ou
 void reset_timers(ps_ctx* c) {
   for (bool& u : c->ev_used) u = false;
   c->probe_split = false;
+  c->shard_pending = false;  // the hit buffer is about to be rewritten
 }
 
 }  // namespace
@@ -401,7 +408,7 @@ ps_status ps_create(const ps_config* cfg, ps_ctx** out) {
             dalloc(c, &c->d_delta, (size_t)dn) == cudaSuccess && dalloc(c, &c->gsync.jobs, c->Rmax) == cudaSuccess &&
             dalloc(c, &c->gsync.done, c->Rmax) == cudaSuccess && dalloc(c, &c->gsync.ready, c->Rmax) == cudaSuccess &&
             dalloc(c, &c->gsync.sums, psk::kSumSlots) == cudaSuccess && dalloc(c, &c->gsync.sready, c->Rmax) == cudaSuccess &&
-            dalloc(c, &c->gsync.stats, 2) == cudaSuccess &&
+            dalloc(c, &c->gsync.stats, psk::kGreedyStats) == cudaSuccess &&
             dalloc(c, &c->gsync.hitring, (size_t)psk::kHitSlots * c->gsync.ring_stride) == cudaSuccess &&
             dalloc(c, &c->gsync.tpfring, (size_t)psk::kHitSlots * c->gsync.ring_stride) == cudaSuccess &&
             dalloc(c, &c->d_rows, c->Rmax) == cudaSuccess && dalloc(c, &c->d_lastslot, c->lastslot_n) == cudaSuccess &&
@@ -420,7 +427,8 @@ ps_status ps_create(const ps_config* cfg, ps_ctx** out) {
        dalloc(c, &c->d_best, c->Rmax) == cudaSuccess && dalloc(c, &c->d_path, c->Rmax) == cudaSuccess &&
        dalloc(c, &c->d_assign, c->Rmax) == cudaSuccess && dalloc(c, &c->d_dpath, c->Rmax) == cudaSuccess &&
        dalloc(c, &c->d_hchosen, c->Rmax) == cudaSuccess && dalloc(c, &c->d_err, 1) == cudaSuccess &&
-       dalloc(c, &c->d_stats, kNumStats) == cudaSuccess &&
+       dalloc(c, &c->d_stats, kNumStats) == cudaSuccess && dalloc(c, &c->d_shard_wmin, c->Rmax) == cudaSuccess &&
+       dalloc(c, &c->d_shard_key, c->Rmax) == cudaSuccess && dalloc(c, &c->d_shard_tie, c->Rmax) == cudaSuccess &&
        dalloc(c, &c->d_cap, I) == cudaSuccess && dalloc(c, &c->d_outtok, c->Rmax) == cudaSuccess;
   if (ok && c->lru) {
     for (uint32_t i = 0; i < I; ++i)
@@ -505,6 +513,7 @@ const char* ps_last_error(const ps_ctx* c) { return c ? c->err.c_str() : "null c
 
 ps_status ps_load_instances(ps_ctx* c, const ps_instance_state* s, uint32_t n) {
   if (!c) return PS_ERR_INVALID;
+  c->shard_pending = false;
   if (!s || n != c->I) return fail(c, PS_ERR_INVALID, "need exactly num_instances states");
   const uint32_t I = c->I;
   std::vector<int32_t> b(I), qr(I), bm(I);
@@ -557,6 +566,7 @@ ps_status ps_get_instances(ps_ctx* c, ps_instance_state* out, uint32_t n) {
 ps_status ps_calibrate(ps_ctx* c, uint32_t n, const int32_t* batch, const int64_t* ctx_tokens,
                        const float* measured_ms, float weight) {
   if (!c) return PS_ERR_INVALID;
+  c->shard_pending = false;
   if (!(weight > 0.0f && weight <= 1.0f)) return fail(c, PS_ERR_INVALID, "calibration weight must be in (0, 1]");
   if (n == 0) return PS_OK;
   if (!batch || !ctx_tokens || !measured_ms) return fail(c, PS_ERR_INVALID, "NULL calibration sample array");
@@ -578,6 +588,7 @@ ps_status ps_get_ema_factors(ps_ctx* c, float* out, uint32_t n) {
 
 ps_status ps_set_model(ps_ctx* c, const ps_model* m) {
   if (!c) return PS_ERR_INVALID;
+  c->shard_pending = false;
   if (!m) return fail(c, PS_ERR_INVALID, "NULL model");
   if (check_model(c, *m) != PS_OK) return PS_ERR_INVALID;
   c->model = to_dev(*m);
@@ -600,6 +611,7 @@ ps_status ps_get_pending_instances(ps_ctx* c, ps_instance_state* out, uint32_t n
 ps_status ps_insert_chains(ps_ctx* c, uint64_t nchains, const uint32_t* inst, const uint64_t* off,
                            const uint64_t* hash, const uint64_t* parent, uint32_t last_use, int32_t on_device) {
   if (!c) return PS_ERR_INVALID;
+  c->shard_pending = false;
   if (nchains == 0) return PS_OK;
   if (!inst || !off || !parent || (on_device != 0 && on_device != 1))
     return fail(c, PS_ERR_INVALID, "bad chain arrays");
@@ -654,6 +666,7 @@ ps_status ps_insert_chains(ps_ctx* c, uint64_t nchains, const uint32_t* inst, co
 ps_status ps_insert_blocks(ps_ctx* c, uint32_t inst, const uint64_t* chain, uint64_t n, uint64_t parent_hash,
                            uint32_t last_use) {
   if (!c) return PS_ERR_INVALID;
+  c->shard_pending = false;
   if (n == 0) return PS_OK;
   const uint64_t off[2] = {0, n};
   return ps_insert_chains(c, 1, &inst, off, chain, &parent_hash, last_use, 0);
@@ -680,6 +693,89 @@ ps_status ps_score_window(ps_ctx* c, const ps_window* w, ps_scores* out) {
   uint32_t* hits = nullptr;
   s = run_probe_and_score(c, wd, out, &hits);
   if (s != PS_OK) return s;
+  return finish(c);
+}
+
+ps_status ps_shard_wmin(ps_ctx* c, const ps_window* w, uint32_t* wmin_ord, int32_t on_device) {
+  if (!c) return PS_ERR_INVALID;
+  if (on_device != 0 && on_device != 1) return fail(c, PS_ERR_INVALID, "on_device must be 0 or 1");
+  DeviceGuard g(c->device);
+  reset_timers(c);
+  psk::WindowDev wd{};
+  ps_status s = stage_window(c, w, &wd);
+  if (s != PS_OK) return s;
+  if (wd.R > 0 && !wmin_ord) return fail(c, PS_ERR_INVALID, "wmin_ord is NULL");
+  uint32_t* hits = nullptr;
+  s = run_probe_and_score(c, wd, nullptr, &hits);  // the probe phase only: hits into the context's buffer
+  if (s != PS_OK) return s;
+  psk::ShardIO sh;
+  sh.wmin_out = on_device ? wmin_ord : c->d_shard_wmin;
+  record(c, kEvScore0);
+  PS_TRY_CUDA(c, pskl::launch_score(hits, c->st, c->I, wd, c->model, nullptr, nullptr, nullptr, nullptr, nullptr,
+                                    c->num_sms, c->stream, sh));
+  record(c, kEvScore1);
+  c->ev_used[1] = true;
+  if (!on_device) PS_TRY_CUDA(c, deliver(c, wmin_ord, c->d_shard_wmin, wd.R, 0));
+  s = finish(c);
+  if (s != PS_OK) return s;
+  c->shard_pending = true;
+  c->shard_win = wd;
+  return PS_OK;
+}
+
+ps_status ps_shard_pick(ps_ctx* c, const uint32_t* wmin_ord, uint32_t id_base, uint64_t* key, uint32_t* tie,
+                        int32_t on_device, ps_scores* opt) {
+  if (!c) return PS_ERR_INVALID;
+  if (!c->shard_pending) return fail(c, PS_ERR_STATE, "no window from ps_shard_wmin (or the context changed since)");
+  if (on_device != 0 && on_device != 1) return fail(c, PS_ERR_INVALID, "on_device must be 0 or 1");
+  if (opt && opt->outputs_on_device != 0 && opt->outputs_on_device != 1)
+    return fail(c, PS_ERR_INVALID, "outputs_on_device must be 0 or 1");
+  const psk::WindowDev wd = c->shard_win;
+  if (wd.R > 0 && (!wmin_ord || !key || !tie)) return fail(c, PS_ERR_INVALID, "wmin_ord, key and tie are required");
+  if ((uint64_t)id_base + c->I > (c->model.sel == psk::kSelHCQ ? 4096ull : 0x7FFFFFFFull))
+    return fail(c, PS_ERR_INVALID, "id_base + num_instances too large (4096 under H-C-Q)");
+  DeviceGuard g(c->device);
+  for (bool& u : c->ev_used) u = false;
+  c->probe_split = false;
+  psk::ShardIO sh;
+  sh.id_base = id_base;
+  if (on_device) {
+    sh.wmin_in = wmin_ord;
+    sh.key_out = reinterpret_cast<unsigned long long*>(key);
+    sh.tie_out = tie;
+  } else {
+    if (wd.R) PS_TRY_CUDA(c, cudaMemcpyAsync(c->d_shard_wmin, wmin_ord, wd.R * sizeof(uint32_t), cudaMemcpyHostToDevice,
+                                             c->stream));
+    sh.wmin_in = c->d_shard_wmin;
+    sh.key_out = c->d_shard_key;
+    sh.tie_out = c->d_shard_tie;
+  }
+  const int dev_out = opt ? opt->outputs_on_device : 0;
+  const size_t RI = (size_t)wd.R * c->I;
+  float* tpot = (opt && opt->tpot) ? (dev_out ? opt->tpot : c->d_tpot_o) : nullptr;
+  float* ttft = (opt && opt->ttft) ? (dev_out ? opt->ttft : c->d_ttft_o) : nullptr;
+  uint8_t* cls = (opt && opt->cls) ? (dev_out ? opt->cls : c->d_cls) : nullptr;
+  int32_t* best = (opt && opt->best) ? (dev_out ? opt->best : c->d_best) : nullptr;
+  uint8_t* path = (opt && opt->path) ? (dev_out ? opt->path : c->d_path) : nullptr;
+  record(c, kEvScore0);
+  PS_TRY_CUDA(c, pskl::launch_score(c->d_hits, c->st, c->I, wd, c->model, tpot, ttft, cls, best, path, c->num_sms,
+                                    c->stream, sh));
+  record(c, kEvScore1);
+  c->ev_used[1] = true;
+  if (!on_device) {
+    PS_TRY_CUDA(c, deliver(c, reinterpret_cast<unsigned long long*>(key), c->d_shard_key, wd.R, 0));
+    PS_TRY_CUDA(c, deliver(c, tie, c->d_shard_tie, wd.R, 0));
+  }
+  if (opt) {
+    PS_TRY_CUDA(c, deliver(c, opt->hits, c->d_hits, RI, dev_out));
+    if (!dev_out) {
+      PS_TRY_CUDA(c, deliver(c, opt->tpot, c->d_tpot_o, RI, 0));
+      PS_TRY_CUDA(c, deliver(c, opt->ttft, c->d_ttft_o, RI, 0));
+      PS_TRY_CUDA(c, deliver(c, opt->cls, c->d_cls, RI, 0));
+      PS_TRY_CUDA(c, deliver(c, opt->best, c->d_best, wd.R, 0));
+      PS_TRY_CUDA(c, deliver(c, opt->path, c->d_path, wd.R, 0));
+    }
+  }
   return finish(c);
 }
 
@@ -725,6 +821,7 @@ ps_status ps_schedule_window(ps_ctx* c, const ps_window* w, ps_decisions* out, p
 
 ps_status ps_commit_window(ps_ctx* c, uint32_t last_use) {
   if (!c) return PS_ERR_INVALID;
+  c->shard_pending = false;
   if (!c->pending) return fail(c, PS_ERR_STATE, "no pending window");
   if (c->rq.M && c->pend_win.R && !c->pend_out)
     return fail(c, PS_ERR_INVALID, "request tracking needs the window's out_tokens");
@@ -749,6 +846,7 @@ ps_status ps_commit_window(ps_ctx* c, uint32_t last_use) {
 ps_status ps_load_requests(ps_ctx* c, uint64_t n, const uint32_t* inst, const uint32_t* state, const uint32_t* L,
                            const uint32_t* out, const uint64_t* rem) {
   if (!c) return PS_ERR_INVALID;
+  c->shard_pending = false;
   if (!c->rq.M) return fail(c, PS_ERR_STATE, "context has no request tracking (max_active_requests = 0)");
   if (n && (!inst || !state || !L || !out || !rem)) return fail(c, PS_ERR_INVALID, "request array is NULL");
   const uint32_t I = c->I, M = c->rq.M;
@@ -795,6 +893,7 @@ ps_status ps_load_requests(ps_ctx* c, uint64_t n, const uint32_t* inst, const ui
 
 ps_status ps_advance_window(ps_ctx* c, const ps_advance_params* p) {
   if (!c) return PS_ERR_INVALID;
+  c->shard_pending = false;
   if (!p || !(p->window_ms > 0.0f) || !std::isfinite(p->window_ms) || (p->evict != 0 && p->evict != 1))
     return fail(c, PS_ERR_INVALID, "advance params: window_ms > 0, evict 0 or 1");
   if (c->pending) return fail(c, PS_ERR_STATE, "commit the pending window before advancing");
@@ -829,16 +928,13 @@ ps_status ps_last_probe_stats(ps_ctx* c, uint64_t* out, uint32_t n) {
   if (!out || n < (uint32_t)kNumStats) return fail(c, PS_ERR_INVALID, "need 6 entries");
   DeviceGuard g(c->device);
   unsigned long long v[kNumStats] = {};
-  unsigned long long gs[2] = {};
+  unsigned long long gs[psk::kGreedyStats] = {};
   if (c->ev_used[0]) PS_TRY_CUDA(c, cudaMemcpyAsync(v, c->d_stats, sizeof(v), cudaMemcpyDeviceToHost, c->stream));
   if (c->ev_used[2] && c->search && n >= 8)
     PS_TRY_CUDA(c, cudaMemcpyAsync(gs, c->gsync.stats, sizeof(gs), cudaMemcpyDeviceToHost, c->stream));
   PS_TRY_CUDA(c, cudaStreamSynchronize(c->stream));
   for (int k = 0; k < kNumStats; ++k) out[k] = v[k];
-  if (n >= 8) {
-    out[6] = gs[0];
-    out[7] = gs[1];
-  }
+  for (uint32_t k = 0; k < (uint32_t)psk::kGreedyStats && 6 + k < n; ++k) out[6 + k] = gs[k];
   return PS_OK;
 }
 

@@ -487,6 +487,7 @@ __device__ void probe_rows(const psk::RowPre* __restrict__ rows, const uint64_t*
   const uint32_t t = threadIdx.x;
   const uint32_t NT = blockDim.x;
   const int lane = t & 31, warp = t >> 5, NW = NT >> 5;
+  unsigned long long cyc_done = 0;  // thread 0: cycles spent waiting for inserts
   for (uint32_t i = t; i < I; i += NT) s_end[i] = 0u;
   if (t == 0) {
     s_replayed = 0;
@@ -563,6 +564,7 @@ __device__ void probe_rows(const psk::RowPre* __restrict__ rows, const uint64_t*
     if (warp == 0) {
       // Wait until the inserts of jobs [done, need) are in: the leading run of done flags among the
       // next 32 is taken, and the first one not yet done is waited for.
+      const long long c0 = clock64();
       uint32_t f = s_done;
       bool abort = false;
       while ((int64_t)f < need && !abort) {
@@ -581,6 +583,7 @@ __device__ void probe_rows(const psk::RowPre* __restrict__ rows, const uint64_t*
       if (lane == 0) {
         s_done = f;
         s_abort = abort ? 1 : 0;
+        cyc_done += (unsigned long long)(clock64() - c0);
       }
     }
     __syncthreads();
@@ -623,6 +626,7 @@ __device__ void probe_rows(const psk::RowPre* __restrict__ rows, const uint64_t*
       psk::st_release_u32(sync.ready + s, 1u);
     }
   }
+  if (t == 0 && sync.stats) atomicAdd(sync.stats + psk::kGsProbeDoneWait, cyc_done);
 }
 
 // q and S within [0, 2^30): with L, n < 2^30 the sums S + L and q + n are exact in 32 bits.
@@ -869,9 +873,12 @@ __device__ void summary_rows(const psk::RowPre* __restrict__ rows, uint32_t R, u
   if (t < 16) s_jm[t] = -1;
   if (t == 0) s_abort = 0;
   uint32_t applied = 0;  // decisions [0, applied) are in this block's state
+  unsigned long long cyc_job = 0, cyc_ready = 0, cyc_eval = 0;
   __syncthreads();
   for (uint32_t s = sb; s < R; s += kSummaryBlocks) {
     const int64_t need = (int64_t)s - psk::kSpecLag;  // decisions [0, need) count for row s
+    const long long c0 = clock64();
+    long long c1 = c0;
     if (warp == 0) {
       // Replay decisions [applied, need), 32 at a time: the adds commute; the last lane of each
       // instance refreshes its terms once every add is in.
@@ -901,6 +908,7 @@ __device__ void summary_rows(const psk::RowPre* __restrict__ rows, uint32_t R, u
         __syncwarp();
         applied += nbatch;
       }
+      c1 = clock64();
       if (lane == 0) {
         if (abort) s_abort = 1;
         else if (!wait_flag(sync.ready + s, err, sync.wait_ns)) s_abort = 1;  // the row's probed hits
@@ -909,7 +917,12 @@ __device__ void summary_rows(const psk::RowPre* __restrict__ rows, uint32_t R, u
         reinterpret_cast<uint4*>(&s_row)[lane] = __ldg(reinterpret_cast<const uint4*>(rows + s) + lane);
     }
     __syncthreads();
-    if (s_abort) return;  // block-uniform
+    const long long c2 = clock64();
+    if (t == 0) {
+      cyc_job += (unsigned long long)(c1 - c0);
+      cyc_ready += (unsigned long long)(c2 - c1);
+    }
+    if (s_abort) break;  // block-uniform
     const psk::RowConst rc = row_of(s_row);
     const uint32_t slot = s % psk::kHitSlots;
     // raises from the picks of requests s - kLcpBack .. s - kSpecLag - 1 (older than the lag)
@@ -1038,8 +1051,14 @@ __device__ void summary_rows(const psk::RowPre* __restrict__ rows, uint32_t R, u
       out->wmin = wmin_o;
       __threadfence();  // every warp's entries (written before the barrier) before the flag
       psk::st_release_u32(sync.sready + s, 1u);
+      cyc_eval += (unsigned long long)(clock64() - c2);
     }
     __syncthreads();  // the next row reuses the reduction slots
+  }
+  if (t == 0 && sync.stats) {
+    atomicAdd(sync.stats + psk::kGsSumJobWait, cyc_job);
+    atomicAdd(sync.stats + psk::kGsSumReadyWait, cyc_ready);
+    atomicAdd(sync.stats + psk::kGsSumEval, cyc_eval);
   }
 }
 
@@ -1071,13 +1090,18 @@ __device__ void decide_spec(const psk::RowPre* __restrict__ rows, uint32_t R, ui
 
   if (t >= 32) {
     // ---- feeder -----------------------------------------------------------------------------------
+    unsigned long long cyc_slot = 0, cyc_sum = 0;
     for (uint32_t x = 0; x < R; ++x) {
       const uint32_t slot = x % kFeedRing;
       // lane 0 waits for the slot to be free and the row's summary to be published; the warp follows
       bool ok = true;
       if (lane == 0) {
+        const long long c0 = clock64();
         if (x >= kFeedRing) ok = wait_smem_at_least(&s_consumed, x - kFeedRing + 1, &s_stop, err, sync.wait_ns);
+        const long long c1 = clock64();
         if (ok) ok = wait_flag(sync.sready + x, err, sync.wait_ns);
+        cyc_slot += (unsigned long long)(c1 - c0);
+        cyc_sum += (unsigned long long)(clock64() - c1);
         if (!ok) s_stop = 1;
       }
       ok = __shfl_sync(full, ok ? 1 : 0, 0) != 0;
@@ -1100,6 +1124,10 @@ __device__ void decide_spec(const psk::RowPre* __restrict__ rows, uint32_t R, ui
       psk::cp_async_wait_all();
       __syncwarp();
       if (lane == 0) psk::st_release_cta_shared_u32(&s_fed, x + 1);
+    }
+    if (lane == 0 && sync.stats) {
+      atomicAdd(sync.stats + psk::kGsFeedSlotWait, cyc_slot);
+      atomicAdd(sync.stats + psk::kGsFeedSumWait, cyc_sum);
     }
     return;
   }
@@ -1124,7 +1152,8 @@ __device__ void decide_spec(const psk::RowPre* __restrict__ rows, uint32_t R, ui
   cor.tie = 0xFFFFFFFFu;
   cor.inA = false;
   uint32_t chit = 0u;
-  unsigned long long n_fast = 0, n_full = 0;
+  unsigned long long n_fast = 0, n_full = 0, cyc_wait = 0;
+  const long long cyc_start = clock64();
   // hit of instance c on a row: its probed hit raised to the common prefix with each of the last
   // kLcpBack requests that went to c; `self` raises by lcp[0] too (c taking the request just before)
   auto raised_hit = [&](const psk::RowPre& rw, const uint32_t* hr, uint32_t c, bool self, int shift) {
@@ -1145,7 +1174,9 @@ __device__ void decide_spec(const psk::RowPre* __restrict__ rows, uint32_t R, ui
     const bool has_next = s + 1 < R;
     bool ok = true;
     if (lane == 0) {
+      const long long c0 = clock64();
       ok = wait_smem_at_least(&s_fed, has_next ? s + 2 : s + 1, &s_stop, err, sync.wait_ns);
+      cyc_wait += (unsigned long long)(clock64() - c0);
       if (!ok) s_stop = 1;
     }
     ok = __shfl_sync(full, ok ? 1 : 0, 0) != 0;
@@ -1315,8 +1346,10 @@ __device__ void decide_spec(const psk::RowPre* __restrict__ rows, uint32_t R, ui
     }
   }
   if (lane == 0 && sync.stats) {
-    atomicAdd(sync.stats, n_fast);
-    atomicAdd(sync.stats + 1, n_full);
+    atomicAdd(sync.stats + psk::kGsFast, n_fast);
+    atomicAdd(sync.stats + psk::kGsFull, n_full);
+    atomicAdd(sync.stats + psk::kGsDecideWait, cyc_wait);
+    atomicAdd(sync.stats + psk::kGsDecideTotal, (unsigned long long)(clock64() - cyc_start));
   }
   for (uint32_t i = (uint32_t)lane; i < I; i += 32) {
     pending.b[i] = a.b[i];
@@ -1409,7 +1442,7 @@ cudaError_t launch_greedy_search(const psk::RowPre* rows, const psk::WindowDev& 
   if (e == cudaSuccess) e = cudaMemsetAsync(sync.ready, 0, (size_t)w.R * sizeof(uint32_t), s);
   if (e == cudaSuccess) e = cudaMemsetAsync(sync.sready, 0, (size_t)w.R * sizeof(uint32_t), s);
   if (e == cudaSuccess) e = cudaMemsetAsync(sync.jobs, 0, (size_t)w.R * sizeof(unsigned long long), s);
-  if (e == cudaSuccess && sync.stats) e = cudaMemsetAsync(sync.stats, 0, 2 * sizeof(unsigned long long), s);
+  if (e == cudaSuccess && sync.stats) e = cudaMemsetAsync(sync.stats, 0, psk::kGreedyStats * sizeof(unsigned long long), s);
   if (e != cudaSuccess) return e;
   // every block has 256 threads; probe and summary threads hold IPT = ceil(I / 256) instances each
   const uint32_t ipt = (I + kPipeThreads - 1) / kPipeThreads;

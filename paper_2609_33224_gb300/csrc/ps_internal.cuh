@@ -139,7 +139,17 @@ struct GreedySync {
   uint64_t wait_ns;          // bound on any cross-block wait (ns); a waiter that gives up sets kErrTimeout
   RowSummary* sums;          // [kSumSlots] published row summaries
   uint32_t* sready;          // [R] 1 once row s's summary is published
-  unsigned long long* stats; // [2] rows decided from the summary, rows decided by a full pass
+  unsigned long long* stats; // [kGreedyStats] counters of the pass (below)
+};
+
+// Counters of one greedy pass (GreedySync::stats): decisions taken from a corrected summary and by a
+// full pass, then SM clock cycles summed over the blocks of each role: the deciding warp waiting for
+// staged rows and in all; the feeder waiting for a free ring slot and for published summaries; the
+// summary blocks waiting for published decisions, for probed rows, and evaluating rows; the probe
+// blocks waiting for the inserts of earlier decisions.
+enum : int {
+  kGsFast = 0, kGsFull, kGsDecideWait, kGsDecideTotal, kGsFeedSlotWait, kGsFeedSumWait, kGsSumJobWait,
+  kGsSumReadyWait, kGsSumEval, kGsProbeDoneWait, kGreedyStats
 };
 
 // Window table from a chain's last block hash to the earliest request ending there.
@@ -993,6 +1003,26 @@ __device__ __forceinline__ void warp_pick_min(uint64_t key, uint32_t inst, uint3
 
 }  // namespace psk
 
+namespace psk {
+// Scoring over one column block of an instance pool (the pool's instances split over contexts, one
+// block each).  Algorithm 1 is a map over instances followed by two reductions per request: W_min
+// over A, then the smallest (key, tie) over C.  A block's kernel computes its part of each, and the
+// caller combines them across blocks (a MIN over blocks):
+//   wmin_out  non-null: write the block's W_min over A (f2ord bits, 0xFFFFFFFF = A empty) per request
+//             and stop after it (no classes, latencies or pick);
+//   wmin_in   non-null: use the pool's W_min (f2ord bits, per request) in the recompute filter instead
+//             of the block's own;
+//   key_out, tie_out  non-null: the block's smallest packed key per request (kNoKey if none) and its
+//             tie word with the pool's instance id (id_base + local id; under H-C-Q qr << 12 | id).
+struct ShardIO {
+  const uint32_t* wmin_in = nullptr;
+  uint32_t* wmin_out = nullptr;
+  unsigned long long* key_out = nullptr;
+  uint32_t* tie_out = nullptr;
+  uint32_t id_base = 0;
+};
+}  // namespace psk
+
 // Kernel launchers (one translation unit each).
 namespace pskl {
 // rows (from launch_relations, or nullptr to probe every request from scratch); tpf (nullable)
@@ -1005,7 +1035,7 @@ cudaError_t launch_probe(const uint64_t* slots, const uint64_t* ovf, const psk::
 int probe_max_grid(uint32_t I, int num_sms);
 cudaError_t launch_score(const uint32_t* hits, psk::StateSoA st, uint32_t I, const psk::WindowDev& w,
                          const psk::DevModel& m, float* tpot, float* ttft, uint8_t* cls, int32_t* best,
-                         uint8_t* path, int num_sms, cudaStream_t s);
+                         uint8_t* path, int num_sms, cudaStream_t s, const psk::ShardIO& sh = psk::ShardIO());
 cudaError_t launch_greedy(const uint64_t* slots, const uint64_t* ovf, const psk::TableDesc* tdesc, uint32_t I,
                           const psk::WindowDev& w, const uint32_t* hit0, psk::StateSoA committed,
                           psk::StateSoA pending, const psk::DevModel& m, psk::DeltaSlot* delta,

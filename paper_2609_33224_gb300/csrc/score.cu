@@ -272,7 +272,7 @@ __global__ void __launch_bounds__(kScoreThreads, 2)
 score_rows_kernel(const uint32_t* __restrict__ hits, psk::StateSoA st, uint32_t I, psk::WindowDev w,
                   psk::DevModel m, float* __restrict__ tpot_out, float* __restrict__ ttft_out,
                   uint8_t* __restrict__ cls_out, int32_t* __restrict__ best_out,
-                  uint8_t* __restrict__ path_out) {
+                  uint8_t* __restrict__ path_out, psk::ShardIO sh) {
   extern __shared__ __align__(16) unsigned long long smem_raw[];
   const uint32_t Ip = (I + 3u) & ~3u;
   const ScoreSmem s = score_smem(smem_raw, Ip);
@@ -326,6 +326,12 @@ score_rows_kernel(const uint32_t* __restrict__ hits, psk::StateSoA st, uint32_t 
     }
     __syncwarp();  // the stash row is read back by other lanes of the warp
     wbest = __reduce_min_sync(0xffffffffu, wbest);
+    if (sh.wmin_out) {  // column block, first reduction only
+      if (lane == 0) sh.wmin_out[r] = wbest;
+      __syncwarp();
+      continue;
+    }
+    if (sh.wmin_in) wbest = __ldg(sh.wmin_in + r);  // the pool's W_min
     const bool anyA = wbest != 0xFFFFFFFFu;  // a W of a pair in A is never NaN, so never all ones
     const float wmin = psk::ord2f(wbest);
     uint64_t bkey = psk::kNoKey;
@@ -353,6 +359,10 @@ score_rows_kernel(const uint32_t* __restrict__ hits, psk::StateSoA st, uint32_t 
       const bool pick = anyA && key != psk::kNoKey;
       if (best_out) best_out[r] = pick ? (int32_t)(tie & psk::kTieInstMask) : -1;
       if (path_out) path_out[r] = pick ? (uint8_t)(key >> 62) : (uint8_t)2;
+      if (sh.key_out) {
+        sh.key_out[r] = pick ? key : psk::kNoKey;
+        sh.tie_out[r] = pick ? tie + sh.id_base : 0xFFFFFFFFu;
+      }
     }
   }
 }
@@ -360,7 +370,7 @@ score_rows_kernel(const uint32_t* __restrict__ hits, psk::StateSoA st, uint32_t 
 template <int NV>
 cudaError_t score_launch(const uint32_t* hits, psk::StateSoA st, uint32_t I, const psk::WindowDev& w,
                          const psk::DevModel& m, float* tpot, float* ttft, uint8_t* cls, int32_t* best,
-                         uint8_t* path, int num_sms, cudaStream_t s) {
+                         uint8_t* path, int num_sms, cudaStream_t s, const psk::ShardIO& sh) {
   const uint32_t Ip = (I + 3u) & ~3u;
   size_t smem = (size_t)Ip * (3 * sizeof(int64_t) + 7 * sizeof(uint32_t));
   if (Ip <= kStashMax) smem += (size_t)(kScoreThreads / 32) * Ip * sizeof(float);
@@ -387,7 +397,7 @@ cudaError_t score_launch(const uint32_t* hits, psk::StateSoA st, uint32_t I, con
   uint32_t grid = (w.R + rows_per_block - 1) / rows_per_block;
   const uint32_t cap = (uint32_t)num_sms * 2u;
   if (grid > cap) grid = cap;
-  kern<<<grid, kScoreThreads, smem, s>>>(hits, st, I, w, m, tpot, ttft, cls, best, path);
+  kern<<<grid, kScoreThreads, smem, s>>>(hits, st, I, w, m, tpot, ttft, cls, best, path, sh);
   return cudaGetLastError();
 }
 
@@ -397,11 +407,11 @@ namespace pskl {
 
 cudaError_t launch_score(const uint32_t* hits, psk::StateSoA st, uint32_t I, const psk::WindowDev& w,
                          const psk::DevModel& m, float* tpot, float* ttft, uint8_t* cls, int32_t* best,
-                         uint8_t* path, int num_sms, cudaStream_t s) {
+                         uint8_t* path, int num_sms, cudaStream_t s, const psk::ShardIO& sh) {
   if (w.R == 0) return cudaSuccess;
-  if (I <= 128u) return score_launch<1>(hits, st, I, w, m, tpot, ttft, cls, best, path, num_sms, s);
-  if (I <= 256u) return score_launch<2>(hits, st, I, w, m, tpot, ttft, cls, best, path, num_sms, s);
-  return score_launch<4>(hits, st, I, w, m, tpot, ttft, cls, best, path, num_sms, s);
+  if (I <= 128u) return score_launch<1>(hits, st, I, w, m, tpot, ttft, cls, best, path, num_sms, s, sh);
+  if (I <= 256u) return score_launch<2>(hits, st, I, w, m, tpot, ttft, cls, best, path, num_sms, s, sh);
+  return score_launch<4>(hits, st, I, w, m, tpot, ttft, cls, best, path, num_sms, s, sh);
 }
 
 }  // namespace pskl

@@ -180,6 +180,22 @@ class Instances:
         return int(self.b.shape[0])
 
 
+def column_block(ins: Instances, lo: int, hi: int) -> Instances:
+    """Instances lo .. hi - 1 of a pool as a pool of their own (ids renumbered from 0): the seed
+    chains cached on them and their state."""
+    sel = np.nonzero((ins.chain_inst >= lo) & (ins.chain_inst < hi))[0]
+    lens = np.diff(ins.chain_off)[sel].astype(np.uint64)
+    off = np.zeros(sel.shape[0] + 1, np.uint64)
+    off[1:] = np.cumsum(lens)
+    hashes = [ins.chain_hash[int(ins.chain_off[c]):int(ins.chain_off[c + 1])] for c in sel]
+    return Instances(b=ins.b[lo:hi].copy(), qr=ins.qr[lo:hi].copy(), q=ins.q[lo:hi].copy(),
+                     S=ins.S[lo:hi].copy(), M_KV=ins.M_KV[lo:hi].copy(), B_max=ins.B_max[lo:hi].copy(),
+                     cap_blocks=ins.cap_blocks[lo:hi].copy(),
+                     chain_inst=(ins.chain_inst[sel] - lo).astype(np.uint32), chain_off=off,
+                     chain_hash=(np.concatenate(hashes) if hashes else np.zeros(0, np.uint64)).astype(np.uint64),
+                     chain_parent=ins.chain_parent[sel].copy())
+
+
 @dataclass
 class Workload:
     config: int
