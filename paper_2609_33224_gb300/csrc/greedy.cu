@@ -836,20 +836,29 @@ __device__ __forceinline__ unsigned long long warp_min_u64w(unsigned long long v
   return ((unsigned long long)mhi << 32) | mlo;
 }
 
-// Bounded spin on a shared-memory counter (acquire) until it reaches `want` or *abort is set; false
-// on timeout (error bit set) or abort.
+// Bounded spin on a shared-memory counter until it reaches `want` (then an acquire fence) or *abort
+// is set; false on timeout (error bit set) or abort.  An iteration is one shared load and a compare;
+// the bound is counted in SM cycles, 3 per ns (at least the time limit at any clock up to 3 GHz).
 __device__ __forceinline__ bool wait_smem_at_least(const uint32_t* p, uint32_t want, const volatile int* abort,
                                                    uint32_t* err, uint64_t limit_ns) {
-  if (psk::ld_acquire_cta_shared_u32(p) >= want) return true;
-  const uint64_t t0 = psk::globaltimer_ns();
-  for (;;) {
-    if (psk::ld_acquire_cta_shared_u32(p) >= want) return true;
-    if (*abort) return false;
-    if (psk::globaltimer_ns() - t0 > limit_ns) {
-      atomicOr(err, psk::kErrTimeout);
-      return false;
+  if (psk::ld_relaxed_cta_shared_u32(p) >= want) {
+    psk::fence_acq_rel_cta();
+    return true;
+  }
+  const long long c0 = clock64();
+  const long long lim = (long long)(limit_ns * 3ull);
+  for (uint32_t it = 1;; ++it) {
+    if (psk::ld_relaxed_cta_shared_u32(p) >= want) {
+      psk::fence_acq_rel_cta();
+      return true;
     }
-    __nanosleep(20);
+    if ((it & 31u) == 0u) {
+      if (*abort) return false;
+      if (clock64() - c0 > lim) {
+        atomicOr(err, psk::kErrTimeout);
+        return false;
+      }
+    }
   }
 }
 
@@ -1062,42 +1071,149 @@ __device__ void summary_rows(const psk::RowPre* __restrict__ rows, uint32_t R, u
   }
 }
 
-// Deciding block (warps 0 and 1; the block's other warps return at once).
+// Deciding block: warp 0 decides, warp 1 (the feeder) stages rows in a shared-memory ring, warps 2, 3
+// and 7 (the helpers A, B, C) prepare each step's inputs one step ahead, warp 5 hands decisions to
+// them (and stores each pick's new state and writes the outputs); warps 4 and 6 return at once.  A
+// warp's scheduler is warp id mod 4, so the spinning roles (deciding warp, feeder, warp 5) and the
+// computing ones sit on different schedulers where they can.
+//
+// The decision of request s needs, besides row s's summary, the pairs on row s of the instances
+// picked by decisions s - kSpecLag .. s - 1 under the current state: lane 0 the pick of s - 1, lane k
+// the pick of s - 1 - k.  All but lane 0's depend only on decisions up to s - 2, and lane 0's is the
+// winner of step s - 1 taking request s - 1.  So while step s - 1 is decided, the helpers compute for
+// step s (their phase s - 1, started once decision s - 2 is published):
+//   A[l]  summary entry l of row s - 1 as if it took request s - 1: its state after that, and its
+//         pair on row s;
+//   B[l]  the same for lane l's touched instance of step s - 1;
+//   C[k]  the pick of s - 1 - k (k = 1 .. kSpecLag - 1) on row s under the state after s - 2.
+// Step s then reads lane 0's pair from A, B (or, after a full pass or at the last request, from what
+// the deciding warp computed itself, X) at the winner's index, and lane k's from C[k].  The deciding
+// warp's own path is the W_min and key reductions of the corrected summary (whose entries it loads
+// a step ahead) and one shared-memory publish; the helpers store each pick's new state into the
+// instance arrays and write the decision outputs to global memory.
+struct HelpSlot {
+  PairKey a_pk[32];
+  InstVals a_nv[32];
+  uint32_t a_hit[32];
+  int32_t a_qr[32];
+  PairKey b_pk[psk::kSpecLag];
+  InstVals b_nv[psk::kSpecLag];
+  uint32_t b_hit[psk::kSpecLag];
+  int32_t b_qr[psk::kSpecLag];
+  PairKey c_pk[psk::kSpecLag];
+  uint32_t c_hit[psk::kSpecLag];
+  PairKey x_pk;
+  InstVals x_nv;
+  uint32_t x_hit;
+  int32_t x_qr;
+};
+enum : uint32_t { kSrcA = 0, kSrcB = 1, kSrcX = 2 };
+constexpr uint32_t kLogSlots = 64;  // decisions kept for the helpers (more than kLcpBack + 2)
+
+// hit of instance c on row rw: its probed hit raised to the common prefix with each of the last
+// kLcpBack requests that went to c (hist[k]: the pick of request s - 1 - k, s the step the history is
+// taken at); `self` raises by lcp[0] too (c taking request s).  shift 0: rw is row s (lcp[k2] is with
+// request s - 1 - k2 = hist[k2]); shift 1: rw is row s + 1 (lcp[k2] is with request s - k2 =
+// hist[k2 - 1]).
+__device__ __forceinline__ uint32_t raised_hit(const psk::RowPre& rw, const uint32_t* hr, uint32_t c, bool self, int shift,
+                                               const int32_t (&hist)[psk::kLcpBack]) {
+  uint32_t h = hr[c];
+  if (self && rw.lcp[0] > h) h = rw.lcp[0];
+#pragma unroll
+  for (int k2 = 0; k2 < psk::kLcpBack; ++k2) {
+    const int kk = k2 - shift;
+    if (kk >= 0 && hist[kk < 0 ? 0 : kk] == (int32_t)c && rw.lcp[k2] > h) h = rw.lcp[k2];
+  }
+  return h;
+}
+
+// The as-if values of a decision's winner in a helper slot.
+__device__ __forceinline__ const InstVals& slot_nv(const HelpSlot& hb, uint32_t src, uint32_t idx) {
+  return src == kSrcA ? hb.a_nv[idx] : (src == kSrcB ? hb.b_nv[idx] : hb.x_nv);
+}
+__device__ __forceinline__ int32_t slot_qr(const HelpSlot& hb, uint32_t src, uint32_t idx) {
+  return src == kSrcA ? hb.a_qr[idx] : (src == kSrcB ? hb.b_qr[idx] : hb.x_qr);
+}
+__device__ __forceinline__ uint32_t slot_hit(const HelpSlot& hb, uint32_t src, uint32_t idx) {
+  return src == kSrcA ? hb.a_hit[idx] : (src == kSrcB ? hb.b_hit[idx] : hb.x_hit);
+}
+
+// Instance state v (of an instance with decode batch b, KV capacity M, slot limit Bmax and qr queued
+// requests) after it takes a request of L tokens at hit h: inst_vals_after on given values.
+__device__ __forceinline__ InstVals vals_after(const psk::DevModel& m, int32_t b, int64_t M, int32_t Bmax, int32_t qr0,
+                                               const InstVals& v0, uint32_t L, uint32_t h, int32_t* qr_out) {
+  const int32_t qr = qr0 + 1;
+  InstVals v;
+  v.q = v0.q + (int64_t)L - 16 * (int64_t)h;
+  v.S = v0.S + (int64_t)L;
+  const psk::InstTerms it = psk::inst_terms(m, b, qr, v.q, Bmax);
+  v.dec0 = it.dec0;
+  v.f = it.f;
+  v.tq = it.tq;
+  v.Bp = it.Bp;
+  v.room = it.okB ? psk::kv_room(v.S, M) : -1;
+  v.kd = psk::dcq_key0(b, qr);
+  *qr_out = qr;
+  return v;
+}
+
 __device__ void decide_spec(const psk::RowPre* __restrict__ rows, uint32_t R, uint32_t I, psk::StateSoA committed,
                             psk::StateSoA pending, const psk::DevModel& m, int32_t* assign, uint8_t* __restrict__ path,
                             uint32_t* __restrict__ hit_chosen, uint32_t* err, const psk::GreedySync& sync,
                             unsigned long long* smem_raw) {
-  if (threadIdx.x >= 64) return;
+  const int wid = (int)(threadIdx.x >> 5);
+  if (wid == 4 || wid == 6) return;
   const uint32_t Ip = sync.ring_stride;
   const InstSmem a = inst_smem(smem_raw, Ip);
   uint32_t* s_hitr = reinterpret_cast<uint32_t*>(a.Bmax + Ip);  // [kFeedRing][Ip] probed hits
   uint32_t* s_tpfr = s_hitr + kFeedRing * Ip;                   // [kFeedRing][Ip] T_pf at them (bits)
   __shared__ psk::RowSummary s_sum[kFeedRing];
   __shared__ psk::RowPre s_rowc[kFeedRing];
+  __shared__ HelpSlot s_help[2];               // helper phase p writes s_help[p & 1]
+  __shared__ int32_t s_logpick[kLogSlots];     // decision x: its pick (-1 rejected) ...
+  __shared__ uint32_t s_logsrc[kLogSlots];     // ... where its as-if values are (kSrc*) and at which index
+  __shared__ uint32_t s_logidx[kLogSlots];
+  __shared__ uint32_t s_loghit[kLogSlots];     // ... its hit and path (the decision outputs)
+  __shared__ uint32_t s_logpath[kLogSlots];
   __shared__ uint32_t s_fed;       // rows [0, s_fed) are staged (release / acquire)
-  __shared__ uint32_t s_consumed;  // rows [0, s_consumed) are decided (release / acquire)
-  __shared__ volatile int s_stop;           // the feeder or the decider gave up
+  __shared__ uint32_t s_dec;       // decisions [0, s_dec) are published (their rows are consumed)
+  __shared__ uint32_t s_stored;    // the state after decisions [0, s_stored) is in the instance arrays
+  __shared__ uint32_t s_ph[3];     // helper w (A, B, C) finished phases [0, s_ph[w])
+  __shared__ int s_hgo[2];         // helper phase p goes ahead (s_hgo[p & 1]), set before its barrier
+  __shared__ volatile int s_stop;  // a role gave up (a bounded wait ran out)
   const uint32_t t = threadIdx.x;
-  const int lane = (int)(t & 31u);
+  const int lane = (int)(t & 31u), warp = (int)(t >> 5);
   const unsigned full = 0xffffffffu;
-  for (uint32_t i = t; i < I; i += 64) inst_load(a, committed, m, i);
+  if (t < 64)
+    for (uint32_t i = t; i < I; i += 64) inst_load(a, committed, m, i);
   if (t == 0) {
     s_fed = 0u;
-    s_consumed = 0u;
+    s_dec = 0u;
+    s_stored = 0u;
+    s_ph[0] = 0u;
+    s_ph[1] = 0u;
+    s_ph[2] = 0u;
     s_stop = 0;
   }
-  asm volatile("bar.sync 1, 64;" ::: "memory");
+  asm volatile("bar.sync 1, 192;" ::: "memory");  // warps 0, 1, 2, 3, 5, 7
 
-  if (t >= 32) {
-    // ---- feeder -----------------------------------------------------------------------------------
+  if (warp == 1) {
+    // ---- feeder ---------------------------------------------------------------------------------
+    // Row x's slot held row x - kFeedRing, which the deciding warp reads up to its decision
+    // x - kFeedRing and the helpers up to their phase x - kFeedRing.
     unsigned long long cyc_slot = 0, cyc_sum = 0;
     for (uint32_t x = 0; x < R; ++x) {
       const uint32_t slot = x % kFeedRing;
-      // lane 0 waits for the slot to be free and the row's summary to be published; the warp follows
       bool ok = true;
       if (lane == 0) {
         const long long c0 = clock64();
-        if (x >= kFeedRing) ok = wait_smem_at_least(&s_consumed, x - kFeedRing + 1, &s_stop, err, sync.wait_ns);
+        if (x >= kFeedRing) {
+          const uint32_t want = x - kFeedRing + 1;
+          ok = wait_smem_at_least(&s_dec, want, &s_stop, err, sync.wait_ns) &&
+               wait_smem_at_least(&s_ph[0], want, &s_stop, err, sync.wait_ns) &&
+               wait_smem_at_least(&s_ph[1], want, &s_stop, err, sync.wait_ns) &&
+               wait_smem_at_least(&s_ph[2], want, &s_stop, err, sync.wait_ns);
+        }
         const long long c1 = clock64();
         if (ok) ok = wait_flag(sync.sready + x, err, sync.wait_ns);
         cyc_slot += (unsigned long long)(c1 - c0);
@@ -1132,42 +1248,151 @@ __device__ void decide_spec(const psk::RowPre* __restrict__ rows, uint32_t R, ui
     return;
   }
 
+  if (warp >= 2) {
+    // ---- helpers ----------------------------------------------------------------------------------
+    // Phase p (p = 0 .. R): once decision p - 1 is published, warp 5 stores its pick's new state and
+    // writes its outputs, and for p < R - 1 the helpers compute A (warp 2), B (warp 3) and C (warp 7)
+    // for step p + 1 into s_help[p & 1].  Lanes whose instance is the pick of p - 1 take its state from
+    // the winner's as-if values, so nothing waits for the store: the others' instances were not
+    // picked at p - 1.
+    const int role = warp == 2 ? 0 : (warp == 3 ? 1 : (warp == 7 ? 2 : 3));  // 3: warp 5
+    for (uint32_t p = 0; p <= R; ++p) {
+      if (role == 3 && lane == 0) {
+        bool ok = wait_smem_at_least(&s_dec, p, &s_stop, err, sync.wait_ns);
+        if (ok && p < R) ok = wait_smem_at_least(&s_fed, p + 2 < R ? p + 2 : R, &s_stop, err, sync.wait_ns);
+        if (!ok) s_stop = 1;
+        s_hgo[p & 1u] = ok ? 1 : 0;
+      }
+      asm volatile("bar.sync 2, 128;" ::: "memory");  // warps 2, 3, 5, 7
+      if (!s_hgo[p & 1u]) break;  // uniform across the helper warps
+      const HelpSlot& hp = s_help[(p - 1) & 1u];  // phase p - 1's slot (p >= 1)
+      const uint32_t xp = (p - 1) % kLogSlots;     // decision p - 1 in the log (p >= 1)
+      int32_t j0 = -1;                              // the pick of p - 1
+      uint32_t src0 = kSrcX, idx0 = 0u;
+      if (p >= 1) {
+        j0 = s_logpick[xp];
+        src0 = s_logsrc[xp];
+        idx0 = s_logidx[xp];
+      }
+      if (role == 3) {
+        if (lane == 0) {
+          if (j0 >= 0) inst_store(a, (uint32_t)j0, slot_qr(hp, src0, idx0), slot_nv(hp, src0, idx0));
+          psk::st_release_cta_shared_u32(&s_stored, p);
+        } else if (lane == 1 && p >= 1) {
+          assign[p - 1] = j0;
+          path[p - 1] = (uint8_t)s_logpath[xp];
+          hit_chosen[p - 1] = s_loghit[xp];
+        }
+        continue;
+      }
+      if (p == R) break;
+      if (p + 1 >= R) {  // no row R: nothing to compute
+        __syncwarp();
+        if (lane == 0) psk::st_release_cta_shared_u32(&s_ph[role], p + 1);
+        continue;
+      }
+      int32_t hist[psk::kLcpBack];
+#pragma unroll
+      for (int k = 0; k < psk::kLcpBack; ++k)
+        hist[k] = (int64_t)p - 1 - k >= 0 ? s_logpick[(p - 1 - k) % kLogSlots] : -1;
+      const uint32_t slot = p % kFeedRing, slot1 = (p + 1) % kFeedRing;
+      const psk::RowPre& row = s_rowc[slot];
+      const psk::RowPre& row1 = s_rowc[slot1];
+      const psk::RowConst rc1 = row_of(row1);
+      const uint32_t* hrow1 = s_hitr + slot1 * Ip;
+      const uint32_t* trow1 = s_tpfr + slot1 * Ip;
+      HelpSlot& out = s_help[p & 1u];
+      // instance c (state v0, qr0) taking request p at hit h: its state after, and its pair on row p + 1
+      auto as_if = [&](uint32_t c, const InstVals& v0, int32_t qr0, uint32_t h, PairKey* pk, InstVals* nv,
+                       uint32_t* hit, int32_t* qr) {
+        *nv = vals_after(m, a.b[c], a.M[c], a.Bmax[c], qr0, v0, row.L, h, qr);
+        *hit = raised_hit(row1, hrow1, c, true, 1, hist);
+        *pk = pair_key_v(m, rc1, *nv, c, *hit, *hit == hrow1[c] ? trow1[c] : psk::kNoTpfBits);
+      };
+      if (role == 0) {
+        // A: summary entry `lane` of row p, when no decision of the last kSpecLag picked it (its state
+        // is then the one in the instance arrays)
+        const psk::RowSummary& sm = s_sum[slot];
+        const uint64_t ek = sm.key[lane];
+        const uint32_t e = sm.tie[lane] & psk::kTieInstMask;
+        bool touched = false;
+#pragma unroll
+        for (int k = 0; k < psk::kSpecLag; ++k) touched |= hist[k] == (int32_t)e;
+        if (ek != psk::kNoKey && !touched) {
+          PairKey pk;
+          InstVals nv;
+          uint32_t hit;
+          int32_t qr;
+          as_if(e, inst_vals(a, e), a.qr[e], sm.hit[lane], &pk, &nv, &hit, &qr);
+          out.a_pk[lane] = pk;
+          out.a_nv[lane] = nv;
+          out.a_hit[lane] = hit;
+          out.a_qr[lane] = qr;
+        }
+      } else if (role == 1) {
+        // B: lane's touched instance of step p (the pick of p - 1 - lane) as if it took request p, at
+        // its hit on row p (from phase p - 1)
+        const int32_t u = lane < psk::kSpecLag && (int64_t)p - 1 - lane >= 0 ? s_logpick[(p - 1 - lane) % kLogSlots] : -1;
+        if (u >= 0) {
+          PairKey pk;
+          InstVals nv;
+          uint32_t hit;
+          int32_t qr;
+          // lane 0's instance is the pick of p - 1: its state is the winner's as-if values (one call for
+          // every lane, so the lanes do not diverge)
+          const InstVals v0 = lane == 0 ? slot_nv(hp, src0, idx0) : inst_vals(a, (uint32_t)u);
+          const int32_t qr0 = lane == 0 ? slot_qr(hp, src0, idx0) : a.qr[u];
+          const uint32_t h0 = lane == 0 ? slot_hit(hp, src0, idx0) : hp.c_hit[lane];
+          as_if((uint32_t)u, v0, qr0, h0, &pk, &nv, &hit, &qr);
+          out.b_pk[lane] = pk;
+          out.b_nv[lane] = nv;
+          out.b_hit[lane] = hit;
+          out.b_qr[lane] = qr;
+        }
+      } else {
+        // C: the pick of p - k (k = lane, 1 .. kSpecLag - 1) on row p + 1, current state
+        const int k = lane;
+        const int32_t u = k >= 1 && k < psk::kSpecLag && (int64_t)p - k >= 0 ? s_logpick[(p - k) % kLogSlots] : -1;
+        if (u >= 0) {
+          const uint32_t h = raised_hit(row1, hrow1, (uint32_t)u, false, 1, hist);
+          const uint32_t tb = h == hrow1[u] ? trow1[u] : psk::kNoTpfBits;
+          out.c_pk[k] = pair_key_v(m, rc1, k == 1 ? slot_nv(hp, src0, idx0) : inst_vals(a, (uint32_t)u), (uint32_t)u, h, tb);
+          out.c_hit[k] = h;
+        }
+      }
+      __syncwarp();
+      if (lane == 0) psk::st_release_cta_shared_u32(&s_ph[role], p + 1);
+    }
+    return;
+  }
+
   // ---- deciding warp --------------------------------------------------------------------------------
-  // Carried from step s to step s + 1 (software pipelining: what step s + 1 needs of its touched
-  // instances is computed in step s, beside step s's reductions):
-  //   pk          lane k < kLcpBack: the pick of request s - 1 - k (-1: none or rejected)
-  //   hist        the same picks in every lane
-  //   cor, chit   lane k < kSpecLag: that instance's pair (key, tie, W, capacity) and hit on row s on
-  //               the current state.  Lane 0's is the pick of request s - 1, which each candidate lane
-  //               of step s - 1 evaluated as if it were picked; lanes 1 .. kSpecLag - 1 evaluated
-  //               theirs on row s in step s - 1 (stale only when step s - 1 picked the same instance,
-  //               and then lane 0 holds it and the duplicate is dropped).
+  //   pk     lane k < kLcpBack: the pick of request s - 1 - k (-1: none or rejected)
+  //   hist   the same picks in every lane
+  //   cor    lane k < kSpecLag: that instance's pair on row s under the current state, chit its hit
+  //   e*, w* this lane's summary entries of row s, loaded a step ahead
   int32_t pk = -1;
   int32_t hist[psk::kLcpBack];
 #pragma unroll
   for (int k = 0; k < psk::kLcpBack; ++k) hist[k] = -1;
-  PairKey cor;
-  cor.W = 0.0f;
-  cor.key = psk::kNoKey;
-  cor.tie = 0xFFFFFFFFu;
-  cor.inA = false;
-  uint32_t chit = 0u;
+  uint32_t w_src = kSrcA, w_idx = 0;  // where the previous winner's as-if values are
   unsigned long long n_fast = 0, n_full = 0, cyc_wait = 0;
   const long long cyc_start = clock64();
-  // hit of instance c on a row: its probed hit raised to the common prefix with each of the last
-  // kLcpBack requests that went to c; `self` raises by lcp[0] too (c taking the request just before)
-  auto raised_hit = [&](const psk::RowPre& rw, const uint32_t* hr, uint32_t c, bool self, int shift) {
-    const uint32_t hb = hr[c];
-    uint32_t h = hb;
-    if (self && rw.lcp[0] > h) h = rw.lcp[0];
-#pragma unroll
-    for (int k2 = 0; k2 < psk::kLcpBack; ++k2) {
-      // shift 0: lcp[k2] is with request s - 1 - k2 = hist[k2]; shift 1 (the next row): lcp[k2] is with
-      // request s - k2 = hist[k2 - 1]
-      const int kk = k2 - shift;
-      if (kk >= 0 && hist[kk < 0 ? 0 : kk] == (int32_t)c && rw.lcp[k2] > h) h = rw.lcp[k2];
-    }
-    return h;
+  uint64_t ek = psk::kNoKey, wv = ~0ull, kbound = psk::kNoKey;
+  uint32_t et = 0u, ew = 0u, eh = 0u, wbound = 0u, wsum = 0u, tbound = 0u;
+  psk::RowConst rc{};
+  auto load_row = [&](uint32_t x) {
+    const psk::RowSummary& sm = s_sum[x % kFeedRing];
+    ek = sm.key[lane];
+    et = sm.tie[lane];
+    ew = sm.word[lane];
+    eh = sm.hit[lane];
+    wv = lane < psk::kSumWarps * psk::kWPerWarp ? sm.w[lane] : ~0ull;
+    wbound = sm.w_bound;
+    wsum = sm.wmin;
+    kbound = sm.key_bound;
+    tbound = sm.tie_bound;
+    rc = row_of(s_rowc[x % kFeedRing]);
   };
   for (uint32_t s = 0; s < R; ++s) {
     const uint32_t slot = s % kFeedRing;
@@ -1176,17 +1401,33 @@ __device__ void decide_spec(const psk::RowPre* __restrict__ rows, uint32_t R, ui
     if (lane == 0) {
       const long long c0 = clock64();
       ok = wait_smem_at_least(&s_fed, has_next ? s + 2 : s + 1, &s_stop, err, sync.wait_ns);
+      if (ok && s >= 1)
+        ok = wait_smem_at_least(&s_ph[0], s, &s_stop, err, sync.wait_ns) &&
+             wait_smem_at_least(&s_ph[1], s, &s_stop, err, sync.wait_ns) &&
+             wait_smem_at_least(&s_ph[2], s, &s_stop, err, sync.wait_ns);
       cyc_wait += (unsigned long long)(clock64() - c0);
       if (!ok) s_stop = 1;
     }
     ok = __shfl_sync(full, ok ? 1 : 0, 0) != 0;
     __syncwarp();
     if (!ok) break;  // warp-uniform
-    const psk::RowPre& row = s_rowc[slot];
-    const psk::RowSummary& sm = s_sum[slot];
-    const uint32_t* hrow = s_hitr + slot * Ip;
-    const uint32_t* trow = s_tpfr + slot * Ip;
-    const psk::RowConst rc = row_of(row);
+    if (s == 0) load_row(0);
+    PairKey cor;
+    cor.W = 0.0f;
+    cor.key = psk::kNoKey;
+    cor.tie = 0xFFFFFFFFu;
+    cor.inA = false;
+    uint32_t chit = 0u;
+    if (s >= 1 && lane < psk::kSpecLag && pk >= 0) {
+      const HelpSlot& hb = s_help[(s - 1) & 1u];
+      if (lane == 0) {
+        cor = w_src == kSrcA ? hb.a_pk[w_idx] : (w_src == kSrcB ? hb.b_pk[w_idx] : hb.x_pk);
+        chit = slot_hit(hb, w_src, w_idx);
+      } else {
+        cor = hb.c_pk[lane];
+        chit = hb.c_hit[lane];
+      }
+    }
     auto touched = [&](uint32_t i) {
       bool r = false;
 #pragma unroll
@@ -1198,78 +1439,59 @@ __device__ void decide_spec(const psk::RowPre* __restrict__ rows, uint32_t R, ui
     const unsigned same = __match_any_sync(full, tk);
     const bool corr = tk >= 0 && (__ffs(same) - 1) == lane;
     // W_min of the current state
-    const unsigned long long wv = lane < psk::kSumWarps * psk::kWPerWarp ? sm.w[lane] : ~0ull;
     const bool w_untouched = wv != ~0ull && !touched((uint32_t)wv);
     const uint32_t mu = __reduce_min_sync(full, w_untouched ? (uint32_t)(wv >> 32) : 0xFFFFFFFFu);
     const uint32_t mt = __reduce_min_sync(full, (corr && cor.inA) ? psk::f2ord(cor.W) : 0xFFFFFFFFu);
     uint32_t wmin_o = min(mu, mt);
     bool anyA = wmin_o != 0xFFFFFFFFu;
-    bool fast = sm.w_bound == 0xFFFFFFFFu || mu <= sm.w_bound;
-    if (fast && anyA && rc.Z > 0.0f && wmin_o > sm.wmin) fast = false;
+    bool fast = wbound == 0xFFFFFFFFu || mu <= wbound;
+    if (fast && anyA && rc.Z > 0.0f && wmin_o > wsum) fast = false;
     // this lane's candidate: its summary entry or its touched instance, whichever is smaller
     uint64_t bk = psk::kNoKey;
-    uint32_t bt = 0xFFFFFFFFu, bh = 0u;
+    uint32_t bt = 0xFFFFFFFFu, bh = 0u, bsrc = kSrcA;
     if (fast && anyA) {
       const float wmin = psk::ord2f(wmin_o);
-      const uint64_t ek = sm.key[lane];
-      const uint32_t et = sm.tie[lane];
-      if (ek != psk::kNoKey && !touched(et & psk::kTieInstMask) && psk::pair_in_c(rc, psk::ord2f(sm.word[lane]), wmin)) {
+      if (ek != psk::kNoKey && !touched(et & psk::kTieInstMask) && psk::pair_in_c(rc, psk::ord2f(ew), wmin)) {
         bk = ek;
         bt = et;
-        bh = sm.hit[lane];
+        bh = eh;
       }
       if (corr && cor.inA && psk::pair_in_c(rc, cor.W, wmin) && kt_less(cor.key, cor.tie, bk, bt)) {
         bk = cor.key;
         bt = cor.tie;
         bh = chit;
-      }
-    }
-    // next row, computed beside this row's reductions: (a) this lane's candidate as the pick of
-    // request s (its state after the pick, its pair on row s + 1); (b) lanes 1 .. kSpecLag - 1: the
-    // instance picked by request s - lane, on row s + 1 with its current state
-    const uint32_t slot1 = (s + 1) % kFeedRing;
-    const psk::RowPre& row1 = s_rowc[slot1];
-    const uint32_t* hrow1 = s_hitr + slot1 * Ip;
-    const uint32_t* trow1 = s_tpfr + slot1 * Ip;
-    const int32_t u = __shfl_up_sync(full, pk, 1);  // lane k >= 1: the pick of request s - k
-    PairKey nx, nt;
-    nx.W = nt.W = 0.0f;
-    nx.key = nt.key = psk::kNoKey;
-    nx.tie = nt.tie = 0xFFFFFFFFu;
-    nx.inA = nt.inA = false;
-    uint32_t nxh = 0u, nth = 0u;
-    InstVals nv;
-    int32_t nqr = 0;
-    if (bk != psk::kNoKey) nv = inst_vals_after(a, m, bt & psk::kTieInstMask, rc.L, bh, &nqr);
-    if (has_next) {
-      const psk::RowConst rc1 = row_of(row1);
-      if (bk != psk::kNoKey) {
-        const uint32_t c = bt & psk::kTieInstMask;
-        nxh = raised_hit(row1, hrow1, c, true, 1);
-        nx = pair_key_v(m, rc1, nv, c, nxh, nxh == hrow1[c] ? trow1[c] : psk::kNoTpfBits);
-      }
-      if (lane >= 1 && lane < psk::kSpecLag && u >= 0) {
-        const uint32_t c = (uint32_t)u;
-        nth = raised_hit(row1, hrow1, c, false, 1);
-        nt = pair_key_of(m, rc1, a, c, nth, nth == hrow1[c] ? trow1[c] : psk::kNoTpfBits);
+        bsrc = kSrcB;
       }
     }
     uint64_t K = psk::kNoKey;
     uint32_t T = 0xFFFFFFFFu, H = 0u;
     if (fast && anyA) {
       psk::warp_pick_min(bk, bt, bh, &K, &T, &H);
-      fast = K != psk::kNoKey && (sm.key_bound == psk::kNoKey || kt_less(K, T, sm.key_bound, sm.tie_bound));
+      fast = K != psk::kNoKey && (kbound == psk::kNoKey || kt_less(K, T, kbound, tbound));
     }
     const bool won = fast && bk != psk::kNoKey && bk == K && bt == T;  // one lane at most (tie words are unique)
+    const psk::RowPre& row = s_rowc[slot];
+    const uint32_t* hrow = s_hitr + slot * Ip;
+    const uint32_t* trow = s_tpfr + slot * Ip;
+    bool stored = false;  // the state after decision s - 1 is known to be in the instance arrays
     if (fast) {
       ++n_fast;
     } else {
-      // full pass over the row on the current state
+      // full pass over the row on the current state (which needs the previous pick's state stored)
       ++n_full;
+      bool ok2 = true;
+      if (lane == 0) {
+        ok2 = wait_smem_at_least(&s_stored, s, &s_stop, err, sync.wait_ns);
+        if (!ok2) s_stop = 1;
+      }
+      ok2 = __shfl_sync(full, ok2 ? 1 : 0, 0) != 0;
+      __syncwarp();
+      if (!ok2) break;  // warp-uniform
+      stored = true;
       uint32_t wo = 0xFFFFFFFFu;
       for (uint32_t i = (uint32_t)lane; i < I; i += 32) {
         if ((int32_t)rc.L <= a.room[i]) {
-          const uint32_t h = raised_hit(row, hrow, i, false, 0);
+          const uint32_t h = raised_hit(row, hrow, i, false, 0, hist);
           const float tpf = (h == hrow[i] && trow[i] != psk::kNoTpfBits) ? __uint_as_float(trow[i]) : psk::t_pf32(m, rc.L, h);
           wo = min(wo, psk::f2ord(__fsub_rn(tpf, rc.t_cached)));
         }
@@ -1281,7 +1503,7 @@ __device__ void decide_spec(const psk::RowPre* __restrict__ rows, uint32_t R, ui
       uint32_t ft = 0xFFFFFFFFu, fh = 0u;
       if (anyA) {
         for (uint32_t i = (uint32_t)lane; i < I; i += 32) {
-          const uint32_t h = raised_hit(row, hrow, i, false, 0);
+          const uint32_t h = raised_hit(row, hrow, i, false, 0, hist);
           const PairKey p = pair_key_of(m, rc, a, i, h, h == hrow[i] ? trow[i] : psk::kNoTpfBits);
           if (p.inA && psk::pair_in_c(rc, p.W, wmin) && kt_less(p.key, p.tie, fk, ft)) {
             fk = p.key;
@@ -1295,55 +1517,59 @@ __device__ void decide_spec(const psk::RowPre* __restrict__ rows, uint32_t R, ui
     const bool pick = anyA && K != psk::kNoKey;
     const uint32_t j = T & psk::kTieInstMask;
     if (!pick) H = 0u;
-    __syncwarp();  // every lane's reads of this step are done before the pick's state changes
-    // the pick's state after the decision, and its pair on row s + 1 for lane 0 of the next step
-    PairKey pn;
-    uint32_t pnh = 0u;
+    // where the pick's as-if values (its state after this decision, its pair on row s + 1) are
+    uint32_t src = kSrcX, idx = 0u;
     const unsigned wm = __ballot_sync(full, won);
-    if (wm) {
+    if (wm && has_next) {
       const int wl = __ffs(wm) - 1;
-      if (won) inst_store(a, j, nqr, nv);
-      pn.W = __shfl_sync(full, nx.W, wl);
-      pn.key = ((uint64_t)__shfl_sync(full, (uint32_t)(nx.key >> 32), wl) << 32) | __shfl_sync(full, (uint32_t)nx.key, wl);
-      pn.tie = __shfl_sync(full, nx.tie, wl);
-      pn.inA = __shfl_sync(full, nx.inA ? 1 : 0, wl) != 0;
-      pnh = __shfl_sync(full, nxh, wl);
-    } else {
-      pn.W = 0.0f;
-      pn.key = psk::kNoKey;
-      pn.tie = 0xFFFFFFFFu;
-      pn.inA = false;
-      if (pick && lane == 0) {
-        int32_t qr2;
-        const InstVals v2 = inst_vals_after(a, m, j, rc.L, H, &qr2);
-        inst_store(a, j, qr2, v2);
-        if (has_next) {
-          pnh = raised_hit(row1, hrow1, j, true, 1);
-          pn = pair_key_v(m, row_of(row1), v2, j, pnh, pnh == hrow1[j] ? trow1[j] : psk::kNoTpfBits);
+      src = __shfl_sync(full, bsrc, wl);
+      idx = (uint32_t)wl;
+    } else if (pick) {
+      // a full pass picked it (the helpers prepared no such candidate), or the last request (there is
+      // no next row): its values are computed here, on the stored state
+      bool ok3 = true;
+      if (lane == 0) {
+        if (!stored) ok3 = wait_smem_at_least(&s_stored, s, &s_stop, err, sync.wait_ns);
+        if (ok3) {
+          HelpSlot& xb = s_help[s & 1u];
+          int32_t qr2;
+          const InstVals v2 = inst_vals_after(a, m, j, rc.L, H, &qr2);
+          xb.x_nv = v2;
+          xb.x_qr = qr2;
+          if (has_next) {
+            const uint32_t slot1 = (s + 1) % kFeedRing;
+            const psk::RowPre& row1 = s_rowc[slot1];
+            const uint32_t* hrow1 = s_hitr + slot1 * Ip;
+            const uint32_t* trow1 = s_tpfr + slot1 * Ip;
+            const uint32_t h1 = raised_hit(row1, hrow1, j, true, 1, hist);
+            xb.x_pk = pair_key_v(m, row_of(row1), v2, j, h1, h1 == hrow1[j] ? trow1[j] : psk::kNoTpfBits);
+            xb.x_hit = h1;
+          }
+        } else {
+          s_stop = 1;
         }
       }
+      __syncwarp();
     }
     if (lane == 0) {
-      assign[s] = pick ? (int32_t)j : -1;
-      path[s] = pick ? (uint8_t)(K >> 62) : (uint8_t)2;
-      hit_chosen[s] = H;
+      const uint32_t x = s % kLogSlots;
+      s_logpick[x] = pick ? (int32_t)j : -1;
+      s_logsrc[x] = src;
+      s_logidx[x] = idx;
+      s_loghit[x] = H;
+      s_logpath[x] = pick ? (uint32_t)(K >> 62) : 2u;
+      psk::st_release_cta_shared_u32(&s_dec, s + 1);
       psk::st_relaxed_u64(sync.jobs + s, kJobValid | ((unsigned long long)H << 32) | (pick ? j : 0xFFFFFFFFu));
-      psk::st_release_cta_shared_u32(&s_consumed, s + 1);
     }
-    __syncwarp();
     const int32_t pj = pick ? (int32_t)j : -1;
     pk = __shfl_up_sync(full, pk, 1);
     if (lane == 0) pk = pj;
 #pragma unroll
     for (int k = psk::kLcpBack - 1; k > 0; --k) hist[k] = hist[k - 1];
     hist[0] = pj;
-    if (lane == 0) {
-      cor = pn;
-      chit = pnh;
-    } else {
-      cor = nt;
-      chit = nth;
-    }
+    w_src = src;
+    w_idx = idx;
+    if (has_next) load_row(s + 1);  // staged: s_fed >= s + 2 was waited for
   }
   if (lane == 0 && sync.stats) {
     atomicAdd(sync.stats + psk::kGsFast, n_fast);
@@ -1351,6 +1577,11 @@ __device__ void decide_spec(const psk::RowPre* __restrict__ rows, uint32_t R, ui
     atomicAdd(sync.stats + psk::kGsDecideWait, cyc_wait);
     atomicAdd(sync.stats + psk::kGsDecideTotal, (unsigned long long)(clock64() - cyc_start));
   }
+  // the pending state: every decision's state stored by the helpers (their phase R)
+  bool ok = true;
+  if (lane == 0) ok = !s_stop && wait_smem_at_least(&s_stored, R, &s_stop, err, sync.wait_ns);
+  ok = __shfl_sync(full, ok ? 1 : 0, 0) != 0;
+  if (!ok) return;
   for (uint32_t i = (uint32_t)lane; i < I; i += 32) {
     pending.b[i] = a.b[i];
     pending.qr[i] = a.qr[i];

@@ -550,6 +550,16 @@ __device__ __forceinline__ uint32_t ld_acquire_cta_shared_u32(const uint32_t* p)
   return v;
 }
 
+__device__ __forceinline__ uint32_t ld_relaxed_cta_shared_u32(const uint32_t* p) {
+  uint32_t v;
+  asm volatile("ld.relaxed.cta.shared::cta.u32 %0, [%1];" : "=r"(v) : "r"((uint32_t)__cvta_generic_to_shared(p))
+               : "memory");
+  return v;
+}
+
+// With a relaxed load before it that observed a release store, an acquire (CTA scope).
+__device__ __forceinline__ void fence_acq_rel_cta() { asm volatile("fence.acq_rel.cta;" ::: "memory"); }
+
 __device__ __forceinline__ uint64_t globaltimer_ns() {
   uint64_t x;
   asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(x));

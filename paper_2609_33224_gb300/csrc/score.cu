@@ -367,6 +367,248 @@ score_rows_kernel(const uint32_t* __restrict__ hits, psk::StateSoA st, uint32_t 
   }
 }
 
+// ---- rows of 257 .. 1024 instances: one thread block per row, instance terms in registers ----------
+//
+// Thread t owns the instances 4t .. 4t + 3 and keeps their request-independent terms in registers
+// for the whole launch, so a pair needs no shared-memory load.  A block takes a contiguous range of
+// rows; their row constants (T_pf(0, L), Z, eta Z, the TTFT budget) are computed once per 256 rows
+// into shared memory.  Per row: each thread loads its four hits (one 16-byte load, the next row's
+// issued before this row's pass 2), evaluates pass 1, and the block reduces W_min over A (warp
+// reduction, one barrier, every thread combines the warps' values); pass 2 writes the per-pair
+// outputs with 16-byte (TPOT, TTFT) and 4-byte (classes) stores and the block reduces the pick
+// (warp reduction, one barrier, one thread combines).  Shared reduction slots alternate between even
+// and odd rows, so two barriers per row suffice.
+constexpr uint32_t kBlkRowsAhead = 256;  // row constants computed per refill
+
+struct BlkRow {
+  float t_cached, Z, etaZ, ttft_budget, tpot_target;
+  uint32_t L;
+};
+
+template <bool GEN, bool VEC>
+__global__ void __launch_bounds__(256, 3)
+score_block_kernel(const uint32_t* __restrict__ hits, psk::StateSoA st, uint32_t I, psk::WindowDev w, psk::DevModel m,
+                   float* __restrict__ tpot_out, float* __restrict__ ttft_out, uint8_t* __restrict__ cls_out,
+                   int32_t* __restrict__ best_out, uint8_t* __restrict__ path_out, psk::ShardIO sh) {
+  __shared__ BlkRow s_rc[kBlkRowsAhead];
+  __shared__ uint32_t s_w[2][8];
+  __shared__ unsigned long long s_k[2][8];
+  __shared__ uint32_t s_t[2][8];
+  const uint32_t t = threadIdx.x;
+  const int lane = (int)(t & 31u), warp = (int)(t >> 5);
+  const int nw = (int)(blockDim.x >> 5);
+  const uint32_t i0 = 4u * t;
+  const bool all_pairs = tpot_out || ttft_out || cls_out;
+  // instance terms (padding instances past I fail the capacity guard: room -1)
+  int32_t room[4], q32[4], S32[4], Bp[4];
+  float dec0[4], fe[4], tq[4];
+  uint64_t k0[4];
+  bool wide = false;
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    const uint32_t i = i0 + (uint32_t)k;
+    room[k] = -1;
+    q32[k] = S32[k] = 0;
+    Bp[k] = 1;
+    dec0[k] = fe[k] = tq[k] = 0.0f;
+    k0[k] = 0ull;
+    if (i < I) {
+      const int32_t b = __ldg(st.b + i), qr = __ldg(st.qr + i), Bmax = __ldg(st.Bmax + i);
+      const int64_t q = __ldg(st.q + i), S = __ldg(st.S + i), M = __ldg(st.M + i);
+      const psk::InstTerms it = psk::inst_terms(m, b, qr, q, Bmax);
+      room[k] = it.okB ? psk::kv_room(S, M) : -1;
+      dec0[k] = it.dec0;
+      fe[k] = it.f;
+      tq[k] = it.tq;
+      Bp[k] = it.Bp;
+      k0[k] = psk::dcq_key0(b, qr);
+      wide |= !(q >= 0 && q < (1ll << 30) && S >= 0 && S < (1ll << 30));
+      q32[k] = (int32_t)q;
+      S32[k] = (int32_t)S;
+    }
+  }
+  // every instance's q and S below 2^30: the 32-bit sums are exact (else 64-bit state per pair)
+  const bool narrow = __syncthreads_or(wide ? 1 : 0) == 0;
+  const uint32_t per = (w.R + gridDim.x - 1) / gridDim.x;
+  const uint32_t r_lo = blockIdx.x * per;
+  const uint32_t r_hi = min(w.R, r_lo + per);
+  auto load_hits = [&](uint32_t r, uint32_t (&h)[4]) {
+    const uint32_t* hrow = hits + (uint64_t)r * I;
+    if (VEC) {
+      uint4 x = make_uint4(0u, 0u, 0u, 0u);
+      if (i0 < I) x = __ldcs(reinterpret_cast<const uint4*>(hrow + i0));
+      h[0] = x.x;
+      h[1] = x.y;
+      h[2] = x.z;
+      h[3] = x.w;
+    } else {
+#pragma unroll
+      for (int k = 0; k < 4; ++k) h[k] = (i0 + k < I) ? __ldcs(hrow + i0 + k) : 0u;
+    }
+  };
+  uint32_t hn[4] = {0u, 0u, 0u, 0u};
+  if (r_lo < r_hi) load_hits(r_lo, hn);
+  uint32_t par = 0;
+  for (uint32_t r = r_lo; r < r_hi; ++r, par ^= 1u) {
+    const uint32_t rr = (r - r_lo) % kBlkRowsAhead;
+    if (rr == 0) {
+      __syncthreads();  // every thread is done with the previous batch of row constants
+      const uint32_t x = r + t;
+      if (t < kBlkRowsAhead && x < r_hi) {
+        const psk::RowConst rc = psk::row_const(m, __ldg(w.L + x), __ldg(w.ttft_t + x), __ldg(w.tpot_t + x));
+        s_rc[t] = BlkRow{rc.t_cached, rc.Z, rc.etaZ, rc.ttft_budget, rc.tpot_target, rc.L};
+      }
+      __syncthreads();
+    }
+    psk::RowConst rc;
+    {
+      const BlkRow& b = s_rc[rr];
+      rc.t_cached = b.t_cached;
+      rc.Z = b.Z;
+      rc.etaZ = b.etaZ;
+      rc.ttft_budget = b.ttft_budget;
+      rc.tpot_target = b.tpot_target;
+      rc.L = b.L;
+    }
+    uint32_t h[4] = {hn[0], hn[1], hn[2], hn[3]};
+    if (r + 1 < r_hi) load_hits(r + 1, hn);  // in flight during this row
+    // pass 1: capacity guard, T_pf at the hit, W over A
+    float tp[4];
+    uint32_t am = 0u, wbest = 0xFFFFFFFFu;
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const bool inA = (int32_t)rc.L <= room[k];
+      am |= (inA ? 1u : 0u) << k;
+      tp[k] = (inA || all_pairs) ? t_pf32(m, rc.L, h[k]) : 0.0f;
+      if (inA) wbest = min(wbest, psk::f2ord(__fsub_rn(tp[k], rc.t_cached)));
+    }
+    wbest = __reduce_min_sync(0xffffffffu, wbest);
+    if (lane == 0) s_w[par][warp] = wbest;
+    __syncthreads();
+    wbest = 0xFFFFFFFFu;
+    for (int v = 0; v < nw; ++v) wbest = min(wbest, s_w[par][v]);
+    if (sh.wmin_out) {  // column block, first reduction only
+      if (t == 0) sh.wmin_out[r] = wbest;
+      continue;
+    }
+    if (sh.wmin_in) wbest = __ldg(sh.wmin_in + r);  // the pool's W_min
+    const bool anyA = wbest != 0xFFFFFFFFu;
+    const float wmin = psk::ord2f(wbest);
+    // pass 2: classes, latencies, keys
+    uint64_t bkey = psk::kNoKey;
+    uint32_t btie = 0xFFFFFFFFu;
+    float to[4], tt[4];
+    uint32_t cw = 0u;
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const uint32_t i = i0 + (uint32_t)k;
+      const bool inA = (am >> k) & 1u;
+      const bool inC = inA && psk::pair_in_c(rc, __fsub_rn(tp[k], rc.t_cached), wmin);
+      const int32_t n = (int32_t)rc.L - (int32_t)(h[k] << 4);
+      to[k] = tt[k] = 0.0f;
+      uint32_t cls = 3u;
+      if (all_pairs || inC) {
+        if (narrow) {
+          pair_lat32(m, rc, tp[k], n, dec0[k], fe[k], tq[k], Bp[k], q32[k], S32[k], &to[k], &tt[k]);
+        } else if (i < I) {
+          psk::InstTerms it;
+          it.dec0 = dec0[k];
+          it.f = fe[k];
+          it.tq = tq[k];
+          it.Bp = Bp[k];
+          it.okB = 1;
+          psk::PairW x;
+          x.tpf = tp[k];
+          x.W = __fsub_rn(x.tpf, rc.t_cached);
+          x.n = n;
+          x.inA = true;
+          psk::pair_lat(m, rc, x, it, __ldg(st.q + i), __ldg(st.S + i), &to[k], &tt[k]);
+        }
+        if (inA) cls = inC ? (psk::pair_admitted(m, rc, to[k], tt[k]) ? 0u : 1u) : 2u;
+      }
+      cw |= cls << (8 * k);
+      if (cls <= 1u) {
+        const uint64_t qn = narrow ? (uint64_t)(uint32_t)(q32[k] + n)
+                                   : (uint64_t)__ldg(st.q + i) + (uint64_t)(int64_t)n;
+        uint64_t key;
+        uint32_t tie = i;
+        if (!GEN) {
+          key = cls == 0u ? psk::packed_key(0u, k0[k] | ((uint64_t)((1u << 26) - 1u - h[k]) << 18))
+                          : psk::packed_key(1u, qn * (uint64_t)(uint32_t)Bp[k]);
+        } else if (cls == 0u) {
+          key = psk::packed_key(0u, psk::value_in_t(m, psk::key0_from_dcq(m, k0[k]), h[k], to[k], rc.tpot_target));
+          if (m.sel == psk::kSelHCQ) tie |= (uint32_t)(k0[k] & 0x3FFFFull) << 12;
+        } else {
+          key = psk::packed_key(1u, psk::value_fallback(m, qn, (uint32_t)Bp[k], k0[k], h[k]));
+        }
+        if (key < bkey || (GEN && key == bkey && tie < btie)) {  // this thread's instances ascend
+          bkey = key;
+          btie = tie;
+        }
+      }
+    }
+    if (all_pairs && i0 < I) {
+      const uint64_t x = (uint64_t)r * I + i0;
+      if (VEC) {
+        if (tpot_out) __stcs(reinterpret_cast<float4*>(tpot_out + x), make_float4(to[0], to[1], to[2], to[3]));
+        if (ttft_out) __stcs(reinterpret_cast<float4*>(ttft_out + x), make_float4(tt[0], tt[1], tt[2], tt[3]));
+        if (cls_out) __stcs(reinterpret_cast<uint32_t*>(cls_out + x), cw);
+      } else {
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          if (i0 + k >= I) break;
+          if (tpot_out) tpot_out[x + k] = to[k];
+          if (ttft_out) ttft_out[x + k] = tt[k];
+          if (cls_out) cls_out[x + k] = (uint8_t)(cw >> (8 * k));
+        }
+      }
+    }
+    uint64_t key;
+    uint32_t tie, hj;
+    psk::warp_pick_min(bkey, btie, 0u, &key, &tie, &hj);
+    if (lane == 0) {
+      s_k[par][warp] = key;
+      s_t[par][warp] = tie;
+    }
+    __syncthreads();
+    if (t == 0) {
+      uint64_t kb = psk::kNoKey;
+      uint32_t tb = 0xFFFFFFFFu;
+      for (int v = 0; v < nw; ++v) {
+        const uint64_t kv = s_k[par][v];
+        const uint32_t tv = s_t[par][v];
+        if (kv < kb || (kv == kb && tv < tb)) {
+          kb = kv;
+          tb = tv;
+        }
+      }
+      const bool pick = anyA && kb != psk::kNoKey;
+      if (best_out) best_out[r] = pick ? (int32_t)(tb & psk::kTieInstMask) : -1;
+      if (path_out) path_out[r] = pick ? (uint8_t)(kb >> 62) : (uint8_t)2;
+      if (sh.key_out) {
+        sh.key_out[r] = pick ? kb : psk::kNoKey;
+        sh.tie_out[r] = pick ? tb + sh.id_base : 0xFFFFFFFFu;
+      }
+    }
+  }
+}
+
+cudaError_t score_block_launch(const uint32_t* hits, psk::StateSoA st, uint32_t I, const psk::WindowDev& w,
+                               const psk::DevModel& m, float* tpot, float* ttft, uint8_t* cls, int32_t* best,
+                               uint8_t* path, int num_sms, cudaStream_t s, const psk::ShardIO& sh) {
+  const bool vec = (I & 3u) == 0u && (reinterpret_cast<uintptr_t>(hits) & 15u) == 0u &&
+                   (reinterpret_cast<uintptr_t>(tpot) & 15u) == 0u && (reinterpret_cast<uintptr_t>(ttft) & 15u) == 0u &&
+                   (reinterpret_cast<uintptr_t>(cls) & 3u) == 0u;
+  const bool gen = m.sel != psk::kSelDCQ || m.fb_dcq;
+  const uint32_t threads = 256u;  // 4 instances a thread, up to 1024 instances
+  uint32_t grid = (uint32_t)num_sms * 3u;
+  if (grid > w.R) grid = w.R;
+  auto kern = vec ? (gen ? score_block_kernel<true, true> : score_block_kernel<false, true>)
+                  : (gen ? score_block_kernel<true, false> : score_block_kernel<false, false>);
+  kern<<<grid, threads, 0, s>>>(hits, st, I, w, m, tpot, ttft, cls, best, path, sh);
+  return cudaGetLastError();
+}
+
 template <int NV>
 cudaError_t score_launch(const uint32_t* hits, psk::StateSoA st, uint32_t I, const psk::WindowDev& w,
                          const psk::DevModel& m, float* tpot, float* ttft, uint8_t* cls, int32_t* best,
@@ -411,6 +653,7 @@ cudaError_t launch_score(const uint32_t* hits, psk::StateSoA st, uint32_t I, con
   if (w.R == 0) return cudaSuccess;
   if (I <= 128u) return score_launch<1>(hits, st, I, w, m, tpot, ttft, cls, best, path, num_sms, s, sh);
   if (I <= 256u) return score_launch<2>(hits, st, I, w, m, tpot, ttft, cls, best, path, num_sms, s, sh);
+  if (I <= 1024u) return score_block_launch(hits, st, I, w, m, tpot, ttft, cls, best, path, num_sms, s, sh);
   return score_launch<4>(hits, st, I, w, m, tpot, ttft, cls, best, path, num_sms, s, sh);
 }
 
