@@ -13,6 +13,8 @@
 // C when T is empty, Reject when A is empty (or the model's policy variant of Table 3 / Table 4).
 // Pass 2 takes the hits from registers; rows of more than 128 NV instances are taken in pieces of
 // NV chunks, each read again for pass 2.
+#include <type_traits>
+
 #include "ps_internal.cuh"
 
 namespace {
@@ -367,38 +369,40 @@ score_rows_kernel(const uint32_t* __restrict__ hits, psk::StateSoA st, uint32_t 
   }
 }
 
-// ---- rows of 257 .. 1024 instances: one thread block per row, instance terms in registers ----------
+// ---- rows of 257 .. 1024 instances: a thread block per row, instance terms in registers ------------
 //
 // Thread t owns the instances 4t .. 4t + 3 and keeps their request-independent terms in registers
 // for the whole launch, so a pair needs no shared-memory load.  A block takes a contiguous range of
-// rows; their row constants (T_pf(0, L), Z, eta Z, the TTFT budget) are computed once per 256 rows
-// into shared memory.  Per row: each thread loads its four hits (one 16-byte load, the next row's
-// issued before this row's pass 2), evaluates pass 1, and the block reduces W_min over A (warp
-// reduction, one barrier, every thread combines the warps' values); pass 2 writes the per-pair
-// outputs with 16-byte (TPOT, TTFT) and 4-byte (classes) stores and the block reduces the pick
-// (warp reduction, one barrier, one thread combines).  Shared reduction slots alternate between even
-// and odd rows, so two barriers per row suffice.
+// rows, two at a time; their row constants (T_pf(0, L), Z, eta Z, the TTFT budget) are computed once
+// per 256 rows into shared memory.  Per pair of rows: each thread loads its four hits of each (16-byte
+// loads, the next pair's issued before this pair's work), evaluates pass 1 on both, and the block
+// reduces both rows' W_min over A (warp reductions, one barrier, every thread combines the warps'
+// values); pass 2 writes the per-pair outputs with 16-byte (TPOT, TTFT) and 4-byte (classes) stores
+// and the warps' picks go to shared slots, which one thread per row combines after the next pair's
+// barrier.  Shared reduction slots alternate between iterations, so one barrier per pair of rows
+// suffices.
 constexpr uint32_t kBlkRowsAhead = 256;  // row constants computed per refill
+constexpr uint32_t kBlkThreads = 256;    // 4 instances a thread, up to 1024 instances
 
 struct BlkRow {
   float t_cached, Z, etaZ, ttft_budget, tpot_target;
   uint32_t L;
 };
 
-template <bool GEN, bool VEC>
-__global__ void __launch_bounds__(256, 3)
+template <bool GEN, bool VEC, bool ALL>
+__global__ void __launch_bounds__(kBlkThreads, 2)
 score_block_kernel(const uint32_t* __restrict__ hits, psk::StateSoA st, uint32_t I, psk::WindowDev w, psk::DevModel m,
                    float* __restrict__ tpot_out, float* __restrict__ ttft_out, uint8_t* __restrict__ cls_out,
                    int32_t* __restrict__ best_out, uint8_t* __restrict__ path_out, psk::ShardIO sh) {
   __shared__ BlkRow s_rc[kBlkRowsAhead];
-  __shared__ uint32_t s_w[2][8];
-  __shared__ unsigned long long s_k[2][8];
-  __shared__ uint32_t s_t[2][8];
+  __shared__ __align__(16) uint32_t s_w[2][2][8];  // [parity][row of the pair][warp]
+  __shared__ unsigned long long s_k[2][2][8];
+  __shared__ uint32_t s_t[2][2][8];
   const uint32_t t = threadIdx.x;
   const int lane = (int)(t & 31u), warp = (int)(t >> 5);
-  const int nw = (int)(blockDim.x >> 5);
+  constexpr int nw = kBlkThreads / 32;  // the launch's block size
   const uint32_t i0 = 4u * t;
-  const bool all_pairs = tpot_out || ttft_out || cls_out;
+  constexpr bool all_pairs = ALL;  // some per-pair output is wanted (the launch checks)
   // instance terms (padding instances past I fail the capacity guard: room -1)
   int32_t room[4], q32[4], S32[4], Bp[4];
   float dec0[4], fe[4], tq[4];
@@ -429,168 +433,246 @@ score_block_kernel(const uint32_t* __restrict__ hits, psk::StateSoA st, uint32_t
   }
   // every instance's q and S below 2^30: the 32-bit sums are exact (else 64-bit state per pair)
   const bool narrow = __syncthreads_or(wide ? 1 : 0) == 0;
-  const uint32_t per = (w.R + gridDim.x - 1) / gridDim.x;
-  const uint32_t r_lo = blockIdx.x * per;
-  const uint32_t r_hi = min(w.R, r_lo + per);
-  auto load_hits = [&](uint32_t r, uint32_t (&h)[4]) {
-    const uint32_t* hrow = hits + (uint64_t)r * I;
-    if (VEC) {
-      uint4 x = make_uint4(0u, 0u, 0u, 0u);
-      if (i0 < I) x = __ldcs(reinterpret_cast<const uint4*>(hrow + i0));
-      h[0] = x.x;
-      h[1] = x.y;
-      h[2] = x.z;
-      h[3] = x.w;
-    } else {
+  // the row loop, compiled for the narrow and the wide state separately (a block-uniform choice)
+  auto rows_loop = [&](auto narrow_tag) {
+    constexpr bool NARROW = decltype(narrow_tag)::value;
+    const uint32_t per = (w.R + gridDim.x - 1) / gridDim.x;
+    const uint32_t r_lo = blockIdx.x * per;
+    const uint32_t r_hi = min(w.R, r_lo + per);
+    auto load_hits = [&](uint32_t r, uint32_t (&h)[4]) {
+      const uint32_t* hrow = hits + (uint64_t)r * I;
+      if (VEC) {
+        uint4 x = make_uint4(0u, 0u, 0u, 0u);
+        if (i0 < I) x = __ldcs(reinterpret_cast<const uint4*>(hrow + i0));
+        h[0] = x.x;
+        h[1] = x.y;
+        h[2] = x.z;
+        h[3] = x.w;
+      } else {
 #pragma unroll
-      for (int k = 0; k < 4; ++k) h[k] = (i0 + k < I) ? __ldcs(hrow + i0 + k) : 0u;
-    }
-  };
-  uint32_t hn[4] = {0u, 0u, 0u, 0u};
-  if (r_lo < r_hi) load_hits(r_lo, hn);
-  uint32_t par = 0;
-  for (uint32_t r = r_lo; r < r_hi; ++r, par ^= 1u) {
-    const uint32_t rr = (r - r_lo) % kBlkRowsAhead;
-    if (rr == 0) {
-      __syncthreads();  // every thread is done with the previous batch of row constants
-      const uint32_t x = r + t;
-      if (t < kBlkRowsAhead && x < r_hi) {
-        const psk::RowConst rc = psk::row_const(m, __ldg(w.L + x), __ldg(w.ttft_t + x), __ldg(w.tpot_t + x));
-        s_rc[t] = BlkRow{rc.t_cached, rc.Z, rc.etaZ, rc.ttft_budget, rc.tpot_target, rc.L};
+        for (int k = 0; k < 4; ++k) h[k] = (i0 + k < I) ? __ldcs(hrow + i0 + k) : 0u;
       }
-      __syncthreads();
-    }
-    psk::RowConst rc;
-    {
+    };
+    auto rc_of = [&](uint32_t rr) {
       const BlkRow& b = s_rc[rr];
+      psk::RowConst rc;
       rc.t_cached = b.t_cached;
       rc.Z = b.Z;
       rc.etaZ = b.etaZ;
       rc.ttft_budget = b.ttft_budget;
       rc.tpot_target = b.tpot_target;
       rc.L = b.L;
-    }
-    uint32_t h[4] = {hn[0], hn[1], hn[2], hn[3]};
-    if (r + 1 < r_hi) load_hits(r + 1, hn);  // in flight during this row
-    // pass 1: capacity guard, T_pf at the hit, W over A
-    float tp[4];
-    uint32_t am = 0u, wbest = 0xFFFFFFFFu;
+      return rc;
+    };
+    // pass 1 of a row: capacity guard, T_pf at the hit, this thread's W_min over A.  T_pf depends on
+    // the row and the hit only, and most of a row's instances share a hit (the shared system prompt),
+    // so a thread evaluates it at its first instance's hit and again only where a hit differs (a
+    // warp-uniform test: the warp skips the evaluation when no lane's hit differs).
+    auto pass1 = [&](const psk::RowConst& rc, const uint32_t (&h)[4], float (&tp)[4], uint32_t& am) {
+      uint32_t wbest = 0xFFFFFFFFu;
+      am = 0u;
+      const float tb = t_pf32(m, rc.L, h[0]);
 #pragma unroll
-    for (int k = 0; k < 4; ++k) {
-      const bool inA = (int32_t)rc.L <= room[k];
-      am |= (inA ? 1u : 0u) << k;
-      tp[k] = (inA || all_pairs) ? t_pf32(m, rc.L, h[k]) : 0.0f;
-      if (inA) wbest = min(wbest, psk::f2ord(__fsub_rn(tp[k], rc.t_cached)));
-    }
-    wbest = __reduce_min_sync(0xffffffffu, wbest);
-    if (lane == 0) s_w[par][warp] = wbest;
-    __syncthreads();
-    wbest = 0xFFFFFFFFu;
-    for (int v = 0; v < nw; ++v) wbest = min(wbest, s_w[par][v]);
-    if (sh.wmin_out) {  // column block, first reduction only
-      if (t == 0) sh.wmin_out[r] = wbest;
-      continue;
-    }
-    if (sh.wmin_in) wbest = __ldg(sh.wmin_in + r);  // the pool's W_min
-    const bool anyA = wbest != 0xFFFFFFFFu;
-    const float wmin = psk::ord2f(wbest);
-    // pass 2: classes, latencies, keys
-    uint64_t bkey = psk::kNoKey;
-    uint32_t btie = 0xFFFFFFFFu;
-    float to[4], tt[4];
-    uint32_t cw = 0u;
-#pragma unroll
-    for (int k = 0; k < 4; ++k) {
-      const uint32_t i = i0 + (uint32_t)k;
-      const bool inA = (am >> k) & 1u;
-      const bool inC = inA && psk::pair_in_c(rc, __fsub_rn(tp[k], rc.t_cached), wmin);
-      const int32_t n = (int32_t)rc.L - (int32_t)(h[k] << 4);
-      to[k] = tt[k] = 0.0f;
-      uint32_t cls = 3u;
-      if (all_pairs || inC) {
-        if (narrow) {
-          pair_lat32(m, rc, tp[k], n, dec0[k], fe[k], tq[k], Bp[k], q32[k], S32[k], &to[k], &tt[k]);
-        } else if (i < I) {
-          psk::InstTerms it;
-          it.dec0 = dec0[k];
-          it.f = fe[k];
-          it.tq = tq[k];
-          it.Bp = Bp[k];
-          it.okB = 1;
-          psk::PairW x;
-          x.tpf = tp[k];
-          x.W = __fsub_rn(x.tpf, rc.t_cached);
-          x.n = n;
-          x.inA = true;
-          psk::pair_lat(m, rc, x, it, __ldg(st.q + i), __ldg(st.S + i), &to[k], &tt[k]);
+      for (int k = 0; k < 4; ++k) {
+        const bool inA = (int32_t)rc.L <= room[k];
+        am |= (inA ? 1u : 0u) << k;
+        tp[k] = tb;
+        const bool other = h[k] != h[0] && (inA || all_pairs);
+        if (k > 0 && __any_sync(0xffffffffu, other)) {
+          if (other) tp[k] = t_pf32(m, rc.L, h[k]);
         }
-        if (inA) cls = inC ? (psk::pair_admitted(m, rc, to[k], tt[k]) ? 0u : 1u) : 2u;
+        if (inA) wbest = min(wbest, psk::f2ord(__fsub_rn(tp[k], rc.t_cached)));
       }
-      cw |= cls << (8 * k);
-      if (cls <= 1u) {
-        const uint64_t qn = narrow ? (uint64_t)(uint32_t)(q32[k] + n)
-                                   : (uint64_t)__ldg(st.q + i) + (uint64_t)(int64_t)n;
-        uint64_t key;
-        uint32_t tie = i;
-        if (!GEN) {
-          key = cls == 0u ? psk::packed_key(0u, k0[k] | ((uint64_t)((1u << 26) - 1u - h[k]) << 18))
-                          : psk::packed_key(1u, qn * (uint64_t)(uint32_t)Bp[k]);
-        } else if (cls == 0u) {
-          key = psk::packed_key(0u, psk::value_in_t(m, psk::key0_from_dcq(m, k0[k]), h[k], to[k], rc.tpot_target));
-          if (m.sel == psk::kSelHCQ) tie |= (uint32_t)(k0[k] & 0x3FFFFull) << 12;
+      return wbest;
+    };
+    // pass 2 of row r: classes, latencies, the per-pair outputs, this thread's best (key, tie)
+    auto pass2 = [&](uint32_t r, const psk::RowConst& rc, const uint32_t (&h)[4], const float (&tp)[4], uint32_t am,
+                     float wmin, uint64_t& bkey, uint32_t& btie) {
+      bkey = psk::kNoKey;
+      btie = 0xFFFFFFFFu;
+      float to[4], tt[4];
+      uint32_t cw = 0u;
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const uint32_t i = i0 + (uint32_t)k;
+        const bool inA = (am >> k) & 1u;
+        const bool inC = inA && psk::pair_in_c(rc, __fsub_rn(tp[k], rc.t_cached), wmin);
+        const int32_t n = (int32_t)rc.L - (int32_t)(h[k] << 4);
+        to[k] = tt[k] = 0.0f;
+        uint32_t cls = 3u;
+        if (all_pairs || inC) {
+          if (NARROW) {
+            pair_lat32(m, rc, tp[k], n, dec0[k], fe[k], tq[k], Bp[k], q32[k], S32[k], &to[k], &tt[k]);
+          } else if (i < I) {
+            psk::InstTerms it;
+            it.dec0 = dec0[k];
+            it.f = fe[k];
+            it.tq = tq[k];
+            it.Bp = Bp[k];
+            it.okB = 1;
+            psk::PairW x;
+            x.tpf = tp[k];
+            x.W = __fsub_rn(x.tpf, rc.t_cached);
+            x.n = n;
+            x.inA = true;
+            psk::pair_lat(m, rc, x, it, __ldg(st.q + i), __ldg(st.S + i), &to[k], &tt[k]);
+          }
+          if (inA) cls = inC ? (psk::pair_admitted(m, rc, to[k], tt[k]) ? 0u : 1u) : 2u;
+        }
+        cw |= cls << (8 * k);
+        if (cls <= 1u) {
+          const uint64_t qn = NARROW ? (uint64_t)(uint32_t)(q32[k] + n)
+                                     : (uint64_t)__ldg(st.q + i) + (uint64_t)(int64_t)n;
+          uint64_t key;
+          uint32_t tie = i;
+          if (!GEN) {
+            key = cls == 0u ? psk::packed_key(0u, k0[k] | ((uint64_t)((1u << 26) - 1u - h[k]) << 18))
+                            : psk::packed_key(1u, qn * (uint64_t)(uint32_t)Bp[k]);
+          } else if (cls == 0u) {
+            key = psk::packed_key(0u, psk::value_in_t(m, psk::key0_from_dcq(m, k0[k]), h[k], to[k], rc.tpot_target));
+            if (m.sel == psk::kSelHCQ) tie |= (uint32_t)(k0[k] & 0x3FFFFull) << 12;
+          } else {
+            key = psk::packed_key(1u, psk::value_fallback(m, qn, (uint32_t)Bp[k], k0[k], h[k]));
+          }
+          if (key < bkey || (GEN && key == bkey && tie < btie)) {  // this thread's instances ascend
+            bkey = key;
+            btie = tie;
+          }
+        }
+      }
+      if (all_pairs && i0 < I) {
+        const uint64_t x = (uint64_t)r * I + i0;
+        if (VEC) {
+          if (tpot_out) __stcs(reinterpret_cast<float4*>(tpot_out + x), make_float4(to[0], to[1], to[2], to[3]));
+          if (ttft_out) __stcs(reinterpret_cast<float4*>(ttft_out + x), make_float4(tt[0], tt[1], tt[2], tt[3]));
+          if (cls_out) __stcs(reinterpret_cast<uint32_t*>(cls_out + x), cw);
         } else {
-          key = psk::packed_key(1u, psk::value_fallback(m, qn, (uint32_t)Bp[k], k0[k], h[k]));
-        }
-        if (key < bkey || (GEN && key == bkey && tie < btie)) {  // this thread's instances ascend
-          bkey = key;
-          btie = tie;
-        }
-      }
-    }
-    if (all_pairs && i0 < I) {
-      const uint64_t x = (uint64_t)r * I + i0;
-      if (VEC) {
-        if (tpot_out) __stcs(reinterpret_cast<float4*>(tpot_out + x), make_float4(to[0], to[1], to[2], to[3]));
-        if (ttft_out) __stcs(reinterpret_cast<float4*>(ttft_out + x), make_float4(tt[0], tt[1], tt[2], tt[3]));
-        if (cls_out) __stcs(reinterpret_cast<uint32_t*>(cls_out + x), cw);
-      } else {
 #pragma unroll
-        for (int k = 0; k < 4; ++k) {
-          if (i0 + k >= I) break;
-          if (tpot_out) tpot_out[x + k] = to[k];
-          if (ttft_out) ttft_out[x + k] = tt[k];
-          if (cls_out) cls_out[x + k] = (uint8_t)(cw >> (8 * k));
+          for (int k = 0; k < 4; ++k) {
+            if (i0 + k >= I) break;
+            if (tpot_out) tpot_out[x + k] = to[k];
+            if (ttft_out) ttft_out[x + k] = tt[k];
+            if (cls_out) cls_out[x + k] = (uint8_t)(cw >> (8 * k));
+          }
         }
       }
-    }
-    uint64_t key;
-    uint32_t tie, hj;
-    psk::warp_pick_min(bkey, btie, 0u, &key, &tie, &hj);
-    if (lane == 0) {
-      s_k[par][warp] = key;
-      s_t[par][warp] = tie;
-    }
-    __syncthreads();
-    if (t == 0) {
+    };
+    // Rows two at a time: both rows' W_min in one barrier.  The picks of a pair of rows are combined
+    // after the next pair's barrier (their slots alternate between iterations), so an iteration has
+    // one barrier.
+    auto merge = [&](uint32_t rp, int q, uint32_t pw, uint32_t pp) {
+      // row rp's pick from the warps' (key, tie) in slot s_k[pp][q]
       uint64_t kb = psk::kNoKey;
       uint32_t tb = 0xFFFFFFFFu;
       for (int v = 0; v < nw; ++v) {
-        const uint64_t kv = s_k[par][v];
-        const uint32_t tv = s_t[par][v];
+        const uint64_t kv = s_k[pp][q][v];
+        const uint32_t tv = s_t[pp][q][v];
         if (kv < kb || (kv == kb && tv < tb)) {
           kb = kv;
           tb = tv;
         }
       }
-      const bool pick = anyA && kb != psk::kNoKey;
-      if (best_out) best_out[r] = pick ? (int32_t)(tb & psk::kTieInstMask) : -1;
-      if (path_out) path_out[r] = pick ? (uint8_t)(kb >> 62) : (uint8_t)2;
+      const bool pick = pw != 0xFFFFFFFFu && kb != psk::kNoKey;
+      if (best_out) best_out[rp] = pick ? (int32_t)(tb & psk::kTieInstMask) : -1;
+      if (path_out) path_out[rp] = pick ? (uint8_t)(kb >> 62) : (uint8_t)2;
       if (sh.key_out) {
-        sh.key_out[r] = pick ? kb : psk::kNoKey;
-        sh.tie_out[r] = pick ? tb + sh.id_base : 0xFFFFFFFFu;
+        sh.key_out[rp] = pick ? kb : psk::kNoKey;
+        sh.tie_out[rp] = pick ? tb + sh.id_base : 0xFFFFFFFFu;
       }
+    };
+    uint32_t hn[2][4] = {{0u, 0u, 0u, 0u}, {0u, 0u, 0u, 0u}};
+    if (r_lo < r_hi) load_hits(r_lo, hn[0]);
+    if (r_lo + 1 < r_hi) load_hits(r_lo + 1, hn[1]);
+    uint32_t par = 0;
+    bool prev = false;          // a pair of rows whose picks are still to be combined
+    uint32_t prev_r = 0, pw0 = 0u, pw1 = 0u;
+    bool prev_two = false;
+    for (uint32_t r = r_lo; r < r_hi; r += 2, par ^= 1u) {
+      const bool two = r + 1 < r_hi;
+      const uint32_t rr = (r - r_lo) % kBlkRowsAhead;  // even, so row r + 1 is in the same batch
+      if (rr == 0) {
+        __syncthreads();  // every thread is done with the previous batch of row constants
+        const uint32_t x = r + t;
+        if (t < kBlkRowsAhead && x < r_hi) {
+          const psk::RowConst rc = psk::row_const(m, __ldg(w.L + x), __ldg(w.ttft_t + x), __ldg(w.tpot_t + x));
+          s_rc[t] = BlkRow{rc.t_cached, rc.Z, rc.etaZ, rc.ttft_budget, rc.tpot_target, rc.L};
+        }
+        __syncthreads();
+      }
+      const psk::RowConst rc0 = rc_of(rr);
+      const psk::RowConst rc1 = rc_of(two ? rr + 1 : rr);
+      uint32_t h0[4], h1[4];
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        h0[k] = hn[0][k];
+        h1[k] = hn[1][k];
+      }
+      if (r + 2 < r_hi) load_hits(r + 2, hn[0]);  // in flight during these rows
+      if (r + 3 < r_hi) load_hits(r + 3, hn[1]);
+      float tp0[4], tp1[4];
+      uint32_t am0, am1;
+      uint32_t w0 = pass1(rc0, h0, tp0, am0);
+      uint32_t w1 = two ? pass1(rc1, h1, tp1, am1) : 0xFFFFFFFFu;
+      if (!two) {
+        am1 = 0u;
+#pragma unroll
+        for (int k = 0; k < 4; ++k) tp1[k] = 0.0f;
+      }
+      w0 = __reduce_min_sync(0xffffffffu, w0);
+      w1 = __reduce_min_sync(0xffffffffu, w1);
+      if (lane == 0) {
+        s_w[par][0][warp] = w0;
+        s_w[par][1][warp] = w1;
+      }
+      __syncthreads();
+      // the previous pair's picks (its warps' slots were written before this barrier)
+      if (prev && (t == 0 || (t == 32 && prev_two))) {
+        const int q = t == 0 ? 0 : 1;
+        merge(prev_r + (uint32_t)q, q, q == 0 ? pw0 : pw1, par ^ 1u);
+      }
+      {  // the eight warps' values of both rows, four 16-byte loads
+        const uint4* sw = reinterpret_cast<const uint4*>(&s_w[par][0][0]);
+        const uint4 a0 = sw[0], a1 = sw[1], b0 = sw[2], b1 = sw[3];
+        w0 = min(min(min(a0.x, a0.y), min(a0.z, a0.w)), min(min(a1.x, a1.y), min(a1.z, a1.w)));
+        w1 = min(min(min(b0.x, b0.y), min(b0.z, b0.w)), min(min(b1.x, b1.y), min(b1.z, b1.w)));
+      }
+      if (sh.wmin_out) {  // column block, first reduction only
+        if (t == 0) sh.wmin_out[r] = w0;
+        if (t == 32 && two) sh.wmin_out[r + 1] = w1;
+        continue;
+      }
+      if (sh.wmin_in) {  // the pool's W_min
+        w0 = __ldg(sh.wmin_in + r);
+        if (two) w1 = __ldg(sh.wmin_in + r + 1);
+      }
+      uint64_t bk0, bk1 = psk::kNoKey;
+      uint32_t bt0, bt1 = 0xFFFFFFFFu;
+      pass2(r, rc0, h0, tp0, am0, psk::ord2f(w0), bk0, bt0);
+      if (two) pass2(r + 1, rc1, h1, tp1, am1, psk::ord2f(w1), bk1, bt1);
+      uint64_t key0, key1;
+      uint32_t tie0, tie1, hj;
+      psk::warp_pick_min(bk0, bt0, 0u, &key0, &tie0, &hj);
+      psk::warp_pick_min(bk1, bt1, 0u, &key1, &tie1, &hj);
+      if (lane == 0) {
+        s_k[par][0][warp] = key0;
+        s_t[par][0][warp] = tie0;
+        s_k[par][1][warp] = key1;
+        s_t[par][1][warp] = tie1;
+      }
+      prev = true;
+      prev_r = r;
+      prev_two = two;
+      pw0 = w0;
+      pw1 = w1;
     }
-  }
+    __syncthreads();
+    if (prev && (t == 0 || (t == 32 && prev_two))) {
+      const int q = t == 0 ? 0 : 1;
+      merge(prev_r + (uint32_t)q, q, q == 0 ? pw0 : pw1, par ^ 1u);
+    }
+  };
+  if (narrow) rows_loop(std::integral_constant<bool, true>());
+  else rows_loop(std::integral_constant<bool, false>());
 }
 
 cudaError_t score_block_launch(const uint32_t* hits, psk::StateSoA st, uint32_t I, const psk::WindowDev& w,
@@ -600,11 +682,20 @@ cudaError_t score_block_launch(const uint32_t* hits, psk::StateSoA st, uint32_t 
                    (reinterpret_cast<uintptr_t>(tpot) & 15u) == 0u && (reinterpret_cast<uintptr_t>(ttft) & 15u) == 0u &&
                    (reinterpret_cast<uintptr_t>(cls) & 3u) == 0u;
   const bool gen = m.sel != psk::kSelDCQ || m.fb_dcq;
-  const uint32_t threads = 256u;  // 4 instances a thread, up to 1024 instances
-  uint32_t grid = (uint32_t)num_sms * 3u;
+  const uint32_t threads = kBlkThreads;
+  const bool all = tpot || ttft || cls;
+  decltype(&score_block_kernel<true, true, true>) kern;
+  if (all)
+    kern = vec ? (gen ? score_block_kernel<true, true, true> : score_block_kernel<false, true, true>)
+               : (gen ? score_block_kernel<true, false, true> : score_block_kernel<false, false, true>);
+  else
+    kern = vec ? (gen ? score_block_kernel<true, true, false> : score_block_kernel<false, true, false>)
+               : (gen ? score_block_kernel<true, false, false> : score_block_kernel<false, false, false>);
+  int per_sm = 0;  // one wave of resident blocks, each taking a contiguous range of rows
+  cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, (int)threads, 0);
+  if (e != cudaSuccess) return e;
+  uint32_t grid = (uint32_t)num_sms * (uint32_t)(per_sm > 0 ? per_sm : 1);
   if (grid > w.R) grid = w.R;
-  auto kern = vec ? (gen ? score_block_kernel<true, true> : score_block_kernel<false, true>)
-                  : (gen ? score_block_kernel<true, false> : score_block_kernel<false, false>);
   kern<<<grid, threads, 0, s>>>(hits, st, I, w, m, tpot, ttft, cls, best, path, sh);
   return cudaGetLastError();
 }
