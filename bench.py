@@ -444,9 +444,13 @@ def main():
     dominant = max(phases, key=phases.get)
     peak, peak_src = _peaks()
     probe_ms = km["probe_scratch"] + max(0.0, km["probe_derived"])
-    greedy_traffic = profile_figure("step_kernels_production_window_1024x8192.md", "DRAM bytes per request")
-    probe_traffic = profile_figure("step_kernels_production_window_1024x8192.md", "DRAM bytes per lookup")
-    score_traffic = profile_figure("score_rows_production_window_1024x8192.md", "DRAM bytes per request")
+    # DRAM traffic per unit from the committed ncu summaries of the production window (scaled by this
+    # run's units; None for another workload, whose kernels those captures do not cover)
+    prod = args.config == 2 and args.probe_mode == 1
+    greedy_traffic = profile_figure("greedy_pipe_production_window_1024x8192.md", "DRAM bytes per request") if prod else None
+    probe_traffic = profile_figure("probe_search_production_window_1024x16384.md", "DRAM bytes per lookup") if prod else None
+    score_traffic = profile_figure("score_block_production_window_1024x16384.md", "DRAM bytes per request") if prod else None
+    score_kernel = "score_block_kernel" if 256 < I <= 1024 else "score_rows_kernel"
     if dominant == "probe":
         achieved = probe_bytes / (probe_ms / 1000) / 1e9
         roof = {"bound": "hbm", "kernel": "probe_search_kernel + probe_derived_kernel", "achieved": achieved,
@@ -485,7 +489,7 @@ def main():
                                      "per-request pick written to device buffers",
                              "ms": score_call_ms, "scorings_per_s": job_rate(world, R * I, score_call_ms),
                              "kernel_ms": skm,
-                             "score_roofline": {"bound": "hbm", "kernel": "score_rows_kernel",
+                             "score_roofline": {"bound": "hbm", "kernel": score_kernel,
                                                 "achieved": score_achieved, "peak": peak, "unit": "GB/s",
                                                 "frac": score_achieved / peak, "peak_source": peak_src,
                                                 "algorithmic_bytes_per_launch": score_bytes,
