@@ -871,6 +871,7 @@ __device__ void summary_rows(const psk::RowPre* __restrict__ rows, uint32_t R, u
   const InstSmem a = inst_smem(smem_raw, Ip);
   __shared__ psk::RowPre s_row;
   __shared__ int32_t s_jm[16];  // pick of request x in s_jm[x & 15] (-1: rejected)
+  static_assert(psk::kLcpBack <= psk::kSpecLag + 16, "the ring holds the picks the row's raises need");
   __shared__ uint32_t s_wmin[psk::kSumWarps];
   __shared__ uint32_t s_wb[psk::kSumWarps];
   __shared__ unsigned long long s_kb[psk::kSumWarps];
@@ -888,6 +889,28 @@ __device__ void summary_rows(const psk::RowPre* __restrict__ rows, uint32_t R, u
     const int64_t need = (int64_t)s - psk::kSpecLag;  // decisions [0, need) count for row s
     const long long c0 = clock64();
     long long c1 = c0;
+    // Each warp waits for the row's probed hits and loads its threads' hits and T_pf right away, so
+    // the loads are in flight while warp 0 replays the decisions the row must see.
+    const uint32_t slot = s % psk::kHitSlots;
+    uint32_t hl[IPT], tl[IPT];
+    {
+      bool rdy = true;
+      if (lane == 0) {
+        rdy = wait_flag(sync.ready + s, err, sync.wait_ns);
+        if (!rdy) s_abort = 1;
+      }
+      rdy = __shfl_sync(0xffffffffu, rdy ? 1 : 0, 0) != 0;
+#pragma unroll
+      for (int k = 0; k < IPT; ++k) {
+        const uint32_t i = t + (uint32_t)k * kPipeThreads;
+        hl[k] = 0u;
+        tl[k] = psk::kNoTpfBits;
+        if (rdy && i < I) {
+          hl[k] = __ldcg(sync.hitring + (uint64_t)slot * Ip + i);
+          tl[k] = __float_as_uint(__ldcg(sync.tpfring + (uint64_t)slot * Ip + i));
+        }
+      }
+    }
     if (warp == 0) {
       // Replay decisions [applied, need), 32 at a time: the adds commute; the last lane of each
       // instance refreshes its terms once every add is in.
@@ -918,10 +941,7 @@ __device__ void summary_rows(const psk::RowPre* __restrict__ rows, uint32_t R, u
         applied += nbatch;
       }
       c1 = clock64();
-      if (lane == 0) {
-        if (abort) s_abort = 1;
-        else if (!wait_flag(sync.ready + s, err, sync.wait_ns)) s_abort = 1;  // the row's probed hits
-      }
+      if (lane == 0 && abort) s_abort = 1;
       if (lane < psk::kRowWords)
         reinterpret_cast<uint4*>(&s_row)[lane] = __ldg(reinterpret_cast<const uint4*>(rows + s) + lane);
     }
@@ -933,7 +953,6 @@ __device__ void summary_rows(const psk::RowPre* __restrict__ rows, uint32_t R, u
     }
     if (s_abort) break;  // block-uniform
     const psk::RowConst rc = row_of(s_row);
-    const uint32_t slot = s % psk::kHitSlots;
     // raises from the picks of requests s - kLcpBack .. s - kSpecLag - 1 (older than the lag)
     constexpr int kNR = psk::kLcpBack - psk::kSpecLag;
     int32_t rj[kNR > 0 ? kNR : 1];
@@ -955,8 +974,8 @@ __device__ void summary_rows(const psk::RowPre* __restrict__ rows, uint32_t R, u
       pk[k].key = psk::kNoKey;
       hk[k] = 0u;
       if (i < I) {
-        const uint32_t h0 = __ldcg(sync.hitring + (uint64_t)slot * Ip + i);
-        const uint32_t tp0 = __float_as_uint(__ldcg(sync.tpfring + (uint64_t)slot * Ip + i));
+        const uint32_t h0 = hl[k];
+        const uint32_t tp0 = tl[k];
         uint32_t h = h0;
 #pragma unroll
         for (int q = 0; q < kNR; ++q)

@@ -63,12 +63,12 @@ struct DeltaSlot {
 
 // Greedy pipeline depth: a probe for request s sees every delta insert of requests <= s - kLag, and
 // the requests s - 1 .. s - (kLag - 1) are covered by their common chain prefix with s (RowPre::lcp).
-constexpr int kLag = 13;
+constexpr int kLag = 21;
 constexpr int kLcpBack = kLag - 1;
 
 // Per-request constants of one window, computed in parallel before the greedy pass: the request's
 // chain range, the Algorithm 1 / Eq. 8 row constants, and its relations to earlier requests of the
-// window (longest common chain prefix with each of the four requests before it; the deepest earlier
+// window (longest common chain prefix with each of the kLcpBack requests before it; the deepest earlier
 // request whose whole chain is a prefix of this one).
 struct __align__(16) RowPre {
   uint64_t off;
@@ -87,7 +87,7 @@ struct __align__(16) RowPre {
   uint32_t lcp[kLcpBack];  // common chain prefix with requests r - 1 .. r - kLcpBack (blocks)
 };
 constexpr int kRowWords = (int)(sizeof(RowPre) / 16);
-static_assert(sizeof(RowPre) % 16 == 0 && kRowWords == 7, "RowPre is seven 16-byte words");
+static_assert(sizeof(RowPre) % 16 == 0 && kRowWords <= 32, "RowPre is whole 16-byte words, staged by one warp");
 
 // Hand-offs between the blocks of the pipelined greedy (one cooperative launch): the deciding
 // block publishes each decision as a job, insert blocks put the job's chain blocks into the delta

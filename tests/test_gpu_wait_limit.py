@@ -3,7 +3,7 @@
 The pipelined greedy pass (search mode) is a cooperative launch whose thread blocks hand each other
 decisions, inserted blocks and probed hit rows through flags in device memory, each wait bounded by
 the context's wait limit.  Here the limit is set to 1 us on a window whose first request must cache
-a 65536-block chain tail: the rows 13 requests later can be probed only after that insert is done,
+a 65536-block chain tail: the rows a fixed lag (21 requests) later can be probed only after that insert is done,
 which takes far longer than 1 us, so some wait must give up.  The call has to return
 PS_ERR_TIMEOUT (every block of the launch ended, or the call would not return), and the same context
 with the default limit must then schedule the same window exactly as the oracle does.
