@@ -253,8 +253,11 @@ def run_streaming(args):
     """Streaming workload (1024 instances, 1000-request windows, state carried across windows):
     per window one schedule, commit and advance (engine progress + leaf-first LRU eviction), with
     the window's arrays copied from page-locked host memory inside the timed region.  Windows are
-    drawn by the generator before timing (its cost is not the scheduler's).  Prints one JSON line:
-    end-to-end decisions/s and the share of each kernel."""
+    drawn by the generator outside the timed region (its cost is not the scheduler's): all before
+    timing for short runs, each just before it is scheduled for long ones (more than 64 windows, whose
+    pinned copies would not all fit).  The time of a window is the device time of its three calls
+    (CUDA events around them); the run's time is their sum.  Prints one JSON line: decisions/s and the
+    share of each kernel."""
     import torch
     import workload as W
     import paper_2609_33224_gb300 as P
@@ -266,15 +269,20 @@ def run_streaming(args):
     ins = wl.instances
     Rw = wl.window.R
     n_win = args.warmup + args.steps
-    wins = [wl.window] + [wl.next_window() for _ in range(n_win - 1)]
-    maxb = max(int(w.chain_off[-1]) for w in wins)
+    lazy = n_win > 64
 
     def pinned(w):
         view = {np.dtype(np.uint64): np.int64, np.dtype(np.uint32): np.int32}
         return W.Window(**{k: torch.from_numpy(np.ascontiguousarray(getattr(w, k)).view(
             view.get(getattr(w, k).dtype, getattr(w, k).dtype))).pin_memory() for k in w.__dataclass_fields__})
 
-    hwins = [pinned(w) for w in wins]
+    if lazy:
+        maxb = 8192 * Rw  # every chain is at most 8192 blocks (128K tokens)
+        hwins = None
+    else:
+        wins = [wl.window] + [wl.next_window() for _ in range(n_win - 1)]
+        maxb = max(int(w.chain_off[-1]) for w in wins)
+        hwins = [pinned(w) for w in wins]
     stream = torch.cuda.current_stream()
     sched = P.Scheduler(ins.I, ins.cap_blocks, Rw, maxb, wl.model, table_load_factor=wl.table_load_factor,
                         device=local, stream=stream.cuda_stream, probe_mode=P.PS_PROBE_SEARCH, track_lru=True,
@@ -285,27 +293,32 @@ def run_streaming(args):
     paths = np.zeros(3, np.int64)
     ea, eb = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    total_ms = 0.0
     with ClockSampler(local) as clk:
         for w in range(n_win):
-            if w == args.warmup:
-                torch.cuda.synchronize()
-                e0.record(stream)
-            out = sched.schedule_window(hwins[w])
+            if lazy:
+                hw = pinned(wl.window if w == 0 else wl.next_window())
+            else:
+                hw = hwins[w]
+            torch.cuda.synchronize()
+            e0.record(stream)
+            out = sched.schedule_window(hw)
             sched.commit_window(last_use=w + 1)
             t = sched.timings()
             ea.record(stream)
             sched.advance_window(20.0, 1000, evict=True)
             eb.record(stream)
+            e1.record(stream)
+            torch.cuda.synchronize()
             if w >= args.warmup:
-                torch.cuda.synchronize()
+                total_ms += e0.elapsed_time(e1)
                 for k in ("probe", "score", "greedy", "commit"):
                     kern[k] += max(0.0, t[k])
                 kern["advance"] += ea.elapsed_time(eb)
                 paths += np.bincount(out["path"].astype(np.int64), minlength=3)
-        e1.record(stream)
-        torch.cuda.synchronize()
-    ms = max_over_ranks(e0.elapsed_time(e1) / args.steps, f"cuda:{local}")
+    ms = max_over_ranks(total_ms / args.steps, f"cuda:{local}")
     km = {k: v / args.steps for k, v in kern.items()}
+    cached = sched.cached_blocks()
     sched.close()
     line = {"metric": "streaming scheduling decisions/sec (schedule + commit + advance per window) at 1 GB300",
             "value": job_rate(world, Rw, ms), "unit": "decisions/s", "n_gpus": world, "steps": args.steps,
@@ -318,6 +331,9 @@ def run_streaming(args):
                        "path_counts": paths.tolist()},
             "kernel_ms_per_window": km,
             "greedy_share": km["greedy"] / ms if ms > 0 else None,
+            "advance_share": km["advance"] / ms if ms > 0 else None,
+            "cached_blocks_after": {"min": int(cached.min()), "max": int(cached.max()),
+                                    "capacity": int(np.max(ins.cap_blocks))},
             "scorings_per_s": job_rate(world, Rw * ins.I, ms),
             "clocks": clk.summary()}
     if rank == 0:

@@ -30,6 +30,7 @@ def test_probe_algorithmic_bytes_from_launch_counters():
 def test_traffic_figures_are_read_from_the_committed_profiles():
     assert bench.profile_figure("greedy_pipe_production_window_1024x8192.md", "DRAM bytes per request") > 8 * 1024
     assert bench.profile_figure("score_block_production_window_1024x16384.md", "DRAM bytes per request") > 0
+    assert bench.profile_figure("probe_search_production_window_1024x16384.md", "DRAM bytes per lookup") > 32
     assert bench.profile_figure("no_such_summary.md", "DRAM bytes per request") is None
 
 
