@@ -418,21 +418,33 @@ def main():
     ms = max_over_ranks(e0.elapsed_time(e1) / args.steps, f"cuda:{local}")
     path_counts = np.bincount(out["path"].cpu().numpy().astype(np.int64), minlength=3).tolist()
 
-    # e2e: same step through the C ABI with page-locked host inputs and host outputs
-    hwin = W.Window(**{k: torch.from_numpy(np.ascontiguousarray(getattr(win, k)).view(
-        {np.dtype(np.uint64): np.int64, np.dtype(np.uint32): np.int32}.get(getattr(win, k).dtype,
-                                                                           getattr(win, k).dtype))).pin_memory()
-        for k in win.__dataclass_fields__})
-    sched.schedule_window(hwin, scores=("best", "path"))
-    torch.cuda.synchronize()
-    if dist_on:
-        dist.barrier()
-    t0 = time.perf_counter()
-    for _ in range(args.steps):
-        sched.schedule_window(hwin, scores=("best", "path"))
-    torch.cuda.synchronize()
-    e2e_ms = max_over_ranks(1000 * (time.perf_counter() - t0) / args.steps, f"cuda:{local}")
-    h2d = int(8 * (R + 1) + 8 * nb.sum() + 12 * R)
+    # e2e: the same step through the C ABI with page-locked host inputs and host outputs, the window
+    # in the shared-prefix form (each request's own blocks and a parent link, ps_window.parent: what a
+    # gateway that tracks sessions sends; the library rebuilds the chains on the device), and again
+    # with every chain sent whole.
+    def pinned(w):
+        return type(w)(**{k: torch.from_numpy(np.ascontiguousarray(getattr(w, k)).view(
+            {np.dtype(np.uint64): np.int64, np.dtype(np.uint32): np.int32}.get(getattr(w, k).dtype,
+                                                                               getattr(w, k).dtype))).pin_memory()
+            for k in w.__dataclass_fields__})
+
+    def e2e_time(hw):
+        sched.schedule_window(hw, scores=("best", "path"))
+        torch.cuda.synchronize()
+        if dist_on:
+            dist.barrier()
+        t0 = time.perf_counter()
+        for _ in range(args.steps):
+            sched.schedule_window(hw, scores=("best", "path"))
+        torch.cuda.synchronize()
+        return max_over_ranks(1000 * (time.perf_counter() - t0) / args.steps, f"cuda:{local}")
+
+    twin = W.tree_window(win)
+    own_blocks = int(twin.chain_off[-1])
+    e2e_ms = e2e_time(pinned(twin))
+    e2e_full_ms = e2e_time(pinned(win))
+    h2d = int(8 * (R + 1) + 8 * own_blocks + 4 * R + 12 * R)
+    h2d_full = int(8 * (R + 1) + 8 * nb.sum() + 12 * R)
     d2h = int(R * (4 + 1 + 4) + R * (4 + 1))
 
     # The scoring call alone (ps_score_window, rows A1-A6): every per-pair output (hits, TPOT, TTFT,
@@ -512,7 +524,11 @@ def main():
                                                 "traffic": (None if score_traffic is None
                                                             else score_traffic * R)}},
             "e2e": {"value": job_rate(world, R * I, e2e_ms), "unit": "scorings/s", "ms_per_step": e2e_ms,
-                    "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+                    "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+                    "window_form": f"shared-prefix: {own_blocks} own blocks of {int(nb.sum())}, parent links"},
+            "e2e_full_chains": {"value": job_rate(world, R * I, e2e_full_ms), "unit": "scorings/s",
+                                "ms_per_step": e2e_full_ms, "h2d_bytes_per_step": h2d_full,
+                                "d2h_bytes_per_step": d2h},
             # per step: window validation, last-block table, relations, base, probe (scratch rows),
             # probe (derived rows), score, greedy
             "gpu_launches": 8 * args.steps,

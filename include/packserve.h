@@ -162,7 +162,7 @@ typedef struct {
 /* One window of requests in arrival order (Algorithm 1's request r: a session's token prefix as a
  * chain of block hashes, plus its SLO targets).
  *   chain_off      [R+1], chain_off[0] = 0, non-decreasing; request r's chain is
- *                  chain_hash[chain_off[r] .. chain_off[r+1]).
+ *                  chain_hash[chain_off[r] .. chain_off[r+1]) (with parent: its own blocks, below).
  *   chain_hash     [chain_off[R]] block hashes.
  *   prompt_tokens  [R] input length L_r in tokens; its chain must have exactly L_r / 16 blocks
  *                  (full blocks only).  L_r < 2^30.
@@ -170,6 +170,14 @@ typedef struct {
  *   out_tokens     [R] output length of each request (only read by ps_commit_window on a context
  *                  with request tracking, to queue the admitted requests; may be NULL otherwise).
  *   inputs_on_device  0: all arrays are host memory, 1: all are device memory.
+ *   parent         [R] or NULL.  The shared-prefix (prefix-tree) form of the window: an agentic
+ *                  session resends its whole history with every step (Section 3), so a request's
+ *                  prompt usually extends an earlier request's.  parent[r] = p (0 <= p < r) says that
+ *                  request r's chain starts with request p's whole chain, and chain_hash[chain_off[r]
+ *                  .. chain_off[r+1]) then holds only the blocks after it (L_r/16 - L_p/16 of them);
+ *                  parent[r] = -1 gives the whole chain as usual.  The library rebuilds every chain on
+ *                  the device (one pass over the window), so the host sends each shared prefix once.
+ *                  Host inputs only (inputs_on_device 0); NULL: every chain is given whole.
  * A window with device inputs is read in place; its buffers must stay unchanged until the window is
  * committed or discarded (ps_commit_window / the next ps_schedule_window). */
 typedef struct {
@@ -181,6 +189,7 @@ typedef struct {
   const float* tpot_target;
   const uint32_t* out_tokens;
   int32_t inputs_on_device;
+  const int32_t* parent;
 } ps_window;
 
 /* Per-pair and per-request scoring outputs.  Any pointer may be NULL (not wanted).
@@ -451,7 +460,8 @@ PS_API ps_status ps_last_probe_stats(ps_ctx* ctx, uint64_t* out, uint32_t n);
  *            full when it was inserted, it is stored in the first bucket after b1 (wrapping) that
  *            had a free slot, and b1 and every bucket passed on the way carry overflow bit 1.
  *   state    device arrays of the instance state (ps_instance_state fields, structure of arrays).
- *   window   inputs_on_device must be 1; out->outputs_on_device must be 1 (all device buffers).
+ *   window   inputs_on_device must be 1 and parent NULL; out->outputs_on_device must be 1 (all
+ *            device buffers).
  *   probe_mode  as ps_config.probe_mode (PS_PROBE_SEARCH only for prefix-closed caches).
  *   cuda_stream  the stream to run on; the call synchronises it before returning.
  * The hit matrix it needs in between is kept in a fixed device array inside the library

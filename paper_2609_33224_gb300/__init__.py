@@ -68,7 +68,7 @@ class PsWindow(ctypes.Structure):
     _fields_ = [("R", ctypes.c_uint32), ("chain_off", ctypes.c_void_p), ("chain_hash", ctypes.c_void_p),
                 ("prompt_tokens", ctypes.c_void_p), ("ttft_target", ctypes.c_void_p),
                 ("tpot_target", ctypes.c_void_p), ("out_tokens", ctypes.c_void_p),
-                ("inputs_on_device", ctypes.c_int32)]
+                ("inputs_on_device", ctypes.c_int32), ("parent", ctypes.c_void_p)]
 
 
 class PsScores(ctypes.Structure):
@@ -358,14 +358,16 @@ class Scheduler:
         w = PsWindow()
         arrs = [(window.chain_off, np.uint64), (window.chain_hash, np.uint64),
                 (window.prompt_tokens, np.uint32), (window.ttft_target, np.float32),
-                (window.tpot_target, np.float32), (getattr(window, "out_tokens", None), np.uint32)]
+                (window.tpot_target, np.float32), (getattr(window, "out_tokens", None), np.uint32),
+                (getattr(window, "parent", None), np.int32)]
         ptrs = [_ptr(a, d) for a, d in arrs]
         dev = {p[1] for p in ptrs if p[1] is not None}
         if len(dev) > 1:
             raise ValueError("window arrays must all be host or all be device")
         n_off = window.chain_off.numel() if _is_torch(window.chain_off) else window.chain_off.shape[0]
         w.R = int(n_off) - 1
-        w.chain_off, w.chain_hash, w.prompt_tokens, w.ttft_target, w.tpot_target, w.out_tokens = (p[0] for p in ptrs)
+        (w.chain_off, w.chain_hash, w.prompt_tokens, w.ttft_target, w.tpot_target, w.out_tokens,
+         w.parent) = (p[0] for p in ptrs)
         w.inputs_on_device = 1 if dev == {True} else 0
         return w
 

@@ -16,7 +16,7 @@ ROOT = os.path.dirname(HERE)
 CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(BUILD, "libpackserve.so")
-SOURCES = ["api.cu", "probe.cu", "score.cu", "greedy.cu", "relations.cu", "table.cu", "noalloc.cu"]
+SOURCES = ["api.cu", "probe.cu", "score.cu", "greedy.cu", "relations.cu", "table.cu", "noalloc.cu", "window.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 # host code is compiled without floating-point contraction (calibrate.h is exact fp32, op by op)
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-fvisibility=hidden",

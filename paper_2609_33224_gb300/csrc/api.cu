@@ -65,6 +65,11 @@ struct ps_ctx {
   psk::StateSoA st{}, pend{};
   uint64_t* d_off = nullptr;
   uint64_t* d_hash = nullptr;
+  // shared-prefix windows (ps_window.parent): each request's own blocks and parent link, staged
+  uint64_t* d_own_off = nullptr;
+  uint64_t* d_own_hash = nullptr;
+  int32_t* d_parent = nullptr;
+  std::vector<uint64_t> h_full_off;
   uint32_t* d_L = nullptr;
   float* d_ttft = nullptr;
   float* d_tpot = nullptr;
@@ -218,6 +223,66 @@ ps_status check_capacity(ps_ctx* c) {
   return PS_OK;
 }
 
+// Copies the request arrays shared by both window forms (L, targets, output lengths) to the device.
+ps_status stage_request_arrays(ps_ctx* c, const ps_window* w) {
+  if (!w->R) return PS_OK;
+  PS_TRY_CUDA(c, cudaMemcpyAsync(c->d_L, w->prompt_tokens, w->R * sizeof(uint32_t), cudaMemcpyHostToDevice, c->stream));
+  PS_TRY_CUDA(c, cudaMemcpyAsync(c->d_ttft, w->ttft_target, w->R * sizeof(float), cudaMemcpyHostToDevice, c->stream));
+  PS_TRY_CUDA(c, cudaMemcpyAsync(c->d_tpot, w->tpot_target, w->R * sizeof(float), cudaMemcpyHostToDevice, c->stream));
+  if (w->out_tokens) {
+    PS_TRY_CUDA(c, cudaMemcpyAsync(c->d_outtok, w->out_tokens, w->R * sizeof(uint32_t), cudaMemcpyHostToDevice,
+                                   c->stream));
+    c->pend_out = c->d_outtok;
+  }
+  return PS_OK;
+}
+
+// Shared-prefix form (host inputs): validate the parent links and own-block counts, send each
+// request's own blocks, and rebuild the full chains on the device.
+ps_status stage_window_tree(ps_ctx* c, const ps_window* w, psk::WindowDev* out) {
+  const uint32_t R = w->R;
+  const uint64_t* own = w->chain_off;
+  if (own[0] != 0) return fail(c, PS_ERR_INVALID, "chain_off[0] must be 0");
+  std::vector<uint64_t>& full = c->h_full_off;
+  full.assign((size_t)R + 1, 0);
+  for (uint32_t r = 0; r < R; ++r) {
+    const uint32_t L = w->prompt_tokens[r];
+    const int32_t p = w->parent[r];
+    if (L >= (1u << 30)) return fail(c, PS_ERR_INVALID, "request " + std::to_string(r) + ": L must be < 2^30");
+    if (p < -1 || p >= (int64_t)r)
+      return fail(c, PS_ERR_INVALID, "request " + std::to_string(r) + ": parent must be -1 or an earlier request");
+    const uint64_t nb = L / 16u;
+    const uint64_t pb = p >= 0 ? full[(size_t)p + 1] - full[(size_t)p] : 0;
+    if (own[r + 1] < own[r] || nb < pb || own[r + 1] - own[r] != nb - pb)
+      return fail(c, PS_ERR_INVALID, "request " + std::to_string(r) +
+                                         ": own blocks must be L/16 minus the parent's chain length");
+    full[(size_t)r + 1] = full[r] + nb;
+  }
+  const uint64_t nblk = full[R], nown = own[R];
+  if (nblk > c->max_blocks) return fail(c, PS_ERR_INVALID, "window exceeds max_window_chain_blocks");
+  if (nown > 0 && !w->chain_hash) return fail(c, PS_ERR_INVALID, "chain_hash is NULL");
+  PS_TRY_CUDA(c, cudaMemcpyAsync(c->d_off, full.data(), ((size_t)R + 1) * sizeof(uint64_t), cudaMemcpyHostToDevice,
+                                 c->stream));
+  if (R) {
+    PS_TRY_CUDA(c, cudaMemcpyAsync(c->d_own_off, own, ((size_t)R + 1) * sizeof(uint64_t), cudaMemcpyHostToDevice,
+                                   c->stream));
+    PS_TRY_CUDA(c, cudaMemcpyAsync(c->d_parent, w->parent, R * sizeof(int32_t), cudaMemcpyHostToDevice, c->stream));
+  }
+  if (nown)
+    PS_TRY_CUDA(c, cudaMemcpyAsync(c->d_own_hash, w->chain_hash, nown * sizeof(uint64_t), cudaMemcpyHostToDevice,
+                                   c->stream));
+  ps_status s = stage_request_arrays(c, w);
+  if (s != PS_OK) return s;
+  PS_TRY_CUDA(c, pskl::launch_expand_chains(c->d_off, c->d_own_off, c->d_own_hash, c->d_parent, R, c->d_hash, c->d_err,
+                                            c->num_sms, c->stream));
+  out->off = c->d_off;
+  out->hash = c->d_hash;
+  out->L = c->d_L;
+  out->ttft_t = c->d_ttft;
+  out->tpot_t = c->d_tpot;
+  return PS_OK;
+}
+
 // Validate a window and make its arrays available on the device.
 ps_status stage_window(ps_ctx* c, const ps_window* w, psk::WindowDev* out) {
   if (!w) return fail(c, PS_ERR_INVALID, "window is NULL");
@@ -229,6 +294,7 @@ ps_status stage_window(ps_ctx* c, const ps_window* w, psk::WindowDev* out) {
   out->R = w->R;
   c->pend_out = nullptr;
   if (w->inputs_on_device) {
+    if (w->parent) return fail(c, PS_ERR_INVALID, "a window with parent links must be in host memory");
     c->pend_out = w->out_tokens;
     out->off = w->chain_off;
     out->hash = w->chain_hash;
@@ -245,6 +311,7 @@ ps_status stage_window(ps_ctx* c, const ps_window* w, psk::WindowDev* out) {
     }
     return PS_OK;
   }
+  if (w->parent) return stage_window_tree(c, w, out);
   const uint64_t* off = w->chain_off;
   if (off[0] != 0) return fail(c, PS_ERR_INVALID, "chain_off[0] must be 0");
   for (uint32_t r = 0; r < w->R; ++r) {
@@ -258,16 +325,8 @@ ps_status stage_window(ps_ctx* c, const ps_window* w, psk::WindowDev* out) {
   PS_TRY_CUDA(c, cudaMemcpyAsync(c->d_off, off, (w->R + 1) * sizeof(uint64_t), cudaMemcpyHostToDevice, c->stream));
   if (nblk)
     PS_TRY_CUDA(c, cudaMemcpyAsync(c->d_hash, w->chain_hash, nblk * sizeof(uint64_t), cudaMemcpyHostToDevice, c->stream));
-  if (w->R) {
-    PS_TRY_CUDA(c, cudaMemcpyAsync(c->d_L, w->prompt_tokens, w->R * sizeof(uint32_t), cudaMemcpyHostToDevice, c->stream));
-    PS_TRY_CUDA(c, cudaMemcpyAsync(c->d_ttft, w->ttft_target, w->R * sizeof(float), cudaMemcpyHostToDevice, c->stream));
-    PS_TRY_CUDA(c, cudaMemcpyAsync(c->d_tpot, w->tpot_target, w->R * sizeof(float), cudaMemcpyHostToDevice, c->stream));
-    if (w->out_tokens) {
-      PS_TRY_CUDA(c, cudaMemcpyAsync(c->d_outtok, w->out_tokens, w->R * sizeof(uint32_t), cudaMemcpyHostToDevice,
-                                     c->stream));
-      c->pend_out = c->d_outtok;
-    }
-  }
+  ps_status s = stage_request_arrays(c, w);
+  if (s != PS_OK) return s;
   out->off = c->d_off;
   out->hash = c->d_hash;
   out->L = c->d_L;
@@ -420,7 +479,9 @@ ps_status ps_create(const ps_config* cfg, ps_ctx** out) {
          dalloc(c, &s->M, I) == cudaSuccess && dalloc(c, &s->Bmax, I) == cudaSuccess;
   }
   ok = ok && dalloc(c, &c->d_off, (size_t)c->Rmax + 1) == cudaSuccess &&
-       dalloc(c, &c->d_hash, c->max_blocks) == cudaSuccess && dalloc(c, &c->d_L, c->Rmax) == cudaSuccess &&
+       dalloc(c, &c->d_hash, c->max_blocks) == cudaSuccess &&
+       dalloc(c, &c->d_own_off, (size_t)c->Rmax + 1) == cudaSuccess &&
+       dalloc(c, &c->d_own_hash, c->max_blocks) == cudaSuccess && dalloc(c, &c->d_parent, c->Rmax) == cudaSuccess && dalloc(c, &c->d_L, c->Rmax) == cudaSuccess &&
        dalloc(c, &c->d_ttft, c->Rmax) == cudaSuccess && dalloc(c, &c->d_tpot, c->Rmax) == cudaSuccess &&
        dalloc(c, &c->d_hits, RI) == cudaSuccess && dalloc(c, &c->d_tpf, RI) == cudaSuccess && dalloc(c, &c->d_tpot_o, RI) == cudaSuccess &&
        dalloc(c, &c->d_ttft_o, RI) == cudaSuccess && dalloc(c, &c->d_cls, RI) == cudaSuccess &&

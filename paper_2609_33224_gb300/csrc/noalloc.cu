@@ -113,7 +113,7 @@ ps_status ps_score_window_noalloc(const uint64_t* slots, const uint64_t* overflo
       (reinterpret_cast<uintptr_t>(tables) & 7u))
     return PS_ERR_INVALID;
   if (num_instances < 1 || num_instances > 4096) return PS_ERR_INVALID;
-  if (w->inputs_on_device != 1 || out->outputs_on_device != 1) return PS_ERR_INVALID;
+  if (w->inputs_on_device != 1 || out->outputs_on_device != 1 || w->parent) return PS_ERR_INVALID;
   if (probe_mode != PS_PROBE_LINEAR && probe_mode != PS_PROBE_SEARCH) return PS_ERR_INVALID;
   if (!state->b || !state->qr || !state->q_tokens || !state->S_tokens || !state->M_KV_tokens || !state->B_max)
     return PS_ERR_INVALID;

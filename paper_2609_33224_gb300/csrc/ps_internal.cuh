@@ -1052,6 +1052,11 @@ cudaError_t launch_greedy(const uint64_t* slots, const uint64_t* ovf, const psk:
                           uint64_t delta_nslots, int32_t* assign, uint8_t* path, uint32_t* hit_chosen,
                           uint32_t* err, int search, cudaStream_t s);
 cudaError_t launch_delta_clear(psk::DeltaSlot* delta, uint64_t nslots, cudaStream_t s);
+// Rebuilds every chain of a window in the shared-prefix form (ps_window.parent) into hash (CSR at
+// full_off) from each request's own blocks (CSR at own_off) and its parent link.
+cudaError_t launch_expand_chains(const uint64_t* full_off, const uint64_t* own_off, const uint64_t* own_hash,
+                                 const int32_t* parent, uint32_t R, uint64_t* hash, uint32_t* err, int num_sms,
+                                 cudaStream_t s);
 cudaError_t launch_relations(const psk::WindowDev& w, const psk::DevModel& m, psk::LastSlot* tab, uint32_t tab_n,
                              psk::RowPre* rows, psk::RowList list, int num_sms, cudaStream_t s);
 cudaError_t launch_greedy_search(const psk::RowPre* rows, const psk::WindowDev& w, uint32_t I, const uint32_t* hit0,

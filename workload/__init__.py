@@ -180,6 +180,53 @@ class Instances:
         return int(self.b.shape[0])
 
 
+@dataclass
+class TreeWindow:
+    """A window in the shared-prefix form: request r's chain is request parent[r]'s whole chain
+    followed by its own blocks chain_hash[chain_off[r]:chain_off[r+1]] (parent -1: the whole chain)."""
+    chain_off: np.ndarray      # u64[R+1] own blocks
+    chain_hash: np.ndarray     # u64[sum own]
+    prompt_tokens: np.ndarray  # u32[R]
+    ttft_target: np.ndarray    # f32[R]
+    tpot_target: np.ndarray    # f32[R]
+    session: np.ndarray        # u32[R]
+    out_tokens: np.ndarray     # u32[R]
+    parent: np.ndarray         # i32[R]
+
+    @property
+    def R(self) -> int:
+        return int(self.prompt_tokens.shape[0])
+
+
+def tree_window(win: Window) -> TreeWindow:
+    """The shared-prefix form of a window: each request's parent is the latest earlier request of its
+    session whose chain is a prefix of its own (chained block hashes: equal hashes at the parent's
+    last position mean equal prefixes), and only the blocks after the parent's chain are kept."""
+    off = win.chain_off.astype(np.int64)
+    R = win.R
+    parent = np.full(R, -1, np.int32)
+    by_session: dict = {}
+    for r in range(R):
+        a, b = int(off[r]), int(off[r + 1])
+        for p in reversed(by_session.get(int(win.session[r]), [])):
+            pa, pb = int(off[p]), int(off[p + 1])
+            n = pb - pa
+            if 0 < n <= b - a and win.chain_hash[pb - 1] == win.chain_hash[a + n - 1]:
+                parent[r] = p
+                break
+        by_session.setdefault(int(win.session[r]), []).append(r)
+    keep = np.ones(int(off[-1]), bool)
+    own = np.zeros(R + 1, np.uint64)
+    for r in range(R):
+        p = int(parent[r])
+        n = int(off[p + 1] - off[p]) if p >= 0 else 0
+        keep[int(off[r]):int(off[r]) + n] = False
+        own[r + 1] = own[r] + np.uint64(int(off[r + 1] - off[r]) - n)
+    return TreeWindow(chain_off=own, chain_hash=win.chain_hash[keep].astype(np.uint64),
+                      prompt_tokens=win.prompt_tokens, ttft_target=win.ttft_target, tpot_target=win.tpot_target,
+                      session=win.session, out_tokens=win.out_tokens, parent=parent)
+
+
 def column_block(ins: Instances, lo: int, hi: int) -> Instances:
     """Instances lo .. hi - 1 of a pool as a pool of their own (ids renumbered from 0): the seed
     chains cached on them and their state."""
