@@ -836,31 +836,7 @@ __device__ __forceinline__ unsigned long long warp_min_u64w(unsigned long long v
   return ((unsigned long long)mhi << 32) | mlo;
 }
 
-// Bounded spin on a shared-memory counter until it reaches `want` (then an acquire fence) or *abort
-// is set; false on timeout (error bit set) or abort.  An iteration is one shared load and a compare;
-// the bound is counted in SM cycles, 3 per ns (at least the time limit at any clock up to 3 GHz).
-__device__ __forceinline__ bool wait_smem_at_least(const uint32_t* p, uint32_t want, const volatile int* abort,
-                                                   uint32_t* err, uint64_t limit_ns) {
-  if (psk::ld_relaxed_cta_shared_u32(p) >= want) {
-    psk::fence_acq_rel_cta();
-    return true;
-  }
-  const long long c0 = clock64();
-  const long long lim = (long long)(limit_ns * 3ull);
-  for (uint32_t it = 1;; ++it) {
-    if (psk::ld_relaxed_cta_shared_u32(p) >= want) {
-      psk::fence_acq_rel_cta();
-      return true;
-    }
-    if ((it & 31u) == 0u) {
-      if (*abort) return false;
-      if (clock64() - c0 > lim) {
-        atomicOr(err, psk::kErrTimeout);
-        return false;
-      }
-    }
-  }
-}
+using psk::wait_smem_at_least;
 
 // Summary block sb: rows sb, sb + kSummaryBlocks, ...  Thread t holds instances t, t + 256, ...
 template <int IPT>

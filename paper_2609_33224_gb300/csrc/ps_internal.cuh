@@ -566,6 +566,32 @@ __device__ __forceinline__ uint64_t globaltimer_ns() {
   return x;
 }
 
+// Bounded spin on a shared-memory counter until it reaches `want` (then an acquire fence) or *abort
+// is set; false on timeout (error bit set) or abort.  An iteration is one shared load and a compare;
+// the bound is counted in SM cycles, 3 per ns (at least the time limit at any clock up to 3 GHz).
+__device__ __forceinline__ bool wait_smem_at_least(const uint32_t* p, uint32_t want, const volatile int* abort,
+                                                   uint32_t* err, uint64_t limit_ns) {
+  if (ld_relaxed_cta_shared_u32(p) >= want) {
+    fence_acq_rel_cta();
+    return true;
+  }
+  const long long c0 = clock64();
+  const long long lim = (long long)(limit_ns * 3ull);
+  for (uint32_t it = 1;; ++it) {
+    if (ld_relaxed_cta_shared_u32(p) >= want) {
+      fence_acq_rel_cta();
+      return true;
+    }
+    if ((it & 31u) == 0u) {
+      if (*abort) return false;
+      if (clock64() - c0 > lim) {
+        atomicOr(err, kErrTimeout);
+        return false;
+      }
+    }
+  }
+}
+
 // 16-byte asynchronous global -> shared copy (completes at cp_async_wait_all of the same thread).
 __device__ __forceinline__ void cp_async16(void* smem, const void* gmem) {
   asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"((uint32_t)__cvta_generic_to_shared(smem)), "l"(gmem)

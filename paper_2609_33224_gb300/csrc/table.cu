@@ -363,9 +363,23 @@ __global__ void advance_kernel(psk::StateSoA st, uint32_t I, psk::ReqStore rq, p
 // Every evicted block only ever makes its parent a leaf, and a leaf outside the first E sorted ones
 // can never be among E evictions, so a round of at most kHeapMax evictions reproduces the
 // one-at-a-time rule exactly; the host repeats rounds while an instance is still over capacity.
+//
+// The ordered loop touches shared memory only.  A loader warp reads each parent's metadata from
+// global memory ahead of it: for the sorted leaves, up to kRing leaves past the loop's position; for
+// a parent that became a leaf, as soon as it is pushed.  Children counts are not written during the
+// loop, so every load sees the round's starting count; the loop keeps the decremented counts in a
+// shared hash table, written back at the end of the round.  A block's metadata changes in a round
+// only when it is evicted, which happens after every record that names it as a parent has been read.
+// Most evictions climb a chain (a parent goes right after its last child, when its key is below the
+// next candidate's), and such a step still waits for its record: the parent's parent is known only
+// from the parent's metadata.
 constexpr int kLeafMax = 4096;
-constexpr int kHeapMax = 1536;  // with kLeafMax, two eviction blocks fit on an SM
+constexpr int kHeapMax = 1536;
 constexpr int kEvictThreads = 256;
+constexpr int kRing = 32;          // sorted leaves whose parent records the loader keeps ready
+constexpr int kDeltaSlots = 2048;  // children counts a round changes (at most kHeapMax parents)
+constexpr uint64_t kEvictWaitNs = 1000000000ull;  // bound on any wait inside an eviction block
+static_assert(kHeapMax < kDeltaSlots, "the count table never fills");
 constexpr int kCollectThreads = 256;
 constexpr uint32_t kCollectSlotsPerThread = 8;
 
@@ -424,6 +438,113 @@ __device__ __forceinline__ Leaf heap_pop(Leaf* h, int& n) {
   return top;
 }
 
+// A parent's metadata as the loader reads it: children count at the start of the round, last_use,
+// hash and its own parent's slot.  A pool record also holds the slot it describes (a parent that
+// became a leaf names its record by index, in the heap entry's parent word).
+struct ParentRec {
+  uint32_t pc, plu, ph_lo, ph_hi, ppp;
+};
+struct PoolRec {
+  uint32_t pp;
+  ParentRec r;
+};
+static_assert(sizeof(ParentRec) == 20 && sizeof(PoolRec) == 24, "records are 32-bit words");
+
+// Shared memory of an eviction block.  The sort uses all kLeafMax leaves; a round then reads only
+// the first kHeapMax sorted ones, and the rest of that space holds the records and the count table.
+constexpr size_t kOffPool = (size_t)kHeapMax * sizeof(Leaf);
+constexpr size_t kOffRing = kOffPool + (size_t)kHeapMax * sizeof(PoolRec);
+constexpr size_t kOffDKey = kOffRing + (size_t)kRing * sizeof(ParentRec);
+constexpr size_t kOffDVal = kOffDKey + (size_t)kDeltaSlots * sizeof(uint32_t);
+constexpr size_t kOffHeapRaw = kOffDVal + (size_t)kDeltaSlots * sizeof(uint32_t);
+constexpr size_t kOffHeap =
+    kOffHeapRaw > (size_t)kLeafMax * sizeof(Leaf) ? kOffHeapRaw : (size_t)kLeafMax * sizeof(Leaf);
+constexpr size_t kEvictSmem = kOffHeap + (size_t)kHeapMax * sizeof(Leaf);
+// two eviction blocks per SM: 2 x (kEvictSmem + the static flags + 1 KB reserved) <= 228 KB
+static_assert(2 * (kEvictSmem + 64 + 1024) <= 228 * 1024, "two eviction blocks fit on an SM");
+__device__ __forceinline__ ParentRec load_parent(const uint64_t* slots, const psk::LruMeta& meta, uint32_t ps) {
+  ParentRec r{0u, 0u, 0u, 0u, kLeafNoParent};
+  if (ps != kLeafNoParent) {
+    const uint32_t pc = meta.children[ps], plu = meta.last_use[ps];
+    const uint64_t ph = slots[ps], pp = meta.parent[ps];
+    r = ParentRec{pc, plu, (uint32_t)ph, (uint32_t)(ph >> 32), parent32(pp)};
+  }
+  return r;
+}
+// The decremented children count of ps (first touch: from the round's starting count pc).
+__device__ __forceinline__ uint32_t count_dec(uint32_t* dkey, uint32_t* dval, uint32_t ps, uint32_t pc) {
+  uint32_t h = (ps * 0x9E3779B1u) >> 21;  // 11 bits: kDeltaSlots entries
+  for (int probe = 0; probe < kDeltaSlots; ++probe) {
+    const uint32_t k = dkey[h];
+    if (k == ps) return --dval[h];
+    if (k == kLeafNoParent) {
+      dkey[h] = ps;
+      dval[h] = pc - 1u;
+      return pc - 1u;
+    }
+    h = (h + 1u) & (uint32_t)(kDeltaSlots - 1);
+  }
+  return 1u;  // not reached: a round changes fewer counts than the table holds
+}
+static_assert(kDeltaSlots == 1 << 11, "count_dec hashes to 11 bits");
+
+struct EvictFlags {
+  uint32_t ptr;        // sorted leaves the loop has taken (their records may be overwritten)
+  uint32_t ring_done;  // sorted leaves whose parent records are in the ring
+  uint32_t req;        // pool records the loop has asked for
+  uint32_t pool_done;  // pool records filled
+  uint32_t exit;       // the loop has ended
+  int abort;           // the loader gave up
+};
+
+// The loader warp: fills ring records for sorted leaves [ring_done, min(m, ptr + kRing)) and pool
+// records [pool_done, req), one record of each kind per lane per pass, loads issued before any
+// record is written.  Every control value is the warp's minimum of what its lanes observed, so the
+// warp stays converged and each lane's acquire covers what it reads.
+__device__ void evict_loader(const uint64_t* slots, const psk::LruMeta& meta, const Leaf* leaves, ParentRec* ring,
+                             PoolRec* pool, uint32_t m, EvictFlags* f, uint32_t* err) {
+  const uint32_t lane = threadIdx.x & 31u;
+  uint32_t ring_done = 0, pool_done = 0;
+  const long long c0 = clock64();
+  const long long lim = (long long)(kEvictWaitNs * 3ull);
+  for (uint32_t it = 1;; ++it) {
+    uint32_t ex = psk::ld_relaxed_cta_shared_u32(&f->exit);
+    uint32_t ptr = psk::ld_relaxed_cta_shared_u32(&f->ptr);
+    uint32_t req = psk::ld_relaxed_cta_shared_u32(&f->req);
+    psk::fence_acq_rel_cta();
+    ex = __reduce_min_sync(0xffffffffu, ex);
+    ptr = __reduce_min_sync(0xffffffffu, ptr);
+    req = __reduce_min_sync(0xffffffffu, req);
+    if (ex) return;
+    const uint32_t rhi = ptr + (uint32_t)kRing < m ? ptr + (uint32_t)kRing : m;
+    const uint32_t phi = req < pool_done + 32u ? req : pool_done + 32u;
+    if (ring_done >= rhi && pool_done >= phi) {
+      if ((it & 31u) == 0u && __any_sync(0xffffffffu, clock64() - c0 > lim)) {
+        if (lane == 0) {
+          atomicOr(err, psk::kErrTimeout);
+          f->abort = 1;
+        }
+        return;
+      }
+      continue;
+    }
+    const uint32_t j = ring_done + lane, k = pool_done + lane;
+    const bool rj = j < rhi, pk = k < phi;
+    const ParentRec a = load_parent(slots, meta, rj ? leaves[j].parent : kLeafNoParent);
+    const uint32_t pp = pk ? pool[k].pp : kLeafNoParent;
+    const ParentRec b = load_parent(slots, meta, pp);
+    if (rj) ring[j % (uint32_t)kRing] = a;
+    if (pk) pool[k].r = b;
+    __syncwarp();
+    if (lane == 0) {
+      if (rhi > ring_done) psk::st_release_cta_shared_u32(&f->ring_done, rhi);
+      if (phi > pool_done) psk::st_release_cta_shared_u32(&f->pool_done, phi);
+    }
+    if (rhi > ring_done) ring_done = rhi;
+    if (phi > pool_done) pool_done = phi;
+  }
+}
+
 // grid: (slot chunks, instances)
 __global__ void __launch_bounds__(kCollectThreads)
 leaf_collect_kernel(const uint64_t* __restrict__ slots, const psk::TableDesc* __restrict__ tdesc,
@@ -447,12 +568,19 @@ leaf_collect_kernel(const uint64_t* __restrict__ slots, const psk::TableDesc* __
 __global__ void __launch_bounds__(kEvictThreads)
 evict_kernel(uint64_t* slots, unsigned long long* count, const uint64_t* __restrict__ cap, psk::LruMeta meta,
              const Leaf* __restrict__ leafbuf, const uint32_t* __restrict__ nleaf, uint32_t* more, uint32_t* err) {
-  extern __shared__ unsigned long long ev_smem[];
+  extern __shared__ __align__(16) unsigned char ev_smem[];
+  __shared__ EvictFlags flags;
   Leaf* leaves = reinterpret_cast<Leaf*>(ev_smem);
-  Leaf* heap = leaves + kLeafMax;
+  PoolRec* pool = reinterpret_cast<PoolRec*>(ev_smem + kOffPool);
+  ParentRec* ring = reinterpret_cast<ParentRec*>(ev_smem + kOffRing);
+  uint32_t* dkey = reinterpret_cast<uint32_t*>(ev_smem + kOffDKey);
+  uint32_t* dval = reinterpret_cast<uint32_t*>(ev_smem + kOffDVal);
+  Leaf* heap = reinterpret_cast<Leaf*>(ev_smem + kOffHeap);
   const uint32_t i = blockIdx.x;
   const unsigned long long cnt = count[i];
   if (cnt <= cap[i]) return;  // block-uniform
+  // an earlier round gave up: no more rounds (read once, so that the whole block leaves together)
+  if (__syncthreads_or(threadIdx.x == 0 && (*(volatile uint32_t*)err & psk::kErrTimeout) != 0u)) return;
   const uint32_t n = nleaf[i];
   if (n > (uint32_t)kLeafMax || n == 0) {
     if (threadIdx.x == 0) atomicOr(err, psk::kErrLeavesFull);
@@ -480,40 +608,73 @@ evict_kernel(uint64_t* slots, unsigned long long* count, const uint64_t* __restr
       __syncthreads();
     }
   }
-  if (threadIdx.x == 0) {
-    const uint64_t E = cnt - cap[i];
-    const uint64_t todo = E < (uint64_t)kHeapMax ? E : (uint64_t)kHeapMax;
-    uint32_t ptr = 0;
+  const uint64_t E = cnt - cap[i];
+  const uint32_t todo = E < (uint64_t)kHeapMax ? (uint32_t)E : (uint32_t)kHeapMax;
+  const uint32_t m = n < todo ? n : todo;  // sorted leaves a round can take
+  for (uint32_t x = threadIdx.x; x < (uint32_t)kDeltaSlots; x += kEvictThreads) dkey[x] = kLeafNoParent;
+  if (threadIdx.x == 0) flags = EvictFlags{0u, 0u, 0u, 0u, 0u, 0};
+  __syncthreads();
+  const uint32_t warp = threadIdx.x >> 5;
+  if (warp >= 2) return;
+  if (warp == 1) {
+    evict_loader(slots, meta, leaves, ring, pool, m, &flags, err);
+  } else if (threadIdx.x == 0) {
+    uint32_t ptr = 0, npush = 0;
     int hn = 0;
-    uint64_t evicted = 0;
+    uint32_t evicted = 0;
+    bool ok = true;
     while (evicted < todo) {
       const bool from_sorted = ptr < n && (hn == 0 || leaf_less(leaves[ptr], heap[0]));
       if (!from_sorted && hn == 0) break;
-      const Leaf v = from_sorted ? leaves[ptr++] : heap_pop(heap, hn);
-      const uint32_t ps = v.parent;
-      // the parent's metadata, all four words requested together
-      uint32_t pc = 0u, plu = 0u;
-      uint64_t ph = 0ull, pp = psk::kNoParent;
-      if (ps != kLeafNoParent) {
-        pc = meta.children[ps];
-        plu = meta.last_use[ps];
-        ph = slots[ps];
-        pp = meta.parent[ps];
+      Leaf v;
+      uint32_t ps = kLeafNoParent;
+      ParentRec r{0u, 0u, 0u, 0u, kLeafNoParent};
+      if (from_sorted) {
+        v = leaves[ptr];
+        ps = v.parent;
+        if (ps != kLeafNoParent) {
+          if (!psk::wait_smem_at_least(&flags.ring_done, ptr + 1u, &flags.abort, err, kEvictWaitNs)) {
+            ok = false;
+            break;
+          }
+          r = ring[ptr % (uint32_t)kRing];
+        }
+        ++ptr;
+        psk::st_release_cta_shared_u32(&flags.ptr, ptr);  // the record is read: its slot may be refilled
+      } else {
+        v = heap_pop(heap, hn);
+        if (v.parent != kLeafNoParent) {
+          if (!psk::wait_smem_at_least(&flags.pool_done, v.parent + 1u, &flags.abort, err, kEvictWaitNs)) {
+            ok = false;
+            break;
+          }
+          ps = pool[v.parent].pp;
+          r = pool[v.parent].r;
+        }
       }
       slots[v.slot] = psk::kEmpty;
       meta.last_use[v.slot] = 0;
       meta.children[v.slot] = 0;
       meta.parent[v.slot] = psk::kNoParent;
       ++evicted;
-      if (ps != kLeafNoParent) {
-        const uint32_t c = pc - 1;
-        meta.children[ps] = c;
-        if (c == 0) heap_push(heap, hn, make_leaf(plu, ps, ph, pp));
+      if (ps != kLeafNoParent && count_dec(dkey, dval, ps, r.pc) == 0u) {
+        uint32_t link = kLeafNoParent;
+        if (r.ppp != kLeafNoParent) {  // ask the loader for the record of its parent now
+          link = npush;
+          pool[npush].pp = r.ppp;
+          psk::st_release_cta_shared_u32(&flags.req, ++npush);
+        }
+        heap_push(heap, hn, Leaf{r.plu, ps, r.ph_lo, r.ph_hi, link});
       }
     }
     count[i] = cnt - evicted;
-    if (evicted > 0 && cnt - evicted > cap[i]) atomicOr(more, 1u);
+    if (ok && evicted > 0 && cnt - evicted > cap[i]) atomicOr(more, 1u);
+    psk::st_release_cta_shared_u32(&flags.exit, 1u);
   }
+  __syncwarp();
+  asm volatile("bar.sync 1, 64;" ::: "memory");  // warps 0 and 1: the loop and the loader are done
+  for (uint32_t x = threadIdx.x; x < (uint32_t)kDeltaSlots; x += 64u)
+    if (dkey[x] != kLeafNoParent) meta.children[dkey[x]] = dval[x];
 }
 
 // Prefix closure check (search mode): every chain's parent must be cached once the chains are in.
@@ -604,7 +765,7 @@ cudaError_t launch_advance(psk::StateSoA st, uint32_t I, const psk::ReqStore& rq
 cudaError_t launch_evict(uint64_t* slots, const psk::TableDesc* tdesc, uint32_t I, unsigned long long* count,
                          const uint64_t* cap, psk::LruMeta meta, void* leafbuf, uint32_t* nleaf, uint32_t* more,
                          uint32_t* more_host, uint64_t max_instance_slots, uint32_t* err, cudaStream_t s) {
-  const size_t smem = (size_t)(kLeafMax + kHeapMax) * sizeof(Leaf);
+  const size_t smem = kEvictSmem;
   cudaError_t e = cudaFuncSetAttribute(evict_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   const uint64_t per_block = (uint64_t)kCollectThreads * kCollectSlotsPerThread;
