@@ -364,21 +364,22 @@ __global__ void advance_kernel(psk::StateSoA st, uint32_t I, psk::ReqStore rq, p
 // can never be among E evictions, so a round of at most kHeapMax evictions reproduces the
 // one-at-a-time rule exactly; the host repeats rounds while an instance is still over capacity.
 //
-// The ordered loop touches shared memory only.  A loader warp reads each parent's metadata from
-// global memory ahead of it: for the sorted leaves, up to kRing leaves past the loop's position; for
-// a parent that became a leaf, as soon as it is pushed.  Children counts are not written during the
-// loop, so every load sees the round's starting count; the loop keeps the decremented counts in a
-// shared hash table, written back at the end of the round.  A block's metadata changes in a round
-// only when it is evicted, which happens after every record that names it as a parent has been read.
-// Most evictions climb a chain (a parent goes right after its last child, when its key is below the
-// next candidate's), and such a step still waits for its record: the parent's parent is known only
-// from the parent's metadata.
+// A loader warp reads each parent's metadata from global memory ahead of the ordered loop: for the
+// sorted leaves, up to kRing leaves past the loop's position; for a parent that became a leaf, as
+// soon as it is pushed.  The loop never waits for it: a record not filled yet is read by the loop
+// itself, with the same result.  Children counts are not written during the loop, so every read
+// sees the round's starting count; the loop keeps the decremented counts in a shared hash table,
+// written back at the end of the round.  A block's metadata changes in a round only when it is
+// evicted, which happens after every record that names it as a parent has been read.  Most
+// evictions climb a chain (a parent goes right after its last child, when its key is below the next
+// candidate's); such a step reads its record itself, since the parent's parent is known only from
+// the parent's metadata.
 constexpr int kLeafMax = 4096;
 constexpr int kHeapMax = 1536;
 constexpr int kEvictThreads = 256;
 constexpr int kRing = 32;          // sorted leaves whose parent records the loader keeps ready
 constexpr int kDeltaSlots = 2048;  // children counts a round changes (at most kHeapMax parents)
-constexpr uint64_t kEvictWaitNs = 1000000000ull;  // bound on any wait inside an eviction block
+constexpr uint64_t kEvictWaitNs = 1000000000ull;  // bound on the loader's idle wait
 static_assert(kHeapMax < kDeltaSlots, "the count table never fills");
 constexpr int kCollectThreads = 256;
 constexpr uint32_t kCollectSlotsPerThread = 8;
@@ -494,7 +495,6 @@ struct EvictFlags {
   uint32_t req;        // pool records the loop has asked for
   uint32_t pool_done;  // pool records filled
   uint32_t exit;       // the loop has ended
-  int abort;           // the loader gave up
 };
 
 // The loader warp: fills ring records for sorted leaves [ring_done, min(m, ptr + kRing)) and pool
@@ -520,10 +520,7 @@ __device__ void evict_loader(const uint64_t* slots, const psk::LruMeta& meta, co
     const uint32_t phi = req < pool_done + 32u ? req : pool_done + 32u;
     if (ring_done >= rhi && pool_done >= phi) {
       if ((it & 31u) == 0u && __any_sync(0xffffffffu, clock64() - c0 > lim)) {
-        if (lane == 0) {
-          atomicOr(err, psk::kErrTimeout);
-          f->abort = 1;
-        }
+        if (lane == 0) atomicOr(err, psk::kErrTimeout);
         return;
       }
       continue;
@@ -612,7 +609,7 @@ evict_kernel(uint64_t* slots, unsigned long long* count, const uint64_t* __restr
   const uint32_t todo = E < (uint64_t)kHeapMax ? (uint32_t)E : (uint32_t)kHeapMax;
   const uint32_t m = n < todo ? n : todo;  // sorted leaves a round can take
   for (uint32_t x = threadIdx.x; x < (uint32_t)kDeltaSlots; x += kEvictThreads) dkey[x] = kLeafNoParent;
-  if (threadIdx.x == 0) flags = EvictFlags{0u, 0u, 0u, 0u, 0u, 0};
+  if (threadIdx.x == 0) flags = EvictFlags{0u, 0u, 0u, 0u, 0u};
   __syncthreads();
   const uint32_t warp = threadIdx.x >> 5;
   if (warp >= 2) return;
@@ -622,7 +619,6 @@ evict_kernel(uint64_t* slots, unsigned long long* count, const uint64_t* __restr
     uint32_t ptr = 0, npush = 0;
     int hn = 0;
     uint32_t evicted = 0;
-    bool ok = true;
     while (evicted < todo) {
       const bool from_sorted = ptr < n && (hn == 0 || leaf_less(leaves[ptr], heap[0]));
       if (!from_sorted && hn == 0) break;
@@ -633,23 +629,25 @@ evict_kernel(uint64_t* slots, unsigned long long* count, const uint64_t* __restr
         v = leaves[ptr];
         ps = v.parent;
         if (ps != kLeafNoParent) {
-          if (!psk::wait_smem_at_least(&flags.ring_done, ptr + 1u, &flags.abort, err, kEvictWaitNs)) {
-            ok = false;
-            break;
+          if (psk::ld_relaxed_cta_shared_u32(&flags.ring_done) > ptr) {
+            psk::fence_acq_rel_cta();
+            r = ring[ptr % (uint32_t)kRing];
+          } else {
+            r = load_parent(slots, meta, ps);
           }
-          r = ring[ptr % (uint32_t)kRing];
         }
         ++ptr;
         psk::st_release_cta_shared_u32(&flags.ptr, ptr);  // the record is read: its slot may be refilled
       } else {
         v = heap_pop(heap, hn);
         if (v.parent != kLeafNoParent) {
-          if (!psk::wait_smem_at_least(&flags.pool_done, v.parent + 1u, &flags.abort, err, kEvictWaitNs)) {
-            ok = false;
-            break;
-          }
           ps = pool[v.parent].pp;
-          r = pool[v.parent].r;
+          if (psk::ld_relaxed_cta_shared_u32(&flags.pool_done) > v.parent) {
+            psk::fence_acq_rel_cta();
+            r = pool[v.parent].r;
+          } else {
+            r = load_parent(slots, meta, ps);
+          }
         }
       }
       slots[v.slot] = psk::kEmpty;
@@ -659,7 +657,7 @@ evict_kernel(uint64_t* slots, unsigned long long* count, const uint64_t* __restr
       ++evicted;
       if (ps != kLeafNoParent && count_dec(dkey, dval, ps, r.pc) == 0u) {
         uint32_t link = kLeafNoParent;
-        if (r.ppp != kLeafNoParent) {  // ask the loader for the record of its parent now
+        if (r.ppp != kLeafNoParent) {  // ask the loader for the record of its parent
           link = npush;
           pool[npush].pp = r.ppp;
           psk::st_release_cta_shared_u32(&flags.req, ++npush);
@@ -668,7 +666,7 @@ evict_kernel(uint64_t* slots, unsigned long long* count, const uint64_t* __restr
       }
     }
     count[i] = cnt - evicted;
-    if (ok && evicted > 0 && cnt - evicted > cap[i]) atomicOr(more, 1u);
+    if (evicted > 0 && cnt - evicted > cap[i]) atomicOr(more, 1u);
     psk::st_release_cta_shared_u32(&flags.exit, 1u);
   }
   __syncwarp();
