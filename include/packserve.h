@@ -403,7 +403,9 @@ typedef struct {
  * engine's progress simulated).  Errors: PS_ERR_STATE (a scheduled window
  * is still pending, or no request tracking), PS_ERR_INVALID (params), PS_ERR_CAPACITY (a decoding
  * list is full), PS_ERR_TABLE_FULL (an instance has more leaves than the eviction buffer holds,
- * 4096; its eviction stops). */
+ * 4096; its eviction stops), PS_ERR_TIMEOUT (an eviction block's metadata-prefetch warp found no
+ * work for 1 s, which a round of at most 1536 evictions never takes; the evictions already made
+ * stand, with counts and parent links consistent, and no further round runs). */
 PS_API ps_status ps_advance_window(ps_ctx* ctx, const ps_advance_params* p);
 
 /* Scheduling overhead, the quantity Section 8.3.3 reports as arrival-to-decision latency: device
