@@ -201,10 +201,6 @@ __device__ __forceinline__ uint32_t fastrange32(uint64_t h, uint32_t n) {
 // independent of the ones that pick the first bucket.
 __device__ __forceinline__ uint64_t remix(uint64_t k) { return (k ^ (k >> 31)) * 0x7FB5D329728EA185ull; }
 
-__device__ __forceinline__ bool ovf_bit(const uint64_t* ovf, const TableDesc& d, uint32_t b) {
-  return (ovf[d.ovf + (b >> 6)] >> (b & 63)) & 1ull;
-}
-
 // Membership in an instance's main table, in two parts so that several lookups can have their
 // loads in flight together: lookup_issue requests both candidate buckets (2 x 4 x 16-byte loads)
 // and the overflow word, lookup_finish compares (and, rarely, follows the overflow run after b1).
@@ -536,18 +532,11 @@ __device__ __forceinline__ void st_relaxed_u64(unsigned long long* p, unsigned l
   asm volatile("st.relaxed.gpu.global.u64 [%0], %1;" ::"l"(p), "l"(v) : "memory");
 }
 
-// Shared-memory flags between the warps of one block: release store / acquire load at CTA scope
-// (orders this thread's earlier accesses / its later accesses, without waiting for global stores).
+// Shared-memory flags between the warps of one block: a release store at CTA scope (orders this
+// thread's earlier accesses, without waiting for global stores).
 __device__ __forceinline__ void st_release_cta_shared_u32(uint32_t* p, uint32_t v) {
   asm volatile("st.release.cta.shared::cta.u32 [%0], %1;" ::"r"((uint32_t)__cvta_generic_to_shared(p)), "r"(v)
                : "memory");
-}
-
-__device__ __forceinline__ uint32_t ld_acquire_cta_shared_u32(const uint32_t* p) {
-  uint32_t v;
-  asm volatile("ld.acquire.cta.shared::cta.u32 %0, [%1];" : "=r"(v) : "r"((uint32_t)__cvta_generic_to_shared(p))
-               : "memory");
-  return v;
 }
 
 __device__ __forceinline__ uint32_t ld_relaxed_cta_shared_u32(const uint32_t* p) {
@@ -598,30 +587,13 @@ __device__ __forceinline__ void cp_async16(void* smem, const void* gmem) {
                : "memory");
 }
 
-// 4-, 8- or 16-byte asynchronous global -> shared copy (both addresses aligned to the size).
-template <int BYTES>
-__device__ __forceinline__ void cp_async_bytes(void* smem, const void* gmem) {
-  static_assert(BYTES == 4 || BYTES == 8 || BYTES == 16, "cp.async copies 4, 8 or 16 bytes");
-  if (BYTES == 16) {
-    cp_async16(smem, gmem);
-  } else {
-    asm volatile("cp.async.ca.shared.global [%0], [%1], %2;" ::"r"((uint32_t)__cvta_generic_to_shared(smem)),
-                 "l"(gmem), "n"(BYTES)
-                 : "memory");
-  }
-}
-
 __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
 
 __device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_all;" ::: "memory"); }
 
-// Wait until at most N of this thread's most recent copy groups are still pending.
-template <int N>
-__device__ __forceinline__ void cp_async_wait_group() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
-
 // ------------------------------------------------------------------------------- first-miss walks --
 // All 32 lanes of a warp call these with the same arguments; present(k) is evaluated per lane.
-// Both return the first position k in [lo, nb) with present(k) false (nb if there is none), given
+// Each returns the first position k in [lo, nb) with present(k) false (nb if there is none), given
 // that every position below lo is known present.
 
 // Linear walk, 32 consecutive positions per step: exact for any membership pattern.
@@ -662,11 +634,6 @@ __device__ __forceinline__ uint64_t warp_search_range(uint64_t lo, uint64_t hi, 
     lo = lo + (j * span) / 32;
     hi = pj;
   }
-}
-
-template <class Pred>
-__device__ __forceinline__ uint64_t warp_first_miss_search(uint64_t lo, uint64_t nb, Pred present) {
-  return warp_search_range(lo, nb, present);
 }
 
 __device__ __forceinline__ uint64_t warp_min_u64(uint64_t x) {
