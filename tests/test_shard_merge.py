@@ -211,3 +211,46 @@ def test_thread_ranks_merge_to_the_unsharded_oracle():
     for k, (merged, cls, _) in enumerate(out):
         assert np.array_equal(merged["best"], full["best"]) and np.array_equal(merged["path"], full["path"])
         assert np.array_equal(cls, full["cls"][:, cuts[k]:cuts[k + 1]])
+
+
+def test_blocks_without_capacity_and_rows_rejected_everywhere():
+    """Edge cases of the merge, blocks as threads: the first block has no instance with a free
+    decode slot (b + qr + 1 > B_max), so its W_min and its key are the 'none' values on every row,
+    and the second block's KV room fits only the shorter prompts (S + L <= M_KV), so the longer
+    requests pass the capacity guard nowhere and are rejected (Algorithm 1: A empty)."""
+    import threading
+    wl = W.generate(0)
+    ins = wl.instances
+    cut = 3
+    ins.b[:cut] = ins.B_max[:cut]
+    med = int(np.median(wl.window.prompt_tokens))
+    ins.M_KV[cut:] = ins.S[cut:] + med
+    I = ins.I
+    full = Oracle(I, wl.model).load(ins).score_rows(wl.window)
+    assert (full["best"] < 0).any() and (full["best"] >= 0).any()
+    assert (full["best"][full["best"] >= 0] >= cut).all()
+    rows = np.arange(wl.window.R, dtype=np.uint32)
+    cuts = [0, cut, I]
+    grp = shard.LocalGroup(2)
+    out, errs = [None, None], []
+
+    def work(k):
+        try:
+            out[k] = block_partials(wl, cuts[k], cuts[k + 1], rows, grp.allreduce_min(k))
+        except BaseException as e:  # noqa: BLE001 - reported below
+            errs.append(e)
+            grp.abort()
+
+    th = [threading.Thread(target=work, args=(k,)) for k in range(2)]
+    for t in th:
+        t.start()
+    for t in th:
+        t.join(timeout=120)
+    assert not errs, errs
+    for k, (merged, cls, wpool) in enumerate(out):
+        assert np.array_equal(merged["best"], full["best"]), k
+        assert np.array_equal(merged["path"], full["path"]), k
+        assert np.array_equal(cls, full["cls"][:, cuts[k]:cuts[k + 1]]), k
+    # a row rejected everywhere has no pool W_min at all
+    rej = full["best"] < 0
+    assert (out[0][2][rej] == np.uint32(NO_W)).all()
