@@ -1,9 +1,13 @@
 // Greedy in-window assignment (Algorithm 1 applied to the window's requests in arrival order).
 //
 // The paper's gateway decides each request online and updates the instance records along the
-// request path before the next decision (Section 4, Metadata service; Section 7).  This kernel
-// replays that sequence for a whole window on the GPU: one persistent thread block whose threads
-// each own up to IPT instances.  Per request r:
+// request path before the next decision (Section 4, Metadata service; Section 7).  Two kernels
+// replay that sequence for a whole window on the GPU:
+//   greedy_kernel       any cache (the probe's linear mode), described here;
+//   greedy_pipe_kernel  prefix-closed caches (the search mode), a pipelined cooperative launch of
+//                       deciding, insert, probe and summary blocks, described at its section below.
+// greedy_kernel is one persistent thread block whose threads each own up to IPT instances.  Per
+// request r:
 //   1. hit of r on instance i = hit0[r][i] (the probe kernel's result on the committed tables)
 //      extended through the window's delta table: an instance that has received blocks in this
 //      window is re-probed at position hit0, and if that block is now cached a warp finds the new
