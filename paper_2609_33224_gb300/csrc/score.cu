@@ -1,7 +1,9 @@
 // Fused score kernel: hit lengths + instance state -> predicted latencies, Algorithm 1's admission
 // sets and the per-request pick, each request independently against the same state.
 //
-// The instance terms that do not depend on the request (InstTerms, the free KV room with the
+// Two forms: score_block_kernel for rows of 257 .. 1024 instances (a thread block per row, the
+// instance terms in registers; described at its section below) and score_rows_kernel for the other
+// sizes, described here.  The instance terms that do not depend on the request (InstTerms, the free KV room with the
 // decode-slot guard folded in, q, S and the class-0 key bits of (b, qr)) are computed once per
 // thread block into shared memory as padded structure-of-arrays.  One warp then takes one request
 // at a time: lane l owns the instances 128 v + 4 l .. 128 v + 4 l + 3 of each 128-instance chunk v,
