@@ -497,6 +497,9 @@ def main():
                 "note": "serial per-request dependency chain decided on one SM: latency-bound, not "
                         "bandwidth-bound; traffic scaled by request count from the 8192-request ncu capture"}
     probe_achieved = probe_bytes / (probe_ms / 1000) / 1e9
+    # the whole A2 phase: the relations pass exists only to serve the probe, so it is counted too
+    a2_ms = probe_ms + max(0.0, km["relations"])
+    a2_achieved = probe_bytes / (a2_ms / 1000) / 1e9 if a2_ms > 0 else None
     line = {"metric": METRIC, "value": job_rate(world, R * I, ms), "unit": "scorings/s", "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f32+u64", "data": "synthetic (seeded generator)",
@@ -511,7 +514,10 @@ def main():
                                "unit": "GB/s", "peak": peak, "frac": probe_achieved / peak,
                                "frac_vs_8tbs": probe_achieved / 8000.0, "ms": probe_ms,
                                "algorithmic_bytes_per_launch": probe_bytes, "stats": pstats,
-                               "traffic": None if probe_traffic is None else probe_traffic * n_probes},
+                               "traffic": None if probe_traffic is None else probe_traffic * n_probes,
+                               "a2_phase": {"kernels": "relations_kernel + probe_search_kernel + probe_derived_kernel",
+                                            "ms": a2_ms, "achieved": a2_achieved,
+                                            "frac": None if a2_achieved is None else a2_achieved / peak}},
             "roofline": roof,
             "scoring_call": {"what": "ps_score_window with hits, TPOT, TTFT and class of every pair and the "
                                      "per-request pick written to device buffers",
